@@ -1,0 +1,340 @@
+"""Benchmark: packed-ensemble training throughput on GB300.
+
+One step = one pass of the whole training path over one batch: gather,
+forward through every member, per-member loss, backward, per-member AdamW.
+Metric: member-samples/s = (active members) x (batch rows) x steps / time.
+
+  python bench.py [--gpus N --steps K --warmup W --workload medium]
+  python bench.py --impl reference ...   # the CPU fp64 oracle on host cores
+
+Under torchrun (N > 1) every rank trains its own full pack (members are
+independent; no collective on the data path), so scaling is weak and the
+reported value is the sum over ranks of member-samples / max-over-ranks time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from workloads import SEED_HP, SEED_INIT, WORKLOADS, make_data, sample_hparams  # noqa: E402
+
+METRIC = "member-samples/sec (fwd+bwd+AdamW)"
+UNIT = "member-samples/s"
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"], bf16_sus=d.get("bf16_tflops_sustained", d["bf16_tflops"]),
+                    source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
+
+
+def work_per_step(wl, hp, B):
+    """Algorithmic work of one step, from the shapes (no padding):
+    matrix-product flops (forward 2, dgrad 2 except layer 0, wgrad 2 per MAC)
+    and AdamW bytes (read p, g, m, v; write p, m, v fp32 + the bf16 copy)."""
+    flops = 0.0
+    n_params = 0
+    for L, w in zip(hp["depth"], hp["width"]):
+        L, w = int(L), int(w)
+        macs_fwd = wl.d_in * w + (L - 1) * w * w
+        macs_dgrad = (L - 1) * w * w
+        flops += 2.0 * B * (2 * macs_fwd + macs_dgrad)
+        n_params += wl.d_in * w + w + (L - 1) * (w * w + w) + wl.d_out * w + wl.d_out
+    return flops, n_params
+
+
+def workload_desc(wl, B):
+    return (f"{wl.name}: {wl.task}, m={wl.m} members, depth U{{{wl.depth[0]}..{wl.depth[1]}}}, width multiples of "
+            f"{wl.width[2]} in [{wl.width[0]},{wl.width[1]}], dropout U[{wl.dropout[0]},{wl.dropout[1]}], "
+            f"d_in={wl.d_in}, d_out={wl.d_out}, batch={B}, n_train={wl.n_train}")
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples during the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id):
+        self.gpu_id = gpu_id
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu_id}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.out = ""
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if not getattr(self, "out", ""):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm, smax, reasons = [], [], set()
+        names = ["active", "hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[0]))
+                smax.append(float(f[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names[1:], f[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def cpu_baseline(wl, hp, data_np, B, budget_s=20.0):
+    """The oracle as it stands, on the host cores, on a bounded sample of the
+    same workload: the first k members (independent of the others), timed
+    over whole steps until about budget_s seconds of CPU work."""
+    import oracle
+    oracle.build()
+    X, y = data_np
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    k = min(wl.m, max(1, cores))
+    rng = np.random.default_rng(3)
+    members = list(range(k))
+    pk = oracle.OraclePack(wl.d_in, wl.d_out, wl.task, hp["depth"][members], hp["width"][members],
+                           hp["dropout"][members], hp["lr"][members], hp["wd"][members], seed=SEED_INIT,
+                           member_id=members)
+    steps = 0
+    t0 = time.perf_counter()
+    while True:
+        idx = rng.choice(X.shape[0], B, replace=False).astype(np.int32)
+        pk.train_step(X, idx, y, steps)
+        steps += 1
+        el = time.perf_counter() - t0
+        if el > budget_s or steps >= 50:
+            break
+    value = k * B * steps / el
+    return {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"members 0..{k - 1} of {wl.m} (independent), {steps} full steps of batch {B}, {el:.1f} s"}
+
+
+def run_reference(args, wl, rank):
+    """Reference arm: the CPU fp64 oracle timed on the host cores (rank 0)."""
+    if rank != 0:
+        return
+    hp = sample_hparams(wl, seed=SEED_HP)
+    B = wl.batch
+    n = min(wl.n_train, 20000)
+    d = make_data(wl, device="cpu", n_train=n, n_val=0)
+    data = (d["X_train"].numpy(), d["y_train"].numpy())
+    per = max(3.0, min(30.0, 120.0 / max(1, args.steps)))
+    vals = []
+    for _ in range(args.warmup if args.warmup < 1 else 1):
+        pass
+    base = None
+    for s in range(max(1, args.steps)):
+        base = cpu_baseline(wl, hp, data, B, budget_s=per)
+        vals.append(base["value"])
+    value = float(np.mean(vals))
+    ms = float(1000.0 * wl.m * B / value)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": workload_desc(wl, B)},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": base["cores"], "kind": "oracle",
+                             "sample": base["sample"]},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--workload", default="medium", choices=sorted(WORKLOADS))
+    ap.add_argument("--precision", default="bf16", choices=["bf16", "fp32"])
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    wl = WORKLOADS[args.workload]
+
+    if args.impl == "reference":
+        run_reference(args, wl, rank)
+        return
+
+    import torch
+    import torch.distributed as dist
+    import paper_2607_05380_gb300 as tp
+
+    if world > 1:
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    tp.load_library()
+
+    B = wl.batch
+    hp = sample_hparams(wl, seed=SEED_HP)
+    d = make_data(wl, device=dev)
+    X, y = d["X_train"], d["y_train"]
+    n_train = X.shape[0]
+    total = args.warmup + args.steps
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(3)
+    idx_all = torch.stack([torch.randperm(n_train, generator=gen, device=dev)[:B] for _ in range(total)])
+    idx_all = idx_all.to(torch.int32).contiguous()
+
+    stream = torch.cuda.current_stream()
+    pack = tp.Pack(wl.d_in, wl.d_out, wl.task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
+                   max_batch=B, seed=SEED_INIT, precision=args.precision, stream=stream)
+    loss = torch.zeros(wl.m, dtype=torch.float32, device=dev)
+
+    for s in range(args.warmup):
+        pack.train_step(X, idx_all[s], y, s, loss)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+
+    gpu_id = getattr(torch.cuda.get_device_properties(dev), "uuid", None)
+    gpu_id = f"GPU-{gpu_id}" if gpu_id is not None and not str(gpu_id).startswith("GPU-") else (gpu_id or local)
+    l0 = pack.launch_count()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(gpu_id) as clk:
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for s in range(args.warmup, total):
+            pack.train_step(X, idx_all[s], y, s, loss)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    launches = pack.launch_count() - l0
+    ms_total = ev0.elapsed_time(ev1)
+    if world > 1:
+        t = torch.tensor([ms_total], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_total = float(t.item())
+        dist.barrier()
+    ms_step = ms_total / args.steps
+    value = world * wl.m * B * args.steps / (ms_total / 1000.0)
+    lossv = loss.cpu().numpy()
+
+    # per-kernel-family times over a second timed region (CUDA events on the pack's stream)
+    pack.profile_enable(True)
+    pack.profile_read(reset=True)
+    n_prof = min(args.steps, 50)
+    for s in range(n_prof):
+        pack.train_step(X, idx_all[args.warmup + s], y, total + s, loss)
+    prof = pack.profile_read(reset=True)
+    pack.profile_enable(False)
+    flops, n_params = work_per_step(wl, hp, B)
+    pk = peaks()
+    fam = {k: v for k, v in prof.items() if v[1] > 0}
+    dominant = max(fam, key=lambda k: fam[k][0])
+    shares = {k: round(v[0] / sum(x[0] for x in fam.values()), 4) for k, v in fam.items()}
+    if dominant in ("fwd", "bwd"):
+        gemm_ms = (prof["fwd"][0] + prof["bwd"][0]) / n_prof
+        n_l = (prof["fwd"][1] + prof["bwd"][1]) / n_prof
+        ach = flops / (gemm_ms / 1000.0) / 1e12
+        roof = {"kernel": "grouped GEMM (fwd+dgrad+wgrad launches of one step)", "bound": "tensor",
+                "achieved": ach, "peak": pk["bf16_sus"], "unit": "TFLOP/s", "frac": ach / pk["bf16_sus"],
+                "traffic": None, "per_launch_ms": gemm_ms / max(1, n_l), "peak_source": pk["source"] + " sustained"}
+    else:
+        per_launch_ms = prof[dominant][0] / max(1, prof[dominant][1])
+        byts = 30.0 * n_params if dominant == "adamw" else None
+        ach = byts / (per_launch_ms / 1000.0) / 1e9 if byts else None
+        roof = {"kernel": dominant, "bound": "hbm", "achieved": ach, "peak": pk["hbm"], "unit": "GB/s",
+                "frac": (ach / pk["hbm"]) if ach else None, "traffic": None, "per_launch_ms": per_launch_ms,
+                "peak_source": pk["source"]}
+    roof["shares"] = shares
+
+    # end to end through the public API with host buffers: per step the batch
+    # rows and labels go host -> device (pinned), the member losses come back
+    e2e = None
+    if not args.no_e2e:
+        Xh = X.cpu().pin_memory()
+        yh = y.cpu().pin_memory()
+        idx_h = idx_all.cpu()
+        xb_h = [Xh[idx_h[s].long()].pin_memory() for s in range(min(total, 64))]
+        yb_h = [yh[idx_h[s].long()].pin_memory() for s in range(min(total, 64))]
+        ident = torch.arange(B, dtype=torch.int32, device=dev)
+        xb_d = torch.empty(B, wl.d_in, dtype=torch.float32, device=dev)
+        yb_d = torch.empty(B, dtype=y.dtype, device=dev)
+        loss_h = torch.empty(wl.m, dtype=torch.float32).pin_memory()
+        n_e2e = min(args.steps, 64)
+        for s in range(3):
+            xb_d.copy_(xb_h[s], non_blocking=True)
+            yb_d.copy_(yb_h[s], non_blocking=True)
+            pack.train_step(xb_d, ident, yb_d, s, loss)
+            loss_h.copy_(loss, non_blocking=True)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for s in range(n_e2e):
+            xb_d.copy_(xb_h[s % len(xb_h)], non_blocking=True)
+            yb_d.copy_(yb_h[s % len(yb_h)], non_blocking=True)
+            pack.train_step(xb_d, ident, yb_d, 10_000 + s, loss)
+            loss_h.copy_(loss, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+        ms_e2e = max(e0.elapsed_time(e1), wall * 1000.0)
+        e2e = {"value": world * wl.m * B * n_e2e / (ms_e2e / 1000.0), "unit": UNIT,
+               "h2d_bytes_per_step": B * wl.d_in * 4 + B * 4, "d2h_bytes_per_step": wl.m * 4, "steps": n_e2e}
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        n = min(n_train, 20000)
+        data_np = (X[:n].cpu().numpy(), y[:n].cpu().numpy())
+        cpu = cpu_baseline(wl, hp, data_np, B, budget_s=20.0)
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": args.precision, "data": "synthetic",
+                "config": {"workload": workload_desc(wl, B), "precision": args.precision,
+                           "params": n_params, "gemm_flop_per_step": flops,
+                           "l2": "inputs larger than L2: each step streams ~%.2f GB of parameters and optimizer state"
+                                 % (30.0 * n_params / 1e9),
+                           "parallelism": "one independent pack per GPU" if world > 1 else "single GPU"},
+                "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
+                "clocks": clk.summary(), "final_losses_mean": float(np.nanmean(lossv))}
+        print(json.dumps(line), flush=True)
+    pack.close()
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

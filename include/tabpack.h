@@ -1,0 +1,202 @@
+/*
+ * tabpack.h -- C ABI of the GB300 (sm_103a) library for training a packed
+ * hyperparameter ensemble of tabular MLPs, after "TabPack: Efficient
+ * Hyperparameter Ensembles for Tabular Deep Learning".
+ *
+ * A pack holds m base MLPs ("base models", Sec. 3.3).  Member i is a stack of
+ * depth[i] Linear-ReLU-Dropout blocks of width width[i] with dropout rate
+ * dropout[i], followed by a linear head with d_out outputs; it is trained by
+ * its own AdamW optimizer with learning rate lr[i] and weight decay wd[i]
+ * (the optimizer pack, Sec. 3.4).  All members see the same input batch and
+ * are trained independently: the per-member losses are summed, so each
+ * member's gradient is that of its own loss (Sec. 3.6 "Training").
+ *
+ * Conventions for every entry point:
+ *   - Pointers documented "device" are CUDA device pointers; they are read or
+ *     written asynchronously on the pack's stream and must stay valid until
+ *     the work on that stream has finished.  Pointers documented "host" are
+ *     ordinary host memory, read or written before the call returns.
+ *   - The caller owns every pointer argument; the pack owns its own device
+ *     memory (parameters, optimizer state, activations), allocated at
+ *     pack_create and freed at pack_destroy.
+ *   - Matrices are row-major.  Weights of a layer are [out, in]; biases [out].
+ *     Layer index l is 0-based: 0 .. depth-1 are the hidden blocks and
+ *     l == depth is the head.
+ *   - Labels y are device int32 class indices (binary: 0/1, multiclass:
+ *     0..d_out-1) or device float32 targets (regression), with one entry per
+ *     row of X.
+ *   - No C++ exception crosses the ABI.  Every entry point returns a
+ *     tp_status; on failure pack_last_error() describes the cause.  A
+ *     TP_ECUDA status means a CUDA call failed; the pack should then be
+ *     destroyed.
+ *   - A pack is not thread-safe: use it from one host thread at a time.
+ */
+#ifndef TABPACK_H
+#define TABPACK_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct tabpack tabpack_t;
+
+typedef enum {
+  TP_OK = 0,
+  TP_EINVAL = 1,    /* an argument is out of range or inconsistent        */
+  TP_ENOMEM = 2,    /* device or pinned-host allocation failed            */
+  TP_ECUDA = 3,     /* a CUDA runtime/driver call failed                  */
+  TP_ESTATE = 4,    /* call not valid in the pack's current state         */
+  TP_ETIMEOUT = 5,  /* a bounded device-side wait gave up                 */
+  TP_ENOTSUP = 6    /* configuration not supported on this device         */
+} tp_status;
+
+typedef enum { TP_BINARY = 0, TP_MULTICLASS = 1, TP_REGRESSION = 2 } tp_task;
+typedef enum { TP_BF16 = 0, TP_FP32 = 1 } tp_precision;
+typedef enum { TP_SCORE_LOSS = 0, TP_SCORE_ACCURACY = 1, TP_SCORE_RMSE = 2 } tp_score;
+
+typedef struct {
+  int32_t m;          /* number of base models in the pack, >= 1                        */
+  int32_t d_in;       /* input features, >= 1                                           */
+  int32_t d_out;      /* 1 for binary / regression, number of classes (2..32) otherwise  */
+  int32_t max_batch;  /* largest B passed to pack_train_step, >= 1                      */
+  int32_t task;       /* tp_task                                                        */
+  int32_t precision;  /* tp_precision: TP_BF16 runs the matrix products on bf16 tensor
+                         cores with fp32 accumulation and stores activations in bf16;
+                         TP_FP32 keeps everything in fp32 (CUDA-core products)           */
+  uint64_t seed;      /* Philox key of parameter init and dropout masks                 */
+  float beta1, beta2, eps;  /* AdamW constants shared by all members (0.9, 0.999, 1e-8) */
+  int32_t wd_on_bias; /* 1: weight decay also applies to biases                         */
+} tp_config;
+
+/* Create a pack (Sec. 3.3 model pack + Sec. 3.4 optimizer pack).
+ * depth, width, dropout, lr, wd: host arrays of length cfg->m, copied.
+ *   depth[i] in 1..14; width[i] a positive multiple of 16 (<= 4096);
+ *   0 <= dropout[i] < 1; lr[i] >= 0; wd[i] >= 0.
+ * cuda_stream: the cudaStream_t all work of this pack runs on (NULL: the
+ *   legacy default stream).
+ * Parameters are initialised on the device from Philox4x32-10: element e of
+ * layer l of member i (weights row-major, then biases) takes the word at
+ * counter (e >> 2, 0, 0, 1 << 28 | i << 4 | l), word e & 3, key cfg->seed;
+ * with u = ((r >> 8) + 1/2) 2^-24 its value is (2u - 1) / sqrt(fan_in),
+ * rounded to fp32 (U(-1/sqrt(fan_in), 1/sqrt(fan_in)), the PyTorch Linear
+ * default; the paper does not state its init).
+ * On success *out receives the handle; on failure *out is NULL.             */
+tp_status pack_create(const tp_config* cfg, const int32_t* depth, const int32_t* width,
+                      const float* dropout, const float* lr, const float* wd,
+                      void* cuda_stream, tabpack_t** out);
+
+/* Free the pack and its device memory (waits for the pack's stream). NULL ok. */
+void pack_destroy(tabpack_t* pack);
+
+/* Change the stream subsequent work is enqueued on. */
+tp_status pack_set_stream(tabpack_t* pack, void* cuda_stream);
+
+/* One training step of every active member (Sec. 3.6): gather rows
+ * idx[0..B) of X, forward through each member's blocks with its own dropout
+ * rate, per-member mean loss (cross-entropy for multiclass, logistic loss on
+ * one logit for binary, MSE for regression), backward, and one AdamW update
+ * per member with its own lr and wd and its own step count t (PyTorch AdamW
+ * semantics: p <- p - lr wd p, then the bias-corrected Adam step).
+ *   X: device float32 [n_rows, d_in];  idx: device int32 [B], 0 <= idx < n_rows
+ *   (not checked on the device);  y: device labels [n_rows] (see above);
+ *   1 <= B <= max_batch;  step: dropout counter of this step (masks are a
+ *   function of (seed, member, layer, step, row, col): keep iff the Philox
+ *   word at counter (row, col >> 2, step, member << 4 | layer), word col & 3,
+ *   is >= floor(dropout * 2^32));
+ *   loss_out: device float32 [m] (may be NULL): member i's mean loss, NaN for
+ *   inactive members.
+ * Asynchronous: returns once the work is enqueued.                          */
+tp_status pack_train_step(tabpack_t* pack, const float* X, int64_t n_rows, const int32_t* idx,
+                          const void* y, int32_t B, uint32_t step, float* loss_out);
+
+/* Same as pack_train_step without the optimizer update: the gradients of
+ * the step stay readable through pack_get_grads and the step counts do not
+ * advance.  For tests and diagnostics.                                       */
+tp_status pack_forward_backward(tabpack_t* pack, const float* X, int64_t n_rows, const int32_t* idx,
+                                const void* y, int32_t B, uint32_t step, float* loss_out);
+
+/* Per-member validation predictions (Sec. 3.5 "Online ensemble"): forward
+ * without dropout of every active member on all N rows of X.
+ *   X: device float32 [N, d_in];  out: device float32 [m, N, d_out]:
+ *   softmax probabilities (multiclass), sigmoid probability of class 1
+ *   (binary) or the regression value.  Rows of inactive members are left
+ *   untouched.  Asynchronous.                                                */
+tp_status pack_predict(tabpack_t* pack, const float* X, int64_t N, float* out);
+
+/* Greedy ensemble selection over a pool of P candidates (Sec. 3.5 "Greedy
+ * ensembling"): start from the candidate with the best ensemble score, then
+ * repeatedly add the unused candidate whose addition gives the best score of
+ * the averaged prediction; stop after m_ens members or when the best
+ * addition does not strictly improve the score.  Ties go to the lowest
+ * candidate index.  Scores (lower is better): TP_SCORE_LOSS = mean CE / BCE
+ * of the averaged probabilities clipped to [1e-7, 1 - 1e-7], or MSE;
+ * TP_SCORE_ACCURACY = minus the accuracy (classification);
+ * TP_SCORE_RMSE = root MSE (regression).  Per-row terms are taken in fp32
+ * and summed in fp64 in a fixed order; the running ensemble sum is fp64.
+ *   preds: device float32 [P, N, d_out] (probabilities or values as written
+ *   by pack_predict);  y: device labels [N];  cuda_stream: stream to run on;
+ *   selected: host int32 [m_ens] receives the selection order;
+ *   n_selected, final_score: host outputs.
+ * Allocates its scratch with cudaMallocAsync on the stream and synchronises
+ * the stream before returning.                                              */
+tp_status pack_select_greedy(const float* preds, int32_t P, int64_t N, int32_t d_out, const void* y,
+                             int32_t task, int32_t score, int32_t m_ens, void* cuda_stream,
+                             int32_t* selected, int32_t* n_selected, double* final_score);
+
+/* Base-model early stopping hook (Sec. 3.6): active is a host uint8 [m];
+ * inactive members are skipped by every kernel and keep their parameters,
+ * optimizer state and step count.                                           */
+tp_status pack_set_active(tabpack_t* pack, const uint8_t* active);
+
+/* Copy one layer's fp32 master parameters to / from host memory.
+ * W: host float32 [out, in] (may be NULL), b: host float32 [out] (may be
+ * NULL).  Synchronises the pack's stream.  pack_set_params also refreshes
+ * the bf16 copy used by the tensor-core products.                           */
+tp_status pack_get_params(tabpack_t* pack, int32_t member, int32_t layer, float* W, float* b);
+tp_status pack_set_params(tabpack_t* pack, int32_t member, int32_t layer, const float* W, const float* b);
+
+/* Gradients of the last pack_forward_backward, same layout as the params.  */
+tp_status pack_get_grads(tabpack_t* pack, int32_t member, int32_t layer, float* W, float* b);
+
+/* Logits of the last step for one member: host float32 [B, d_out].        */
+tp_status pack_get_logits(tabpack_t* pack, int32_t member, float* out);
+
+/* Dropout keep mask (1 keep, 0 drop) that step `step` applies to hidden
+ * layer `layer` of `member`, evaluated on the device by the same function
+ * the forward epilogue uses: host uint8 [B, width].                        */
+tp_status pack_debug_masks(tabpack_t* pack, int32_t member, int32_t layer, uint32_t step,
+                           int32_t B, uint8_t* keep);
+
+/* Activations of the last forward for hidden layer `layer` of `member`
+ * (the stored output of that layer, after ReLU and dropout): host float32
+ * [B, width] with B the last step's batch size.  For tests and diagnostics. */
+tp_status pack_debug_activations(tabpack_t* pack, int32_t member, int32_t layer, float* out);
+
+/* Per-kernel-family timing with CUDA events recorded on the pack's stream.
+ * Enable, run work, then read the accumulated milliseconds and launch counts
+ * (synchronises).  Families: see tp_phase.                                  */
+typedef enum {
+  TP_PH_GATHER = 0, TP_PH_FWD = 1, TP_PH_HEAD = 2, TP_PH_BWD = 3, TP_PH_BIAS = 4,
+  TP_PH_ADAMW = 5, TP_PH_PREDICT = 6, TP_PH_COUNT = 7
+} tp_phase;
+tp_status pack_profile_enable(tabpack_t* pack, int32_t enable);
+tp_status pack_profile_read(tabpack_t* pack, double* ms /* [TP_PH_COUNT] */,
+                            int64_t* launches /* [TP_PH_COUNT] */, int32_t reset);
+
+/* Number of kernels this pack has launched since creation.                 */
+int64_t pack_launch_count(const tabpack_t* pack);
+
+/* Sizes of the pack: number of fp32 parameters (as stored, including the
+ * zero padding of layer-0 columns to a multiple of 8) and device bytes held. */
+tp_status pack_sizes(const tabpack_t* pack, int64_t* n_params, int64_t* device_bytes);
+
+/* Description of the last error on this pack (or, for pack == NULL, of the
+ * last failed pack_create / pack_select_greedy on this thread).            */
+const char* pack_last_error(const tabpack_t* pack);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

@@ -81,6 +81,7 @@ def lib():
                 "orc_get_logits": (ctypes.c_int, [P, i32, P]),
                 "orc_get_keep": (ctypes.c_int, [P, i32, i32, P]),
                 "orc_get_margin": (f64, [P, i32]),
+                "orc_get_preact": (ctypes.c_int, [P, i32, i32, P]),
                 "orc_member_steps": (i64, [P, i32]),
                 "orc_greedy": (ctypes.c_int, [P, i32, i64, i32, P, P, i32, i32, i32, i32,
                                               P, P, P, P, P]),
@@ -221,6 +222,12 @@ class OraclePack:
     def keep(self, member, layer):
         out = np.zeros((self._B, int(self.width[member])), dtype=np.uint8)
         if lib().orc_get_keep(self._h, member, layer, _ptr(out)):
+            raise IndexError((member, layer))
+        return out
+
+    def preact(self, member, layer):
+        out = np.zeros((self._B, int(self.width[member])), dtype=np.float64)
+        if lib().orc_get_preact(self._h, member, layer, _ptr(out)):
             raise IndexError((member, layer))
         return out
 

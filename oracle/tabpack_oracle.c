@@ -529,6 +529,13 @@ int orc_get_keep(const orc_pack* h, int32_t member, int32_t layer, uint8_t* out)
   return 0;
 }
 
+int orc_get_preact(const orc_pack* h, int32_t member, int32_t layer, double* out) {
+  if (orc_check_ml(h, member, layer) || layer >= h->mem[member].L || !h->mem[member].Z) return 1;
+  const orc_member* M = &h->mem[member];
+  memcpy(out, M->Z[layer], (size_t)M->B * M->w * sizeof(double));
+  return 0;
+}
+
 double orc_get_margin(const orc_pack* h, int32_t member) {
   if (orc_check_ml(h, member, 0)) return NAN;
   return h->mem[member].margin;

@@ -108,6 +108,8 @@ int orc_get_adam_state(const orc_pack* h, int32_t member, int32_t layer,
 int orc_get_logits(const orc_pack* h, int32_t member, double* out);
 /* dropout keep mask of the last step for hidden layer `layer` [B, width] */
 int orc_get_keep(const orc_pack* h, int32_t member, int32_t layer, uint8_t* out);
+/* pre-activations Z of the last forward for hidden layer `layer` [B, width]   */
+int orc_get_preact(const orc_pack* h, int32_t member, int32_t layer, double* out);
 /* smallest |Z| / rms(Z) over the pre-activations of the last forward          */
 double orc_get_margin(const orc_pack* h, int32_t member);
 int64_t orc_member_steps(const orc_pack* h, int32_t member);

@@ -1,0 +1,262 @@
+"""Python binding of the tabpack C ABI (``include/tabpack.h``).
+
+Argument marshalling only: every step of the training path runs in the CUDA
+kernels of ``libtabpack.so``; PyTorch provides device memory and streams.
+The library must have been built (``build.build()``); importing the binding
+without it raises, there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+from . import build as _build
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = _build.LIB
+
+TP_OK, TP_EINVAL, TP_ENOMEM, TP_ECUDA, TP_ESTATE, TP_ETIMEOUT, TP_ENOTSUP = range(7)
+BINARY, MULTICLASS, REGRESSION = 0, 1, 2
+BF16, FP32 = 0, 1
+SCORE_LOSS, SCORE_ACCURACY, SCORE_RMSE = 0, 1, 2
+TASKS = {"binary": BINARY, "multiclass": MULTICLASS, "regression": REGRESSION}
+PRECISIONS = {"bf16": BF16, "fp32": FP32}
+SCORES = {"loss": SCORE_LOSS, "accuracy": SCORE_ACCURACY, "rmse": SCORE_RMSE}
+PHASES = ["gather", "fwd", "head", "bwd", "bias", "adamw", "predict"]
+
+# every entry point declared in include/tabpack.h
+SYMBOLS = ["pack_create", "pack_destroy", "pack_set_stream", "pack_train_step", "pack_forward_backward",
+           "pack_predict", "pack_select_greedy", "pack_set_active", "pack_get_params", "pack_set_params",
+           "pack_get_grads", "pack_get_logits", "pack_debug_masks", "pack_debug_activations", "pack_profile_enable",
+           "pack_profile_read", "pack_launch_count", "pack_sizes", "pack_last_error"]
+
+
+class TabpackError(RuntimeError):
+    def __init__(self, status, msg):
+        super().__init__(f"tabpack status {status}: {msg}")
+        self.status = status
+
+
+class Config(ctypes.Structure):
+    _fields_ = [("m", ctypes.c_int32), ("d_in", ctypes.c_int32), ("d_out", ctypes.c_int32),
+                ("max_batch", ctypes.c_int32), ("task", ctypes.c_int32), ("precision", ctypes.c_int32),
+                ("seed", ctypes.c_uint64), ("beta1", ctypes.c_float), ("beta2", ctypes.c_float),
+                ("eps", ctypes.c_float), ("wd_on_bias", ctypes.c_int32)]
+
+
+_lib = None
+
+
+def load_library(path: str = LIB_PATH):
+    """Load libtabpack.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise ImportError(f"libtabpack.so not built at {path}: run paper_2607_05380_gb300.build.build()")
+    L = ctypes.CDLL(path)
+    P, i32, i64, u32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32
+    st = ctypes.c_int
+    sig = {
+        "pack_create": (st, [ctypes.POINTER(Config), P, P, P, P, P, P, ctypes.POINTER(P)]),
+        "pack_destroy": (None, [P]),
+        "pack_set_stream": (st, [P, P]),
+        "pack_train_step": (st, [P, P, i64, P, P, i32, u32, P]),
+        "pack_forward_backward": (st, [P, P, i64, P, P, i32, u32, P]),
+        "pack_predict": (st, [P, P, i64, P]),
+        "pack_select_greedy": (st, [P, i32, i64, i32, P, i32, i32, i32, P, P, P, P]),
+        "pack_set_active": (st, [P, P]),
+        "pack_get_params": (st, [P, i32, i32, P, P]),
+        "pack_set_params": (st, [P, i32, i32, P, P]),
+        "pack_get_grads": (st, [P, i32, i32, P, P]),
+        "pack_get_logits": (st, [P, i32, P]),
+        "pack_debug_masks": (st, [P, i32, i32, u32, i32, P]),
+        "pack_debug_activations": (st, [P, i32, i32, P]),
+        "pack_profile_enable": (st, [P, i32]),
+        "pack_profile_read": (st, [P, P, P, i32]),
+        "pack_launch_count": (i64, [P]),
+        "pack_sizes": (st, [P, P, P]),
+        "pack_last_error": (ctypes.c_char_p, [P]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(L, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = L
+    return L
+
+
+def _check(status, handle=None):
+    if status != TP_OK:
+        msg = load_library().pack_last_error(handle)
+        raise TabpackError(status, msg.decode() if msg else "")
+
+
+def _dptr(t, dtype=None):
+    """Device pointer of a contiguous CUDA tensor (None for None)."""
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("expected a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError("expected a contiguous tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"expected {dtype}, got {t.dtype}")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _hptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _stream_ptr(stream):
+    if stream is None:
+        import torch
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+class Pack:
+    """A pack of m base MLPs with per-member hyperparameters on one GPU."""
+
+    def __init__(self, d_in, d_out, task, depth, width, dropout, lr, wd, max_batch, seed=2,
+                 precision="bf16", beta1=0.9, beta2=0.999, eps=1e-8, wd_on_bias=True, stream=None):
+        import torch
+        L = load_library()
+        self.torch = torch
+        self.depth = np.ascontiguousarray(depth, dtype=np.int32)
+        self.width = np.ascontiguousarray(width, dtype=np.int32)
+        self.m = len(self.depth)
+        self.d_in, self.d_out = int(d_in), int(d_out)
+        self.task = TASKS[task] if isinstance(task, str) else int(task)
+        self.precision = PRECISIONS[precision] if isinstance(precision, str) else int(precision)
+        cfg = Config(self.m, self.d_in, self.d_out, int(max_batch), self.task, self.precision, int(seed),
+                     beta1, beta2, eps, int(bool(wd_on_bias)))
+        drop = np.ascontiguousarray(dropout, dtype=np.float32)
+        lr_ = np.ascontiguousarray(lr, dtype=np.float32)
+        wd_ = np.ascontiguousarray(wd, dtype=np.float32)
+        h = ctypes.c_void_p()
+        _check(L.pack_create(ctypes.byref(cfg), _hptr(self.depth), _hptr(self.width), _hptr(drop), _hptr(lr_),
+                             _hptr(wd_), _stream_ptr(stream), ctypes.byref(h)))
+        self._h = h
+        self._B = 0
+
+    def close(self):
+        if getattr(self, "_h", None):
+            load_library().pack_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _y_dtype(self):
+        return self.torch.float32 if self.task == REGRESSION else self.torch.int32
+
+    def train_step(self, X, idx, y, step, loss_out=None, update=True):
+        """X float32 [n, d_in], idx int32 [B], y labels [n] (CUDA tensors);
+        loss_out: optional float32 [m] CUDA tensor."""
+        fn = load_library().pack_train_step if update else load_library().pack_forward_backward
+        t = self.torch
+        _check(fn(self._h, _dptr(X, t.float32), X.shape[0], _dptr(idx, t.int32), _dptr(y, self._y_dtype()),
+                  int(idx.shape[0]), int(step), _dptr(loss_out, t.float32)), self._h)
+        self._B = int(idx.shape[0])
+
+    def forward_backward(self, X, idx, y, step, loss_out=None):
+        self.train_step(X, idx, y, step, loss_out, update=False)
+
+    def predict(self, X, out=None):
+        t = self.torch
+        if out is None:
+            out = t.empty((self.m, X.shape[0], self.d_out), dtype=t.float32, device=X.device)
+        _check(load_library().pack_predict(self._h, _dptr(X, t.float32), X.shape[0], _dptr(out, t.float32)), self._h)
+        return out
+
+    def set_active(self, active):
+        a = np.ascontiguousarray(active, dtype=np.uint8)
+        _check(load_library().pack_set_active(self._h, _hptr(a)), self._h)
+
+    def layer_shape(self, member, layer):
+        L, w = int(self.depth[member]), int(self.width[member])
+        return (self.d_out if layer == L else w), (self.d_in if layer == 0 else w)
+
+    def _valid(self, member, layer):
+        return 0 <= member < self.m and 0 <= layer <= int(self.depth[member])
+
+    def _two(self, fn, member, layer):
+        if not self._valid(member, layer):   # let the library report the error
+            _check(fn(self._h, int(member), int(layer), None, None), self._h)
+        o, i = self.layer_shape(member, layer)
+        W = np.zeros((o, i), dtype=np.float32)
+        b = np.zeros(o, dtype=np.float32)
+        _check(fn(self._h, member, layer, _hptr(W), _hptr(b)), self._h)
+        return W, b
+
+    def get_params(self, member, layer):
+        return self._two(load_library().pack_get_params, member, layer)
+
+    def get_grads(self, member, layer):
+        return self._two(load_library().pack_get_grads, member, layer)
+
+    def set_params(self, member, layer, W, b):
+        if not self._valid(member, layer):
+            _check(load_library().pack_set_params(self._h, int(member), int(layer), None, None), self._h)
+        W = np.ascontiguousarray(W, dtype=np.float32)
+        b = np.ascontiguousarray(b, dtype=np.float32)
+        if W.shape != self.layer_shape(member, layer) or b.shape != (W.shape[0],):
+            raise ValueError("shape mismatch")
+        _check(load_library().pack_set_params(self._h, member, layer, _hptr(W), _hptr(b)), self._h)
+
+    def logits(self, member):
+        out = np.zeros((self._B, self.d_out), dtype=np.float32)
+        _check(load_library().pack_get_logits(self._h, member, _hptr(out)), self._h)
+        return out
+
+    def debug_masks(self, member, layer, step, B):
+        out = np.zeros((B, int(self.width[member])), dtype=np.uint8)
+        _check(load_library().pack_debug_masks(self._h, member, layer, int(step), int(B), _hptr(out)), self._h)
+        return out
+
+    def debug_activations(self, member, layer):
+        out = np.zeros((self._B, int(self.width[member])), dtype=np.float32)
+        _check(load_library().pack_debug_activations(self._h, member, layer, _hptr(out)), self._h)
+        return out
+
+    def profile_enable(self, on=True):
+        _check(load_library().pack_profile_enable(self._h, int(bool(on))), self._h)
+
+    def profile_read(self, reset=True):
+        ms = np.zeros(len(PHASES), dtype=np.float64)
+        n = np.zeros(len(PHASES), dtype=np.int64)
+        _check(load_library().pack_profile_read(self._h, _hptr(ms), _hptr(n), int(bool(reset))), self._h)
+        return {p: (float(ms[k]), int(n[k])) for k, p in enumerate(PHASES)}
+
+    def launch_count(self):
+        return int(load_library().pack_launch_count(self._h))
+
+    def sizes(self):
+        n = ctypes.c_int64()
+        b = ctypes.c_int64()
+        _check(load_library().pack_sizes(self._h, ctypes.byref(n), ctypes.byref(b)), self._h)
+        return n.value, b.value
+
+
+def select_greedy(preds, y, task, score="loss", m_ens=32, stream=None):
+    """Greedy ensemble selection on the GPU.  preds float32 [P, N, d_out] and
+    y [N] CUDA tensors.  Returns (selected indices, final score)."""
+    import torch
+    t = TASKS[task] if isinstance(task, str) else int(task)
+    s = SCORES[score] if isinstance(score, str) else int(score)
+    P, N, d_out = preds.shape
+    ydt = torch.float32 if t == REGRESSION else torch.int32
+    sel = np.zeros(m_ens, dtype=np.int32)
+    n = ctypes.c_int32()
+    fin = ctypes.c_double()
+    _check(load_library().pack_select_greedy(_dptr(preds, torch.float32), P, N, d_out, _dptr(y, ydt), t, s,
+                                             int(m_ens), _stream_ptr(stream), _hptr(sel), ctypes.byref(n),
+                                             ctypes.byref(fin)))
+    return sel[:n.value].copy(), fin.value

@@ -1,0 +1,501 @@
+// kernels.cu -- element-wise, reduction and CUDA-core matrix kernels of the
+// packed training step (gather, CUDA-core grouped GEMM, head + loss, bias
+// gradients, AdamW, init, predict head, mask dump).
+#include "kernels.cuh"
+
+namespace tp {
+
+// ------------------------------------------------------------------ gather
+// xb[b, k] = X[idx[b], k] for b < B, k < d_in; zeros elsewhere in [B_pad, d_in_pad].
+// Block 0 also advances the step count of every active member and stores the
+// AdamW bias corrections 1 - beta^t of the new step (when `advance`).
+template <typename T>
+__global__ void k_gather(const float* __restrict__ X, const int32_t* __restrict__ idx, int32_t B,
+                         int32_t B_pad, int32_t d_in, int32_t d_in_pad, T* __restrict__ xb,
+                         int32_t advance, int32_t* __restrict__ t_dev, float2* __restrict__ bias_corr,
+                         const int32_t* __restrict__ active_ids, int32_t n_active, float beta1,
+                         float beta2) {
+  if (advance && blockIdx.x == 0) {
+    for (int a = threadIdx.x; a < n_active; a += blockDim.x) {
+      int i = active_ids[a];
+      int t = t_dev[i] + 1;
+      t_dev[i] = t;
+      bias_corr[i] = make_float2((float)(1.0 - pow((double)beta1, (double)t)),
+                                 (float)(1.0 - pow((double)beta2, (double)t)));
+    }
+  }
+  const int64_t total = (int64_t)B_pad * d_in_pad;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    int b = (int)(e / d_in_pad), k = (int)(e % d_in_pad);
+    float v = 0.f;
+    if (b < B && k < d_in) {
+      int64_t row = idx ? (int64_t)idx[b] : (int64_t)b;
+      v = X[row * d_in + k];
+    }
+    xb[e] = Elem<T>::from_f(v);
+  }
+}
+
+// ------------------------------------------------------- CUDA-core GEMM
+// One 64 x 64 output tile per block, 256 threads, 4 x 4 outputs per thread,
+// k-slabs of 16 staged in shared memory.  Each output accumulates its k terms
+// in increasing k order with fused multiply-adds (fp32).
+template <typename T>
+__global__ void __launch_bounds__(256) k_gemm_simt(GemmArgs<T> g, int32_t tile_base) {
+  const GemmTile t = g.tiles[tile_base + blockIdx.x];
+  const GemmProblem P = g.probs[t.prob];
+  const int M = P.M ? P.M : g.B_pad;
+  const int N = P.N;
+  const int K = P.K ? P.K : g.B_pad;
+  if (t.m0 >= M) return;
+  const T* bases[4] = {g.xb, g.act, g.dz, g.wq};
+  const T* A = bases[P.a_src] + P.a_off;
+  const T* Bm = bases[P.b_src] + P.b_off;
+  int64_t a_rs, a_ks, b_rs, b_ks;
+  if (P.kind == kFwd) {
+    a_rs = P.lda; a_ks = 1; b_rs = P.ldb; b_ks = 1;
+  } else if (P.kind == kDgrad) {
+    a_rs = P.lda; a_ks = 1; b_rs = 1; b_ks = P.ldb;
+  } else {
+    a_rs = 1; a_ks = P.lda; b_rs = 1; b_ks = P.ldb;
+  }
+  __shared__ float As[16][68];
+  __shared__ float Bs[16][68];
+  float acc[4][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+  for (int k0 = 0; k0 < K; k0 += 16) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      int e = threadIdx.x + q * 256;
+      int r, kk;
+      if (a_ks == 1) { kk = e & 15; r = e >> 4; } else { r = e & 63; kk = e >> 6; }
+      int gr = t.m0 + r, gk = k0 + kk;
+      float v = 0.f;
+      if (gr < M && gk < K) v = Elem<T>::to_f(A[gr * a_rs + gk * a_ks]);
+      As[kk][r] = v;
+      int c, kb;
+      if (b_ks == 1) { kb = e & 15; c = e >> 4; } else { c = e & 63; kb = e >> 6; }
+      int gc = t.n0 + c, gkb = k0 + kb;
+      float u = 0.f;
+      if (gc < N && gkb < K) u = Elem<T>::to_f(Bm[gc * b_rs + gkb * b_ks]);
+      Bs[kb][c] = u;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < 16; ++kk) {
+      float a[4], b[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) a[i] = As[kk][ty + 16 * i];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) b[j] = Bs[kk][tx * 4 + j];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+  const int c0 = t.n0 + tx * 4;
+  if (c0 >= N) return;  // N is a multiple of 4, so c0 < N covers c0 .. c0 + 3
+  const MemberDev md = g.mem[P.member];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int r = t.m0 + ty + 16 * i;
+    if (r >= M) continue;
+    if (P.kind == kFwd) {
+      uint32_t keep = g.train ? keep_bits4(g.seed, (uint32_t)P.member, (uint32_t)P.layer, g.step,
+                                           (uint32_t)r, (uint32_t)(c0 >> 2), md.drop_T)
+                              : 0xFu;
+      const float sc = g.train ? md.scale : 1.f;
+      T* C = g.act + P.c_off;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        float z = acc[i][j] + g.params[P.aux_off + c0 + j];
+        float a = z > 0.f ? z : 0.f;
+        float h = ((keep >> j) & 1u) ? a * sc : 0.f;
+        C[(int64_t)r * P.ldc + c0 + j] = Elem<T>::from_f(h);
+      }
+    } else if (P.kind == kDgrad) {
+      const T* Hm = g.act + P.aux_off;
+      T* C = g.dz + P.c_off;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        int64_t o = (int64_t)r * P.ldc + c0 + j;
+        float h = Elem<T>::to_f(Hm[o]);
+        C[o] = Elem<T>::from_f(h > 0.f ? acc[i][j] * md.scale : 0.f);
+      }
+    } else {
+      float* C = g.grads + P.c_off;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) C[(int64_t)r * P.ldc + c0 + j] = acc[i][j];
+    }
+  }
+}
+
+// ------------------------------------------------------------- head + loss
+// One block per (member, 128-row block).  Warps compute one row's logits at
+// a time, then the per-row loss and d(mean loss)/d(logits); the block then
+// forms dZ of the last hidden layer and its partial head-weight gradient.
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+template <typename T, int DO>
+__global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
+  const HeadJob jb = g.jobs[blockIdx.x];
+  const int r0 = jb.blk * kRowTile;
+  if (r0 >= g.B_pad) return;
+  const MemberDev md = g.mem[jb.member];
+  const int w = md.w, d_out = g.d_out;
+  const T* H = g.act + jb.h_off;
+  const float* Wh = g.params + jb.w_off;
+  const float* bh = g.params + jb.b_off;
+  __shared__ float dlog[kRowTile][DO];
+  __shared__ float lrow[kRowTile];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float invB = 1.f / (float)g.B;
+  for (int rr = warp; rr < kRowTile; rr += 8) {
+    const int r = r0 + rr;
+    float acc[DO];
+#pragma unroll
+    for (int c = 0; c < DO; ++c) acc[c] = 0.f;
+    for (int j = lane; j < w; j += 32) {
+      float h = Elem<T>::to_f(H[(int64_t)r * w + j]);
+#pragma unroll
+      for (int c = 0; c < DO; ++c)
+        if (c < d_out) acc[c] = fmaf(h, Wh[(int64_t)c * w + j], acc[c]);
+    }
+#pragma unroll
+    for (int c = 0; c < DO; ++c)
+      if (c < d_out) acc[c] = warp_sum(acc[c]) + bh[c];
+    float loss = 0.f;
+    float dl[DO];
+#pragma unroll
+    for (int c = 0; c < DO; ++c) dl[c] = 0.f;
+    if (r < g.B) {
+      const int64_t row = g.idx ? (int64_t)g.idx[r] : (int64_t)r;
+      if (g.task == 1) {  // multiclass: softmax cross-entropy
+        const int yv = ((const int32_t*)g.y)[row];
+        float mx = acc[0];
+#pragma unroll
+        for (int c = 1; c < DO; ++c) if (c < d_out) mx = fmaxf(mx, acc[c]);
+        float s = 0.f;
+#pragma unroll
+        for (int c = 0; c < DO; ++c) if (c < d_out) s += expf(acc[c] - mx);
+        const float lse = mx + logf(s);
+        float zy = 0.f;
+#pragma unroll
+        for (int c = 0; c < DO; ++c)
+          if (c < d_out) {
+            if (c == yv) zy = acc[c];
+            dl[c] = (expf(acc[c] - lse) - (c == yv ? 1.f : 0.f)) * invB;
+          }
+        loss = lse - zy;
+      } else if (g.task == 0) {  // binary: logistic loss on one logit
+        const float yv = (float)((const int32_t*)g.y)[row];
+        const float x = acc[0];
+        loss = fmaxf(x, 0.f) - x * yv + log1pf(expf(-fabsf(x)));
+        dl[0] = (1.f / (1.f + expf(-x)) - yv) * invB;
+      } else {  // regression: squared error
+        const float d = acc[0] - ((const float*)g.y)[row];
+        loss = d * d;
+        dl[0] = 2.f * d * invB;
+      }
+      if (lane < d_out) {
+        float z = 0.f;
+#pragma unroll
+        for (int c = 0; c < DO; ++c) if (c == lane) z = acc[c];
+        g.logits[((int64_t)jb.member * g.B_cap + r) * d_out + lane] = z;
+      }
+    }
+    if (lane == 0) {
+#pragma unroll
+      for (int c = 0; c < DO; ++c) dlog[rr][c] = dl[c];
+      lrow[rr] = loss;
+    }
+  }
+  __syncthreads();
+  // dZ of the last hidden layer: (dlogits W_h) * [H > 0] / (1 - p)
+  T* dZ = g.dz + jb.dz_off;
+  for (int e = threadIdx.x; e < kRowTile * w; e += blockDim.x) {
+    const int rr = e / w, j = e % w;
+    const int64_t o = (int64_t)(r0 + rr) * w + j;
+    float s = 0.f;
+#pragma unroll
+    for (int c = 0; c < DO; ++c) if (c < d_out) s = fmaf(dlog[rr][c], Wh[(int64_t)c * w + j], s);
+    const float h = Elem<T>::to_f(H[o]);
+    dZ[o] = Elem<T>::from_f(h > 0.f ? s * md.scale : 0.f);
+  }
+  // partial head gradients of this block
+  float* part = g.head_part + jb.part_off;
+  for (int j = threadIdx.x; j < w; j += blockDim.x) {
+    float a[DO];
+#pragma unroll
+    for (int c = 0; c < DO; ++c) a[c] = 0.f;
+    for (int rr = 0; rr < kRowTile; ++rr) {
+      const float h = Elem<T>::to_f(H[(int64_t)(r0 + rr) * w + j]);
+#pragma unroll
+      for (int c = 0; c < DO; ++c) if (c < d_out) a[c] = fmaf(dlog[rr][c], h, a[c]);
+    }
+#pragma unroll
+    for (int c = 0; c < DO; ++c) if (c < d_out) part[(int64_t)c * w + j] = a[c];
+  }
+  if (threadIdx.x < d_out) {
+    float s = 0.f;
+    for (int rr = 0; rr < kRowTile; ++rr) s += dlog[rr][threadIdx.x];
+    part[(int64_t)d_out * w + threadIdx.x] = s;
+  }
+  if (threadIdx.x == 0) {
+    float s = 0.f;
+    for (int rr = 0; rr < kRowTile; ++rr) s += lrow[rr];
+    g.loss_part[(int64_t)jb.member * g.n_blk_cap + jb.blk] = s;
+  }
+}
+
+// Sum the per-block head partials (fixed order) into the head gradients and
+// the per-member mean loss.  One block per member; inactive members get NaN.
+__global__ void k_head_reduce(HeadReduceArgs g) {
+  const int i = blockIdx.x;
+  const HeadReduceJob jb = g.jobs[i];
+  const int n_blk = g.B_pad / kRowTile;
+  if (!g.active[i]) {
+    if (threadIdx.x == 0 && g.loss_out) g.loss_out[i] = __int_as_float(0x7fc00000);
+    return;
+  }
+  const int w = jb.w, d_out = g.d_out;
+  const int64_t stride = g.part_stride[i];
+  for (int e = threadIdx.x; e < d_out * w + d_out; e += blockDim.x) {
+    float s = 0.f;
+    for (int b = 0; b < n_blk; ++b) s += g.head_part[jb.part_off + b * stride + e];
+    if (e < d_out * w) g.grads[jb.gw_off + e] = s;
+    else g.grads[jb.gb_off + (e - d_out * w)] = s;
+  }
+  if (threadIdx.x == 0) {
+    float s = 0.f;
+    for (int b = 0; b < n_blk; ++b) s += g.loss_part[(int64_t)i * g.n_blk_cap + b];
+    const float loss = s / (float)g.B;
+    if (g.loss_out) g.loss_out[i] = loss;
+    g.loss_last[i] = loss;
+  }
+}
+
+// ------------------------------------------------------------- bias grads
+// db_l[c] = sum over the B_pad batch rows of dZ_l[r, c] (padded rows are 0).
+template <typename T>
+__global__ void k_bias_grad(const BiasJob* __restrict__ jobs, const T* __restrict__ dz,
+                            float* __restrict__ grads, int32_t B_pad) {
+  const BiasJob jb = jobs[blockIdx.x];
+  const int c = jb.c0 + threadIdx.x;
+  if (c >= jb.w) return;
+  const T* z = dz + jb.dz_off + c;
+  float s = 0.f;
+  for (int r = 0; r < B_pad; ++r) s += Elem<T>::to_f(z[(int64_t)r * jb.w]);
+  grads[jb.b_off + c] = s;
+}
+
+// ------------------------------------------------------------------ AdamW
+// Per element of the chunk, with the member's lr and wd and its step's bias
+// corrections (bc1, bc2) = (1 - beta1^t, 1 - beta2^t):
+//   p <- p - lr wd p;  m <- b1 m + (1 - b1) g;  v <- b2 v + (1 - b2) g^2;
+//   p <- p - lr (m / bc1) / (sqrt(v / bc2) + eps)
+// and the bf16 copy of p (bf16 mode).
+__global__ void __launch_bounds__(256) k_adamw(AdamArgs g) {
+  const Chunk ch = g.chunks[blockIdx.x];
+  const Segment s = g.segs[ch.seg];
+  const MemberDev md = g.mem[s.member];
+  const float2 bc = g.bias_corr[s.member];
+  const float lr = md.lr;
+  const float wd = (s.is_bias && !g.wd_on_bias) ? 0.f : md.wd;
+  const float b1 = g.beta1, b2 = g.beta2, eps = g.eps;
+  const float ib1 = 1.f / bc.x, ib2 = 1.f / bc.y;
+  for (int e = threadIdx.x; e < ch.len; e += blockDim.x) {
+    const int64_t o = ch.off + e;
+    float p = g.params[o], gr = g.grads[o], m = g.m[o], v = g.v[o];
+    p = p - lr * wd * p;
+    m = b1 * m + (1.f - b1) * gr;
+    v = b2 * v + (1.f - b2) * gr * gr;
+    p = p - lr * (m * ib1) / (sqrtf(v * ib2) + eps);
+    g.params[o] = p;
+    g.m[o] = m;
+    g.v[o] = v;
+    if (g.wq) g.wq[o] = __float2bfloat16_rn(p);
+  }
+}
+
+// ------------------------------------------------------------------- init
+// Element of the padded arena -> the oracle's element index within the layer
+// (weights row-major unpadded, then biases) -> Philox word -> U(-b, b), fp32.
+__global__ void k_init(InitArgs g) {
+  const Chunk ch = g.chunks[blockIdx.x];
+  const Segment s = g.segs[ch.seg];
+  for (int e = threadIdx.x; e < ch.len; e += blockDim.x) {
+    const int64_t o = ch.off + e;
+    const int64_t local = o - s.off;
+    float val = 0.f;
+    bool real = true;
+    uint32_t idx;
+    if (s.is_bias) {
+      idx = (uint32_t)(s.w_elems + local);
+    } else {
+      const int64_t row = local / s.cols_pad, col = local % s.cols_pad;
+      real = col < s.cols;
+      idx = (uint32_t)(row * s.cols + col);
+    }
+    if (real) {
+      U4 r4 = philox10(idx >> 2, 0u, 0u, (1u << 28) | ((uint32_t)s.member << 4) | (uint32_t)s.layer,
+                       (uint32_t)g.seed, (uint32_t)(g.seed >> 32));
+      const uint32_t q = idx & 3u;
+      const uint32_t r = q == 0 ? r4.x : q == 1 ? r4.y : q == 2 ? r4.z : r4.w;
+      const double u = ((double)(r >> 8) + 0.5) * 5.9604644775390625e-08;  // 2^-24
+      const double bound = 1.0 / sqrt((double)s.fan_in);
+      val = (float)((2.0 * u - 1.0) * bound);
+    }
+    g.params[o] = val;
+    g.grads[o] = 0.f;
+    g.m[o] = 0.f;
+    g.v[o] = 0.f;
+    if (g.wq) g.wq[o] = __float2bfloat16_rn(val);
+  }
+}
+
+// bf16 copy of the whole arena (after pack_set_params).
+__global__ void k_refresh_wq(const float* __restrict__ p, __nv_bfloat16* __restrict__ wq, int64_t n) {
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x)
+    wq[e] = __float2bfloat16_rn(p[e]);
+}
+
+// ----------------------------------------------------------- predict head
+// Forward-only head: probabilities (softmax / sigmoid) or values into
+// out[member, n0 + r, :] for r < rows.
+template <typename T, int DO>
+__global__ void __launch_bounds__(256) k_predict_head(PredictHeadArgs<T> g) {
+  const HeadJob jb = g.jobs[blockIdx.x];
+  const int r0 = jb.blk * kRowTile;
+  if (r0 >= g.rows) return;
+  const MemberDev md = g.mem[jb.member];
+  const int w = md.w, d_out = g.d_out;
+  const T* H = g.act + jb.h_off;
+  const float* Wh = g.params + jb.w_off;
+  const float* bh = g.params + jb.b_off;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int rr = warp; rr < kRowTile; rr += 8) {
+    const int r = r0 + rr;
+    if (r >= g.rows) break;
+    float acc[DO];
+#pragma unroll
+    for (int c = 0; c < DO; ++c) acc[c] = 0.f;
+    for (int j = lane; j < w; j += 32) {
+      float h = Elem<T>::to_f(H[(int64_t)r * w + j]);
+#pragma unroll
+      for (int c = 0; c < DO; ++c)
+        if (c < d_out) acc[c] = fmaf(h, Wh[(int64_t)c * w + j], acc[c]);
+    }
+#pragma unroll
+    for (int c = 0; c < DO; ++c)
+      if (c < d_out) acc[c] = warp_sum(acc[c]) + bh[c];
+    float* o = g.out + ((int64_t)jb.member * g.N + g.n0 + r) * d_out;
+    if (g.task == 1) {
+      float mx = acc[0];
+#pragma unroll
+      for (int c = 1; c < DO; ++c) if (c < d_out) mx = fmaxf(mx, acc[c]);
+      float s = 0.f;
+#pragma unroll
+      for (int c = 0; c < DO; ++c) if (c < d_out) s += expf(acc[c] - mx);
+      const float inv = 1.f / s;
+#pragma unroll
+      for (int c = 0; c < DO; ++c)
+        if (c < d_out && c == lane) o[c] = expf(acc[c] - mx) * inv;
+    } else if (lane == 0) {
+      o[0] = g.task == 0 ? 1.f / (1.f + expf(-acc[0])) : acc[0];
+    }
+  }
+}
+
+// ------------------------------------------------------------- mask dump
+__global__ void k_debug_masks(uint8_t* __restrict__ out, int32_t B, int32_t w, uint64_t seed,
+                              uint32_t member, uint32_t layer, uint32_t step, uint32_t T) {
+  const int64_t n4 = (int64_t)B * (w / 4);
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n4; e += (int64_t)gridDim.x * blockDim.x) {
+    const int r = (int)(e / (w / 4)), c4 = (int)(e % (w / 4));
+    const uint32_t k = keep_bits4(seed, member, layer, step, (uint32_t)r, (uint32_t)c4, T);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) out[(int64_t)r * w + c4 * 4 + q] = (uint8_t)((k >> q) & 1u);
+  }
+}
+
+// ------------------------------------------------------------- launchers
+template <typename T>
+void launch_gather(cudaStream_t st, const float* X, const int32_t* idx, int B, int B_pad, int d_in,
+                   int d_in_pad, T* xb, int advance, int32_t* t_dev, float2* bias_corr,
+                   const int32_t* active_ids, int n_active, float beta1, float beta2) {
+  int64_t total = (int64_t)B_pad * d_in_pad;
+  int blocks = (int)std::min<int64_t>(ceil_div(total, 256), 152 * 8);
+  if (blocks < 1) blocks = 1;
+  k_gather<T><<<blocks, 256, 0, st>>>(X, idx, B, B_pad, d_in, d_in_pad, xb, advance, t_dev, bias_corr,
+                                       active_ids, n_active, beta1, beta2);
+}
+
+template <typename T>
+void launch_gemm_simt(cudaStream_t st, const GemmArgs<T>& g, int tile_base, int n_tiles) {
+  if (n_tiles > 0) k_gemm_simt<T><<<n_tiles, 256, 0, st>>>(g, tile_base);
+}
+
+template <typename T>
+void launch_head(cudaStream_t st, const HeadArgs<T>& g, int n_jobs) {
+  if (n_jobs <= 0) return;
+  if (g.d_out == 1) k_head<T, 1><<<n_jobs, 256, 0, st>>>(g);
+  else k_head<T, kMaxDout><<<n_jobs, 256, 0, st>>>(g);
+}
+
+void launch_head_reduce(cudaStream_t st, const HeadReduceArgs& g, int m) {
+  k_head_reduce<<<m, 256, 0, st>>>(g);
+}
+
+template <typename T>
+void launch_bias_grad(cudaStream_t st, const BiasJob* jobs, int n_jobs, const T* dz, float* grads, int B_pad) {
+  if (n_jobs > 0) k_bias_grad<T><<<n_jobs, 128, 0, st>>>(jobs, dz, grads, B_pad);
+}
+
+void launch_adamw(cudaStream_t st, const AdamArgs& g, int n_chunks) {
+  if (n_chunks > 0) k_adamw<<<n_chunks, 256, 0, st>>>(g);
+}
+
+void launch_init(cudaStream_t st, const InitArgs& g, int n_chunks) {
+  if (n_chunks > 0) k_init<<<n_chunks, 256, 0, st>>>(g);
+}
+
+void launch_refresh_wq(cudaStream_t st, const float* p, __nv_bfloat16* wq, int64_t n) {
+  k_refresh_wq<<<152 * 4, 256, 0, st>>>(p, wq, n);
+}
+
+template <typename T>
+void launch_predict_head(cudaStream_t st, const PredictHeadArgs<T>& g, int n_jobs) {
+  if (n_jobs <= 0) return;
+  if (g.d_out == 1) k_predict_head<T, 1><<<n_jobs, 256, 0, st>>>(g);
+  else k_predict_head<T, kMaxDout><<<n_jobs, 256, 0, st>>>(g);
+}
+
+void launch_debug_masks(cudaStream_t st, uint8_t* out, int B, int w, uint64_t seed, uint32_t member,
+                        uint32_t layer, uint32_t step, uint32_t T) {
+  k_debug_masks<<<64, 256, 0, st>>>(out, B, w, seed, member, layer, step, T);
+}
+
+#define TP_INSTANTIATE(T)                                                                        \
+  template void launch_gather<T>(cudaStream_t, const float*, const int32_t*, int, int, int, int, T*, \
+                                 int, int32_t*, float2*, const int32_t*, int, float, float);      \
+  template void launch_gemm_simt<T>(cudaStream_t, const GemmArgs<T>&, int, int);                 \
+  template void launch_head<T>(cudaStream_t, const HeadArgs<T>&, int);                           \
+  template void launch_bias_grad<T>(cudaStream_t, const BiasJob*, int, const T*, float*, int);   \
+  template void launch_predict_head<T>(cudaStream_t, const PredictHeadArgs<T>&, int);
+
+TP_INSTANTIATE(float)
+TP_INSTANTIATE(__nv_bfloat16)
+
+}  // namespace tp

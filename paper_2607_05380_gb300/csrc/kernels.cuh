@@ -1,0 +1,122 @@
+// kernels.cuh -- kernel argument blocks and launchers of the tabpack library.
+#pragma once
+
+#include <algorithm>
+
+#include "tp_internal.cuh"
+
+namespace tp {
+
+template <typename T>
+struct GemmArgs {
+  const GemmProblem* probs;
+  const GemmTile* tiles;
+  const T* xb;
+  T* act;
+  T* dz;
+  const T* wq;            // matrix-product copy of the weights (bf16 copy, or the fp32 params)
+  const float* params;    // fp32 master (biases)
+  float* grads;
+  const MemberDev* mem;
+  int32_t B, B_pad;
+  uint32_t step;
+  int32_t train;          // 1: dropout on
+  uint64_t seed;
+};
+
+template <typename T>
+struct HeadArgs {
+  const HeadJob* jobs;
+  const MemberDev* mem;
+  const T* act;
+  T* dz;
+  const float* params;
+  float* head_part;
+  float* loss_part;
+  float* logits;          // [m, B_cap, d_out]
+  const int32_t* idx;
+  const void* y;
+  int32_t B, B_pad, B_cap, d_out, task, n_blk_cap;
+};
+
+struct HeadReduceArgs {
+  const HeadReduceJob* jobs;
+  const uint8_t* active;
+  const int64_t* part_stride;
+  const float* head_part;
+  const float* loss_part;
+  float* grads;
+  float* loss_out;        // caller's [m] or NULL
+  float* loss_last;       // pack's own copy [m]
+  int32_t B, B_pad, d_out, n_blk_cap;
+};
+
+struct AdamArgs {
+  const Chunk* chunks;
+  const Segment* segs;
+  const MemberDev* mem;
+  const float2* bias_corr;
+  float* params;
+  const float* grads;
+  float* m;
+  float* v;
+  __nv_bfloat16* wq;      // NULL in fp32 mode
+  float beta1, beta2, eps;
+  int32_t wd_on_bias;
+};
+
+struct InitArgs {
+  const Chunk* chunks;
+  const Segment* segs;
+  float* params;
+  float* grads;
+  float* m;
+  float* v;
+  __nv_bfloat16* wq;
+  uint64_t seed;
+};
+
+template <typename T>
+struct PredictHeadArgs {
+  const HeadJob* jobs;
+  const MemberDev* mem;
+  const T* act;
+  const float* params;
+  float* out;
+  int64_t N, n0;
+  int32_t rows, d_out, task, _pad;
+};
+
+template <typename T>
+void launch_gather(cudaStream_t st, const float* X, const int32_t* idx, int B, int B_pad, int d_in,
+                   int d_in_pad, T* xb, int advance, int32_t* t_dev, float2* bias_corr,
+                   const int32_t* active_ids, int n_active, float beta1, float beta2);
+template <typename T>
+void launch_gemm_simt(cudaStream_t st, const GemmArgs<T>& g, int tile_base, int n_tiles);
+template <typename T>
+void launch_head(cudaStream_t st, const HeadArgs<T>& g, int n_jobs);
+void launch_head_reduce(cudaStream_t st, const HeadReduceArgs& g, int m);
+template <typename T>
+void launch_bias_grad(cudaStream_t st, const BiasJob* jobs, int n_jobs, const T* dz, float* grads, int B_pad);
+void launch_adamw(cudaStream_t st, const AdamArgs& g, int n_chunks);
+void launch_init(cudaStream_t st, const InitArgs& g, int n_chunks);
+void launch_refresh_wq(cudaStream_t st, const float* p, __nv_bfloat16* wq, int64_t n);
+template <typename T>
+void launch_predict_head(cudaStream_t st, const PredictHeadArgs<T>& g, int n_jobs);
+void launch_debug_masks(cudaStream_t st, uint8_t* out, int B, int w, uint64_t seed, uint32_t member,
+                        uint32_t layer, uint32_t step, uint32_t T);
+
+// greedy selection (select.cu)
+struct SelectScratch {
+  double* S;              // running ensemble sum [N, d_out]
+  double* partial;        // [P, n_blk]
+  int32_t* state;         // [4 + m_ens + P]: n, done, last, pad | selected | used
+  double* cur;            // [1]: current score
+};
+int64_t select_scratch_bytes(int32_t P, int64_t N, int32_t d_out, int32_t m_ens);
+SelectScratch select_carve(void* base, int32_t P, int64_t N, int32_t d_out, int32_t m_ens);
+int select_enqueue(cudaStream_t st, const SelectScratch& s, const float* preds, int32_t P, int64_t N,
+                   int32_t d_out, const void* y, int32_t task, int32_t score, int32_t m_ens,
+                   int64_t* launches);
+
+}  // namespace tp

@@ -1,0 +1,843 @@
+// tabpack.cu -- host side of the C ABI declared in include/tabpack.h: pack
+// layout, schedule construction (which member/layer/tile runs in which
+// launch), the step orchestration on the pack's stream, and error handling.
+#include <cuda_runtime.h>
+
+#include <array>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "kernels.cuh"
+#include "tabpack.h"
+#include "tc_gemm.cuh"
+
+using namespace tp;
+
+namespace {
+
+thread_local std::string g_thread_error;
+
+struct PhaseEvents {
+  std::vector<cudaEvent_t> pool;
+  std::vector<std::pair<int, int>> pending;  // (phase, event index of start; stop = +1)
+  double ms[TP_PH_COUNT] = {0};
+  int64_t launches[TP_PH_COUNT] = {0};
+};
+
+}  // namespace
+
+struct tabpack {
+  tp_config cfg{};
+  int d_in_pad = 0, B_cap = 0, n_blk_cap = 0, Lmax = 0;
+  cudaStream_t st = nullptr;
+  bool bf16 = true;
+  std::vector<int32_t> depth, width;
+  std::vector<float> dropout, lr, wd;
+  std::vector<std::array<int64_t, kMaxDepth + 1>> W_off, b_off;
+  std::vector<std::array<int64_t, kMaxDepth>> act_off, dz_off;
+  std::vector<uint8_t> active;
+  std::vector<Segment> segs;
+  std::vector<MemberDev> mem;
+  std::vector<int64_t> part_off, part_stride;
+  int64_t n_params = 0, act_elems = 0, dz_elems = 0, xb_elems = 0, head_part_elems = 0;
+  size_t elem = 2;
+
+  // device memory
+  float *params = nullptr, *grads = nullptr, *adam_m = nullptr, *adam_v = nullptr;
+  __nv_bfloat16* wq = nullptr;
+  void *xb = nullptr, *act = nullptr, *dz = nullptr;
+  float *logits = nullptr, *head_part = nullptr, *loss_part = nullptr, *loss_last = nullptr;
+  int32_t* t_dev = nullptr;
+  float2* bias_corr = nullptr;
+  uint8_t* active_dev = nullptr;
+  int32_t* active_ids_dev = nullptr;
+  MemberDev* mem_dev = nullptr;
+  Segment* segs_dev = nullptr;
+  Chunk* chunks_dev = nullptr;
+  GemmProblem* probs_dev = nullptr;
+  GemmTile* tiles_dev = nullptr;
+  HeadJob* head_jobs_dev = nullptr;
+  HeadReduceJob* hred_dev = nullptr;
+  int64_t* part_stride_dev = nullptr;
+  BiasJob* bias_jobs_dev = nullptr;
+  TcPlan tc;  // tensor-core GEMM plan (bf16 mode)
+
+  // schedule (active members)
+  int n_active = 0, n_chunks = 0, n_head_jobs = 0, n_bias_jobs = 0;
+  std::vector<std::pair<int, int>> fwd_rng, bwd_rng;  // tile ranges per depth index
+  int cap_chunks = 0, cap_probs = 0, cap_tiles = 0, cap_head = 0, cap_bias = 0;
+
+  int last_B = 0;
+  int64_t launches = 0;
+  size_t dev_bytes = 0;
+  std::vector<void*> allocs;
+  std::string err;
+  bool profiling = false;
+  PhaseEvents prof;
+};
+
+namespace {
+
+tp_status fail(tabpack* h, tp_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  if (h) h->err = buf;
+  else g_thread_error = buf;
+  return s;
+}
+
+#define TP_CUDA(h, call)                                                                   \
+  do {                                                                                     \
+    cudaError_t e_ = (call);                                                               \
+    if (e_ != cudaSuccess)                                                                 \
+      return fail((h), e_ == cudaErrorMemoryAllocation ? TP_ENOMEM : TP_ECUDA, "%s: %s (%s:%d)", \
+                  #call, cudaGetErrorString(e_), __FILE__, __LINE__);                      \
+  } while (0)
+
+#define TP_LAUNCHED(h)                                                                     \
+  do {                                                                                     \
+    cudaError_t e_ = cudaGetLastError();                                                   \
+    if (e_ != cudaSuccess)                                                                 \
+      return fail((h), TP_ECUDA, "kernel launch: %s (%s:%d)", cudaGetErrorString(e_), __FILE__, __LINE__); \
+  } while (0)
+
+template <typename P>
+tp_status dalloc(tabpack* h, P** ptr, size_t bytes) {
+  void* p = nullptr;
+  if (bytes == 0) bytes = 16;
+  cudaError_t e = cudaMalloc(&p, bytes);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return fail(h, TP_ENOMEM, "cudaMalloc(%zu bytes): %s", bytes, cudaGetErrorString(e));
+  }
+  h->allocs.push_back(p);
+  h->dev_bytes += bytes;
+  *ptr = (P*)p;
+  return TP_OK;
+}
+
+#define TP_TRY(expr)                 \
+  do {                               \
+    tp_status s_ = (expr);           \
+    if (s_ != TP_OK) return s_;      \
+  } while (0)
+
+void prof_begin(tabpack* h, int phase, int* slot) {
+  *slot = -1;
+  if (!h->profiling) return;
+  auto& P = h->prof;
+  int idx = (int)P.pending.size() * 2;
+  while ((int)P.pool.size() < idx + 2) {
+    cudaEvent_t e;
+    cudaEventCreate(&e);
+    P.pool.push_back(e);
+  }
+  cudaEventRecord(P.pool[idx], h->st);
+  P.pending.push_back({phase, idx});
+  *slot = idx;
+}
+
+void prof_end(tabpack* h, int slot, int n_launch, int phase) {
+  if (slot < 0) return;
+  cudaEventRecord(h->prof.pool[slot + 1], h->st);
+  h->prof.launches[phase] += n_launch;
+}
+
+void prof_flush(tabpack* h) {
+  auto& P = h->prof;
+  if (P.pending.empty()) return;
+  cudaStreamSynchronize(h->st);
+  for (auto& pr : P.pending) {
+    float ms = 0.f;
+    cudaEventElapsedTime(&ms, P.pool[pr.second], P.pool[pr.second + 1]);
+    P.ms[pr.first] += ms;
+  }
+  P.pending.clear();
+}
+
+// ------------------------------------------------------------------ layout
+tp_status build_layout(tabpack* h) {
+  const auto& c = h->cfg;
+  const int m = c.m;
+  h->d_in_pad = (int)round_up(c.d_in, 8);
+  h->B_cap = (int)round_up(c.max_batch, kRowTile);
+  h->n_blk_cap = h->B_cap / kRowTile;
+  h->W_off.resize(m);
+  h->b_off.resize(m);
+  h->act_off.resize(m);
+  h->dz_off.resize(m);
+  h->mem.resize(m);
+  h->part_off.resize(m);
+  h->part_stride.resize(m);
+  int64_t off = 0, aoff = 0, hoff = 0;
+  h->Lmax = 0;
+  for (int i = 0; i < m; ++i) {
+    const int L = h->depth[i], w = h->width[i];
+    h->Lmax = std::max(h->Lmax, L);
+    for (int l = 0; l <= L; ++l) {
+      const int in = l == 0 ? c.d_in : w, in_pad = l == 0 ? h->d_in_pad : w;
+      const int out = l == L ? c.d_out : w;
+      off = round_up(off, kSegAlign);
+      h->W_off[i][l] = off;
+      h->segs.push_back(Segment{off, i, l, out, in, in_pad, 0, in, out * in});
+      off += (int64_t)out * in_pad;
+      off = round_up(off, kSegAlign);
+      h->b_off[i][l] = off;
+      h->segs.push_back(Segment{off, i, l, out, 1, 1, 1, in, out * in});
+      off += out;
+    }
+    for (int l = 0; l < L; ++l) {
+      h->act_off[i][l] = aoff;
+      aoff += round_up((int64_t)h->B_cap * w, 128);
+      h->dz_off[i][l] = aoff;  // dz uses its own arena; same offsets scheme
+    }
+    const float p = h->dropout[i];
+    double T = std::floor((double)p * 4294967296.0);
+    if (T > 4294967295.0) T = 4294967295.0;
+    MemberDev md;
+    md.L = L;
+    md.w = w;
+    md.p = p;
+    md.scale = 1.f / (1.f - p);
+    md.lr = h->lr[i];
+    md.wd = h->wd[i];
+    md.drop_T = (uint32_t)T;
+    md._pad = 0;
+    h->mem[i] = md;
+    h->part_stride[i] = round_up((int64_t)c.d_out * (w + 1), 32);
+    h->part_off[i] = hoff;
+    hoff += h->part_stride[i] * h->n_blk_cap;
+  }
+  for (int i = 0; i < m; ++i)
+    for (int l = 0; l < h->depth[i]; ++l) h->dz_off[i][l] = h->act_off[i][l];
+  h->n_params = round_up(off, kSegAlign);
+  h->act_elems = std::max<int64_t>(aoff, 128);
+  h->dz_elems = h->act_elems;
+  h->xb_elems = (int64_t)h->B_cap * h->d_in_pad;
+  h->head_part_elems = std::max<int64_t>(hoff, 32);
+  return TP_OK;
+}
+
+// --------------------------------------------------------------- schedule
+// Rebuilt whenever the active set changes: per depth index the forward and
+// backward GEMM work of the active members, head / bias / AdamW work lists.
+tp_status build_schedule(tabpack* h) {
+  const auto& c = h->cfg;
+  const int m = c.m;
+  std::vector<int32_t> ids;
+  for (int i = 0; i < m; ++i)
+    if (h->active[i]) ids.push_back(i);
+  h->n_active = (int)ids.size();
+
+  std::vector<GemmProblem> probs;
+  std::vector<GemmTile> tiles;
+  h->fwd_rng.assign(h->Lmax, {0, 0});
+  h->bwd_rng.assign(h->Lmax, {0, 0});
+  auto add_tiles = [&](int prob, int M_rows, int N) {
+    const int tm = 64, tn = 64;
+    for (int m0 = 0; m0 < M_rows; m0 += tm)
+      for (int n0 = 0; n0 < N; n0 += tn) tiles.push_back(GemmTile{prob, m0, n0, std::min(tn, N - n0)});
+  };
+  for (int l = 0; l < h->Lmax; ++l) {
+    const int base = (int)tiles.size();
+    for (int i : ids) {
+      if (h->depth[i] <= l) continue;
+      const int w = h->width[i];
+      GemmProblem P{};
+      P.kind = kFwd; P.member = i; P.layer = l;
+      P.M = 0; P.N = w; P.K = l == 0 ? h->d_in_pad : w;
+      P.a_src = l == 0 ? kSrcXb : kSrcAct;
+      P.a_off = l == 0 ? 0 : h->act_off[i][l - 1];
+      P.lda = l == 0 ? h->d_in_pad : w;
+      P.b_src = kSrcWq; P.b_off = h->W_off[i][l]; P.ldb = P.K;
+      P.c_off = h->act_off[i][l]; P.ldc = w;
+      P.aux_off = h->b_off[i][l];
+      probs.push_back(P);
+      add_tiles((int)probs.size() - 1, h->B_cap, w);
+    }
+    h->fwd_rng[l] = {base, (int)tiles.size() - base};
+  }
+  for (int l = h->Lmax - 1; l >= 0; --l) {
+    const int base = (int)tiles.size();
+    for (int i : ids) {
+      if (h->depth[i] <= l) continue;
+      const int w = h->width[i];
+      const int in_pad = l == 0 ? h->d_in_pad : w;
+      if (l > 0) {
+        GemmProblem P{};
+        P.kind = kDgrad; P.member = i; P.layer = l;
+        P.M = 0; P.N = w; P.K = w;
+        P.a_src = kSrcDz; P.a_off = h->dz_off[i][l]; P.lda = w;
+        P.b_src = kSrcWq; P.b_off = h->W_off[i][l]; P.ldb = w;
+        P.c_off = h->dz_off[i][l - 1]; P.ldc = w;
+        P.aux_off = h->act_off[i][l - 1];
+        probs.push_back(P);
+        add_tiles((int)probs.size() - 1, h->B_cap, w);
+      }
+      GemmProblem Q{};
+      Q.kind = kWgrad; Q.member = i; Q.layer = l;
+      Q.M = w; Q.N = in_pad; Q.K = 0;
+      Q.a_src = kSrcDz; Q.a_off = h->dz_off[i][l]; Q.lda = w;
+      Q.b_src = l == 0 ? kSrcXb : kSrcAct; Q.b_off = l == 0 ? 0 : h->act_off[i][l - 1];
+      Q.ldb = in_pad;
+      Q.c_off = h->W_off[i][l]; Q.ldc = in_pad;
+      probs.push_back(Q);
+      add_tiles((int)probs.size() - 1, w, in_pad);
+    }
+    h->bwd_rng[l] = {base, (int)tiles.size() - base};
+  }
+
+  std::vector<HeadJob> hj;
+  std::vector<HeadReduceJob> hr(m);
+  for (int i = 0; i < m; ++i) {
+    const int L = h->depth[i];
+    hr[i] = HeadReduceJob{i, h->n_blk_cap, h->part_off[i], h->W_off[i][L], h->b_off[i][L], h->width[i], 0};
+  }
+  for (int i : ids) {
+    const int L = h->depth[i];
+    for (int b = 0; b < h->n_blk_cap; ++b)
+      hj.push_back(HeadJob{i, b, h->act_off[i][L - 1], h->dz_off[i][L - 1], h->W_off[i][L], h->b_off[i][L],
+                           h->part_off[i] + b * h->part_stride[i]});
+  }
+  std::vector<BiasJob> bj;
+  for (int i : ids)
+    for (int l = 0; l < h->depth[i]; ++l)
+      for (int c0 = 0; c0 < h->width[i]; c0 += 128)
+        bj.push_back(BiasJob{h->dz_off[i][l], h->b_off[i][l], h->width[i], c0});
+  std::vector<Chunk> ch;
+  for (int s = 0; s < (int)h->segs.size(); ++s) {
+    const Segment& S = h->segs[s];
+    if (!h->active[S.member]) continue;
+    const int64_t len = S.is_bias ? S.rows : (int64_t)S.rows * S.cols_pad;
+    for (int64_t o = 0; o < len; o += 4096)
+      ch.push_back(Chunk{S.off + o, (int32_t)std::min<int64_t>(4096, len - o), s});
+  }
+
+  // capacities are fixed at create (all members active)
+  if (h->probs_dev == nullptr) {
+    h->cap_probs = (int)probs.size() + 1;
+    h->cap_tiles = (int)tiles.size() + 1;
+    h->cap_head = (int)hj.size() + 1;
+    h->cap_bias = (int)bj.size() + 1;
+    h->cap_chunks = (int)ch.size() + 1;
+    TP_TRY(dalloc(h, &h->probs_dev, sizeof(GemmProblem) * h->cap_probs));
+    TP_TRY(dalloc(h, &h->tiles_dev, sizeof(GemmTile) * h->cap_tiles));
+    TP_TRY(dalloc(h, &h->head_jobs_dev, sizeof(HeadJob) * h->cap_head));
+    TP_TRY(dalloc(h, &h->hred_dev, sizeof(HeadReduceJob) * m));
+    TP_TRY(dalloc(h, &h->bias_jobs_dev, sizeof(BiasJob) * h->cap_bias));
+    TP_TRY(dalloc(h, &h->chunks_dev, sizeof(Chunk) * h->cap_chunks));
+    TP_TRY(dalloc(h, &h->active_ids_dev, sizeof(int32_t) * m));
+  }
+  if ((int)probs.size() > h->cap_probs || (int)tiles.size() > h->cap_tiles || (int)hj.size() > h->cap_head ||
+      (int)bj.size() > h->cap_bias || (int)ch.size() > h->cap_chunks)
+    return fail(h, TP_ESTATE, "schedule grew beyond its capacity");
+  TP_CUDA(h, cudaStreamSynchronize(h->st));
+  if (!probs.empty()) TP_CUDA(h, cudaMemcpy(h->probs_dev, probs.data(), sizeof(GemmProblem) * probs.size(), cudaMemcpyHostToDevice));
+  if (!tiles.empty()) TP_CUDA(h, cudaMemcpy(h->tiles_dev, tiles.data(), sizeof(GemmTile) * tiles.size(), cudaMemcpyHostToDevice));
+  if (!hj.empty()) TP_CUDA(h, cudaMemcpy(h->head_jobs_dev, hj.data(), sizeof(HeadJob) * hj.size(), cudaMemcpyHostToDevice));
+  TP_CUDA(h, cudaMemcpy(h->hred_dev, hr.data(), sizeof(HeadReduceJob) * m, cudaMemcpyHostToDevice));
+  if (!bj.empty()) TP_CUDA(h, cudaMemcpy(h->bias_jobs_dev, bj.data(), sizeof(BiasJob) * bj.size(), cudaMemcpyHostToDevice));
+  if (!ch.empty()) TP_CUDA(h, cudaMemcpy(h->chunks_dev, ch.data(), sizeof(Chunk) * ch.size(), cudaMemcpyHostToDevice));
+  if (!ids.empty()) TP_CUDA(h, cudaMemcpy(h->active_ids_dev, ids.data(), sizeof(int32_t) * ids.size(), cudaMemcpyHostToDevice));
+  TP_CUDA(h, cudaMemcpy(h->active_dev, h->active.data(), m, cudaMemcpyHostToDevice));
+  h->n_head_jobs = (int)hj.size();
+  h->n_bias_jobs = (int)bj.size();
+  h->n_chunks = (int)ch.size();
+  if (h->bf16) TP_TRY(tc_build_plan(h->tc, h->cfg, h->depth, h->width, h->active, h->W_off, h->act_off,
+                                    h->dz_off, h->d_in_pad, h->B_cap, h->wq, h->xb, h->act, h->dz, h->err));
+  return TP_OK;
+}
+
+tp_status alloc_all(tabpack* h) {
+  const int m = h->cfg.m;
+  h->elem = h->bf16 ? 2 : 4;
+  TP_TRY(dalloc(h, &h->params, sizeof(float) * h->n_params));
+  TP_TRY(dalloc(h, &h->grads, sizeof(float) * h->n_params));
+  TP_TRY(dalloc(h, &h->adam_m, sizeof(float) * h->n_params));
+  TP_TRY(dalloc(h, &h->adam_v, sizeof(float) * h->n_params));
+  if (h->bf16) TP_TRY(dalloc(h, &h->wq, sizeof(__nv_bfloat16) * h->n_params));
+  TP_TRY(dalloc(h, &h->xb, h->elem * h->xb_elems));
+  TP_TRY(dalloc(h, &h->act, h->elem * h->act_elems));
+  TP_TRY(dalloc(h, &h->dz, h->elem * h->dz_elems));
+  TP_TRY(dalloc(h, &h->logits, sizeof(float) * (size_t)m * h->B_cap * h->cfg.d_out));
+  TP_TRY(dalloc(h, &h->head_part, sizeof(float) * h->head_part_elems));
+  TP_TRY(dalloc(h, &h->loss_part, sizeof(float) * (size_t)m * h->n_blk_cap));
+  TP_TRY(dalloc(h, &h->loss_last, sizeof(float) * m));
+  TP_TRY(dalloc(h, &h->t_dev, sizeof(int32_t) * m));
+  TP_TRY(dalloc(h, &h->bias_corr, sizeof(float2) * m));
+  TP_TRY(dalloc(h, &h->active_dev, m));
+  TP_TRY(dalloc(h, &h->mem_dev, sizeof(MemberDev) * m));
+  TP_TRY(dalloc(h, &h->segs_dev, sizeof(Segment) * h->segs.size()));
+  TP_TRY(dalloc(h, &h->part_stride_dev, sizeof(int64_t) * m));
+  TP_CUDA(h, cudaMemset(h->t_dev, 0, sizeof(int32_t) * m));
+  TP_CUDA(h, cudaMemset(h->bias_corr, 0, sizeof(float2) * m));
+  TP_CUDA(h, cudaMemset(h->xb, 0, h->elem * h->xb_elems));
+  TP_CUDA(h, cudaMemset(h->act, 0, h->elem * h->act_elems));
+  TP_CUDA(h, cudaMemset(h->dz, 0, h->elem * h->dz_elems));
+  TP_CUDA(h, cudaMemset(h->logits, 0, sizeof(float) * (size_t)m * h->B_cap * h->cfg.d_out));
+  TP_CUDA(h, cudaMemcpy(h->mem_dev, h->mem.data(), sizeof(MemberDev) * m, cudaMemcpyHostToDevice));
+  TP_CUDA(h, cudaMemcpy(h->segs_dev, h->segs.data(), sizeof(Segment) * h->segs.size(), cudaMemcpyHostToDevice));
+  TP_CUDA(h, cudaMemcpy(h->part_stride_dev, h->part_stride.data(), sizeof(int64_t) * m, cudaMemcpyHostToDevice));
+  return TP_OK;
+}
+
+void free_all(tabpack* h) {
+  if (h->st) cudaStreamSynchronize(h->st);
+  tc_free_plan(h->tc);
+  for (void* p : h->allocs) cudaFree(p);
+  h->allocs.clear();
+  for (auto e : h->prof.pool) cudaEventDestroy(e);
+  h->prof.pool.clear();
+}
+
+template <typename T>
+GemmArgs<T> gemm_args(tabpack* h, int B, int B_pad, uint32_t step, int train) {
+  GemmArgs<T> g;
+  g.probs = h->probs_dev;
+  g.tiles = h->tiles_dev;
+  g.xb = (const T*)h->xb;
+  g.act = (T*)h->act;
+  g.dz = (T*)h->dz;
+  g.wq = h->bf16 ? (const T*)h->wq : (const T*)h->params;
+  g.params = h->params;
+  g.grads = h->grads;
+  g.mem = h->mem_dev;
+  g.B = B;
+  g.B_pad = B_pad;
+  g.step = step;
+  g.train = train;
+  g.seed = h->cfg.seed;
+  return g;
+}
+
+template <typename T>
+tp_status run_forward(tabpack* h, int B, int B_pad, uint32_t step, int train) {
+  for (int l = 0; l < h->Lmax; ++l) {
+    int slot;
+    prof_begin(h, train ? TP_PH_FWD : TP_PH_PREDICT, &slot);
+    if (h->bf16 && h->tc.enabled) {
+      TP_TRY(tc_run_fwd(h->tc, h->st, l, B, B_pad, step, train, h->cfg.seed, h->params, h->mem_dev, h->err));
+    } else {
+      auto g = gemm_args<T>(h, B, B_pad, step, train);
+      launch_gemm_simt<T>(h->st, g, h->fwd_rng[l].first, h->fwd_rng[l].second);
+    }
+    TP_LAUNCHED(h);
+    h->launches++;
+    prof_end(h, slot, 1, train ? TP_PH_FWD : TP_PH_PREDICT);
+  }
+  return TP_OK;
+}
+
+template <typename T>
+tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* idx, const void* y, int B,
+                   uint32_t step, float* loss_out, bool update) {
+  const int B_pad = (int)round_up(B, kRowTile);
+  int slot;
+  // gather + step counters
+  prof_begin(h, TP_PH_GATHER, &slot);
+  launch_gather<T>(h->st, X, idx, B, B_pad, h->cfg.d_in, h->d_in_pad, (T*)h->xb, update ? 1 : 0, h->t_dev,
+                   h->bias_corr, h->active_ids_dev, h->n_active, h->cfg.beta1, h->cfg.beta2);
+  TP_LAUNCHED(h);
+  h->launches++;
+  prof_end(h, slot, 1, TP_PH_GATHER);
+  TP_TRY(run_forward<T>(h, B, B_pad, step, 1));
+  // head + loss
+  prof_begin(h, TP_PH_HEAD, &slot);
+  HeadArgs<T> hg;
+  hg.jobs = h->head_jobs_dev;
+  hg.mem = h->mem_dev;
+  hg.act = (const T*)h->act;
+  hg.dz = (T*)h->dz;
+  hg.params = h->params;
+  hg.head_part = h->head_part;
+  hg.loss_part = h->loss_part;
+  hg.logits = h->logits;
+  hg.idx = idx;
+  hg.y = y;
+  hg.B = B;
+  hg.B_pad = B_pad;
+  hg.B_cap = h->B_cap;
+  hg.d_out = h->cfg.d_out;
+  hg.task = h->cfg.task;
+  hg.n_blk_cap = h->n_blk_cap;
+  launch_head<T>(h->st, hg, h->n_head_jobs);
+  TP_LAUNCHED(h);
+  h->launches++;
+  prof_end(h, slot, 1, TP_PH_HEAD);
+  // backward GEMMs, deepest layer first
+  for (int l = h->Lmax - 1; l >= 0; --l) {
+    prof_begin(h, TP_PH_BWD, &slot);
+    if (h->bf16 && h->tc.enabled) {
+      TP_TRY(tc_run_bwd(h->tc, h->st, l, B, B_pad, h->grads, h->mem_dev, h->err));
+    } else {
+      auto g = gemm_args<T>(h, B, B_pad, step, 1);
+      launch_gemm_simt<T>(h->st, g, h->bwd_rng[l].first, h->bwd_rng[l].second);
+    }
+    TP_LAUNCHED(h);
+    h->launches++;
+    prof_end(h, slot, 1, TP_PH_BWD);
+  }
+  // bias gradients + head gradients / losses
+  prof_begin(h, TP_PH_BIAS, &slot);
+  launch_bias_grad<T>(h->st, h->bias_jobs_dev, h->n_bias_jobs, (const T*)h->dz, h->grads, B_pad);
+  TP_LAUNCHED(h);
+  HeadReduceArgs rg;
+  rg.jobs = h->hred_dev;
+  rg.active = h->active_dev;
+  rg.part_stride = h->part_stride_dev;
+  rg.head_part = h->head_part;
+  rg.loss_part = h->loss_part;
+  rg.grads = h->grads;
+  rg.loss_out = loss_out;
+  rg.loss_last = h->loss_last;
+  rg.B = B;
+  rg.B_pad = B_pad;
+  rg.d_out = h->cfg.d_out;
+  rg.n_blk_cap = h->n_blk_cap;
+  launch_head_reduce(h->st, rg, h->cfg.m);
+  TP_LAUNCHED(h);
+  h->launches += 2;
+  prof_end(h, slot, 2, TP_PH_BIAS);
+  if (update) {
+    prof_begin(h, TP_PH_ADAMW, &slot);
+    AdamArgs ag;
+    ag.chunks = h->chunks_dev;
+    ag.segs = h->segs_dev;
+    ag.mem = h->mem_dev;
+    ag.bias_corr = h->bias_corr;
+    ag.params = h->params;
+    ag.grads = h->grads;
+    ag.m = h->adam_m;
+    ag.v = h->adam_v;
+    ag.wq = h->bf16 ? h->wq : nullptr;
+    ag.beta1 = h->cfg.beta1;
+    ag.beta2 = h->cfg.beta2;
+    ag.eps = h->cfg.eps;
+    ag.wd_on_bias = h->cfg.wd_on_bias;
+    launch_adamw(h->st, ag, h->n_chunks);
+    TP_LAUNCHED(h);
+    h->launches++;
+    prof_end(h, slot, 1, TP_PH_ADAMW);
+  }
+  h->last_B = B;
+  (void)n_rows;
+  return TP_OK;
+}
+
+template <typename T>
+tp_status run_predict(tabpack* h, const float* X, int64_t N, float* out) {
+  for (int64_t n0 = 0; n0 < N; n0 += h->B_cap) {
+    const int rows = (int)std::min<int64_t>(h->B_cap, N - n0);
+    const int B_pad = (int)round_up(rows, kRowTile);
+    int slot;
+    prof_begin(h, TP_PH_PREDICT, &slot);
+    launch_gather<T>(h->st, X + n0 * h->cfg.d_in, nullptr, rows, B_pad, h->cfg.d_in, h->d_in_pad, (T*)h->xb, 0,
+                     h->t_dev, h->bias_corr, h->active_ids_dev, 0, h->cfg.beta1, h->cfg.beta2);
+    TP_LAUNCHED(h);
+    h->launches++;
+    prof_end(h, slot, 1, TP_PH_PREDICT);
+    TP_TRY(run_forward<T>(h, rows, B_pad, 0u, 0));
+    prof_begin(h, TP_PH_PREDICT, &slot);
+    PredictHeadArgs<T> pg;
+    pg.jobs = h->head_jobs_dev;
+    pg.mem = h->mem_dev;
+    pg.act = (const T*)h->act;
+    pg.params = h->params;
+    pg.out = out;
+    pg.N = N;
+    pg.n0 = n0;
+    pg.rows = rows;
+    pg.d_out = h->cfg.d_out;
+    pg.task = h->cfg.task;
+    pg._pad = 0;
+    launch_predict_head<T>(h->st, pg, h->n_head_jobs);
+    TP_LAUNCHED(h);
+    h->launches++;
+    prof_end(h, slot, 1, TP_PH_PREDICT);
+  }
+  return TP_OK;
+}
+
+tp_status check_step_args(tabpack* h, const float* X, int64_t n_rows, const int32_t* idx, const void* y, int B) {
+  if (!h) return fail(nullptr, TP_EINVAL, "null pack");
+  if (!X || !idx || !y) return fail(h, TP_EINVAL, "X, idx and y must be device pointers");
+  if (B < 1 || B > h->cfg.max_batch) return fail(h, TP_EINVAL, "B=%d outside [1, max_batch=%d]", B, h->cfg.max_batch);
+  if (n_rows < 1) return fail(h, TP_EINVAL, "n_rows=%lld", (long long)n_rows);
+  return TP_OK;
+}
+
+tp_status check_ml(tabpack* h, int member, int layer) {
+  if (!h) return fail(nullptr, TP_EINVAL, "null pack");
+  if (member < 0 || member >= h->cfg.m) return fail(h, TP_EINVAL, "member %d out of range", member);
+  if (layer < 0 || layer > h->depth[member]) return fail(h, TP_EINVAL, "layer %d out of range", layer);
+  return TP_OK;
+}
+
+}  // namespace
+
+// ====================================================================== ABI
+extern "C" {
+
+tp_status pack_create(const tp_config* cfg, const int32_t* depth, const int32_t* width, const float* dropout,
+                      const float* lr, const float* wd, void* cuda_stream, tabpack_t** out) {
+  if (out) *out = nullptr;
+  if (!cfg || !depth || !width || !dropout || !lr || !wd || !out)
+    return fail(nullptr, TP_EINVAL, "null argument");
+  if (cfg->m < 1 || cfg->d_in < 1 || cfg->max_batch < 1) return fail(nullptr, TP_EINVAL, "m, d_in, max_batch must be >= 1");
+  if (cfg->task < 0 || cfg->task > 2) return fail(nullptr, TP_EINVAL, "unknown task %d", cfg->task);
+  if (cfg->precision != TP_BF16 && cfg->precision != TP_FP32) return fail(nullptr, TP_EINVAL, "unknown precision");
+  if (cfg->task == TP_MULTICLASS ? (cfg->d_out < 2 || cfg->d_out > kMaxDout) : cfg->d_out != 1)
+    return fail(nullptr, TP_EINVAL, "d_out=%d invalid for task %d", cfg->d_out, cfg->task);
+  if (!(cfg->beta1 >= 0.f && cfg->beta1 < 1.f && cfg->beta2 >= 0.f && cfg->beta2 < 1.f && cfg->eps >= 0.f))
+    return fail(nullptr, TP_EINVAL, "AdamW constants out of range");
+  for (int i = 0; i < cfg->m; ++i) {
+    if (depth[i] < 1 || depth[i] > kMaxDepth) return fail(nullptr, TP_EINVAL, "depth[%d]=%d not in 1..%d", i, depth[i], kMaxDepth);
+    if (width[i] < 16 || width[i] > 4096 || width[i] % 16)
+      return fail(nullptr, TP_EINVAL, "width[%d]=%d must be a multiple of 16 in [16, 4096]", i, width[i]);
+    if (!(dropout[i] >= 0.f && dropout[i] < 1.f)) return fail(nullptr, TP_EINVAL, "dropout[%d] not in [0, 1)", i);
+    if (!(lr[i] >= 0.f) || !(wd[i] >= 0.f)) return fail(nullptr, TP_EINVAL, "lr/wd[%d] must be >= 0", i);
+  }
+  if (cfg->m >= (1 << 24)) return fail(nullptr, TP_EINVAL, "too many members");
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(nullptr, TP_ECUDA, "no CUDA device: %s", cudaGetErrorString(e));
+  cudaDeviceProp prop;
+  e = cudaGetDeviceProperties(&prop, dev);
+  if (e != cudaSuccess) return fail(nullptr, TP_ECUDA, "cudaGetDeviceProperties: %s", cudaGetErrorString(e));
+  if (prop.major != 10) return fail(nullptr, TP_ENOTSUP, "needs a Blackwell (sm_10x) GPU, found sm_%d%d", prop.major, prop.minor);
+
+  tabpack* h = new tabpack();
+  h->cfg = *cfg;
+  h->st = (cudaStream_t)cuda_stream;
+  h->bf16 = cfg->precision == TP_BF16;
+  h->depth.assign(depth, depth + cfg->m);
+  h->width.assign(width, width + cfg->m);
+  h->dropout.assign(dropout, dropout + cfg->m);
+  h->lr.assign(lr, lr + cfg->m);
+  h->wd.assign(wd, wd + cfg->m);
+  h->active.assign(cfg->m, 1);
+  tp_status s = build_layout(h);
+  if (s == TP_OK) s = alloc_all(h);
+  if (s == TP_OK) s = build_schedule(h);
+  if (s == TP_OK) {
+    // Philox init of every parameter (all members active here)
+    InitArgs ig{h->chunks_dev, h->segs_dev, h->params, h->grads, h->adam_m, h->adam_v, h->wq, cfg->seed};
+    launch_init(h->st, ig, h->n_chunks);
+    h->launches++;
+    cudaError_t le = cudaGetLastError();
+    if (le == cudaSuccess) le = cudaStreamSynchronize(h->st);
+    if (le != cudaSuccess) s = fail(h, TP_ECUDA, "init: %s", cudaGetErrorString(le));
+  }
+  if (s != TP_OK) {
+    g_thread_error = h->err;
+    free_all(h);
+    delete h;
+    return s;
+  }
+  *out = h;
+  return TP_OK;
+}
+
+void pack_destroy(tabpack_t* h) {
+  if (!h) return;
+  free_all(h);
+  delete h;
+}
+
+tp_status pack_set_stream(tabpack_t* h, void* cuda_stream) {
+  if (!h) return fail(nullptr, TP_EINVAL, "null pack");
+  TP_CUDA(h, cudaStreamSynchronize(h->st));
+  h->st = (cudaStream_t)cuda_stream;
+  return TP_OK;
+}
+
+tp_status pack_train_step(tabpack_t* h, const float* X, int64_t n_rows, const int32_t* idx, const void* y,
+                          int32_t B, uint32_t step, float* loss_out) {
+  TP_TRY(check_step_args(h, X, n_rows, idx, y, B));
+  if (h->n_active == 0) return fail(h, TP_ESTATE, "no active member");
+  return h->bf16 ? run_step<__nv_bfloat16>(h, X, n_rows, idx, y, B, step, loss_out, true)
+                 : run_step<float>(h, X, n_rows, idx, y, B, step, loss_out, true);
+}
+
+tp_status pack_forward_backward(tabpack_t* h, const float* X, int64_t n_rows, const int32_t* idx, const void* y,
+                                int32_t B, uint32_t step, float* loss_out) {
+  TP_TRY(check_step_args(h, X, n_rows, idx, y, B));
+  if (h->n_active == 0) return fail(h, TP_ESTATE, "no active member");
+  return h->bf16 ? run_step<__nv_bfloat16>(h, X, n_rows, idx, y, B, step, loss_out, false)
+                 : run_step<float>(h, X, n_rows, idx, y, B, step, loss_out, false);
+}
+
+tp_status pack_predict(tabpack_t* h, const float* X, int64_t N, float* out) {
+  if (!h) return fail(nullptr, TP_EINVAL, "null pack");
+  if (!X || !out || N < 1) return fail(h, TP_EINVAL, "X/out null or N < 1");
+  if (h->n_active == 0) return fail(h, TP_ESTATE, "no active member");
+  return h->bf16 ? run_predict<__nv_bfloat16>(h, X, N, out) : run_predict<float>(h, X, N, out);
+}
+
+tp_status pack_set_active(tabpack_t* h, const uint8_t* active) {
+  if (!h || !active) return fail(h, TP_EINVAL, "null argument");
+  for (int i = 0; i < h->cfg.m; ++i) h->active[i] = active[i] ? 1 : 0;
+  return build_schedule(h);
+}
+
+static tp_status copy_layer(tabpack_t* h, int member, int layer, float* W, float* b, const float* src) {
+  TP_TRY(check_ml(h, member, layer));
+  TP_CUDA(h, cudaStreamSynchronize(h->st));
+  const int L = h->depth[member], w = h->width[member];
+  const int in = layer == 0 ? h->cfg.d_in : w, in_pad = layer == 0 ? h->d_in_pad : w;
+  const int out = layer == L ? h->cfg.d_out : w;
+  if (W) {
+    std::vector<float> tmp((size_t)out * in_pad);
+    TP_CUDA(h, cudaMemcpy(tmp.data(), src + h->W_off[member][layer], tmp.size() * 4, cudaMemcpyDeviceToHost));
+    for (int r = 0; r < out; ++r) std::memcpy(W + (size_t)r * in, tmp.data() + (size_t)r * in_pad, (size_t)in * 4);
+  }
+  if (b) TP_CUDA(h, cudaMemcpy(b, src + h->b_off[member][layer], (size_t)out * 4, cudaMemcpyDeviceToHost));
+  return TP_OK;
+}
+
+tp_status pack_get_params(tabpack_t* h, int32_t member, int32_t layer, float* W, float* b) {
+  if (!h) return fail(nullptr, TP_EINVAL, "null pack");
+  return copy_layer(h, member, layer, W, b, h->params);
+}
+
+tp_status pack_get_grads(tabpack_t* h, int32_t member, int32_t layer, float* W, float* b) {
+  if (!h) return fail(nullptr, TP_EINVAL, "null pack");
+  return copy_layer(h, member, layer, W, b, h->grads);
+}
+
+tp_status pack_set_params(tabpack_t* h, int32_t member, int32_t layer, const float* W, const float* b) {
+  TP_TRY(check_ml(h, member, layer));
+  TP_CUDA(h, cudaStreamSynchronize(h->st));
+  const int L = h->depth[member], w = h->width[member];
+  const int in = layer == 0 ? h->cfg.d_in : w, in_pad = layer == 0 ? h->d_in_pad : w;
+  const int out = layer == L ? h->cfg.d_out : w;
+  if (W) {
+    std::vector<float> tmp((size_t)out * in_pad, 0.f);
+    for (int r = 0; r < out; ++r) std::memcpy(tmp.data() + (size_t)r * in_pad, W + (size_t)r * in, (size_t)in * 4);
+    TP_CUDA(h, cudaMemcpy(h->params + h->W_off[member][layer], tmp.data(), tmp.size() * 4, cudaMemcpyHostToDevice));
+  }
+  if (b) TP_CUDA(h, cudaMemcpy(h->params + h->b_off[member][layer], b, (size_t)out * 4, cudaMemcpyHostToDevice));
+  if (h->bf16) {
+    launch_refresh_wq(h->st, h->params, h->wq, h->n_params);
+    TP_LAUNCHED(h);
+    h->launches++;
+    TP_CUDA(h, cudaStreamSynchronize(h->st));
+  }
+  return TP_OK;
+}
+
+tp_status pack_get_logits(tabpack_t* h, int32_t member, float* out) {
+  TP_TRY(check_ml(h, member, 0));
+  if (!out) return fail(h, TP_EINVAL, "null out");
+  TP_CUDA(h, cudaStreamSynchronize(h->st));
+  TP_CUDA(h, cudaMemcpy(out, h->logits + (size_t)member * h->B_cap * h->cfg.d_out,
+                        sizeof(float) * (size_t)h->last_B * h->cfg.d_out, cudaMemcpyDeviceToHost));
+  return TP_OK;
+}
+
+tp_status pack_debug_masks(tabpack_t* h, int32_t member, int32_t layer, uint32_t step, int32_t B, uint8_t* keep) {
+  TP_TRY(check_ml(h, member, layer));
+  if (layer >= h->depth[member]) return fail(h, TP_EINVAL, "layer %d is the head", layer);
+  if (B < 1 || !keep) return fail(h, TP_EINVAL, "bad B or null keep");
+  const int w = h->width[member];
+  uint8_t* d = nullptr;
+  TP_CUDA(h, cudaMalloc(&d, (size_t)B * w));
+  launch_debug_masks(h->st, d, B, w, h->cfg.seed, (uint32_t)member, (uint32_t)layer, step, h->mem[member].drop_T);
+  h->launches++;
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+  if (e == cudaSuccess) e = cudaMemcpy(keep, d, (size_t)B * w, cudaMemcpyDeviceToHost);
+  cudaFree(d);
+  if (e != cudaSuccess) return fail(h, TP_ECUDA, "debug masks: %s", cudaGetErrorString(e));
+  return TP_OK;
+}
+
+tp_status pack_debug_activations(tabpack_t* h, int32_t member, int32_t layer, float* out) {
+  TP_TRY(check_ml(h, member, layer));
+  if (layer >= h->depth[member]) return fail(h, TP_EINVAL, "layer %d is the head", layer);
+  if (!out) return fail(h, TP_EINVAL, "null out");
+  TP_CUDA(h, cudaStreamSynchronize(h->st));
+  const size_t n = (size_t)h->last_B * h->width[member];
+  if (h->bf16) {
+    std::vector<__nv_bfloat16> tmp(n);
+    TP_CUDA(h, cudaMemcpy(tmp.data(), (const __nv_bfloat16*)h->act + h->act_off[member][layer], n * 2,
+                          cudaMemcpyDeviceToHost));
+    for (size_t e = 0; e < n; ++e) out[e] = __bfloat162float(tmp[e]);
+  } else {
+    TP_CUDA(h, cudaMemcpy(out, (const float*)h->act + h->act_off[member][layer], n * 4, cudaMemcpyDeviceToHost));
+  }
+  return TP_OK;
+}
+
+tp_status pack_select_greedy(const float* preds, int32_t P, int64_t N, int32_t d_out, const void* y, int32_t task,
+                             int32_t score, int32_t m_ens, void* cuda_stream, int32_t* selected,
+                             int32_t* n_selected, double* final_score) {
+  if (!preds || !y || !selected || !n_selected) return fail(nullptr, TP_EINVAL, "null argument");
+  if (P < 1 || N < 1 || m_ens < 1) return fail(nullptr, TP_EINVAL, "P, N, m_ens must be >= 1");
+  if (task < 0 || task > 2 || score < 0 || score > 2) return fail(nullptr, TP_EINVAL, "unknown task/score");
+  if (score == TP_SCORE_ACCURACY && task == TP_REGRESSION) return fail(nullptr, TP_EINVAL, "accuracy needs classification");
+  if (score == TP_SCORE_RMSE && task != TP_REGRESSION) return fail(nullptr, TP_EINVAL, "rmse needs regression");
+  if (task == TP_MULTICLASS ? (d_out < 2 || d_out > kMaxDout) : d_out != 1) return fail(nullptr, TP_EINVAL, "bad d_out");
+  if (P > 65535) return fail(nullptr, TP_EINVAL, "P > 65535");
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  const int64_t bytes = select_scratch_bytes(P, N, d_out, m_ens);
+  void* scratch = nullptr;
+  cudaError_t e = cudaMallocAsync(&scratch, (size_t)bytes, st);
+  if (e != cudaSuccess) return fail(nullptr, TP_ENOMEM, "cudaMallocAsync(%lld): %s", (long long)bytes, cudaGetErrorString(e));
+  SelectScratch s = select_carve(scratch, P, N, d_out, m_ens);
+  const int n_words = select_enqueue(st, s, preds, P, N, d_out, y, task, score, m_ens, nullptr);
+  std::vector<int32_t> host(n_words);
+  double cur = 0.0;
+  e = cudaGetLastError();
+  if (e == cudaSuccess) e = cudaMemcpyAsync(host.data(), s.state, sizeof(int32_t) * n_words, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(&cur, s.cur, sizeof(double), cudaMemcpyDeviceToHost, st);
+  cudaError_t fe = cudaFreeAsync(scratch, st);
+  if (e == cudaSuccess) e = fe;
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return fail(nullptr, TP_ECUDA, "select: %s", cudaGetErrorString(e));
+  const int n = host[0];
+  *n_selected = n;
+  for (int k = 0; k < n; ++k) selected[k] = host[4 + k];
+  if (final_score) *final_score = cur;
+  return TP_OK;
+}
+
+tp_status pack_profile_enable(tabpack_t* h, int32_t enable) {
+  if (!h) return fail(nullptr, TP_EINVAL, "null pack");
+  h->profiling = enable != 0;
+  return TP_OK;
+}
+
+tp_status pack_profile_read(tabpack_t* h, double* ms, int64_t* launches, int32_t reset) {
+  if (!h) return fail(nullptr, TP_EINVAL, "null pack");
+  prof_flush(h);
+  for (int p = 0; p < TP_PH_COUNT; ++p) {
+    if (ms) ms[p] = h->prof.ms[p];
+    if (launches) launches[p] = h->prof.launches[p];
+    if (reset) {
+      h->prof.ms[p] = 0;
+      h->prof.launches[p] = 0;
+    }
+  }
+  return TP_OK;
+}
+
+int64_t pack_launch_count(const tabpack_t* h) { return h ? h->launches : -1; }
+
+tp_status pack_sizes(const tabpack_t* h, int64_t* n_params, int64_t* device_bytes) {
+  if (!h) return fail(nullptr, TP_EINVAL, "null pack");
+  if (n_params) *n_params = h->n_params;
+  if (device_bytes) *device_bytes = (int64_t)h->dev_bytes;
+  return TP_OK;
+}
+
+const char* pack_last_error(const tabpack_t* h) { return h ? h->err.c_str() : g_thread_error.c_str(); }
+
+}  // extern "C"

@@ -1,0 +1,140 @@
+// tp_internal.cuh -- shared internals of the tabpack CUDA library (sm_103a).
+//
+// Device data layout (one pack):
+//   params / grads / adam_m / adam_v : fp32 arenas of n_params elements.  Member i
+//       owns one contiguous run: for l = 0..L_i (L_i = head) the weight block
+//       [out, in_pad] row-major then the bias [out]; every block starts on a
+//       32-element boundary.  Layer 0 has in_pad = round_up(d_in, 8) columns
+//       (the pad columns stay exactly zero); other layers in_pad = in.
+//   wq[2]  : bf16 copies of the whole param arena (same offsets), written by
+//       AdamW; the matrix products read them (bf16 mode).  Two copies so a
+//       step can read one while AdamW of the same step writes the other.
+//   xb     : the gathered batch [B_cap, d_in_pad] (T).
+//   act    : H_{l+1} = output of hidden layer l of member i, [B_cap, w_i] (T).
+//   dz     : dL/dZ_l of hidden layer l of member i, [B_cap, w_i] (T).
+// T = __nv_bfloat16 in bf16 mode, float in fp32 mode.  Batches are padded to
+// B_pad = round_up(B, 128) rows; padded rows carry zero loss gradient, so they
+// add nothing to weight gradients.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace tp {
+
+constexpr int kMaxDepth = 14;   // hidden blocks per member (4-bit layer field of the Philox counter)
+constexpr int kMaxDout = 32;
+constexpr int kRowTile = 128;   // batch rows per tile; B_pad is a multiple of this
+constexpr int kSegAlign = 32;   // elements
+
+enum GemmKind : int32_t { kFwd = 0, kDgrad = 1, kWgrad = 2 };
+enum Src : int32_t { kSrcXb = 0, kSrcAct = 1, kSrcDz = 2, kSrcWq = 3 };
+
+// One matrix product of one member and layer.  Output C[r, c] = sum_k A(r, k) B(c, k).
+//   kFwd   : A = H_l [B, in] (act or xb), B = W_l [w, in] (wq);  C = H_{l+1} [B, w]
+//   kDgrad : A = dZ_l [B, w] (dz), B(c, k) = W_l[k, c];          C = dZ_{l-1} [B, in]
+//   kWgrad : A(r, k) = dZ_l[k, r], B(c, k) = H_l[k, c];          C = dW_l [w, in_pad] (grads)
+struct GemmProblem {
+  int32_t kind, member, layer, _pad0;
+  int32_t M, N, K;        // M == 0 / K == 0: the step's B_pad rows
+  int32_t a_src, b_src;
+  int32_t lda, ldb, ldc;  // row pitches in elements
+  int64_t a_off, b_off, c_off;
+  int64_t aux_off;        // kFwd: bias offset in params; kDgrad: offset of H_l (mask source) in act
+  int64_t _pad1;
+};
+
+struct GemmTile {
+  int32_t prob, m0, n0, n_len;  // output tile origin; n_len = columns of this tile
+};
+
+struct MemberDev {
+  int32_t L, w;
+  float p, scale;         // dropout rate, 1 / (1 - p)
+  float lr, wd;
+  uint32_t drop_T;        // drop iff Philox word < drop_T
+  int32_t _pad;
+};
+
+// Contiguous run of parameters of one layer (weights or bias) of one member.
+struct Segment {
+  int64_t off;            // element offset in the param arena
+  int32_t member, layer;
+  int32_t rows, cols, cols_pad;  // weights: [rows, cols_pad], cols real; bias: rows x 1
+  int32_t is_bias, fan_in;
+  int32_t w_elems;        // unpadded weight count of the layer (bias init index base)
+};
+
+struct Chunk {            // element-wise work unit (init, AdamW): never crosses a segment
+  int64_t off;
+  int32_t len, seg;
+};
+
+struct BiasJob {          // bias gradient: column sums of dZ_l over the batch rows
+  int64_t dz_off, b_off;  // dZ_l in dz arena, bias in grads arena
+  int32_t w, c0;          // pitch / width of dZ_l, first column of this job
+};
+
+struct HeadJob {          // head forward / loss / backward of one member on one 128-row block
+  int32_t member, blk;
+  int64_t h_off;          // H_L in act (or xb never: L >= 1)
+  int64_t dz_off;         // dZ_{L-1} in dz
+  int64_t w_off, b_off;   // head weight / bias offsets in params
+  int64_t part_off;       // partial dW_h of this block: [d_out, w] + [d_out] db
+};
+
+struct HeadReduceJob {
+  int32_t member, n_blk;
+  int64_t part_off;       // first block's partial; blocks are consecutive, stride (d_out + 1) * w... see kernel
+  int64_t gw_off, gb_off; // head grads in grads arena
+  int32_t w, _pad;
+};
+
+// ---------------------------------------------------------------- Philox4x32-10
+// Salmon, Moraes, Dror, Shaw (SC'11): ten rounds of
+//   (c0, c1, c2, c3) -> (hi(Mb c2) ^ c1 ^ k0, lo(Mb c2), hi(Ma c0) ^ c3 ^ k1, lo(Ma c0)),
+// keys bumped by the Weyl increments between rounds.
+struct U4 { uint32_t x, y, z, w; };
+
+__device__ __forceinline__ U4 philox10(uint32_t c0, uint32_t c1, uint32_t c2, uint32_t c3,
+                                       uint32_t k0, uint32_t k1) {
+  const uint32_t Ma = 0xD2511F53u, Mb = 0xCD9E8D57u;
+  const uint32_t Wa = 0x9E3779B9u, Wb = 0xBB67AE85u;
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    uint32_t lo_a = Ma * c0, hi_a = __umulhi(Ma, c0);
+    uint32_t lo_b = Mb * c2, hi_b = __umulhi(Mb, c2);
+    uint32_t n0 = hi_b ^ c1 ^ k0, n2 = hi_a ^ c3 ^ k1;
+    c0 = n0; c1 = lo_b; c2 = n2; c3 = lo_a;
+    k0 += Wa; k1 += Wb;
+  }
+  return U4{c0, c1, c2, c3};
+}
+
+// Keep bits of columns (col4 * 4 .. col4 * 4 + 3) of row `row`: bit q = keep(col4 * 4 + q).
+__device__ __forceinline__ uint32_t keep_bits4(uint64_t seed, uint32_t member, uint32_t layer,
+                                               uint32_t step, uint32_t row, uint32_t col4,
+                                               uint32_t T) {
+  if (T == 0u) return 0xFu;
+  U4 r = philox10(row, col4, step, (member << 4) | layer, (uint32_t)seed, (uint32_t)(seed >> 32));
+  return (uint32_t)(r.x >= T) | ((uint32_t)(r.y >= T) << 1) | ((uint32_t)(r.z >= T) << 2) |
+         ((uint32_t)(r.w >= T) << 3);
+}
+
+// ---------------------------------------------------------------- element types
+template <typename T> struct Elem;
+template <> struct Elem<float> {
+  static __device__ __forceinline__ float load(const float* p) { return *p; }
+  static __device__ __forceinline__ float to_f(float v) { return v; }
+  static __device__ __forceinline__ float from_f(float v) { return v; }
+};
+template <> struct Elem<__nv_bfloat16> {
+  static __device__ __forceinline__ float to_f(__nv_bfloat16 v) { return __bfloat162float(v); }
+  static __device__ __forceinline__ __nv_bfloat16 from_f(float v) { return __float2bfloat16_rn(v); }
+};
+
+__host__ __device__ constexpr int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+__host__ __device__ constexpr int64_t ceil_div(int64_t x, int64_t a) { return (x + a - 1) / a; }
+
+}  // namespace tp

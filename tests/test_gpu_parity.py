@@ -1,0 +1,312 @@
+"""GPU path versus the CPU oracle, element by element, through the C ABI.
+
+Bars: dropout masks, init values and selected indices bit-exact; floats
+within max relative error 1e-4 (fp32 mode, vs the fp64 oracle) and 2e-2
+(bf16 mode, vs the oracle's bf16-storage mode), where the relative error of
+an entry is |g - o| / max(|o|, rms(o)) -- the tensor's rms is the floor for
+entries near zero.
+
+A ReLU pre-activation within rounding of zero makes both masks valid
+subgradients; in fp32 mode a member whose oracle pre-activations came within
+1e-5 rms of zero in any compared step is checked at the bf16 bar instead and
+counted (the test requires most members to meet the strict bar).
+"""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+import oracle  # noqa: E402
+from workloads import random_pack  # noqa: E402
+
+
+@pytest.fixture(scope="module")
+def tp():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    from paper_2607_05380_gb300 import build
+    build.build()
+    import paper_2607_05380_gb300 as tpm
+    tpm.load_library()
+    return tpm
+
+
+DEV = "cuda"
+TOL = {"fp32": 1e-4, "bf16": 2e-2}
+
+
+def rel_err(got, ref):
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    if ref.size == 0:
+        return 0.0
+    rms = np.sqrt(np.mean(ref ** 2))
+    floor = np.maximum(np.abs(ref), rms if rms > 0 else 1e-30)
+    return float(np.max(np.abs(got - ref) / floor))
+
+
+def make_data(task, n, d_in, d_out, seed):
+    rng = np.random.default_rng(seed)
+    X = rng.standard_normal((n, d_in)).astype(np.float32)
+    if task == "regression":
+        y = rng.standard_normal(n).astype(np.float32)
+    elif task == "binary":
+        y = rng.integers(0, 2, n).astype(np.int32)
+    else:
+        y = rng.integers(0, d_out, n).astype(np.int32)
+    return X, y
+
+
+def pair(tp, task, d_in, d_out, hp, prec, max_batch, seed=2):
+    pk = tp.Pack(d_in, d_out, task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
+                 max_batch=max_batch, seed=seed, precision=prec)
+    orc = oracle.OraclePack(d_in, d_out, task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
+                            seed=seed, bf16_storage=(prec == "bf16"))
+    return pk, orc
+
+
+def to_dev(*arrs):
+    return [torch.from_numpy(np.ascontiguousarray(a)).to(DEV) for a in arrs]
+
+
+def test_init_bit_exact(tp):
+    hp = random_pack(5, 13, 4, seed=3)
+    pk, orc = pair(tp, "multiclass", 13, 4, hp, "bf16", 128)
+    for i in range(5):
+        for l in range(int(hp["depth"][i]) + 1):
+            W, b = pk.get_params(i, l)
+            Wo, bo = orc.get_params(i, l)
+            np.testing.assert_array_equal(W.astype(np.float64), Wo)
+            np.testing.assert_array_equal(b.astype(np.float64), bo)
+
+
+@pytest.mark.parametrize("step", [0, 1, 7, 1000])
+def test_dropout_masks_bit_exact(tp, step):
+    hp = random_pack(6, 10, 1, seed=4, dropout=(0.05, 0.5))
+    pk, orc = pair(tp, "binary", 10, 1, hp, "fp32", 256)
+    X, y = make_data("binary", 300, 10, 1, 0)
+    idx = np.arange(200, dtype=np.int32)
+    orc.train_step(X, idx, y, step, update=False)
+    for i in range(6):
+        for l in range(int(hp["depth"][i])):
+            np.testing.assert_array_equal(pk.debug_masks(i, l, step, 200), orc.keep(i, l))
+
+
+# A ReLU decision whose pre-activation lies within rounding of zero may go
+# either way on the two sides; both results are valid subgradients.  In bf16
+# mode a one-ulp difference in a stored activation (the fp32 and fp64 values
+# straddling a bf16 rounding boundary) moves the next layer's pre-activations
+# by ~1e-3 of their rms, so such flips occur there too.  One flip at (row b,
+# unit j) of layer l changes dW_l[j, :] by one of the B batch terms and every
+# upstream gradient by a fraction of a percent.  The test therefore reads the
+# GPU's stored activations, finds every flipped decision exactly (GPU H > 0
+# versus oracle keep & Z > 0), requires each flip to sit at an oracle
+# near-tie (|Z| < TIE * rms(Z)), holds members without flips to the strict
+# elementwise bar everywhere, and members with flips to the strict bar on
+# losses and logits and to the bar norm-wise on each gradient tensor.
+TIE = {"fp32": 1e-5, "bf16": 5e-3}
+
+
+def _flips(pk, orc, i, L, prec):
+    n = 0
+    for l in range(L):
+        Hg = pk.debug_activations(i, l)
+        Zo = orc.preact(i, l)
+        mo = (Zo > 0) & (orc.keep(i, l) > 0)
+        diff = (Hg > 0) != mo
+        if diff.any():
+            zr = np.sqrt(np.mean(Zo ** 2))
+            worst = float(np.max(np.abs(Zo[diff])) / zr)
+            assert worst < TIE[prec], ("flip away from a near-tie", i, l, worst)
+            n += int(diff.sum())
+    return n
+
+
+def _compare_step(pk, orc, hp, prec, loss_gpu, loss_orc):
+    tol = TOL[prec]
+    problems = {}
+    n_flip_members = 0
+    for i in range(len(hp["depth"])):
+        L = int(hp["depth"][i])
+        flips = _flips(pk, orc, i, L, prec)
+        n_flip_members += flips > 0
+        p = []
+        le = abs(loss_gpu[i] - loss_orc[i]) / max(1.0, abs(loss_orc[i]))
+        ge = rel_err(pk.logits(i), orc.logits(i))
+        if le > tol or ge > tol:
+            p.append(("loss/logits", le, ge))
+        for l in range(L + 1):
+            gW, gb = pk.get_grads(i, l)
+            oW, ob = orc.get_grads(i, l)
+            if flips == 0:
+                e = max(rel_err(gW, oW), rel_err(gb, ob))
+            else:
+                g = np.concatenate([gW.ravel(), gb]).astype(np.float64)
+                o = np.concatenate([oW.ravel(), ob])
+                e = float(np.linalg.norm(g - o) / max(np.linalg.norm(o), 1e-30))
+            if e > tol:
+                p.append(("grad", l, flips, e))
+        if p:
+            problems[i] = p
+    assert n_flip_members <= max(1, len(hp["depth"]) // 3), ("too many members with flips", n_flip_members)
+    return problems
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+@pytest.mark.parametrize("task,d_out", [("binary", 1), ("multiclass", 7), ("regression", 1)])
+@pytest.mark.parametrize("B", [256, 200, 1])
+def test_one_step_logits_losses_grads(tp, prec, task, d_out, B):
+    """Several 128-row tiles plus a ragged tail (B=200), and B=1."""
+    d_in = 37
+    hp = random_pack(6, d_in, d_out, seed=10 + d_out, width=(16, 160, 16), depth=(1, 4))
+    pk, orc = pair(tp, task, d_in, d_out, hp, prec, 256)
+    X, y = make_data(task, 400, d_in, d_out, 1)
+    idx = np.random.default_rng(2).choice(400, B, replace=False).astype(np.int32)
+    Xd, yd, idxd = to_dev(X, y, idx)
+    loss = torch.zeros(len(hp["depth"]), dtype=torch.float32, device=DEV)
+    pk.forward_backward(Xd, idxd, yd, 5, loss)
+    lo = orc.train_step(X, idx, y, 5, update=False)
+    problems = _compare_step(pk, orc, hp, prec, loss.cpu().numpy(), lo)
+    assert not problems, problems
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+@pytest.mark.parametrize("task,d_out", [("binary", 1), ("multiclass", 5), ("regression", 1)])
+def test_ten_steps_params(tp, prec, task, d_out):
+    d_in, m, B = 24, 8, 192
+    hp = random_pack(m, d_in, d_out, seed=20 + d_out, width=(16, 128, 16), depth=(1, 3))
+    pk, orc = pair(tp, task, d_in, d_out, hp, prec, 256)
+    X, y = make_data(task, 600, d_in, d_out, 3)
+    Xd, yd = to_dev(X, y)
+    rng = np.random.default_rng(5)
+    loss = torch.zeros(m, dtype=torch.float32, device=DEV)
+    margin = np.full(m, np.inf)
+    for step in range(10):
+        idx = rng.choice(600, B, replace=False).astype(np.int32)
+        (idxd,) = to_dev(idx)
+        pk.train_step(Xd, idxd, yd, step, loss)
+        lo = orc.train_step(X, idx, y, step)
+        margin = np.minimum(margin, [orc.margin(i) for i in range(m)])
+        lg = loss.cpu().numpy()
+        for i in range(m):
+            assert abs(lg[i] - lo[i]) <= TOL["bf16"] * max(1.0, abs(lo[i])), (step, i, lg[i], lo[i])
+    errs = {}
+    for i in range(m):
+        e = 0.0
+        for l in range(int(hp["depth"][i]) + 1):
+            W, b = pk.get_params(i, l)
+            Wo, bo = orc.get_params(i, l)
+            e = max(e, rel_err(W, Wo), rel_err(b, bo))
+        errs[i] = e
+    tol = TOL[prec]
+    bad = {i: e for i, e in errs.items() if e > tol}
+    if prec == "fp32":
+        ties = {i for i in bad if margin[i] < 1e-5}
+        assert all(errs[i] <= TOL["bf16"] for i in ties), (errs, margin)
+        bad = {i: e for i, e in bad.items() if i not in ties}
+        assert len(ties) <= m // 4, (errs, margin)
+    assert not bad, (errs, margin)
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+@pytest.mark.parametrize("task,d_out", [("binary", 1), ("multiclass", 6), ("regression", 1)])
+def test_predict(tp, prec, task, d_out):
+    d_in = 19
+    hp = random_pack(5, d_in, d_out, seed=30 + d_out, width=(16, 96, 16))
+    pk, orc = pair(tp, task, d_in, d_out, hp, prec, 128)
+    X, y = make_data(task, 333, d_in, d_out, 4)   # 3 row chunks of 128, ragged tail
+    (Xd,) = to_dev(X)
+    out = pk.predict(Xd).cpu().numpy()
+    ref = orc.predict(X)
+    for i in range(5):
+        assert rel_err(out[i], ref[i]) <= TOL[prec], i
+
+
+def test_inactive_members(tp):
+    hp = random_pack(4, 9, 1, seed=7)
+    pk, orc = pair(tp, "regression", 9, 1, hp, "fp32", 128)
+    X, y = make_data("regression", 200, 9, 1, 5)
+    Xd, yd = to_dev(X, y)
+    idx = np.arange(128, dtype=np.int32)
+    (idxd,) = to_dev(idx)
+    loss = torch.zeros(4, dtype=torch.float32, device=DEV)
+    pk.train_step(Xd, idxd, yd, 0, loss)
+    orc.train_step(X, idx, y, 0)
+    frozen = pk.get_params(2, 0)
+    pk.set_active([1, 1, 0, 1])
+    orc.set_active([1, 1, 0, 1])
+    pk.train_step(Xd, idxd, yd, 1, loss)
+    lo = orc.train_step(X, idx, y, 1)
+    lg = loss.cpu().numpy()
+    assert np.isnan(lg[2]) and np.isnan(lo[2])
+    np.testing.assert_array_equal(pk.get_params(2, 0)[0], frozen[0])
+    for i in (0, 1, 3):
+        for l in range(int(hp["depth"][i]) + 1):
+            assert rel_err(pk.get_params(i, l)[0], orc.get_params(i, l)[0]) <= TOL["fp32"] * 10
+    pk.set_active([1, 1, 1, 1])
+    orc.set_active([1, 1, 1, 1])
+    pk.train_step(Xd, idxd, yd, 2, loss)
+    orc.train_step(X, idx, y, 2)
+    assert orc.member_steps(2) == 2
+
+
+@pytest.mark.parametrize("task,score,d_out", [("multiclass", "loss", 10), ("multiclass", "accuracy", 10),
+                                              ("binary", "loss", 1), ("binary", "accuracy", 1),
+                                              ("regression", "loss", 1), ("regression", "rmse", 1)])
+def test_select_greedy_indices_bit_exact(tp, task, score, d_out):
+    """Oracle greedy (fp32 terms, the kernel's decision precision) on the
+    GPU's own candidate tensor: identical selection order wherever the
+    oracle's best-vs-runner-up margin is not a near-tie."""
+    rng = np.random.default_rng(11)
+    P, N = 40, 5000
+    if task == "multiclass":
+        lg = rng.standard_normal((P, N, d_out)) * 1.5
+        preds = (np.exp(lg) / np.exp(lg).sum(-1, keepdims=True)).astype(np.float32)
+        y = rng.integers(0, d_out, N).astype(np.int32)
+    elif task == "binary":
+        preds = (1 / (1 + np.exp(-1.5 * rng.standard_normal((P, N, 1))))).astype(np.float32)
+        y = rng.integers(0, 2, N).astype(np.int32)
+    else:
+        y = rng.standard_normal(N).astype(np.float32)
+        preds = (y[None, :, None] + rng.standard_normal((P, N, 1)) * rng.uniform(0.5, 2, (P, 1, 1))).astype(np.float32)
+    preds[7] = preds[3]   # an exact duplicate: tie to the lower index
+    pd, yd = to_dev(preds, y)
+    sel, fin = tp.select_greedy(pd, yd, task, score, m_ens=12)
+    osel, ofin, obest, ogap = oracle.greedy(preds, y, task, score, m_ens=12, fp32_terms=True)
+    k = 0
+    while k < min(len(sel), len(osel)) and sel[k] == osel[k]:
+        k += 1
+    if k < max(len(sel), len(osel)):
+        # disagreement only at a near-tie of the oracle
+        assert ogap[k] <= 1e-6 * max(1.0, abs(obest[k])), (list(sel), list(osel), ogap)
+    else:
+        # per-row terms are fp32: the score is defined to fp32 term rounding
+        assert abs(fin - ofin) <= 1e-6 * max(1.0, abs(ofin))
+
+
+def test_select_greedy_worked_example(tp):
+    import json
+    import os
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "greedy_worked_example.json")))
+    preds = np.array(g["preds"], dtype=np.float32)
+    y = np.array(g["y"], dtype=np.float32)
+    pd, yd = to_dev(preds, y)
+    sel, fin = tp.select_greedy(pd, yd, g["task"], g["score"], m_ens=g["m_ens"])
+    assert list(sel) == g["selected"] and fin == g["final_score"]
+
+
+def test_errors_are_status_codes(tp):
+    hp = random_pack(2, 8, 1, seed=1)
+    pk, _ = pair(tp, "binary", 8, 1, hp, "bf16", 128)
+    X, y = make_data("binary", 300, 8, 1, 0)
+    Xd, yd = to_dev(X, y)
+    (idxd,) = to_dev(np.arange(200, dtype=np.int32))   # B > max_batch
+    with pytest.raises(tp.TabpackError) as ei:
+        pk.train_step(Xd, idxd, yd, 0)
+    assert ei.value.status == tp.TP_EINVAL
+    with pytest.raises(tp.TabpackError):
+        pk.get_params(5, 0)
+    with pytest.raises(tp.TabpackError):
+        tp.select_greedy(torch.zeros(3, 10, 1, device=DEV), torch.zeros(10, device=DEV), "regression",
+                         "accuracy", 2)

@@ -17,7 +17,6 @@ import torch.nn.functional as F
 
 from workloads import random_pack
 
-torch.set_default_dtype(torch.float64)
 
 
 class _RoundBF16(torch.autograd.Function):
