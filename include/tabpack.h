@@ -145,6 +145,31 @@ tp_status pack_select_greedy(const float* preds, int32_t P, int64_t N, int32_t d
                              int32_t task, int32_t score, int32_t m_ens, void* cuda_stream,
                              int32_t* selected, int32_t* n_selected, double* final_score);
 
+/* pack_select_greedy without any memory allocation.  (The paper has no
+ * counterpart: this is a deployment variant of the same selection.)
+ * Same arguments, results and stream behaviour as pack_select_greedy, but
+ * the scratch lives in one fixed 16 MiB array of device memory that the
+ * library defines at file scope; every GPU that loads the library holds it
+ * until the process exits.  It is for callers that cannot call cudaMalloc /
+ * cudaMallocAsync when they select: processes whose device memory is already
+ * fully reserved by another framework's caching allocator, loops that must
+ * not risk an out-of-memory failure or an allocator synchronisation, and
+ * embedding runtimes that forbid allocation calls after start-up.  It calls
+ * no allocating routine.
+ *   Limit: the problem must fit, N*d_out*8 + P*ceil(N/1024)*8 +
+ *   (4 + m_ens + P)*4 + 768 <= 16 MiB (e.g. N = 100000 rows of 10 classes
+ *   with P = 96 candidates); larger problems return TP_EINVAL with a message
+ *   in pack_last_error(NULL) and do nothing.
+ *   The first call on each device looks up the array's device address
+ *   (cudaGetSymbolAddress, with that device current); make that first call
+ *   before any stream capture.
+ *   All calls share the one array and each call starts by clearing what it
+ *   needs, so calls that overlap on the GPU (concurrent streams) race and
+ *   must be serialised by the caller.                                        */
+tp_status pack_select_greedy_static(const float* preds, int32_t P, int64_t N, int32_t d_out, const void* y,
+                                    int32_t task, int32_t score, int32_t m_ens, void* cuda_stream,
+                                    int32_t* selected, int32_t* n_selected, double* final_score);
+
 /* Base-model early stopping hook (Sec. 3.6): active is a host uint8 [m];
  * inactive members are skipped by every kernel and keep their parameters,
  * optimizer state and step count.                                           */
@@ -193,7 +218,8 @@ int64_t pack_launch_count(const tabpack_t* pack);
 tp_status pack_sizes(const tabpack_t* pack, int64_t* n_params, int64_t* device_bytes);
 
 /* Description of the last error on this pack (or, for pack == NULL, of the
- * last failed pack_create / pack_select_greedy on this thread).            */
+ * last failed pack_create / pack_select_greedy / pack_select_greedy_static
+ * on this thread).                                                         */
 const char* pack_last_error(const tabpack_t* pack);
 
 #ifdef __cplusplus

@@ -28,7 +28,7 @@ PHASES = ["gather", "fwd", "head", "bwd", "bias", "adamw", "predict"]
 
 # every entry point declared in include/tabpack.h
 SYMBOLS = ["pack_create", "pack_destroy", "pack_set_stream", "pack_train_step", "pack_forward_backward",
-           "pack_predict", "pack_select_greedy", "pack_set_active", "pack_get_params", "pack_set_params",
+           "pack_predict", "pack_select_greedy", "pack_select_greedy_static", "pack_set_active", "pack_get_params", "pack_set_params",
            "pack_get_grads", "pack_get_logits", "pack_debug_masks", "pack_debug_activations", "pack_profile_enable",
            "pack_profile_read", "pack_launch_count", "pack_sizes", "pack_last_error"]
 
@@ -67,6 +67,7 @@ def load_library(path: str = LIB_PATH):
         "pack_forward_backward": (st, [P, P, i64, P, P, i32, u32, P]),
         "pack_predict": (st, [P, P, i64, P]),
         "pack_select_greedy": (st, [P, i32, i64, i32, P, i32, i32, i32, P, P, P, P]),
+        "pack_select_greedy_static": (st, [P, i32, i64, i32, P, i32, i32, i32, P, P, P, P]),
         "pack_set_active": (st, [P, P]),
         "pack_get_params": (st, [P, i32, i32, P, P]),
         "pack_set_params": (st, [P, i32, i32, P, P]),
@@ -245,9 +246,11 @@ class Pack:
         return n.value, b.value
 
 
-def select_greedy(preds, y, task, score="loss", m_ens=32, stream=None):
+def select_greedy(preds, y, task, score="loss", m_ens=32, stream=None, static_scratch=False):
     """Greedy ensemble selection on the GPU.  preds float32 [P, N, d_out] and
-    y [N] CUDA tensors.  Returns (selected indices, final score)."""
+    y [N] CUDA tensors.  Returns (selected indices, final score).
+    static_scratch=True calls pack_select_greedy_static, the variant that
+    allocates no device memory (its scratch is a fixed array in the library)."""
     import torch
     t = TASKS[task] if isinstance(task, str) else int(task)
     s = SCORES[score] if isinstance(score, str) else int(score)
@@ -256,7 +259,7 @@ def select_greedy(preds, y, task, score="loss", m_ens=32, stream=None):
     sel = np.zeros(m_ens, dtype=np.int32)
     n = ctypes.c_int32()
     fin = ctypes.c_double()
-    _check(load_library().pack_select_greedy(_dptr(preds, torch.float32), P, N, d_out, _dptr(y, ydt), t, s,
-                                             int(m_ens), _stream_ptr(stream), _hptr(sel), ctypes.byref(n),
-                                             ctypes.byref(fin)))
+    fn = load_library().pack_select_greedy_static if static_scratch else load_library().pack_select_greedy
+    _check(fn(_dptr(preds, torch.float32), P, N, d_out, _dptr(y, ydt), t, s, int(m_ens), _stream_ptr(stream),
+              _hptr(sel), ctypes.byref(n), ctypes.byref(fin)))
     return sel[:n.value].copy(), fin.value

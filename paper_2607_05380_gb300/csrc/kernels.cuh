@@ -106,6 +106,9 @@ void launch_predict_head(cudaStream_t st, const PredictHeadArgs<T>& g, int n_job
 void launch_debug_masks(cudaStream_t st, uint8_t* out, int B, int w, uint64_t seed, uint32_t member,
                         uint32_t layer, uint32_t step, uint32_t T);
 
+// Sets the per-thread message pack_last_error(NULL) returns (tabpack.cu).
+void record_thread_error(const char* msg);
+
 // greedy selection (select.cu)
 struct SelectScratch {
   double* S;              // running ensemble sum [N, d_out]

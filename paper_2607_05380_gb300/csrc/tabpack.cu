@@ -582,6 +582,8 @@ tp_status check_ml(tabpack* h, int member, int layer) {
 
 }  // namespace
 
+void tp::record_thread_error(const char* msg) { g_thread_error = msg; }
+
 // ====================================================================== ABI
 extern "C" {
 
