@@ -350,7 +350,7 @@ tp_status build_schedule(tabpack* h) {
   h->n_head_jobs = (int)hj.size();
   h->n_bias_jobs = (int)bj.size();
   h->n_chunks = (int)ch.size();
-  if (h->bf16) TP_TRY(tc_build_plan(h->tc, h->cfg, h->depth, h->width, h->active, h->W_off, h->act_off,
+  if (h->bf16) TP_TRY(tc_build_plan(h->tc, h->cfg, h->depth, h->width, h->active, h->W_off, h->b_off, h->act_off,
                                     h->dz_off, h->d_in_pad, h->B_cap, h->wq, h->xb, h->act, h->dz, h->err));
   return TP_OK;
 }
@@ -423,7 +423,7 @@ tp_status run_forward(tabpack* h, int B, int B_pad, uint32_t step, int train) {
     int slot;
     prof_begin(h, train ? TP_PH_FWD : TP_PH_PREDICT, &slot);
     if (h->bf16 && h->tc.enabled) {
-      TP_TRY(tc_run_fwd(h->tc, h->st, l, B, B_pad, step, train, h->cfg.seed, h->params, h->mem_dev, h->err));
+      TP_TRY(tc_run_fwd(h->tc, h->st, l, B, B_pad, step, train, h->cfg.seed, h->params, h->mem_dev, h->act, h->err));
     } else {
       auto g = gemm_args<T>(h, B, B_pad, step, train);
       launch_gemm_simt<T>(h->st, g, h->fwd_rng[l].first, h->fwd_rng[l].second);
@@ -475,7 +475,7 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
   for (int l = h->Lmax - 1; l >= 0; --l) {
     prof_begin(h, TP_PH_BWD, &slot);
     if (h->bf16 && h->tc.enabled) {
-      TP_TRY(tc_run_bwd(h->tc, h->st, l, B, B_pad, h->grads, h->mem_dev, h->err));
+      TP_TRY(tc_run_bwd(h->tc, h->st, l, B, B_pad, h->grads, h->mem_dev, h->act, h->dz, h->err));
     } else {
       auto g = gemm_args<T>(h, B, B_pad, step, 1);
       launch_gemm_simt<T>(h->st, g, h->bwd_rng[l].first, h->bwd_rng[l].second);

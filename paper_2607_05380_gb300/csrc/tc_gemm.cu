@@ -1,25 +1,650 @@
-// tc_gemm.cu -- tensor-core grouped GEMM plan (placeholder: disabled).
+// tc_gemm.cu -- persistent warp-specialised grouped GEMM on tcgen05 (sm_103a).
+//
+// Every launch processes a list of 128 x N output tiles (N <= 256, a
+// multiple of 16) of many members' products; each persistent CTA (one per
+// SM) walks the list with stride gridDim.x (the list is sorted by cost,
+// largest first).  Warp roles:
+//   warp 0     TMA producer: per 64-wide K block, loads the A tile
+//              (2 boxes of 64 x 64 bf16) and the B tile (N/64 boxes) into a
+//              4-stage shared-memory ring, 128-byte swizzled.
+//   warp 1     MMA issuer: one thread issues tcgen05.mma (M=128, K=16 per
+//              instruction) into one of two TMEM accumulators (2 x 256
+//              fp32 columns) and commits each stage back to the producer.
+//   warps 2-5  epilogue: tcgen05.ld of the accumulator (warp w reads TMEM
+//              lanes 32 (w % 4) .. +31, i.e. those output rows) and the
+//              fused epilogue of the product kind:
+//                kFwd   z = acc + b; h = dropout(relu(z)) / (1 - p)   -> bf16
+//                kDgrad dz_prev = acc * [H_prev > 0] / (1 - p)          -> bf16
+//                kWgrad dW = acc                                        -> fp32
+// Ragged K (member widths that are multiples of 16 but not of 64) issues
+// only the K=16 steps that exist; out-of-range operand rows and columns are
+// zero-filled by TMA.  Operands are read K-major or MN-major straight from
+// their row-major arrays through the descriptor's major-ness bits, so no
+// transposed copies are kept.
+//
+// Every mbarrier wait is bounded (2 s): a role that gives up sets the
+// pack's device error word and an abort flag in shared memory; the other
+// roles then stop, the producer waits (bounded) for its own copies in
+// flight, the MMA thread for its own MMAs, TMEM is freed and the CTA exits.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+
 #include "tc_gemm.cuh"
 
 namespace tp {
+namespace {
 
-tp_status tc_build_plan(TcPlan& plan, const tp_config&, const std::vector<int32_t>&, const std::vector<int32_t>&,
-                        const std::vector<uint8_t>&, const std::vector<std::array<int64_t, kMaxDepth + 1>>&,
-                        const std::vector<std::array<int64_t, kMaxDepth>>&,
-                        const std::vector<std::array<int64_t, kMaxDepth>>&, int, int, const __nv_bfloat16*,
-                        const void*, const void*, const void*, std::string&) {
-  plan.enabled = false;
+constexpr int kStages = 4;
+constexpr int kBoxBytes = 64 * 64 * 2;  // one 64 x 64 bf16 TMA box
+constexpr int kABytes = 2 * kBoxBytes;  // 128 rows
+constexpr int kBBytes = 4 * kBoxBytes;  // up to 256 rows / columns
+constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kThreads = 192;
+constexpr uint32_t kTmemCols = 512;
+constexpr int kAccCols = 256;
+constexpr uint64_t kWaitNs = 2000000000ull;
+
+struct SmemTail {
+  uint64_t full[kStages];
+  uint64_t empty[kStages];
+  uint64_t tfull[2];
+  uint64_t tempty[2];
+  uint64_t done;
+  uint32_t tmem_base;
+  int abort;
+};
+constexpr int kSmemBytes = kStages * kStageBytes + 1024 + (int)sizeof(SmemTail) + 64;
+
+struct TcArgs {
+  const TcTile* tiles;
+  int32_t n_tiles;
+  int32_t B, B_pad;
+  uint32_t step;
+  int32_t train;
+  uint64_t seed;
+  const CUtensorMap* maps;
+  const float* params;
+  const MemberDev* mem;
+  __nv_bfloat16* act;
+  __nv_bfloat16* dz;
+  float* grads;
+  int* err;
+};
+
+// ------------------------------------------------------------ PTX helpers
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait: false if the abort flag is raised or the budget runs out
+// (then the flag and the device error word are set).
+__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* err,
+                                       uint64_t budget_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (global_ns() - t0 > budget_ns) {
+      *abort_flag = 1;
+      atomicExch(err, 1);
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint64_t* bar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
+      "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y)
+      : "memory");
+}
+__device__ __forceinline__ void tensormap_acquire(const CUtensorMap* map) {
+  asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(map) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Shared-memory matrix descriptor: start, leading / stride byte offsets,
+// version 1 (bits 46-48), 128-byte swizzle (layout 2, bits 61-63).
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = (uint64_t)((addr >> 4) & 0x3FFFu);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulate, bf16 A and B.
+__device__ __forceinline__ uint32_t instr_desc(int n, int a_mn, int b_mn) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)a_mn << 15) | ((uint32_t)b_mn << 16) |
+         ((uint32_t)(n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+}
+
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
+          d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]), "=r"(v[8]),
+        "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]),
+        "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]),
+        "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+  __nv_bfloat162 t = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&t);
+}
+
+__device__ __forceinline__ bool tile_live(const TcTile& t, int B_pad) { return t.kind == kWgrad || t.m0 < B_pad; }
+
+// ------------------------------------------------------------------ kernel
+__global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  SmemTail* tl = (SmemTail*)(smem + kStages * kStageBytes);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&tl->full[s], 1);
+      mbar_init(&tl->empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tl->tfull[b], 1);
+      mbar_init(&tl->tempty[b], 128);
+    }
+    mbar_init(&tl->done, 1);
+    tl->abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tl->tmem_base)),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tl->tmem_base;
+  volatile int* abort_flag = &tl->abort;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------------------------------------------------- producer
+      uint32_t stage = 0, phase = 0;
+      uint32_t issued_mask = 0, last_parity = 0;  // per stage: ever issued, parity of the last issue
+      bool ok = true;
+      for (int t = blockIdx.x; ok && t < g.n_tiles; t += gridDim.x) {
+        const TcTile tile = g.tiles[t];
+        if (!tile_live(tile, g.B_pad)) continue;
+        const int K = tile.k_len ? tile.k_len : g.B_pad;
+        const CUtensorMap* ma = g.maps + tile.map_a;
+        const CUtensorMap* mb = g.maps + tile.map_b;
+        tensormap_acquire(ma);
+        tensormap_acquire(mb);
+        const int nb = (tile.n_len + 63) >> 6;
+        const uint32_t bytes = (uint32_t)(2 + nb) * kBoxBytes;
+        for (int k0 = 0; k0 < K; k0 += 64) {
+          if (!mbar_wait(&tl->empty[stage], phase ^ 1u, abort_flag, g.err, kWaitNs)) {
+            ok = false;
+            break;
+          }
+          uint64_t* fb = &tl->full[stage];
+          mbar_expect_tx(fb, bytes);
+          const uint32_t a = smem_u32(smem + stage * kStageBytes);
+          const uint32_t b = a + kABytes;
+          if (tile.kind == kWgrad) {  // A = dZ, MN-major: x = output row (unit), y = batch row
+            tma_load_2d(a, ma, fb, tile.m0, k0);
+            tma_load_2d(a + kBoxBytes, ma, fb, tile.m0 + 64, k0);
+          } else {  // A K-major: x = k, y = batch row
+            tma_load_2d(a, ma, fb, k0, tile.m0);
+            tma_load_2d(a + kBoxBytes, ma, fb, k0, tile.m0 + 64);
+          }
+          for (int q = 0; q < nb; ++q) {
+            if (tile.kind == kFwd) tma_load_2d(b + q * kBoxBytes, mb, fb, k0, tile.n0 + 64 * q);
+            else tma_load_2d(b + q * kBoxBytes, mb, fb, tile.n0 + 64 * q, k0);
+          }
+          issued_mask |= 1u << stage;
+          last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      // wait (bounded) until every copy this thread issued has landed
+      for (int s = 0; s < kStages; ++s)
+        if (issued_mask & (1u << s)) {
+          int dummy_abort = 0;
+          mbar_wait(&tl->full[s], (last_parity >> s) & 1u, &dummy_abort, g.err, kWaitNs);
+        }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // --------------------------------------------------------------- MMA
+      uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; ok && t < g.n_tiles; t += gridDim.x) {
+        const TcTile tile = g.tiles[t];
+        if (!tile_live(tile, g.B_pad)) continue;
+        const int K = tile.k_len ? tile.k_len : g.B_pad;
+        if (!mbar_wait(&tl->tempty[acc], acc_phase ^ 1u, abort_flag, g.err, kWaitNs)) break;
+        tc_fence_after();
+        const uint32_t d = tmem + acc * kAccCols;
+        const int a_mn = tile.kind == kWgrad, b_mn = tile.kind != kFwd;
+        const uint32_t idesc = instr_desc(tile.n_len, a_mn, b_mn);
+        for (int k0 = 0; k0 < K; k0 += 64) {
+          if (!mbar_wait(&tl->full[stage], phase, abort_flag, g.err, kWaitNs)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a = smem_u32(smem + stage * kStageBytes);
+          const uint32_t b = a + kABytes;
+          const int nk = min(4, (K - k0 + 15) >> 4);
+          for (int kk = 0; kk < nk; ++kk) {
+            const uint64_t ad = a_mn ? smem_desc(a + kk * 2048, kBoxBytes, 1024) : smem_desc(a + kk * 32, 16, 1024);
+            const uint64_t bd = b_mn ? smem_desc(b + kk * 2048, kBoxBytes, 1024) : smem_desc(b + kk * 32, 16, 1024);
+            umma_bf16(d, ad, bd, idesc, (k0 | kk) != 0);
+          }
+          umma_commit(&tl->empty[stage]);
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit(&tl->tfull[acc]);
+        acc ^= 1u;
+        if (acc == 0) acc_phase ^= 1u;
+      }
+      // all MMAs this thread issued have completed before TMEM is freed
+      umma_commit(&tl->done);
+      int dummy_abort = 0;
+      mbar_wait(&tl->done, 0, &dummy_abort, g.err, kWaitNs);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;
+    const int row = 32 * q + lane;
+    uint32_t acc = 0, acc_phase = 0;
+    for (int t = blockIdx.x; t < g.n_tiles; t += gridDim.x) {
+      const TcTile tile = g.tiles[t];
+      if (!tile_live(tile, g.B_pad)) continue;
+      if (!mbar_wait(&tl->tfull[acc], acc_phase, abort_flag, g.err, kWaitNs)) break;
+      tc_fence_after();
+      const MemberDev md = g.mem[tile.member];
+      const int m_lim = tile.m_real ? tile.m_real : g.B_pad;
+      const int r = tile.m0 + row;
+      const bool row_ok = r < m_lim;
+      const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + acc * kAccCols;
+      for (int c = 0; c < tile.n_len; c += 32) {
+        uint32_t v[32];
+        tmem_ld32(taddr + c, v);
+        if (!row_ok) continue;
+        const int col0 = tile.n0 + c;
+        const int ncols = min(32, tile.n_real - col0);  // a multiple of 8 (widths are multiples of 16)
+        if (ncols <= 0) continue;
+        if (tile.kind == kFwd) {
+          uint32_t keep = 0xFFFFFFFFu;
+          if (g.train && md.drop_T) {
+            keep = 0;
+#pragma unroll
+            for (int g4 = 0; g4 < 8; ++g4)
+              keep |= keep_bits4(g.seed, (uint32_t)tile.member, (uint32_t)tile.layer, g.step, (uint32_t)r,
+                                 (uint32_t)((col0 >> 2) + g4), md.drop_T)
+                      << (4 * g4);
+          }
+          const float sc = g.train ? md.scale : 1.f;
+          const float* bias = g.params + tile.aux_off + col0;
+          __nv_bfloat16* out = g.act + tile.c_off + (int64_t)r * tile.ldc + col0;
+#pragma unroll
+          for (int s = 0; s < 4; ++s) {
+            if (8 * s >= ncols) break;
+            uint32_t pk[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              float h2[2];
+#pragma unroll
+              for (int u = 0; u < 2; ++u) {
+                const int j = 8 * s + 2 * e + u;
+                const float z = __uint_as_float(v[j]) + __ldg(bias + j);
+                const float a = z > 0.f ? z : 0.f;
+                h2[u] = ((keep >> j) & 1u) ? a * sc : 0.f;
+              }
+              pk[e] = pack_bf16x2(h2[0], h2[1]);
+            }
+            *reinterpret_cast<uint4*>(out + 8 * s) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          }
+        } else if (tile.kind == kDgrad) {
+          const __nv_bfloat16* hm = g.act + tile.aux_off + (int64_t)r * tile.ldc + col0;
+          __nv_bfloat16* out = g.dz + tile.c_off + (int64_t)r * tile.ldc + col0;
+#pragma unroll
+          for (int s = 0; s < 4; ++s) {
+            if (8 * s >= ncols) break;
+            const uint4 hv = *reinterpret_cast<const uint4*>(hm + 8 * s);
+            const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&hv);
+            uint32_t pk[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const int j = 8 * s + 2 * e;
+              const float x0 = __bfloat162float(hb[2 * e]) > 0.f ? __uint_as_float(v[j]) * md.scale : 0.f;
+              const float x1 = __bfloat162float(hb[2 * e + 1]) > 0.f ? __uint_as_float(v[j + 1]) * md.scale : 0.f;
+              pk[e] = pack_bf16x2(x0, x1);
+            }
+            *reinterpret_cast<uint4*>(out + 8 * s) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          }
+        } else {
+          float* out = g.grads + tile.c_off + (int64_t)r * tile.ldc + col0;
+#pragma unroll
+          for (int s = 0; s < 8; ++s) {
+            if (4 * s >= ncols) break;
+            *reinterpret_cast<float4*>(out + 4 * s) =
+                make_float4(__uint_as_float(v[4 * s]), __uint_as_float(v[4 * s + 1]), __uint_as_float(v[4 * s + 2]),
+                            __uint_as_float(v[4 * s + 3]));
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&tl->tempty[acc]);
+      acc ^= 1u;
+      if (acc == 0) acc_phase ^= 1u;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+  }
+}
+
+// ------------------------------------------------------------------- host
+PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = (PFN_cuTensorMapEncodeTiled_v12000)p;
+  }
+  return fn;
+}
+
+// 2-D bf16 row-major matrix [rows, cols] with 64 x 64 boxes, 128-byte swizzle.
+bool encode_map(CUtensorMap* m, const void* base, int64_t cols, int64_t rows, std::string& err) {
+  auto fn = get_encode();
+  if (!fn) {
+    err = "cuTensorMapEncodeTiled unavailable";
+    return false;
+  }
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+  cuuint32_t box[2] = {64, 64};
+  cuuint32_t es[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    err = "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")";
+    return false;
+  }
+  return true;
+}
+
+}  // namespace
+
+tp_status tc_build_plan(TcPlan& plan, const tp_config& cfg, const std::vector<int32_t>& depth,
+                        const std::vector<int32_t>& width, const std::vector<uint8_t>& active,
+                        const std::vector<std::array<int64_t, kMaxDepth + 1>>& W_off,
+                        const std::vector<std::array<int64_t, kMaxDepth + 1>>& b_off,
+                        const std::vector<std::array<int64_t, kMaxDepth>>& act_off,
+                        const std::vector<std::array<int64_t, kMaxDepth>>& dz_off, int d_in_pad, int B_cap,
+                        const __nv_bfloat16* wq, const void* xb, const void* act, const void* dz,
+                        std::string& err) {
+  const int m = cfg.m;
+  if (plan.maps_dev == nullptr) {
+    // tensor maps: 0 = gathered batch; then per (member, layer) act, dz, W
+    std::vector<CUtensorMap> maps;
+    plan.map_act.assign((size_t)m * kMaxDepth, -1);
+    plan.map_dz.assign((size_t)m * kMaxDepth, -1);
+    plan.map_w.assign((size_t)m * kMaxDepth, -1);
+    CUtensorMap mp;
+    if (!encode_map(&mp, xb, d_in_pad, B_cap, err)) return TP_ECUDA;
+    maps.push_back(mp);
+    const __nv_bfloat16* actb = (const __nv_bfloat16*)act;
+    const __nv_bfloat16* dzb = (const __nv_bfloat16*)dz;
+    for (int i = 0; i < m; ++i)
+      for (int l = 0; l < depth[i]; ++l) {
+        const int w = width[i], in_pad = l == 0 ? d_in_pad : w;
+        if (!encode_map(&mp, actb + act_off[i][l], w, B_cap, err)) return TP_ECUDA;
+        plan.map_act[(size_t)i * kMaxDepth + l] = (int)maps.size();
+        maps.push_back(mp);
+        if (!encode_map(&mp, dzb + dz_off[i][l], w, B_cap, err)) return TP_ECUDA;
+        plan.map_dz[(size_t)i * kMaxDepth + l] = (int)maps.size();
+        maps.push_back(mp);
+        if (!encode_map(&mp, wq + W_off[i][l], in_pad, w, err)) return TP_ECUDA;
+        plan.map_w[(size_t)i * kMaxDepth + l] = (int)maps.size();
+        maps.push_back(mp);
+      }
+    plan.n_maps = (int)maps.size();
+    if (cudaMalloc(&plan.maps_dev, sizeof(CUtensorMap) * maps.size()) != cudaSuccess) {
+      err = "cudaMalloc(tensor maps) failed";
+      return TP_ENOMEM;
+    }
+    if (cudaMemcpy(plan.maps_dev, maps.data(), sizeof(CUtensorMap) * maps.size(), cudaMemcpyHostToDevice) !=
+        cudaSuccess) {
+      err = "cudaMemcpy(tensor maps) failed";
+      return TP_ECUDA;
+    }
+    if (cudaMalloc(&plan.err_dev, sizeof(int)) != cudaSuccess || cudaMemset(plan.err_dev, 0, sizeof(int)) != cudaSuccess) {
+      err = "cudaMalloc(error word) failed";
+      return TP_ENOMEM;
+    }
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&plan.n_sm, cudaDevAttrMultiProcessorCount, dev);
+    if (cudaFuncSetAttribute(k_tc_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess) {
+      err = "cudaFuncSetAttribute(smem) failed";
+      return TP_ECUDA;
+    }
+  }
+
+  // tiles of the active members, per launch, largest first
+  int Lmax = 0;
+  for (int i = 0; i < m; ++i) Lmax = std::max(Lmax, depth[i]);
+  std::vector<TcTile> all;
+  plan.fwd_rng.assign(Lmax, {0, 0});
+  plan.bwd_rng.assign(Lmax, {0, 0});
+  auto cost = [&](const TcTile& t) { return (int64_t)(t.k_len ? t.k_len : B_cap) * t.n_len; };
+  auto sorted_append = [&](std::vector<TcTile>& v) {
+    std::stable_sort(v.begin(), v.end(), [&](const TcTile& a, const TcTile& b) { return cost(a) > cost(b); });
+    const int base = (int)all.size();
+    all.insert(all.end(), v.begin(), v.end());
+    return std::make_pair(base, (int)v.size());
+  };
+  for (int l = 0; l < Lmax; ++l) {
+    std::vector<TcTile> v;
+    for (int i = 0; i < m; ++i) {
+      if (!active[i] || depth[i] <= l) continue;
+      const int w = width[i];
+      for (int m0 = 0; m0 < B_cap; m0 += 128)
+        for (int n0 = 0; n0 < w; n0 += 256) {
+          TcTile t{};
+          t.kind = kFwd; t.member = i; t.layer = l;
+          t.m0 = m0; t.n0 = n0; t.n_len = std::min(256, w - n0);
+          t.m_real = 0; t.n_real = w;
+          t.k_len = l == 0 ? d_in_pad : w;
+          t.map_a = l == 0 ? 0 : plan.map_act[(size_t)i * kMaxDepth + l - 1];
+          t.map_b = plan.map_w[(size_t)i * kMaxDepth + l];
+          t.ldc = w;
+          t.c_off = act_off[i][l];
+          t.aux_off = b_off[i][l];
+          v.push_back(t);
+        }
+    }
+    plan.fwd_rng[l] = sorted_append(v);
+  }
+  for (int l = Lmax - 1; l >= 0; --l) {
+    std::vector<TcTile> v;
+    for (int i = 0; i < m; ++i) {
+      if (!active[i] || depth[i] <= l) continue;
+      const int w = width[i], in_pad = l == 0 ? d_in_pad : w;
+      if (l > 0)
+        for (int m0 = 0; m0 < B_cap; m0 += 128)
+          for (int n0 = 0; n0 < w; n0 += 256) {
+            TcTile t{};
+            t.kind = kDgrad; t.member = i; t.layer = l;
+            t.m0 = m0; t.n0 = n0; t.n_len = std::min(256, w - n0);
+            t.m_real = 0; t.n_real = w;
+            t.k_len = w;
+            t.map_a = plan.map_dz[(size_t)i * kMaxDepth + l];
+            t.map_b = plan.map_w[(size_t)i * kMaxDepth + l];
+            t.ldc = w;
+            t.c_off = dz_off[i][l - 1];
+            t.aux_off = act_off[i][l - 1];
+            v.push_back(t);
+          }
+      for (int m0 = 0; m0 < w; m0 += 128)
+        for (int n0 = 0; n0 < in_pad; n0 += 256) {
+          TcTile t{};
+          t.kind = kWgrad; t.member = i; t.layer = l;
+          t.m0 = m0; t.n0 = n0; t.n_len = (int)round_up(std::min(256, in_pad - n0), 16);
+          t.m_real = w; t.n_real = in_pad;
+          t.k_len = 0;
+          t.map_a = plan.map_dz[(size_t)i * kMaxDepth + l];
+          t.map_b = l == 0 ? 0 : plan.map_act[(size_t)i * kMaxDepth + l - 1];
+          t.ldc = in_pad;
+          t.c_off = W_off[i][l];
+          t.aux_off = 0;
+          v.push_back(t);
+        }
+    }
+    plan.bwd_rng[l] = sorted_append(v);
+  }
+  if ((int)all.size() + 1 > plan.cap_tiles) {
+    if (plan.tiles_dev) cudaFree(plan.tiles_dev);
+    plan.cap_tiles = (int)all.size() + 1;
+    if (cudaMalloc(&plan.tiles_dev, sizeof(TcTile) * plan.cap_tiles) != cudaSuccess) {
+      err = "cudaMalloc(tc tiles) failed";
+      return TP_ENOMEM;
+    }
+  }
+  if (!all.empty() &&
+      cudaMemcpy(plan.tiles_dev, all.data(), sizeof(TcTile) * all.size(), cudaMemcpyHostToDevice) != cudaSuccess) {
+    err = "cudaMemcpy(tc tiles) failed";
+    return TP_ECUDA;
+  }
+  plan.enabled = true;
   return TP_OK;
 }
-tp_status tc_run_fwd(TcPlan&, cudaStream_t, int, int, int, uint32_t, int, uint64_t, const float*, const MemberDev*,
-                     std::string& err) {
-  err = "tensor-core plan disabled";
-  return TP_ESTATE;
+
+static tp_status launch(TcPlan& plan, cudaStream_t st, const std::pair<int, int>& rng, int B, int B_pad,
+                        uint32_t step, int train, uint64_t seed, const float* params, const MemberDev* mem,
+                        void* act, void* dz, float* grads, std::string& err) {
+  if (rng.second <= 0) return TP_OK;
+  TcArgs a;
+  a.tiles = plan.tiles_dev + rng.first;
+  a.n_tiles = rng.second;
+  a.B = B;
+  a.B_pad = B_pad;
+  a.step = step;
+  a.train = train;
+  a.seed = seed;
+  a.maps = plan.maps_dev;
+  a.params = params;
+  a.mem = mem;
+  a.act = (__nv_bfloat16*)act;
+  a.dz = (__nv_bfloat16*)dz;
+  a.grads = grads;
+  a.err = plan.err_dev;
+  const int grid = std::max(1, std::min(rng.second, plan.n_sm));
+  k_tc_gemm<<<grid, kThreads, kSmemBytes, st>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    err = std::string("tcgen05 GEMM launch: ") + cudaGetErrorString(e);
+    return TP_ECUDA;
+  }
+  return TP_OK;
 }
-tp_status tc_run_bwd(TcPlan&, cudaStream_t, int, int, int, float*, const MemberDev*, std::string& err) {
-  err = "tensor-core plan disabled";
-  return TP_ESTATE;
+
+tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, uint32_t step, int train,
+                     uint64_t seed, const float* params, const MemberDev* mem, void* act, std::string& err) {
+  return launch(plan, st, plan.fwd_rng[layer], B, B_pad, step, train, seed, params, mem, act, nullptr, nullptr, err);
 }
-void tc_free_plan(TcPlan& plan) { plan.enabled = false; }
+
+tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, float* grads,
+                     const MemberDev* mem, void* act, void* dz, std::string& err) {
+  return launch(plan, st, plan.bwd_rng[layer], B, B_pad, 0, 0, 0, nullptr, mem, act, dz, grads, err);
+}
+
+tp_status tc_check(TcPlan& plan, cudaStream_t st, std::string& err) {
+  if (!plan.err_dev) return TP_OK;
+  int v = 0;
+  if (cudaMemcpyAsync(&v, plan.err_dev, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess) {
+    err = "reading the tcgen05 error word failed";
+    return TP_ECUDA;
+  }
+  if (v) {
+    cudaMemsetAsync(plan.err_dev, 0, sizeof(int), st);
+    err = "a tcgen05 GEMM pipeline wait timed out";
+    return TP_ETIMEOUT;
+  }
+  return TP_OK;
+}
+
+void tc_free_plan(TcPlan& plan) {
+  if (plan.maps_dev) cudaFree(plan.maps_dev);
+  if (plan.tiles_dev) cudaFree(plan.tiles_dev);
+  if (plan.err_dev) cudaFree(plan.err_dev);
+  plan.maps_dev = nullptr;
+  plan.tiles_dev = nullptr;
+  plan.err_dev = nullptr;
+  plan.enabled = false;
+}
 
 }  // namespace tp
