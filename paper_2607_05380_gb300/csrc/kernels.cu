@@ -147,30 +147,67 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
+// 8 consecutive activations of a row as floats (16-byte bf16 / 2 x 16-byte fp32 loads).
+__device__ __forceinline__ void load8(const __nv_bfloat16* p, float (&h)[8]) {
+  const uint4 u = *reinterpret_cast<const uint4*>(p);
+  const __nv_bfloat16* b = reinterpret_cast<const __nv_bfloat16*>(&u);
+#pragma unroll
+  for (int k = 0; k < 8; ++k) h[k] = __bfloat162float(b[k]);
+}
+__device__ __forceinline__ void load8(const float* p, float (&h)[8]) {
+  const float4 a = *reinterpret_cast<const float4*>(p), b = *reinterpret_cast<const float4*>(p + 4);
+  h[0] = a.x; h[1] = a.y; h[2] = a.z; h[3] = a.w; h[4] = b.x; h[5] = b.y; h[6] = b.z; h[7] = b.w;
+}
+__device__ __forceinline__ void store8(__nv_bfloat16* p, const float (&v)[8]) {
+  uint4 u;
+  __nv_bfloat162* b = reinterpret_cast<__nv_bfloat162*>(&u);
+#pragma unroll
+  for (int k = 0; k < 4; ++k) b[k] = __floats2bfloat162_rn(v[2 * k], v[2 * k + 1]);
+  *reinterpret_cast<uint4*>(p) = u;
+}
+__device__ __forceinline__ void store8(float* p, const float (&v)[8]) {
+  *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+  *reinterpret_cast<float4*>(p + 4) = make_float4(v[4], v[5], v[6], v[7]);
+}
+
+// Head kernel.  Per row (one warp, lanes over 8-column groups): logits,
+// per-row loss and dlogits, then dZ of the last hidden layer for the same
+// row while it is in L1.  Then per column group (threads) the block's
+// partial head-weight gradient sum over its 128 rows, in row order.
 template <typename T, int DO>
 __global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
   const HeadJob jb = g.jobs[blockIdx.x];
-  const int r0 = jb.blk * kRowTile;
+  const int r0 = jb.blk * kHeadRows;
   if (r0 >= g.B_pad) return;
   const MemberDev md = g.mem[jb.member];
   const int w = md.w, d_out = g.d_out;
+  const int ng = w >> 3;  // 8-column groups (widths are multiples of 16)
   const T* H = g.act + jb.h_off;
   const float* Wh = g.params + jb.w_off;
   const float* bh = g.params + jb.b_off;
-  __shared__ float dlog[kRowTile][DO];
-  __shared__ float lrow[kRowTile];
+  __shared__ float dlog[kHeadRows][DO];
+  __shared__ float lrow[kHeadRows];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float invB = 1.f / (float)g.B;
-  for (int rr = warp; rr < kRowTile; rr += 8) {
+  T* dZ = g.dz + jb.dz_off;
+  for (int rr = warp; rr < kHeadRows; rr += 8) {
     const int r = r0 + rr;
+    const T* Hr = H + (int64_t)r * w;
     float acc[DO];
 #pragma unroll
     for (int c = 0; c < DO; ++c) acc[c] = 0.f;
-    for (int j = lane; j < w; j += 32) {
-      float h = Elem<T>::to_f(H[(int64_t)r * w + j]);
+    for (int gi = lane; gi < ng; gi += 32) {
+      float h[8];
+      load8(Hr + 8 * gi, h);
 #pragma unroll
-      for (int c = 0; c < DO; ++c)
-        if (c < d_out) acc[c] = fmaf(h, Wh[(int64_t)c * w + j], acc[c]);
+      for (int c = 0; c < DO; ++c) {
+        if (c < d_out) {
+          float w8[8];
+          load8(Wh + (int64_t)c * w + 8 * gi, w8);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) acc[c] = fmaf(h[k], w8[k], acc[c]);
+        }
+      }
     }
 #pragma unroll
     for (int c = 0; c < DO; ++c)
@@ -220,41 +257,70 @@ __global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
       for (int c = 0; c < DO; ++c) dlog[rr][c] = dl[c];
       lrow[rr] = loss;
     }
+    // dZ of the last hidden layer for this row: (dlogits W_h) * [H > 0] / (1 - p)
+    T* dZr = dZ + (int64_t)r * w;
+    for (int gi = lane; gi < ng; gi += 32) {
+      float h[8], s[8];
+      load8(Hr + 8 * gi, h);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) s[k] = 0.f;
+#pragma unroll
+      for (int c = 0; c < DO; ++c) {
+        if (c < d_out) {
+          float w8[8];
+          load8(Wh + (int64_t)c * w + 8 * gi, w8);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) s[k] = fmaf(dl[c], w8[k], s[k]);
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 8; ++k) s[k] = h[k] > 0.f ? s[k] * md.scale : 0.f;
+      store8(dZr + 8 * gi, s);
+    }
   }
   __syncthreads();
-  // dZ of the last hidden layer: (dlogits W_h) * [H > 0] / (1 - p)
-  T* dZ = g.dz + jb.dz_off;
-  for (int e = threadIdx.x; e < kRowTile * w; e += blockDim.x) {
-    const int rr = e / w, j = e % w;
-    const int64_t o = (int64_t)(r0 + rr) * w + j;
-    float s = 0.f;
-#pragma unroll
-    for (int c = 0; c < DO; ++c) if (c < d_out) s = fmaf(dlog[rr][c], Wh[(int64_t)c * w + j], s);
-    const float h = Elem<T>::to_f(H[o]);
-    dZ[o] = Elem<T>::from_f(h > 0.f ? s * md.scale : 0.f);
-  }
-  // partial head gradients of this block
+  // partial head gradients of this block: per group of G columns, all
+  // classes, rows in increasing order
+  constexpr int G = DO == 1 ? 8 : (DO <= 16 ? 4 : 2);
   float* part = g.head_part + jb.part_off;
-  for (int j = threadIdx.x; j < w; j += blockDim.x) {
-    float a[DO];
+  for (int gi = threadIdx.x; gi < w / G; gi += blockDim.x) {
+    float a[DO][G];
 #pragma unroll
-    for (int c = 0; c < DO; ++c) a[c] = 0.f;
-    for (int rr = 0; rr < kRowTile; ++rr) {
-      const float h = Elem<T>::to_f(H[(int64_t)(r0 + rr) * w + j]);
+    for (int c = 0; c < DO; ++c)
 #pragma unroll
-      for (int c = 0; c < DO; ++c) if (c < d_out) a[c] = fmaf(dlog[rr][c], h, a[c]);
+      for (int k = 0; k < G; ++k) a[c][k] = 0.f;
+#pragma unroll 4
+    for (int rr = 0; rr < kHeadRows; ++rr) {
+      const T* hp = H + (int64_t)(r0 + rr) * w + G * gi;
+      float h[G];
+      if constexpr (G == 8) {
+        load8(hp, h);
+      } else {
+#pragma unroll
+        for (int k = 0; k < G; ++k) h[k] = Elem<T>::to_f(hp[k]);
+      }
+#pragma unroll
+      for (int c = 0; c < DO; ++c)
+        if (c < d_out) {
+          const float d = dlog[rr][c];
+#pragma unroll
+          for (int k = 0; k < G; ++k) a[c][k] = fmaf(d, h[k], a[c][k]);
+        }
     }
 #pragma unroll
-    for (int c = 0; c < DO; ++c) if (c < d_out) part[(int64_t)c * w + j] = a[c];
+    for (int c = 0; c < DO; ++c)
+      if (c < d_out)
+#pragma unroll
+        for (int k = 0; k < G; ++k) part[(int64_t)c * w + G * gi + k] = a[c][k];
   }
   if (threadIdx.x < d_out) {
     float s = 0.f;
-    for (int rr = 0; rr < kRowTile; ++rr) s += dlog[rr][threadIdx.x];
+    for (int rr = 0; rr < kHeadRows; ++rr) s += dlog[rr][threadIdx.x];
     part[(int64_t)d_out * w + threadIdx.x] = s;
   }
   if (threadIdx.x == 0) {
     float s = 0.f;
-    for (int rr = 0; rr < kRowTile; ++rr) s += lrow[rr];
+    for (int rr = 0; rr < kHeadRows; ++rr) s += lrow[rr];
     g.loss_part[(int64_t)jb.member * g.n_blk_cap + jb.blk] = s;
   }
 }
@@ -264,7 +330,7 @@ __global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
 __global__ void k_head_reduce(HeadReduceArgs g) {
   const int i = blockIdx.x;
   const HeadReduceJob jb = g.jobs[i];
-  const int n_blk = g.B_pad / kRowTile;
+  const int n_blk = g.B_pad / kHeadRows;
   if (!g.active[i]) {
     if (threadIdx.x == 0 && g.loss_out) g.loss_out[i] = __int_as_float(0x7fc00000);
     return;
@@ -288,16 +354,38 @@ __global__ void k_head_reduce(HeadReduceArgs g) {
 
 // ------------------------------------------------------------- bias grads
 // db_l[c] = sum over the B_pad batch rows of dZ_l[r, c] (padded rows are 0).
+// One block per 256 columns of one layer: lane l of warp q sums columns
+// c0 + 8 l .. + 7 over rows q, q + 8, ... (16-byte loads), then the 8 warp
+// partials are added in warp order.
 template <typename T>
-__global__ void k_bias_grad(const BiasJob* __restrict__ jobs, const T* __restrict__ dz,
-                            float* __restrict__ grads, int32_t B_pad) {
+__global__ void __launch_bounds__(256) k_bias_grad(const BiasJob* __restrict__ jobs, const T* __restrict__ dz,
+                                                   float* __restrict__ grads, int32_t B_pad) {
   const BiasJob jb = jobs[blockIdx.x];
-  const int c = jb.c0 + threadIdx.x;
-  if (c >= jb.w) return;
-  const T* z = dz + jb.dz_off + c;
-  float s = 0.f;
-  for (int r = 0; r < B_pad; ++r) s += Elem<T>::to_f(z[(int64_t)r * jb.w]);
-  grads[jb.b_off + c] = s;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int c = jb.c0 + 8 * lane;
+  __shared__ float part[8][256];
+  float s[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) s[k] = 0.f;
+  if (c < jb.w) {
+    const T* z = dz + jb.dz_off + c;
+    for (int r = warp; r < B_pad; r += 8) {
+      float h[8];
+      load8(z + (int64_t)r * jb.w, h);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) s[k] += h[k];
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < 8; ++k) part[warp][8 * lane + k] = s[k];
+  __syncthreads();
+  const int cc = jb.c0 + threadIdx.x;
+  if (cc < jb.w) {
+    float t = 0.f;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) t += part[q][threadIdx.x];
+    grads[jb.b_off + cc] = t;
+  }
 }
 
 // ------------------------------------------------------------------ AdamW
@@ -315,7 +403,38 @@ __global__ void __launch_bounds__(256) k_adamw(AdamArgs g) {
   const float wd = (s.is_bias && !g.wd_on_bias) ? 0.f : md.wd;
   const float b1 = g.beta1, b2 = g.beta2, eps = g.eps;
   const float ib1 = 1.f / bc.x, ib2 = 1.f / bc.y;
-  for (int e = threadIdx.x; e < ch.len; e += blockDim.x) {
+  // chunk offsets are multiples of 4 elements: float4 body, scalar tail
+  const int n4 = ch.len >> 2;
+  float4* P4 = reinterpret_cast<float4*>(g.params + ch.off);
+  const float4* G4 = reinterpret_cast<const float4*>(g.grads + ch.off);
+  float4* M4 = reinterpret_cast<float4*>(g.m + ch.off);
+  float4* V4 = reinterpret_cast<float4*>(g.v + ch.off);
+  for (int e = threadIdx.x; e < n4; e += blockDim.x) {
+    float4 p = P4[e], m = M4[e], v = V4[e];
+    const float4 gr = __ldcs(G4 + e);
+    float* pp = &p.x;
+    float* mm = &m.x;
+    float* vv = &v.x;
+    const float* gg = &gr.x;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      pp[k] = pp[k] - lr * wd * pp[k];
+      mm[k] = b1 * mm[k] + (1.f - b1) * gg[k];
+      vv[k] = b2 * vv[k] + (1.f - b2) * gg[k] * gg[k];
+      pp[k] = pp[k] - lr * (mm[k] * ib1) / (sqrtf(vv[k] * ib2) + eps);
+    }
+    P4[e] = p;
+    M4[e] = m;
+    V4[e] = v;
+    if (g.wq) {
+      __nv_bfloat162 lo = __floats2bfloat162_rn(p.x, p.y), hi = __floats2bfloat162_rn(p.z, p.w);
+      uint2 u;
+      u.x = *reinterpret_cast<uint32_t*>(&lo);
+      u.y = *reinterpret_cast<uint32_t*>(&hi);
+      *reinterpret_cast<uint2*>(g.wq + ch.off + 4 * e) = u;
+    }
+  }
+  for (int e = 4 * n4 + threadIdx.x; e < ch.len; e += blockDim.x) {
     const int64_t o = ch.off + e;
     float p = g.params[o], gr = g.grads[o], m = g.m[o], v = g.v[o];
     p = p - lr * wd * p;
@@ -377,7 +496,7 @@ __global__ void k_refresh_wq(const float* __restrict__ p, __nv_bfloat16* __restr
 template <typename T, int DO>
 __global__ void __launch_bounds__(256) k_predict_head(PredictHeadArgs<T> g) {
   const HeadJob jb = g.jobs[blockIdx.x];
-  const int r0 = jb.blk * kRowTile;
+  const int r0 = jb.blk * kHeadRows;
   if (r0 >= g.rows) return;
   const MemberDev md = g.mem[jb.member];
   const int w = md.w, d_out = g.d_out;
@@ -385,17 +504,24 @@ __global__ void __launch_bounds__(256) k_predict_head(PredictHeadArgs<T> g) {
   const float* Wh = g.params + jb.w_off;
   const float* bh = g.params + jb.b_off;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int rr = warp; rr < kRowTile; rr += 8) {
+  for (int rr = warp; rr < kHeadRows; rr += 8) {
     const int r = r0 + rr;
     if (r >= g.rows) break;
     float acc[DO];
 #pragma unroll
     for (int c = 0; c < DO; ++c) acc[c] = 0.f;
-    for (int j = lane; j < w; j += 32) {
-      float h = Elem<T>::to_f(H[(int64_t)r * w + j]);
+    for (int gi = lane; gi < (w >> 3); gi += 32) {
+      float h[8];
+      load8(H + (int64_t)r * w + 8 * gi, h);
 #pragma unroll
-      for (int c = 0; c < DO; ++c)
-        if (c < d_out) acc[c] = fmaf(h, Wh[(int64_t)c * w + j], acc[c]);
+      for (int c = 0; c < DO; ++c) {
+        if (c < d_out) {
+          float w8[8];
+          load8(Wh + (int64_t)c * w + 8 * gi, w8);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) acc[c] = fmaf(h[k], w8[k], acc[c]);
+        }
+      }
     }
 #pragma unroll
     for (int c = 0; c < DO; ++c)
@@ -460,7 +586,7 @@ void launch_head_reduce(cudaStream_t st, const HeadReduceArgs& g, int m) {
 
 template <typename T>
 void launch_bias_grad(cudaStream_t st, const BiasJob* jobs, int n_jobs, const T* dz, float* grads, int B_pad) {
-  if (n_jobs > 0) k_bias_grad<T><<<n_jobs, 128, 0, st>>>(jobs, dz, grads, B_pad);
+  if (n_jobs > 0) k_bias_grad<T><<<n_jobs, 256, 0, st>>>(jobs, dz, grads, B_pad);
 }
 
 void launch_adamw(cudaStream_t st, const AdamArgs& g, int n_chunks) {

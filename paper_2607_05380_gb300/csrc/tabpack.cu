@@ -168,7 +168,7 @@ tp_status build_layout(tabpack* h) {
   const int m = c.m;
   h->d_in_pad = (int)round_up(c.d_in, 8);
   h->B_cap = (int)round_up(c.max_batch, kRowTile);
-  h->n_blk_cap = h->B_cap / kRowTile;
+  h->n_blk_cap = h->B_cap / kHeadRows;
   h->W_off.resize(m);
   h->b_off.resize(m);
   h->act_off.resize(m);
@@ -309,7 +309,7 @@ tp_status build_schedule(tabpack* h) {
   std::vector<BiasJob> bj;
   for (int i : ids)
     for (int l = 0; l < h->depth[i]; ++l)
-      for (int c0 = 0; c0 < h->width[i]; c0 += 128)
+      for (int c0 = 0; c0 < h->width[i]; c0 += 256)
         bj.push_back(BiasJob{h->dz_off[i][l], h->b_off[i][l], h->width[i], c0});
   std::vector<Chunk> ch;
   for (int s = 0; s < (int)h->segs.size(); ++s) {

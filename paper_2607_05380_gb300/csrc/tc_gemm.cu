@@ -10,9 +10,10 @@
 //   warp 1     MMA issuer: one thread issues tcgen05.mma (M=128, K=16 per
 //              instruction) into one of two TMEM accumulators (2 x 256
 //              fp32 columns) and commits each stage back to the producer.
-//   warps 2-5  epilogue: tcgen05.ld of the accumulator (warp w reads TMEM
-//              lanes 32 (w % 4) .. +31, i.e. those output rows) and the
-//              fused epilogue of the product kind:
+//   warps 2-9  epilogue: tcgen05.ld of the accumulator (warp w reads TMEM
+//              lanes 32 (w % 4) .. +31, i.e. those output rows; the two
+//              warps of a lane quarter take alternate 32-column chunks) and
+//              the fused epilogue of the product kind:
 //                kFwd   z = acc + b; h = dropout(relu(z)) / (1 - p)   -> bf16
 //                kDgrad dz_prev = acc * [H_prev > 0] / (1 - p)          -> bf16
 //                kWgrad dW = acc                                        -> fp32
@@ -40,7 +41,7 @@ constexpr int kBoxBytes = 64 * 64 * 2;  // one 64 x 64 bf16 TMA box
 constexpr int kABytes = 2 * kBoxBytes;  // 128 rows
 constexpr int kBBytes = 4 * kBoxBytes;  // up to 256 rows / columns
 constexpr int kStageBytes = kABytes + kBBytes;
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;  // 2 role warps + 8 epilogue warps
 constexpr uint32_t kTmemCols = 512;
 constexpr int kAccCols = 256;
 constexpr uint64_t kWaitNs = 2000000000ull;
@@ -191,7 +192,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tl->tfull[b], 1);
-      mbar_init(&tl->tempty[b], 128);
+      mbar_init(&tl->tempty[b], 256);
     }
     mbar_init(&tl->done, 1);
     tl->abort = 0;
@@ -306,7 +307,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    const int q = warp & 3;
+    const int q = warp & 3;             // TMEM lane quarter this warp may access
+    const int half = (warp - 2) >> 2;   // 0 for warps 2-5, 1 for warps 6-9
     const int row = 32 * q + lane;
     uint32_t acc = 0, acc_phase = 0;
     for (int t = blockIdx.x; t < g.n_tiles; t += gridDim.x) {
@@ -319,15 +321,22 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       const int r = tile.m0 + row;
       const bool row_ok = r < m_lim;
       const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + acc * kAccCols;
-      for (int c = 0; c < tile.n_len; c += 32) {
-        uint32_t v[32];
-        tmem_ld32(taddr + c, v);
-        if (!row_ok) continue;
+      // the two warps of a lane quarter take alternate 32-column chunks
+      for (int c = 32 * half; c < tile.n_len; c += 64) {
         const int col0 = tile.n0 + c;
         const int ncols = min(32, tile.n_real - col0);  // a multiple of 8 (widths are multiples of 16)
-        if (ncols <= 0) continue;
-        if (tile.kind == kFwd) {
-          uint32_t keep = 0xFFFFFFFFu;
+        const bool live = row_ok && ncols > 0;
+        // forward: bias and dropout bits do not depend on the accumulator,
+        // so they are fetched / generated before the TMEM load
+        float bias[32];
+        uint32_t keep = 0xFFFFFFFFu;
+        if (tile.kind == kFwd && live) {
+          const float4* b4 = reinterpret_cast<const float4*>(g.params + tile.aux_off + col0);
+#pragma unroll
+          for (int s = 0; s < 8; ++s) {
+            const float4 t4 = 4 * s < ncols ? __ldg(b4 + s) : make_float4(0.f, 0.f, 0.f, 0.f);
+            bias[4 * s] = t4.x; bias[4 * s + 1] = t4.y; bias[4 * s + 2] = t4.z; bias[4 * s + 3] = t4.w;
+          }
           if (g.train && md.drop_T) {
             keep = 0;
 #pragma unroll
@@ -336,8 +345,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
                                  (uint32_t)((col0 >> 2) + g4), md.drop_T)
                       << (4 * g4);
           }
+        }
+        uint32_t v[32];
+        tmem_ld32(taddr + c, v);
+        if (!live) continue;
+        if (tile.kind == kFwd) {
           const float sc = g.train ? md.scale : 1.f;
-          const float* bias = g.params + tile.aux_off + col0;
           __nv_bfloat16* out = g.act + tile.c_off + (int64_t)r * tile.ldc + col0;
 #pragma unroll
           for (int s = 0; s < 4; ++s) {
@@ -349,7 +362,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
 #pragma unroll
               for (int u = 0; u < 2; ++u) {
                 const int j = 8 * s + 2 * e + u;
-                const float z = __uint_as_float(v[j]) + __ldg(bias + j);
+                const float z = __uint_as_float(v[j]) + bias[j];
                 const float a = z > 0.f ? z : 0.f;
                 h2[u] = ((keep >> j) & 1u) ? a * sc : 0.f;
               }

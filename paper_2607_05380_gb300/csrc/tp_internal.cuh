@@ -26,6 +26,7 @@ namespace tp {
 constexpr int kMaxDepth = 14;   // hidden blocks per member (4-bit layer field of the Philox counter)
 constexpr int kMaxDout = 32;
 constexpr int kRowTile = 128;   // batch rows per tile; B_pad is a multiple of this
+constexpr int kHeadRows = 32;   // batch rows per head-kernel block
 constexpr int kSegAlign = 32;   // elements
 
 enum GemmKind : int32_t { kFwd = 0, kDgrad = 1, kWgrad = 2 };
