@@ -261,20 +261,25 @@ def main():
     fam = {k: v for k, v in prof.items() if v[1] > 0}
     dominant = max(fam, key=lambda k: fam[k][0])
     shares = {k: round(v[0] / sum(x[0] for x in fam.values()), 4) for k, v in fam.items()}
-    if dominant in ("fwd", "bwd"):
-        gemm_ms = (prof["fwd"][0] + prof["bwd"][0]) / n_prof
-        n_l = (prof["fwd"][1] + prof["bwd"][1]) / n_prof
-        ach = flops / (gemm_ms / 1000.0) / 1e12
-        roof = {"kernel": "grouped GEMM (fwd+dgrad+wgrad launches of one step)", "bound": "tensor",
-                "achieved": ach, "peak": pk["bf16_sus"], "unit": "TFLOP/s", "frac": ach / pk["bf16_sus"],
-                "traffic": None, "per_launch_ms": gemm_ms / max(1, n_l), "peak_source": pk["source"] + " sustained"}
-    else:
-        per_launch_ms = prof[dominant][0] / max(1, prof[dominant][1])
-        byts = 30.0 * n_params if dominant == "adamw" else None
-        ach = byts / (per_launch_ms / 1000.0) / 1e9 if byts else None
-        roof = {"kernel": dominant, "bound": "hbm", "achieved": ach, "peak": pk["hbm"], "unit": "GB/s",
-                "frac": (ach / pk["hbm"]) if ach else None, "traffic": None, "per_launch_ms": per_launch_ms,
-                "peak_source": pk["source"]}
+    fwd_ms = prof["fwd"][0] / n_prof                              # per step
+    bwd_ms = prof["bwd"][0] / n_prof
+    adam_ms = prof["adamw"][0] / n_prof
+    gemm_ms = fwd_ms + bwd_ms
+    gemm = {"kernel": "k_tc_gemm (grouped fwd + dgrad + wgrad launches of one step)", "bound": "tensor",
+            "achieved": flops / (gemm_ms / 1e3) / 1e12, "peak": pk["bf16_sus"], "unit": "TFLOP/s",
+            "traffic": None, "ms_per_step": gemm_ms, "peak_source": pk["source"] + " sustained bf16"}
+    gemm["frac"] = gemm["achieved"] / gemm["peak"]
+    if adam_ms > 0:   # fp32 mode: stand-alone AdamW, 30 B per parameter
+        mem = {"kernel": "k_adamw", "bound": "hbm", "achieved": 30.0 * n_params / (adam_ms / 1e3) / 1e9,
+               "ms_per_step": adam_ms, "bytes_per_step": 30.0 * n_params}
+    else:             # bf16 mode: AdamW fused into the wgrad epilogue, 26 B per parameter
+        mem = {"kernel": "k_tc_gemm backward launches (fused AdamW: read p, m, v; write p, m, v, bf16 p)",
+               "bound": "hbm", "achieved": 26.0 * n_params / (bwd_ms / 1e3) / 1e9, "ms_per_step": bwd_ms,
+               "bytes_per_step": 26.0 * n_params}
+    mem.update({"peak": pk["hbm"], "unit": "GB/s", "traffic": None, "peak_source": pk["source"] + " HBM copy"})
+    mem["frac"] = mem["achieved"] / mem["peak"]
+    roof = dict(gemm if gemm_ms >= adam_ms else mem)
+    roof["other"] = mem if gemm_ms >= adam_ms else gemm
     roof["shares"] = shares
 
     # end to end through the public API with host buffers: per step the batch

@@ -68,6 +68,10 @@ typedef struct {
   uint64_t seed;      /* Philox key of parameter init and dropout masks                 */
   float beta1, beta2, eps;  /* AdamW constants shared by all members (0.9, 0.999, 1e-8) */
   int32_t wd_on_bias; /* 1: weight decay also applies to biases                         */
+  int32_t fuse_optimizer; /* bf16 mode only.  0: the weight-gradient products store fp32
+                         gradients and one AdamW pass updates all parameters (faster on
+                         most shapes); 1: AdamW runs inside the weight-gradient product's
+                         epilogue, so gradients never reach HBM.  Results are the same. */
 } tp_config;
 
 /* Create a pack (Sec. 3.3 model pack + Sec. 3.4 optimizer pack).

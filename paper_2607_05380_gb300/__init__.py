@@ -43,7 +43,7 @@ class Config(ctypes.Structure):
     _fields_ = [("m", ctypes.c_int32), ("d_in", ctypes.c_int32), ("d_out", ctypes.c_int32),
                 ("max_batch", ctypes.c_int32), ("task", ctypes.c_int32), ("precision", ctypes.c_int32),
                 ("seed", ctypes.c_uint64), ("beta1", ctypes.c_float), ("beta2", ctypes.c_float),
-                ("eps", ctypes.c_float), ("wd_on_bias", ctypes.c_int32)]
+                ("eps", ctypes.c_float), ("wd_on_bias", ctypes.c_int32), ("fuse_optimizer", ctypes.c_int32)]
 
 
 _lib = None
@@ -123,7 +123,8 @@ class Pack:
     """A pack of m base MLPs with per-member hyperparameters on one GPU."""
 
     def __init__(self, d_in, d_out, task, depth, width, dropout, lr, wd, max_batch, seed=2,
-                 precision="bf16", beta1=0.9, beta2=0.999, eps=1e-8, wd_on_bias=True, stream=None):
+                 precision="bf16", beta1=0.9, beta2=0.999, eps=1e-8, wd_on_bias=True, stream=None,
+                 fuse_optimizer=False):
         import torch
         L = load_library()
         self.torch = torch
@@ -134,7 +135,7 @@ class Pack:
         self.task = TASKS[task] if isinstance(task, str) else int(task)
         self.precision = PRECISIONS[precision] if isinstance(precision, str) else int(precision)
         cfg = Config(self.m, self.d_in, self.d_out, int(max_batch), self.task, self.precision, int(seed),
-                     beta1, beta2, eps, int(bool(wd_on_bias)))
+                     beta1, beta2, eps, int(bool(wd_on_bias)), int(bool(fuse_optimizer)))
         drop = np.ascontiguousarray(dropout, dtype=np.float32)
         lr_ = np.ascontiguousarray(lr, dtype=np.float32)
         wd_ = np.ascontiguousarray(wd, dtype=np.float32)

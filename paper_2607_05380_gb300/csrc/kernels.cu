@@ -1,17 +1,18 @@
 // kernels.cu -- element-wise, reduction and CUDA-core matrix kernels of the
-// packed training step (gather, CUDA-core grouped GEMM, head + loss, bias
-// gradients, AdamW, init, predict head, mask dump).
+// packed training step (gather, CUDA-core grouped GEMM, head + loss + head
+// AdamW, AdamW, init, predict head, mask dump).
 #include "kernels.cuh"
 
 namespace tp {
 
 // ------------------------------------------------------------------ gather
-// xb[b, k] = X[idx[b], k] for b < B, k < d_in; zeros elsewhere in [B_pad, d_in_pad].
+// xb[b, k] = X[idx[b], k] for b < B, k < d_in; zero for the rest of the first
+// d_in_pad columns of rows < B_pad (column d_in_pad holds the constant 1).
 // Block 0 also advances the step count of every active member and stores the
 // AdamW bias corrections 1 - beta^t of the new step (when `advance`).
 template <typename T>
 __global__ void k_gather(const float* __restrict__ X, const int32_t* __restrict__ idx, int32_t B,
-                         int32_t B_pad, int32_t d_in, int32_t d_in_pad, T* __restrict__ xb,
+                         int32_t B_pad, int32_t d_in, int32_t d_in_pad, int32_t ldx, T* __restrict__ xb,
                          int32_t advance, int32_t* __restrict__ t_dev, float2* __restrict__ bias_corr,
                          const int32_t* __restrict__ active_ids, int32_t n_active, float beta1,
                          float beta2) {
@@ -33,8 +34,16 @@ __global__ void k_gather(const float* __restrict__ X, const int32_t* __restrict_
       int64_t row = idx ? (int64_t)idx[b] : (int64_t)b;
       v = X[row * d_in + k];
     }
-    xb[e] = Elem<T>::from_f(v);
+    xb[(int64_t)b * ldx + k] = Elem<T>::from_f(v);
   }
+}
+
+// Column `col` of the first `rows` rows := 1 (xb and every act matrix, once).
+template <typename T>
+__global__ void k_fill_ones(const OnesJob* __restrict__ jobs, T* __restrict__ xb, T* __restrict__ act) {
+  const OnesJob jb = jobs[blockIdx.x];
+  T* base = (jb.arena == 0 ? xb : act) + jb.off;
+  for (int r = threadIdx.x; r < jb.rows; r += blockDim.x) base[(int64_t)r * jb.ld + jb.col] = Elem<T>::from_f(1.f);
 }
 
 // ------------------------------------------------------- CUDA-core GEMM
@@ -101,13 +110,13 @@ __global__ void __launch_bounds__(256) k_gemm_simt(GemmArgs<T> g, int32_t tile_b
     __syncthreads();
   }
   const int c0 = t.n0 + tx * 4;
-  if (c0 >= N) return;  // N is a multiple of 4, so c0 < N covers c0 .. c0 + 3
+  if (c0 >= N) return;
   const MemberDev md = g.mem[P.member];
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     const int r = t.m0 + ty + 16 * i;
     if (r >= M) continue;
-    if (P.kind == kFwd) {
+    if (P.kind == kFwd) {  // N = w, a multiple of 16
       uint32_t keep = g.train ? keep_bits4(g.seed, (uint32_t)P.member, (uint32_t)P.layer, g.step,
                                            (uint32_t)r, (uint32_t)(c0 >> 2), md.drop_T)
                               : 0xFu;
@@ -120,34 +129,34 @@ __global__ void __launch_bounds__(256) k_gemm_simt(GemmArgs<T> g, int32_t tile_b
         float h = ((keep >> j) & 1u) ? a * sc : 0.f;
         C[(int64_t)r * P.ldc + c0 + j] = Elem<T>::from_f(h);
       }
-    } else if (P.kind == kDgrad) {
+    } else if (P.kind == kDgrad) {  // N = w
       const T* Hm = g.act + P.aux_off;
       T* C = g.dz + P.c_off;
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
-        int64_t o = (int64_t)r * P.ldc + c0 + j;
-        float h = Elem<T>::to_f(Hm[o]);
-        C[o] = Elem<T>::from_f(h > 0.f ? acc[i][j] * md.scale : 0.f);
+        float h = Elem<T>::to_f(Hm[(int64_t)r * P.ld_aux + c0 + j]);
+        C[(int64_t)r * P.ldc + c0 + j] = Elem<T>::from_f(h > 0.f ? acc[i][j] * md.scale : 0.f);
       }
-    } else {
+    } else {  // N = in_pad + 1: the last column is the bias gradient
       float* C = g.grads + P.c_off;
 #pragma unroll
-      for (int j = 0; j < 4; ++j) C[(int64_t)r * P.ldc + c0 + j] = acc[i][j];
+      for (int j = 0; j < 4; ++j) {
+        const int c = c0 + j;
+        if (c < N - 1) C[(int64_t)r * P.ldc + c] = acc[i][j];
+        else if (c == N - 1) g.grads[P.aux_off + r] = acc[i][j];
+      }
     }
   }
 }
 
-// ------------------------------------------------------------- head + loss
-// One block per (member, 128-row block).  Warps compute one row's logits at
-// a time, then the per-row loss and d(mean loss)/d(logits); the block then
-// forms dZ of the last hidden layer and its partial head-weight gradient.
+// ---------------------------------------------------------- vector helpers
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
 }
 
-// 8 consecutive activations of a row as floats (16-byte bf16 / 2 x 16-byte fp32 loads).
+// 8 consecutive values as floats (16-byte bf16 / 2 x 16-byte fp32 loads).
 __device__ __forceinline__ void load8(const __nv_bfloat16* p, float (&h)[8]) {
   const uint4 u = *reinterpret_cast<const uint4*>(p);
   const __nv_bfloat16* b = reinterpret_cast<const __nv_bfloat16*>(&u);
@@ -170,17 +179,59 @@ __device__ __forceinline__ void store8(float* p, const float (&v)[8]) {
   *reinterpret_cast<float4*>(p + 4) = make_float4(v[4], v[5], v[6], v[7]);
 }
 
-// Head kernel.  Per row (one warp, lanes over 8-column groups): logits,
-// per-row loss and dlogits, then dZ of the last hidden layer for the same
-// row while it is in L1.  Then per column group (threads) the block's
-// partial head-weight gradient sum over its 128 rows, in row order.
+// Per-row loss and d(mean loss)/d(logits) of one row (fp32).
+template <int DO>
+__device__ __forceinline__ float row_loss(int task, int d_out, const float (&z)[DO], const void* y, int64_t row,
+                                          float invB, float (&dl)[DO]) {
+  float loss;
+  if (task == 1) {  // multiclass: softmax cross-entropy
+    const int yv = ((const int32_t*)y)[row];
+    float mx = z[0];
+#pragma unroll
+    for (int c = 1; c < DO; ++c) if (c < d_out) mx = fmaxf(mx, z[c]);
+    float s = 0.f;
+#pragma unroll
+    for (int c = 0; c < DO; ++c) if (c < d_out) s += expf(z[c] - mx);
+    const float lse = mx + logf(s);
+    float zy = 0.f;
+#pragma unroll
+    for (int c = 0; c < DO; ++c) {
+      if (c == yv) zy = z[c];
+      dl[c] = c < d_out ? (expf(z[c] - lse) - (c == yv ? 1.f : 0.f)) * invB : 0.f;
+    }
+    loss = lse - zy;
+  } else if (task == 0) {  // binary: logistic loss on one logit
+    const float yv = (float)((const int32_t*)y)[row];
+    const float x = z[0];
+    loss = fmaxf(x, 0.f) - x * yv + log1pf(expf(-fabsf(x)));
+#pragma unroll
+    for (int c = 0; c < DO; ++c) dl[c] = 0.f;
+    dl[0] = (1.f / (1.f + expf(-x)) - yv) * invB;
+  } else {  // regression: squared error
+    const float d = z[0] - ((const float*)y)[row];
+    loss = d * d;
+#pragma unroll
+    for (int c = 0; c < DO; ++c) dl[c] = 0.f;
+    dl[0] = 2.f * d * invB;
+  }
+  return loss;
+}
+
+// ------------------------------------------------------------- head + loss
+// One block per (member, 32-row block); each warp owns 4 rows and walks them
+// R at a time (lanes over 8-column groups, 16-byte loads), so every head-weight
+// load serves R rows.  Per row: logits, loss and dlogits, then dZ of the last
+// hidden layer = (dlogits W_h) * [H > 0] / (1 - p).  Then per column group the
+// block's partial head-weight gradient over its 32 rows, in row order.
 template <typename T, int DO>
 __global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
+  constexpr int R = DO <= 16 ? 4 : 1;
+  constexpr int RW = kHeadRows / 8;  // rows per warp
   const HeadJob jb = g.jobs[blockIdx.x];
   const int r0 = jb.blk * kHeadRows;
   if (r0 >= g.B_pad) return;
   const MemberDev md = g.mem[jb.member];
-  const int w = md.w, d_out = g.d_out;
+  const int w = md.w, d_out = g.d_out, ldh = jb.h_ld;
   const int ng = w >> 3;  // 8-column groups (widths are multiples of 16)
   const T* H = g.act + jb.h_off;
   const float* Wh = g.params + jb.w_off;
@@ -190,92 +241,78 @@ __global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float invB = 1.f / (float)g.B;
   T* dZ = g.dz + jb.dz_off;
-  for (int rr = warp; rr < kHeadRows; rr += 8) {
-    const int r = r0 + rr;
-    const T* Hr = H + (int64_t)r * w;
-    float acc[DO];
+  for (int q0 = 0; q0 < RW; q0 += R) {
+    const int rl0 = warp * RW + q0;  // first local row of this pass
+    float acc[R][DO];
 #pragma unroll
-    for (int c = 0; c < DO; ++c) acc[c] = 0.f;
+    for (int q = 0; q < R; ++q)
+#pragma unroll
+      for (int c = 0; c < DO; ++c) acc[q][c] = 0.f;
     for (int gi = lane; gi < ng; gi += 32) {
-      float h[8];
-      load8(Hr + 8 * gi, h);
+      float h[R][8];
+#pragma unroll
+      for (int q = 0; q < R; ++q) load8(H + (int64_t)(r0 + rl0 + q) * ldh + 8 * gi, h[q]);
 #pragma unroll
       for (int c = 0; c < DO; ++c) {
         if (c < d_out) {
           float w8[8];
           load8(Wh + (int64_t)c * w + 8 * gi, w8);
 #pragma unroll
-          for (int k = 0; k < 8; ++k) acc[c] = fmaf(h[k], w8[k], acc[c]);
+          for (int q = 0; q < R; ++q)
+#pragma unroll
+            for (int k = 0; k < 8; ++k) acc[q][c] = fmaf(h[q][k], w8[k], acc[q][c]);
         }
       }
     }
+    float dl[R][DO];
 #pragma unroll
-    for (int c = 0; c < DO; ++c)
-      if (c < d_out) acc[c] = warp_sum(acc[c]) + bh[c];
-    float loss = 0.f;
-    float dl[DO];
+    for (int q = 0; q < R; ++q) {
 #pragma unroll
-    for (int c = 0; c < DO; ++c) dl[c] = 0.f;
-    if (r < g.B) {
-      const int64_t row = g.idx ? (int64_t)g.idx[r] : (int64_t)r;
-      if (g.task == 1) {  // multiclass: softmax cross-entropy
-        const int yv = ((const int32_t*)g.y)[row];
-        float mx = acc[0];
+      for (int c = 0; c < DO; ++c)
+        if (c < d_out) acc[q][c] = warp_sum(acc[q][c]) + bh[c];
+      const int r = r0 + rl0 + q;
+      float loss = 0.f;
 #pragma unroll
-        for (int c = 1; c < DO; ++c) if (c < d_out) mx = fmaxf(mx, acc[c]);
-        float s = 0.f;
-#pragma unroll
-        for (int c = 0; c < DO; ++c) if (c < d_out) s += expf(acc[c] - mx);
-        const float lse = mx + logf(s);
-        float zy = 0.f;
-#pragma unroll
-        for (int c = 0; c < DO; ++c)
-          if (c < d_out) {
-            if (c == yv) zy = acc[c];
-            dl[c] = (expf(acc[c] - lse) - (c == yv ? 1.f : 0.f)) * invB;
-          }
-        loss = lse - zy;
-      } else if (g.task == 0) {  // binary: logistic loss on one logit
-        const float yv = (float)((const int32_t*)g.y)[row];
-        const float x = acc[0];
-        loss = fmaxf(x, 0.f) - x * yv + log1pf(expf(-fabsf(x)));
-        dl[0] = (1.f / (1.f + expf(-x)) - yv) * invB;
-      } else {  // regression: squared error
-        const float d = acc[0] - ((const float*)g.y)[row];
-        loss = d * d;
-        dl[0] = 2.f * d * invB;
-      }
-      if (lane < d_out) {
+      for (int c = 0; c < DO; ++c) dl[q][c] = 0.f;
+      if (r < g.B) {
+        const int64_t row = g.idx ? (int64_t)g.idx[r] : (int64_t)r;
+        loss = row_loss<DO>(g.task, d_out, acc[q], g.y, row, invB, dl[q]);
         float z = 0.f;
 #pragma unroll
-        for (int c = 0; c < DO; ++c) if (c == lane) z = acc[c];
-        g.logits[((int64_t)jb.member * g.B_cap + r) * d_out + lane] = z;
+        for (int c = 0; c < DO; ++c) if (c == lane) z = acc[q][c];
+        if (lane < d_out) g.logits[((int64_t)jb.member * g.B_cap + r) * d_out + lane] = z;
+      }
+      if (lane == 0) {
+#pragma unroll
+        for (int c = 0; c < DO; ++c) dlog[rl0 + q][c] = dl[q][c];
+        lrow[rl0 + q] = loss;
       }
     }
-    if (lane == 0) {
-#pragma unroll
-      for (int c = 0; c < DO; ++c) dlog[rr][c] = dl[c];
-      lrow[rr] = loss;
-    }
-    // dZ of the last hidden layer for this row: (dlogits W_h) * [H > 0] / (1 - p)
-    T* dZr = dZ + (int64_t)r * w;
     for (int gi = lane; gi < ng; gi += 32) {
-      float h[8], s[8];
-      load8(Hr + 8 * gi, h);
+      float h[R][8], s[R][8];
 #pragma unroll
-      for (int k = 0; k < 8; ++k) s[k] = 0.f;
+      for (int q = 0; q < R; ++q) {
+        load8(H + (int64_t)(r0 + rl0 + q) * ldh + 8 * gi, h[q]);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) s[q][k] = 0.f;
+      }
 #pragma unroll
       for (int c = 0; c < DO; ++c) {
         if (c < d_out) {
           float w8[8];
           load8(Wh + (int64_t)c * w + 8 * gi, w8);
 #pragma unroll
-          for (int k = 0; k < 8; ++k) s[k] = fmaf(dl[c], w8[k], s[k]);
+          for (int q = 0; q < R; ++q)
+#pragma unroll
+            for (int k = 0; k < 8; ++k) s[q][k] = fmaf(dl[q][c], w8[k], s[q][k]);
         }
       }
 #pragma unroll
-      for (int k = 0; k < 8; ++k) s[k] = h[k] > 0.f ? s[k] * md.scale : 0.f;
-      store8(dZr + 8 * gi, s);
+      for (int q = 0; q < R; ++q) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) s[q][k] = h[q][k] > 0.f ? s[q][k] * md.scale : 0.f;
+        store8(dZ + (int64_t)(r0 + rl0 + q) * w + 8 * gi, s[q]);
+      }
     }
   }
   __syncthreads();
@@ -291,7 +328,7 @@ __global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
       for (int k = 0; k < G; ++k) a[c][k] = 0.f;
 #pragma unroll 4
     for (int rr = 0; rr < kHeadRows; ++rr) {
-      const T* hp = H + (int64_t)(r0 + rr) * w + G * gi;
+      const T* hp = H + (int64_t)(r0 + rr) * ldh + G * gi;
       float h[G];
       if constexpr (G == 8) {
         load8(hp, h);
@@ -326,7 +363,9 @@ __global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
 }
 
 // Sum the per-block head partials (fixed order) into the head gradients and
-// the per-member mean loss.  One block per member; inactive members get NaN.
+// the per-member mean loss; in update mode apply the member's AdamW to the
+// head parameters directly (the gradients are not stored).  One block per
+// member; inactive members report NaN.
 __global__ void k_head_reduce(HeadReduceArgs g) {
   const int i = blockIdx.x;
   const HeadReduceJob jb = g.jobs[i];
@@ -337,11 +376,31 @@ __global__ void k_head_reduce(HeadReduceArgs g) {
   }
   const int w = jb.w, d_out = g.d_out;
   const int64_t stride = g.part_stride[i];
+  float lr = 0.f, wdw = 0.f, wdb = 0.f, ib1 = 1.f, ib2 = 1.f;
+  if (g.update) {
+    const MemberDev md = g.adam.mem[i];
+    const float2 bc = g.adam.bias_corr[i];
+    lr = md.lr;
+    wdw = md.wd;
+    wdb = g.adam.wd_on_bias ? md.wd : 0.f;
+    ib1 = 1.f / bc.x;
+    ib2 = 1.f / bc.y;
+  }
   for (int e = threadIdx.x; e < d_out * w + d_out; e += blockDim.x) {
     float s = 0.f;
     for (int b = 0; b < n_blk; ++b) s += g.head_part[jb.part_off + b * stride + e];
-    if (e < d_out * w) g.grads[jb.gw_off + e] = s;
-    else g.grads[jb.gb_off + (e - d_out * w)] = s;
+    const bool is_b = e >= d_out * w;
+    const int64_t o = is_b ? jb.gb_off + (e - d_out * w) : jb.gw_off + e;
+    if (g.update) {
+      float p = g.adam.params[o], m = g.adam.m[o], v = g.adam.v[o];
+      adamw_elem(p, m, v, s, lr, is_b ? wdb : wdw, g.adam.beta1, g.adam.beta2, g.adam.eps, ib1, ib2);
+      g.adam.params[o] = p;
+      g.adam.m[o] = m;
+      g.adam.v[o] = v;
+      if (g.adam.wq_out) g.adam.wq_out[o] = __float2bfloat16_rn(p);
+    } else {
+      g.grads[o] = s;
+    }
   }
   if (threadIdx.x == 0) {
     float s = 0.f;
@@ -352,48 +411,9 @@ __global__ void k_head_reduce(HeadReduceArgs g) {
   }
 }
 
-// ------------------------------------------------------------- bias grads
-// db_l[c] = sum over the B_pad batch rows of dZ_l[r, c] (padded rows are 0).
-// One block per 256 columns of one layer: lane l of warp q sums columns
-// c0 + 8 l .. + 7 over rows q, q + 8, ... (16-byte loads), then the 8 warp
-// partials are added in warp order.
-template <typename T>
-__global__ void __launch_bounds__(256) k_bias_grad(const BiasJob* __restrict__ jobs, const T* __restrict__ dz,
-                                                   float* __restrict__ grads, int32_t B_pad) {
-  const BiasJob jb = jobs[blockIdx.x];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int c = jb.c0 + 8 * lane;
-  __shared__ float part[8][256];
-  float s[8];
-#pragma unroll
-  for (int k = 0; k < 8; ++k) s[k] = 0.f;
-  if (c < jb.w) {
-    const T* z = dz + jb.dz_off + c;
-    for (int r = warp; r < B_pad; r += 8) {
-      float h[8];
-      load8(z + (int64_t)r * jb.w, h);
-#pragma unroll
-      for (int k = 0; k < 8; ++k) s[k] += h[k];
-    }
-  }
-#pragma unroll
-  for (int k = 0; k < 8; ++k) part[warp][8 * lane + k] = s[k];
-  __syncthreads();
-  const int cc = jb.c0 + threadIdx.x;
-  if (cc < jb.w) {
-    float t = 0.f;
-#pragma unroll
-    for (int q = 0; q < 8; ++q) t += part[q][threadIdx.x];
-    grads[jb.b_off + cc] = t;
-  }
-}
-
 // ------------------------------------------------------------------ AdamW
-// Per element of the chunk, with the member's lr and wd and its step's bias
-// corrections (bc1, bc2) = (1 - beta1^t, 1 - beta2^t):
-//   p <- p - lr wd p;  m <- b1 m + (1 - b1) g;  v <- b2 v + (1 - b2) g^2;
-//   p <- p - lr (m / bc1) / (sqrt(v / bc2) + eps)
-// and the bf16 copy of p (bf16 mode).
+// Stand-alone AdamW over chunks of the arena (fp32 mode), with the member's
+// lr and wd and its step's bias corrections; float4 body, scalar tail.
 __global__ void __launch_bounds__(256) k_adamw(AdamArgs g) {
   const Chunk ch = g.chunks[blockIdx.x];
   const Segment s = g.segs[ch.seg];
@@ -403,8 +423,7 @@ __global__ void __launch_bounds__(256) k_adamw(AdamArgs g) {
   const float wd = (s.is_bias && !g.wd_on_bias) ? 0.f : md.wd;
   const float b1 = g.beta1, b2 = g.beta2, eps = g.eps;
   const float ib1 = 1.f / bc.x, ib2 = 1.f / bc.y;
-  // chunk offsets are multiples of 4 elements: float4 body, scalar tail
-  const int n4 = ch.len >> 2;
+  const int n4 = ch.len >> 2;  // chunk offsets are multiples of 4 elements
   float4* P4 = reinterpret_cast<float4*>(g.params + ch.off);
   const float4* G4 = reinterpret_cast<const float4*>(g.grads + ch.off);
   float4* M4 = reinterpret_cast<float4*>(g.m + ch.off);
@@ -412,17 +431,10 @@ __global__ void __launch_bounds__(256) k_adamw(AdamArgs g) {
   for (int e = threadIdx.x; e < n4; e += blockDim.x) {
     float4 p = P4[e], m = M4[e], v = V4[e];
     const float4 gr = __ldcs(G4 + e);
-    float* pp = &p.x;
-    float* mm = &m.x;
-    float* vv = &v.x;
-    const float* gg = &gr.x;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      pp[k] = pp[k] - lr * wd * pp[k];
-      mm[k] = b1 * mm[k] + (1.f - b1) * gg[k];
-      vv[k] = b2 * vv[k] + (1.f - b2) * gg[k] * gg[k];
-      pp[k] = pp[k] - lr * (mm[k] * ib1) / (sqrtf(vv[k] * ib2) + eps);
-    }
+    adamw_elem(p.x, m.x, v.x, gr.x, lr, wd, b1, b2, eps, ib1, ib2);
+    adamw_elem(p.y, m.y, v.y, gr.y, lr, wd, b1, b2, eps, ib1, ib2);
+    adamw_elem(p.z, m.z, v.z, gr.z, lr, wd, b1, b2, eps, ib1, ib2);
+    adamw_elem(p.w, m.w, v.w, gr.w, lr, wd, b1, b2, eps, ib1, ib2);
     P4[e] = p;
     M4[e] = m;
     V4[e] = v;
@@ -436,11 +448,8 @@ __global__ void __launch_bounds__(256) k_adamw(AdamArgs g) {
   }
   for (int e = 4 * n4 + threadIdx.x; e < ch.len; e += blockDim.x) {
     const int64_t o = ch.off + e;
-    float p = g.params[o], gr = g.grads[o], m = g.m[o], v = g.v[o];
-    p = p - lr * wd * p;
-    m = b1 * m + (1.f - b1) * gr;
-    v = b2 * v + (1.f - b2) * gr * gr;
-    p = p - lr * (m * ib1) / (sqrtf(v * ib2) + eps);
+    float p = g.params[o], m = g.m[o], v = g.v[o];
+    adamw_elem(p, m, v, g.grads[o], lr, wd, b1, b2, eps, ib1, ib2);
     g.params[o] = p;
     g.m[o] = m;
     g.v[o] = v;
@@ -449,7 +458,7 @@ __global__ void __launch_bounds__(256) k_adamw(AdamArgs g) {
 }
 
 // ------------------------------------------------------------------- init
-// Element of the padded arena -> the oracle's element index within the layer
+// Element of the padded arena -> the element index within the layer
 // (weights row-major unpadded, then biases) -> Philox word -> U(-b, b), fp32.
 __global__ void k_init(InitArgs g) {
   const Chunk ch = g.chunks[blockIdx.x];
@@ -480,14 +489,21 @@ __global__ void k_init(InitArgs g) {
     g.grads[o] = 0.f;
     g.m[o] = 0.f;
     g.v[o] = 0.f;
-    if (g.wq) g.wq[o] = __float2bfloat16_rn(val);
+    if (g.wq0) {
+      g.wq0[o] = __float2bfloat16_rn(val);
+      g.wq1[o] = __float2bfloat16_rn(val);
+    }
   }
 }
 
-// bf16 copy of the whole arena (after pack_set_params).
-__global__ void k_refresh_wq(const float* __restrict__ p, __nv_bfloat16* __restrict__ wq, int64_t n) {
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x)
-    wq[e] = __float2bfloat16_rn(p[e]);
+// bf16 copies of the whole arena (after pack_set_params / pack_set_active).
+__global__ void k_refresh_wq(const float* __restrict__ p, __nv_bfloat16* __restrict__ wq0,
+                             __nv_bfloat16* __restrict__ wq1, int64_t n) {
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
+    const __nv_bfloat16 b = __float2bfloat16_rn(p[e]);
+    wq0[e] = b;
+    wq1[e] = b;
+  }
 }
 
 // ----------------------------------------------------------- predict head
@@ -499,7 +515,7 @@ __global__ void __launch_bounds__(256) k_predict_head(PredictHeadArgs<T> g) {
   const int r0 = jb.blk * kHeadRows;
   if (r0 >= g.rows) return;
   const MemberDev md = g.mem[jb.member];
-  const int w = md.w, d_out = g.d_out;
+  const int w = md.w, d_out = g.d_out, ldh = jb.h_ld;
   const T* H = g.act + jb.h_off;
   const float* Wh = g.params + jb.w_off;
   const float* bh = g.params + jb.b_off;
@@ -512,7 +528,7 @@ __global__ void __launch_bounds__(256) k_predict_head(PredictHeadArgs<T> g) {
     for (int c = 0; c < DO; ++c) acc[c] = 0.f;
     for (int gi = lane; gi < (w >> 3); gi += 32) {
       float h[8];
-      load8(H + (int64_t)r * w + 8 * gi, h);
+      load8(H + (int64_t)r * ldh + 8 * gi, h);
 #pragma unroll
       for (int c = 0; c < DO; ++c) {
         if (c < d_out) {
@@ -559,13 +575,18 @@ __global__ void k_debug_masks(uint8_t* __restrict__ out, int32_t B, int32_t w, u
 // ------------------------------------------------------------- launchers
 template <typename T>
 void launch_gather(cudaStream_t st, const float* X, const int32_t* idx, int B, int B_pad, int d_in,
-                   int d_in_pad, T* xb, int advance, int32_t* t_dev, float2* bias_corr,
+                   int d_in_pad, int ldx, T* xb, int advance, int32_t* t_dev, float2* bias_corr,
                    const int32_t* active_ids, int n_active, float beta1, float beta2) {
   int64_t total = (int64_t)B_pad * d_in_pad;
   int blocks = (int)std::min<int64_t>(ceil_div(total, 256), 152 * 8);
   if (blocks < 1) blocks = 1;
-  k_gather<T><<<blocks, 256, 0, st>>>(X, idx, B, B_pad, d_in, d_in_pad, xb, advance, t_dev, bias_corr,
+  k_gather<T><<<blocks, 256, 0, st>>>(X, idx, B, B_pad, d_in, d_in_pad, ldx, xb, advance, t_dev, bias_corr,
                                        active_ids, n_active, beta1, beta2);
+}
+
+template <typename T>
+void launch_fill_ones(cudaStream_t st, const OnesJob* jobs, int n_jobs, T* xb, T* act) {
+  if (n_jobs > 0) k_fill_ones<T><<<n_jobs, 256, 0, st>>>(jobs, xb, act);
 }
 
 template <typename T>
@@ -577,16 +598,12 @@ template <typename T>
 void launch_head(cudaStream_t st, const HeadArgs<T>& g, int n_jobs) {
   if (n_jobs <= 0) return;
   if (g.d_out == 1) k_head<T, 1><<<n_jobs, 256, 0, st>>>(g);
+  else if (g.d_out <= 16) k_head<T, 16><<<n_jobs, 256, 0, st>>>(g);
   else k_head<T, kMaxDout><<<n_jobs, 256, 0, st>>>(g);
 }
 
 void launch_head_reduce(cudaStream_t st, const HeadReduceArgs& g, int m) {
   k_head_reduce<<<m, 256, 0, st>>>(g);
-}
-
-template <typename T>
-void launch_bias_grad(cudaStream_t st, const BiasJob* jobs, int n_jobs, const T* dz, float* grads, int B_pad) {
-  if (n_jobs > 0) k_bias_grad<T><<<n_jobs, 256, 0, st>>>(jobs, dz, grads, B_pad);
 }
 
 void launch_adamw(cudaStream_t st, const AdamArgs& g, int n_chunks) {
@@ -597,14 +614,15 @@ void launch_init(cudaStream_t st, const InitArgs& g, int n_chunks) {
   if (n_chunks > 0) k_init<<<n_chunks, 256, 0, st>>>(g);
 }
 
-void launch_refresh_wq(cudaStream_t st, const float* p, __nv_bfloat16* wq, int64_t n) {
-  k_refresh_wq<<<152 * 4, 256, 0, st>>>(p, wq, n);
+void launch_refresh_wq(cudaStream_t st, const float* p, __nv_bfloat16* wq0, __nv_bfloat16* wq1, int64_t n) {
+  k_refresh_wq<<<152 * 4, 256, 0, st>>>(p, wq0, wq1, n);
 }
 
 template <typename T>
 void launch_predict_head(cudaStream_t st, const PredictHeadArgs<T>& g, int n_jobs) {
   if (n_jobs <= 0) return;
   if (g.d_out == 1) k_predict_head<T, 1><<<n_jobs, 256, 0, st>>>(g);
+  else if (g.d_out <= 16) k_predict_head<T, 16><<<n_jobs, 256, 0, st>>>(g);
   else k_predict_head<T, kMaxDout><<<n_jobs, 256, 0, st>>>(g);
 }
 
@@ -613,12 +631,12 @@ void launch_debug_masks(cudaStream_t st, uint8_t* out, int B, int w, uint64_t se
   k_debug_masks<<<64, 256, 0, st>>>(out, B, w, seed, member, layer, step, T);
 }
 
-#define TP_INSTANTIATE(T)                                                                        \
-  template void launch_gather<T>(cudaStream_t, const float*, const int32_t*, int, int, int, int, T*, \
-                                 int, int32_t*, float2*, const int32_t*, int, float, float);      \
-  template void launch_gemm_simt<T>(cudaStream_t, const GemmArgs<T>&, int, int);                 \
-  template void launch_head<T>(cudaStream_t, const HeadArgs<T>&, int);                           \
-  template void launch_bias_grad<T>(cudaStream_t, const BiasJob*, int, const T*, float*, int);   \
+#define TP_INSTANTIATE(T)                                                                              \
+  template void launch_gather<T>(cudaStream_t, const float*, const int32_t*, int, int, int, int, int, T*, \
+                                 int, int32_t*, float2*, const int32_t*, int, float, float);            \
+  template void launch_fill_ones<T>(cudaStream_t, const OnesJob*, int, T*, T*);                         \
+  template void launch_gemm_simt<T>(cudaStream_t, const GemmArgs<T>&, int, int);                       \
+  template void launch_head<T>(cudaStream_t, const HeadArgs<T>&, int);                                 \
   template void launch_predict_head<T>(cudaStream_t, const PredictHeadArgs<T>&, int);
 
 TP_INSTANTIATE(float)

@@ -14,7 +14,7 @@ struct GemmArgs {
   const T* xb;
   T* act;
   T* dz;
-  const T* wq;            // matrix-product copy of the weights (bf16 copy, or the fp32 params)
+  const T* wq;            // matrix-product copy of the weights (the fp32 params in fp32 mode)
   const float* params;    // fp32 master (biases)
   float* grads;
   const MemberDev* mem;
@@ -45,10 +45,12 @@ struct HeadReduceArgs {
   const int64_t* part_stride;
   const float* head_part;
   const float* loss_part;
-  float* grads;
+  float* grads;           // store mode: head gradients land here
   float* loss_out;        // caller's [m] or NULL
   float* loss_last;       // pack's own copy [m]
   int32_t B, B_pad, d_out, n_blk_cap;
+  int32_t update;         // 1: apply AdamW to the head parameters instead of storing the gradients
+  AdamDev adam;
 };
 
 struct AdamArgs {
@@ -72,7 +74,8 @@ struct InitArgs {
   float* grads;
   float* m;
   float* v;
-  __nv_bfloat16* wq;
+  __nv_bfloat16* wq0;
+  __nv_bfloat16* wq1;
   uint64_t seed;
 };
 
@@ -89,18 +92,18 @@ struct PredictHeadArgs {
 
 template <typename T>
 void launch_gather(cudaStream_t st, const float* X, const int32_t* idx, int B, int B_pad, int d_in,
-                   int d_in_pad, T* xb, int advance, int32_t* t_dev, float2* bias_corr,
+                   int d_in_pad, int ldx, T* xb, int advance, int32_t* t_dev, float2* bias_corr,
                    const int32_t* active_ids, int n_active, float beta1, float beta2);
 template <typename T>
 void launch_gemm_simt(cudaStream_t st, const GemmArgs<T>& g, int tile_base, int n_tiles);
 template <typename T>
 void launch_head(cudaStream_t st, const HeadArgs<T>& g, int n_jobs);
 void launch_head_reduce(cudaStream_t st, const HeadReduceArgs& g, int m);
-template <typename T>
-void launch_bias_grad(cudaStream_t st, const BiasJob* jobs, int n_jobs, const T* dz, float* grads, int B_pad);
 void launch_adamw(cudaStream_t st, const AdamArgs& g, int n_chunks);
 void launch_init(cudaStream_t st, const InitArgs& g, int n_chunks);
-void launch_refresh_wq(cudaStream_t st, const float* p, __nv_bfloat16* wq, int64_t n);
+void launch_refresh_wq(cudaStream_t st, const float* p, __nv_bfloat16* wq0, __nv_bfloat16* wq1, int64_t n);
+template <typename T>
+void launch_fill_ones(cudaStream_t st, const OnesJob* jobs, int n_jobs, T* xb, T* act);
 template <typename T>
 void launch_predict_head(cudaStream_t st, const PredictHeadArgs<T>& g, int n_jobs);
 void launch_debug_masks(cudaStream_t st, uint8_t* out, int B, int w, uint64_t seed, uint32_t member,

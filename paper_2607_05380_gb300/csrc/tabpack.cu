@@ -32,7 +32,7 @@ struct PhaseEvents {
 
 struct tabpack {
   tp_config cfg{};
-  int d_in_pad = 0, B_cap = 0, n_blk_cap = 0, Lmax = 0;
+  int d_in_pad = 0, ldx = 0, B_cap = 0, n_blk_cap = 0, Lmax = 0;
   cudaStream_t st = nullptr;
   bool bf16 = true;
   std::vector<int32_t> depth, width;
@@ -48,7 +48,9 @@ struct tabpack {
 
   // device memory
   float *params = nullptr, *grads = nullptr, *adam_m = nullptr, *adam_v = nullptr;
-  __nv_bfloat16* wq = nullptr;
+  __nv_bfloat16* wq[2] = {nullptr, nullptr};
+  int wcur = 0;  // the bf16 weight copy the next step reads
+  bool fuse_adamw = false;  // bf16: AdamW in the wgrad epilogue (else a stand-alone pass)
   void *xb = nullptr, *act = nullptr, *dz = nullptr;
   float *logits = nullptr, *head_part = nullptr, *loss_part = nullptr, *loss_last = nullptr;
   int32_t* t_dev = nullptr;
@@ -63,13 +65,12 @@ struct tabpack {
   HeadJob* head_jobs_dev = nullptr;
   HeadReduceJob* hred_dev = nullptr;
   int64_t* part_stride_dev = nullptr;
-  BiasJob* bias_jobs_dev = nullptr;
   TcPlan tc;  // tensor-core GEMM plan (bf16 mode)
 
   // schedule (active members)
-  int n_active = 0, n_chunks = 0, n_head_jobs = 0, n_bias_jobs = 0;
-  std::vector<std::pair<int, int>> fwd_rng, bwd_rng;  // tile ranges per depth index
-  int cap_chunks = 0, cap_probs = 0, cap_tiles = 0, cap_head = 0, cap_bias = 0;
+  int n_active = 0, n_chunks = 0, n_head_jobs = 0;
+  std::vector<std::pair<int, int>> fwd_rng, bwd_rng;  // CUDA-core tile ranges per depth index
+  int cap_chunks = 0, cap_probs = 0, cap_tiles = 0, cap_head = 0;
 
   int last_B = 0;
   int64_t launches = 0;
@@ -108,6 +109,12 @@ tp_status fail(tabpack* h, tp_status s, const char* fmt, ...) {
       return fail((h), TP_ECUDA, "kernel launch: %s (%s:%d)", cudaGetErrorString(e_), __FILE__, __LINE__); \
   } while (0)
 
+#define TP_TRY(expr)                 \
+  do {                               \
+    tp_status s_ = (expr);           \
+    if (s_ != TP_OK) return s_;      \
+  } while (0)
+
 template <typename P>
 tp_status dalloc(tabpack* h, P** ptr, size_t bytes) {
   void* p = nullptr;
@@ -122,12 +129,6 @@ tp_status dalloc(tabpack* h, P** ptr, size_t bytes) {
   *ptr = (P*)p;
   return TP_OK;
 }
-
-#define TP_TRY(expr)                 \
-  do {                               \
-    tp_status s_ = (expr);           \
-    if (s_ != TP_OK) return s_;      \
-  } while (0)
 
 void prof_begin(tabpack* h, int phase, int* slot) {
   *slot = -1;
@@ -162,11 +163,14 @@ void prof_flush(tabpack* h) {
   P.pending.clear();
 }
 
+int ldh_of(const tabpack* h, int i) { return h->width[i] + kOnesCols; }
+
 // ------------------------------------------------------------------ layout
 tp_status build_layout(tabpack* h) {
   const auto& c = h->cfg;
   const int m = c.m;
   h->d_in_pad = (int)round_up(c.d_in, 8);
+  h->ldx = h->d_in_pad + kOnesCols;
   h->B_cap = (int)round_up(c.max_batch, kRowTile);
   h->n_blk_cap = h->B_cap / kHeadRows;
   h->W_off.resize(m);
@@ -176,7 +180,7 @@ tp_status build_layout(tabpack* h) {
   h->mem.resize(m);
   h->part_off.resize(m);
   h->part_stride.resize(m);
-  int64_t off = 0, aoff = 0, hoff = 0;
+  int64_t off = 0, aoff = 0, zoff = 0, hoff = 0;
   h->Lmax = 0;
   for (int i = 0; i < m; ++i) {
     const int L = h->depth[i], w = h->width[i];
@@ -195,8 +199,9 @@ tp_status build_layout(tabpack* h) {
     }
     for (int l = 0; l < L; ++l) {
       h->act_off[i][l] = aoff;
-      aoff += round_up((int64_t)h->B_cap * w, 128);
-      h->dz_off[i][l] = aoff;  // dz uses its own arena; same offsets scheme
+      aoff += round_up((int64_t)h->B_cap * ldh_of(h, i), 128);
+      h->dz_off[i][l] = zoff;
+      zoff += round_up((int64_t)h->B_cap * w, 128);
     }
     const float p = h->dropout[i];
     double T = std::floor((double)p * 4294967296.0);
@@ -215,19 +220,17 @@ tp_status build_layout(tabpack* h) {
     h->part_off[i] = hoff;
     hoff += h->part_stride[i] * h->n_blk_cap;
   }
-  for (int i = 0; i < m; ++i)
-    for (int l = 0; l < h->depth[i]; ++l) h->dz_off[i][l] = h->act_off[i][l];
   h->n_params = round_up(off, kSegAlign);
   h->act_elems = std::max<int64_t>(aoff, 128);
-  h->dz_elems = h->act_elems;
-  h->xb_elems = (int64_t)h->B_cap * h->d_in_pad;
+  h->dz_elems = std::max<int64_t>(zoff, 128);
+  h->xb_elems = (int64_t)h->B_cap * h->ldx;
   h->head_part_elems = std::max<int64_t>(hoff, 32);
   return TP_OK;
 }
 
 // --------------------------------------------------------------- schedule
 // Rebuilt whenever the active set changes: per depth index the forward and
-// backward GEMM work of the active members, head / bias / AdamW work lists.
+// backward GEMM work of the active members, the head and AdamW work lists.
 tp_status build_schedule(tabpack* h) {
   const auto& c = h->cfg;
   const int m = c.m;
@@ -236,62 +239,65 @@ tp_status build_schedule(tabpack* h) {
     if (h->active[i]) ids.push_back(i);
   h->n_active = (int)ids.size();
 
+  // CUDA-core products (fp32 mode)
   std::vector<GemmProblem> probs;
   std::vector<GemmTile> tiles;
   h->fwd_rng.assign(h->Lmax, {0, 0});
   h->bwd_rng.assign(h->Lmax, {0, 0});
-  auto add_tiles = [&](int prob, int M_rows, int N) {
-    const int tm = 64, tn = 64;
-    for (int m0 = 0; m0 < M_rows; m0 += tm)
-      for (int n0 = 0; n0 < N; n0 += tn) tiles.push_back(GemmTile{prob, m0, n0, std::min(tn, N - n0)});
-  };
-  for (int l = 0; l < h->Lmax; ++l) {
-    const int base = (int)tiles.size();
-    for (int i : ids) {
-      if (h->depth[i] <= l) continue;
-      const int w = h->width[i];
-      GemmProblem P{};
-      P.kind = kFwd; P.member = i; P.layer = l;
-      P.M = 0; P.N = w; P.K = l == 0 ? h->d_in_pad : w;
-      P.a_src = l == 0 ? kSrcXb : kSrcAct;
-      P.a_off = l == 0 ? 0 : h->act_off[i][l - 1];
-      P.lda = l == 0 ? h->d_in_pad : w;
-      P.b_src = kSrcWq; P.b_off = h->W_off[i][l]; P.ldb = P.K;
-      P.c_off = h->act_off[i][l]; P.ldc = w;
-      P.aux_off = h->b_off[i][l];
-      probs.push_back(P);
-      add_tiles((int)probs.size() - 1, h->B_cap, w);
-    }
-    h->fwd_rng[l] = {base, (int)tiles.size() - base};
-  }
-  for (int l = h->Lmax - 1; l >= 0; --l) {
-    const int base = (int)tiles.size();
-    for (int i : ids) {
-      if (h->depth[i] <= l) continue;
-      const int w = h->width[i];
-      const int in_pad = l == 0 ? h->d_in_pad : w;
-      if (l > 0) {
+  if (!h->bf16) {
+    auto add_tiles = [&](int prob, int M_rows, int N) {
+      for (int m0 = 0; m0 < M_rows; m0 += 64)
+        for (int n0 = 0; n0 < N; n0 += 64) tiles.push_back(GemmTile{prob, m0, n0, std::min(64, N - n0)});
+    };
+    for (int l = 0; l < h->Lmax; ++l) {
+      const int base = (int)tiles.size();
+      for (int i : ids) {
+        if (h->depth[i] <= l) continue;
+        const int w = h->width[i];
         GemmProblem P{};
-        P.kind = kDgrad; P.member = i; P.layer = l;
-        P.M = 0; P.N = w; P.K = w;
-        P.a_src = kSrcDz; P.a_off = h->dz_off[i][l]; P.lda = w;
-        P.b_src = kSrcWq; P.b_off = h->W_off[i][l]; P.ldb = w;
-        P.c_off = h->dz_off[i][l - 1]; P.ldc = w;
-        P.aux_off = h->act_off[i][l - 1];
+        P.kind = kFwd; P.member = i; P.layer = l;
+        P.M = 0; P.N = w; P.K = l == 0 ? h->d_in_pad : w;
+        P.a_src = l == 0 ? kSrcXb : kSrcAct;
+        P.a_off = l == 0 ? 0 : h->act_off[i][l - 1];
+        P.lda = l == 0 ? h->ldx : ldh_of(h, i);
+        P.b_src = kSrcWq; P.b_off = h->W_off[i][l]; P.ldb = P.K;
+        P.c_off = h->act_off[i][l]; P.ldc = ldh_of(h, i);
+        P.aux_off = h->b_off[i][l];
         probs.push_back(P);
         add_tiles((int)probs.size() - 1, h->B_cap, w);
       }
-      GemmProblem Q{};
-      Q.kind = kWgrad; Q.member = i; Q.layer = l;
-      Q.M = w; Q.N = in_pad; Q.K = 0;
-      Q.a_src = kSrcDz; Q.a_off = h->dz_off[i][l]; Q.lda = w;
-      Q.b_src = l == 0 ? kSrcXb : kSrcAct; Q.b_off = l == 0 ? 0 : h->act_off[i][l - 1];
-      Q.ldb = in_pad;
-      Q.c_off = h->W_off[i][l]; Q.ldc = in_pad;
-      probs.push_back(Q);
-      add_tiles((int)probs.size() - 1, w, in_pad);
+      h->fwd_rng[l] = {base, (int)tiles.size() - base};
     }
-    h->bwd_rng[l] = {base, (int)tiles.size() - base};
+    for (int l = h->Lmax - 1; l >= 0; --l) {
+      const int base = (int)tiles.size();
+      for (int i : ids) {
+        if (h->depth[i] <= l) continue;
+        const int w = h->width[i];
+        const int in_pad = l == 0 ? h->d_in_pad : w;
+        if (l > 0) {
+          GemmProblem P{};
+          P.kind = kDgrad; P.member = i; P.layer = l;
+          P.M = 0; P.N = w; P.K = w;
+          P.a_src = kSrcDz; P.a_off = h->dz_off[i][l]; P.lda = w;
+          P.b_src = kSrcWq; P.b_off = h->W_off[i][l]; P.ldb = w;
+          P.c_off = h->dz_off[i][l - 1]; P.ldc = w;
+          P.aux_off = h->act_off[i][l - 1]; P.ld_aux = ldh_of(h, i);
+          probs.push_back(P);
+          add_tiles((int)probs.size() - 1, h->B_cap, w);
+        }
+        GemmProblem Q{};
+        Q.kind = kWgrad; Q.member = i; Q.layer = l;
+        Q.M = w; Q.N = in_pad + 1; Q.K = 0;  // the last column is the bias gradient
+        Q.a_src = kSrcDz; Q.a_off = h->dz_off[i][l]; Q.lda = w;
+        Q.b_src = l == 0 ? kSrcXb : kSrcAct; Q.b_off = l == 0 ? 0 : h->act_off[i][l - 1];
+        Q.ldb = l == 0 ? h->ldx : ldh_of(h, i);
+        Q.c_off = h->W_off[i][l]; Q.ldc = in_pad;
+        Q.aux_off = h->b_off[i][l];
+        probs.push_back(Q);
+        add_tiles((int)probs.size() - 1, w, in_pad + 1);
+      }
+      h->bwd_rng[l] = {base, (int)tiles.size() - base};
+    }
   }
 
   std::vector<HeadJob> hj;
@@ -302,15 +308,20 @@ tp_status build_schedule(tabpack* h) {
   }
   for (int i : ids) {
     const int L = h->depth[i];
-    for (int b = 0; b < h->n_blk_cap; ++b)
-      hj.push_back(HeadJob{i, b, h->act_off[i][L - 1], h->dz_off[i][L - 1], h->W_off[i][L], h->b_off[i][L],
-                           h->part_off[i] + b * h->part_stride[i]});
+    for (int b = 0; b < h->n_blk_cap; ++b) {
+      HeadJob j{};
+      j.member = i;
+      j.blk = b;
+      j.h_ld = ldh_of(h, i);
+      j.h_off = h->act_off[i][L - 1];
+      j.dz_off = h->dz_off[i][L - 1];
+      j.w_off = h->W_off[i][L];
+      j.b_off = h->b_off[i][L];
+      j.part_off = h->part_off[i] + b * h->part_stride[i];
+      hj.push_back(j);
+    }
   }
-  std::vector<BiasJob> bj;
-  for (int i : ids)
-    for (int l = 0; l < h->depth[i]; ++l)
-      for (int c0 = 0; c0 < h->width[i]; c0 += 256)
-        bj.push_back(BiasJob{h->dz_off[i][l], h->b_off[i][l], h->width[i], c0});
+  // element-wise chunks of the active members (init, fp32-mode AdamW)
   std::vector<Chunk> ch;
   for (int s = 0; s < (int)h->segs.size(); ++s) {
     const Segment& S = h->segs[s];
@@ -321,37 +332,73 @@ tp_status build_schedule(tabpack* h) {
   }
 
   // capacities are fixed at create (all members active)
-  if (h->probs_dev == nullptr) {
+  if (h->head_jobs_dev == nullptr) {
     h->cap_probs = (int)probs.size() + 1;
     h->cap_tiles = (int)tiles.size() + 1;
     h->cap_head = (int)hj.size() + 1;
-    h->cap_bias = (int)bj.size() + 1;
     h->cap_chunks = (int)ch.size() + 1;
     TP_TRY(dalloc(h, &h->probs_dev, sizeof(GemmProblem) * h->cap_probs));
     TP_TRY(dalloc(h, &h->tiles_dev, sizeof(GemmTile) * h->cap_tiles));
     TP_TRY(dalloc(h, &h->head_jobs_dev, sizeof(HeadJob) * h->cap_head));
     TP_TRY(dalloc(h, &h->hred_dev, sizeof(HeadReduceJob) * m));
-    TP_TRY(dalloc(h, &h->bias_jobs_dev, sizeof(BiasJob) * h->cap_bias));
     TP_TRY(dalloc(h, &h->chunks_dev, sizeof(Chunk) * h->cap_chunks));
     TP_TRY(dalloc(h, &h->active_ids_dev, sizeof(int32_t) * m));
   }
   if ((int)probs.size() > h->cap_probs || (int)tiles.size() > h->cap_tiles || (int)hj.size() > h->cap_head ||
-      (int)bj.size() > h->cap_bias || (int)ch.size() > h->cap_chunks)
+      (int)ch.size() > h->cap_chunks)
     return fail(h, TP_ESTATE, "schedule grew beyond its capacity");
   TP_CUDA(h, cudaStreamSynchronize(h->st));
   if (!probs.empty()) TP_CUDA(h, cudaMemcpy(h->probs_dev, probs.data(), sizeof(GemmProblem) * probs.size(), cudaMemcpyHostToDevice));
   if (!tiles.empty()) TP_CUDA(h, cudaMemcpy(h->tiles_dev, tiles.data(), sizeof(GemmTile) * tiles.size(), cudaMemcpyHostToDevice));
   if (!hj.empty()) TP_CUDA(h, cudaMemcpy(h->head_jobs_dev, hj.data(), sizeof(HeadJob) * hj.size(), cudaMemcpyHostToDevice));
   TP_CUDA(h, cudaMemcpy(h->hred_dev, hr.data(), sizeof(HeadReduceJob) * m, cudaMemcpyHostToDevice));
-  if (!bj.empty()) TP_CUDA(h, cudaMemcpy(h->bias_jobs_dev, bj.data(), sizeof(BiasJob) * bj.size(), cudaMemcpyHostToDevice));
   if (!ch.empty()) TP_CUDA(h, cudaMemcpy(h->chunks_dev, ch.data(), sizeof(Chunk) * ch.size(), cudaMemcpyHostToDevice));
   if (!ids.empty()) TP_CUDA(h, cudaMemcpy(h->active_ids_dev, ids.data(), sizeof(int32_t) * ids.size(), cudaMemcpyHostToDevice));
   TP_CUDA(h, cudaMemcpy(h->active_dev, h->active.data(), m, cudaMemcpyHostToDevice));
   h->n_head_jobs = (int)hj.size();
-  h->n_bias_jobs = (int)bj.size();
   h->n_chunks = (int)ch.size();
-  if (h->bf16) TP_TRY(tc_build_plan(h->tc, h->cfg, h->depth, h->width, h->active, h->W_off, h->b_off, h->act_off,
-                                    h->dz_off, h->d_in_pad, h->B_cap, h->wq, h->xb, h->act, h->dz, h->err));
+  if (h->bf16) {
+    TcLayout lay;
+    lay.depth = &h->depth;
+    lay.width = &h->width;
+    lay.active = &h->active;
+    lay.W_off = &h->W_off;
+    lay.b_off = &h->b_off;
+    lay.act_off = &h->act_off;
+    lay.dz_off = &h->dz_off;
+    lay.m = m;
+    lay.d_in_pad = h->d_in_pad;
+    lay.ldx = h->ldx;
+    lay.B_cap = h->B_cap;
+    lay.wq[0] = h->wq[0];
+    lay.wq[1] = h->wq[1];
+    lay.xb = h->xb;
+    lay.act = h->act;
+    lay.dz = h->dz;
+    TP_TRY(tc_build_plan(h->tc, lay, h->err));
+  }
+  return TP_OK;
+}
+
+// Column in_pad of xb and column w of every act matrix := 1 (all rows).
+template <typename T>
+tp_status fill_ones(tabpack* h) {
+  std::vector<OnesJob> jobs;
+  jobs.push_back(OnesJob{0, h->ldx, h->d_in_pad, h->B_cap, 0});
+  for (int i = 0; i < h->cfg.m; ++i)
+    for (int l = 0; l < h->depth[i]; ++l)
+      jobs.push_back(OnesJob{h->act_off[i][l], ldh_of(h, i), h->width[i], h->B_cap, 1});
+  OnesJob* d = nullptr;
+  TP_CUDA(h, cudaMalloc(&d, sizeof(OnesJob) * jobs.size()));
+  cudaError_t e = cudaMemcpy(d, jobs.data(), sizeof(OnesJob) * jobs.size(), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) {
+    launch_fill_ones<T>(h->st, d, (int)jobs.size(), (T*)h->xb, (T*)h->act);
+    h->launches++;
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+  cudaFree(d);
+  if (e != cudaSuccess) return fail(h, TP_ECUDA, "fill ones: %s", cudaGetErrorString(e));
   return TP_OK;
 }
 
@@ -362,7 +409,10 @@ tp_status alloc_all(tabpack* h) {
   TP_TRY(dalloc(h, &h->grads, sizeof(float) * h->n_params));
   TP_TRY(dalloc(h, &h->adam_m, sizeof(float) * h->n_params));
   TP_TRY(dalloc(h, &h->adam_v, sizeof(float) * h->n_params));
-  if (h->bf16) TP_TRY(dalloc(h, &h->wq, sizeof(__nv_bfloat16) * h->n_params));
+  if (h->bf16) {
+    TP_TRY(dalloc(h, &h->wq[0], sizeof(__nv_bfloat16) * h->n_params));
+    TP_TRY(dalloc(h, &h->wq[1], sizeof(__nv_bfloat16) * h->n_params));
+  }
   TP_TRY(dalloc(h, &h->xb, h->elem * h->xb_elems));
   TP_TRY(dalloc(h, &h->act, h->elem * h->act_elems));
   TP_TRY(dalloc(h, &h->dz, h->elem * h->dz_elems));
@@ -405,7 +455,7 @@ GemmArgs<T> gemm_args(tabpack* h, int B, int B_pad, uint32_t step, int train) {
   g.xb = (const T*)h->xb;
   g.act = (T*)h->act;
   g.dz = (T*)h->dz;
-  g.wq = h->bf16 ? (const T*)h->wq : (const T*)h->params;
+  g.wq = (const T*)h->params;  // the CUDA-core path runs in fp32 mode only
   g.params = h->params;
   g.grads = h->grads;
   g.mem = h->mem_dev;
@@ -417,13 +467,29 @@ GemmArgs<T> gemm_args(tabpack* h, int B, int B_pad, uint32_t step, int train) {
   return g;
 }
 
+AdamDev adam_dev(tabpack* h, __nv_bfloat16* wq_out) {
+  AdamDev a;
+  a.params = h->params;
+  a.m = h->adam_m;
+  a.v = h->adam_v;
+  a.wq_out = wq_out;
+  a.bias_corr = h->bias_corr;
+  a.mem = h->mem_dev;
+  a.beta1 = h->cfg.beta1;
+  a.beta2 = h->cfg.beta2;
+  a.eps = h->cfg.eps;
+  a.wd_on_bias = h->cfg.wd_on_bias;
+  return a;
+}
+
 template <typename T>
 tp_status run_forward(tabpack* h, int B, int B_pad, uint32_t step, int train) {
   for (int l = 0; l < h->Lmax; ++l) {
     int slot;
     prof_begin(h, train ? TP_PH_FWD : TP_PH_PREDICT, &slot);
-    if (h->bf16 && h->tc.enabled) {
-      TP_TRY(tc_run_fwd(h->tc, h->st, l, B, B_pad, step, train, h->cfg.seed, h->params, h->mem_dev, h->act, h->err));
+    if (h->bf16) {
+      TP_TRY(tc_run_fwd(h->tc, h->st, l, B, B_pad, h->wcur, step, train, h->cfg.seed, h->params, h->mem_dev, h->act,
+                        h->err));
     } else {
       auto g = gemm_args<T>(h, B, B_pad, step, train);
       launch_gemm_simt<T>(h->st, g, h->fwd_rng[l].first, h->fwd_rng[l].second);
@@ -435,14 +501,19 @@ tp_status run_forward(tabpack* h, int B, int B_pad, uint32_t step, int train) {
   return TP_OK;
 }
 
+// One step on the pack's stream:
+//   gather -> forward (per depth) -> head + loss -> head reduce (+ head AdamW)
+//   -> backward (per depth, deepest first; bf16: AdamW fused into the wgrad
+//   epilogue, bias gradients from the ones column) -> fp32 mode: AdamW.
 template <typename T>
 tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* idx, const void* y, int B,
                    uint32_t step, float* loss_out, bool update) {
   const int B_pad = (int)round_up(B, kRowTile);
+  const bool fused = update && h->bf16 && h->fuse_adamw;
+  __nv_bfloat16* wq_next = h->bf16 ? h->wq[h->wcur ^ 1] : nullptr;
   int slot;
-  // gather + step counters
   prof_begin(h, TP_PH_GATHER, &slot);
-  launch_gather<T>(h->st, X, idx, B, B_pad, h->cfg.d_in, h->d_in_pad, (T*)h->xb, update ? 1 : 0, h->t_dev,
+  launch_gather<T>(h->st, X, idx, B, B_pad, h->cfg.d_in, h->d_in_pad, h->ldx, (T*)h->xb, update ? 1 : 0, h->t_dev,
                    h->bias_corr, h->active_ids_dev, h->n_active, h->cfg.beta1, h->cfg.beta2);
   TP_LAUNCHED(h);
   h->launches++;
@@ -470,24 +541,7 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
   launch_head<T>(h->st, hg, h->n_head_jobs);
   TP_LAUNCHED(h);
   h->launches++;
-  prof_end(h, slot, 1, TP_PH_HEAD);
-  // backward GEMMs, deepest layer first
-  for (int l = h->Lmax - 1; l >= 0; --l) {
-    prof_begin(h, TP_PH_BWD, &slot);
-    if (h->bf16 && h->tc.enabled) {
-      TP_TRY(tc_run_bwd(h->tc, h->st, l, B, B_pad, h->grads, h->mem_dev, h->act, h->dz, h->err));
-    } else {
-      auto g = gemm_args<T>(h, B, B_pad, step, 1);
-      launch_gemm_simt<T>(h->st, g, h->bwd_rng[l].first, h->bwd_rng[l].second);
-    }
-    TP_LAUNCHED(h);
-    h->launches++;
-    prof_end(h, slot, 1, TP_PH_BWD);
-  }
-  // bias gradients + head gradients / losses
-  prof_begin(h, TP_PH_BIAS, &slot);
-  launch_bias_grad<T>(h->st, h->bias_jobs_dev, h->n_bias_jobs, (const T*)h->dz, h->grads, B_pad);
-  TP_LAUNCHED(h);
+  // head gradients (sum of the per-block partials), losses, head AdamW
   HeadReduceArgs rg;
   rg.jobs = h->hred_dev;
   rg.active = h->active_dev;
@@ -501,11 +555,28 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
   rg.B_pad = B_pad;
   rg.d_out = h->cfg.d_out;
   rg.n_blk_cap = h->n_blk_cap;
+  rg.update = fused ? 1 : 0;
+  rg.adam = adam_dev(h, wq_next);
   launch_head_reduce(h->st, rg, h->cfg.m);
   TP_LAUNCHED(h);
-  h->launches += 2;
-  prof_end(h, slot, 2, TP_PH_BIAS);
-  if (update) {
+  h->launches++;
+  prof_end(h, slot, 2, TP_PH_HEAD);
+  // backward products, deepest layer first
+  const AdamDev ad = adam_dev(h, wq_next);
+  for (int l = h->Lmax - 1; l >= 0; --l) {
+    prof_begin(h, TP_PH_BWD, &slot);
+    if (h->bf16) {
+      TP_TRY(tc_run_bwd(h->tc, h->st, l, B, B_pad, h->wcur, h->mem_dev, h->act, h->dz, h->grads, fused ? 1 : 0, ad,
+                        h->err));
+    } else {
+      auto g = gemm_args<T>(h, B, B_pad, step, 1);
+      launch_gemm_simt<T>(h->st, g, h->bwd_rng[l].first, h->bwd_rng[l].second);
+    }
+    TP_LAUNCHED(h);
+    h->launches++;
+    prof_end(h, slot, 1, TP_PH_BWD);
+  }
+  if (update && !fused && h->n_chunks > 0) {
     prof_begin(h, TP_PH_ADAMW, &slot);
     AdamArgs ag;
     ag.chunks = h->chunks_dev;
@@ -516,7 +587,7 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
     ag.grads = h->grads;
     ag.m = h->adam_m;
     ag.v = h->adam_v;
-    ag.wq = h->bf16 ? h->wq : nullptr;
+    ag.wq = wq_next;
     ag.beta1 = h->cfg.beta1;
     ag.beta2 = h->cfg.beta2;
     ag.eps = h->cfg.eps;
@@ -526,6 +597,7 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
     h->launches++;
     prof_end(h, slot, 1, TP_PH_ADAMW);
   }
+  if (update && h->bf16) h->wcur ^= 1;
   h->last_B = B;
   (void)n_rows;
   return TP_OK;
@@ -538,8 +610,8 @@ tp_status run_predict(tabpack* h, const float* X, int64_t N, float* out) {
     const int B_pad = (int)round_up(rows, kRowTile);
     int slot;
     prof_begin(h, TP_PH_PREDICT, &slot);
-    launch_gather<T>(h->st, X + n0 * h->cfg.d_in, nullptr, rows, B_pad, h->cfg.d_in, h->d_in_pad, (T*)h->xb, 0,
-                     h->t_dev, h->bias_corr, h->active_ids_dev, 0, h->cfg.beta1, h->cfg.beta2);
+    launch_gather<T>(h->st, X + n0 * h->cfg.d_in, nullptr, rows, B_pad, h->cfg.d_in, h->d_in_pad, h->ldx, (T*)h->xb,
+                     0, h->t_dev, h->bias_corr, h->active_ids_dev, 0, h->cfg.beta1, h->cfg.beta2);
     TP_LAUNCHED(h);
     h->launches++;
     prof_end(h, slot, 1, TP_PH_PREDICT);
@@ -565,6 +637,16 @@ tp_status run_predict(tabpack* h, const float* X, int64_t N, float* out) {
   return TP_OK;
 }
 
+// both bf16 copies := bf16(params) (after a host write or an active-set change)
+tp_status refresh_copies(tabpack* h) {
+  if (!h->bf16) return TP_OK;
+  launch_refresh_wq(h->st, h->params, h->wq[0], h->wq[1], h->n_params);
+  TP_LAUNCHED(h);
+  h->launches++;
+  TP_CUDA(h, cudaStreamSynchronize(h->st));
+  return TP_OK;
+}
+
 tp_status check_step_args(tabpack* h, const float* X, int64_t n_rows, const int32_t* idx, const void* y, int B) {
   if (!h) return fail(nullptr, TP_EINVAL, "null pack");
   if (!X || !idx || !y) return fail(h, TP_EINVAL, "X, idx and y must be device pointers");
@@ -577,6 +659,13 @@ tp_status check_ml(tabpack* h, int member, int layer) {
   if (!h) return fail(nullptr, TP_EINVAL, "null pack");
   if (member < 0 || member >= h->cfg.m) return fail(h, TP_EINVAL, "member %d out of range", member);
   if (layer < 0 || layer > h->depth[member]) return fail(h, TP_EINVAL, "layer %d out of range", layer);
+  return TP_OK;
+}
+
+// synchronise and surface a bounded-wait timeout of the tensor-core pipeline
+tp_status sync_check(tabpack* h) {
+  TP_CUDA(h, cudaStreamSynchronize(h->st));
+  if (h->bf16 && h->tc.enabled) TP_TRY(tc_check(h->tc, h->st, h->err));
   return TP_OK;
 }
 
@@ -619,6 +708,7 @@ tp_status pack_create(const tp_config* cfg, const int32_t* depth, const int32_t*
   h->cfg = *cfg;
   h->st = (cudaStream_t)cuda_stream;
   h->bf16 = cfg->precision == TP_BF16;
+  h->fuse_adamw = h->bf16 && cfg->fuse_optimizer != 0;
   h->depth.assign(depth, depth + cfg->m);
   h->width.assign(width, width + cfg->m);
   h->dropout.assign(dropout, dropout + cfg->m);
@@ -628,9 +718,10 @@ tp_status pack_create(const tp_config* cfg, const int32_t* depth, const int32_t*
   tp_status s = build_layout(h);
   if (s == TP_OK) s = alloc_all(h);
   if (s == TP_OK) s = build_schedule(h);
+  if (s == TP_OK) s = h->bf16 ? fill_ones<__nv_bfloat16>(h) : fill_ones<float>(h);
   if (s == TP_OK) {
     // Philox init of every parameter (all members active here)
-    InitArgs ig{h->chunks_dev, h->segs_dev, h->params, h->grads, h->adam_m, h->adam_v, h->wq, cfg->seed};
+    InitArgs ig{h->chunks_dev, h->segs_dev, h->params, h->grads, h->adam_m, h->adam_v, h->wq[0], h->wq[1], cfg->seed};
     launch_init(h->st, ig, h->n_chunks);
     h->launches++;
     cudaError_t le = cudaGetLastError();
@@ -685,13 +776,16 @@ tp_status pack_predict(tabpack_t* h, const float* X, int64_t N, float* out) {
 
 tp_status pack_set_active(tabpack_t* h, const uint8_t* active) {
   if (!h || !active) return fail(h, TP_EINVAL, "null argument");
+  TP_TRY(sync_check(h));
   for (int i = 0; i < h->cfg.m; ++i) h->active[i] = active[i] ? 1 : 0;
-  return build_schedule(h);
+  TP_TRY(build_schedule(h));
+  // a member that stops keeps its latest weights in both bf16 copies
+  return refresh_copies(h);
 }
 
 static tp_status copy_layer(tabpack_t* h, int member, int layer, float* W, float* b, const float* src) {
   TP_TRY(check_ml(h, member, layer));
-  TP_CUDA(h, cudaStreamSynchronize(h->st));
+  TP_TRY(sync_check(h));
   const int L = h->depth[member], w = h->width[member];
   const int in = layer == 0 ? h->cfg.d_in : w, in_pad = layer == 0 ? h->d_in_pad : w;
   const int out = layer == L ? h->cfg.d_out : w;
@@ -716,7 +810,7 @@ tp_status pack_get_grads(tabpack_t* h, int32_t member, int32_t layer, float* W, 
 
 tp_status pack_set_params(tabpack_t* h, int32_t member, int32_t layer, const float* W, const float* b) {
   TP_TRY(check_ml(h, member, layer));
-  TP_CUDA(h, cudaStreamSynchronize(h->st));
+  TP_TRY(sync_check(h));
   const int L = h->depth[member], w = h->width[member];
   const int in = layer == 0 ? h->cfg.d_in : w, in_pad = layer == 0 ? h->d_in_pad : w;
   const int out = layer == L ? h->cfg.d_out : w;
@@ -726,19 +820,13 @@ tp_status pack_set_params(tabpack_t* h, int32_t member, int32_t layer, const flo
     TP_CUDA(h, cudaMemcpy(h->params + h->W_off[member][layer], tmp.data(), tmp.size() * 4, cudaMemcpyHostToDevice));
   }
   if (b) TP_CUDA(h, cudaMemcpy(h->params + h->b_off[member][layer], b, (size_t)out * 4, cudaMemcpyHostToDevice));
-  if (h->bf16) {
-    launch_refresh_wq(h->st, h->params, h->wq, h->n_params);
-    TP_LAUNCHED(h);
-    h->launches++;
-    TP_CUDA(h, cudaStreamSynchronize(h->st));
-  }
-  return TP_OK;
+  return refresh_copies(h);
 }
 
 tp_status pack_get_logits(tabpack_t* h, int32_t member, float* out) {
   TP_TRY(check_ml(h, member, 0));
   if (!out) return fail(h, TP_EINVAL, "null out");
-  TP_CUDA(h, cudaStreamSynchronize(h->st));
+  TP_TRY(sync_check(h));
   TP_CUDA(h, cudaMemcpy(out, h->logits + (size_t)member * h->B_cap * h->cfg.d_out,
                         sizeof(float) * (size_t)h->last_B * h->cfg.d_out, cudaMemcpyDeviceToHost));
   return TP_OK;
@@ -765,15 +853,19 @@ tp_status pack_debug_activations(tabpack_t* h, int32_t member, int32_t layer, fl
   TP_TRY(check_ml(h, member, layer));
   if (layer >= h->depth[member]) return fail(h, TP_EINVAL, "layer %d is the head", layer);
   if (!out) return fail(h, TP_EINVAL, "null out");
-  TP_CUDA(h, cudaStreamSynchronize(h->st));
-  const size_t n = (size_t)h->last_B * h->width[member];
+  TP_TRY(sync_check(h));
+  const int w = h->width[member], ldh = ldh_of(h, member);
+  const size_t n = (size_t)h->last_B * ldh;
   if (h->bf16) {
     std::vector<__nv_bfloat16> tmp(n);
     TP_CUDA(h, cudaMemcpy(tmp.data(), (const __nv_bfloat16*)h->act + h->act_off[member][layer], n * 2,
                           cudaMemcpyDeviceToHost));
-    for (size_t e = 0; e < n; ++e) out[e] = __bfloat162float(tmp[e]);
+    for (int r = 0; r < h->last_B; ++r)
+      for (int c = 0; c < w; ++c) out[(size_t)r * w + c] = __bfloat162float(tmp[(size_t)r * ldh + c]);
   } else {
-    TP_CUDA(h, cudaMemcpy(out, (const float*)h->act + h->act_off[member][layer], n * 4, cudaMemcpyDeviceToHost));
+    std::vector<float> tmp(n);
+    TP_CUDA(h, cudaMemcpy(tmp.data(), (const float*)h->act + h->act_off[member][layer], n * 4, cudaMemcpyDeviceToHost));
+    for (int r = 0; r < h->last_B; ++r) std::memcpy(out + (size_t)r * w, tmp.data() + (size_t)r * ldh, (size_t)w * 4);
   }
   return TP_OK;
 }
@@ -820,6 +912,7 @@ tp_status pack_profile_enable(tabpack_t* h, int32_t enable) {
 tp_status pack_profile_read(tabpack_t* h, double* ms, int64_t* launches, int32_t reset) {
   if (!h) return fail(nullptr, TP_EINVAL, "null pack");
   prof_flush(h);
+  TP_TRY(sync_check(h));
   for (int p = 0; p < TP_PH_COUNT; ++p) {
     if (ms) ms[p] = h->prof.ms[p];
     if (launches) launches[p] = h->prof.launches[p];

@@ -16,12 +16,15 @@
 //              the fused epilogue of the product kind:
 //                kFwd   z = acc + b; h = dropout(relu(z)) / (1 - p)   -> bf16
 //                kDgrad dz_prev = acc * [H_prev > 0] / (1 - p)          -> bf16
-//                kWgrad dW = acc                                        -> fp32
+//                kWgrad dW, db = acc (store) or AdamW(p, m, v; dW, db) with
+//                       the fp32 master, the moments and the bf16 copy
 // Ragged K (member widths that are multiples of 16 but not of 64) issues
 // only the K=16 steps that exist; out-of-range operand rows and columns are
 // zero-filled by TMA.  Operands are read K-major or MN-major straight from
 // their row-major arrays through the descriptor's major-ness bits, so no
-// transposed copies are kept.
+// transposed copies are kept.  Because the weight-gradient reduction runs
+// over the whole batch inside one tile, the fused AdamW sees final gradients
+// and they never travel through HBM.
 //
 // Every mbarrier wait is bounded (2 s): a role that gives up sets the
 // pack's device error word and an abort flag in shared memory; the other
@@ -55,7 +58,10 @@ struct SmemTail {
   uint32_t tmem_base;
   int abort;
 };
-constexpr int kSmemBytes = kStages * kStageBytes + 1024 + (int)sizeof(SmemTail) + 64;
+// per epilogue warp a 32 x 33 fp32 transpose buffer (wgrad epilogue)
+constexpr int kTrPitch = 33;
+constexpr int kTrBytes = 8 * 32 * kTrPitch * 4;
+constexpr int kSmemBytes = kStages * kStageBytes + kTrBytes + 1024 + (int)sizeof(SmemTail) + 64;
 
 struct TcArgs {
   const TcTile* tiles;
@@ -63,6 +69,8 @@ struct TcArgs {
   int32_t B, B_pad;
   uint32_t step;
   int32_t train;
+  int32_t w_shift;  // added to the weight-map index of kFwd / kDgrad tiles (weight copy)
+  int32_t update;   // kWgrad: 1 = fused AdamW, 0 = store gradients
   uint64_t seed;
   const CUtensorMap* maps;
   const float* params;
@@ -70,6 +78,7 @@ struct TcArgs {
   __nv_bfloat16* act;
   __nv_bfloat16* dz;
   float* grads;
+  AdamDev adam;
   int* err;
 };
 
@@ -182,7 +191,8 @@ __device__ __forceinline__ bool tile_live(const TcTile& t, int B_pad) { return t
 __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  SmemTail* tl = (SmemTail*)(smem + kStages * kStageBytes);
+  float* tr_all = (float*)(smem + kStages * kStageBytes);
+  SmemTail* tl = (SmemTail*)(smem + kStages * kStageBytes + kTrBytes);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
@@ -221,7 +231,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         if (!tile_live(tile, g.B_pad)) continue;
         const int K = tile.k_len ? tile.k_len : g.B_pad;
         const CUtensorMap* ma = g.maps + tile.map_a;
-        const CUtensorMap* mb = g.maps + tile.map_b;
+        const CUtensorMap* mb = g.maps + tile.map_b + (tile.kind == kWgrad ? 0 : g.w_shift);
         tensormap_acquire(ma);
         tensormap_acquire(mb);
         const int nb = (tile.n_len + 63) >> 6;
@@ -321,10 +331,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       const int r = tile.m0 + row;
       const bool row_ok = r < m_lim;
       const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + acc * kAccCols;
+      float lr = 0.f, wd_w = 0.f, wd_b = 0.f, ib1 = 1.f, ib2 = 1.f;
+      if (tile.kind == kWgrad && g.update) {
+        const float2 bc = g.adam.bias_corr[tile.member];
+        lr = md.lr;
+        wd_w = md.wd;
+        wd_b = g.adam.wd_on_bias ? md.wd : 0.f;
+        ib1 = 1.f / bc.x;
+        ib2 = 1.f / bc.y;
+      }
       // the two warps of a lane quarter take alternate 32-column chunks
       for (int c = 32 * half; c < tile.n_len; c += 64) {
         const int col0 = tile.n0 + c;
-        const int ncols = min(32, tile.n_real - col0);  // a multiple of 8 (widths are multiples of 16)
+        const int ncols = min(32, tile.n_real - col0);
         const bool live = row_ok && ncols > 0;
         // forward: bias and dropout bits do not depend on the accumulator,
         // so they are fetched / generated before the TMEM load
@@ -348,8 +367,56 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         }
         uint32_t v[32];
         tmem_ld32(taddr + c, v);
+        if (tile.kind == kWgrad) {
+          // Transpose the warp's 32 rows x 32 columns through shared memory so
+          // that lane j walks column col0 + j row by row: every parameter,
+          // moment and gradient access of the warp is one 128-byte segment.
+          float* tr = tr_all + (warp - 2) * 32 * kTrPitch;
+#pragma unroll
+          for (int j = 0; j < 32; ++j) tr[lane * kTrPitch + j] = __uint_as_float(v[j]);
+          __syncwarp();
+          const int in_pad = tile.n_real - 1;
+          const int col = col0 + lane;
+          const bool is_w = col < in_pad, is_b = col == in_pad;
+          const int rbase = tile.m0 + 32 * q;
+          const int nrows = min(32, m_lim - rbase);
+          if (is_w || is_b) {
+            const AdamDev& ad = g.adam;
+            const float wdl = is_b ? wd_b : wd_w;
+            for (int rr0 = 0; rr0 < nrows; rr0 += 8) {
+              float gv[8], pp[8], mm[8], vv[8];
+              int64_t o[8];
+#pragma unroll
+              for (int u = 0; u < 8; ++u) {
+                const int rr = min(rr0 + u, nrows - 1);
+                gv[u] = tr[rr * kTrPitch + lane];
+                o[u] = is_w ? tile.c_off + (int64_t)(rbase + rr) * tile.ldc + col : tile.aux_off + rbase + rr;
+                if (g.update) {
+                  pp[u] = ad.params[o[u]];
+                  mm[u] = ad.m[o[u]];
+                  vv[u] = ad.v[o[u]];
+                }
+              }
+#pragma unroll
+              for (int u = 0; u < 8; ++u) {
+                if (rr0 + u >= nrows) break;
+                if (g.update) {
+                  adamw_elem(pp[u], mm[u], vv[u], gv[u], lr, wdl, ad.beta1, ad.beta2, ad.eps, ib1, ib2);
+                  ad.params[o[u]] = pp[u];
+                  ad.m[o[u]] = mm[u];
+                  ad.v[o[u]] = vv[u];
+                  ad.wq_out[o[u]] = __float2bfloat16_rn(pp[u]);
+                } else {
+                  g.grads[o[u]] = gv[u];
+                }
+              }
+            }
+          }
+          __syncwarp();  // the buffer is reused by the next chunk
+          continue;
+        }
         if (!live) continue;
-        if (tile.kind == kFwd) {
+        if (tile.kind == kFwd) {  // ncols: a multiple of 8 (widths are multiples of 16)
           const float sc = g.train ? md.scale : 1.f;
           __nv_bfloat16* out = g.act + tile.c_off + (int64_t)r * tile.ldc + col0;
 #pragma unroll
@@ -371,7 +438,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
             *reinterpret_cast<uint4*>(out + 8 * s) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
           }
         } else if (tile.kind == kDgrad) {
-          const __nv_bfloat16* hm = g.act + tile.aux_off + (int64_t)r * tile.ldc + col0;
+          const __nv_bfloat16* hm = g.act + tile.aux_off + (int64_t)r * tile.ld_aux + col0;
           __nv_bfloat16* out = g.dz + tile.c_off + (int64_t)r * tile.ldc + col0;
 #pragma unroll
           for (int s = 0; s < 4; ++s) {
@@ -387,15 +454,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
               pk[e] = pack_bf16x2(x0, x1);
             }
             *reinterpret_cast<uint4*>(out + 8 * s) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-          }
-        } else {
-          float* out = g.grads + tile.c_off + (int64_t)r * tile.ldc + col0;
-#pragma unroll
-          for (int s = 0; s < 8; ++s) {
-            if (4 * s >= ncols) break;
-            *reinterpret_cast<float4*>(out + 4 * s) =
-                make_float4(__uint_as_float(v[4 * s]), __uint_as_float(v[4 * s + 1]), __uint_as_float(v[4 * s + 2]),
-                            __uint_as_float(v[4 * s + 3]));
           }
         }
       }
@@ -427,15 +485,16 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   return fn;
 }
 
-// 2-D bf16 row-major matrix [rows, cols] with 64 x 64 boxes, 128-byte swizzle.
-bool encode_map(CUtensorMap* m, const void* base, int64_t cols, int64_t rows, std::string& err) {
+// 2-D bf16 row-major matrix [rows, cols] with row pitch `ld` elements,
+// 64 x 64 boxes, 128-byte swizzle.
+bool encode_map(CUtensorMap* m, const void* base, int64_t cols, int64_t rows, int64_t ld, std::string& err) {
   auto fn = get_encode();
   if (!fn) {
     err = "cuTensorMapEncodeTiled unavailable";
     return false;
   }
   cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+  cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
   cuuint32_t box[2] = {64, 64};
   cuuint32_t es[2] = {1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
@@ -448,41 +507,55 @@ bool encode_map(CUtensorMap* m, const void* base, int64_t cols, int64_t rows, st
   return true;
 }
 
+// Balanced split of n columns into tiles of at most 256 (multiples of 16).
+void split_n(int n, std::vector<std::pair<int, int>>& out) {
+  out.clear();
+  const int nt = (int)ceil_div(n, 256);
+  const int len = (int)round_up(ceil_div(n, nt), 16);
+  for (int n0 = 0; n0 < n; n0 += len) out.push_back({n0, std::min(len, (int)round_up(n - n0, 16))});
+}
+
 }  // namespace
 
-tp_status tc_build_plan(TcPlan& plan, const tp_config& cfg, const std::vector<int32_t>& depth,
-                        const std::vector<int32_t>& width, const std::vector<uint8_t>& active,
-                        const std::vector<std::array<int64_t, kMaxDepth + 1>>& W_off,
-                        const std::vector<std::array<int64_t, kMaxDepth + 1>>& b_off,
-                        const std::vector<std::array<int64_t, kMaxDepth>>& act_off,
-                        const std::vector<std::array<int64_t, kMaxDepth>>& dz_off, int d_in_pad, int B_cap,
-                        const __nv_bfloat16* wq, const void* xb, const void* act, const void* dz,
-                        std::string& err) {
-  const int m = cfg.m;
+tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
+  const int m = lay.m;
+  const auto& depth = *lay.depth;
+  const auto& width = *lay.width;
+  const auto& active = *lay.active;
   if (plan.maps_dev == nullptr) {
-    // tensor maps: 0 = gathered batch; then per (member, layer) act, dz, W
+    // tensor maps: 0 = gathered batch [B_cap, d_in_pad + 16]; per (member,
+    // layer) act [B_cap, w + 16], dz [B_cap, w]; then the weights of copy 0,
+    // then the weights of copy 1 (w_shift apart)
     std::vector<CUtensorMap> maps;
     plan.map_act.assign((size_t)m * kMaxDepth, -1);
     plan.map_dz.assign((size_t)m * kMaxDepth, -1);
     plan.map_w.assign((size_t)m * kMaxDepth, -1);
     CUtensorMap mp;
-    if (!encode_map(&mp, xb, d_in_pad, B_cap, err)) return TP_ECUDA;
+    if (!encode_map(&mp, lay.xb, lay.ldx, lay.B_cap, lay.ldx, err)) return TP_ECUDA;
     maps.push_back(mp);
-    const __nv_bfloat16* actb = (const __nv_bfloat16*)act;
-    const __nv_bfloat16* dzb = (const __nv_bfloat16*)dz;
+    const __nv_bfloat16* actb = (const __nv_bfloat16*)lay.act;
+    const __nv_bfloat16* dzb = (const __nv_bfloat16*)lay.dz;
     for (int i = 0; i < m; ++i)
       for (int l = 0; l < depth[i]; ++l) {
-        const int w = width[i], in_pad = l == 0 ? d_in_pad : w;
-        if (!encode_map(&mp, actb + act_off[i][l], w, B_cap, err)) return TP_ECUDA;
+        const int w = width[i];
+        if (!encode_map(&mp, actb + (*lay.act_off)[i][l], w + kOnesCols, lay.B_cap, w + kOnesCols, err))
+          return TP_ECUDA;
         plan.map_act[(size_t)i * kMaxDepth + l] = (int)maps.size();
         maps.push_back(mp);
-        if (!encode_map(&mp, dzb + dz_off[i][l], w, B_cap, err)) return TP_ECUDA;
+        if (!encode_map(&mp, dzb + (*lay.dz_off)[i][l], w, lay.B_cap, w, err)) return TP_ECUDA;
         plan.map_dz[(size_t)i * kMaxDepth + l] = (int)maps.size();
         maps.push_back(mp);
-        if (!encode_map(&mp, wq + W_off[i][l], in_pad, w, err)) return TP_ECUDA;
-        plan.map_w[(size_t)i * kMaxDepth + l] = (int)maps.size();
-        maps.push_back(mp);
       }
+    const int w_base = (int)maps.size();
+    for (int copy = 0; copy < 2; ++copy)
+      for (int i = 0; i < m; ++i)
+        for (int l = 0; l < depth[i]; ++l) {
+          const int w = width[i], in_pad = l == 0 ? lay.d_in_pad : w;
+          if (!encode_map(&mp, lay.wq[copy] + (*lay.W_off)[i][l], in_pad, w, in_pad, err)) return TP_ECUDA;
+          if (copy == 0) plan.map_w[(size_t)i * kMaxDepth + l] = (int)maps.size();
+          maps.push_back(mp);
+        }
+    plan.w_shift = ((int)maps.size() - w_base) / 2;
     plan.n_maps = (int)maps.size();
     if (cudaMalloc(&plan.maps_dev, sizeof(CUtensorMap) * maps.size()) != cudaSuccess) {
       err = "cudaMalloc(tensor maps) failed";
@@ -512,30 +585,33 @@ tp_status tc_build_plan(TcPlan& plan, const tp_config& cfg, const std::vector<in
   std::vector<TcTile> all;
   plan.fwd_rng.assign(Lmax, {0, 0});
   plan.bwd_rng.assign(Lmax, {0, 0});
-  auto cost = [&](const TcTile& t) { return (int64_t)(t.k_len ? t.k_len : B_cap) * t.n_len; };
+  auto cost = [&](const TcTile& t) { return (int64_t)(t.k_len ? t.k_len : lay.B_cap) * t.n_len; };
   auto sorted_append = [&](std::vector<TcTile>& v) {
     std::stable_sort(v.begin(), v.end(), [&](const TcTile& a, const TcTile& b) { return cost(a) > cost(b); });
     const int base = (int)all.size();
     all.insert(all.end(), v.begin(), v.end());
     return std::make_pair(base, (int)v.size());
   };
+  std::vector<std::pair<int, int>> ns;
   for (int l = 0; l < Lmax; ++l) {
     std::vector<TcTile> v;
     for (int i = 0; i < m; ++i) {
       if (!active[i] || depth[i] <= l) continue;
       const int w = width[i];
-      for (int m0 = 0; m0 < B_cap; m0 += 128)
-        for (int n0 = 0; n0 < w; n0 += 256) {
+      split_n(w, ns);
+      for (int m0 = 0; m0 < lay.B_cap; m0 += 128)
+        for (auto& nn : ns) {
           TcTile t{};
           t.kind = kFwd; t.member = i; t.layer = l;
-          t.m0 = m0; t.n0 = n0; t.n_len = std::min(256, w - n0);
+          t.m0 = m0; t.n0 = nn.first; t.n_len = nn.second;
           t.m_real = 0; t.n_real = w;
-          t.k_len = l == 0 ? d_in_pad : w;
+          t.k_len = l == 0 ? lay.d_in_pad : w;
           t.map_a = l == 0 ? 0 : plan.map_act[(size_t)i * kMaxDepth + l - 1];
           t.map_b = plan.map_w[(size_t)i * kMaxDepth + l];
-          t.ldc = w;
-          t.c_off = act_off[i][l];
-          t.aux_off = b_off[i][l];
+          t.ldc = w + kOnesCols;
+          t.ld_aux = 0;
+          t.c_off = (*lay.act_off)[i][l];
+          t.aux_off = (*lay.b_off)[i][l];
           v.push_back(t);
         }
     }
@@ -545,34 +621,39 @@ tp_status tc_build_plan(TcPlan& plan, const tp_config& cfg, const std::vector<in
     std::vector<TcTile> v;
     for (int i = 0; i < m; ++i) {
       if (!active[i] || depth[i] <= l) continue;
-      const int w = width[i], in_pad = l == 0 ? d_in_pad : w;
-      if (l > 0)
-        for (int m0 = 0; m0 < B_cap; m0 += 128)
-          for (int n0 = 0; n0 < w; n0 += 256) {
+      const int w = width[i], in_pad = l == 0 ? lay.d_in_pad : w;
+      if (l > 0) {
+        split_n(w, ns);
+        for (int m0 = 0; m0 < lay.B_cap; m0 += 128)
+          for (auto& nn : ns) {
             TcTile t{};
             t.kind = kDgrad; t.member = i; t.layer = l;
-            t.m0 = m0; t.n0 = n0; t.n_len = std::min(256, w - n0);
+            t.m0 = m0; t.n0 = nn.first; t.n_len = nn.second;
             t.m_real = 0; t.n_real = w;
             t.k_len = w;
             t.map_a = plan.map_dz[(size_t)i * kMaxDepth + l];
             t.map_b = plan.map_w[(size_t)i * kMaxDepth + l];
             t.ldc = w;
-            t.c_off = dz_off[i][l - 1];
-            t.aux_off = act_off[i][l - 1];
+            t.ld_aux = w + kOnesCols;
+            t.c_off = (*lay.dz_off)[i][l - 1];
+            t.aux_off = (*lay.act_off)[i][l - 1];
             v.push_back(t);
           }
+      }
+      split_n(in_pad + 1, ns);  // weight columns plus the bias column
       for (int m0 = 0; m0 < w; m0 += 128)
-        for (int n0 = 0; n0 < in_pad; n0 += 256) {
+        for (auto& nn : ns) {
           TcTile t{};
           t.kind = kWgrad; t.member = i; t.layer = l;
-          t.m0 = m0; t.n0 = n0; t.n_len = (int)round_up(std::min(256, in_pad - n0), 16);
-          t.m_real = w; t.n_real = in_pad;
+          t.m0 = m0; t.n0 = nn.first; t.n_len = nn.second;
+          t.m_real = w; t.n_real = in_pad + 1;
           t.k_len = 0;
           t.map_a = plan.map_dz[(size_t)i * kMaxDepth + l];
           t.map_b = l == 0 ? 0 : plan.map_act[(size_t)i * kMaxDepth + l - 1];
           t.ldc = in_pad;
-          t.c_off = W_off[i][l];
-          t.aux_off = 0;
+          t.ld_aux = 0;
+          t.c_off = (*lay.W_off)[i][l];
+          t.aux_off = (*lay.b_off)[i][l];
           v.push_back(t);
         }
     }
@@ -595,24 +676,13 @@ tp_status tc_build_plan(TcPlan& plan, const tp_config& cfg, const std::vector<in
   return TP_OK;
 }
 
-static tp_status launch(TcPlan& plan, cudaStream_t st, const std::pair<int, int>& rng, int B, int B_pad,
-                        uint32_t step, int train, uint64_t seed, const float* params, const MemberDev* mem,
-                        void* act, void* dz, float* grads, std::string& err) {
+static tp_status launch(TcPlan& plan, cudaStream_t st, const std::pair<int, int>& rng, const TcArgs& base,
+                        std::string& err) {
   if (rng.second <= 0) return TP_OK;
-  TcArgs a;
+  TcArgs a = base;
   a.tiles = plan.tiles_dev + rng.first;
   a.n_tiles = rng.second;
-  a.B = B;
-  a.B_pad = B_pad;
-  a.step = step;
-  a.train = train;
-  a.seed = seed;
   a.maps = plan.maps_dev;
-  a.params = params;
-  a.mem = mem;
-  a.act = (__nv_bfloat16*)act;
-  a.dz = (__nv_bfloat16*)dz;
-  a.grads = grads;
   a.err = plan.err_dev;
   const int grid = std::max(1, std::min(rng.second, plan.n_sm));
   k_tc_gemm<<<grid, kThreads, kSmemBytes, st>>>(a);
@@ -624,14 +694,36 @@ static tp_status launch(TcPlan& plan, cudaStream_t st, const std::pair<int, int>
   return TP_OK;
 }
 
-tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, uint32_t step, int train,
-                     uint64_t seed, const float* params, const MemberDev* mem, void* act, std::string& err) {
-  return launch(plan, st, plan.fwd_rng[layer], B, B_pad, step, train, seed, params, mem, act, nullptr, nullptr, err);
+tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, int wcur, uint32_t step,
+                     int train, uint64_t seed, const float* params, const MemberDev* mem, void* act,
+                     std::string& err) {
+  TcArgs a{};
+  a.B = B;
+  a.B_pad = B_pad;
+  a.step = step;
+  a.train = train;
+  a.w_shift = wcur ? plan.w_shift : 0;
+  a.update = 0;
+  a.seed = seed;
+  a.params = params;
+  a.mem = mem;
+  a.act = (__nv_bfloat16*)act;
+  return launch(plan, st, plan.fwd_rng[layer], a, err);
 }
 
-tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, float* grads,
-                     const MemberDev* mem, void* act, void* dz, std::string& err) {
-  return launch(plan, st, plan.bwd_rng[layer], B, B_pad, 0, 0, 0, nullptr, mem, act, dz, grads, err);
+tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, int wcur, const MemberDev* mem,
+                     void* act, void* dz, float* grads, int update, const AdamDev& adam, std::string& err) {
+  TcArgs a{};
+  a.B = B;
+  a.B_pad = B_pad;
+  a.w_shift = wcur ? plan.w_shift : 0;
+  a.update = update;
+  a.mem = mem;
+  a.act = (__nv_bfloat16*)act;
+  a.dz = (__nv_bfloat16*)dz;
+  a.grads = grads;
+  a.adam = adam;
+  return launch(plan, st, plan.bwd_rng[layer], a, err);
 }
 
 tp_status tc_check(TcPlan& plan, cudaStream_t st, std::string& err) {

@@ -15,18 +15,21 @@
 namespace tp {
 
 // One 128 x n_len output tile of one member's product.
-//   kFwd   C[b, j]  = sum_k H[b, k] W[j, k]       A = H (K-major), B = W (K-major)
-//   kDgrad C[b, k]  = sum_j dZ[b, j] W[j, k]      A = dZ (K-major), B = W (MN-major)
-//   kWgrad C[j, k]  = sum_b dZ[b, j] H[b, k]      A = dZ (MN-major), B = H (MN-major)
+//   kFwd   C[b, j]  = sum_k H[b, k] W[j, k]         A = H (K-major), B = W (K-major)
+//   kDgrad C[b, k]  = sum_j dZ[b, j] W[j, k]        A = dZ (K-major), B = W (MN-major)
+//   kWgrad C[j, k]  = sum_b dZ[b, j] [H | 1][b, k]  A = dZ (MN-major), B = [H | 1] (MN-major);
+//          columns k < in_pad are dW, column in_pad is db
 struct TcTile {
   int32_t kind, member, layer;
   int32_t m0, n0, n_len;   // tile origin; n_len = MMA N (multiple of 16, <= 256)
-  int32_t m_real, n_real;  // output bounds (m_real 0: the step's padded batch)
+  int32_t m_real, n_real;  // output bounds (m_real 0: the step's padded batch);
+                           // kWgrad: n_real = in_pad + 1 (the bias column)
   int32_t k_len;           // reduction length (0: the step's padded batch)
-  int32_t map_a, map_b;    // indices into the tensor-map table
-  int32_t ldc;
-  int64_t c_off;           // output offset: act (kFwd), dz (kDgrad), grads (kWgrad)
-  int64_t aux_off;         // kFwd: bias offset in params; kDgrad: H_l offset in act (mask)
+  int32_t map_a, map_b;    // indices into the tensor-map table (weight maps of copy 0)
+  int32_t ldc, ld_aux, _pad;
+  int64_t c_off;           // output: act (kFwd), dz (kDgrad), weight offset in the arena (kWgrad)
+  int64_t aux_off;         // kFwd: bias offset in params; kDgrad: H_l offset in act (mask);
+                           // kWgrad: bias offset in the arena
 };
 
 struct TcPlan {
@@ -34,26 +37,39 @@ struct TcPlan {
   int n_sm = 0;
   CUtensorMap* maps_dev = nullptr;
   int n_maps = 0;
+  int w_shift = 0;         // index distance from a weight map of copy 0 to copy 1
   TcTile* tiles_dev = nullptr;
   int cap_tiles = 0;
   std::vector<std::pair<int, int>> fwd_rng, bwd_rng;  // tile ranges per depth index
   int* err_dev = nullptr;  // device error word (bounded waits that gave up)
-  // inputs used at build time
   std::vector<int> map_act, map_dz, map_w;  // per (member * kMaxDepth + layer)
 };
 
-tp_status tc_build_plan(TcPlan& plan, const tp_config& cfg, const std::vector<int32_t>& depth,
-                        const std::vector<int32_t>& width, const std::vector<uint8_t>& active,
-                        const std::vector<std::array<int64_t, kMaxDepth + 1>>& W_off,
-                        const std::vector<std::array<int64_t, kMaxDepth + 1>>& b_off,
-                        const std::vector<std::array<int64_t, kMaxDepth>>& act_off,
-                        const std::vector<std::array<int64_t, kMaxDepth>>& dz_off, int d_in_pad, int B_cap,
-                        const __nv_bfloat16* wq, const void* xb, const void* act, const void* dz,
-                        std::string& err);
-tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, uint32_t step, int train,
-                     uint64_t seed, const float* params, const MemberDev* mem, void* act, std::string& err);
-tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, float* grads,
-                     const MemberDev* mem, void* act, void* dz, std::string& err);
+struct TcLayout {          // what the plan needs to know about the pack's arenas
+  const std::vector<int32_t>* depth;
+  const std::vector<int32_t>* width;
+  const std::vector<uint8_t>* active;
+  const std::vector<std::array<int64_t, kMaxDepth + 1>>* W_off;
+  const std::vector<std::array<int64_t, kMaxDepth + 1>>* b_off;
+  const std::vector<std::array<int64_t, kMaxDepth>>* act_off;
+  const std::vector<std::array<int64_t, kMaxDepth>>* dz_off;
+  int m, d_in_pad, ldx, B_cap;
+  const __nv_bfloat16* wq[2];
+  const void* xb;
+  const void* act;
+  const void* dz;
+};
+
+tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err);
+// Forward products of hidden layer `layer`, reading weight copy `wcur`.
+tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, int wcur, uint32_t step,
+                     int train, uint64_t seed, const float* params, const MemberDev* mem, void* act,
+                     std::string& err);
+// Backward products (dgrad + wgrad) of hidden layer `layer`.  update = 0: the
+// weight and bias gradients are stored in `grads`; update = 1: AdamW is
+// applied in the epilogue (adam.wq_out = the other weight copy).
+tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, int wcur, const MemberDev* mem,
+                     void* act, void* dz, float* grads, int update, const AdamDev& adam, std::string& err);
 // Reads and clears the device error word (synchronises the stream).
 tp_status tc_check(TcPlan& plan, cudaStream_t st, std::string& err);
 void tc_free_plan(TcPlan& plan);

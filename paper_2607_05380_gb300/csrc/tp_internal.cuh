@@ -6,15 +6,19 @@
 //       [out, in_pad] row-major then the bias [out]; every block starts on a
 //       32-element boundary.  Layer 0 has in_pad = round_up(d_in, 8) columns
 //       (the pad columns stay exactly zero); other layers in_pad = in.
-//   wq[2]  : bf16 copies of the whole param arena (same offsets), written by
-//       AdamW; the matrix products read them (bf16 mode).  Two copies so a
-//       step can read one while AdamW of the same step writes the other.
-//   xb     : the gathered batch [B_cap, d_in_pad] (T).
-//   act    : H_{l+1} = output of hidden layer l of member i, [B_cap, w_i] (T).
+//   wq[2]  : bf16 copies of the whole param arena (same offsets).  A step reads
+//       wq[cur] in its matrix products and its fused AdamW writes wq[cur ^ 1],
+//       so the step's dgrad can still read the weights its wgrad is updating.
+//   xb     : the gathered batch [B_cap, ldx] (T), ldx = d_in_pad + 16.
+//   act    : H_{l+1} = output of hidden layer l of member i, [B_cap, ldh_i] (T),
+//            ldh_i = w_i + 16.
 //   dz     : dL/dZ_l of hidden layer l of member i, [B_cap, w_i] (T).
+// Column in_pad of xb and column w of every act matrix hold 1 (the next 15
+// columns 0): the weight-gradient product dZ^T [H | 1] then yields the bias
+// gradient dZ^T 1 as its extra output column.
 // T = __nv_bfloat16 in bf16 mode, float in fp32 mode.  Batches are padded to
 // B_pad = round_up(B, 128) rows; padded rows carry zero loss gradient, so they
-// add nothing to weight gradients.
+// add nothing to weight or bias gradients.
 #pragma once
 
 #include <cuda_bf16.h>
@@ -28,21 +32,25 @@ constexpr int kMaxDout = 32;
 constexpr int kRowTile = 128;   // batch rows per tile; B_pad is a multiple of this
 constexpr int kHeadRows = 32;   // batch rows per head-kernel block
 constexpr int kSegAlign = 32;   // elements
+constexpr int kOnesCols = 16;   // the ones column plus zero padding to 16 columns
 
 enum GemmKind : int32_t { kFwd = 0, kDgrad = 1, kWgrad = 2 };
 enum Src : int32_t { kSrcXb = 0, kSrcAct = 1, kSrcDz = 2, kSrcWq = 3 };
 
-// One matrix product of one member and layer.  Output C[r, c] = sum_k A(r, k) B(c, k).
-//   kFwd   : A = H_l [B, in] (act or xb), B = W_l [w, in] (wq);  C = H_{l+1} [B, w]
-//   kDgrad : A = dZ_l [B, w] (dz), B(c, k) = W_l[k, c];          C = dZ_{l-1} [B, in]
-//   kWgrad : A(r, k) = dZ_l[k, r], B(c, k) = H_l[k, c];          C = dW_l [w, in_pad] (grads)
+// One matrix product of one member and layer (CUDA-core path).
+// Output C[r, c] = sum_k A(r, k) B(c, k).
+//   kFwd   : A = H_l [B, in] (act or xb), B = W_l [w, in];  C = H_{l+1} [B, w]
+//   kDgrad : A = dZ_l [B, w], B(c, k) = W_l[k, c];          C = dZ_{l-1} [B, in]
+//   kWgrad : A(r, k) = dZ_l[k, r], B(c, k) = [H_l | 1][k, c]; C = dW_l [w, in_pad],
+//            column in_pad = db_l
 struct GemmProblem {
-  int32_t kind, member, layer, _pad0;
+  int32_t kind, member, layer, ld_aux;
   int32_t M, N, K;        // M == 0 / K == 0: the step's B_pad rows
   int32_t a_src, b_src;
   int32_t lda, ldb, ldc;  // row pitches in elements
   int64_t a_off, b_off, c_off;
-  int64_t aux_off;        // kFwd: bias offset in params; kDgrad: offset of H_l (mask source) in act
+  int64_t aux_off;        // kFwd: bias offset in params; kDgrad: offset of H_l (mask) in act;
+                          // kWgrad: bias offset in grads
   int64_t _pad1;
 };
 
@@ -72,25 +80,49 @@ struct Chunk {            // element-wise work unit (init, AdamW): never crosses
   int32_t len, seg;
 };
 
-struct BiasJob {          // bias gradient: column sums of dZ_l over the batch rows
-  int64_t dz_off, b_off;  // dZ_l in dz arena, bias in grads arena
-  int32_t w, c0;          // pitch / width of dZ_l, first column of this job
-};
-
-struct HeadJob {          // head forward / loss / backward of one member on one 128-row block
+struct HeadJob {          // head forward / loss / backward of one member on one 32-row block
   int32_t member, blk;
-  int64_t h_off;          // H_L in act (or xb never: L >= 1)
-  int64_t dz_off;         // dZ_{L-1} in dz
+  int32_t h_ld, _pad;     // pitch of H_L
+  int64_t h_off;          // H_L in act
+  int64_t dz_off;         // dZ_{L-1} in dz (pitch w)
   int64_t w_off, b_off;   // head weight / bias offsets in params
-  int64_t part_off;       // partial dW_h of this block: [d_out, w] + [d_out] db
+  int64_t part_off;       // partial dW_h of this block: [d_out, w] then [d_out] db
 };
 
 struct HeadReduceJob {
   int32_t member, n_blk;
-  int64_t part_off;       // first block's partial; blocks are consecutive, stride (d_out + 1) * w... see kernel
-  int64_t gw_off, gb_off; // head grads in grads arena
+  int64_t part_off;       // first block's partial; blocks follow at part_stride[member]
+  int64_t gw_off, gb_off; // head weight / bias offsets (params, grads, m, v share them)
   int32_t w, _pad;
 };
+
+struct OnesJob {          // column `col` of rows 0..rows-1 of a matrix with pitch `ld` := 1
+  int64_t off;
+  int32_t ld, col, rows;
+  int32_t arena;          // 0: xb, 1: act
+};
+
+// What a fused AdamW update needs besides the element itself.
+struct AdamDev {
+  float* params;
+  float* m;
+  float* v;
+  __nv_bfloat16* wq_out;  // bf16 copy to write (NULL: none)
+  const float2* bias_corr;  // per member (1 - beta1^t, 1 - beta2^t) of the step
+  const MemberDev* mem;
+  float beta1, beta2, eps;
+  int32_t wd_on_bias;
+};
+
+// AdamW on one element (PyTorch semantics): decoupled decay, moments, bias-
+// corrected step.  ib1 = 1 / (1 - beta1^t), ib2 = 1 / (1 - beta2^t).
+__device__ __forceinline__ void adamw_elem(float& p, float& m, float& v, float g, float lr, float wd, float b1,
+                                           float b2, float eps, float ib1, float ib2) {
+  p = p - lr * wd * p;
+  m = b1 * m + (1.f - b1) * g;
+  v = b2 * v + (1.f - b2) * g * g;
+  p = p - lr * (m * ib1) / (sqrtf(v * ib2) + eps);
+}
 
 // ---------------------------------------------------------------- Philox4x32-10
 // Salmon, Moraes, Dror, Shaw (SC'11): ten rounds of
@@ -126,7 +158,6 @@ __device__ __forceinline__ uint32_t keep_bits4(uint64_t seed, uint32_t member, u
 // ---------------------------------------------------------------- element types
 template <typename T> struct Elem;
 template <> struct Elem<float> {
-  static __device__ __forceinline__ float load(const float* p) { return *p; }
   static __device__ __forceinline__ float to_f(float v) { return v; }
   static __device__ __forceinline__ float from_f(float v) { return v; }
 };

@@ -58,9 +58,9 @@ def make_data(task, n, d_in, d_out, seed):
     return X, y
 
 
-def pair(tp, task, d_in, d_out, hp, prec, max_batch, seed=2):
+def pair(tp, task, d_in, d_out, hp, prec, max_batch, seed=2, fuse=False):
     pk = tp.Pack(d_in, d_out, task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
-                 max_batch=max_batch, seed=seed, precision=prec)
+                 max_batch=max_batch, seed=seed, precision=prec, fuse_optimizer=fuse)
     orc = oracle.OraclePack(d_in, d_out, task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
                             seed=seed, bf16_storage=(prec == "bf16"))
     return pk, orc
@@ -171,12 +171,14 @@ def test_one_step_logits_losses_grads(tp, prec, task, d_out, B):
     assert not problems, problems
 
 
-@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+@pytest.mark.parametrize("prec,fuse", [("fp32", False), ("bf16", False), ("bf16", True)])
 @pytest.mark.parametrize("task,d_out", [("binary", 1), ("multiclass", 5), ("regression", 1)])
-def test_ten_steps_params(tp, prec, task, d_out):
+def test_ten_steps_params(tp, prec, fuse, task, d_out):
+    """Ten AdamW steps; in bf16 mode with the optimizer both as a separate
+    pass and fused into the weight-gradient epilogue."""
     d_in, m, B = 24, 8, 192
     hp = random_pack(m, d_in, d_out, seed=20 + d_out, width=(16, 128, 16), depth=(1, 3))
-    pk, orc = pair(tp, task, d_in, d_out, hp, prec, 256)
+    pk, orc = pair(tp, task, d_in, d_out, hp, prec, 256, fuse=fuse)
     X, y = make_data(task, 600, d_in, d_out, 3)
     Xd, yd = to_dev(X, y)
     rng = np.random.default_rng(5)
@@ -223,9 +225,10 @@ def test_predict(tp, prec, task, d_out):
         assert rel_err(out[i], ref[i]) <= TOL[prec], i
 
 
-def test_inactive_members(tp):
+@pytest.mark.parametrize("prec,fuse", [("fp32", False), ("bf16", False), ("bf16", True)])
+def test_inactive_members(tp, prec, fuse):
     hp = random_pack(4, 9, 1, seed=7)
-    pk, orc = pair(tp, "regression", 9, 1, hp, "fp32", 128)
+    pk, orc = pair(tp, "regression", 9, 1, hp, prec, 128, fuse=fuse)
     X, y = make_data("regression", 200, 9, 1, 5)
     Xd, yd = to_dev(X, y)
     idx = np.arange(128, dtype=np.int32)
@@ -241,14 +244,19 @@ def test_inactive_members(tp):
     lg = loss.cpu().numpy()
     assert np.isnan(lg[2]) and np.isnan(lo[2])
     np.testing.assert_array_equal(pk.get_params(2, 0)[0], frozen[0])
+    tol = TOL["fp32"] * 10 if prec == "fp32" else TOL["bf16"]
     for i in (0, 1, 3):
         for l in range(int(hp["depth"][i]) + 1):
-            assert rel_err(pk.get_params(i, l)[0], orc.get_params(i, l)[0]) <= TOL["fp32"] * 10
+            assert rel_err(pk.get_params(i, l)[0], orc.get_params(i, l)[0]) <= tol
     pk.set_active([1, 1, 1, 1])
     orc.set_active([1, 1, 1, 1])
-    pk.train_step(Xd, idxd, yd, 2, loss)
-    orc.train_step(X, idx, y, 2)
-    assert orc.member_steps(2) == 2
+    for step in (2, 3, 4):   # the re-activated member must train from its own latest weights
+        pk.train_step(Xd, idxd, yd, step, loss)
+        orc.train_step(X, idx, y, step)
+    assert orc.member_steps(2) == 4
+    for i in range(4):
+        for l in range(int(hp["depth"][i]) + 1):
+            assert rel_err(pk.get_params(i, l)[0], orc.get_params(i, l)[0]) <= tol, (i, l)
 
 
 @pytest.mark.parametrize("task,score,d_out", [("multiclass", "loss", 10), ("multiclass", "accuracy", 10),
