@@ -181,6 +181,9 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--members", type=int, default=0,
+                    help="train only the first N members of the workload (profiling small cases)")
+    ap.add_argument("--fuse-optimizer", action="store_true", help="AdamW inside the weight-gradient epilogue")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -189,6 +192,9 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     wl = WORKLOADS[args.workload]
+    if args.members > 0:
+        import dataclasses
+        wl = dataclasses.replace(wl, m=min(wl.m, args.members))
 
     if args.impl == "reference":
         run_reference(args, wl, rank)
@@ -205,7 +211,7 @@ def main():
     tp.load_library()
 
     B = wl.batch
-    hp = sample_hparams(wl, seed=SEED_HP)
+    hp = {k: v[:wl.m] for k, v in sample_hparams(WORKLOADS[args.workload], seed=SEED_HP).items()}
     d = make_data(wl, device=dev)
     X, y = d["X_train"], d["y_train"]
     n_train = X.shape[0]
@@ -217,7 +223,8 @@ def main():
 
     stream = torch.cuda.current_stream()
     pack = tp.Pack(wl.d_in, wl.d_out, wl.task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
-                   max_batch=B, seed=SEED_INIT, precision=args.precision, stream=stream)
+                   max_batch=B, seed=SEED_INIT, precision=args.precision, stream=stream,
+                   fuse_optimizer=args.fuse_optimizer)
     loss = torch.zeros(wl.m, dtype=torch.float32, device=dev)
 
     for s in range(args.warmup):

@@ -225,7 +225,9 @@ __device__ __forceinline__ float row_loss(int task, int d_out, const float (&z)[
 // block's partial head-weight gradient over its 32 rows, in row order.
 template <typename T, int DO>
 __global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
-  constexpr int R = DO <= 16 ? 4 : 1;
+  // rows per head-weight load: 4 for the one-logit head; 1 for class heads,
+  // whose per-row state (DO logits and dlogits) would otherwise cost occupancy
+  constexpr int R = DO == 1 ? 4 : (DO <= 4 ? 2 : 1);
   constexpr int RW = kHeadRows / 8;  // rows per warp
   const HeadJob jb = g.jobs[blockIdx.x];
   const int r0 = jb.blk * kHeadRows;
@@ -318,7 +320,7 @@ __global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
   __syncthreads();
   // partial head gradients of this block: per group of G columns, all
   // classes, rows in increasing order
-  constexpr int G = DO == 1 ? 8 : (DO <= 16 ? 4 : 2);
+  constexpr int G = DO <= 2 ? 8 : (DO <= 16 ? 4 : 2);
   float* part = g.head_part + jb.part_off;
   for (int gi = threadIdx.x; gi < w / G; gi += blockDim.x) {
     float a[DO][G];
@@ -364,17 +366,19 @@ __global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
 
 // Sum the per-block head partials (fixed order) into the head gradients and
 // the per-member mean loss; in update mode apply the member's AdamW to the
-// head parameters directly (the gradients are not stored).  One block per
-// member; inactive members report NaN.
+// head parameters directly (the gradients are not stored).  Grid: member x
+// chunks of 256 head parameters; inactive members report NaN.
 __global__ void k_head_reduce(HeadReduceArgs g) {
   const int i = blockIdx.x;
   const HeadReduceJob jb = g.jobs[i];
   const int n_blk = g.B_pad / kHeadRows;
   if (!g.active[i]) {
-    if (threadIdx.x == 0 && g.loss_out) g.loss_out[i] = __int_as_float(0x7fc00000);
+    if (blockIdx.y == 0 && threadIdx.x == 0 && g.loss_out) g.loss_out[i] = __int_as_float(0x7fc00000);
     return;
   }
   const int w = jb.w, d_out = g.d_out;
+  const int e0 = blockIdx.y * blockDim.x;
+  if (e0 >= d_out * w + d_out) return;
   const int64_t stride = g.part_stride[i];
   float lr = 0.f, wdw = 0.f, wdb = 0.f, ib1 = 1.f, ib2 = 1.f;
   if (g.update) {
@@ -386,7 +390,7 @@ __global__ void k_head_reduce(HeadReduceArgs g) {
     ib1 = 1.f / bc.x;
     ib2 = 1.f / bc.y;
   }
-  for (int e = threadIdx.x; e < d_out * w + d_out; e += blockDim.x) {
+  for (int e = e0 + threadIdx.x; e < min(e0 + (int)blockDim.x, d_out * w + d_out); e += blockDim.x) {
     float s = 0.f;
     for (int b = 0; b < n_blk; ++b) s += g.head_part[jb.part_off + b * stride + e];
     const bool is_b = e >= d_out * w;
@@ -402,7 +406,7 @@ __global__ void k_head_reduce(HeadReduceArgs g) {
       g.grads[o] = s;
     }
   }
-  if (threadIdx.x == 0) {
+  if (blockIdx.y == 0 && threadIdx.x == 0) {
     float s = 0.f;
     for (int b = 0; b < n_blk; ++b) s += g.loss_part[(int64_t)i * g.n_blk_cap + b];
     const float loss = s / (float)g.B;
@@ -597,13 +601,18 @@ void launch_gemm_simt(cudaStream_t st, const GemmArgs<T>& g, int tile_base, int 
 template <typename T>
 void launch_head(cudaStream_t st, const HeadArgs<T>& g, int n_jobs) {
   if (n_jobs <= 0) return;
+  // class-count buckets: the loops over classes are unrolled to the bucket size
   if (g.d_out == 1) k_head<T, 1><<<n_jobs, 256, 0, st>>>(g);
+  else if (g.d_out <= 2) k_head<T, 2><<<n_jobs, 256, 0, st>>>(g);
+  else if (g.d_out <= 4) k_head<T, 4><<<n_jobs, 256, 0, st>>>(g);
+  else if (g.d_out <= 8) k_head<T, 8><<<n_jobs, 256, 0, st>>>(g);
+  else if (g.d_out <= 10) k_head<T, 10><<<n_jobs, 256, 0, st>>>(g);
   else if (g.d_out <= 16) k_head<T, 16><<<n_jobs, 256, 0, st>>>(g);
   else k_head<T, kMaxDout><<<n_jobs, 256, 0, st>>>(g);
 }
 
-void launch_head_reduce(cudaStream_t st, const HeadReduceArgs& g, int m) {
-  k_head_reduce<<<m, 256, 0, st>>>(g);
+void launch_head_reduce(cudaStream_t st, const HeadReduceArgs& g, int m, int max_elems) {
+  k_head_reduce<<<dim3(m, (unsigned)ceil_div(max_elems, 256)), 256, 0, st>>>(g);
 }
 
 void launch_adamw(cudaStream_t st, const AdamArgs& g, int n_chunks) {
@@ -622,6 +631,8 @@ template <typename T>
 void launch_predict_head(cudaStream_t st, const PredictHeadArgs<T>& g, int n_jobs) {
   if (n_jobs <= 0) return;
   if (g.d_out == 1) k_predict_head<T, 1><<<n_jobs, 256, 0, st>>>(g);
+  else if (g.d_out <= 4) k_predict_head<T, 4><<<n_jobs, 256, 0, st>>>(g);
+  else if (g.d_out <= 10) k_predict_head<T, 10><<<n_jobs, 256, 0, st>>>(g);
   else if (g.d_out <= 16) k_predict_head<T, 16><<<n_jobs, 256, 0, st>>>(g);
   else k_predict_head<T, kMaxDout><<<n_jobs, 256, 0, st>>>(g);
 }

@@ -98,7 +98,8 @@ template <typename T>
 void launch_gemm_simt(cudaStream_t st, const GemmArgs<T>& g, int tile_base, int n_tiles);
 template <typename T>
 void launch_head(cudaStream_t st, const HeadArgs<T>& g, int n_jobs);
-void launch_head_reduce(cudaStream_t st, const HeadReduceArgs& g, int m);
+// grid: m members x ceil(max_elems / 256) chunks (max_elems = max_i d_out (w_i + 1))
+void launch_head_reduce(cudaStream_t st, const HeadReduceArgs& g, int m, int max_elems);
 void launch_adamw(cudaStream_t st, const AdamArgs& g, int n_chunks);
 void launch_init(cudaStream_t st, const InitArgs& g, int n_chunks);
 void launch_refresh_wq(cudaStream_t st, const float* p, __nv_bfloat16* wq0, __nv_bfloat16* wq1, int64_t n);

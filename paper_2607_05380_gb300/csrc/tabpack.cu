@@ -557,7 +557,9 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
   rg.n_blk_cap = h->n_blk_cap;
   rg.update = fused ? 1 : 0;
   rg.adam = adam_dev(h, wq_next);
-  launch_head_reduce(h->st, rg, h->cfg.m);
+  int w_max = 0;
+  for (int w : h->width) w_max = std::max(w_max, w);
+  launch_head_reduce(h->st, rg, h->cfg.m, h->cfg.d_out * (w_max + 1));
   TP_LAUNCHED(h);
   h->launches++;
   prof_end(h, slot, 2, TP_PH_HEAD);
