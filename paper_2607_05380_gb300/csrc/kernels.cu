@@ -11,11 +11,15 @@ namespace tp {
 // Block 0 also advances the step count of every active member and stores the
 // AdamW bias corrections 1 - beta^t of the new step (when `advance`).
 template <typename T>
-__global__ void k_gather(const float* __restrict__ X, const int32_t* __restrict__ idx, int32_t B,
-                         int32_t B_pad, int32_t d_in, int32_t d_in_pad, int32_t ldx, T* __restrict__ xb,
+__global__ void k_gather(const float* __restrict__ X, const int32_t* __restrict__ idx, const StepDyn* dyn,
+                         int32_t B, int32_t B_pad, int32_t d_in, int32_t d_in_pad, int32_t ldx, T* __restrict__ xb,
                          int32_t advance, int32_t* __restrict__ t_dev, float2* __restrict__ bias_corr,
                          const int32_t* __restrict__ active_ids, int32_t n_active, float beta1,
                          float beta2) {
+  if (dyn) {
+    X = dyn->X;
+    idx = dyn->idx;
+  }
   if (advance && blockIdx.x == 0) {
     for (int a = threadIdx.x; a < n_active; a += blockDim.x) {
       int i = active_ids[a];
@@ -58,6 +62,7 @@ __global__ void __launch_bounds__(256) k_gemm_simt(GemmArgs<T> g, int32_t tile_b
   const int N = P.N;
   const int K = P.K ? P.K : g.B_pad;
   if (t.m0 >= M) return;
+  const uint32_t step = g.dyn ? g.dyn->step : g.step;
   const T* bases[4] = {g.xb, g.act, g.dz, g.wq};
   const T* A = bases[P.a_src] + P.a_off;
   const T* Bm = bases[P.b_src] + P.b_off;
@@ -117,7 +122,7 @@ __global__ void __launch_bounds__(256) k_gemm_simt(GemmArgs<T> g, int32_t tile_b
     const int r = t.m0 + ty + 16 * i;
     if (r >= M) continue;
     if (P.kind == kFwd) {  // N = w, a multiple of 16
-      uint32_t keep = g.train ? keep_bits4(g.seed, (uint32_t)P.member, (uint32_t)P.layer, g.step,
+      uint32_t keep = g.train ? keep_bits4(g.seed, (uint32_t)P.member, (uint32_t)P.layer, step,
                                            (uint32_t)r, (uint32_t)(c0 >> 2), md.drop_T)
                               : 0xFu;
       const float sc = g.train ? md.scale : 1.f;
@@ -277,8 +282,10 @@ __global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
 #pragma unroll
       for (int c = 0; c < DO; ++c) dl[q][c] = 0.f;
       if (r < g.B) {
-        const int64_t row = g.idx ? (int64_t)g.idx[r] : (int64_t)r;
-        loss = row_loss<DO>(g.task, d_out, acc[q], g.y, row, invB, dl[q]);
+        const int32_t* idx = g.dyn ? g.dyn->idx : g.idx;
+        const void* yv = g.dyn ? g.dyn->y : g.y;
+        const int64_t row = idx ? (int64_t)idx[r] : (int64_t)r;
+        loss = row_loss<DO>(g.task, d_out, acc[q], yv, row, invB, dl[q]);
         float z = 0.f;
 #pragma unroll
         for (int c = 0; c < DO; ++c) if (c == lane) z = acc[q][c];
@@ -373,7 +380,8 @@ __global__ void k_head_reduce(HeadReduceArgs g) {
   const HeadReduceJob jb = g.jobs[i];
   const int n_blk = g.B_pad / kHeadRows;
   if (!g.active[i]) {
-    if (blockIdx.y == 0 && threadIdx.x == 0 && g.loss_out) g.loss_out[i] = __int_as_float(0x7fc00000);
+    float* lo = g.dyn ? g.dyn->loss_out : g.loss_out;
+    if (blockIdx.y == 0 && threadIdx.x == 0 && lo) lo[i] = __int_as_float(0x7fc00000);
     return;
   }
   const int w = jb.w, d_out = g.d_out;
@@ -410,7 +418,8 @@ __global__ void k_head_reduce(HeadReduceArgs g) {
     float s = 0.f;
     for (int b = 0; b < n_blk; ++b) s += g.loss_part[(int64_t)i * g.n_blk_cap + b];
     const float loss = s / (float)g.B;
-    if (g.loss_out) g.loss_out[i] = loss;
+    float* lo = g.dyn ? g.dyn->loss_out : g.loss_out;
+    if (lo) lo[i] = loss;
     g.loss_last[i] = loss;
   }
 }
@@ -578,13 +587,13 @@ __global__ void k_debug_masks(uint8_t* __restrict__ out, int32_t B, int32_t w, u
 
 // ------------------------------------------------------------- launchers
 template <typename T>
-void launch_gather(cudaStream_t st, const float* X, const int32_t* idx, int B, int B_pad, int d_in,
-                   int d_in_pad, int ldx, T* xb, int advance, int32_t* t_dev, float2* bias_corr,
+void launch_gather(cudaStream_t st, const float* X, const int32_t* idx, const StepDyn* dyn, int B, int B_pad,
+                   int d_in, int d_in_pad, int ldx, T* xb, int advance, int32_t* t_dev, float2* bias_corr,
                    const int32_t* active_ids, int n_active, float beta1, float beta2) {
   int64_t total = (int64_t)B_pad * d_in_pad;
   int blocks = (int)std::min<int64_t>(ceil_div(total, 256), 152 * 8);
   if (blocks < 1) blocks = 1;
-  k_gather<T><<<blocks, 256, 0, st>>>(X, idx, B, B_pad, d_in, d_in_pad, ldx, xb, advance, t_dev, bias_corr,
+  k_gather<T><<<blocks, 256, 0, st>>>(X, idx, dyn, B, B_pad, d_in, d_in_pad, ldx, xb, advance, t_dev, bias_corr,
                                        active_ids, n_active, beta1, beta2);
 }
 
@@ -643,8 +652,8 @@ void launch_debug_masks(cudaStream_t st, uint8_t* out, int B, int w, uint64_t se
 }
 
 #define TP_INSTANTIATE(T)                                                                              \
-  template void launch_gather<T>(cudaStream_t, const float*, const int32_t*, int, int, int, int, int, T*, \
-                                 int, int32_t*, float2*, const int32_t*, int, float, float);            \
+  template void launch_gather<T>(cudaStream_t, const float*, const int32_t*, const StepDyn*, int, int, int, int, \
+                                 int, T*, int, int32_t*, float2*, const int32_t*, int, float, float);   \
   template void launch_fill_ones<T>(cudaStream_t, const OnesJob*, int, T*, T*);                         \
   template void launch_gemm_simt<T>(cudaStream_t, const GemmArgs<T>&, int, int);                       \
   template void launch_head<T>(cudaStream_t, const HeadArgs<T>&, int);                                 \

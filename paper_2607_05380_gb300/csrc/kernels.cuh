@@ -22,6 +22,7 @@ struct GemmArgs {
   uint32_t step;
   int32_t train;          // 1: dropout on
   uint64_t seed;
+  const StepDyn* dyn;     // non-NULL: take the step from here
 };
 
 template <typename T>
@@ -37,6 +38,7 @@ struct HeadArgs {
   const int32_t* idx;
   const void* y;
   int32_t B, B_pad, B_cap, d_out, task, n_blk_cap;
+  const StepDyn* dyn;     // non-NULL: take idx and y from here
 };
 
 struct HeadReduceArgs {
@@ -51,6 +53,7 @@ struct HeadReduceArgs {
   int32_t B, B_pad, d_out, n_blk_cap;
   int32_t update;         // 1: apply AdamW to the head parameters instead of storing the gradients
   AdamDev adam;
+  const StepDyn* dyn;     // non-NULL: take loss_out from here
 };
 
 struct AdamArgs {
@@ -90,9 +93,10 @@ struct PredictHeadArgs {
   int32_t rows, d_out, task, _pad;
 };
 
+// dyn non-NULL: X and idx are taken from it
 template <typename T>
-void launch_gather(cudaStream_t st, const float* X, const int32_t* idx, int B, int B_pad, int d_in,
-                   int d_in_pad, int ldx, T* xb, int advance, int32_t* t_dev, float2* bias_corr,
+void launch_gather(cudaStream_t st, const float* X, const int32_t* idx, const StepDyn* dyn, int B, int B_pad,
+                   int d_in, int d_in_pad, int ldx, T* xb, int advance, int32_t* t_dev, float2* bias_corr,
                    const int32_t* active_ids, int n_active, float beta1, float beta2);
 template <typename T>
 void launch_gemm_simt(cudaStream_t st, const GemmArgs<T>& g, int tile_base, int n_tiles);

@@ -72,6 +72,23 @@ struct tabpack {
   std::vector<std::pair<int, int>> fwd_rng, bwd_rng;  // CUDA-core tile ranges per depth index
   int cap_chunks = 0, cap_probs = 0, cap_tiles = 0, cap_head = 0;
 
+  // CUDA graphs of the training step, one per (B, update, weight copy); the
+  // per-call arguments travel through dyn_dev, filled from a pinned ring
+  struct GraphEntry {
+    int B, update, wcur;
+    cudaGraphExec_t exec;
+    int64_t n_launch;
+  };
+  std::vector<GraphEntry> graphs;
+  bool use_graphs = true;
+  cudaStream_t st_cap = nullptr;  // graphs are captured here (the legacy stream cannot capture)
+  StepDyn* dyn_dev = nullptr;
+  static constexpr int kRing = 16;
+  StepDyn* dyn_host = nullptr;    // pinned [kRing]
+  cudaEvent_t dyn_ev[kRing] = {};
+  bool dyn_used[kRing] = {};
+  int dyn_next = 0;
+
   int last_B = 0;
   int64_t launches = 0;
   size_t dev_bytes = 0;
@@ -164,6 +181,8 @@ void prof_flush(tabpack* h) {
 }
 
 int ldh_of(const tabpack* h, int i) { return h->width[i] + kOnesCols; }
+
+void drop_graphs(tabpack* h);
 
 // ------------------------------------------------------------------ layout
 tp_status build_layout(tabpack* h) {
@@ -348,6 +367,7 @@ tp_status build_schedule(tabpack* h) {
       (int)ch.size() > h->cap_chunks)
     return fail(h, TP_ESTATE, "schedule grew beyond its capacity");
   TP_CUDA(h, cudaStreamSynchronize(h->st));
+  drop_graphs(h);  // captured launches carry the old work-list sizes
   if (!probs.empty()) TP_CUDA(h, cudaMemcpy(h->probs_dev, probs.data(), sizeof(GemmProblem) * probs.size(), cudaMemcpyHostToDevice));
   if (!tiles.empty()) TP_CUDA(h, cudaMemcpy(h->tiles_dev, tiles.data(), sizeof(GemmTile) * tiles.size(), cudaMemcpyHostToDevice));
   if (!hj.empty()) TP_CUDA(h, cudaMemcpy(h->head_jobs_dev, hj.data(), sizeof(HeadJob) * hj.size(), cudaMemcpyHostToDevice));
@@ -426,6 +446,10 @@ tp_status alloc_all(tabpack* h) {
   TP_TRY(dalloc(h, &h->mem_dev, sizeof(MemberDev) * m));
   TP_TRY(dalloc(h, &h->segs_dev, sizeof(Segment) * h->segs.size()));
   TP_TRY(dalloc(h, &h->part_stride_dev, sizeof(int64_t) * m));
+  TP_TRY(dalloc(h, &h->dyn_dev, sizeof(StepDyn)));
+  TP_CUDA(h, cudaHostAlloc((void**)&h->dyn_host, sizeof(StepDyn) * tabpack::kRing, cudaHostAllocDefault));
+  for (int k = 0; k < tabpack::kRing; ++k) TP_CUDA(h, cudaEventCreateWithFlags(&h->dyn_ev[k], cudaEventDisableTiming));
+  TP_CUDA(h, cudaStreamCreateWithFlags(&h->st_cap, cudaStreamNonBlocking));
   TP_CUDA(h, cudaMemset(h->t_dev, 0, sizeof(int32_t) * m));
   TP_CUDA(h, cudaMemset(h->bias_corr, 0, sizeof(float2) * m));
   TP_CUDA(h, cudaMemset(h->xb, 0, h->elem * h->xb_elems));
@@ -438,8 +462,20 @@ tp_status alloc_all(tabpack* h) {
   return TP_OK;
 }
 
+void drop_graphs(tabpack* h) {
+  for (auto& ge : h->graphs) cudaGraphExecDestroy(ge.exec);
+  h->graphs.clear();
+}
+
 void free_all(tabpack* h) {
   if (h->st) cudaStreamSynchronize(h->st);
+  drop_graphs(h);
+  if (h->st_cap) cudaStreamDestroy(h->st_cap);
+  h->st_cap = nullptr;
+  for (auto& e : h->dyn_ev)
+    if (e) cudaEventDestroy(e);
+  if (h->dyn_host) cudaFreeHost(h->dyn_host);
+  h->dyn_host = nullptr;
   tc_free_plan(h->tc);
   for (void* p : h->allocs) cudaFree(p);
   h->allocs.clear();
@@ -464,6 +500,7 @@ GemmArgs<T> gemm_args(tabpack* h, int B, int B_pad, uint32_t step, int train) {
   g.step = step;
   g.train = train;
   g.seed = h->cfg.seed;
+  g.dyn = nullptr;
   return g;
 }
 
@@ -483,15 +520,16 @@ AdamDev adam_dev(tabpack* h, __nv_bfloat16* wq_out) {
 }
 
 template <typename T>
-tp_status run_forward(tabpack* h, int B, int B_pad, uint32_t step, int train) {
+tp_status run_forward(tabpack* h, int B, int B_pad, uint32_t step, const StepDyn* dyn, int train) {
   for (int l = 0; l < h->Lmax; ++l) {
     int slot;
     prof_begin(h, train ? TP_PH_FWD : TP_PH_PREDICT, &slot);
     if (h->bf16) {
-      TP_TRY(tc_run_fwd(h->tc, h->st, l, B, B_pad, h->wcur, step, train, h->cfg.seed, h->params, h->mem_dev, h->act,
-                        h->err));
+      TP_TRY(tc_run_fwd(h->tc, h->st, l, B, B_pad, h->wcur, step, dyn, train, h->cfg.seed, h->params, h->mem_dev,
+                        h->act, h->err));
     } else {
       auto g = gemm_args<T>(h, B, B_pad, step, train);
+      g.dyn = dyn;
       launch_gemm_simt<T>(h->st, g, h->fwd_rng[l].first, h->fwd_rng[l].second);
     }
     TP_LAUNCHED(h);
@@ -501,24 +539,26 @@ tp_status run_forward(tabpack* h, int B, int B_pad, uint32_t step, int train) {
   return TP_OK;
 }
 
-// One step on the pack's stream:
+// One step on the pack's stream (enqueue only; the caller flips the weight
+// copy for the next step):
 //   gather -> forward (per depth) -> head + loss -> head reduce (+ head AdamW)
-//   -> backward (per depth, deepest first; bf16: AdamW fused into the wgrad
-//   epilogue, bias gradients from the ones column) -> fp32 mode: AdamW.
+//   -> backward (per depth, deepest first; bias gradients from the ones
+//   column; AdamW fused into the wgrad epilogue or) -> one AdamW pass.
+// dyn non-NULL: X, idx, y, loss_out and step are read from it on the device.
 template <typename T>
 tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* idx, const void* y, int B,
-                   uint32_t step, float* loss_out, bool update) {
+                   uint32_t step, float* loss_out, bool update, const StepDyn* dyn) {
   const int B_pad = (int)round_up(B, kRowTile);
   const bool fused = update && h->bf16 && h->fuse_adamw;
   __nv_bfloat16* wq_next = h->bf16 ? h->wq[h->wcur ^ 1] : nullptr;
   int slot;
   prof_begin(h, TP_PH_GATHER, &slot);
-  launch_gather<T>(h->st, X, idx, B, B_pad, h->cfg.d_in, h->d_in_pad, h->ldx, (T*)h->xb, update ? 1 : 0, h->t_dev,
-                   h->bias_corr, h->active_ids_dev, h->n_active, h->cfg.beta1, h->cfg.beta2);
+  launch_gather<T>(h->st, X, idx, dyn, B, B_pad, h->cfg.d_in, h->d_in_pad, h->ldx, (T*)h->xb, update ? 1 : 0,
+                   h->t_dev, h->bias_corr, h->active_ids_dev, h->n_active, h->cfg.beta1, h->cfg.beta2);
   TP_LAUNCHED(h);
   h->launches++;
   prof_end(h, slot, 1, TP_PH_GATHER);
-  TP_TRY(run_forward<T>(h, B, B_pad, step, 1));
+  TP_TRY(run_forward<T>(h, B, B_pad, step, dyn, 1));
   // head + loss
   prof_begin(h, TP_PH_HEAD, &slot);
   HeadArgs<T> hg;
@@ -538,6 +578,7 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
   hg.d_out = h->cfg.d_out;
   hg.task = h->cfg.task;
   hg.n_blk_cap = h->n_blk_cap;
+  hg.dyn = dyn;
   launch_head<T>(h->st, hg, h->n_head_jobs);
   TP_LAUNCHED(h);
   h->launches++;
@@ -557,6 +598,7 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
   rg.n_blk_cap = h->n_blk_cap;
   rg.update = fused ? 1 : 0;
   rg.adam = adam_dev(h, wq_next);
+  rg.dyn = dyn;
   int w_max = 0;
   for (int w : h->width) w_max = std::max(w_max, w);
   launch_head_reduce(h->st, rg, h->cfg.m, h->cfg.d_out * (w_max + 1));
@@ -599,9 +641,59 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
     h->launches++;
     prof_end(h, slot, 1, TP_PH_ADAMW);
   }
+  (void)n_rows;
+  return TP_OK;
+}
+
+// A training (update) or forward-backward step: replay the captured graph
+// of this (B, update, weight copy) after copying the per-call arguments to
+// the device, or launch the kernels directly while profiling.
+template <typename T>
+tp_status step_entry(tabpack* h, const float* X, int64_t n_rows, const int32_t* idx, const void* y, int B,
+                     uint32_t step, float* loss_out, bool update) {
+  if (!h->use_graphs || h->profiling) {
+    TP_TRY(run_step<T>(h, X, n_rows, idx, y, B, step, loss_out, update, nullptr));
+  } else {
+    // per-call arguments: pinned ring slot -> dyn_dev, ordered before the graph
+    const int k = h->dyn_next;
+    h->dyn_next = (k + 1) % tabpack::kRing;
+    if (h->dyn_used[k]) TP_CUDA(h, cudaEventSynchronize(h->dyn_ev[k]));
+    h->dyn_host[k] = StepDyn{X, idx, y, loss_out, step, 0};
+    TP_CUDA(h, cudaMemcpyAsync(h->dyn_dev, &h->dyn_host[k], sizeof(StepDyn), cudaMemcpyHostToDevice, h->st));
+    TP_CUDA(h, cudaEventRecord(h->dyn_ev[k], h->st));
+    h->dyn_used[k] = true;
+    tabpack::GraphEntry* ge = nullptr;
+    for (auto& e : h->graphs)
+      if (e.B == B && e.update == (int)update && e.wcur == h->wcur) ge = &e;
+    if (!ge) {
+      cudaStream_t user = h->st;
+      h->st = h->st_cap;
+      const int64_t l0 = h->launches;
+      cudaError_t e = cudaStreamBeginCapture(h->st, cudaStreamCaptureModeThreadLocal);
+      tp_status s = e == cudaSuccess ? run_step<T>(h, X, n_rows, idx, y, B, step, loss_out, update, h->dyn_dev)
+                                     : fail(h, TP_ECUDA, "cudaStreamBeginCapture: %s", cudaGetErrorString(e));
+      cudaGraph_t graph = nullptr;
+      cudaError_t e2 = e == cudaSuccess ? cudaStreamEndCapture(h->st, &graph) : cudaSuccess;
+      h->st = user;
+      const int64_t n_launch = h->launches - l0;
+      h->launches = l0;
+      if (s != TP_OK) {
+        if (graph) cudaGraphDestroy(graph);
+        return s;
+      }
+      if (e2 != cudaSuccess) return fail(h, TP_ECUDA, "cudaStreamEndCapture: %s", cudaGetErrorString(e2));
+      cudaGraphExec_t exec = nullptr;
+      e = cudaGraphInstantiate(&exec, graph, 0);
+      cudaGraphDestroy(graph);
+      if (e != cudaSuccess) return fail(h, TP_ECUDA, "cudaGraphInstantiate: %s", cudaGetErrorString(e));
+      h->graphs.push_back(tabpack::GraphEntry{B, (int)update, h->wcur, exec, n_launch});
+      ge = &h->graphs.back();
+    }
+    TP_CUDA(h, cudaGraphLaunch(ge->exec, h->st));
+    h->launches += ge->n_launch;
+  }
   if (update && h->bf16) h->wcur ^= 1;
   h->last_B = B;
-  (void)n_rows;
   return TP_OK;
 }
 
@@ -612,12 +704,13 @@ tp_status run_predict(tabpack* h, const float* X, int64_t N, float* out) {
     const int B_pad = (int)round_up(rows, kRowTile);
     int slot;
     prof_begin(h, TP_PH_PREDICT, &slot);
-    launch_gather<T>(h->st, X + n0 * h->cfg.d_in, nullptr, rows, B_pad, h->cfg.d_in, h->d_in_pad, h->ldx, (T*)h->xb,
+    launch_gather<T>(h->st, X + n0 * h->cfg.d_in, nullptr, nullptr, rows, B_pad, h->cfg.d_in, h->d_in_pad, h->ldx,
+                     (T*)h->xb,
                      0, h->t_dev, h->bias_corr, h->active_ids_dev, 0, h->cfg.beta1, h->cfg.beta2);
     TP_LAUNCHED(h);
     h->launches++;
     prof_end(h, slot, 1, TP_PH_PREDICT);
-    TP_TRY(run_forward<T>(h, rows, B_pad, 0u, 0));
+    TP_TRY(run_forward<T>(h, rows, B_pad, 0u, nullptr, 0));
     prof_begin(h, TP_PH_PREDICT, &slot);
     PredictHeadArgs<T> pg;
     pg.jobs = h->head_jobs_dev;
@@ -757,16 +850,16 @@ tp_status pack_train_step(tabpack_t* h, const float* X, int64_t n_rows, const in
                           int32_t B, uint32_t step, float* loss_out) {
   TP_TRY(check_step_args(h, X, n_rows, idx, y, B));
   if (h->n_active == 0) return fail(h, TP_ESTATE, "no active member");
-  return h->bf16 ? run_step<__nv_bfloat16>(h, X, n_rows, idx, y, B, step, loss_out, true)
-                 : run_step<float>(h, X, n_rows, idx, y, B, step, loss_out, true);
+  return h->bf16 ? step_entry<__nv_bfloat16>(h, X, n_rows, idx, y, B, step, loss_out, true)
+                 : step_entry<float>(h, X, n_rows, idx, y, B, step, loss_out, true);
 }
 
 tp_status pack_forward_backward(tabpack_t* h, const float* X, int64_t n_rows, const int32_t* idx, const void* y,
                                 int32_t B, uint32_t step, float* loss_out) {
   TP_TRY(check_step_args(h, X, n_rows, idx, y, B));
   if (h->n_active == 0) return fail(h, TP_ESTATE, "no active member");
-  return h->bf16 ? run_step<__nv_bfloat16>(h, X, n_rows, idx, y, B, step, loss_out, false)
-                 : run_step<float>(h, X, n_rows, idx, y, B, step, loss_out, false);
+  return h->bf16 ? step_entry<__nv_bfloat16>(h, X, n_rows, idx, y, B, step, loss_out, false)
+                 : step_entry<float>(h, X, n_rows, idx, y, B, step, loss_out, false);
 }
 
 tp_status pack_predict(tabpack_t* h, const float* X, int64_t N, float* out) {

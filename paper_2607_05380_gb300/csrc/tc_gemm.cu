@@ -80,6 +80,7 @@ struct TcArgs {
   float* grads;
   AdamDev adam;
   int* err;
+  const StepDyn* dyn;  // non-NULL: the dropout step counter is read from here
 };
 
 // ------------------------------------------------------------ PTX helpers
@@ -320,6 +321,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
     const int q = warp & 3;             // TMEM lane quarter this warp may access
     const int half = (warp - 2) >> 2;   // 0 for warps 2-5, 1 for warps 6-9
     const int row = 32 * q + lane;
+    const uint32_t step = g.dyn ? g.dyn->step : g.step;
     uint32_t acc = 0, acc_phase = 0;
     for (int t = blockIdx.x; t < g.n_tiles; t += gridDim.x) {
       const TcTile tile = g.tiles[t];
@@ -360,7 +362,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
             keep = 0;
 #pragma unroll
             for (int g4 = 0; g4 < 8; ++g4)
-              keep |= keep_bits4(g.seed, (uint32_t)tile.member, (uint32_t)tile.layer, g.step, (uint32_t)r,
+              keep |= keep_bits4(g.seed, (uint32_t)tile.member, (uint32_t)tile.layer, step, (uint32_t)r,
                                  (uint32_t)((col0 >> 2) + g4), md.drop_T)
                       << (4 * g4);
           }
@@ -695,12 +697,13 @@ static tp_status launch(TcPlan& plan, cudaStream_t st, const std::pair<int, int>
 }
 
 tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, int wcur, uint32_t step,
-                     int train, uint64_t seed, const float* params, const MemberDev* mem, void* act,
-                     std::string& err) {
+                     const StepDyn* dyn, int train, uint64_t seed, const float* params, const MemberDev* mem,
+                     void* act, std::string& err) {
   TcArgs a{};
   a.B = B;
   a.B_pad = B_pad;
   a.step = step;
+  a.dyn = dyn;
   a.train = train;
   a.w_shift = wcur ? plan.w_shift : 0;
   a.update = 0;

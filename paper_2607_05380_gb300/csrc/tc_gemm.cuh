@@ -62,9 +62,10 @@ struct TcLayout {          // what the plan needs to know about the pack's arena
 
 tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err);
 // Forward products of hidden layer `layer`, reading weight copy `wcur`.
+// The dropout step counter is `step`, or dyn->step when dyn is non-NULL.
 tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, int wcur, uint32_t step,
-                     int train, uint64_t seed, const float* params, const MemberDev* mem, void* act,
-                     std::string& err);
+                     const StepDyn* dyn, int train, uint64_t seed, const float* params, const MemberDev* mem,
+                     void* act, std::string& err);
 // Backward products (dgrad + wgrad) of hidden layer `layer`.  update = 0: the
 // weight and bias gradients are stored in `grads`; update = 1: AdamW is
 // applied in the epilogue (adam.wq_out = the other weight copy).

@@ -102,6 +102,17 @@ struct OnesJob {          // column `col` of rows 0..rows-1 of a matrix with pit
   int32_t arena;          // 0: xb, 1: act
 };
 
+// The per-call arguments of a training step, read from device memory by the
+// kernels of a replayed CUDA graph (the graph itself stays unchanged).
+struct StepDyn {
+  const float* X;
+  const int32_t* idx;
+  const void* y;
+  float* loss_out;
+  uint32_t step;
+  uint32_t _pad;
+};
+
 // What a fused AdamW update needs besides the element itself.
 struct AdamDev {
   float* params;
