@@ -16,6 +16,8 @@ __global__ void k_gather(const float* __restrict__ X, const int32_t* __restrict_
                          int32_t advance, int32_t* __restrict__ t_dev, float2* __restrict__ bias_corr,
                          const int32_t* __restrict__ active_ids, int32_t n_active, float beta1,
                          float beta2) {
+  pdl_trigger();
+  pdl_wait();
   if (dyn) {
     X = dyn->X;
     idx = dyn->idx;
@@ -56,6 +58,8 @@ __global__ void k_fill_ones(const OnesJob* __restrict__ jobs, T* __restrict__ xb
 // in increasing k order with fused multiply-adds (fp32).
 template <typename T>
 __global__ void __launch_bounds__(256) k_gemm_simt(GemmArgs<T> g, int32_t tile_base) {
+  pdl_trigger();
+  pdl_wait();
   const GemmTile t = g.tiles[tile_base + blockIdx.x];
   const GemmProblem P = g.probs[t.prob];
   const int M = P.M ? P.M : g.B_pad;
@@ -234,6 +238,8 @@ __global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
   // whose per-row state (DO logits and dlogits) would otherwise cost occupancy
   constexpr int R = DO == 1 ? 4 : (DO <= 4 ? 2 : 1);
   constexpr int RW = kHeadRows / 8;  // rows per warp
+  pdl_trigger();
+  pdl_wait();
   const HeadJob jb = g.jobs[blockIdx.x];
   const int r0 = jb.blk * kHeadRows;
   if (r0 >= g.B_pad) return;
@@ -376,6 +382,8 @@ __global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
 // head parameters directly (the gradients are not stored).  Grid: member x
 // chunks of 256 head parameters; inactive members report NaN.
 __global__ void k_head_reduce(HeadReduceArgs g) {
+  pdl_trigger();
+  pdl_wait();
   const int i = blockIdx.x;
   const HeadReduceJob jb = g.jobs[i];
   const int n_blk = g.B_pad / kHeadRows;
@@ -428,6 +436,8 @@ __global__ void k_head_reduce(HeadReduceArgs g) {
 // Stand-alone AdamW over chunks of the arena (fp32 mode), with the member's
 // lr and wd and its step's bias corrections; float4 body, scalar tail.
 __global__ void __launch_bounds__(256) k_adamw(AdamArgs g) {
+  pdl_trigger();
+  pdl_wait();
   const Chunk ch = g.chunks[blockIdx.x];
   const Segment s = g.segs[ch.seg];
   const MemberDev md = g.mem[s.member];
@@ -524,6 +534,7 @@ __global__ void k_refresh_wq(const float* __restrict__ p, __nv_bfloat16* __restr
 // out[member, n0 + r, :] for r < rows.
 template <typename T, int DO>
 __global__ void __launch_bounds__(256) k_predict_head(PredictHeadArgs<T> g) {
+  pdl_wait();
   const HeadJob jb = g.jobs[blockIdx.x];
   const int r0 = jb.blk * kHeadRows;
   if (r0 >= g.rows) return;
@@ -593,7 +604,7 @@ void launch_gather(cudaStream_t st, const float* X, const int32_t* idx, const St
   int64_t total = (int64_t)B_pad * d_in_pad;
   int blocks = (int)std::min<int64_t>(ceil_div(total, 256), 152 * 8);
   if (blocks < 1) blocks = 1;
-  k_gather<T><<<blocks, 256, 0, st>>>(X, idx, dyn, B, B_pad, d_in, d_in_pad, ldx, xb, advance, t_dev, bias_corr,
+  launch_pdl(k_gather<T>, dim3(blocks), dim3(256), 0, st, X, idx, dyn, B, B_pad, d_in, d_in_pad, ldx, xb, advance, t_dev, bias_corr,
                                        active_ids, n_active, beta1, beta2);
 }
 
@@ -604,28 +615,28 @@ void launch_fill_ones(cudaStream_t st, const OnesJob* jobs, int n_jobs, T* xb, T
 
 template <typename T>
 void launch_gemm_simt(cudaStream_t st, const GemmArgs<T>& g, int tile_base, int n_tiles) {
-  if (n_tiles > 0) k_gemm_simt<T><<<n_tiles, 256, 0, st>>>(g, tile_base);
+  if (n_tiles > 0) launch_pdl(k_gemm_simt<T>, dim3(n_tiles), dim3(256), 0, st, g, tile_base);
 }
 
 template <typename T>
 void launch_head(cudaStream_t st, const HeadArgs<T>& g, int n_jobs) {
   if (n_jobs <= 0) return;
   // class-count buckets: the loops over classes are unrolled to the bucket size
-  if (g.d_out == 1) k_head<T, 1><<<n_jobs, 256, 0, st>>>(g);
-  else if (g.d_out <= 2) k_head<T, 2><<<n_jobs, 256, 0, st>>>(g);
-  else if (g.d_out <= 4) k_head<T, 4><<<n_jobs, 256, 0, st>>>(g);
-  else if (g.d_out <= 8) k_head<T, 8><<<n_jobs, 256, 0, st>>>(g);
-  else if (g.d_out <= 10) k_head<T, 10><<<n_jobs, 256, 0, st>>>(g);
-  else if (g.d_out <= 16) k_head<T, 16><<<n_jobs, 256, 0, st>>>(g);
-  else k_head<T, kMaxDout><<<n_jobs, 256, 0, st>>>(g);
+  if (g.d_out == 1) launch_pdl(k_head<T, 1>, dim3(n_jobs), dim3(256), 0, st, g);
+  else if (g.d_out <= 2) launch_pdl(k_head<T, 2>, dim3(n_jobs), dim3(256), 0, st, g);
+  else if (g.d_out <= 4) launch_pdl(k_head<T, 4>, dim3(n_jobs), dim3(256), 0, st, g);
+  else if (g.d_out <= 8) launch_pdl(k_head<T, 8>, dim3(n_jobs), dim3(256), 0, st, g);
+  else if (g.d_out <= 10) launch_pdl(k_head<T, 10>, dim3(n_jobs), dim3(256), 0, st, g);
+  else if (g.d_out <= 16) launch_pdl(k_head<T, 16>, dim3(n_jobs), dim3(256), 0, st, g);
+  else launch_pdl(k_head<T, kMaxDout>, dim3(n_jobs), dim3(256), 0, st, g);
 }
 
 void launch_head_reduce(cudaStream_t st, const HeadReduceArgs& g, int m, int max_elems) {
-  k_head_reduce<<<dim3(m, (unsigned)ceil_div(max_elems, 256)), 256, 0, st>>>(g);
+  launch_pdl(k_head_reduce, dim3(m, (unsigned)ceil_div(max_elems, 256)), dim3(256), 0, st, g);
 }
 
 void launch_adamw(cudaStream_t st, const AdamArgs& g, int n_chunks) {
-  if (n_chunks > 0) k_adamw<<<n_chunks, 256, 0, st>>>(g);
+  if (n_chunks > 0) launch_pdl(k_adamw, dim3(n_chunks), dim3(256), 0, st, g);
 }
 
 void launch_init(cudaStream_t st, const InitArgs& g, int n_chunks) {

@@ -218,6 +218,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // The set-up above overlaps the previous kernel; data reads start here.  The
+  // GEMM itself never triggers its dependents early: CTAs of the next kernel
+  // parked beside a running GEMM measurably slow it down.
+  pdl_wait();
   const uint32_t tmem = tl->tmem_base;
   volatile int* abort_flag = &tl->abort;
 
@@ -687,7 +691,7 @@ static tp_status launch(TcPlan& plan, cudaStream_t st, const std::pair<int, int>
   a.maps = plan.maps_dev;
   a.err = plan.err_dev;
   const int grid = std::max(1, std::min(rng.second, plan.n_sm));
-  k_tc_gemm<<<grid, kThreads, kSmemBytes, st>>>(a);
+  launch_pdl(k_tc_gemm, dim3(grid), dim3(kThreads), kSmemBytes, st, a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {
     err = std::string("tcgen05 GEMM launch: ") + cudaGetErrorString(e);
