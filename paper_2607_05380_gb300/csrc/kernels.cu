@@ -9,15 +9,17 @@ namespace tp {
 // xb[b, k] = X[idx[b], k] for b < B, k < d_in; zero for the rest of the first
 // d_in_pad columns of rows < B_pad (column d_in_pad holds the constant 1).
 // Block 0 also advances the step count of every active member and stores the
-// AdamW bias corrections 1 - beta^t of the new step (when `advance`).
+// AdamW bias corrections 1 - beta^t of the new step (when `advance`); the
+// grid clears `zero[0 .. n_zero)` (the GEMMs' row-block completion counters).
 template <typename T>
 __global__ void k_gather(const float* __restrict__ X, const int32_t* __restrict__ idx, const StepDyn* dyn,
                          int32_t B, int32_t B_pad, int32_t d_in, int32_t d_in_pad, int32_t ldx, T* __restrict__ xb,
                          int32_t advance, int32_t* __restrict__ t_dev, float2* __restrict__ bias_corr,
                          const int32_t* __restrict__ active_ids, int32_t n_active, float beta1,
-                         float beta2) {
+                         float beta2, int32_t* __restrict__ zero, int32_t n_zero) {
   pdl_trigger();
   pdl_wait();
+  for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < n_zero; e += gridDim.x * blockDim.x) zero[e] = 0;
   if (dyn) {
     X = dyn->X;
     idx = dyn->idx;
@@ -600,12 +602,12 @@ __global__ void k_debug_masks(uint8_t* __restrict__ out, int32_t B, int32_t w, u
 template <typename T>
 void launch_gather(cudaStream_t st, const float* X, const int32_t* idx, const StepDyn* dyn, int B, int B_pad,
                    int d_in, int d_in_pad, int ldx, T* xb, int advance, int32_t* t_dev, float2* bias_corr,
-                   const int32_t* active_ids, int n_active, float beta1, float beta2) {
+                   const int32_t* active_ids, int n_active, float beta1, float beta2, int* zero, int n_zero) {
   int64_t total = (int64_t)B_pad * d_in_pad;
   int blocks = (int)std::min<int64_t>(ceil_div(total, 256), 152 * 8);
   if (blocks < 1) blocks = 1;
   launch_pdl(k_gather<T>, dim3(blocks), dim3(256), 0, st, X, idx, dyn, B, B_pad, d_in, d_in_pad, ldx, xb, advance, t_dev, bias_corr,
-                                       active_ids, n_active, beta1, beta2);
+             active_ids, n_active, beta1, beta2, zero, n_zero);
 }
 
 template <typename T>
@@ -664,7 +666,8 @@ void launch_debug_masks(cudaStream_t st, uint8_t* out, int B, int w, uint64_t se
 
 #define TP_INSTANTIATE(T)                                                                              \
   template void launch_gather<T>(cudaStream_t, const float*, const int32_t*, const StepDyn*, int, int, int, int, \
-                                 int, T*, int, int32_t*, float2*, const int32_t*, int, float, float);   \
+                                 int, T*, int, int32_t*, float2*, const int32_t*, int, float, float,    \
+                                 int*, int);                                                           \
   template void launch_fill_ones<T>(cudaStream_t, const OnesJob*, int, T*, T*);                         \
   template void launch_gemm_simt<T>(cudaStream_t, const GemmArgs<T>&, int, int);                       \
   template void launch_head<T>(cudaStream_t, const HeadArgs<T>&, int);                                 \

@@ -97,7 +97,8 @@ struct PredictHeadArgs {
 template <typename T>
 void launch_gather(cudaStream_t st, const float* X, const int32_t* idx, const StepDyn* dyn, int B, int B_pad,
                    int d_in, int d_in_pad, int ldx, T* xb, int advance, int32_t* t_dev, float2* bias_corr,
-                   const int32_t* active_ids, int n_active, float beta1, float beta2);
+                   const int32_t* active_ids, int n_active, float beta1, float beta2, int* zero = nullptr,
+                   int n_zero = 0);
 template <typename T>
 void launch_gemm_simt(cudaStream_t st, const GemmArgs<T>& g, int tile_base, int n_tiles);
 template <typename T>

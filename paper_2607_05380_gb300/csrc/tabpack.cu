@@ -521,17 +521,22 @@ AdamDev adam_dev(tabpack* h, __nv_bfloat16* wq_out) {
 
 template <typename T>
 tp_status run_forward(tabpack* h, int B, int B_pad, uint32_t step, const StepDyn* dyn, int train) {
-  for (int l = 0; l < h->Lmax; ++l) {
+  if (h->bf16) {  // every layer in one launch
     int slot;
     prof_begin(h, train ? TP_PH_FWD : TP_PH_PREDICT, &slot);
-    if (h->bf16) {
-      TP_TRY(tc_run_fwd(h->tc, h->st, l, B, B_pad, h->wcur, step, dyn, train, h->cfg.seed, h->params, h->mem_dev,
-                        h->act, h->err));
-    } else {
-      auto g = gemm_args<T>(h, B, B_pad, step, train);
-      g.dyn = dyn;
-      launch_gemm_simt<T>(h->st, g, h->fwd_rng[l].first, h->fwd_rng[l].second);
-    }
+    TP_TRY(tc_run_fwd(h->tc, h->st, B, B_pad, h->wcur, step, dyn, train, h->cfg.seed, h->params, h->mem_dev, h->act,
+                      h->err));
+    TP_LAUNCHED(h);
+    h->launches++;
+    prof_end(h, slot, 1, train ? TP_PH_FWD : TP_PH_PREDICT);
+    return TP_OK;
+  }
+  for (int l = 0; l < h->Lmax; ++l) {  // CUDA-core path: one launch per depth
+    int slot;
+    prof_begin(h, train ? TP_PH_FWD : TP_PH_PREDICT, &slot);
+    auto g = gemm_args<T>(h, B, B_pad, step, train);
+    g.dyn = dyn;
+    launch_gemm_simt<T>(h->st, g, h->fwd_rng[l].first, h->fwd_rng[l].second);
     TP_LAUNCHED(h);
     h->launches++;
     prof_end(h, slot, 1, train ? TP_PH_FWD : TP_PH_PREDICT);
@@ -554,7 +559,8 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
   int slot;
   prof_begin(h, TP_PH_GATHER, &slot);
   launch_gather<T>(h->st, X, idx, dyn, B, B_pad, h->cfg.d_in, h->d_in_pad, h->ldx, (T*)h->xb, update ? 1 : 0,
-                   h->t_dev, h->bias_corr, h->active_ids_dev, h->n_active, h->cfg.beta1, h->cfg.beta2);
+                   h->t_dev, h->bias_corr, h->active_ids_dev, h->n_active, h->cfg.beta1, h->cfg.beta2,
+                   h->tc.cnt_dev, h->tc.n_cnt);
   TP_LAUNCHED(h);
   h->launches++;
   prof_end(h, slot, 1, TP_PH_GATHER);
@@ -605,20 +611,25 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
   TP_LAUNCHED(h);
   h->launches++;
   prof_end(h, slot, 2, TP_PH_HEAD);
-  // backward products, deepest layer first
+  // backward products: tensor cores, every layer in one launch; CUDA cores,
+  // one launch per depth, deepest first
   const AdamDev ad = adam_dev(h, wq_next);
-  for (int l = h->Lmax - 1; l >= 0; --l) {
+  if (h->bf16) {
     prof_begin(h, TP_PH_BWD, &slot);
-    if (h->bf16) {
-      TP_TRY(tc_run_bwd(h->tc, h->st, l, B, B_pad, h->wcur, h->mem_dev, h->act, h->dz, h->grads, fused ? 1 : 0, ad,
-                        h->err));
-    } else {
-      auto g = gemm_args<T>(h, B, B_pad, step, 1);
-      launch_gemm_simt<T>(h->st, g, h->bwd_rng[l].first, h->bwd_rng[l].second);
-    }
+    TP_TRY(tc_run_bwd(h->tc, h->st, B, B_pad, h->wcur, h->mem_dev, h->act, h->dz, h->grads, fused ? 1 : 0, ad,
+                      h->err));
     TP_LAUNCHED(h);
     h->launches++;
     prof_end(h, slot, 1, TP_PH_BWD);
+  } else {
+    for (int l = h->Lmax - 1; l >= 0; --l) {
+      prof_begin(h, TP_PH_BWD, &slot);
+      auto g = gemm_args<T>(h, B, B_pad, step, 1);
+      launch_gemm_simt<T>(h->st, g, h->bwd_rng[l].first, h->bwd_rng[l].second);
+      TP_LAUNCHED(h);
+      h->launches++;
+      prof_end(h, slot, 1, TP_PH_BWD);
+    }
   }
   if (update && !fused && h->n_chunks > 0) {
     prof_begin(h, TP_PH_ADAMW, &slot);
@@ -706,7 +717,8 @@ tp_status run_predict(tabpack* h, const float* X, int64_t N, float* out) {
     prof_begin(h, TP_PH_PREDICT, &slot);
     launch_gather<T>(h->st, X + n0 * h->cfg.d_in, nullptr, nullptr, rows, B_pad, h->cfg.d_in, h->d_in_pad, h->ldx,
                      (T*)h->xb,
-                     0, h->t_dev, h->bias_corr, h->active_ids_dev, 0, h->cfg.beta1, h->cfg.beta2);
+                     0, h->t_dev, h->bias_corr, h->active_ids_dev, 0, h->cfg.beta1, h->cfg.beta2, h->tc.cnt_dev,
+                     h->tc.n_cnt);
     TP_LAUNCHED(h);
     h->launches++;
     prof_end(h, slot, 1, TP_PH_PREDICT);

@@ -1,9 +1,16 @@
 // tc_gemm.cu -- persistent warp-specialised grouped GEMM on tcgen05 (sm_103a).
 //
-// Every launch processes a list of 128 x N output tiles (N <= 256, a
-// multiple of 16) of many members' products; each persistent CTA (one per
-// SM) walks the list with stride gridDim.x (the list is sorted by cost,
-// largest first).  Warp roles:
+// One launch runs every forward product of the step (all members, all
+// depths), another every backward product: a list of 128 x N output tiles
+// (N <= 256, a multiple of 16) that each persistent CTA (one per SM) walks
+// with stride gridDim.x.  The list is ordered by dependency level (forward:
+// the layer; backward: the distance from the head) and by cost, largest
+// first, within a level.  A tile whose A operand is produced in the same
+// launch waits for a row-block completion counter (the producer polls it
+// with acquire loads, bounded); every epilogue warp publishes its stores
+// with a release add when it finishes a tile.  All CTAs are resident at once
+// (grid <= SMs, one CTA per SM), and a tile only waits on tiles earlier in
+// the list, so the waits always end.  Warp roles:
 //   warp 0     TMA producer: per 64-wide K block, loads the A tile
 //              (2 boxes of 64 x 64 bf16) and the B tile (N/64 boxes) into a
 //              4-stage shared-memory ring, 128-byte swizzled.
@@ -81,6 +88,7 @@ struct TcArgs {
   AdamDev adam;
   int* err;
   const StepDyn* dyn;  // non-NULL: the dropout step counter is read from here
+  int* cnt;            // row-block completion counters
 };
 
 // ------------------------------------------------------------ PTX helpers
@@ -125,6 +133,39 @@ __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile 
       return false;
     }
   }
+}
+
+__device__ __forceinline__ int ld_acquire(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void red_release_add(int* p, int v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+// Generic-proxy writes of other CTAs, acquired through a counter, become
+// visible to this thread's subsequent TMA (async-proxy) reads.
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+// Bounded wait until counters p[0 .. n-1] each reach `need`.
+__device__ __noinline__ bool dep_wait(const int* p, int n, int need, volatile int* abort_flag, int* err) {
+  for (int j = 0; j < n; ++j) {
+    if (ld_acquire(p + j) >= need) continue;
+    const uint64_t t0 = global_ns();
+    while (ld_acquire(p + j) < need) {
+      if (*abort_flag) return false;
+      if (global_ns() - t0 > kWaitNs) {
+        *abort_flag = 1;
+        atomicExch(err, 1);
+        return false;
+      }
+      __nanosleep(32);
+    }
+  }
+  fence_proxy_async_global();
+  return true;
 }
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint64_t* bar, int x, int y) {
@@ -241,6 +282,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         tensormap_acquire(mb);
         const int nb = (tile.n_len + 63) >> 6;
         const uint32_t bytes = (uint32_t)(2 + nb) * kBoxBytes;
+        if (tile.dep >= 0 &&
+            !dep_wait(g.cnt + tile.dep, tile.dep_n ? tile.dep_n : g.B_pad / 128, tile.dep_need, abort_flag, g.err)) {
+          ok = false;
+          break;
+        }
         for (int k0 = 0; k0 < K; k0 += 64) {
           if (!mbar_wait(&tl->empty[stage], phase ^ 1u, abort_flag, g.err, kWaitNs)) {
             ok = false;
@@ -467,6 +513,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       mbar_arrive(&tl->tempty[acc]);
       acc ^= 1u;
       if (acc == 0) acc_phase ^= 1u;
+      if (tile.sig >= 0) {  // publish this warp's part of the tile
+        __syncwarp();
+        if (lane == 0) {
+          fence_proxy_async_global();
+          __threadfence();
+          red_release_add(g.cnt + tile.sig, 1);
+        }
+      }
     }
   }
 
@@ -585,18 +639,28 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
     }
   }
 
-  // tiles of the active members, per launch, largest first
+  // Tiles of the active members.  Forward: level = layer.  Backward: level
+  // = distance from the head (each member's top hidden layer first); within a
+  // level the dgrad tiles (which the next level waits for) precede the wgrad
+  // tiles, each group sorted largest first.
+  const int nrb = lay.B_cap / kRowTile;
+  if (plan.cnt_dev == nullptr) {
+    plan.n_cnt = 2 * m * kMaxDepth * nrb;
+    if (cudaMalloc(&plan.cnt_dev, sizeof(int) * plan.n_cnt) != cudaSuccess ||
+        cudaMemset(plan.cnt_dev, 0, sizeof(int) * plan.n_cnt) != cudaSuccess) {
+      err = "cudaMalloc(tc counters) failed";
+      return TP_ENOMEM;
+    }
+  }
+  auto cnt_act = [&](int i, int l) { return (i * kMaxDepth + l) * nrb; };
+  auto cnt_dz = [&](int i, int l) { return ((m + i) * kMaxDepth + l) * nrb; };
   int Lmax = 0;
   for (int i = 0; i < m; ++i) Lmax = std::max(Lmax, depth[i]);
   std::vector<TcTile> all;
-  plan.fwd_rng.assign(Lmax, {0, 0});
-  plan.bwd_rng.assign(Lmax, {0, 0});
   auto cost = [&](const TcTile& t) { return (int64_t)(t.k_len ? t.k_len : lay.B_cap) * t.n_len; };
   auto sorted_append = [&](std::vector<TcTile>& v) {
     std::stable_sort(v.begin(), v.end(), [&](const TcTile& a, const TcTile& b) { return cost(a) > cost(b); });
-    const int base = (int)all.size();
     all.insert(all.end(), v.begin(), v.end());
-    return std::make_pair(base, (int)v.size());
   };
   std::vector<std::pair<int, int>> ns;
   for (int l = 0; l < Lmax; ++l) {
@@ -605,7 +669,8 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
       if (!active[i] || depth[i] <= l) continue;
       const int w = width[i];
       split_n(w, ns);
-      for (int m0 = 0; m0 < lay.B_cap; m0 += 128)
+      const int need = 8 * (int)ns.size();  // every epilogue warp of every N tile of a row block
+      for (int m0 = 0; m0 < lay.B_cap; m0 += kRowTile)
         for (auto& nn : ns) {
           TcTile t{};
           t.kind = kFwd; t.member = i; t.layer = l;
@@ -616,21 +681,29 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
           t.map_b = plan.map_w[(size_t)i * kMaxDepth + l];
           t.ldc = w + kOnesCols;
           t.ld_aux = 0;
+          t.dep = l == 0 ? -1 : cnt_act(i, l - 1) + m0 / kRowTile;
+          t.dep_n = 1;
+          t.dep_need = need;
+          t.sig = l + 1 < depth[i] ? cnt_act(i, l) + m0 / kRowTile : -1;
           t.c_off = (*lay.act_off)[i][l];
           t.aux_off = (*lay.b_off)[i][l];
           v.push_back(t);
         }
     }
-    plan.fwd_rng[l] = sorted_append(v);
+    sorted_append(v);
   }
-  for (int l = Lmax - 1; l >= 0; --l) {
-    std::vector<TcTile> v;
+  plan.fwd_rng = {0, (int)all.size()};
+  for (int lev = 0; lev < Lmax; ++lev) {
+    std::vector<TcTile> vd, vw;
     for (int i = 0; i < m; ++i) {
-      if (!active[i] || depth[i] <= l) continue;
+      if (!active[i] || depth[i] <= lev) continue;
+      const int l = depth[i] - 1 - lev;
       const int w = width[i], in_pad = l == 0 ? lay.d_in_pad : w;
+      split_n(w, ns);
+      const int need = 8 * (int)ns.size();  // dgrad tiles of layer l + 1 per row block of dz_l
+      const bool from_head = l == depth[i] - 1;
       if (l > 0) {
-        split_n(w, ns);
-        for (int m0 = 0; m0 < lay.B_cap; m0 += 128)
+        for (int m0 = 0; m0 < lay.B_cap; m0 += kRowTile)
           for (auto& nn : ns) {
             TcTile t{};
             t.kind = kDgrad; t.member = i; t.layer = l;
@@ -641,14 +714,19 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
             t.map_b = plan.map_w[(size_t)i * kMaxDepth + l];
             t.ldc = w;
             t.ld_aux = w + kOnesCols;
+            t.dep = from_head ? -1 : cnt_dz(i, l) + m0 / kRowTile;
+            t.dep_n = 1;
+            t.dep_need = need;
+            t.sig = cnt_dz(i, l - 1) + m0 / kRowTile;
             t.c_off = (*lay.dz_off)[i][l - 1];
             t.aux_off = (*lay.act_off)[i][l - 1];
-            v.push_back(t);
+            vd.push_back(t);
           }
       }
-      split_n(in_pad + 1, ns);  // weight columns plus the bias column
-      for (int m0 = 0; m0 < w; m0 += 128)
-        for (auto& nn : ns) {
+      std::vector<std::pair<int, int>> nw;
+      split_n(in_pad + 1, nw);  // weight columns plus the bias column
+      for (int m0 = 0; m0 < w; m0 += kRowTile)
+        for (auto& nn : nw) {
           TcTile t{};
           t.kind = kWgrad; t.member = i; t.layer = l;
           t.m0 = m0; t.n0 = nn.first; t.n_len = nn.second;
@@ -658,13 +736,19 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
           t.map_b = l == 0 ? 0 : plan.map_act[(size_t)i * kMaxDepth + l - 1];
           t.ldc = in_pad;
           t.ld_aux = 0;
+          t.dep = from_head ? -1 : cnt_dz(i, l);  // every row block of dz_l
+          t.dep_n = 0;
+          t.dep_need = need;
+          t.sig = -1;
           t.c_off = (*lay.W_off)[i][l];
           t.aux_off = (*lay.b_off)[i][l];
-          v.push_back(t);
+          vw.push_back(t);
         }
     }
-    plan.bwd_rng[l] = sorted_append(v);
+    sorted_append(vd);
+    sorted_append(vw);
   }
+  plan.bwd_rng = {plan.fwd_rng.second, (int)all.size() - plan.fwd_rng.second};
   if ((int)all.size() + 1 > plan.cap_tiles) {
     if (plan.tiles_dev) cudaFree(plan.tiles_dev);
     plan.cap_tiles = (int)all.size() + 1;
@@ -690,6 +774,7 @@ static tp_status launch(TcPlan& plan, cudaStream_t st, const std::pair<int, int>
   a.n_tiles = rng.second;
   a.maps = plan.maps_dev;
   a.err = plan.err_dev;
+  a.cnt = plan.cnt_dev;
   const int grid = std::max(1, std::min(rng.second, plan.n_sm));
   launch_pdl(k_tc_gemm, dim3(grid), dim3(kThreads), kSmemBytes, st, a);
   cudaError_t e = cudaGetLastError();
@@ -700,9 +785,9 @@ static tp_status launch(TcPlan& plan, cudaStream_t st, const std::pair<int, int>
   return TP_OK;
 }
 
-tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, int wcur, uint32_t step,
-                     const StepDyn* dyn, int train, uint64_t seed, const float* params, const MemberDev* mem,
-                     void* act, std::string& err) {
+tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, uint32_t step, const StepDyn* dyn,
+                     int train, uint64_t seed, const float* params, const MemberDev* mem, void* act,
+                     std::string& err) {
   TcArgs a{};
   a.B = B;
   a.B_pad = B_pad;
@@ -715,11 +800,11 @@ tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad,
   a.params = params;
   a.mem = mem;
   a.act = (__nv_bfloat16*)act;
-  return launch(plan, st, plan.fwd_rng[layer], a, err);
+  return launch(plan, st, plan.fwd_rng, a, err);
 }
 
-tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, int wcur, const MemberDev* mem,
-                     void* act, void* dz, float* grads, int update, const AdamDev& adam, std::string& err) {
+tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, const MemberDev* mem, void* act,
+                     void* dz, float* grads, int update, const AdamDev& adam, std::string& err) {
   TcArgs a{};
   a.B = B;
   a.B_pad = B_pad;
@@ -730,7 +815,7 @@ tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad,
   a.dz = (__nv_bfloat16*)dz;
   a.grads = grads;
   a.adam = adam;
-  return launch(plan, st, plan.bwd_rng[layer], a, err);
+  return launch(plan, st, plan.bwd_rng, a, err);
 }
 
 tp_status tc_check(TcPlan& plan, cudaStream_t st, std::string& err) {
@@ -753,6 +838,9 @@ void tc_free_plan(TcPlan& plan) {
   if (plan.maps_dev) cudaFree(plan.maps_dev);
   if (plan.tiles_dev) cudaFree(plan.tiles_dev);
   if (plan.err_dev) cudaFree(plan.err_dev);
+  if (plan.cnt_dev) cudaFree(plan.cnt_dev);
+  plan.cnt_dev = nullptr;
+  plan.n_cnt = 0;
   plan.maps_dev = nullptr;
   plan.tiles_dev = nullptr;
   plan.err_dev = nullptr;

@@ -26,7 +26,12 @@ struct TcTile {
                            // kWgrad: n_real = in_pad + 1 (the bias column)
   int32_t k_len;           // reduction length (0: the step's padded batch)
   int32_t map_a, map_b;    // indices into the tensor-map table (weight maps of copy 0)
-  int32_t ldc, ld_aux, _pad;
+  int32_t ldc, ld_aux;
+  // Dataflow within one launch: before loading A the producer waits until
+  // counters dep .. dep + n - 1 (n = dep_n, or the step's B_pad / 128 when
+  // dep_n is 0) each reach dep_need; after storing its output every
+  // epilogue warp adds 1 to counter sig.  -1: none.
+  int32_t dep, dep_n, dep_need, sig;
   int64_t c_off;           // output: act (kFwd), dz (kDgrad), weight offset in the arena (kWgrad)
   int64_t aux_off;         // kFwd: bias offset in params; kDgrad: H_l offset in act (mask);
                            // kWgrad: bias offset in the arena
@@ -40,7 +45,12 @@ struct TcPlan {
   int w_shift = 0;         // index distance from a weight map of copy 0 to copy 1
   TcTile* tiles_dev = nullptr;
   int cap_tiles = 0;
-  std::vector<std::pair<int, int>> fwd_rng, bwd_rng;  // tile ranges per depth index
+  std::pair<int, int> fwd_rng, bwd_rng;  // tile ranges of the forward / backward launch
+  // Row-block completion counters: act of (member, layer) then dz of
+  // (member, layer), B_cap / 128 each.  They must be zero before a launch
+  // (the gather kernel that precedes every forward clears them).
+  int* cnt_dev = nullptr;
+  int n_cnt = 0;
   int* err_dev = nullptr;  // device error word (bounded waits that gave up)
   std::vector<int> map_act, map_dz, map_w;  // per (member * kMaxDepth + layer)
 };
@@ -61,16 +71,18 @@ struct TcLayout {          // what the plan needs to know about the pack's arena
 };
 
 tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err);
-// Forward products of hidden layer `layer`, reading weight copy `wcur`.
-// The dropout step counter is `step`, or dyn->step when dyn is non-NULL.
-tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, int wcur, uint32_t step,
-                     const StepDyn* dyn, int train, uint64_t seed, const float* params, const MemberDev* mem,
-                     void* act, std::string& err);
-// Backward products (dgrad + wgrad) of hidden layer `layer`.  update = 0: the
-// weight and bias gradients are stored in `grads`; update = 1: AdamW is
-// applied in the epilogue (adam.wq_out = the other weight copy).
-tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int layer, int B, int B_pad, int wcur, const MemberDev* mem,
-                     void* act, void* dz, float* grads, int update, const AdamDev& adam, std::string& err);
+// Forward products of every hidden layer of every active member (one
+// launch), reading weight copy `wcur`.  The dropout step counter is `step`,
+// or dyn->step when dyn is non-NULL.
+tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, uint32_t step, const StepDyn* dyn,
+                     int train, uint64_t seed, const float* params, const MemberDev* mem, void* act,
+                     std::string& err);
+// Backward products (dgrad + wgrad) of every hidden layer (one launch).
+// update = 0: the weight and bias gradients are stored in `grads`;
+// update = 1: AdamW is applied in the epilogue (adam.wq_out = the other
+// weight copy).
+tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, const MemberDev* mem, void* act,
+                     void* dz, float* grads, int update, const AdamDev& adam, std::string& err);
 // Reads and clears the device error word (synchronises the stream).
 tp_status tc_check(TcPlan& plan, cudaStream_t st, std::string& err);
 void tc_free_plan(TcPlan& plan);
