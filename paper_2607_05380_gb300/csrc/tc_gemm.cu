@@ -40,6 +40,8 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cstdio>
+#include <cstdlib>
 
 #include "tc_gemm.cuh"
 
@@ -89,6 +91,8 @@ struct TcArgs {
   int* err;
   const StepDyn* dyn;  // non-NULL: the dropout step counter is read from here
   int* cnt;            // row-block completion counters
+  int32_t cm, cn;      // cluster shape: cm row blocks x cn column tiles per cluster tile
+  int32_t kmaj_off;    // index distance to the same matrix's map with 128-row boxes (K-major loads)
 };
 
 // ------------------------------------------------------------ PTX helpers
@@ -120,8 +124,8 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 // Bounded wait: false if the abort flag is raised or the budget runs out
 // (then the flag and the device error word are set).
-__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* err,
-                                       uint64_t budget_ns) {
+__device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* err,
+                                            uint64_t budget_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_ns();
   while (true) {
@@ -133,6 +137,11 @@ __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile 
       return false;
     }
   }
+}
+
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* err,
+                                          uint64_t budget_ns) {
+  return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity, abort_flag, err, budget_ns);
 }
 
 __device__ __forceinline__ int ld_acquire(const int* p) {
@@ -174,8 +183,23 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y)
       : "memory");
 }
-__device__ __forceinline__ void tensormap_acquire(const CUtensorMap* map) {
-  asm volatile("fence.proxy.tensormap::generic.acquire.gpu [%0], 128;" ::"l"(map) : "memory");
+// The same box into the same shared-memory offset of every CTA in `mask`;
+// each destination's mbarrier at `bar`'s offset receives its bytes.
+__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const CUtensorMap* map, uint64_t* bar, int x, int y,
+                                               uint16_t mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster [%0], [%1, {%3, "
+      "%4}], [%2], %5;" ::"r"(dst),
+      "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y), "h"(mask)
+      : "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
@@ -209,6 +233,14 @@ __device__ __forceinline__ void umma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
                : "memory");
 }
+// Arrive on the mbarrier at `bar`'s offset in every CTA of `mask` once this
+// thread's MMAs so far have completed.
+__device__ __forceinline__ void umma_commit_mc(uint64_t* bar, uint16_t mask) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+                   smem_u32(bar)),
+               "h"(mask)
+               : "memory");
+}
 
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
   asm volatile(
@@ -229,6 +261,23 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 
 __device__ __forceinline__ bool tile_live(const TcTile& t, int B_pad) { return t.kind == kWgrad || t.m0 < B_pad; }
 
+// This CTA's part of a cluster tile: row block mi (rows m0 .. m0 + 127) and
+// column tile ni.  A part whose rows or columns lie beyond the product still
+// loads its share of the operands for its cluster peers but stores nothing.
+struct SubTile {
+  int m0, n0, n_len;
+  bool rows_live, n_live;
+};
+__device__ __forceinline__ SubTile sub_tile(const TcTile& t, int mi, int ni, int B_pad) {
+  SubTile u;
+  u.m0 = t.m0 + kRowTile * mi;
+  u.rows_live = u.m0 < (t.m_real ? t.m_real : B_pad);
+  u.n_live = ni == 0 || t.n_lenb > 0;
+  u.n0 = ni ? t.n0b : t.n0;
+  u.n_len = (ni && t.n_lenb) ? t.n_lenb : t.n_len;
+  return u;
+}
+
 // ------------------------------------------------------------------ kernel
 __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
   extern __shared__ uint8_t smem_raw[];
@@ -236,11 +285,22 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
   float* tr_all = (float*)(smem + kStages * kStageBytes);
   SmemTail* tl = (SmemTail*)(smem + kStages * kStageBytes + kTrBytes);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // Cluster of cm x cn CTAs: the cn CTAs of a row block share (multicast)
+  // its A tile, the cm CTAs of a column tile share its B tile, so each CTA
+  // reads 1 / cn of A and 1 / cm of B from L2.
+  const int cs = g.cm * g.cn;
+  const int rank = cs > 1 ? (int)cluster_rank() : 0;
+  const int mi = rank % g.cm, ni = rank / g.cm;
+  uint16_t row_mask = 0, col_mask = 0;
+  for (int q = 0; q < g.cn; ++q) row_mask |= (uint16_t)(1u << (mi + g.cm * q));
+  for (int q = 0; q < g.cm; ++q) col_mask |= (uint16_t)(1u << (q + g.cm * ni));
+  const uint16_t writers = row_mask | col_mask;  // CTAs whose copies land in this CTA's stages
+  const int clu = blockIdx.x / cs, n_clu = gridDim.x / cs;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&tl->full[s], 1);
-      mbar_init(&tl->empty[s], 1);
+      mbar_init(&tl->empty[s], g.cm + g.cn - 1);  // one MMA commit per writer CTA
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tl->tfull[b], 1);
@@ -259,6 +319,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  if (cs > 1) cluster_sync();  // every peer's barriers exist before the first multicast
   // The set-up above overlaps the previous kernel; data reads start here.  The
   // GEMM itself never triggers its dependents early: CTAs of the next kernel
   // parked beside a running GEMM measurably slow it down.
@@ -272,18 +333,28 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       uint32_t stage = 0, phase = 0;
       uint32_t issued_mask = 0, last_parity = 0;  // per stage: ever issued, parity of the last issue
       bool ok = true;
-      for (int t = blockIdx.x; ok && t < g.n_tiles; t += gridDim.x) {
+      for (int t = clu; ok && t < g.n_tiles; t += n_clu) {
         const TcTile tile = g.tiles[t];
         if (!tile_live(tile, g.B_pad)) continue;
+        const SubTile u = sub_tile(tile, mi, ni, g.B_pad);
         const int K = tile.k_len ? tile.k_len : g.B_pad;
-        const CUtensorMap* ma = g.maps + tile.map_a;
-        const CUtensorMap* mb = g.maps + tile.map_b + (tile.kind == kWgrad ? 0 : g.w_shift);
-        tensormap_acquire(ma);
-        tensormap_acquire(mb);
-        const int nb = (tile.n_len + 63) >> 6;
-        const uint32_t bytes = (uint32_t)(2 + nb) * kBoxBytes;
-        if (tile.dep >= 0 &&
-            !dep_wait(g.cnt + tile.dep, tile.dep_n ? tile.dep_n : g.B_pad / 128, tile.dep_need, abort_flag, g.err)) {
+        // Issue plan of the tile.  K-major operands (A of kFwd / kDgrad, B of
+        // kFwd) load 128-row boxes, MN-major ones 64 x 64 boxes; a box is
+        // issued by one CTA of its row (A) or column (B) group and
+        // multicast to the others.
+        const bool a_k = tile.kind != kWgrad, b_k = tile.kind == kFwd;
+        const CUtensorMap* ma = g.maps + tile.map_a + (a_k ? g.kmaj_off : 0);
+        const CUtensorMap* mb =
+            g.maps + tile.map_b + (tile.kind == kWgrad ? 0 : g.w_shift) + (b_k ? g.kmaj_off : 0);
+        const int nbB = b_k ? (u.n_len + 127) >> 7 : (u.n_len + 63) >> 6;
+        const uint32_t boxB = b_k ? 2 * kBoxBytes : kBoxBytes;
+        const uint32_t bytes = 2 * kBoxBytes + (uint32_t)nbB * boxB;
+        const uint32_t a_mine = a_k ? (ni == 0 ? 1u : 0u) : (g.cn > 1 ? 1u << ni : 3u);
+        uint32_t b_mine = 0;
+        for (int q = mi; q < nbB; q += g.cm) b_mine |= 1u << q;
+        if (u.rows_live && tile.dep >= 0 &&
+            !dep_wait(g.cnt + tile.dep + (tile.dep_n ? mi : 0), tile.dep_n ? tile.dep_n : g.B_pad / kRowTile,
+                      tile.dep_need, abort_flag, g.err)) {
           ok = false;
           break;
         }
@@ -296,16 +367,24 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           mbar_expect_tx(fb, bytes);
           const uint32_t a = smem_u32(smem + stage * kStageBytes);
           const uint32_t b = a + kABytes;
-          if (tile.kind == kWgrad) {  // A = dZ, MN-major: x = output row (unit), y = batch row
-            tma_load_2d(a, ma, fb, tile.m0, k0);
-            tma_load_2d(a + kBoxBytes, ma, fb, tile.m0 + 64, k0);
-          } else {  // A K-major: x = k, y = batch row
-            tma_load_2d(a, ma, fb, k0, tile.m0);
-            tma_load_2d(a + kBoxBytes, ma, fb, k0, tile.m0 + 64);
+          if (a_k) {
+            if (a_mine) {
+              if (g.cn > 1) tma_load_2d_mc(a, ma, fb, k0, u.m0, row_mask);
+              else tma_load_2d(a, ma, fb, k0, u.m0);
+            }
+          } else {
+            for (int h = 0; h < 2; ++h) {
+              if (!((a_mine >> h) & 1u)) continue;
+              if (g.cn > 1) tma_load_2d_mc(a + h * kBoxBytes, ma, fb, u.m0 + 64 * h, k0, row_mask);
+              else tma_load_2d(a + h * kBoxBytes, ma, fb, u.m0 + 64 * h, k0);
+            }
           }
-          for (int q = 0; q < nb; ++q) {
-            if (tile.kind == kFwd) tma_load_2d(b + q * kBoxBytes, mb, fb, k0, tile.n0 + 64 * q);
-            else tma_load_2d(b + q * kBoxBytes, mb, fb, tile.n0 + 64 * q, k0);
+          for (int q = 0; q < nbB; ++q) {
+            if (!((b_mine >> q) & 1u)) continue;
+            const int x = b_k ? k0 : u.n0 + 64 * q;
+            const int y = b_k ? u.n0 + 128 * q : k0;
+            if (g.cm > 1) tma_load_2d_mc(b + q * boxB, mb, fb, x, y, col_mask);
+            else tma_load_2d(b + q * boxB, mb, fb, x, y);
           }
           issued_mask |= 1u << stage;
           last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
@@ -315,7 +394,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           }
         }
       }
-      // wait (bounded) until every copy this thread issued has landed
+      // wait (bounded) until every copy into this CTA's stages has landed
       for (int s = 0; s < kStages; ++s)
         if (issued_mask & (1u << s)) {
           int dummy_abort = 0;
@@ -327,15 +406,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       // --------------------------------------------------------------- MMA
       uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
       bool ok = true;
-      for (int t = blockIdx.x; ok && t < g.n_tiles; t += gridDim.x) {
+      for (int t = clu; ok && t < g.n_tiles; t += n_clu) {
         const TcTile tile = g.tiles[t];
         if (!tile_live(tile, g.B_pad)) continue;
+        const SubTile u = sub_tile(tile, mi, ni, g.B_pad);
         const int K = tile.k_len ? tile.k_len : g.B_pad;
         if (!mbar_wait(&tl->tempty[acc], acc_phase ^ 1u, abort_flag, g.err, kWaitNs)) break;
         tc_fence_after();
         const uint32_t d = tmem + acc * kAccCols;
         const int a_mn = tile.kind == kWgrad, b_mn = tile.kind != kFwd;
-        const uint32_t idesc = instr_desc(tile.n_len, a_mn, b_mn);
+        const uint32_t idesc = instr_desc(u.n_len, a_mn, b_mn);
         for (int k0 = 0; k0 < K; k0 += 64) {
           if (!mbar_wait(&tl->full[stage], phase, abort_flag, g.err, kWaitNs)) {
             ok = false;
@@ -350,7 +430,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
             const uint64_t bd = b_mn ? smem_desc(b + kk * 2048, kBoxBytes, 1024) : smem_desc(b + kk * 32, 16, 1024);
             umma_bf16(d, ad, bd, idesc, (k0 | kk) != 0);
           }
-          umma_commit(&tl->empty[stage]);
+          // the stage is free once the MMAs of every CTA that reads a copy
+          // this CTA's producer wrote have completed
+          if (cs > 1) umma_commit_mc(&tl->empty[stage], writers);
+          else umma_commit(&tl->empty[stage]);
           if (++stage == kStages) {
             stage = 0;
             phase ^= 1u;
@@ -373,14 +456,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
     const int row = 32 * q + lane;
     const uint32_t step = g.dyn ? g.dyn->step : g.step;
     uint32_t acc = 0, acc_phase = 0;
-    for (int t = blockIdx.x; t < g.n_tiles; t += gridDim.x) {
+    for (int t = clu; t < g.n_tiles; t += n_clu) {
       const TcTile tile = g.tiles[t];
       if (!tile_live(tile, g.B_pad)) continue;
+      const SubTile u = sub_tile(tile, mi, ni, g.B_pad);
       if (!mbar_wait(&tl->tfull[acc], acc_phase, abort_flag, g.err, kWaitNs)) break;
       tc_fence_after();
       const MemberDev md = g.mem[tile.member];
       const int m_lim = tile.m_real ? tile.m_real : g.B_pad;
-      const int r = tile.m0 + row;
+      const int r = u.m0 + row;
       const bool row_ok = r < m_lim;
       const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + acc * kAccCols;
       float lr = 0.f, wd_w = 0.f, wd_b = 0.f, ib1 = 1.f, ib2 = 1.f;
@@ -393,8 +477,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         ib2 = 1.f / bc.y;
       }
       // the two warps of a lane quarter take alternate 32-column chunks
-      for (int c = 32 * half; c < tile.n_len; c += 64) {
-        const int col0 = tile.n0 + c;
+      const int n_end = u.rows_live && u.n_live ? u.n_len : 0;
+      for (int c = 32 * half; c < n_end; c += 64) {
+        const int col0 = u.n0 + c;
         const int ncols = min(32, tile.n_real - col0);
         const bool live = row_ok && ncols > 0;
         // forward: bias and dropout bits do not depend on the accumulator,
@@ -430,7 +515,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           const int in_pad = tile.n_real - 1;
           const int col = col0 + lane;
           const bool is_w = col < in_pad, is_b = col == in_pad;
-          const int rbase = tile.m0 + 32 * q;
+          const int rbase = u.m0 + 32 * q;
           const int nrows = min(32, m_lim - rbase);
           if (is_w || is_b) {
             const AdamDev& ad = g.adam;
@@ -513,12 +598,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       mbar_arrive(&tl->tempty[acc]);
       acc ^= 1u;
       if (acc == 0) acc_phase ^= 1u;
-      if (tile.sig >= 0) {  // publish this warp's part of the tile
+      if (tile.sig >= 0 && u.rows_live && u.n_live) {  // publish this warp's part of the tile
         __syncwarp();
         if (lane == 0) {
           fence_proxy_async_global();
           __threadfence();
-          red_release_add(g.cnt + tile.sig, 1);
+          red_release_add(g.cnt + tile.sig + mi, 1);
         }
       }
     }
@@ -527,6 +612,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  if (cs > 1) cluster_sync();  // no peer copies into or signals this CTA any more
   if (warp == 1) {
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
   }
@@ -546,8 +632,9 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
 }
 
 // 2-D bf16 row-major matrix [rows, cols] with row pitch `ld` elements,
-// 64 x 64 boxes, 128-byte swizzle.
-bool encode_map(CUtensorMap* m, const void* base, int64_t cols, int64_t rows, int64_t ld, std::string& err) {
+// boxes of 64 columns x box_rows rows, 128-byte swizzle.
+bool encode_map(CUtensorMap* m, const void* base, int64_t cols, int64_t rows, int64_t ld, int box_rows,
+                std::string& err) {
   auto fn = get_encode();
   if (!fn) {
     err = "cuTensorMapEncodeTiled unavailable";
@@ -555,7 +642,7 @@ bool encode_map(CUtensorMap* m, const void* base, int64_t cols, int64_t rows, in
   }
   cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
   cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
-  cuuint32_t box[2] = {64, 64};
+  cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
   cuuint32_t es[2] = {1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -583,39 +670,46 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
   const auto& width = *lay.width;
   const auto& active = *lay.active;
   if (plan.maps_dev == nullptr) {
-    // tensor maps: 0 = gathered batch [B_cap, d_in_pad + 16]; per (member,
-    // layer) act [B_cap, w + 16], dz [B_cap, w]; then the weights of copy 0,
-    // then the weights of copy 1 (w_shift apart)
+    // tensor maps, twice (64-row boxes for MN-major loads, then 128-row
+    // boxes for K-major loads, kmaj_off apart): 0 = gathered batch
+    // [B_cap, d_in_pad + 16]; per (member, layer) act [B_cap, w + 16],
+    // dz [B_cap, w]; then the weights of copy 0, then the weights of copy 1
+    // (w_shift apart)
     std::vector<CUtensorMap> maps;
     plan.map_act.assign((size_t)m * kMaxDepth, -1);
     plan.map_dz.assign((size_t)m * kMaxDepth, -1);
     plan.map_w.assign((size_t)m * kMaxDepth, -1);
     CUtensorMap mp;
-    if (!encode_map(&mp, lay.xb, lay.ldx, lay.B_cap, lay.ldx, err)) return TP_ECUDA;
-    maps.push_back(mp);
     const __nv_bfloat16* actb = (const __nv_bfloat16*)lay.act;
     const __nv_bfloat16* dzb = (const __nv_bfloat16*)lay.dz;
-    for (int i = 0; i < m; ++i)
-      for (int l = 0; l < depth[i]; ++l) {
-        const int w = width[i];
-        if (!encode_map(&mp, actb + (*lay.act_off)[i][l], w + kOnesCols, lay.B_cap, w + kOnesCols, err))
-          return TP_ECUDA;
-        plan.map_act[(size_t)i * kMaxDepth + l] = (int)maps.size();
-        maps.push_back(mp);
-        if (!encode_map(&mp, dzb + (*lay.dz_off)[i][l], w, lay.B_cap, w, err)) return TP_ECUDA;
-        plan.map_dz[(size_t)i * kMaxDepth + l] = (int)maps.size();
-        maps.push_back(mp);
-      }
-    const int w_base = (int)maps.size();
-    for (int copy = 0; copy < 2; ++copy)
+    for (int set = 0; set < 2; ++set) {
+      const int br = set ? 128 : 64;
+      const int base = (int)maps.size();
+      if (!encode_map(&mp, lay.xb, lay.ldx, lay.B_cap, lay.ldx, br, err)) return TP_ECUDA;
+      maps.push_back(mp);
       for (int i = 0; i < m; ++i)
         for (int l = 0; l < depth[i]; ++l) {
-          const int w = width[i], in_pad = l == 0 ? lay.d_in_pad : w;
-          if (!encode_map(&mp, lay.wq[copy] + (*lay.W_off)[i][l], in_pad, w, in_pad, err)) return TP_ECUDA;
-          if (copy == 0) plan.map_w[(size_t)i * kMaxDepth + l] = (int)maps.size();
+          const int w = width[i];
+          if (!encode_map(&mp, actb + (*lay.act_off)[i][l], w + kOnesCols, lay.B_cap, w + kOnesCols, br, err))
+            return TP_ECUDA;
+          if (set == 0) plan.map_act[(size_t)i * kMaxDepth + l] = (int)maps.size();
+          maps.push_back(mp);
+          if (!encode_map(&mp, dzb + (*lay.dz_off)[i][l], w, lay.B_cap, w, br, err)) return TP_ECUDA;
+          if (set == 0) plan.map_dz[(size_t)i * kMaxDepth + l] = (int)maps.size();
           maps.push_back(mp);
         }
-    plan.w_shift = ((int)maps.size() - w_base) / 2;
+      const int w_base = (int)maps.size();
+      for (int copy = 0; copy < 2; ++copy)
+        for (int i = 0; i < m; ++i)
+          for (int l = 0; l < depth[i]; ++l) {
+            const int w = width[i], in_pad = l == 0 ? lay.d_in_pad : w;
+            if (!encode_map(&mp, lay.wq[copy] + (*lay.W_off)[i][l], in_pad, w, in_pad, br, err)) return TP_ECUDA;
+            if (set == 0 && copy == 0) plan.map_w[(size_t)i * kMaxDepth + l] = (int)maps.size();
+            maps.push_back(mp);
+          }
+      plan.w_shift = ((int)maps.size() - w_base) / 2;
+      if (set == 1) plan.kmaj_off = base;
+    }
     plan.n_maps = (int)maps.size();
     if (cudaMalloc(&plan.maps_dev, sizeof(CUtensorMap) * maps.size()) != cudaSuccess) {
       err = "cudaMalloc(tensor maps) failed";
@@ -636,6 +730,48 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
     if (cudaFuncSetAttribute(k_tc_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess) {
       err = "cudaFuncSetAttribute(smem) failed";
       return TP_ECUDA;
+    }
+    // Cluster shape.  Sharing the weight tile between two row blocks (2 x 1)
+    // cuts the L2 -> SM operand traffic by a third; it pays when every SM has
+    // many K blocks to stream (wide members, large batches) and costs a few
+    // resident CTAs and idle halves otherwise.  TP_CLUSTER=<cm>x<cn> (each 1
+    // or 2) overrides the choice.
+    int64_t fwd_kblocks = 0;
+    for (int i = 0; i < m; ++i)
+      for (int l = 0; l < depth[i]; ++l) {
+        const int in_pad = l == 0 ? lay.d_in_pad : width[i];
+        fwd_kblocks += (lay.B_cap / kRowTile) * ceil_div(width[i], 256) * ceil_div(in_pad, 64);
+      }
+    plan.cm = fwd_kblocks >= 100 * (int64_t)plan.n_sm ? 2 : 1;
+    plan.cn = 1;
+    if (const char* e = getenv("TP_CLUSTER")) {
+      int a = 0, b = 0;
+      if (sscanf(e, "%dx%d", &a, &b) == 2 && (a == 1 || a == 2) && (b == 1 || b == 2)) {
+        plan.cm = a;
+        plan.cn = b;
+      }
+    }
+    plan.max_clusters = plan.n_sm;
+    const int cs = plan.cm * plan.cn;
+    if (cs > 1) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(cs * plan.n_sm);
+      cfg.blockDim = dim3(kThreads);
+      cfg.dynamicSmemBytes = kSmemBytes;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = cs;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      int n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, (void*)k_tc_gemm, &cfg) == cudaSuccess && n >= 1) {
+        plan.max_clusters = n;
+      } else {
+        cudaGetLastError();
+        plan.cm = plan.cn = 1;
+      }
     }
   }
 
@@ -662,6 +798,25 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
     std::stable_sort(v.begin(), v.end(), [&](const TcTile& a, const TcTile& b) { return cost(a) > cost(b); });
     all.insert(all.end(), v.begin(), v.end());
   };
+  // The cluster tiles of one product: R row blocks and the column tiles ns,
+  // cm x cn at a time; proto.dep / proto.sig are the counters of row block 0.
+  const int cm = plan.cm, cn = plan.cn;
+  auto emit = [&](std::vector<TcTile>& v, const TcTile& proto, int R, const std::vector<std::pair<int, int>>& ns) {
+    const int n_pad = (int)round_up(proto.n_real, 64);  // a column origin past the product (TMA zero fill)
+    for (int rb = 0; rb < R; rb += cm)
+      for (int j = 0; j < (int)ns.size(); j += cn) {
+        TcTile t = proto;
+        t.m0 = rb * kRowTile;
+        t.n0 = ns[j].first;
+        t.n_len = ns[j].second;
+        const bool second = cn > 1 && j + 1 < (int)ns.size();
+        t.n0b = second ? ns[j + 1].first : n_pad;
+        t.n_lenb = second ? ns[j + 1].second : 0;
+        if (proto.dep >= 0 && proto.dep_n == 1) t.dep = proto.dep + rb;
+        if (proto.sig >= 0) t.sig = proto.sig + rb;
+        v.push_back(t);
+      }
+  };
   std::vector<std::pair<int, int>> ns;
   for (int l = 0; l < Lmax; ++l) {
     std::vector<TcTile> v;
@@ -669,26 +824,21 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
       if (!active[i] || depth[i] <= l) continue;
       const int w = width[i];
       split_n(w, ns);
-      const int need = 8 * (int)ns.size();  // every epilogue warp of every N tile of a row block
-      for (int m0 = 0; m0 < lay.B_cap; m0 += kRowTile)
-        for (auto& nn : ns) {
-          TcTile t{};
-          t.kind = kFwd; t.member = i; t.layer = l;
-          t.m0 = m0; t.n0 = nn.first; t.n_len = nn.second;
-          t.m_real = 0; t.n_real = w;
-          t.k_len = l == 0 ? lay.d_in_pad : w;
-          t.map_a = l == 0 ? 0 : plan.map_act[(size_t)i * kMaxDepth + l - 1];
-          t.map_b = plan.map_w[(size_t)i * kMaxDepth + l];
-          t.ldc = w + kOnesCols;
-          t.ld_aux = 0;
-          t.dep = l == 0 ? -1 : cnt_act(i, l - 1) + m0 / kRowTile;
-          t.dep_n = 1;
-          t.dep_need = need;
-          t.sig = l + 1 < depth[i] ? cnt_act(i, l) + m0 / kRowTile : -1;
-          t.c_off = (*lay.act_off)[i][l];
-          t.aux_off = (*lay.b_off)[i][l];
-          v.push_back(t);
-        }
+      TcTile t{};
+      t.kind = kFwd; t.member = i; t.layer = l;
+      t.m_real = 0; t.n_real = w;
+      t.k_len = l == 0 ? lay.d_in_pad : w;
+      t.map_a = l == 0 ? 0 : plan.map_act[(size_t)i * kMaxDepth + l - 1];
+      t.map_b = plan.map_w[(size_t)i * kMaxDepth + l];
+      t.ldc = w + kOnesCols;
+      t.ld_aux = 0;
+      t.dep = l == 0 ? -1 : cnt_act(i, l - 1);
+      t.dep_n = 1;
+      t.dep_need = 8 * (int)ns.size();  // every epilogue warp of every column tile of a row block
+      t.sig = l + 1 < depth[i] ? cnt_act(i, l) : -1;
+      t.c_off = (*lay.act_off)[i][l];
+      t.aux_off = (*lay.b_off)[i][l];
+      emit(v, t, lay.B_cap / kRowTile, ns);
     }
     sorted_append(v);
   }
@@ -700,50 +850,42 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
       const int l = depth[i] - 1 - lev;
       const int w = width[i], in_pad = l == 0 ? lay.d_in_pad : w;
       split_n(w, ns);
-      const int need = 8 * (int)ns.size();  // dgrad tiles of layer l + 1 per row block of dz_l
+      const int need = 8 * (int)ns.size();  // dgrad column tiles of layer l + 1 per row block of dz_l
       const bool from_head = l == depth[i] - 1;
       if (l > 0) {
-        for (int m0 = 0; m0 < lay.B_cap; m0 += kRowTile)
-          for (auto& nn : ns) {
-            TcTile t{};
-            t.kind = kDgrad; t.member = i; t.layer = l;
-            t.m0 = m0; t.n0 = nn.first; t.n_len = nn.second;
-            t.m_real = 0; t.n_real = w;
-            t.k_len = w;
-            t.map_a = plan.map_dz[(size_t)i * kMaxDepth + l];
-            t.map_b = plan.map_w[(size_t)i * kMaxDepth + l];
-            t.ldc = w;
-            t.ld_aux = w + kOnesCols;
-            t.dep = from_head ? -1 : cnt_dz(i, l) + m0 / kRowTile;
-            t.dep_n = 1;
-            t.dep_need = need;
-            t.sig = cnt_dz(i, l - 1) + m0 / kRowTile;
-            t.c_off = (*lay.dz_off)[i][l - 1];
-            t.aux_off = (*lay.act_off)[i][l - 1];
-            vd.push_back(t);
-          }
+        TcTile t{};
+        t.kind = kDgrad; t.member = i; t.layer = l;
+        t.m_real = 0; t.n_real = w;
+        t.k_len = w;
+        t.map_a = plan.map_dz[(size_t)i * kMaxDepth + l];
+        t.map_b = plan.map_w[(size_t)i * kMaxDepth + l];
+        t.ldc = w;
+        t.ld_aux = w + kOnesCols;
+        t.dep = from_head ? -1 : cnt_dz(i, l);
+        t.dep_n = 1;
+        t.dep_need = need;
+        t.sig = cnt_dz(i, l - 1);
+        t.c_off = (*lay.dz_off)[i][l - 1];
+        t.aux_off = (*lay.act_off)[i][l - 1];
+        emit(vd, t, lay.B_cap / kRowTile, ns);
       }
       std::vector<std::pair<int, int>> nw;
       split_n(in_pad + 1, nw);  // weight columns plus the bias column
-      for (int m0 = 0; m0 < w; m0 += kRowTile)
-        for (auto& nn : nw) {
-          TcTile t{};
-          t.kind = kWgrad; t.member = i; t.layer = l;
-          t.m0 = m0; t.n0 = nn.first; t.n_len = nn.second;
-          t.m_real = w; t.n_real = in_pad + 1;
-          t.k_len = 0;
-          t.map_a = plan.map_dz[(size_t)i * kMaxDepth + l];
-          t.map_b = l == 0 ? 0 : plan.map_act[(size_t)i * kMaxDepth + l - 1];
-          t.ldc = in_pad;
-          t.ld_aux = 0;
-          t.dep = from_head ? -1 : cnt_dz(i, l);  // every row block of dz_l
-          t.dep_n = 0;
-          t.dep_need = need;
-          t.sig = -1;
-          t.c_off = (*lay.W_off)[i][l];
-          t.aux_off = (*lay.b_off)[i][l];
-          vw.push_back(t);
-        }
+      TcTile t{};
+      t.kind = kWgrad; t.member = i; t.layer = l;
+      t.m_real = w; t.n_real = in_pad + 1;
+      t.k_len = 0;
+      t.map_a = plan.map_dz[(size_t)i * kMaxDepth + l];
+      t.map_b = l == 0 ? 0 : plan.map_act[(size_t)i * kMaxDepth + l - 1];
+      t.ldc = in_pad;
+      t.ld_aux = 0;
+      t.dep = from_head ? -1 : cnt_dz(i, l);  // every row block of dz_l
+      t.dep_n = 0;
+      t.dep_need = need;
+      t.sig = -1;
+      t.c_off = (*lay.W_off)[i][l];
+      t.aux_off = (*lay.b_off)[i][l];
+      emit(vw, t, (int)ceil_div(w, kRowTile), nw);
     }
     sorted_append(vd);
     sorted_append(vw);
@@ -775,9 +917,28 @@ static tp_status launch(TcPlan& plan, cudaStream_t st, const std::pair<int, int>
   a.maps = plan.maps_dev;
   a.err = plan.err_dev;
   a.cnt = plan.cnt_dev;
-  const int grid = std::max(1, std::min(rng.second, plan.n_sm));
-  launch_pdl(k_tc_gemm, dim3(grid), dim3(kThreads), kSmemBytes, st, a);
-  cudaError_t e = cudaGetLastError();
+  a.cm = plan.cm;
+  a.cn = plan.cn;
+  a.kmaj_off = plan.kmaj_off;
+  const int cs = plan.cm * plan.cn;
+  // every CTA resident at once (the dataflow waits rely on it)
+  const int n_clu = std::max(1, std::min(rng.second, plan.max_clusters));
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(n_clu * cs);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = cs;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = cs > 1 ? 2 : 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, k_tc_gemm, a);
+  if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) {
     err = std::string("tcgen05 GEMM launch: ") + cudaGetErrorString(e);
     return TP_ECUDA;
