@@ -328,79 +328,81 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
   volatile int* abort_flag = &tl->abort;
 
   if (warp == 0) {
-    if (lane == 0) {
-      // ---------------------------------------------------------- producer
-      uint32_t stage = 0, phase = 0;
-      uint32_t issued_mask = 0, last_parity = 0;  // per stage: ever issued, parity of the last issue
-      bool ok = true;
-      for (int t = clu; ok && t < g.n_tiles; t += n_clu) {
-        const TcTile tile = g.tiles[t];
-        if (!tile_live(tile, g.B_pad)) continue;
-        const SubTile u = sub_tile(tile, mi, ni, g.B_pad);
-        const int K = tile.k_len ? tile.k_len : g.B_pad;
-        // Issue plan of the tile.  K-major operands (A of kFwd / kDgrad, B of
-        // kFwd) load 128-row boxes, MN-major ones 64 x 64 boxes; a box is
-        // issued by one CTA of its row (A) or column (B) group and
-        // multicast to the others.
-        const bool a_k = tile.kind != kWgrad, b_k = tile.kind == kFwd;
-        const CUtensorMap* ma = g.maps + tile.map_a + (a_k ? g.kmaj_off : 0);
-        const CUtensorMap* mb =
-            g.maps + tile.map_b + (tile.kind == kWgrad ? 0 : g.w_shift) + (b_k ? g.kmaj_off : 0);
-        const int nbB = b_k ? (u.n_len + 127) >> 7 : (u.n_len + 63) >> 6;
-        const uint32_t boxB = b_k ? 2 * kBoxBytes : kBoxBytes;
-        const uint32_t bytes = 2 * kBoxBytes + (uint32_t)nbB * boxB;
-        const uint32_t a_mine = a_k ? (ni == 0 ? 1u : 0u) : (g.cn > 1 ? 1u << ni : 3u);
-        uint32_t b_mine = 0;
-        for (int q = mi; q < nbB; q += g.cm) b_mine |= 1u << q;
-        if (u.rows_live && tile.dep >= 0 &&
-            !dep_wait(g.cnt + tile.dep + (tile.dep_n ? mi : 0), tile.dep_n ? tile.dep_n : g.B_pad / kRowTile,
-                      tile.dep_need, abort_flag, g.err)) {
+    // ------------------------------------------------------------ producer
+    // The whole warp walks the tiles; lane 0 waits for free stages and posts
+    // the expected bytes, then lane j issues TMA box j of the K block, so the
+    // boxes of a stage leave in parallel instead of one after another.
+    uint32_t stage = 0, phase = 0;
+    uint32_t issued_mask = 0, last_parity = 0;  // per stage: ever issued, parity of the last issue
+    bool ok = true;
+    for (int t = clu; ok && t < g.n_tiles; t += n_clu) {
+      const TcTile tile = g.tiles[t];
+      if (!tile_live(tile, g.B_pad)) continue;
+      const SubTile u = sub_tile(tile, mi, ni, g.B_pad);
+      const int K = tile.k_len ? tile.k_len : g.B_pad;
+      // Issue plan of the tile.  K-major operands (A of kFwd / kDgrad, B of
+      // kFwd) load 128-row boxes, MN-major ones 64 x 64 boxes; a box is
+      // issued by one CTA of its row (A) or column (B) group and multicast
+      // to the others.
+      const bool a_k = tile.kind != kWgrad, b_k = tile.kind == kFwd;
+      const int nbA = a_k ? 1 : 2;
+      const int nbB = b_k ? (u.n_len + 127) >> 7 : (u.n_len + 63) >> 6;
+      const uint32_t boxB = b_k ? 2 * kBoxBytes : kBoxBytes;
+      const uint32_t bytes = 2 * kBoxBytes + (uint32_t)nbB * boxB;
+      // this lane's box: lane < nbA: A box `lane`; then B box `lane - nbA`
+      const bool is_a = lane < nbA;
+      const int qb = lane - nbA;
+      bool mine;
+      if (is_a) mine = a_k ? ni == 0 : (g.cn > 1 ? lane == ni : true);
+      else mine = qb < nbB && qb % g.cm == mi;
+      const CUtensorMap* map =
+          is_a ? g.maps + tile.map_a + (a_k ? g.kmaj_off : 0)
+               : g.maps + tile.map_b + (tile.kind == kWgrad ? 0 : g.w_shift) + (b_k ? g.kmaj_off : 0);
+      const bool mn = is_a ? !a_k : !b_k;                 // MN-major box: x = row / column, y = k
+      const int xy0 = is_a ? u.m0 + 64 * lane : u.n0 + (b_k ? 128 : 64) * qb;
+      const uint32_t off = is_a ? (uint32_t)lane * kBoxBytes : (uint32_t)kABytes + (uint32_t)qb * boxB;
+      const bool mc = is_a ? g.cn > 1 : g.cm > 1;
+      const uint16_t mask = is_a ? row_mask : col_mask;
+      bool dep_ok = true;
+      if (lane == 0 && u.rows_live && tile.dep >= 0)
+        dep_ok = dep_wait(g.cnt + tile.dep + (tile.dep_n ? mi : 0), tile.dep_n ? tile.dep_n : g.B_pad / kRowTile,
+                          tile.dep_need, abort_flag, g.err);
+      if (!__shfl_sync(0xffffffffu, dep_ok, 0)) {
+        ok = false;
+        break;
+      }
+      if (tile.dep >= 0) fence_proxy_async_global();  // every issuing lane, after lane 0's acquire
+      for (int k0 = 0; k0 < K; k0 += 64) {
+        bool got = true;
+        if (lane == 0) {
+          got = mbar_wait(&tl->empty[stage], phase ^ 1u, abort_flag, g.err, kWaitNs);
+          if (got) mbar_expect_tx(&tl->full[stage], bytes);
+        }
+        if (!__shfl_sync(0xffffffffu, got, 0)) {
           ok = false;
           break;
         }
-        for (int k0 = 0; k0 < K; k0 += 64) {
-          if (!mbar_wait(&tl->empty[stage], phase ^ 1u, abort_flag, g.err, kWaitNs)) {
-            ok = false;
-            break;
-          }
-          uint64_t* fb = &tl->full[stage];
-          mbar_expect_tx(fb, bytes);
-          const uint32_t a = smem_u32(smem + stage * kStageBytes);
-          const uint32_t b = a + kABytes;
-          if (a_k) {
-            if (a_mine) {
-              if (g.cn > 1) tma_load_2d_mc(a, ma, fb, k0, u.m0, row_mask);
-              else tma_load_2d(a, ma, fb, k0, u.m0);
-            }
-          } else {
-            for (int h = 0; h < 2; ++h) {
-              if (!((a_mine >> h) & 1u)) continue;
-              if (g.cn > 1) tma_load_2d_mc(a + h * kBoxBytes, ma, fb, u.m0 + 64 * h, k0, row_mask);
-              else tma_load_2d(a + h * kBoxBytes, ma, fb, u.m0 + 64 * h, k0);
-            }
-          }
-          for (int q = 0; q < nbB; ++q) {
-            if (!((b_mine >> q) & 1u)) continue;
-            const int x = b_k ? k0 : u.n0 + 64 * q;
-            const int y = b_k ? u.n0 + 128 * q : k0;
-            if (g.cm > 1) tma_load_2d_mc(b + q * boxB, mb, fb, x, y, col_mask);
-            else tma_load_2d(b + q * boxB, mb, fb, x, y);
-          }
-          issued_mask |= 1u << stage;
-          last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
-          if (++stage == kStages) {
-            stage = 0;
-            phase ^= 1u;
-          }
+        if (mine) {
+          const uint32_t dst = smem_u32(smem + stage * kStageBytes) + off;
+          const int x = mn ? xy0 : k0, y = mn ? k0 : xy0;
+          if (mc) tma_load_2d_mc(dst, map, &tl->full[stage], x, y, mask);
+          else tma_load_2d(dst, map, &tl->full[stage], x, y);
+        }
+        issued_mask |= 1u << stage;
+        last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1u;
         }
       }
-      // wait (bounded) until every copy into this CTA's stages has landed
+    }
+    // wait (bounded) until every copy into this CTA's stages has landed
+    if (lane == 0)
       for (int s = 0; s < kStages; ++s)
         if (issued_mask & (1u << s)) {
           int dummy_abort = 0;
           mbar_wait(&tl->full[s], (last_parity >> s) & 1u, &dummy_abort, g.err, kWaitNs);
         }
-    }
   } else if (warp == 1) {
     if (lane == 0) {
       // --------------------------------------------------------------- MMA
