@@ -48,16 +48,29 @@
 namespace tp {
 namespace {
 
-constexpr int kStages = 4;
 constexpr int kBoxBytes = 64 * 64 * 2;  // one 64 x 64 bf16 TMA box
-constexpr int kABytes = 2 * kBoxBytes;  // 128 rows
-constexpr int kBBytes = 4 * kBoxBytes;  // up to 256 rows / columns
-constexpr int kStageBytes = kABytes + kBBytes;
-constexpr int kThreads = 320;  // 2 role warps + 8 epilogue warps
+constexpr int kABytes = 2 * kBoxBytes;  // 128 rows of A per CTA
+constexpr int kThreads = 320;           // 2 role warps + 8 epilogue warps
 constexpr uint32_t kTmemCols = 512;
 constexpr int kAccCols = 256;
 constexpr uint64_t kWaitNs = 2000000000ull;
+// per epilogue warp a 32 x 33 fp32 transpose buffer (wgrad epilogue)
+constexpr int kTrPitch = 33;
+constexpr int kTrBytes = 8 * 32 * kTrPitch * 4;
 
+// Pipeline geometry for tiles of kCta CTAs.  kCta = 1: a CTA computes
+// 128 x N and stages 128 rows of A and up to 256 rows / columns of B per K
+// block (48 KB, 4 stages).  kCta = 2: a CTA pair computes 256 x N with
+// cta_group::2 MMAs; each CTA stages its own 128 rows of A and half of B
+// (32 KB, 6 stages), so a CTA streams two thirds of the bytes per FLOP and
+// keeps half again as many K blocks in flight.
+template <int kCta>
+struct Geo {
+  static constexpr int kStages = kCta == 2 ? 6 : 4;
+  static constexpr int kBBytes = (kCta == 2 ? 2 : 4) * kBoxBytes;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+};
+template <int kStages>
 struct SmemTail {
   uint64_t full[kStages];
   uint64_t empty[kStages];
@@ -67,10 +80,12 @@ struct SmemTail {
   uint32_t tmem_base;
   int abort;
 };
-// per epilogue warp a 32 x 33 fp32 transpose buffer (wgrad epilogue)
-constexpr int kTrPitch = 33;
-constexpr int kTrBytes = 8 * 32 * kTrPitch * 4;
-constexpr int kSmemBytes = kStages * kStageBytes + kTrBytes + 1024 + (int)sizeof(SmemTail) + 64;
+template <int kCta>
+constexpr int smem_bytes() {
+  return Geo<kCta>::kStages * Geo<kCta>::kStageBytes + kTrBytes + 1024 +
+         (int)sizeof(SmemTail<Geo<kCta>::kStages>) + 64;
+}
+static_assert(smem_bytes<1>() <= 232448 && smem_bytes<2>() <= 232448, "shared memory per CTA");
 
 struct TcArgs {
   const TcTile* tiles;
@@ -91,7 +106,6 @@ struct TcArgs {
   int* err;
   const StepDyn* dyn;  // non-NULL: the dropout step counter is read from here
   int* cnt;            // row-block completion counters
-  int32_t cm, cn;      // cluster shape: cm row blocks x cn column tiles per cluster tile
   int32_t kmaj_off;    // index distance to the same matrix's map with 128-row boxes (K-major loads)
 };
 
@@ -183,15 +197,24 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y)
       : "memory");
 }
-// The same box into the same shared-memory offset of every CTA in `mask`;
-// each destination's mbarrier at `bar`'s offset receives its bytes.
-__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const CUtensorMap* map, uint64_t* bar, int x, int y,
-                                               uint16_t mask) {
+// Copy of a box into this CTA's shared memory whose completion is counted on
+// the mbarrier at shared::cluster address `bar`, which may belong to the
+// peer CTA of the pair (cta_group::2).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y) {
   asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster [%0], [%1, {%3, "
-      "%4}], [%2], %5;" ::"r"(dst),
-      "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y), "h"(mask)
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], "
+      "[%2];" ::"r"(dst),
+      "l"(map), "r"(bar), "r"(x), "r"(y)
       : "memory");
+}
+// shared::cluster address of this CTA's shared variable at `addr` in CTA `rank`
+__device__ __forceinline__ uint32_t mapa(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar) : "memory");
 }
 __device__ __forceinline__ uint32_t cluster_rank() {
   uint32_t r;
@@ -217,29 +240,39 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint3
 }
 
 // Instruction descriptor of kind::f16: fp32 accumulate, bf16 A and B.
-__device__ __forceinline__ uint32_t instr_desc(int n, int a_mn, int b_mn) {
+__device__ __forceinline__ uint32_t instr_desc(int m, int n, int a_mn, int b_mn) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)a_mn << 15) | ((uint32_t)b_mn << 16) |
-         ((uint32_t)(n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+         ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
 }
 
+template <int kCta>
 __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
-          d_tmem),
-      "l"(a), "l"(b), "r"(idesc), "r"(acc)
-      : "memory");
+  if constexpr (kCta == 2)
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
+            d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"(acc)
+        : "memory");
+  else
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
+            d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"(acc)
+        : "memory");
 }
+// Arrive on `bar` once this thread's MMAs so far have completed; for a CTA
+// pair on the mbarrier at `bar`'s offset in both CTAs.
+template <int kCta>
 __device__ __forceinline__ void umma_commit(uint64_t* bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
-               : "memory");
-}
-// Arrive on the mbarrier at `bar`'s offset in every CTA of `mask` once this
-// thread's MMAs so far have completed.
-__device__ __forceinline__ void umma_commit_mc(uint64_t* bar, uint16_t mask) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
-                   smem_u32(bar)),
-               "h"(mask)
-               : "memory");
+  if constexpr (kCta == 2)
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+            smem_u32(bar)),
+        "h"((uint16_t)3)
+        : "memory");
+  else
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+                 : "memory");
 }
 
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
@@ -261,65 +294,65 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
 
 __device__ __forceinline__ bool tile_live(const TcTile& t, int B_pad) { return t.kind == kWgrad || t.m0 < B_pad; }
 
-// This CTA's part of a cluster tile: row block mi (rows m0 .. m0 + 127) and
-// column tile ni.  A part whose rows or columns lie beyond the product still
-// loads its share of the operands for its cluster peers but stores nothing.
+// This CTA's rows of a tile: row block `mi` of the tile (rows m0 .. m0 + 127).
+// Rows beyond the product still load their share of the operands for the
+// peer CTA but store nothing.
 struct SubTile {
-  int m0, n0, n_len;
-  bool rows_live, n_live;
+  int m0;
+  bool rows_live;
 };
-__device__ __forceinline__ SubTile sub_tile(const TcTile& t, int mi, int ni, int B_pad) {
+__device__ __forceinline__ SubTile sub_tile(const TcTile& t, int mi, int B_pad) {
   SubTile u;
   u.m0 = t.m0 + kRowTile * mi;
   u.rows_live = u.m0 < (t.m_real ? t.m_real : B_pad);
-  u.n_live = ni == 0 || t.n_lenb > 0;
-  u.n0 = ni ? t.n0b : t.n0;
-  u.n_len = (ni && t.n_lenb) ? t.n_lenb : t.n_len;
   return u;
 }
 
 // ------------------------------------------------------------------ kernel
+template <int kCta>
 __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
+  using G = Geo<kCta>;
+  constexpr int kStages = G::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  float* tr_all = (float*)(smem + kStages * kStageBytes);
-  SmemTail* tl = (SmemTail*)(smem + kStages * kStageBytes + kTrBytes);
+  float* tr_all = (float*)(smem + kStages * G::kStageBytes);
+  SmemTail<kStages>* tl = (SmemTail<kStages>*)(smem + kStages * G::kStageBytes + kTrBytes);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // Cluster of cm x cn CTAs: the cn CTAs of a row block share (multicast)
-  // its A tile, the cm CTAs of a column tile share its B tile, so each CTA
-  // reads 1 / cn of A and 1 / cm of B from L2.
-  const int cs = g.cm * g.cn;
-  const int rank = cs > 1 ? (int)cluster_rank() : 0;
-  const int mi = rank % g.cm, ni = rank / g.cm;
-  uint16_t row_mask = 0, col_mask = 0;
-  for (int q = 0; q < g.cn; ++q) row_mask |= (uint16_t)(1u << (mi + g.cm * q));
-  for (int q = 0; q < g.cm; ++q) col_mask |= (uint16_t)(1u << (q + g.cm * ni));
-  const uint16_t writers = row_mask | col_mask;  // CTAs whose copies land in this CTA's stages
-  const int clu = blockIdx.x / cs, n_clu = gridDim.x / cs;
+  const int rank = kCta == 2 ? (int)cluster_rank() : 0;  // row block of the tile this CTA holds
+  const bool leader = rank == 0;                         // issues the pair's MMAs
+  const int clu = blockIdx.x / kCta, n_clu = gridDim.x / kCta;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&tl->full[s], 1);
-      mbar_init(&tl->empty[s], g.cm + g.cn - 1);  // one MMA commit per writer CTA
+      mbar_init(&tl->empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tl->tfull[b], 1);
-      mbar_init(&tl->tempty[b], 256);
+      mbar_init(&tl->tempty[b], 8 * kCta);  // one arrival per epilogue warp of the pair
     }
     mbar_init(&tl->done, 1);
     tl->abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tl->tmem_base)),
-                 "r"(kTmemCols)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    // one warp of each CTA of the pair allocates collectively
+    if constexpr (kCta == 2) {
+      asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tl->tmem_base)),
+                   "r"(kTmemCols)
+                   : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+    } else {
+      asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tl->tmem_base)),
+                   "r"(kTmemCols)
+                   : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (cs > 1) cluster_sync();  // every peer's barriers exist before the first multicast
+  if (kCta == 2) cluster_sync();  // the peer's barriers exist before any copy or arrival targets them
   // The set-up above overlaps the previous kernel; data reads start here.  The
   // GEMM itself never triggers its dependents early: CTAs of the next kernel
   // parked beside a running GEMM measurably slow it down.
@@ -331,41 +364,39 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
     // ------------------------------------------------------------ producer
     // The whole warp walks the tiles; lane 0 waits for free stages and posts
     // the expected bytes, then lane j issues TMA box j of the K block, so the
-    // boxes of a stage leave in parallel instead of one after another.
+    // boxes of a stage leave in parallel instead of one after another.  In a
+    // CTA pair both CTAs' copies complete on the leader's full barrier, which
+    // the leader expects for both.
     uint32_t stage = 0, phase = 0;
     uint32_t issued_mask = 0, last_parity = 0;  // per stage: ever issued, parity of the last issue
     bool ok = true;
     for (int t = clu; ok && t < g.n_tiles; t += n_clu) {
       const TcTile tile = g.tiles[t];
       if (!tile_live(tile, g.B_pad)) continue;
-      const SubTile u = sub_tile(tile, mi, ni, g.B_pad);
+      const SubTile u = sub_tile(tile, rank, g.B_pad);
       const int K = tile.k_len ? tile.k_len : g.B_pad;
-      // Issue plan of the tile.  K-major operands (A of kFwd / kDgrad, B of
-      // kFwd) load 128-row boxes, MN-major ones 64 x 64 boxes; a box is
-      // issued by one CTA of its row (A) or column (B) group and multicast
-      // to the others.
+      // K-major operands (A of kFwd / kDgrad, B of kFwd) load 128-row boxes,
+      // MN-major ones 64 x 64 boxes.  This CTA's B: all n_len rows / columns
+      // (kCta 1) or its half of them (kCta 2).
       const bool a_k = tile.kind != kWgrad, b_k = tile.kind == kFwd;
       const int nbA = a_k ? 1 : 2;
-      const int nbB = b_k ? (u.n_len + 127) >> 7 : (u.n_len + 63) >> 6;
+      const int nh = tile.n_len / kCta;
+      const int bn0 = tile.n0 + rank * nh;
+      const int nbB = b_k ? (nh + 127) >> 7 : (nh + 63) >> 6;
       const uint32_t boxB = b_k ? 2 * kBoxBytes : kBoxBytes;
-      const uint32_t bytes = 2 * kBoxBytes + (uint32_t)nbB * boxB;
-      // this lane's box: lane < nbA: A box `lane`; then B box `lane - nbA`
-      const bool is_a = lane < nbA;
+      const uint32_t bytes = (uint32_t)kCta * (2 * kBoxBytes + (uint32_t)nbB * boxB);
+      const bool is_a = lane < nbA;  // lane < nbA: A box `lane`; then B box `lane - nbA`
       const int qb = lane - nbA;
-      bool mine;
-      if (is_a) mine = a_k ? ni == 0 : (g.cn > 1 ? lane == ni : true);
-      else mine = qb < nbB && qb % g.cm == mi;
+      const bool mine = is_a || qb < nbB;
       const CUtensorMap* map =
           is_a ? g.maps + tile.map_a + (a_k ? g.kmaj_off : 0)
                : g.maps + tile.map_b + (tile.kind == kWgrad ? 0 : g.w_shift) + (b_k ? g.kmaj_off : 0);
-      const bool mn = is_a ? !a_k : !b_k;                 // MN-major box: x = row / column, y = k
-      const int xy0 = is_a ? u.m0 + 64 * lane : u.n0 + (b_k ? 128 : 64) * qb;
+      const bool mn = is_a ? !a_k : !b_k;  // MN-major box: x = row / column, y = k
+      const int xy0 = is_a ? u.m0 + 64 * lane : bn0 + (b_k ? 128 : 64) * qb;
       const uint32_t off = is_a ? (uint32_t)lane * kBoxBytes : (uint32_t)kABytes + (uint32_t)qb * boxB;
-      const bool mc = is_a ? g.cn > 1 : g.cm > 1;
-      const uint16_t mask = is_a ? row_mask : col_mask;
       bool dep_ok = true;
       if (lane == 0 && u.rows_live && tile.dep >= 0)
-        dep_ok = dep_wait(g.cnt + tile.dep + (tile.dep_n ? mi : 0), tile.dep_n ? tile.dep_n : g.B_pad / kRowTile,
+        dep_ok = dep_wait(g.cnt + tile.dep + (tile.dep_n ? rank : 0), tile.dep_n ? tile.dep_n : g.B_pad / kRowTile,
                           tile.dep_need, abort_flag, g.err);
       if (!__shfl_sync(0xffffffffu, dep_ok, 0)) {
         ok = false;
@@ -376,16 +407,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         bool got = true;
         if (lane == 0) {
           got = mbar_wait(&tl->empty[stage], phase ^ 1u, abort_flag, g.err, kWaitNs);
-          if (got) mbar_expect_tx(&tl->full[stage], bytes);
+          if (got && leader) mbar_expect_tx(&tl->full[stage], bytes);
         }
         if (!__shfl_sync(0xffffffffu, got, 0)) {
           ok = false;
           break;
         }
         if (mine) {
-          const uint32_t dst = smem_u32(smem + stage * kStageBytes) + off;
+          const uint32_t dst = smem_u32(smem + stage * G::kStageBytes) + off;
           const int x = mn ? xy0 : k0, y = mn ? k0 : xy0;
-          if (mc) tma_load_2d_mc(dst, map, &tl->full[stage], x, y, mask);
+          if constexpr (kCta == 2) tma_load_2d_pair(dst, map, mapa(smem_u32(&tl->full[stage]), 0), x, y);
           else tma_load_2d(dst, map, &tl->full[stage], x, y);
         }
         issued_mask |= 1u << stage;
@@ -396,58 +427,55 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         }
       }
     }
-    // wait (bounded) until every copy into this CTA's stages has landed
-    if (lane == 0)
+    // wait (bounded) until every copy counted on this CTA's full barriers has
+    // landed (in a pair the leader's barriers count both CTAs' copies)
+    if (lane == 0 && leader)
       for (int s = 0; s < kStages; ++s)
         if (issued_mask & (1u << s)) {
           int dummy_abort = 0;
           mbar_wait(&tl->full[s], (last_parity >> s) & 1u, &dummy_abort, g.err, kWaitNs);
         }
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && leader) {
       // --------------------------------------------------------------- MMA
       uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
       bool ok = true;
       for (int t = clu; ok && t < g.n_tiles; t += n_clu) {
         const TcTile tile = g.tiles[t];
         if (!tile_live(tile, g.B_pad)) continue;
-        const SubTile u = sub_tile(tile, mi, ni, g.B_pad);
         const int K = tile.k_len ? tile.k_len : g.B_pad;
         if (!mbar_wait(&tl->tempty[acc], acc_phase ^ 1u, abort_flag, g.err, kWaitNs)) break;
         tc_fence_after();
         const uint32_t d = tmem + acc * kAccCols;
         const int a_mn = tile.kind == kWgrad, b_mn = tile.kind != kFwd;
-        const uint32_t idesc = instr_desc(u.n_len, a_mn, b_mn);
+        const uint32_t idesc = instr_desc(128 * kCta, tile.n_len, a_mn, b_mn);
         for (int k0 = 0; k0 < K; k0 += 64) {
           if (!mbar_wait(&tl->full[stage], phase, abort_flag, g.err, kWaitNs)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t a = smem_u32(smem + stage * kStageBytes);
+          const uint32_t a = smem_u32(smem + stage * G::kStageBytes);
           const uint32_t b = a + kABytes;
           const int nk = min(4, (K - k0 + 15) >> 4);
           for (int kk = 0; kk < nk; ++kk) {
             const uint64_t ad = a_mn ? smem_desc(a + kk * 2048, kBoxBytes, 1024) : smem_desc(a + kk * 32, 16, 1024);
             const uint64_t bd = b_mn ? smem_desc(b + kk * 2048, kBoxBytes, 1024) : smem_desc(b + kk * 32, 16, 1024);
-            umma_bf16(d, ad, bd, idesc, (k0 | kk) != 0);
+            umma_bf16<kCta>(d, ad, bd, idesc, (k0 | kk) != 0);
           }
-          // the stage is free once the MMAs of every CTA that reads a copy
-          // this CTA's producer wrote have completed
-          if (cs > 1) umma_commit_mc(&tl->empty[stage], writers);
-          else umma_commit(&tl->empty[stage]);
+          umma_commit<kCta>(&tl->empty[stage]);  // the stage is free in every CTA of the tile
           if (++stage == kStages) {
             stage = 0;
             phase ^= 1u;
           }
         }
         if (!ok) break;
-        umma_commit(&tl->tfull[acc]);
+        umma_commit<kCta>(&tl->tfull[acc]);
         acc ^= 1u;
         if (acc == 0) acc_phase ^= 1u;
       }
       // all MMAs this thread issued have completed before TMEM is freed
-      umma_commit(&tl->done);
+      umma_commit<kCta>(&tl->done);
       int dummy_abort = 0;
       mbar_wait(&tl->done, 0, &dummy_abort, g.err, kWaitNs);
     }
@@ -461,7 +489,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
     for (int t = clu; t < g.n_tiles; t += n_clu) {
       const TcTile tile = g.tiles[t];
       if (!tile_live(tile, g.B_pad)) continue;
-      const SubTile u = sub_tile(tile, mi, ni, g.B_pad);
+      const SubTile u = sub_tile(tile, rank, g.B_pad);
       if (!mbar_wait(&tl->tfull[acc], acc_phase, abort_flag, g.err, kWaitNs)) break;
       tc_fence_after();
       const MemberDev md = g.mem[tile.member];
@@ -479,9 +507,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         ib2 = 1.f / bc.y;
       }
       // the two warps of a lane quarter take alternate 32-column chunks
-      const int n_end = u.rows_live && u.n_live ? u.n_len : 0;
+      const int n_end = u.rows_live ? tile.n_len : 0;
       for (int c = 32 * half; c < n_end; c += 64) {
-        const int col0 = u.n0 + c;
+        const int col0 = tile.n0 + c;
         const int ncols = min(32, tile.n_real - col0);
         const bool live = row_ok && ncols > 0;
         // forward: bias and dropout bits do not depend on the accumulator,
@@ -596,16 +624,22 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           }
         }
       }
+      // this warp has read its part of the accumulator: release it to the
+      // MMA issuer (the leader CTA's barrier in a pair)
       tc_fence_before();
-      mbar_arrive(&tl->tempty[acc]);
+      __syncwarp();
+      if (lane == 0) {
+        if constexpr (kCta == 2) mbar_arrive_cluster(mapa(smem_u32(&tl->tempty[acc]), 0));
+        else mbar_arrive(&tl->tempty[acc]);
+      }
       acc ^= 1u;
       if (acc == 0) acc_phase ^= 1u;
-      if (tile.sig >= 0 && u.rows_live && u.n_live) {  // publish this warp's part of the tile
+      if (tile.sig >= 0 && u.rows_live) {  // publish this warp's part of the tile
         __syncwarp();
         if (lane == 0) {
           fence_proxy_async_global();
           __threadfence();
-          red_release_add(g.cnt + tile.sig + mi, 1);
+          red_release_add(g.cnt + tile.sig + rank, 1);
         }
       }
     }
@@ -614,9 +648,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (cs > 1) cluster_sync();  // no peer copies into or signals this CTA any more
+  if (kCta == 2) cluster_sync();  // the pair's MMAs, copies and arrivals are over
   if (warp == 1) {
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+    if constexpr (kCta == 2)
+      asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+    else
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
   }
 }
 
@@ -729,50 +766,48 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
     int dev = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&plan.n_sm, cudaDevAttrMultiProcessorCount, dev);
-    if (cudaFuncSetAttribute(k_tc_gemm, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess) {
+    if (cudaFuncSetAttribute(k_tc_gemm<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<1>()) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(k_tc_gemm<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<2>()) !=
+            cudaSuccess) {
       err = "cudaFuncSetAttribute(smem) failed";
       return TP_ECUDA;
     }
-    // Cluster shape.  Sharing the weight tile between two row blocks (2 x 1)
-    // cuts the L2 -> SM operand traffic by a third; it pays when every SM has
-    // many K blocks to stream (wide members, large batches) and costs a few
-    // resident CTAs and idle halves otherwise.  TP_CLUSTER=<cm>x<cn> (each 1
-    // or 2) overrides the choice.
+    // CTAs per tile.  A CTA pair (256-row tiles, cta_group::2) streams two
+    // thirds of the operand bytes per FLOP and keeps more K blocks in flight;
+    // it pays when every SM has many K blocks to stream (wide members, large
+    // batches) and costs idle halves and a few resident CTAs otherwise.
+    // TP_GEMM_CTAS=1|2 overrides the choice.
     int64_t fwd_kblocks = 0;
     for (int i = 0; i < m; ++i)
       for (int l = 0; l < depth[i]; ++l) {
         const int in_pad = l == 0 ? lay.d_in_pad : width[i];
         fwd_kblocks += (lay.B_cap / kRowTile) * ceil_div(width[i], 256) * ceil_div(in_pad, 64);
       }
-    plan.cm = fwd_kblocks >= 100 * (int64_t)plan.n_sm ? 2 : 1;
-    plan.cn = 1;
-    if (const char* e = getenv("TP_CLUSTER")) {
-      int a = 0, b = 0;
-      if (sscanf(e, "%dx%d", &a, &b) == 2 && (a == 1 || a == 2) && (b == 1 || b == 2)) {
-        plan.cm = a;
-        plan.cn = b;
-      }
+    plan.cta = fwd_kblocks >= 100 * (int64_t)plan.n_sm ? 2 : 1;
+    if (const char* e = getenv("TP_GEMM_CTAS")) {
+      const int v = atoi(e);
+      if (v == 1 || v == 2) plan.cta = v;
     }
     plan.max_clusters = plan.n_sm;
-    const int cs = plan.cm * plan.cn;
-    if (cs > 1) {
+    if (plan.cta == 2) {
       cudaLaunchConfig_t cfg = {};
-      cfg.gridDim = dim3(cs * plan.n_sm);
+      cfg.gridDim = dim3(2 * plan.n_sm);
       cfg.blockDim = dim3(kThreads);
-      cfg.dynamicSmemBytes = kSmemBytes;
+      cfg.dynamicSmemBytes = smem_bytes<2>();
       cudaLaunchAttribute attr[1];
       attr[0].id = cudaLaunchAttributeClusterDimension;
-      attr[0].val.clusterDim.x = cs;
+      attr[0].val.clusterDim.x = 2;
       attr[0].val.clusterDim.y = 1;
       attr[0].val.clusterDim.z = 1;
       cfg.attrs = attr;
       cfg.numAttrs = 1;
       int n = 0;
-      if (cudaOccupancyMaxActiveClusters(&n, (void*)k_tc_gemm, &cfg) == cudaSuccess && n >= 1) {
+      if (cudaOccupancyMaxActiveClusters(&n, (void*)k_tc_gemm<2>, &cfg) == cudaSuccess && n >= 1) {
         plan.max_clusters = n;
       } else {
         cudaGetLastError();
-        plan.cm = plan.cn = 1;
+        plan.cta = 1;
       }
     }
   }
@@ -800,20 +835,16 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
     std::stable_sort(v.begin(), v.end(), [&](const TcTile& a, const TcTile& b) { return cost(a) > cost(b); });
     all.insert(all.end(), v.begin(), v.end());
   };
-  // The cluster tiles of one product: R row blocks and the column tiles ns,
-  // cm x cn at a time; proto.dep / proto.sig are the counters of row block 0.
-  const int cm = plan.cm, cn = plan.cn;
+  // The tiles of one product: R row blocks (plan.cta at a time) by the
+  // column tiles ns; proto.dep / proto.sig are the counters of row block 0.
+  const int cta = plan.cta;
   auto emit = [&](std::vector<TcTile>& v, const TcTile& proto, int R, const std::vector<std::pair<int, int>>& ns) {
-    const int n_pad = (int)round_up(proto.n_real, 64);  // a column origin past the product (TMA zero fill)
-    for (int rb = 0; rb < R; rb += cm)
-      for (int j = 0; j < (int)ns.size(); j += cn) {
+    for (int rb = 0; rb < R; rb += cta)
+      for (const auto& nn : ns) {
         TcTile t = proto;
         t.m0 = rb * kRowTile;
-        t.n0 = ns[j].first;
-        t.n_len = ns[j].second;
-        const bool second = cn > 1 && j + 1 < (int)ns.size();
-        t.n0b = second ? ns[j + 1].first : n_pad;
-        t.n_lenb = second ? ns[j + 1].second : 0;
+        t.n0 = nn.first;
+        t.n_len = nn.second;
         if (proto.dep >= 0 && proto.dep_n == 1) t.dep = proto.dep + rb;
         if (proto.sig >= 0) t.sig = proto.sig + rb;
         v.push_back(t);
@@ -919,27 +950,25 @@ static tp_status launch(TcPlan& plan, cudaStream_t st, const std::pair<int, int>
   a.maps = plan.maps_dev;
   a.err = plan.err_dev;
   a.cnt = plan.cnt_dev;
-  a.cm = plan.cm;
-  a.cn = plan.cn;
   a.kmaj_off = plan.kmaj_off;
-  const int cs = plan.cm * plan.cn;
+  const int cta = plan.cta;
   // every CTA resident at once (the dataflow waits rely on it)
   const int n_clu = std::max(1, std::min(rng.second, plan.max_clusters));
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(n_clu * cs);
+  cfg.gridDim = dim3(n_clu * cta);
   cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.dynamicSmemBytes = cta == 2 ? smem_bytes<2>() : smem_bytes<1>();
   cfg.stream = st;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   attr[1].id = cudaLaunchAttributeClusterDimension;
-  attr[1].val.clusterDim.x = cs;
+  attr[1].val.clusterDim.x = cta;
   attr[1].val.clusterDim.y = 1;
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = cs > 1 ? 2 : 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, k_tc_gemm, a);
+  cfg.numAttrs = cta == 2 ? 2 : 1;
+  cudaError_t e = cta == 2 ? cudaLaunchKernelEx(&cfg, k_tc_gemm<2>, a) : cudaLaunchKernelEx(&cfg, k_tc_gemm<1>, a);
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) {
     err = std::string("tcgen05 GEMM launch: ") + cudaGetErrorString(e);

@@ -14,10 +14,8 @@
 
 namespace tp {
 
-// One cluster tile of one member's product: cm row blocks of 128 rows from
-// m0 and cn (1 or 2) column tiles, n0 / n_len and n0b / n_lenb (n_lenb = 0:
-// no second column tile; its CTAs only load their operand share).  With a
-// 1 x 1 cluster it is one 128 x n_len output tile.
+// One output tile of one member's product: 128 * (CTAs per tile) rows from
+// m0 (a CTA pair holds row blocks m0 and m0 + 128) by n_len columns from n0.
 //   kFwd   C[b, j]  = sum_k H[b, k] W[j, k]         A = H (K-major), B = W (K-major)
 //   kDgrad C[b, k]  = sum_j dZ[b, j] W[j, k]        A = dZ (K-major), B = W (MN-major)
 //   kWgrad C[j, k]  = sum_b dZ[b, j] [H | 1][b, k]  A = dZ (MN-major), B = [H | 1] (MN-major);
@@ -31,12 +29,11 @@ struct TcTile {
   int32_t map_a, map_b;    // indices into the tensor-map table (weight maps of copy 0)
   int32_t ldc, ld_aux;
   // Dataflow within one launch: before loading A the producer of row block
-  // mi waits until counters d .. d + n - 1 each reach dep_need (dep_n = 1:
-  // d = dep + mi, n = 1; dep_n = 0: d = dep, n = the step's B_pad / 128);
-  // after storing its output every epilogue warp adds 1 to counter sig + mi.
-  // -1: none.
-  int32_t dep, dep_n, dep_need, sig;
-  int32_t n0b, n_lenb;
+  // mi of the tile waits until counters d .. d + n - 1 each reach dep_need
+  // (dep_n = 1: d = dep + mi, n = 1; dep_n = 0: d = dep, n = the step's
+  // B_pad / 128); after storing its output every epilogue warp adds 1 to
+  // counter sig + mi.  -1: none.
+  int32_t dep, dep_n, dep_need, sig, _pad;
   int64_t c_off;           // output: act (kFwd), dz (kDgrad), weight offset in the arena (kWgrad)
   int64_t aux_off;         // kFwd: bias offset in params; kDgrad: H_l offset in act (mask);
                            // kWgrad: bias offset in the arena
@@ -57,8 +54,8 @@ struct TcPlan {
   // (the gather kernel that precedes every forward clears them).
   int* cnt_dev = nullptr;
   int n_cnt = 0;
-  int cm = 1, cn = 1;      // cluster shape (row blocks x column tiles per cluster tile)
-  int max_clusters = 0;    // clusters that can be resident at once
+  int cta = 1;             // CTAs per tile (2: CTA pairs with cta_group::2 MMAs)
+  int max_clusters = 0;    // tiles in flight at once (resident CTAs / cta)
   int* err_dev = nullptr;  // device error word (bounded waits that gave up)
   std::vector<int> map_act, map_dz, map_w;  // per (member * kMaxDepth + layer)
 };
