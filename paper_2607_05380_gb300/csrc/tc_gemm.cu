@@ -292,6 +292,12 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&t);
 }
 
+// a[i] for a runtime i < 4 without indexing (keeps a[] in registers)
+template <typename V>
+__device__ __forceinline__ V pick4(const V (&a)[4], int i) {
+  return i == 0 ? a[0] : i == 1 ? a[1] : i == 2 ? a[2] : a[3];
+}
+
 __device__ __forceinline__ bool tile_live(const TcTile& t, int B_pad) { return t.kind == kWgrad || t.m0 < B_pad; }
 
 // This CTA's rows of a tile: row block `mi` of the tile (rows m0 .. m0 + 127).
@@ -490,12 +496,54 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       const TcTile tile = g.tiles[t];
       if (!tile_live(tile, g.B_pad)) continue;
       const SubTile u = sub_tile(tile, rank, g.B_pad);
-      if (!mbar_wait(&tl->tfull[acc], acc_phase, abort_flag, g.err, kWaitNs)) break;
-      tc_fence_after();
       const MemberDev md = g.mem[tile.member];
       const int m_lim = tile.m_real ? tile.m_real : g.B_pad;
       const int r = u.m0 + row;
       const bool row_ok = r < m_lim;
+      // the two warps of a lane quarter take alternate 32-column chunks:
+      // chunk ci covers columns 32 * half + 64 * ci .. + 31 of the tile
+      const int n_end = u.rows_live ? tile.n_len : 0;
+      // Inputs that do not depend on the accumulator are prepared while the
+      // tile's MMAs run: forward, this lane's bias value of each chunk
+      // (column = lane; broadcast by shuffles) and the 32 dropout keep bits of
+      // its row; dgrad, the 32 ReLU-mask bits of its row.
+      float bias_l[4];
+      uint32_t bits[4];
+#pragma unroll
+      for (int ci = 0; ci < 4; ++ci) {
+        const int c = 32 * half + 64 * ci;
+        const int col0 = tile.n0 + c;
+        const int ncols = min(32, tile.n_real - col0);
+        bias_l[ci] = 0.f;
+        bits[ci] = 0xFFFFFFFFu;
+        if (c >= n_end || ncols <= 0) continue;
+        if (tile.kind == kFwd) {
+          if (lane < ncols) bias_l[ci] = __ldg(g.params + tile.aux_off + col0 + lane);
+          if (row_ok && g.train && md.drop_T) {
+            uint32_t keep = 0;
+#pragma unroll
+            for (int g4 = 0; g4 < 8; ++g4)
+              keep |= keep_bits4(g.seed, (uint32_t)tile.member, (uint32_t)tile.layer, step, (uint32_t)r,
+                                 (uint32_t)((col0 >> 2) + g4), md.drop_T)
+                      << (4 * g4);
+            bits[ci] = keep;
+          }
+        } else if (tile.kind == kDgrad && row_ok) {
+          const __nv_bfloat16* hm = g.act + tile.aux_off + (int64_t)r * tile.ld_aux + col0;
+          uint32_t mb = 0;
+#pragma unroll
+          for (int s = 0; s < 4; ++s) {
+            if (8 * s >= ncols) break;
+            const uint4 hv = *reinterpret_cast<const uint4*>(hm + 8 * s);
+            const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&hv);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) mb |= (uint32_t)(__bfloat162float(hb[e]) > 0.f) << (8 * s + e);
+          }
+          bits[ci] = mb;
+        }
+      }
+      if (!mbar_wait(&tl->tfull[acc], acc_phase, abort_flag, g.err, kWaitNs)) break;
+      tc_fence_after();
       const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + acc * kAccCols;
       float lr = 0.f, wd_w = 0.f, wd_b = 0.f, ib1 = 1.f, ib2 = 1.f;
       if (tile.kind == kWgrad && g.update) {
@@ -506,32 +554,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         ib1 = 1.f / bc.x;
         ib2 = 1.f / bc.y;
       }
-      // the two warps of a lane quarter take alternate 32-column chunks
-      const int n_end = u.rows_live ? tile.n_len : 0;
-      for (int c = 32 * half; c < n_end; c += 64) {
+#pragma unroll 1
+      for (int ci = 0; ci < 4; ++ci) {
+        const int c = 32 * half + 64 * ci;
+        if (c >= n_end) break;
         const int col0 = tile.n0 + c;
         const int ncols = min(32, tile.n_real - col0);
         const bool live = row_ok && ncols > 0;
-        // forward: bias and dropout bits do not depend on the accumulator,
-        // so they are fetched / generated before the TMEM load
-        float bias[32];
-        uint32_t keep = 0xFFFFFFFFu;
-        if (tile.kind == kFwd && live) {
-          const float4* b4 = reinterpret_cast<const float4*>(g.params + tile.aux_off + col0);
-#pragma unroll
-          for (int s = 0; s < 8; ++s) {
-            const float4 t4 = 4 * s < ncols ? __ldg(b4 + s) : make_float4(0.f, 0.f, 0.f, 0.f);
-            bias[4 * s] = t4.x; bias[4 * s + 1] = t4.y; bias[4 * s + 2] = t4.z; bias[4 * s + 3] = t4.w;
-          }
-          if (g.train && md.drop_T) {
-            keep = 0;
-#pragma unroll
-            for (int g4 = 0; g4 < 8; ++g4)
-              keep |= keep_bits4(g.seed, (uint32_t)tile.member, (uint32_t)tile.layer, step, (uint32_t)r,
-                                 (uint32_t)((col0 >> 2) + g4), md.drop_T)
-                      << (4 * g4);
-          }
-        }
         uint32_t v[32];
         tmem_ld32(taddr + c, v);
         if (tile.kind == kWgrad) {
@@ -582,8 +611,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           __syncwarp();  // the buffer is reused by the next chunk
           continue;
         }
-        if (!live) continue;
         if (tile.kind == kFwd) {  // ncols: a multiple of 8 (widths are multiples of 16)
+          float bias[32];
+          const float bl = pick4(bias_l, ci);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) bias[j] = __shfl_sync(0xffffffffu, bl, j);
+          if (!live) continue;
+          const uint32_t keep = pick4(bits, ci);
           const float sc = g.train ? md.scale : 1.f;
           __nv_bfloat16* out = g.act + tile.c_off + (int64_t)r * tile.ldc + col0;
 #pragma unroll
@@ -605,19 +639,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
             *reinterpret_cast<uint4*>(out + 8 * s) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
           }
         } else if (tile.kind == kDgrad) {
-          const __nv_bfloat16* hm = g.act + tile.aux_off + (int64_t)r * tile.ld_aux + col0;
+          if (!live) continue;
+          const uint32_t mb = pick4(bits, ci);
           __nv_bfloat16* out = g.dz + tile.c_off + (int64_t)r * tile.ldc + col0;
 #pragma unroll
           for (int s = 0; s < 4; ++s) {
             if (8 * s >= ncols) break;
-            const uint4 hv = *reinterpret_cast<const uint4*>(hm + 8 * s);
-            const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&hv);
             uint32_t pk[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
               const int j = 8 * s + 2 * e;
-              const float x0 = __bfloat162float(hb[2 * e]) > 0.f ? __uint_as_float(v[j]) * md.scale : 0.f;
-              const float x1 = __bfloat162float(hb[2 * e + 1]) > 0.f ? __uint_as_float(v[j + 1]) * md.scale : 0.f;
+              const float x0 = ((mb >> j) & 1u) ? __uint_as_float(v[j]) * md.scale : 0.f;
+              const float x1 = ((mb >> (j + 1)) & 1u) ? __uint_as_float(v[j + 1]) * md.scale : 0.f;
               pk[e] = pack_bf16x2(x0, x1);
             }
             *reinterpret_cast<uint4*>(out + 8 * s) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
