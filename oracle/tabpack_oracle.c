@@ -132,6 +132,17 @@ struct orc_pack {
 
 static double* orc_zeros(int64_t n) { return (double*)calloc((size_t)(n > 0 ? n : 1), sizeof(double)); }
 
+/* Column-major copy t[c * rows + r] = a[r * cols + c] of a row-major
+ * [rows, cols] matrix: a sum over r then reads consecutive memory.  Only the
+ * memory layout changes; every product and the order of every sum stay those
+ * of the plain loops over the row-major matrix.                              */
+static double* orc_transpose(const double* a, int64_t rows, int64_t cols) {
+  double* t = orc_zeros(rows * cols);
+  for (int64_t r = 0; r < rows; ++r)
+    for (int64_t c = 0; c < cols; ++c) t[c * rows + r] = a[r * cols + c];
+  return t;
+}
+
 static void orc_free_cache(orc_member* M) {
   if (M->Hin) for (int l = 0; l <= M->L; ++l) free(M->Hin[l]);
   if (M->Z) for (int l = 0; l < M->L; ++l) free(M->Z[l]);
@@ -325,17 +336,21 @@ static double orc_member_backward(const orc_pack* h, orc_member* M, const int32_
   loss /= (double)B;
   for (int64_t e = 0; e < (int64_t)B * d_out; ++e) dlog[e] /= (double)B;
 
-  /* head */
+  /* head: dW_h[c, j] = sum_b dlogits[b, c] H_L[b, j] (b increasing) */
+  double* dlogT = orc_transpose(dlog, B, d_out);
+  double* HT = orc_transpose(M->Hin[L], B, w);
   for (int c = 0; c < d_out; ++c) {
     for (int j = 0; j < w; ++j) {
       double g = 0.0;
-      for (int b = 0; b < B; ++b) g += dlog[(int64_t)b * d_out + c] * M->Hin[L][(int64_t)b * w + j];
+      for (int b = 0; b < B; ++b) g += dlogT[(int64_t)c * B + b] * HT[(int64_t)j * B + b];
       M->gW[L][(int64_t)c * w + j] = g;
     }
     double gb = 0.0;
     for (int b = 0; b < B; ++b) gb += dlog[(int64_t)b * d_out + c];
     M->gb[L][c] = gb;
   }
+  free(dlogT);
+  free(HT);
   double* dH = orc_zeros((int64_t)B * w);
   for (int b = 0; b < B; ++b)
     for (int j = 0; j < w; ++j) {
@@ -353,26 +368,36 @@ static double orc_member_backward(const orc_pack* h, orc_member* M, const int32_
       double g = (M->keep[l][e] && M->Z[l][e] > 0.0) ? dH[e] / (1.0 - (double)M->p) : 0.0;
       dZ[e] = orc_st(h, g);
     }
+    /* dW[j, k] = sum_b dZ[b, j] H_l[b, k], db[j] = sum_b dZ[b, j] (b increasing) */
+    double* dZT = orc_transpose(dZ, B, w);
+    double* HT_l = orc_transpose(M->Hin[l], B, in);
     for (int j = 0; j < w; ++j) {
       for (int k = 0; k < in; ++k) {
         double g = 0.0;
-        for (int b = 0; b < B; ++b) g += dZ[(int64_t)b * w + j] * M->Hin[l][(int64_t)b * in + k];
+        for (int b = 0; b < B; ++b) g += dZT[(int64_t)j * B + b] * HT_l[(int64_t)k * B + b];
         M->gW[l][(int64_t)j * in + k] = g;
       }
       double gb = 0.0;
-      for (int b = 0; b < B; ++b) gb += dZ[(int64_t)b * w + j];
+      for (int b = 0; b < B; ++b) gb += dZT[(int64_t)j * B + b];
       M->gb[l][j] = gb;
     }
+    free(dZT);
+    free(HT_l);
     free(dH);
     dH = NULL;
     if (l > 0) {
+      /* dH_l[b, k] = sum_j dZ[b, j] W_l[j, k] (j increasing), W as stored */
+      double* WT = orc_zeros((int64_t)in * w);
+      for (int j = 0; j < w; ++j)
+        for (int k = 0; k < in; ++k) WT[(int64_t)k * w + j] = orc_st(h, M->W[l][(int64_t)j * in + k]);
       dH = orc_zeros((int64_t)B * in);
       for (int b = 0; b < B; ++b)
         for (int k = 0; k < in; ++k) {
           double s = 0.0;
-          for (int j = 0; j < w; ++j) s += dZ[(int64_t)b * w + j] * orc_st(h, M->W[l][(int64_t)j * in + k]);
+          for (int j = 0; j < w; ++j) s += dZ[(int64_t)b * w + j] * WT[(int64_t)k * w + j];
           dH[(int64_t)b * in + k] = s;
         }
+      free(WT);
     }
     free(dZ);
   }
