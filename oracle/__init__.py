@@ -74,6 +74,7 @@ def lib():
                 "orc_train_step": (ctypes.c_int, [P, P, i64, P, P, P, i32, u32, i32, P]),
                 "orc_predict": (ctypes.c_int, [P, P, i64, P]),
                 "orc_set_active": (ctypes.c_int, [P, P]),
+                "orc_adamw_apply": (None, [P, P, P, P, i64, i64, f64, f64, f64, f64, f64]),
                 "orc_get_params": (ctypes.c_int, [P, i32, i32, P, P]),
                 "orc_set_params": (ctypes.c_int, [P, i32, i32, P, P]),
                 "orc_get_grads": (ctypes.c_int, [P, i32, i32, P, P]),
@@ -117,6 +118,21 @@ def round_bf16(x: float) -> float:
 
 def init_value(seed, member_id, layer, e, fan_in) -> float:
     return float(lib().orc_init_value(seed, member_id, layer, e, fan_in))
+
+
+def adamw_apply(p, g, t, lr, wd, m=None, v=None, beta1=0.9, beta2=0.999, eps=1e-8):
+    """One AdamW step (Sec. 3.4; PyTorch semantics) of parameters p with
+    gradients g at step count t, from moments m, v (zeros if None), in fp64.
+    Returns the new (p, m, v)."""
+    p = np.array(p, dtype=np.float64, copy=True).ravel()
+    g = np.ascontiguousarray(g, dtype=np.float64).ravel()
+    m = np.zeros_like(p) if m is None else np.array(m, dtype=np.float64, copy=True).ravel()
+    v = np.zeros_like(p) if v is None else np.array(v, dtype=np.float64, copy=True).ravel()
+    if not (p.size == g.size == m.size == v.size):
+        raise ValueError("shape mismatch")
+    lib().orc_adamw_apply(_ptr(p), _ptr(m), _ptr(v), _ptr(g), p.size, int(t), float(lr), float(wd),
+                          float(beta1), float(beta2), float(eps))
+    return p, m, v
 
 
 def _labels(task, y):

@@ -408,13 +408,10 @@ static double orc_member_backward(const orc_pack* h, orc_member* M, const int32_
 /* AdamW (Loshchilov & Hutter; Sec. 3.4 packs one optimizer per member with
  * its own learning rate and weight decay).  PyTorch semantics: decoupled
  * decay p <- p - lr wd p, then the bias-corrected Adam step.                 */
-static void orc_adamw(const orc_pack* h, const orc_member* M, double* p, double* m, double* v,
-                      const double* g, int64_t n, int is_bias) {
-  const double b1 = h->cfg.beta1, b2 = h->cfg.beta2, eps = h->cfg.eps;
-  const double lr = (double)M->lr;
-  const double wd = (is_bias && !h->cfg.wd_on_bias) ? 0.0 : (double)M->wd;
-  const double bc1 = 1.0 - pow(b1, (double)M->t);
-  const double bc2 = 1.0 - pow(b2, (double)M->t);
+void orc_adamw_apply(double* p, double* m, double* v, const double* g, int64_t n, int64_t t, double lr,
+                     double wd, double b1, double b2, double eps) {
+  const double bc1 = 1.0 - pow(b1, (double)t);
+  const double bc2 = 1.0 - pow(b2, (double)t);
   for (int64_t e = 0; e < n; ++e) {
     p[e] = p[e] - lr * wd * p[e];
     m[e] = b1 * m[e] + (1.0 - b1) * g[e];
@@ -423,6 +420,12 @@ static void orc_adamw(const orc_pack* h, const orc_member* M, double* p, double*
     double vhat = v[e] / bc2;
     p[e] = p[e] - lr * mhat / (sqrt(vhat) + eps);
   }
+}
+
+static void orc_adamw(const orc_pack* h, const orc_member* M, double* p, double* m, double* v,
+                      const double* g, int64_t n, int is_bias) {
+  const double wd = (is_bias && !h->cfg.wd_on_bias) ? 0.0 : (double)M->wd;
+  orc_adamw_apply(p, m, v, g, n, M->t, (double)M->lr, wd, h->cfg.beta1, h->cfg.beta2, h->cfg.eps);
 }
 
 int orc_train_step(orc_pack* h, const float* X, int64_t N, const int32_t* idx,

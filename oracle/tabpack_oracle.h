@@ -98,6 +98,13 @@ int orc_predict(orc_pack* h, const float* X, int64_t N, double* out);
 
 int orc_set_active(orc_pack* h, const uint8_t* active);
 
+/* One AdamW step (PyTorch semantics, the update the training step applies to
+ * every parameter; Sec. 3.4) on n elements in place: decoupled decay
+ * p <- p - lr wd p, moments m, v, then the step bias-corrected for step
+ * count t >= 1.                                                              */
+void orc_adamw_apply(double* p, double* m, double* v, const double* g, int64_t n, int64_t t, double lr,
+                     double wd, double beta1, double beta2, double eps);
+
 /* layer in [0, depth] (depth = head).  W row-major [out, in], b [out].       */
 int orc_get_params(const orc_pack* h, int32_t member, int32_t layer, double* W, double* b);
 int orc_set_params(orc_pack* h, int32_t member, int32_t layer, const double* W, const double* b);

@@ -4,7 +4,8 @@
 // depths), another every backward product: a list of 128 x N output tiles
 // (N <= 256, a multiple of 16) that each persistent CTA (one per SM) walks
 // with stride gridDim.x.  The list is ordered by dependency level (forward:
-// the layer; backward: the distance from the head) and by cost, largest
+// the layer; backward: the distance from the head, with each level's wgrad
+// tiles moved beside the next level's dgrad tiles) and by cost, largest
 // first, within a level.  A tile whose A operand is produced in the same
 // launch waits for a row-block completion counter (the producer polls it
 // with acquire loads, bounded); every epilogue warp publishes its stores
@@ -54,9 +55,8 @@ constexpr int kThreads = 320;           // 2 role warps + 8 epilogue warps
 constexpr uint32_t kTmemCols = 512;
 constexpr int kAccCols = 256;
 constexpr uint64_t kWaitNs = 2000000000ull;
-// per epilogue warp a 32 x 33 fp32 transpose buffer (wgrad epilogue)
-constexpr int kTrPitch = 33;
-constexpr int kTrBytes = 8 * 32 * kTrPitch * 4;
+// per epilogue warp a 32 x 32 fp32 transpose buffer (wgrad epilogue)
+constexpr int kTrBytes = 8 * 32 * 32 * 4;
 
 // Pipeline geometry for tiles of kCta CTAs.  kCta = 1: a CTA computes
 // 128 x N and stages 128 rows of A and up to 256 rows / columns of B per K
@@ -191,6 +191,11 @@ __device__ __noinline__ bool dep_wait(const int* p, int n, int need, volatile in
   return true;
 }
 
+// Bulk prefetch of `bytes` (a multiple of 16; 16-byte aligned address) into L2.
+__device__ __forceinline__ void prefetch_l2(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint64_t* bar, int x, int y) {
   asm volatile(
       "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
@@ -314,6 +319,32 @@ __device__ __forceinline__ SubTile sub_tile(const TcTile& t, int mi, int B_pad) 
   return u;
 }
 
+// Fused-AdamW weight-gradient tile: epilogue warp e (0..7) of this CTA asks
+// L2 for 16 of the CTA's 128 weight rows of the tile's fp32 master, first and
+// second moments (one bulk prefetch per row and array), so that the
+// epilogue's loads of the tile hit L2.  Weight rows are 16-byte aligned and
+// the weight columns of a tile a multiple of 8 (n0 a multiple of 16, in_pad of 8).
+__device__ __forceinline__ void prefetch_adam_rows(const TcArgs& g, const TcTile& t, int rank, int e, int lane) {
+  const SubTile u = sub_tile(t, rank, g.B_pad);
+  const int cols = min(t.n_len, t.n_real - 1 - t.n0);
+  if (!u.rows_live || cols <= 0) return;
+  for (int k = lane; k < 48; k += 32) {
+    const int r = u.m0 + 16 * e + (k & 15);
+    if (r >= t.m_real) continue;
+    const float* base = k < 16 ? g.adam.params : k < 32 ? g.adam.m : g.adam.v;
+    prefetch_l2(base + t.c_off + (int64_t)r * t.ldc + t.n0, (uint32_t)cols * 4u);
+  }
+}
+
+// Prefetch of the tensor map of a tile's A (which = 0) or B (which = 1)
+// operand, as the producer selects it below.
+__device__ __forceinline__ void prefetch_tile_map(const TcArgs& g, const TcTile& t, int which) {
+  const bool a_k = t.kind != kWgrad, b_k = t.kind == kFwd;
+  const CUtensorMap* m = which == 0 ? g.maps + t.map_a + (a_k ? g.kmaj_off : 0)
+                                    : g.maps + t.map_b + (t.kind == kWgrad ? 0 : g.w_shift) + (b_k ? g.kmaj_off : 0);
+  asm volatile("prefetch.tensormap [%0];" ::"l"(m) : "memory");
+}
+
 // ------------------------------------------------------------------ kernel
 template <int kCta>
 __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
@@ -376,8 +407,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
     uint32_t stage = 0, phase = 0;
     uint32_t issued_mask = 0, last_parity = 0;  // per stage: ever issued, parity of the last issue
     bool ok = true;
+    if (lane < 2 && clu < g.n_tiles) prefetch_tile_map(g, g.tiles[clu], lane);
     for (int t = clu; ok && t < g.n_tiles; t += n_clu) {
       const TcTile tile = g.tiles[t];
+      // the descriptors of this CTA's next tile reach the descriptor cache
+      // while this tile's copies stream
+      if (lane < 2 && t + n_clu < g.n_tiles) prefetch_tile_map(g, g.tiles[t + n_clu], lane);
       if (!tile_live(tile, g.B_pad)) continue;
       const SubTile u = sub_tile(tile, rank, g.B_pad);
       const int K = tile.k_len ? tile.k_len : g.B_pad;
@@ -391,15 +426,17 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       const int nbB = b_k ? (nh + 127) >> 7 : (nh + 63) >> 6;
       const uint32_t boxB = b_k ? 2 * kBoxBytes : kBoxBytes;
       const uint32_t bytes = (uint32_t)kCta * (2 * kBoxBytes + (uint32_t)nbB * boxB);
-      const bool is_a = lane < nbA;  // lane < nbA: A box `lane`; then B box `lane - nbA`
-      const int qb = lane - nbA;
+      // lane bl < nbA: A box bl; then B box bl - nbA
+      const int bl = lane;
+      const bool is_a = bl < nbA;
+      const int qb = bl - nbA;
       const bool mine = is_a || qb < nbB;
       const CUtensorMap* map =
           is_a ? g.maps + tile.map_a + (a_k ? g.kmaj_off : 0)
                : g.maps + tile.map_b + (tile.kind == kWgrad ? 0 : g.w_shift) + (b_k ? g.kmaj_off : 0);
       const bool mn = is_a ? !a_k : !b_k;  // MN-major box: x = row / column, y = k
-      const int xy0 = is_a ? u.m0 + 64 * lane : bn0 + (b_k ? 128 : 64) * qb;
-      const uint32_t off = is_a ? (uint32_t)lane * kBoxBytes : (uint32_t)kABytes + (uint32_t)qb * boxB;
+      const int xy0 = is_a ? u.m0 + 64 * bl : bn0 + (b_k ? 128 : 64) * qb;
+      const uint32_t off = is_a ? (uint32_t)bl * kBoxBytes : (uint32_t)kABytes + (uint32_t)qb * boxB;
       bool dep_ok = true;
       if (lane == 0 && u.rows_live && tile.dep >= 0)
         dep_ok = dep_wait(g.cnt + tile.dep + (tile.dep_n ? rank : 0), tile.dep_n ? tile.dep_n : g.B_pad / kRowTile,
@@ -444,6 +481,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
   } else if (warp == 1) {
     if (lane == 0 && leader) {
       // --------------------------------------------------------------- MMA
+      // The issue loop is kept short: it shares its sub-partition's issue
+      // slots with two epilogue warps, and every instruction it spends
+      // between MMAs delays the tensor pipe.  Descriptors are formed once:
+      // stage s adds s * kStageBytes / 16 to the start-address field and K
+      // step kk adds 32 bytes (K-major) or 2048 bytes (MN-major) / 16; the
+      // field (address / 16 < 2^14) never carries into the next field.
+      const uint32_t s0 = smem_u32(smem);
+      const uint64_t dA_k = smem_desc(s0, 16, 1024), dA_mn = smem_desc(s0, kBoxBytes, 1024);
+      const uint64_t dB_k = smem_desc(s0 + kABytes, 16, 1024), dB_mn = smem_desc(s0 + kABytes, kBoxBytes, 1024);
+      constexpr uint32_t kStageStep = G::kStageBytes >> 4;
       uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
       bool ok = true;
       for (int t = clu; ok && t < g.n_tiles; t += n_clu) {
@@ -455,20 +502,25 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         const uint32_t d = tmem + acc * kAccCols;
         const int a_mn = tile.kind == kWgrad, b_mn = tile.kind != kFwd;
         const uint32_t idesc = instr_desc(128 * kCta, tile.n_len, a_mn, b_mn);
+        const uint64_t ta = a_mn ? dA_mn : dA_k, tb = b_mn ? dB_mn : dB_k;
+        const uint32_t ka = a_mn ? 2048 >> 4 : 32 >> 4, kb = b_mn ? 2048 >> 4 : 32 >> 4;
+        uint32_t accum = 0;
         for (int k0 = 0; k0 < K; k0 += 64) {
           if (!mbar_wait(&tl->full[stage], phase, abort_flag, g.err, kWaitNs)) {
             ok = false;
             break;
           }
-          tc_fence_after();
-          const uint32_t a = smem_u32(smem + stage * G::kStageBytes);
-          const uint32_t b = a + kABytes;
-          const int nk = min(4, (K - k0 + 15) >> 4);
-          for (int kk = 0; kk < nk; ++kk) {
-            const uint64_t ad = a_mn ? smem_desc(a + kk * 2048, kBoxBytes, 1024) : smem_desc(a + kk * 32, 16, 1024);
-            const uint64_t bd = b_mn ? smem_desc(b + kk * 2048, kBoxBytes, 1024) : smem_desc(b + kk * 32, 16, 1024);
-            umma_bf16<kCta>(d, ad, bd, idesc, (k0 | kk) != 0);
+          const uint64_t sa = ta + stage * kStageStep, sb = tb + stage * kStageStep;
+          if (K - k0 >= 64) {
+            umma_bf16<kCta>(d, sa, sb, idesc, accum);
+            umma_bf16<kCta>(d, sa + ka, sb + kb, idesc, 1u);
+            umma_bf16<kCta>(d, sa + 2 * ka, sb + 2 * kb, idesc, 1u);
+            umma_bf16<kCta>(d, sa + 3 * ka, sb + 3 * kb, idesc, 1u);
+          } else {
+            const int nk = (K - k0 + 15) >> 4;
+            for (int kk = 0; kk < nk; ++kk) umma_bf16<kCta>(d, sa + kk * ka, sb + kk * kb, idesc, kk ? 1u : accum);
           }
+          accum = 1u;
           umma_commit<kCta>(&tl->empty[stage]);  // the stage is free in every CTA of the tile
           if (++stage == kStages) {
             stage = 0;
@@ -492,8 +544,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
     const int row = 32 * q + lane;
     const uint32_t step = g.dyn ? g.dyn->step : g.step;
     uint32_t acc = 0, acc_phase = 0;
+    // Fused AdamW: the parameter rows of the CTA's next weight-gradient tile
+    // stream into L2 while this tile's products run and its epilogue works.
+    if (g.update && clu < g.n_tiles && g.tiles[clu].kind == kWgrad)
+      prefetch_adam_rows(g, g.tiles[clu], rank, warp - 2, lane);
     for (int t = clu; t < g.n_tiles; t += n_clu) {
       const TcTile tile = g.tiles[t];
+      if (g.update && t + n_clu < g.n_tiles) {
+        const TcTile nx = g.tiles[t + n_clu];
+        if (nx.kind == kWgrad) prefetch_adam_rows(g, nx, rank, warp - 2, lane);
+      }
       if (!tile_live(tile, g.B_pad)) continue;
       const SubTile u = sub_tile(tile, rank, g.B_pad);
       const MemberDev md = g.mem[tile.member];
@@ -503,6 +563,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       // the two warps of a lane quarter take alternate 32-column chunks:
       // chunk ci covers columns 32 * half + 64 * ci .. + 31 of the tile
       const int n_end = u.rows_live ? tile.n_len : 0;
+      // last output column of this tile plus one: a chunk may reach past the
+      // tile (n_len is a multiple of 16, chunks are 32 wide), and the columns
+      // past it belong to the next column tile
+      const int n_hi = min(tile.n_real, tile.n0 + tile.n_len);
       // Inputs that do not depend on the accumulator are prepared while the
       // tile's MMAs run: forward, this lane's bias value of each chunk
       // (column = lane; broadcast by shuffles) and the 32 dropout keep bits of
@@ -513,7 +577,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       for (int ci = 0; ci < 4; ++ci) {
         const int c = 32 * half + 64 * ci;
         const int col0 = tile.n0 + c;
-        const int ncols = min(32, tile.n_real - col0);
+        const int ncols = min(32, n_hi - col0);
         bias_l[ci] = 0.f;
         bits[ci] = 0xFFFFFFFFu;
         if (c >= n_end || ncols <= 0) continue;
@@ -559,53 +623,90 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         const int c = 32 * half + 64 * ci;
         if (c >= n_end) break;
         const int col0 = tile.n0 + c;
-        const int ncols = min(32, tile.n_real - col0);
+        const int ncols = min(32, n_hi - col0);
         const bool live = row_ok && ncols > 0;
         uint32_t v[32];
         tmem_ld32(taddr + c, v);
         if (tile.kind == kWgrad) {
-          // Transpose the warp's 32 rows x 32 columns through shared memory so
-          // that lane j walks column col0 + j row by row: every parameter,
-          // moment and gradient access of the warp is one 128-byte segment.
-          float* tr = tr_all + (warp - 2) * 32 * kTrPitch;
+          // Transpose the warp's 32 rows x 32 columns through shared memory
+          // (float4 groups XOR-swizzled by row, so that both the row-wise
+          // write and the group-wise read are free of bank conflicts).  Then
+          // lane (rsub, gc) = (lane / 8, lane % 8) takes columns col0 + 4 gc ..
+          // + 3 of rows 4 i + rsub, i = 0..7: every warp access covers four
+          // 128-byte row segments.
+          float* tr = tr_all + (warp - 2) * 32 * 32;
 #pragma unroll
-          for (int j = 0; j < 32; ++j) tr[lane * kTrPitch + j] = __uint_as_float(v[j]);
+          for (int gi = 0; gi < 8; ++gi)
+            *reinterpret_cast<float4*>(tr + lane * 32 + 4 * (gi ^ (lane & 7))) =
+                make_float4(__uint_as_float(v[4 * gi]), __uint_as_float(v[4 * gi + 1]),
+                            __uint_as_float(v[4 * gi + 2]), __uint_as_float(v[4 * gi + 3]));
           __syncwarp();
-          const int in_pad = tile.n_real - 1;
-          const int col = col0 + lane;
-          const bool is_w = col < in_pad, is_b = col == in_pad;
+          const int in_pad = tile.n_real - 1;  // a multiple of 8: a group is all weights or starts at the bias
+          const int gc = lane & 7, rsub = lane >> 3;
+          const int col = col0 + 4 * gc;
+          const bool is_w = col < in_pad && col < n_hi, is_b = col == in_pad && col < n_hi;
           const int rbase = u.m0 + 32 * q;
           const int nrows = min(32, m_lim - rbase);
-          if (is_w || is_b) {
+          if (g.update) {
             const AdamDev& ad = g.adam;
-            const float wdl = is_b ? wd_b : wd_w;
-            for (int rr0 = 0; rr0 < nrows; rr0 += 8) {
-              float gv[8], pp[8], mm[8], vv[8];
-              int64_t o[8];
+            if (is_w) {
+              // rounds of three row groups: nine float4 loads in flight per
+              // lane (the 10-warp CTA allows 168 registers per thread)
+#pragma unroll 1
+              for (int i0 = 0; i0 < 8; i0 += 3) {
+                float4 P[3], M[3], V[3];
 #pragma unroll
-              for (int u = 0; u < 8; ++u) {
-                const int rr = min(rr0 + u, nrows - 1);
-                gv[u] = tr[rr * kTrPitch + lane];
-                o[u] = is_w ? tile.c_off + (int64_t)(rbase + rr) * tile.ldc + col : tile.aux_off + rbase + rr;
-                if (g.update) {
-                  pp[u] = ad.params[o[u]];
-                  mm[u] = ad.m[o[u]];
-                  vv[u] = ad.v[o[u]];
+                for (int i = 0; i < 3; ++i) {
+                  const int rr = 4 * (i0 + i) + rsub;
+                  if (i0 + i < 8 && rr < nrows) {
+                    const int64_t o = tile.c_off + (int64_t)(rbase + rr) * tile.ldc + col;
+                    P[i] = *reinterpret_cast<const float4*>(ad.params + o);
+                    M[i] = *reinterpret_cast<const float4*>(ad.m + o);
+                    V[i] = *reinterpret_cast<const float4*>(ad.v + o);
+                  }
+                }
+#pragma unroll
+                for (int i = 0; i < 3; ++i) {
+                  const int rr = 4 * (i0 + i) + rsub;
+                  if (i0 + i >= 8 || rr >= nrows) break;
+                  const float4 G = *reinterpret_cast<const float4*>(tr + rr * 32 + 4 * (gc ^ (rr & 7)));
+                  adamw_elem(P[i].x, M[i].x, V[i].x, G.x, lr, wd_w, ad.beta1, ad.beta2, ad.eps, ib1, ib2);
+                  adamw_elem(P[i].y, M[i].y, V[i].y, G.y, lr, wd_w, ad.beta1, ad.beta2, ad.eps, ib1, ib2);
+                  adamw_elem(P[i].z, M[i].z, V[i].z, G.z, lr, wd_w, ad.beta1, ad.beta2, ad.eps, ib1, ib2);
+                  adamw_elem(P[i].w, M[i].w, V[i].w, G.w, lr, wd_w, ad.beta1, ad.beta2, ad.eps, ib1, ib2);
+                  const int64_t o = tile.c_off + (int64_t)(rbase + rr) * tile.ldc + col;
+                  *reinterpret_cast<float4*>(ad.params + o) = P[i];
+                  *reinterpret_cast<float4*>(ad.m + o) = M[i];
+                  *reinterpret_cast<float4*>(ad.v + o) = V[i];
+                  *reinterpret_cast<uint2*>(ad.wq_out + o) =
+                      make_uint2(pack_bf16x2(P[i].x, P[i].y), pack_bf16x2(P[i].z, P[i].w));
                 }
               }
-#pragma unroll
-              for (int u = 0; u < 8; ++u) {
-                if (rr0 + u >= nrows) break;
-                if (g.update) {
-                  adamw_elem(pp[u], mm[u], vv[u], gv[u], lr, wdl, ad.beta1, ad.beta2, ad.eps, ib1, ib2);
-                  ad.params[o[u]] = pp[u];
-                  ad.m[o[u]] = mm[u];
-                  ad.v[o[u]] = vv[u];
-                  ad.wq_out[o[u]] = __float2bfloat16_rn(pp[u]);
-                } else {
-                  g.grads[o[u]] = gv[u];
-                }
+            } else if (is_b) {
+              for (int i = 0; i < 8; ++i) {
+                const int rr = 4 * i + rsub;
+                if (rr >= nrows) break;
+                const float gb = tr[rr * 32 + 4 * (gc ^ (rr & 7))];
+                const int64_t o = tile.aux_off + rbase + rr;
+                float pb = ad.params[o], mb = ad.m[o], vb = ad.v[o];
+                adamw_elem(pb, mb, vb, gb, lr, wd_b, ad.beta1, ad.beta2, ad.eps, ib1, ib2);
+                ad.params[o] = pb;
+                ad.m[o] = mb;
+                ad.v[o] = vb;
+                ad.wq_out[o] = __float2bfloat16_rn(pb);
               }
+            }
+          } else if (is_w || is_b) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              const int rr = 4 * i + rsub;
+              if (rr >= nrows) break;
+              const float* src = tr + rr * 32 + 4 * (gc ^ (rr & 7));
+              if (is_w)
+                *reinterpret_cast<float4*>(g.grads + tile.c_off + (int64_t)(rbase + rr) * tile.ldc + col) =
+                    *reinterpret_cast<const float4*>(src);
+              else
+                g.grads[tile.aux_off + rbase + rr] = src[0];
             }
           }
           __syncwarp();  // the buffer is reused by the next chunk
@@ -846,9 +947,10 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
   }
 
   // Tiles of the active members.  Forward: level = layer.  Backward: level
-  // = distance from the head (each member's top hidden layer first); within a
-  // level the dgrad tiles (which the next level waits for) precede the wgrad
-  // tiles, each group sorted largest first.
+  // = distance from the head (each member's top hidden layer first); the
+  // dgrad tiles of a level (which the next level waits for) and its wgrad
+  // tiles are each sorted largest first, and the wgrad tiles are interleaved
+  // with the next level's dgrad tiles (below).
   const int nrb = lay.B_cap / kRowTile;
   if (plan.cnt_dev == nullptr) {
     plan.n_cnt = 2 * m * kMaxDepth * nrb;
@@ -909,8 +1011,10 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
     sorted_append(v);
   }
   plan.fwd_rng = {0, (int)all.size()};
+  std::vector<std::vector<TcTile>> VD(Lmax), VW(Lmax);
   for (int lev = 0; lev < Lmax; ++lev) {
-    std::vector<TcTile> vd, vw;
+    std::vector<TcTile>& vd = VD[lev];
+    std::vector<TcTile>& vw = VW[lev];
     for (int i = 0; i < m; ++i) {
       if (!active[i] || depth[i] <= lev) continue;
       const int l = depth[i] - 1 - lev;
@@ -953,8 +1057,36 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
       t.aux_off = (*lay.b_off)[i][l];
       emit(vw, t, (int)ceil_div(w, kRowTile), nw);
     }
-    sorted_append(vd);
-    sorted_append(vw);
+    auto by_cost = [&](const TcTile& a, const TcTile& b) { return cost(a) > cost(b); };
+    std::stable_sort(vd.begin(), vd.end(), by_cost);
+    std::stable_sort(vw.begin(), vw.end(), by_cost);
+  }
+  // Nothing waits for a weight-gradient tile, so the wgrad tiles of level
+  // lev move back beside the dgrad tiles of level lev + 1: in blocks of one
+  // tile per resident CTA (pair), taken from the two lists in proportion to
+  // their lengths, every CTA alternates between tiles whose epilogue streams
+  // parameters (fused AdamW) and tiles whose time goes to the tensor cores.
+  // Each tile still only waits for tiles earlier in the list.
+  auto interleave = [&](const std::vector<TcTile>& a, const std::vector<TcTile>& b) {
+    const size_t blk = (size_t)std::max(1, plan.max_clusters);
+    size_t ia = 0, ib = 0;
+    while (ia < a.size() || ib < b.size()) {
+      const bool take_a = ib >= b.size() || (ia < a.size() && ia * b.size() <= ib * a.size());
+      if (take_a) {
+        const size_t e = std::min(a.size(), ia + blk);
+        all.insert(all.end(), a.begin() + ia, a.begin() + e);
+        ia = e;
+      } else {
+        const size_t e = std::min(b.size(), ib + blk);
+        all.insert(all.end(), b.begin() + ib, b.begin() + e);
+        ib = e;
+      }
+    }
+  };
+  if (Lmax > 0) {
+    all.insert(all.end(), VD[0].begin(), VD[0].end());
+    for (int lev = 1; lev < Lmax; ++lev) interleave(VD[lev], VW[lev - 1]);
+    all.insert(all.end(), VW[Lmax - 1].begin(), VW[Lmax - 1].end());
   }
   plan.bwd_rng = {plan.fwd_rng.second, (int)all.size() - plan.fwd_rng.second};
   if ((int)all.size() + 1 > plan.cap_tiles) {

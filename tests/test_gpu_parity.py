@@ -97,48 +97,67 @@ def test_dropout_masks_bit_exact(tp, step):
 # either way on the two sides; both results are valid subgradients.  In bf16
 # mode a one-ulp difference in a stored activation (the fp32 and fp64 values
 # straddling a bf16 rounding boundary) moves the next layer's pre-activations
-# by ~1e-3 of their rms, so such flips occur there too.  One flip at (row b,
-# unit j) of layer l changes dW_l[j, :] by one of the B batch terms and every
-# upstream gradient by a fraction of a percent.  The test therefore reads the
-# GPU's stored activations, finds every flipped decision exactly (GPU H > 0
-# versus oracle keep & Z > 0), requires each flip to sit at an oracle
-# near-tie (|Z| < TIE * rms(Z)), holds members without flips to the strict
-# elementwise bar everywhere, and members with flips to the strict bar on
-# losses and logits and to the bar norm-wise on each gradient tensor.
+# by a fraction of an ulp of their rms; each layer turns more of them into
+# straddles, so the discrepancy grows with depth (in a 4-layer member of width
+# 1024 on 2048 rows it reaches ~1e-3 rms(Z) at the last layer).  One flip at
+# (row b, unit j) of layer l changes dW_l[j, :] by one of the B batch terms
+# and every upstream gradient by a fraction of a percent.  The test therefore
+# reads the GPU's stored activations, finds every flipped decision exactly
+# (GPU H > 0 versus oracle keep & Z > 0), and requires each flip to sit at an
+# oracle near-tie: |Z| below the larger of TIE * rms(Z) and twice the
+# layer's largest measured GPU-versus-oracle discrepancy of the
+# pre-activations near zero (units kept and positive on both sides with
+# |Z| < 0.05 rms(Z), where the GPU's pre-activation is its stored H times
+# 1 - p; the discrepancy comes from discrete one-ulp events, so its tail and
+# not its rms is what a flip has to be compared with).  Members without
+# flips are held to the strict elementwise bar everywhere, members with flips
+# to the strict bar on losses and logits and to the bar norm-wise on each
+# gradient tensor.
 TIE = {"fp32": 1e-5, "bf16": 5e-3}
 
 
-def _flips(pk, orc, i, L, prec):
+def _flips(pk, orc, i, L, prec, oi=None, p_drop=0.0):
+    """Flipped ReLU / dropout decisions of GPU member i (oracle member oi)."""
+    oi = i if oi is None else oi
     n = 0
     for l in range(L):
-        Hg = pk.debug_activations(i, l)
-        Zo = orc.preact(i, l)
-        mo = (Zo > 0) & (orc.keep(i, l) > 0)
+        Hg = pk.debug_activations(i, l).astype(np.float64)
+        Zo = orc.preact(oi, l)
+        keep = orc.keep(oi, l) > 0
+        mo = (Zo > 0) & keep
         diff = (Hg > 0) != mo
         if diff.any():
             zr = np.sqrt(np.mean(Zo ** 2))
+            near = keep & (Hg > 0) & (Zo > 0) & (Zo < 0.05 * zr)
+            noise = 0.0
+            if near.sum() >= 100:
+                zg = Hg[near] * (1.0 - float(np.float32(p_drop)))
+                noise = float(np.max(np.abs(zg - Zo[near])) / zr)
             worst = float(np.max(np.abs(Zo[diff])) / zr)
-            assert worst < TIE[prec], ("flip away from a near-tie", i, l, worst)
+            assert worst < max(TIE[prec], 2.0 * noise), ("flip away from a near-tie", i, l, worst, noise)
             n += int(diff.sum())
     return n
 
 
-def _compare_step(pk, orc, hp, prec, loss_gpu, loss_orc):
+def _compare_step(pk, orc, hp, prec, loss_gpu, loss_orc, members=None, max_flip_members=None):
+    """GPU members `members` (default: all) against oracle members 0, 1, ...
+    (the oracle may hold only the sampled members; they are independent)."""
     tol = TOL[prec]
+    members = list(range(len(hp["depth"]))) if members is None else list(members)
     problems = {}
     n_flip_members = 0
-    for i in range(len(hp["depth"])):
+    for oi, i in enumerate(members):
         L = int(hp["depth"][i])
-        flips = _flips(pk, orc, i, L, prec)
+        flips = _flips(pk, orc, i, L, prec, oi, float(hp["dropout"][i]))
         n_flip_members += flips > 0
         p = []
-        le = abs(loss_gpu[i] - loss_orc[i]) / max(1.0, abs(loss_orc[i]))
-        ge = rel_err(pk.logits(i), orc.logits(i))
+        le = abs(loss_gpu[i] - loss_orc[oi]) / max(1.0, abs(loss_orc[oi]))
+        ge = rel_err(pk.logits(i), orc.logits(oi))
         if le > tol or ge > tol:
             p.append(("loss/logits", le, ge))
         for l in range(L + 1):
             gW, gb = pk.get_grads(i, l)
-            oW, ob = orc.get_grads(i, l)
+            oW, ob = orc.get_grads(oi, l)
             if flips == 0:
                 e = max(rel_err(gW, oW), rel_err(gb, ob))
             else:
@@ -149,7 +168,9 @@ def _compare_step(pk, orc, hp, prec, loss_gpu, loss_orc):
                 p.append(("grad", l, flips, e))
         if p:
             problems[i] = p
-    assert n_flip_members <= max(1, len(hp["depth"]) // 3), ("too many members with flips", n_flip_members)
+    if max_flip_members is None:
+        max_flip_members = max(1, len(members) // 3)
+    assert n_flip_members <= max_flip_members, ("too many members with flips", n_flip_members)
     return problems
 
 
@@ -209,6 +230,118 @@ def test_ten_steps_params(tp, prec, fuse, task, d_out):
         bad = {i: e for i, e in bad.items() if i not in ties}
         assert len(ties) <= m // 4, (errs, margin)
     assert not bad, (errs, margin)
+
+
+def _adamw_of_own_grads(pk_step, pk_grads, hp, members, step_fn, t=1, tol=1e-5):
+    """AdamW applied by `pk_step` (one training step from fresh moments)
+    against the oracle's AdamW (Sec. 3.4) applied to the gradients the GPU
+    computed for the same step (`pk_grads`, which stores them), so that the
+    optimizer is checked without the gradients' own bf16 error."""
+    before = {(i, l): pk_step.get_params(i, l) for i in members for l in range(int(hp["depth"][i]) + 1)}
+    step_fn()
+    worst = 0.0
+    for (i, l), (W0, b0) in before.items():
+        gW, gb = pk_grads.get_grads(i, l)
+        W1, b1 = pk_step.get_params(i, l)
+        for p0, g, p1 in ((W0, gW, W1), (b0, gb, b1)):
+            ref, _, _ = oracle.adamw_apply(p0, g, t, float(hp["lr"][i]), float(hp["wd"][i]))
+            worst = max(worst, rel_err(p1.ravel(), ref))
+    assert worst <= tol, worst
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_split_column_tiles(tp, prec):
+    """Members wider than one 256-column tile, split into column tiles whose
+    widths are not multiples of 32 (272 -> 2 x 144, 336 -> 2 x 176,
+    704 -> 3 x 240, 528 -> 3 x 176; the weight gradient of layer 1 with
+    d_in = 270 has 273 columns -> 2 x 144): one step's logits, losses and
+    gradients against the oracle, then the AdamW step of the separate pass
+    and of the fused epilogue (bf16) against the oracle's AdamW of the GPU's
+    own gradients, and three steps' parameters against the oracle (fp32, at
+    the bf16 bar: AdamW's first steps divide each gradient by its own
+    magnitude, so an entry whose gradient is near zero carries the gradient's
+    absolute error into a full-size update; the exact check of the update is
+    the one on the GPU's own gradients)."""
+    d_in, d_out, B = 270, 3, 256
+    hp = random_pack(4, d_in, d_out, seed=41, depth=(2, 3), dropout=(0.0, 0.3))
+    hp["width"] = np.array([272, 336, 704, 528], dtype=np.int32)
+    pk, orc = pair(tp, "multiclass", d_in, d_out, hp, prec, 256)
+    X, y = make_data("multiclass", 600, d_in, d_out, 6)
+    Xd, yd = to_dev(X, y)
+    rng = np.random.default_rng(8)
+    idx = rng.choice(600, B, replace=False).astype(np.int32)
+    (idxd,) = to_dev(idx)
+    loss = torch.zeros(4, dtype=torch.float32, device=DEV)
+    pk.forward_backward(Xd, idxd, yd, 3, loss)
+    lo = orc.train_step(X, idx, y, 3, update=False)
+    problems = _compare_step(pk, orc, hp, prec, loss.cpu().numpy(), lo)
+    assert not problems, problems
+    for fuse in ((False, True) if prec == "bf16" else (False,)):
+        pk_s, _ = pair(tp, "multiclass", d_in, d_out, hp, prec, 256, fuse=fuse)
+        _adamw_of_own_grads(pk_s, pk, hp, range(4), lambda: pk_s.train_step(Xd, idxd, yd, 3, loss))
+    if prec == "bf16":
+        return
+    for step in range(3):
+        idx = rng.choice(600, B, replace=False).astype(np.int32)
+        (idxd,) = to_dev(idx)
+        pk.train_step(Xd, idxd, yd, step, loss)
+        orc.train_step(X, idx, y, step)
+    for i in range(4):
+        for l in range(int(hp["depth"][i]) + 1):
+            W, b = pk.get_params(i, l)
+            Wo, bo = orc.get_params(i, l)
+            assert max(rel_err(W, Wo), rel_err(b, bo)) <= TOL["bf16"], (i, l)
+
+
+def _sample_members(wl, hp):
+    """The cheapest member of each depth present (oracle time stays small)."""
+    cost = [wl.d_in * int(w) + (int(L) - 1) * int(w) * int(w) for L, w in zip(hp["depth"], hp["width"])]
+    pick = {}
+    for i in np.argsort(cost, kind="stable"):
+        pick.setdefault(int(hp["depth"][i]), int(i))
+    return sorted(pick.values())
+
+
+@pytest.mark.parametrize("name", ["medium", "large", "wide"])
+def test_full_size_sampled_members(tp, name):
+    """The benchmark's workload in the benchmark's launch configuration (the
+    whole pack, full batch, bf16, the same tile schedule): for sampled
+    members, dropout masks bit-exact, losses, logits and every gradient
+    against the oracle run on those members alone (members are independent,
+    Sec. 3.6), and the AdamW step of the separate pass and of the fused
+    epilogue against the oracle's AdamW of the GPU's own gradients."""
+    from workloads import SEED_HP, SEED_INIT, WORKLOADS, make_data as wl_data, sample_hparams
+    wl = WORKLOADS[name]
+    hp = sample_hparams(wl, seed=SEED_HP)
+    B = wl.batch
+    d = wl_data(wl, device="cpu", n_train=3 * B, n_val=0)
+    X, y = d["X_train"].numpy(), d["y_train"].numpy()
+    Xd, yd = to_dev(X, y)
+    idx = np.random.default_rng(3).permutation(3 * B)[:B].astype(np.int32)
+    (idxd,) = to_dev(idx)
+    sample = _sample_members(wl, hp)
+    sub = {k: v[sample] for k, v in hp.items()}
+
+    def gpu_pack(fuse):
+        return tp.Pack(wl.d_in, wl.d_out, wl.task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
+                       max_batch=B, seed=SEED_INIT, precision="bf16", fuse_optimizer=fuse)
+
+    pk = gpu_pack(False)
+    loss = torch.zeros(wl.m, dtype=torch.float32, device=DEV)
+    pk.forward_backward(Xd, idxd, yd, 0, loss)
+    orc = oracle.OraclePack(wl.d_in, wl.d_out, wl.task, sub["depth"], sub["width"], sub["dropout"], sub["lr"],
+                            sub["wd"], seed=SEED_INIT, bf16_storage=True, member_id=sample)
+    lo = orc.train_step(X, idx, y, 0, update=False)
+    for oi, i in enumerate(sample):
+        for l in range(int(hp["depth"][i])):
+            np.testing.assert_array_equal(pk.debug_masks(i, l, 0, B), orc.keep(oi, l))
+    problems = _compare_step(pk, orc, hp, "bf16", loss.cpu().numpy(), lo, members=sample,
+                             max_flip_members=len(sample))
+    assert not problems, problems
+    for fuse in (False, True):
+        pk_s = gpu_pack(fuse)
+        _adamw_of_own_grads(pk_s, pk, hp, sample, lambda: pk_s.train_step(Xd, idxd, yd, 0, loss))
+        pk_s.close()
 
 
 @pytest.mark.parametrize("prec", ["fp32", "bf16"])

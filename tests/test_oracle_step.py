@@ -293,3 +293,35 @@ def test_rejects_bad_configs(orc):
         orc.OraclePack(4, 1, "binary", [1], [16], [1.0], [1e-3], [0.0], seed=0)
     with pytest.raises(ValueError):
         orc.OraclePack(4, 3, "binary", [1], [16], [0.1], [1e-3], [0.0], seed=0)
+
+
+def test_adamw_apply_matches_torch_adamw(orc):
+    """The oracle's element-wise AdamW (used by parity tests on the GPU's own
+    gradients) against torch.optim.AdamW in fp64, five steps with moments
+    carried, and the pack's own update equals it on the pack's gradients."""
+    rng = np.random.default_rng(3)
+    p0 = rng.standard_normal(257)
+    lr, wd = 2.5e-3, 3e-2
+    tp = torch.tensor(p0.copy(), requires_grad=True)
+    opt = torch.optim.AdamW([tp], lr=lr, betas=(0.9, 0.999), eps=1e-8, weight_decay=wd)
+    p, m, v = p0.copy(), None, None
+    for t in range(1, 6):
+        g = rng.standard_normal(257) * 10.0 ** rng.uniform(-6, 0, 257)
+        tp.grad = torch.tensor(g)
+        opt.step()
+        p, m, v = orc.adamw_apply(p, g, t, lr, wd, m, v)
+        assert _rel(p, tp.detach().numpy()) < 1e-12
+
+    hp = random_pack(2, 6, 1, seed=12)
+    pack = orc.OraclePack(6, 1, "regression", hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
+                          seed=4)
+    X, y = _make_data("regression", 40, 6, 1, seed=6)
+    before = {(i, l): pack.get_params(i, l) for i in range(2) for l in range(int(hp["depth"][i]) + 1)}
+    pack.train_step(X, np.arange(40, dtype=np.int32), y, 0)
+    for (i, l), (W0, b0) in before.items():
+        gW, gb = pack.get_grads(i, l)
+        W1, b1 = pack.get_params(i, l)
+        pW, _, _ = orc.adamw_apply(W0, gW, 1, float(hp["lr"][i]), float(hp["wd"][i]))
+        pb, _, _ = orc.adamw_apply(b0, gb, 1, float(hp["lr"][i]), float(hp["wd"][i]))
+        np.testing.assert_array_equal(pW, W1.ravel())
+        np.testing.assert_array_equal(pb, b1)
