@@ -138,8 +138,12 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 // Bounded wait: false if the abort flag is raised or the budget runs out
 // (then the flag and the device error word are set).
+// A wait that gives up records its site code in the error word (the first
+// one wins): 1 producer stage empty, 3 producer dependency, 5 MMA
+// accumulator free, 6 MMA stage full, 7 epilogue accumulator full, 10 final
+// copy drain, 12 final MMA drain.
 __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* err,
-                                            uint64_t budget_ns) {
+                                            uint64_t budget_ns, int site) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_ns();
   while (true) {
@@ -147,15 +151,15 @@ __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, vola
     if (*abort_flag) return false;
     if (global_ns() - t0 > budget_ns) {
       *abort_flag = 1;
-      atomicExch(err, 1);
+      atomicCAS(err, 0, site);
       return false;
     }
   }
 }
 
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* err,
-                                          uint64_t budget_ns) {
-  return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity, abort_flag, err, budget_ns);
+                                          uint64_t budget_ns, int site) {
+  return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity, abort_flag, err, budget_ns, site);
 }
 
 __device__ __forceinline__ int ld_acquire(const int* p) {
@@ -173,7 +177,7 @@ __device__ __forceinline__ void fence_proxy_async_global() {
 }
 
 // Bounded wait until counters p[0 .. n-1] each reach `need`.
-__device__ __noinline__ bool dep_wait(const int* p, int n, int need, volatile int* abort_flag, int* err) {
+__device__ __noinline__ bool dep_wait(const int* p, int n, int need, volatile int* abort_flag, int* err, int site) {
   for (int j = 0; j < n; ++j) {
     if (ld_acquire(p + j) >= need) continue;
     const uint64_t t0 = global_ns();
@@ -181,7 +185,7 @@ __device__ __noinline__ bool dep_wait(const int* p, int n, int need, volatile in
       if (*abort_flag) return false;
       if (global_ns() - t0 > kWaitNs) {
         *abort_flag = 1;
-        atomicExch(err, 1);
+        atomicCAS(err, 0, site);
         return false;
       }
       __nanosleep(32);
@@ -440,7 +444,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       bool dep_ok = true;
       if (lane == 0 && u.rows_live && tile.dep >= 0)
         dep_ok = dep_wait(g.cnt + tile.dep + (tile.dep_n ? rank : 0), tile.dep_n ? tile.dep_n : g.B_pad / kRowTile,
-                          tile.dep_need, abort_flag, g.err);
+                          tile.dep_need, abort_flag, g.err, 3);
       if (!__shfl_sync(0xffffffffu, dep_ok, 0)) {
         ok = false;
         break;
@@ -449,7 +453,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       for (int k0 = 0; k0 < K; k0 += 64) {
         bool got = true;
         if (lane == 0) {
-          got = mbar_wait(&tl->empty[stage], phase ^ 1u, abort_flag, g.err, kWaitNs);
+          got = mbar_wait(&tl->empty[stage], phase ^ 1u, abort_flag, g.err, kWaitNs, 1);
           if (got && leader) mbar_expect_tx(&tl->full[stage], bytes);
         }
         if (!__shfl_sync(0xffffffffu, got, 0)) {
@@ -476,7 +480,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       for (int s = 0; s < kStages; ++s)
         if (issued_mask & (1u << s)) {
           int dummy_abort = 0;
-          mbar_wait(&tl->full[s], (last_parity >> s) & 1u, &dummy_abort, g.err, kWaitNs);
+          mbar_wait(&tl->full[s], (last_parity >> s) & 1u, &dummy_abort, g.err, kWaitNs, 10);
         }
   } else if (warp == 1) {
     if (lane == 0 && leader) {
@@ -497,7 +501,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         const TcTile tile = g.tiles[t];
         if (!tile_live(tile, g.B_pad)) continue;
         const int K = tile.k_len ? tile.k_len : g.B_pad;
-        if (!mbar_wait(&tl->tempty[acc], acc_phase ^ 1u, abort_flag, g.err, kWaitNs)) break;
+        if (!mbar_wait(&tl->tempty[acc], acc_phase ^ 1u, abort_flag, g.err, kWaitNs, 5)) break;
         tc_fence_after();
         const uint32_t d = tmem + acc * kAccCols;
         const int a_mn = tile.kind == kWgrad, b_mn = tile.kind != kFwd;
@@ -506,7 +510,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         const uint32_t ka = a_mn ? 2048 >> 4 : 32 >> 4, kb = b_mn ? 2048 >> 4 : 32 >> 4;
         uint32_t accum = 0;
         for (int k0 = 0; k0 < K; k0 += 64) {
-          if (!mbar_wait(&tl->full[stage], phase, abort_flag, g.err, kWaitNs)) {
+          if (!mbar_wait(&tl->full[stage], phase, abort_flag, g.err, kWaitNs, 6)) {
             ok = false;
             break;
           }
@@ -535,7 +539,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       // all MMAs this thread issued have completed before TMEM is freed
       umma_commit<kCta>(&tl->done);
       int dummy_abort = 0;
-      mbar_wait(&tl->done, 0, &dummy_abort, g.err, kWaitNs);
+      mbar_wait(&tl->done, 0, &dummy_abort, g.err, kWaitNs, 12);
     }
   } else {
     // ------------------------------------------------------------ epilogue
@@ -606,7 +610,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           bits[ci] = mb;
         }
       }
-      if (!mbar_wait(&tl->tfull[acc], acc_phase, abort_flag, g.err, kWaitNs)) break;
+      if (!mbar_wait(&tl->tfull[acc], acc_phase, abort_flag, g.err, kWaitNs, 7)) break;
       tc_fence_after();
       const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + acc * kAccCols;
       float lr = 0.f, wd_w = 0.f, wd_b = 0.f, ib1 = 1.f, ib2 = 1.f;
@@ -966,8 +970,18 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
   for (int i = 0; i < m; ++i) Lmax = std::max(Lmax, depth[i]);
   std::vector<TcTile> all;
   auto cost = [&](const TcTile& t) { return (int64_t)(t.k_len ? t.k_len : lay.B_cap) * t.n_len; };
+  // Within a level, tiles whose member has the longest chain of dependent
+  // products still ahead go first (list scheduling by remaining chain), then
+  // the costlier tiles.  Forward: layers above; dgrad: layers below.
+  auto chain = [&](const TcTile& t) {
+    return t.kind == kFwd ? depth[t.member] - 1 - t.layer : t.kind == kDgrad ? t.layer : 0;
+  };
+  auto by_chain_cost = [&](const TcTile& a, const TcTile& b) {
+    const int ca = chain(a), cb = chain(b);
+    return ca != cb ? ca > cb : cost(a) > cost(b);
+  };
   auto sorted_append = [&](std::vector<TcTile>& v) {
-    std::stable_sort(v.begin(), v.end(), [&](const TcTile& a, const TcTile& b) { return cost(a) > cost(b); });
+    std::stable_sort(v.begin(), v.end(), by_chain_cost);
     all.insert(all.end(), v.begin(), v.end());
   };
   // The tiles of one product: R row blocks (plan.cta at a time) by the
@@ -1058,7 +1072,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
       emit(vw, t, (int)ceil_div(w, kRowTile), nw);
     }
     auto by_cost = [&](const TcTile& a, const TcTile& b) { return cost(a) > cost(b); };
-    std::stable_sort(vd.begin(), vd.end(), by_cost);
+    std::stable_sort(vd.begin(), vd.end(), by_chain_cost);
     std::stable_sort(vw.begin(), vw.end(), by_cost);
   }
   // Nothing waits for a weight-gradient tile, so the wgrad tiles of level
@@ -1185,7 +1199,7 @@ tp_status tc_check(TcPlan& plan, cudaStream_t st, std::string& err) {
   }
   if (v) {
     cudaMemsetAsync(plan.err_dev, 0, sizeof(int), st);
-    err = "a tcgen05 GEMM pipeline wait timed out";
+    err = "a tcgen05 GEMM pipeline wait timed out (wait site " + std::to_string(v) + ")";
     return TP_ETIMEOUT;
   }
   return TP_OK;
