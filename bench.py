@@ -31,6 +31,15 @@ sys.path.insert(0, ROOT)
 from workloads import SEED_HP, SEED_INIT, WORKLOADS, make_data, sample_hparams  # noqa: E402
 
 METRIC = "member-samples/sec (fwd+bwd+AdamW)"
+
+# DRAM bytes (read + write) per step of the dominant kernels, from ncu captures of
+# the current kernels (summaries in profiles/; the wide figure is scaled from its
+# first 8 members by GEMM flops).  A workload without a capture reports null.
+DRAM_TRAFFIC = {
+    ("medium", "k_tc_gemm"): 245.3e6,
+    ("medium", "k_adamw"): 601.0e6,
+    ("wide", "k_tc_gemm"): 3.563e9,
+}
 UNIT = "member-samples/s"
 
 
@@ -78,7 +87,7 @@ class ClockSampler:
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu_id}", f"--query-gpu={self.FIELDS}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except Exception:
             self.proc = None
@@ -174,7 +183,7 @@ def run_reference(args, wl, rank):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--workload", default="medium", choices=sorted(WORKLOADS))
     ap.add_argument("--precision", default="bf16", choices=["bf16", "fp32"])
@@ -274,16 +283,18 @@ def main():
     gemm_ms = fwd_ms + bwd_ms
     gemm = {"kernel": "k_tc_gemm (grouped fwd + dgrad + wgrad launches of one step)", "bound": "tensor",
             "achieved": flops / (gemm_ms / 1e3) / 1e12, "peak": pk["bf16_sus"], "unit": "TFLOP/s",
-            "traffic": None, "ms_per_step": gemm_ms, "peak_source": pk["source"] + " sustained bf16"}
+            "traffic": DRAM_TRAFFIC.get((args.workload, "k_tc_gemm")) if args.members == 0 else None,
+            "ms_per_step": gemm_ms, "peak_source": pk["source"] + " sustained bf16"}
     gemm["frac"] = gemm["achieved"] / gemm["peak"]
-    if adam_ms > 0:   # fp32 mode: stand-alone AdamW, 30 B per parameter
+    if adam_ms > 0:   # AdamW as a separate pass (the default): 30 B per parameter
         mem = {"kernel": "k_adamw", "bound": "hbm", "achieved": 30.0 * n_params / (adam_ms / 1e3) / 1e9,
                "ms_per_step": adam_ms, "bytes_per_step": 30.0 * n_params}
-    else:             # bf16 mode: AdamW fused into the wgrad epilogue, 26 B per parameter
+    else:             # --fuse-optimizer: AdamW in the wgrad epilogue, 26 B per parameter
         mem = {"kernel": "k_tc_gemm backward launches (fused AdamW: read p, m, v; write p, m, v, bf16 p)",
                "bound": "hbm", "achieved": 26.0 * n_params / (bwd_ms / 1e3) / 1e9, "ms_per_step": bwd_ms,
                "bytes_per_step": 26.0 * n_params}
-    mem.update({"peak": pk["hbm"], "unit": "GB/s", "traffic": None, "peak_source": pk["source"] + " HBM copy"})
+    mem.update({"peak": pk["hbm"], "unit": "GB/s", "peak_source": pk["source"] + " HBM copy",
+                "traffic": DRAM_TRAFFIC.get((args.workload, "k_adamw")) if args.members == 0 and adam_ms > 0 else None})
     mem["frac"] = mem["achieved"] / mem["peak"]
     roof = dict(gemm if gemm_ms >= adam_ms else mem)
     roof["other"] = mem if gemm_ms >= adam_ms else gemm
