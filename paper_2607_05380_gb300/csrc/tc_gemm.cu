@@ -51,12 +51,24 @@ namespace {
 
 constexpr int kBoxBytes = 64 * 64 * 2;  // one 64 x 64 bf16 TMA box
 constexpr int kABytes = 2 * kBoxBytes;  // 128 rows of A per CTA
-constexpr int kThreads = 320;           // 2 role warps + 8 epilogue warps
+// Epilogue warps: one or two per TMEM lane quarter.  Eight (the default)
+// halve each warp's share of a tile's columns; four keep every SM
+// sub-partition at two warps (a 255-register cap, and the MMA issuer shares
+// its sub-partition with one epilogue warp) but were measured slower: the
+// longer epilogue of a tile delays the next accumulator.
+#ifndef TP_EPI_WARPS
+#define TP_EPI_WARPS 8
+#endif
+constexpr int kEpiWarps = TP_EPI_WARPS;
+static_assert(kEpiWarps == 4 || kEpiWarps == 8, "one or two epilogue warps per TMEM lane quarter");
+constexpr int kEpiPerQ = kEpiWarps / 4;         // epilogue warps per lane quarter
+constexpr int kChunks = 8 / kEpiPerQ;           // 32-column chunks per warp of a 256-column tile
+constexpr int kThreads = 64 + 32 * kEpiWarps;   // producer warp, MMA warp, epilogue warps
 constexpr uint32_t kTmemCols = 512;
 constexpr int kAccCols = 256;
 constexpr uint64_t kWaitNs = 2000000000ull;
 // per epilogue warp a 32 x 32 fp32 transpose buffer (wgrad epilogue)
-constexpr int kTrBytes = 8 * 32 * 32 * 4;
+constexpr int kTrBytes = kEpiWarps * 32 * 32 * 4;
 
 // Pipeline geometry for tiles of kCta CTAs.  kCta = 1: a CTA computes
 // 128 x N and stages 128 rows of A and up to 256 rows / columns of B per K
@@ -301,10 +313,13 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&t);
 }
 
-// a[i] for a runtime i < 4 without indexing (keeps a[] in registers)
-template <typename V>
-__device__ __forceinline__ V pick4(const V (&a)[4], int i) {
-  return i == 0 ? a[0] : i == 1 ? a[1] : i == 2 ? a[2] : a[3];
+// a[i] for a runtime i < N (N = 4 or 8) without indexing (keeps a[] in registers)
+template <typename V, int N>
+__device__ __forceinline__ V pick(const V (&a)[N], int i) {
+  V r = a[0];
+#pragma unroll
+  for (int k = 1; k < N; ++k) r = i == k ? a[k] : r;
+  return r;
 }
 
 __device__ __forceinline__ bool tile_live(const TcTile& t, int B_pad) { return t.kind == kWgrad || t.m0 < B_pad; }
@@ -323,8 +338,8 @@ __device__ __forceinline__ SubTile sub_tile(const TcTile& t, int mi, int B_pad) 
   return u;
 }
 
-// Fused-AdamW weight-gradient tile: epilogue warp e (0..7) of this CTA asks
-// L2 for 16 of the CTA's 128 weight rows of the tile's fp32 master, first and
+// Fused-AdamW weight-gradient tile: epilogue warp e of this CTA asks L2 for
+// 128 / kEpiWarps of the CTA's 128 weight rows of the tile's fp32 master, first and
 // second moments (one bulk prefetch per row and array), so that the
 // epilogue's loads of the tile hit L2.  Weight rows are 16-byte aligned and
 // the weight columns of a tile a multiple of 8 (n0 a multiple of 16, in_pad of 8).
@@ -332,10 +347,11 @@ __device__ __forceinline__ void prefetch_adam_rows(const TcArgs& g, const TcTile
   const SubTile u = sub_tile(t, rank, g.B_pad);
   const int cols = min(t.n_len, t.n_real - 1 - t.n0);
   if (!u.rows_live || cols <= 0) return;
-  for (int k = lane; k < 48; k += 32) {
-    const int r = u.m0 + 16 * e + (k & 15);
+  constexpr int kR = 128 / kEpiWarps;
+  for (int k = lane; k < 3 * kR; k += 32) {
+    const int r = u.m0 + kR * e + (k % kR);
     if (r >= t.m_real) continue;
-    const float* base = k < 16 ? g.adam.params : k < 32 ? g.adam.m : g.adam.v;
+    const float* base = k < kR ? g.adam.params : k < 2 * kR ? g.adam.m : g.adam.v;
     prefetch_l2(base + t.c_off + (int64_t)r * t.ldc + t.n0, (uint32_t)cols * 4u);
   }
 }
@@ -370,7 +386,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tl->tfull[b], 1);
-      mbar_init(&tl->tempty[b], 8 * kCta);  // one arrival per epilogue warp of the pair
+      mbar_init(&tl->tempty[b], kEpiWarps * kCta);  // one arrival per epilogue warp of the pair
     }
     mbar_init(&tl->done, 1);
     tl->abort = 0;
@@ -565,7 +581,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       const int r = u.m0 + row;
       const bool row_ok = r < m_lim;
       // the two warps of a lane quarter take alternate 32-column chunks:
-      // chunk ci covers columns 32 * half + 64 * ci .. + 31 of the tile
+      // chunk ci covers columns 32 * half + 32 * kEpiPerQ * ci .. + 31 of the tile
       const int n_end = u.rows_live ? tile.n_len : 0;
       // last output column of this tile plus one: a chunk may reach past the
       // tile (n_len is a multiple of 16, chunks are 32 wide), and the columns
@@ -575,11 +591,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       // tile's MMAs run: forward, this lane's bias value of each chunk
       // (column = lane; broadcast by shuffles) and the 32 dropout keep bits of
       // its row; dgrad, the 32 ReLU-mask bits of its row.
-      float bias_l[4];
-      uint32_t bits[4];
+      float bias_l[kChunks];
+      uint32_t bits[kChunks];
 #pragma unroll
-      for (int ci = 0; ci < 4; ++ci) {
-        const int c = 32 * half + 64 * ci;
+      for (int ci = 0; ci < kChunks; ++ci) {
+        const int c = 32 * half + 32 * kEpiPerQ * ci;
         const int col0 = tile.n0 + c;
         const int ncols = min(32, n_hi - col0);
         bias_l[ci] = 0.f;
@@ -623,8 +639,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         ib2 = 1.f / bc.y;
       }
 #pragma unroll 1
-      for (int ci = 0; ci < 4; ++ci) {
-        const int c = 32 * half + 64 * ci;
+      for (int ci = 0; ci < kChunks; ++ci) {
+        const int c = 32 * half + 32 * kEpiPerQ * ci;
         if (c >= n_end) break;
         const int col0 = tile.n0 + c;
         const int ncols = min(32, n_hi - col0);
@@ -718,11 +734,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         }
         if (tile.kind == kFwd) {  // ncols: a multiple of 8 (widths are multiples of 16)
           float bias[32];
-          const float bl = pick4(bias_l, ci);
+          const float bl = pick(bias_l, ci);
 #pragma unroll
           for (int j = 0; j < 32; ++j) bias[j] = __shfl_sync(0xffffffffu, bl, j);
           if (!live) continue;
-          const uint32_t keep = pick4(bits, ci);
+          const uint32_t keep = pick(bits, ci);
           const float sc = g.train ? md.scale : 1.f;
           __nv_bfloat16* out = g.act + tile.c_off + (int64_t)r * tile.ldc + col0;
 #pragma unroll
@@ -745,7 +761,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           }
         } else if (tile.kind == kDgrad) {
           if (!live) continue;
-          const uint32_t mb = pick4(bits, ci);
+          const uint32_t mb = pick(bits, ci);
           __nv_bfloat16* out = g.dz + tile.c_off + (int64_t)r * tile.ldc + col0;
 #pragma unroll
           for (int s = 0; s < 4; ++s) {
@@ -1016,7 +1032,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
       t.ld_aux = 0;
       t.dep = l == 0 ? -1 : cnt_act(i, l - 1);
       t.dep_n = 1;
-      t.dep_need = 8 * (int)ns.size();  // every epilogue warp of every column tile of a row block
+      t.dep_need = kEpiWarps * (int)ns.size();  // every epilogue warp of every column tile of a row block
       t.sig = l + 1 < depth[i] ? cnt_act(i, l) : -1;
       t.c_off = (*lay.act_off)[i][l];
       t.aux_off = (*lay.b_off)[i][l];
@@ -1034,7 +1050,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
       const int l = depth[i] - 1 - lev;
       const int w = width[i], in_pad = l == 0 ? lay.d_in_pad : w;
       split_n(w, ns);
-      const int need = 8 * (int)ns.size();  // dgrad column tiles of layer l + 1 per row block of dz_l
+      const int need = kEpiWarps * (int)ns.size();  // dgrad column tiles of layer l + 1 per row block of dz_l
       const bool from_head = l == depth[i] - 1;
       if (l > 0) {
         TcTile t{};
