@@ -67,6 +67,21 @@ def work_per_step(wl, hp, B):
     return flops, n_params
 
 
+def max_over_ranks(value, dist, device):
+    """The largest of every rank's `value` (the job's timed region ends when
+    its slowest rank ends)."""
+    import torch
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(world, members, batch, steps, ms_total):
+    """Whole-job member-samples/s: every rank trains its own pack of
+    `members` members on `batch` rows per step (weak scaling)."""
+    return world * members * batch * steps / (ms_total / 1000.0)
+
+
 def workload_desc(wl, B):
     return (f"{wl.name}: {wl.task}, m={wl.m} members, depth U{{{wl.depth[0]}..{wl.depth[1]}}}, width multiples of "
             f"{wl.width[2]} in [{wl.width[0]},{wl.width[1]}], dropout U[{wl.dropout[0]},{wl.dropout[1]}], "
@@ -256,12 +271,10 @@ def main():
     launches = pack.launch_count() - l0
     ms_total = ev0.elapsed_time(ev1)
     if world > 1:
-        t = torch.tensor([ms_total], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_total = float(t.item())
+        ms_total = max_over_ranks(ms_total, dist, dev)
         dist.barrier()
     ms_step = ms_total / args.steps
-    value = world * wl.m * B * args.steps / (ms_total / 1000.0)
+    value = job_rate(world, wl.m, B, args.steps, ms_total)
     lossv = loss.cpu().numpy()
 
     # per-kernel-family times over a second timed region (CUDA events on the pack's stream)
