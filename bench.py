@@ -138,6 +138,60 @@ class ClockSampler:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
+def predict_flops(wl, hp, n_rows):
+    """Matrix-product flops of one forward without dropout of every member
+    over n_rows rows (hidden layers and head)."""
+    f = 0
+    for L, w in zip(hp["depth"], hp["width"]):
+        L, w = int(L), int(w)
+        f += wl.d_in * w + (L - 1) * w * w + w * wl.d_out
+    return 2.0 * n_rows * f
+
+
+def time_online_epoch(tp, torch, pack, wl, hp, d, X, y, idx_all, stream, loss, n_epochs=6, steps_between=8,
+                      m_ens=32, p_base=16, p_ens=32):
+    """Wall time of the online ensemble's epoch end (Sec. 3.5: predict the
+    members on the validation rows, greedy selection over the pool, member
+    snapshots, patience bookkeeping) on the workload's full validation set,
+    with a few training steps between epoch ends so that states change.  The
+    call synchronises, so it is timed on the host around a synchronised
+    stream; the prediction share comes from the pack's CUDA-event profile."""
+    X_val, y_val = d["X_val"], d["y_val"]
+    on = tp.OnlineEnsemble(pack, X_val.shape[0], "loss", m_ens, p_base, p_ens)
+    B = wl.batch
+    times, pred_ms = [], []
+    s_next = 50_000
+    for e in range(n_epochs + 1):
+        for k in range(steps_between):
+            pack.train_step(X, idx_all[k % idx_all.shape[0]], y, s_next, loss)
+            s_next += 1
+        torch.cuda.synchronize()
+        pack.profile_enable(True)
+        pack.profile_read(reset=True)
+        t0 = time.perf_counter()
+        on.epoch(X_val, y_val)
+        dt = (time.perf_counter() - t0) * 1000.0
+        prof = pack.profile_read(reset=True)
+        pack.profile_enable(False)
+        if e > 0:      # the first call warms up
+            times.append(dt)
+            pred_ms.append(prof["predict"][0] + prof["fwd"][0])
+    info = on.info()
+    on.close()
+    pack.set_active(np.ones(wl.m, dtype=np.uint8))
+    ms = float(np.median(times))
+    pm = float(np.median(pred_ms))
+    n_val = int(X_val.shape[0])
+    pool = info["n_pool"]
+    sel_bytes = m_ens * pool * n_val * wl.d_out * 4.0
+    return {"ms": ms, "predict_ms": pm, "select_and_rest_ms": ms - pm, "n_val": n_val, "m_ens": m_ens,
+            "pool": pool, "n_best": info["n_best"], "epochs_timed": len(times),
+            "predict_tflops": predict_flops(wl, hp, n_val) / (pm / 1e3) / 1e12,
+            "select_candidate_bytes": sel_bytes,
+            "note": "epoch-end cost once per epoch of %d steps; predictions on the full validation set"
+                    % -(-wl.n_train // B)}
+
+
 def cpu_baseline(wl, hp, data_np, B, budget_s=20.0):
     """The oracle as it stands, on the host cores, on a bounded sample of the
     same workload: the first k members (independent of the others), timed
@@ -208,6 +262,7 @@ def main():
     ap.add_argument("--members", type=int, default=0,
                     help="train only the first N members of the workload (profiling small cases)")
     ap.add_argument("--fuse-optimizer", action="store_true", help="AdamW inside the weight-gradient epilogue")
+    ap.add_argument("--no-online", action="store_true", help="skip timing the online-ensemble epoch end")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -348,6 +403,8 @@ def main():
         e2e = {"value": world * wl.m * B * n_e2e / (ms_e2e / 1000.0), "unit": UNIT,
                "h2d_bytes_per_step": B * wl.d_in * 4 + B * 4, "d2h_bytes_per_step": wl.m * 4, "steps": n_e2e}
 
+    online = None if args.no_online else time_online_epoch(tp, torch, pack, wl, hp, d, X, y, idx_all, stream, loss)
+
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         n = min(n_train, 20000)
@@ -363,7 +420,7 @@ def main():
                            "l2": "inputs larger than L2: each step streams ~%.2f GB of parameters and optimizer state"
                                  % (30.0 * n_params / 1e9),
                            "parallelism": "one independent pack per GPU" if world > 1 else "single GPU"},
-                "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
+                "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches, "online_epoch": online,
                 "clocks": clk.summary(), "final_losses_mean": float(np.nanmean(lossv))}
         print(json.dumps(line), flush=True)
     pack.close()

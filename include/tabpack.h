@@ -186,6 +186,34 @@ tp_status pack_set_active(tabpack_t* pack, const uint8_t* active);
 tp_status pack_get_params(tabpack_t* pack, int32_t member, int32_t layer, float* W, float* b);
 tp_status pack_set_params(tabpack_t* pack, int32_t member, int32_t layer, const float* W, const float* b);
 
+/* Member snapshots (the "intermediate base-model checkpoints" of Sec. 3.5
+ * that the online ensemble keeps).  Member i's fp32 master parameters are
+ * one contiguous run of the pack's parameter arena, of *n_elems elements:
+ * for l = 0 .. depth[i] in turn, the weights [out, in_pad] row-major and
+ * then the bias [out], each block starting at a multiple of 32 elements
+ * from the start of the run, the gaps zero; in_pad = d_in rounded up to a
+ * multiple of 8 for l = 0 (pad columns zero), width[i] otherwise.  The run
+ * depends only on (d_in, d_out, depth[i], width[i]), so a snapshot of one
+ * pack restores into any member of the same shape in any pack.
+ *   pack_snapshot: copies the run to dst, a device float32 buffer of
+ *     *n_elems elements; asynchronous on the pack's stream (device to
+ *     device), so it captures the state after all work enqueued before it.
+ *   pack_restore: copies a run written by pack_snapshot back from src
+ *     (device) and refreshes the bf16 weight copies; synchronises.  The
+ *     member's optimizer state and step count are left as they are.      */
+tp_status pack_member_size(const tabpack_t* pack, int32_t member, int64_t* n_elems);
+tp_status pack_snapshot(tabpack_t* pack, int32_t member, float* dst);
+tp_status pack_restore(tabpack_t* pack, int32_t member, const float* src);
+
+/* Read back what pack_create was given: the configuration, one member's
+ * hyperparameters (any output pointer may be NULL), the active mask (host
+ * uint8 [m], 1 = trained) and the stream the pack runs on.                 */
+tp_status pack_get_config(const tabpack_t* pack, tp_config* cfg);
+tp_status pack_member_hparams(const tabpack_t* pack, int32_t member, int32_t* depth, int32_t* width,
+                              float* dropout, float* lr, float* wd);
+tp_status pack_get_active(const tabpack_t* pack, uint8_t* active);
+void* pack_get_stream(const tabpack_t* pack);
+
 /* Gradients of the last pack_forward_backward, same layout as the params.  */
 tp_status pack_get_grads(tabpack_t* pack, int32_t member, int32_t layer, float* W, float* b);
 
@@ -220,6 +248,97 @@ int64_t pack_launch_count(const tabpack_t* pack);
 /* Sizes of the pack: number of fp32 parameters (as stored, including the
  * zero padding of layer-0 columns to a multiple of 8) and device bytes held. */
 tp_status pack_sizes(const tabpack_t* pack, int64_t* n_params, int64_t* device_bytes);
+
+/* ------------------------------------------------------------------------
+ * Online ensemble (Sec. 3.5 "Online ensemble", Sec. 3.6 early stopping).
+ *
+ * The caller trains the pack for one epoch (pack_train_step over its
+ * batches) and then calls pack_online_epoch, which
+ *   1. predicts every active member on the validation rows (pack_predict);
+ *   2. forms the candidate pool: the active members' current states
+ *      (candidates 0 .. m-1, inactive members excluded) followed by the
+ *      previous epoch's ensemble members in their selection order
+ *      (candidates m, m+1, ...; their predictions are kept from the epoch
+ *      they were made in), each an instance (member, epoch);
+ *   3. rebuilds the ensemble from scratch by greedy selection over the pool
+ *      (pack_select_greedy's rule and arithmetic, at most m_ens members);
+ *      instances of the same member from different epochs are distinct
+ *      candidates;
+ *   4. snapshots the parameters of every newly selected current state
+ *      (pack_snapshot into memory the object owns);
+ *   5. base-model early stopping: a member's validation score is the score
+ *      of its own prediction alone (the same score function); a score that
+ *      is strictly below the member's best so far resets its count of
+ *      non-improving epochs, any other (including NaN) increments it, and a
+ *      member whose count reaches p_base + 1 is made inactive
+ *      (pack_set_active) after this epoch's selection;
+ *   6. ensemble early stopping: the same rule on the ensemble's score with
+ *      p_ens; the best ensemble so far (lowest score, earliest on ties) is
+ *      kept with its snapshots.  *stop becomes 1 when the count reaches
+ *      p_ens + 1 or no member remains active.
+ * Epochs are numbered from 1.  Scores are lower-is-better as in
+ * pack_select_greedy.  The object works on the pack's stream; the pack must
+ * outlive it.  Device memory it holds: the pool (m + 2 m_ens) * n_val *
+ * d_out floats, 2 m_ens snapshot slots of the largest member's run, and
+ * its selection scratch.                                                    */
+typedef struct tabpack_online tabpack_online_t;
+
+typedef struct {
+  int32_t epoch;        /* epochs processed                                     */
+  int32_t stop;         /* 1 once training should stop (see above)              */
+  int32_t n_active;     /* members still trained                                */
+  int32_t ens_bad;      /* consecutive epochs without ensemble improvement      */
+  int32_t best_epoch;   /* epoch whose ensemble is the best (0: none yet)       */
+  int32_t n_best;       /* members of the best ensemble                         */
+  int32_t n_last;       /* members of the last epoch's ensemble                 */
+  int32_t n_pool;       /* candidates in the last epoch's pool                  */
+  double best_score;    /* score of the best ensemble (+inf: none yet)          */
+  double last_score;    /* score of the last epoch's ensemble                   */
+} tp_online_info;
+
+/* Create the online ensemble of `pack` for validation sets of n_val rows.
+ * score: tp_score (as pack_select_greedy; valid for the pack's task);
+ * m_ens >= 1; p_base, p_ens >= 0 (the paper's defaults are 16 and 32).     */
+tp_status pack_online_create(tabpack_t* pack, int64_t n_val, int32_t score, int32_t m_ens, int32_t p_base,
+                             int32_t p_ens, tabpack_online_t** out);
+void pack_online_destroy(tabpack_online_t* online);
+
+/* End of an epoch (steps 1-6 above).  X_val: device float32 [n_val, d_in];
+ * y_val: device labels [n_val]; stop: host output (may be NULL).
+ * Synchronises the pack's stream.  After *stop = 1 further calls return
+ * TP_ESTATE.                                                               */
+tp_status pack_online_epoch(tabpack_online_t* online, const float* X_val, const void* y_val, int32_t* stop);
+
+tp_status pack_online_info(const tabpack_online_t* online, tp_online_info* info);
+
+/* Per-member state after the last epoch, host arrays of length m (any may be
+ * NULL): score (the member's last validation score; NaN if it was inactive
+ * in that epoch), best (its best score so far; +inf if none), bad (its count
+ * of non-improving epochs).                                                */
+tp_status pack_online_members(const tabpack_online_t* online, double* score, double* best, int32_t* bad);
+
+/* An ensemble as instances: which = 0 the best ensemble, 1 the last
+ * epoch's.  member, epoch: host int32 [m_ens] in selection order (may be
+ * NULL); *n: its size; *score: its score (may be NULL).                     */
+tp_status pack_online_ensemble(const tabpack_online_t* online, int32_t which, int32_t* member, int32_t* epoch,
+                               int32_t* n, double* score);
+
+/* Parameter run of instance j of the best ensemble (layout as
+ * pack_snapshot; pack_member_size of its member gives the length) copied to
+ * dst (device).  Synchronises.                                             */
+tp_status pack_online_snapshot(tabpack_online_t* online, int32_t j, float* dst);
+
+/* Prediction of the best ensemble on N rows: for every row the mean of its
+ * n instances' predictions (probabilities or values as pack_predict writes
+ * them), summed in fp64 in selection order and multiplied by 1/n, rounded
+ * to fp32.  The instances run from their snapshots in a second pack the
+ * object builds (and rebuilds when the best ensemble changes).
+ *   X: device float32 [N, d_in];  out: device float32 [N, d_out].
+ * Asynchronous on the pack's stream.                                       */
+tp_status pack_online_predict(tabpack_online_t* online, const float* X, int64_t N, float* out);
+
+/* Description of the last error of this online object.                    */
+const char* pack_online_last_error(const tabpack_online_t* online);
 
 /* Description of the last error on this pack (or, for pack == NULL, of the
  * last failed pack_create / pack_select_greedy / pack_select_greedy_static

@@ -30,7 +30,11 @@ PHASES = ["gather", "fwd", "head", "bwd", "bias", "adamw", "predict"]
 SYMBOLS = ["pack_create", "pack_destroy", "pack_set_stream", "pack_train_step", "pack_forward_backward",
            "pack_predict", "pack_select_greedy", "pack_select_greedy_static", "pack_set_active", "pack_get_params", "pack_set_params",
            "pack_get_grads", "pack_get_logits", "pack_debug_masks", "pack_debug_activations", "pack_profile_enable",
-           "pack_profile_read", "pack_launch_count", "pack_sizes", "pack_last_error"]
+           "pack_profile_read", "pack_launch_count", "pack_sizes", "pack_last_error", "pack_member_size",
+           "pack_snapshot", "pack_restore", "pack_get_config", "pack_member_hparams", "pack_get_active",
+           "pack_get_stream", "pack_online_create", "pack_online_destroy", "pack_online_epoch", "pack_online_info",
+           "pack_online_members", "pack_online_ensemble", "pack_online_snapshot", "pack_online_predict",
+           "pack_online_last_error"]
 
 
 class TabpackError(RuntimeError):
@@ -44,6 +48,13 @@ class Config(ctypes.Structure):
                 ("max_batch", ctypes.c_int32), ("task", ctypes.c_int32), ("precision", ctypes.c_int32),
                 ("seed", ctypes.c_uint64), ("beta1", ctypes.c_float), ("beta2", ctypes.c_float),
                 ("eps", ctypes.c_float), ("wd_on_bias", ctypes.c_int32), ("fuse_optimizer", ctypes.c_int32)]
+
+
+class OnlineInfo(ctypes.Structure):
+    _fields_ = [("epoch", ctypes.c_int32), ("stop", ctypes.c_int32), ("n_active", ctypes.c_int32),
+                ("ens_bad", ctypes.c_int32), ("best_epoch", ctypes.c_int32), ("n_best", ctypes.c_int32),
+                ("n_last", ctypes.c_int32), ("n_pool", ctypes.c_int32), ("best_score", ctypes.c_double),
+                ("last_score", ctypes.c_double)]
 
 
 _lib = None
@@ -80,6 +91,22 @@ def load_library(path: str = LIB_PATH):
         "pack_launch_count": (i64, [P]),
         "pack_sizes": (st, [P, P, P]),
         "pack_last_error": (ctypes.c_char_p, [P]),
+        "pack_member_size": (st, [P, i32, P]),
+        "pack_snapshot": (st, [P, i32, P]),
+        "pack_restore": (st, [P, i32, P]),
+        "pack_get_config": (st, [P, ctypes.POINTER(Config)]),
+        "pack_member_hparams": (st, [P, i32, P, P, P, P, P]),
+        "pack_get_active": (st, [P, P]),
+        "pack_get_stream": (P, [P]),
+        "pack_online_create": (st, [P, i64, i32, i32, i32, i32, ctypes.POINTER(P)]),
+        "pack_online_destroy": (None, [P]),
+        "pack_online_epoch": (st, [P, P, P, P]),
+        "pack_online_info": (st, [P, ctypes.POINTER(OnlineInfo)]),
+        "pack_online_members": (st, [P, P, P, P]),
+        "pack_online_ensemble": (st, [P, i32, P, P, P, P]),
+        "pack_online_snapshot": (st, [P, i32, P]),
+        "pack_online_predict": (st, [P, P, i64, P]),
+        "pack_online_last_error": (ctypes.c_char_p, [P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -182,6 +209,29 @@ class Pack:
         a = np.ascontiguousarray(active, dtype=np.uint8)
         _check(load_library().pack_set_active(self._h, _hptr(a)), self._h)
 
+    def get_active(self):
+        a = np.zeros(self.m, dtype=np.uint8)
+        _check(load_library().pack_get_active(self._h, _hptr(a)), self._h)
+        return a
+
+    def member_size(self, member):
+        n = ctypes.c_int64()
+        _check(load_library().pack_member_size(self._h, int(member), ctypes.byref(n)), self._h)
+        return n.value
+
+    def snapshot(self, member, out=None):
+        """Member's parameter run (float32 CUDA tensor of member_size elements)."""
+        t = self.torch
+        if out is None:
+            out = t.empty(self.member_size(member), dtype=t.float32, device="cuda")
+        _check(load_library().pack_snapshot(self._h, int(member), _dptr(out, t.float32)), self._h)
+        return out
+
+    def restore(self, member, run):
+        if run.numel() != self.member_size(member):
+            raise ValueError("snapshot size does not match the member")
+        _check(load_library().pack_restore(self._h, int(member), _dptr(run, self.torch.float32)), self._h)
+
     def layer_shape(self, member, layer):
         L, w = int(self.depth[member]), int(self.width[member])
         return (self.d_out if layer == L else w), (self.d_in if layer == 0 else w)
@@ -264,3 +314,82 @@ def select_greedy(preds, y, task, score="loss", m_ens=32, stream=None, static_sc
     _check(fn(_dptr(preds, torch.float32), P, N, d_out, _dptr(y, ydt), t, s, int(m_ens), _stream_ptr(stream),
               _hptr(sel), ctypes.byref(n), ctypes.byref(fin)))
     return sel[:n.value].copy(), fin.value
+
+
+def _ocheck(status, handle):
+    if status != TP_OK:
+        msg = load_library().pack_online_last_error(handle)
+        raise TabpackError(status, msg.decode() if msg else "")
+
+
+class OnlineEnsemble:
+    """Online ensemble of a Pack (Sec. 3.5) with ensemble and base-model
+    early stopping (Sec. 3.6); see pack_online_create."""
+
+    def __init__(self, pack, n_val, score="loss", m_ens=32, p_base=16, p_ens=32):
+        L = load_library()
+        self.pack = pack
+        self.n_val = int(n_val)
+        self.m_ens = int(m_ens)
+        s = SCORES[score] if isinstance(score, str) else int(score)
+        h = ctypes.c_void_p()
+        _ocheck(L.pack_online_create(pack._h, self.n_val, s, self.m_ens, int(p_base), int(p_ens), ctypes.byref(h)),
+                None)
+        self._h = h
+
+    def close(self):
+        if getattr(self, "_h", None):
+            load_library().pack_online_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def epoch(self, X_val, y_val):
+        """End of an epoch; returns the stop flag."""
+        t = self.pack.torch
+        stop = ctypes.c_int32()
+        _ocheck(load_library().pack_online_epoch(self._h, _dptr(X_val, t.float32), _dptr(y_val, self.pack._y_dtype()),
+                                                 ctypes.byref(stop)), self._h)
+        return bool(stop.value)
+
+    def info(self):
+        i = OnlineInfo()
+        _ocheck(load_library().pack_online_info(self._h, ctypes.byref(i)), self._h)
+        return {f: getattr(i, f) for f, _ in OnlineInfo._fields_}
+
+    def members(self):
+        m = self.pack.m
+        sc, best = np.zeros(m), np.zeros(m)
+        bad = np.zeros(m, dtype=np.int32)
+        _ocheck(load_library().pack_online_members(self._h, _hptr(sc), _hptr(best), _hptr(bad)), self._h)
+        return sc, best, bad
+
+    def ensemble(self, which="best"):
+        """(members, epochs, score) of the best or the last ensemble."""
+        w = {"best": 0, "last": 1}[which]
+        mem = np.zeros(self.m_ens, dtype=np.int32)
+        ep = np.zeros(self.m_ens, dtype=np.int32)
+        n = ctypes.c_int32()
+        sc = ctypes.c_double()
+        _ocheck(load_library().pack_online_ensemble(self._h, w, _hptr(mem), _hptr(ep), ctypes.byref(n),
+                                                    ctypes.byref(sc)), self._h)
+        return mem[:n.value].copy(), ep[:n.value].copy(), sc.value
+
+    def snapshot(self, j):
+        mem, _, _ = self.ensemble("best")
+        t = self.pack.torch
+        out = t.empty(self.pack.member_size(int(mem[j])), dtype=t.float32, device="cuda")
+        _ocheck(load_library().pack_online_snapshot(self._h, int(j), _dptr(out, t.float32)), self._h)
+        return out
+
+    def predict(self, X, out=None):
+        t = self.pack.torch
+        if out is None:
+            out = t.empty((X.shape[0], self.pack.d_out), dtype=t.float32, device=X.device)
+        _ocheck(load_library().pack_online_predict(self._h, _dptr(X, t.float32), X.shape[0], _dptr(out, t.float32)),
+                self._h)
+        return out

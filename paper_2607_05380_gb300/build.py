@@ -18,7 +18,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(HERE, "libtabpack.so")
 BUILD_DIR = os.path.join(HERE, "_build")
-SOURCES = ["tabpack.cu", "kernels.cu", "select.cu", "select_static.cu", "tc_gemm.cu"]
+SOURCES = ["tabpack.cu", "kernels.cu", "select.cu", "select_static.cu", "tc_gemm.cu", "online.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

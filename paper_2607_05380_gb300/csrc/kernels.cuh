@@ -127,8 +127,11 @@ struct SelectScratch {
 };
 int64_t select_scratch_bytes(int32_t P, int64_t N, int32_t d_out, int32_t m_ens);
 SelectScratch select_carve(void* base, int32_t P, int64_t N, int32_t d_out, int32_t m_ens);
+// excl: device uint8 [P] or NULL; candidates with excl[c] != 0 take no part.
+// solo: device double [P] or NULL; receives every candidate's score on its
+// own (the first iteration's values; NaN for excluded candidates).
 int select_enqueue(cudaStream_t st, const SelectScratch& s, const float* preds, int32_t P, int64_t N,
                    int32_t d_out, const void* y, int32_t task, int32_t score, int32_t m_ens,
-                   int64_t* launches);
+                   const uint8_t* excl, double* solo, int64_t* launches);
 
 }  // namespace tp

@@ -24,11 +24,13 @@ __device__ __forceinline__ double warp_sum_d(double v) {
 }
 
 __global__ void k_sel_init(double* __restrict__ S, int64_t n_S, int32_t* __restrict__ state, int32_t n_state,
-                           double* __restrict__ cur) {
+                           double* __restrict__ cur, const uint8_t* __restrict__ excl, int32_t m_ens) {
   for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n_S; e += (int64_t)gridDim.x * blockDim.x)
     S[e] = 0.0;
   if (blockIdx.x == 0) {
-    for (int e = threadIdx.x; e < n_state; e += blockDim.x) state[e] = 0;
+    const int used0 = kStHdr + m_ens;  // used[c] starts as excl[c]
+    for (int e = threadIdx.x; e < n_state; e += blockDim.x)
+      state[e] = (excl != nullptr && e >= used0) ? (excl[e - used0] != 0) : 0;
     if (threadIdx.x == 0) {
       state[kStLast] = -1;
       cur[0] = __longlong_as_double(0x7ff0000000000000LL);  // +inf
@@ -96,6 +98,25 @@ __global__ void __launch_bounds__(kSelThreads) k_sel_score(const double* __restr
   }
 }
 
+// Score of candidate c from its per-block partial sums: blocks in index
+// order, then the mean over N rows and the score's transform.
+__device__ __forceinline__ double cand_score(const double* __restrict__ partial, int c, int32_t n_blk, int64_t N,
+                                             int32_t score) {
+  double s = 0.0;
+  for (int b = 0; b < n_blk; ++b) s += partial[(int64_t)c * n_blk + b];
+  const double mean = s / (double)N;
+  return score == 1 ? -mean : (score == 2 ? sqrt(mean) : mean);
+}
+
+// Every candidate's score on its own, from the first iteration's partials.
+__global__ void k_sel_solo(const double* __restrict__ partial, int32_t P, int32_t n_blk, int64_t N, int32_t score,
+                           const int32_t* __restrict__ state, int32_t m_ens, double* __restrict__ solo) {
+  const int c = blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= P) return;
+  const int32_t* used = state + kStHdr + m_ens;
+  solo[c] = used[c] ? __longlong_as_double(0x7ff8000000000000LL) : cand_score(partial, c, n_blk, N, score);
+}
+
 __global__ void __launch_bounds__(1024) k_sel_pick(const double* __restrict__ partial, int32_t P, int32_t n_blk,
                                                    int64_t N, int32_t score, int32_t* __restrict__ state,
                                                    double* __restrict__ cur, int32_t m_ens) {
@@ -109,10 +130,7 @@ __global__ void __launch_bounds__(1024) k_sel_pick(const double* __restrict__ pa
   int best_c = -1;
   for (int c = threadIdx.x; c < P; c += blockDim.x) {
     if (used[c]) continue;
-    double s = 0.0;
-    for (int b = 0; b < n_blk; ++b) s += partial[(int64_t)c * n_blk + b];
-    double mean = s / (double)N;
-    double sc = score == 1 ? -mean : (score == 2 ? sqrt(mean) : mean);
+    const double sc = cand_score(partial, c, n_blk, N, score);
     if (sc < best) { best = sc; best_c = c; }   // ascending c per thread: lowest index wins ties
   }
   // block argmin, ties to the lowest index
@@ -184,16 +202,20 @@ SelectScratch select_carve(void* base, int32_t P, int64_t N, int32_t d_out, int3
 // Returns the number of the state words to copy back (header + selection).
 int select_enqueue(cudaStream_t st, const SelectScratch& s, const float* preds, int32_t P, int64_t N,
                    int32_t d_out, const void* y, int32_t task, int32_t score, int32_t m_ens,
-                   int64_t* launches) {
+                   const uint8_t* excl, double* solo, int64_t* launches) {
   const int32_t n_blk = (int32_t)ceil_div(N, kSelRowsPerBlock);
   const int64_t n_S = N * d_out;
   const int32_t n_state = kStHdr + m_ens + P;
   const int add_blocks = (int)std::min<int64_t>(ceil_div(n_S, 256), 152 * 8);
-  k_sel_init<<<add_blocks, 256, 0, st>>>(s.S, n_S, s.state, n_state, s.cur);
+  k_sel_init<<<add_blocks, 256, 0, st>>>(s.S, n_S, s.state, n_state, s.cur, excl, m_ens);
   int64_t nl = 1;
   for (int it = 0; it < m_ens; ++it) {
     k_sel_score<<<dim3(n_blk, P), kSelThreads, 0, st>>>(s.S, preds, y, N, d_out, task, score, s.state,
                                                         s.partial, n_blk, m_ens);
+    if (it == 0 && solo != nullptr) {
+      k_sel_solo<<<(int)ceil_div(P, 256), 256, 0, st>>>(s.partial, P, n_blk, N, score, s.state, m_ens, solo);
+      ++nl;
+    }
     k_sel_pick<<<1, 1024, 0, st>>>(s.partial, P, n_blk, N, score, s.state, s.cur, m_ens);
     k_sel_add<<<add_blocks, 256, 0, st>>>(s.S, preds, n_S, s.state);
     nl += 3;

@@ -92,7 +92,7 @@ tp_status pack_select_greedy_static(const float* preds, int32_t P, int64_t N, in
   SelectScratch s = select_carve(base, P, N, d_out, m_ens);
   // select_enqueue's first kernel zeroes the running sum and the state, so the
   // previous call's contents do not leak into this one.
-  select_enqueue(st, s, preds, P, N, d_out, y, task, score, m_ens, nullptr);
+  select_enqueue(st, s, preds, P, N, d_out, y, task, score, m_ens, nullptr, nullptr, nullptr);
   int32_t hdr[4] = {0, 0, 0, 0};
   double cur = 0.0;
   e = cudaGetLastError();

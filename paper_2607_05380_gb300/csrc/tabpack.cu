@@ -762,6 +762,13 @@ tp_status check_step_args(tabpack* h, const float* X, int64_t n_rows, const int3
   return TP_OK;
 }
 
+// Member i's contiguous run of the parameter arena: (first element, length).
+std::pair<int64_t, int64_t> member_run(const tabpack* h, int i) {
+  const int L = h->depth[i];
+  const int64_t first = h->W_off[i][0];
+  return {first, h->b_off[i][L] + h->cfg.d_out - first};
+}
+
 tp_status check_ml(tabpack* h, int member, int layer) {
   if (!h) return fail(nullptr, TP_EINVAL, "null pack");
   if (member < 0 || member >= h->cfg.m) return fail(h, TP_EINVAL, "member %d out of range", member);
@@ -930,6 +937,56 @@ tp_status pack_set_params(tabpack_t* h, int32_t member, int32_t layer, const flo
   return refresh_copies(h);
 }
 
+tp_status pack_member_size(const tabpack_t* h, int32_t member, int64_t* n_elems) {
+  if (!h || !n_elems) return fail(const_cast<tabpack_t*>(h), TP_EINVAL, "null argument");
+  if (member < 0 || member >= h->cfg.m) return fail(const_cast<tabpack_t*>(h), TP_EINVAL, "member %d out of range", member);
+  *n_elems = member_run(h, member).second;
+  return TP_OK;
+}
+
+tp_status pack_snapshot(tabpack_t* h, int32_t member, float* dst) {
+  TP_TRY(check_ml(h, member, 0));
+  if (!dst) return fail(h, TP_EINVAL, "null dst");
+  const auto run = member_run(h, member);
+  TP_CUDA(h, cudaMemcpyAsync(dst, h->params + run.first, (size_t)run.second * 4, cudaMemcpyDeviceToDevice, h->st));
+  return TP_OK;
+}
+
+tp_status pack_restore(tabpack_t* h, int32_t member, const float* src) {
+  TP_TRY(check_ml(h, member, 0));
+  if (!src) return fail(h, TP_EINVAL, "null src");
+  TP_TRY(sync_check(h));
+  const auto run = member_run(h, member);
+  TP_CUDA(h, cudaMemcpyAsync(h->params + run.first, src, (size_t)run.second * 4, cudaMemcpyDeviceToDevice, h->st));
+  return refresh_copies(h);
+}
+
+tp_status pack_get_config(const tabpack_t* h, tp_config* cfg) {
+  if (!h || !cfg) return fail(const_cast<tabpack_t*>(h), TP_EINVAL, "null argument");
+  *cfg = h->cfg;
+  return TP_OK;
+}
+
+tp_status pack_member_hparams(const tabpack_t* h, int32_t member, int32_t* depth, int32_t* width, float* dropout,
+                              float* lr, float* wd) {
+  if (!h) return fail(nullptr, TP_EINVAL, "null pack");
+  if (member < 0 || member >= h->cfg.m) return fail(const_cast<tabpack_t*>(h), TP_EINVAL, "member %d out of range", member);
+  if (depth) *depth = h->depth[member];
+  if (width) *width = h->width[member];
+  if (dropout) *dropout = h->dropout[member];
+  if (lr) *lr = h->lr[member];
+  if (wd) *wd = h->wd[member];
+  return TP_OK;
+}
+
+tp_status pack_get_active(const tabpack_t* h, uint8_t* active) {
+  if (!h || !active) return fail(const_cast<tabpack_t*>(h), TP_EINVAL, "null argument");
+  for (int i = 0; i < h->cfg.m; ++i) active[i] = h->active[i];
+  return TP_OK;
+}
+
+void* pack_get_stream(const tabpack_t* h) { return h ? (void*)h->st : nullptr; }
+
 tp_status pack_get_logits(tabpack_t* h, int32_t member, float* out) {
   TP_TRY(check_ml(h, member, 0));
   if (!out) return fail(h, TP_EINVAL, "null out");
@@ -993,7 +1050,7 @@ tp_status pack_select_greedy(const float* preds, int32_t P, int64_t N, int32_t d
   cudaError_t e = cudaMallocAsync(&scratch, (size_t)bytes, st);
   if (e != cudaSuccess) return fail(nullptr, TP_ENOMEM, "cudaMallocAsync(%lld): %s", (long long)bytes, cudaGetErrorString(e));
   SelectScratch s = select_carve(scratch, P, N, d_out, m_ens);
-  const int n_words = select_enqueue(st, s, preds, P, N, d_out, y, task, score, m_ens, nullptr);
+  const int n_words = select_enqueue(st, s, preds, P, N, d_out, y, task, score, m_ens, nullptr, nullptr, nullptr);
   std::vector<int32_t> host(n_words);
   double cur = 0.0;
   e = cudaGetLastError();
