@@ -67,6 +67,20 @@ struct tabpack {
   int64_t* part_stride_dev = nullptr;
   TcPlan tc;  // tensor-core GEMM plan (bf16 mode)
 
+  // bf16 prediction runs in chunks of P_cap rows (up to kPredictRows, built
+  // on first use) with its own forward-only tile plan over its own arenas:
+  // p_xb [P_cap, ldx] and, per member, two activation buffers
+  // [P_cap, w + 16] that consecutive layers use in turn (layer l writes
+  // buffer l & 1; a row block of layer l + 2 starts only after every tile of
+  // layer l + 1 on that row block has finished reading it).
+  TcPlan tcp;
+  int P_cap = 0;
+  void *p_xb = nullptr, *p_act = nullptr;
+  std::vector<std::array<int64_t, kMaxDepth>> p_act_off;
+  HeadJob* p_head_dev = nullptr;
+  int n_p_head = 0;
+  bool p_stale = true;      // active set changed since the prediction plan was built
+
   // schedule (active members)
   int n_active = 0, n_chunks = 0, n_head_jobs = 0;
   std::vector<std::pair<int, int>> fwd_rng, bwd_rng;  // CUDA-core tile ranges per depth index
@@ -183,6 +197,7 @@ void prof_flush(tabpack* h) {
 int ldh_of(const tabpack* h, int i) { return h->width[i] + kOnesCols; }
 
 void drop_graphs(tabpack* h);
+void free_predict(tabpack* h);
 
 // ------------------------------------------------------------------ layout
 tp_status build_layout(tabpack* h) {
@@ -377,6 +392,7 @@ tp_status build_schedule(tabpack* h) {
   TP_CUDA(h, cudaMemcpy(h->active_dev, h->active.data(), m, cudaMemcpyHostToDevice));
   h->n_head_jobs = (int)hj.size();
   h->n_chunks = (int)ch.size();
+  h->p_stale = true;
   if (h->bf16) {
     TcLayout lay;
     lay.depth = &h->depth;
@@ -462,6 +478,17 @@ tp_status alloc_all(tabpack* h) {
   return TP_OK;
 }
 
+void free_predict(tabpack* h) {
+  tc_free_plan(h->tcp);
+  for (void* p : {h->p_xb, h->p_act, (void*)h->p_head_dev})
+    if (p) cudaFree(p);
+  h->p_xb = h->p_act = nullptr;
+  h->p_head_dev = nullptr;
+  h->P_cap = 0;
+  h->n_p_head = 0;
+  h->p_stale = true;
+}
+
 void drop_graphs(tabpack* h) {
   for (auto& ge : h->graphs) cudaGraphExecDestroy(ge.exec);
   h->graphs.clear();
@@ -477,6 +504,7 @@ void free_all(tabpack* h) {
   if (h->dyn_host) cudaFreeHost(h->dyn_host);
   h->dyn_host = nullptr;
   tc_free_plan(h->tc);
+  free_predict(h);
   for (void* p : h->allocs) cudaFree(p);
   h->allocs.clear();
   for (auto e : h->prof.pool) cudaEventDestroy(e);
@@ -708,8 +736,111 @@ tp_status step_entry(tabpack* h, const float* X, int64_t n_rows, const int32_t* 
   return TP_OK;
 }
 
+constexpr int kPredictRows = 8192;
+
+// (Re)build the bf16 prediction plan for chunks of at least P_need rows.
+tp_status build_predict(tabpack* h, int P_need) {
+  if (h->tcp.enabled && !h->p_stale && h->P_cap >= P_need) return TP_OK;
+  const int m = h->cfg.m;
+  if (h->P_cap < P_need) {
+    TP_CUDA(h, cudaStreamSynchronize(h->st));
+    free_predict(h);
+    h->P_cap = P_need;
+    h->p_act_off.assign(m, {});
+    int64_t off = 0;
+    for (int i = 0; i < m; ++i) {
+      const int64_t buf = round_up((int64_t)h->P_cap * ldh_of(h, i), 128);
+      for (int l = 0; l < h->depth[i]; ++l) h->p_act_off[i][l] = off + (l & 1) * buf;
+      off += std::min(h->depth[i], 2) * buf;
+    }
+    const size_t xb_bytes = sizeof(__nv_bfloat16) * (size_t)h->P_cap * h->ldx;
+    const size_t act_bytes = sizeof(__nv_bfloat16) * (size_t)std::max<int64_t>(off, 128);
+    TP_CUDA(h, cudaMalloc(&h->p_xb, xb_bytes));
+    TP_CUDA(h, cudaMalloc(&h->p_act, act_bytes));
+    TP_CUDA(h, cudaMalloc(&h->p_head_dev, sizeof(HeadJob) * (size_t)m * (h->P_cap / kHeadRows)));
+    // columns the forward never writes (ones / pad columns) stay zero
+    TP_CUDA(h, cudaMemset(h->p_xb, 0, xb_bytes));
+    TP_CUDA(h, cudaMemset(h->p_act, 0, act_bytes));
+  }
+  TcLayout lay;
+  lay.depth = &h->depth;
+  lay.width = &h->width;
+  lay.active = &h->active;
+  lay.W_off = &h->W_off;
+  lay.b_off = &h->b_off;
+  lay.act_off = &h->p_act_off;
+  lay.dz_off = &h->dz_off;
+  lay.m = m;
+  lay.d_in_pad = h->d_in_pad;
+  lay.ldx = h->ldx;
+  lay.B_cap = h->P_cap;
+  lay.wq[0] = h->wq[0];
+  lay.wq[1] = h->wq[1];
+  lay.xb = h->p_xb;
+  lay.act = h->p_act;
+  lay.dz = nullptr;
+  lay.fwd_only = true;
+  TP_CUDA(h, cudaStreamSynchronize(h->st));
+  TP_TRY(tc_build_plan(h->tcp, lay, h->err));
+  std::vector<HeadJob> hj;
+  for (int i = 0; i < m; ++i) {
+    if (!h->active[i]) continue;
+    const int L = h->depth[i];
+    for (int b = 0; b < h->P_cap / kHeadRows; ++b) {
+      HeadJob j{};
+      j.member = i;
+      j.blk = b;
+      j.h_ld = ldh_of(h, i);
+      j.h_off = h->p_act_off[i][L - 1];
+      j.w_off = h->W_off[i][L];
+      j.b_off = h->b_off[i][L];
+      hj.push_back(j);
+    }
+  }
+  if (!hj.empty()) TP_CUDA(h, cudaMemcpy(h->p_head_dev, hj.data(), sizeof(HeadJob) * hj.size(), cudaMemcpyHostToDevice));
+  h->n_p_head = (int)hj.size();
+  h->p_stale = false;
+  return TP_OK;
+}
+
+// bf16 prediction: chunks of P_cap rows through the forward-only plan.
+tp_status run_predict_tc(tabpack* h, const float* X, int64_t N, float* out) {
+  TP_TRY(build_predict(h, (int)std::min<int64_t>(round_up(N, kRowTile), kPredictRows)));
+  for (int64_t n0 = 0; n0 < N; n0 += h->P_cap) {
+    const int rows = (int)std::min<int64_t>(h->P_cap, N - n0);
+    const int B_pad = (int)round_up(rows, kRowTile);
+    int slot;
+    prof_begin(h, TP_PH_PREDICT, &slot);
+    launch_gather<__nv_bfloat16>(h->st, X + n0 * h->cfg.d_in, nullptr, nullptr, rows, B_pad, h->cfg.d_in, h->d_in_pad,
+                                 h->ldx, (__nv_bfloat16*)h->p_xb, 0, h->t_dev, h->bias_corr, h->active_ids_dev, 0,
+                                 h->cfg.beta1, h->cfg.beta2, h->tcp.cnt_dev, h->tcp.n_cnt);
+    TP_LAUNCHED(h);
+    TP_TRY(tc_run_fwd(h->tcp, h->st, rows, B_pad, h->wcur, 0u, nullptr, 0, h->cfg.seed, h->params, h->mem_dev, h->p_act,
+                      h->err));
+    TP_LAUNCHED(h);
+    PredictHeadArgs<__nv_bfloat16> pg;
+    pg.jobs = h->p_head_dev;
+    pg.mem = h->mem_dev;
+    pg.act = (const __nv_bfloat16*)h->p_act;
+    pg.params = h->params;
+    pg.out = out;
+    pg.N = N;
+    pg.n0 = n0;
+    pg.rows = rows;
+    pg.d_out = h->cfg.d_out;
+    pg.task = h->cfg.task;
+    pg._pad = 0;
+    launch_predict_head<__nv_bfloat16>(h->st, pg, h->n_p_head);
+    TP_LAUNCHED(h);
+    h->launches += 3;
+    prof_end(h, slot, 3, TP_PH_PREDICT);
+  }
+  return TP_OK;
+}
+
 template <typename T>
 tp_status run_predict(tabpack* h, const float* X, int64_t N, float* out) {
+  if (h->bf16) return run_predict_tc(h, X, N, out);
   for (int64_t n0 = 0; n0 < N; n0 += h->B_cap) {
     const int rows = (int)std::min<int64_t>(h->B_cap, N - n0);
     const int B_pad = (int)round_up(rows, kRowTile);
@@ -780,6 +911,7 @@ tp_status check_ml(tabpack* h, int member, int layer) {
 tp_status sync_check(tabpack* h) {
   TP_CUDA(h, cudaStreamSynchronize(h->st));
   if (h->bf16 && h->tc.enabled) TP_TRY(tc_check(h->tc, h->st, h->err));
+  if (h->bf16 && h->tcp.enabled) TP_TRY(tc_check(h->tcp, h->st, h->err));
   return TP_OK;
 }
 

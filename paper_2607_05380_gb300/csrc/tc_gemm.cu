@@ -887,6 +887,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
             return TP_ECUDA;
           if (set == 0) plan.map_act[(size_t)i * kMaxDepth + l] = (int)maps.size();
           maps.push_back(mp);
+          if (lay.fwd_only) continue;
           if (!encode_map(&mp, dzb + (*lay.dz_off)[i][l], w, lay.B_cap, w, br, err)) return TP_ECUDA;
           if (set == 0) plan.map_dz[(size_t)i * kMaxDepth + l] = (int)maps.size();
           maps.push_back(mp);
@@ -973,7 +974,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
   // with the next level's dgrad tiles (below).
   const int nrb = lay.B_cap / kRowTile;
   if (plan.cnt_dev == nullptr) {
-    plan.n_cnt = 2 * m * kMaxDepth * nrb;
+    plan.n_cnt = (lay.fwd_only ? 1 : 2) * m * kMaxDepth * nrb;
     if (cudaMalloc(&plan.cnt_dev, sizeof(int) * plan.n_cnt) != cudaSuccess ||
         cudaMemset(plan.cnt_dev, 0, sizeof(int) * plan.n_cnt) != cudaSuccess) {
       err = "cudaMalloc(tc counters) failed";
@@ -1041,6 +1042,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
     sorted_append(v);
   }
   plan.fwd_rng = {0, (int)all.size()};
+  if (lay.fwd_only) Lmax = 0;  // no backward tiles
   std::vector<std::vector<TcTile>> VD(Lmax), VW(Lmax);
   for (int lev = 0; lev < Lmax; ++lev) {
     std::vector<TcTile>& vd = VD[lev];

@@ -73,6 +73,7 @@ struct TcLayout {          // what the plan needs to know about the pack's arena
   const void* xb;
   const void* act;
   const void* dz;
+  bool fwd_only = false;   // forward tiles only (prediction): no dz maps, counters or backward tiles
 };
 
 tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err);

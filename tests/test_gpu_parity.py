@@ -350,12 +350,35 @@ def test_predict(tp, prec, task, d_out):
     d_in = 19
     hp = random_pack(5, d_in, d_out, seed=30 + d_out, width=(16, 96, 16))
     pk, orc = pair(tp, task, d_in, d_out, hp, prec, 128)
-    X, y = make_data(task, 333, d_in, d_out, 4)   # 3 row chunks of 128, ragged tail
+    X, y = make_data(task, 333, d_in, d_out, 4)   # fp32: 3 row chunks of 128, ragged tail; bf16: one of 384
     (Xd,) = to_dev(X)
     out = pk.predict(Xd).cpu().numpy()
     ref = orc.predict(X)
     for i in range(5):
         assert rel_err(out[i], ref[i]) <= TOL[prec], i
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_predict_chunks(tp, prec):
+    """8525 rows: bf16 prediction runs in chunks of 8192 rows (a full chunk and
+    a ragged one), fp32 in chunks of max_batch.  Each row's prediction does
+    not depend on the chunk it falls in (bit-exact), and a change of the
+    active set rebuilds the prediction plan without changing the others."""
+    d_in, d_out = 19, 6
+    hp = random_pack(5, d_in, d_out, seed=44, width=(16, 96, 16))
+    pk, orc = pair(tp, "multiclass", d_in, d_out, hp, prec, 128)
+    X, _ = make_data("multiclass", 8525, d_in, d_out, 8)
+    (Xd,) = to_dev(X)
+    full = pk.predict(Xd).cpu().numpy()
+    ref = orc.predict(X)
+    for i in range(5):
+        assert rel_err(full[i], ref[i]) <= TOL[prec], i
+    np.testing.assert_array_equal(pk.predict(Xd[8192:].contiguous()).cpu().numpy(), full[:, 8192:])
+    np.testing.assert_array_equal(pk.predict(Xd[:100].contiguous()).cpu().numpy(), full[:, :100])
+    pk.set_active([1, 0, 1, 1, 1])
+    part = pk.predict(Xd[:300].contiguous()).cpu().numpy()
+    for i in (0, 2, 3, 4):
+        np.testing.assert_array_equal(part[i], full[i, :300])
 
 
 @pytest.mark.parametrize("prec,fuse", [("fp32", False), ("bf16", False), ("bf16", True)])
