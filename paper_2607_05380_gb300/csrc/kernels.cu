@@ -1,6 +1,8 @@
 // kernels.cu -- element-wise, reduction and CUDA-core matrix kernels of the
 // packed training step (gather, CUDA-core grouped GEMM, head + loss + head
 // AdamW, AdamW, init, predict head, mask dump).
+#include <type_traits>
+
 #include "kernels.cuh"
 
 namespace tp {
@@ -229,17 +231,181 @@ __device__ __forceinline__ float row_loss(int task, int d_out, const float (&z)[
 }
 
 // ------------------------------------------------------------- head + loss
-// One block per (member, 32-row block); each warp owns 4 rows and walks them
-// R at a time (lanes over 8-column groups, 16-byte loads), so every head-weight
-// load serves R rows.  Per row: logits, loss and dlogits, then dZ of the last
-// hidden layer = (dlogits W_h) * [H > 0] / (1 - p).  Then per column group the
-// block's partial head-weight gradient over its 32 rows, in row order.
+// Values of G consecutive columns as floats, and back.
+template <int G>
+__device__ __forceinline__ void loadG(const __nv_bfloat16* p, float (&h)[G]) {
+  if constexpr (G == 8) {
+    load8(p, h);
+  } else if constexpr (G == 4) {
+    const uint2 u = *reinterpret_cast<const uint2*>(p);
+    const __nv_bfloat16* b = reinterpret_cast<const __nv_bfloat16*>(&u);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) h[k] = __bfloat162float(b[k]);
+  } else if constexpr (G == 2) {
+    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(p));
+    h[0] = f.x;
+    h[1] = f.y;
+  } else {
+    h[0] = __bfloat162float(*p);
+  }
+}
+template <int G>
+__device__ __forceinline__ void loadG(const float* p, float (&h)[G]) {
+  if constexpr (G == 8) {
+    load8(p, h);
+  } else if constexpr (G == 4) {
+    const float4 a = *reinterpret_cast<const float4*>(p);
+    h[0] = a.x; h[1] = a.y; h[2] = a.z; h[3] = a.w;
+  } else if constexpr (G == 2) {
+    const float2 a = *reinterpret_cast<const float2*>(p);
+    h[0] = a.x; h[1] = a.y;
+  } else {
+    h[0] = *p;
+  }
+}
+template <int G>
+__device__ __forceinline__ void storeG(__nv_bfloat16* p, const float (&v)[G]) {
+  if constexpr (G == 8) {
+    store8(p, v);
+  } else if constexpr (G == 4) {
+    uint2 u;
+    __nv_bfloat162* b = reinterpret_cast<__nv_bfloat162*>(&u);
+    b[0] = __floats2bfloat162_rn(v[0], v[1]);
+    b[1] = __floats2bfloat162_rn(v[2], v[3]);
+    *reinterpret_cast<uint2*>(p) = u;
+  } else if constexpr (G == 2) {
+    *reinterpret_cast<__nv_bfloat162*>(p) = __floats2bfloat162_rn(v[0], v[1]);
+  } else {
+    *p = __float2bfloat16_rn(v[0]);
+  }
+}
+template <int G>
+__device__ __forceinline__ void storeG(float* p, const float (&v)[G]) {
+  if constexpr (G == 8) {
+    store8(p, v);
+  } else if constexpr (G == 4) {
+    *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+  } else if constexpr (G == 2) {
+    *reinterpret_cast<float2*>(p) = make_float2(v[0], v[1]);
+  } else {
+    *p = v[0];
+  }
+}
+
+// G consecutive elements of T loaded with one vector load and converted to
+// float when used, so that several rows' loads can be in flight at once.
+template <typename T, int G>
+struct RawG;
+template <int G>
+struct RawG<__nv_bfloat16, G> {
+  using V = std::conditional_t<G == 8, uint4, std::conditional_t<G == 4, uint2,
+                               std::conditional_t<G == 2, uint32_t, unsigned short>>>;
+  V v;
+  __device__ __forceinline__ void load(const __nv_bfloat16* p) { v = *reinterpret_cast<const V*>(p); }
+  __device__ __forceinline__ void to_float(float (&h)[G]) const {
+    const __nv_bfloat16* b = reinterpret_cast<const __nv_bfloat16*>(&v);
+#pragma unroll
+    for (int k = 0; k < G; ++k) h[k] = __bfloat162float(b[k]);
+  }
+};
+template <int G>
+struct RawG<float, G> {
+  float v[G];
+  __device__ __forceinline__ void load(const float* p) { loadG<G>(p, v); }
+  __device__ __forceinline__ void to_float(float (&h)[G]) const {
+#pragma unroll
+    for (int k = 0; k < G; ++k) h[k] = v[k];
+  }
+};
+
+// The logit pass of a head block (128 rows of one member, 8 warps of 16
+// rows).  LPR lanes share a row (the smallest power of two >= the row's
+// 8-column groups, at most 32; lanes walk the groups with 16-byte loads) and
+// a warp's 32 / LPR lane groups take different rows, R rows per group at a
+// time, so that every head-weight load serves R rows.  After the call the
+// group's lane 0 holds the R rows' logits (bias added); `rl0` is the block-
+// local index of the group's first row and `live` whether the group has
+// rows in this pass.  Returns the number of passes.
+template <typename T, int DO, int R>
+struct HeadLogits {
+  static constexpr int kRowsPerWarp = kHeadRows / 8;
+  int lpr, groups, grp, gl;
+  __device__ __forceinline__ HeadLogits(int w, int lane) {
+    const int ng = w >> 3;
+    lpr = 1;
+    while (lpr < ng && lpr < 32) lpr <<= 1;
+    groups = min(32 / lpr, kRowsPerWarp / R);
+    grp = lane / lpr;
+    gl = lane % lpr;
+  }
+  __device__ __forceinline__ int step() const { return groups * R; }
+  // rows rl0 .. rl0 + R - 1 (block-local) of H (block origin), head weights Wh [d_out, w]
+  __device__ __forceinline__ void run(const T* __restrict__ H, int ldh, const float* __restrict__ Wh,
+                                      const float* __restrict__ bh, int w, int d_out,
+                                      int rl0, bool live, float (&acc)[R][DO]) const {
+#pragma unroll
+    for (int q = 0; q < R; ++q)
+#pragma unroll
+      for (int c = 0; c < DO; ++c) acc[q][c] = 0.f;
+    if (live) {
+      // two-deep register pipeline over the column groups: the next group's
+      // rows are in flight while this group's products run
+      const int ng = w >> 3;
+      RawG<T, 8> cur[R], nxt[R];
+      if (gl < ng)
+#pragma unroll
+        for (int q = 0; q < R; ++q) cur[q].load(H + (int64_t)(rl0 + q) * ldh + 8 * gl);
+      for (int gi = gl; gi < ng; gi += lpr) {
+        if (gi + lpr < ng)
+#pragma unroll
+          for (int q = 0; q < R; ++q) nxt[q].load(H + (int64_t)(rl0 + q) * ldh + 8 * (gi + lpr));
+        float h[R][8];
+#pragma unroll
+        for (int q = 0; q < R; ++q) cur[q].to_float(h[q]);
+#pragma unroll
+        for (int c = 0; c < DO; ++c) {
+          if (c < d_out) {
+            float w8[8];
+            load8(Wh + (int64_t)c * w + 8 * gi, w8);
+#pragma unroll
+            for (int q = 0; q < R; ++q)
+#pragma unroll
+              for (int k = 0; k < 8; ++k) acc[q][c] = fmaf(h[q][k], w8[k], acc[q][c]);
+          }
+        }
+#pragma unroll
+        for (int q = 0; q < R; ++q) cur[q] = nxt[q];
+      }
+    }
+    // sum over the group's lanes (every lane of the warp takes part)
+    for (int o = lpr >> 1; o > 0; o >>= 1)
+#pragma unroll
+      for (int q = 0; q < R; ++q)
+#pragma unroll
+        for (int c = 0; c < DO; ++c)
+          if (c < d_out) acc[q][c] += __shfl_xor_sync(0xffffffffu, acc[q][c], o);
+#pragma unroll
+    for (int q = 0; q < R; ++q)
+#pragma unroll
+      for (int c = 0; c < DO; ++c)
+        if (c < d_out) acc[q][c] += bh[c];
+  }
+};
+
+// One block per (member, 128-row block), 256 threads.
+//   1. logits, per-row loss and dlogits (HeadLogits; the group's lane 0 takes
+//      the loss of its rows) into shared memory;
+//   2. the gradient pass: a thread owns G = head_cols(DO) columns and keeps
+//      their head weights and partial weight gradients in registers while it
+//      walks its rows in order: dZ of the last hidden layer
+//      = (dlogits W_h) * [H > 0] / (1 - p), and dW_h += dlogits^T H.  Narrow
+//      heads split the rows into jb.split sets, added in order in shared
+//      memory, so that every block writes one partial.
 template <typename T, int DO>
-__global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
-  // rows per head-weight load: 4 for the one-logit head; 1 for class heads,
-  // whose per-row state (DO logits and dlogits) would otherwise cost occupancy
-  constexpr int R = DO == 1 ? 4 : (DO <= 4 ? 2 : 1);
-  constexpr int RW = kHeadRows / 8;  // rows per warp
+__global__ void __launch_bounds__(256, 2) k_head(HeadArgs<T> g) {
+  constexpr int R = DO <= 10 ? 4 : 2;
+  constexpr int G = head_cols(DO);
+  constexpr int DOP = DO == 1 ? 1 : (DO + 3) & ~3;  // padded row of dlogits in shared memory
   pdl_trigger();
   pdl_wait();
   const HeadJob jb = g.jobs[blockIdx.x];
@@ -247,130 +413,129 @@ __global__ void __launch_bounds__(256) k_head(HeadArgs<T> g) {
   if (r0 >= g.B_pad) return;
   const MemberDev md = g.mem[jb.member];
   const int w = md.w, d_out = g.d_out, ldh = jb.h_ld;
-  const int ng = w >> 3;  // 8-column groups (widths are multiples of 16)
-  const T* H = g.act + jb.h_off;
-  const float* Wh = g.params + jb.w_off;
-  const float* bh = g.params + jb.b_off;
-  __shared__ float dlog[kHeadRows][DO];
+  const T* __restrict__ H = g.act + jb.h_off + (int64_t)r0 * ldh;
+  const float* __restrict__ Wh = g.params + jb.w_off;
+  const float* __restrict__ bh = g.params + jb.b_off;
+  __shared__ __align__(16) float dlog[kHeadRows][DOP];
   __shared__ float lrow[kHeadRows];
+  __shared__ __align__(16) float red[256 * G * DO];  // row-set partials when the rows are split
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float invB = 1.f / (float)g.B;
-  T* dZ = g.dz + jb.dz_off;
-  for (int q0 = 0; q0 < RW; q0 += R) {
-    const int rl0 = warp * RW + q0;  // first local row of this pass
+
+  const HeadLogits<T, DO, R> hl(w, lane);
+  for (int p0 = 0; p0 < HeadLogits<T, DO, R>::kRowsPerWarp; p0 += hl.step()) {
+    const int rl0 = warp * HeadLogits<T, DO, R>::kRowsPerWarp + p0 + hl.grp * R;
+    const bool live = hl.grp < hl.groups;
     float acc[R][DO];
+    hl.run(H, ldh, Wh, bh, w, d_out, rl0, live, acc);
+    if (live && hl.gl == 0) {
+      const int32_t* idx = g.dyn ? g.dyn->idx : g.idx;
+      const void* yv = g.dyn ? g.dyn->y : g.y;
 #pragma unroll
-    for (int q = 0; q < R; ++q)
+      for (int q = 0; q < R; ++q) {
+        const int r = r0 + rl0 + q;
+        float dl[DO];
+        float loss = 0.f;
 #pragma unroll
-      for (int c = 0; c < DO; ++c) acc[q][c] = 0.f;
-    for (int gi = lane; gi < ng; gi += 32) {
-      float h[R][8];
+        for (int c = 0; c < DO; ++c) dl[c] = 0.f;
+        if (r < g.B) {
+          const int64_t row = idx ? (int64_t)idx[r] : (int64_t)r;
+          loss = row_loss<DO>(g.task, d_out, acc[q], yv, row, invB, dl);
+          float* lg = g.logits + ((int64_t)jb.member * g.B_cap + r) * d_out;
 #pragma unroll
-      for (int q = 0; q < R; ++q) load8(H + (int64_t)(r0 + rl0 + q) * ldh + 8 * gi, h[q]);
-#pragma unroll
-      for (int c = 0; c < DO; ++c) {
-        if (c < d_out) {
-          float w8[8];
-          load8(Wh + (int64_t)c * w + 8 * gi, w8);
-#pragma unroll
-          for (int q = 0; q < R; ++q)
-#pragma unroll
-            for (int k = 0; k < 8; ++k) acc[q][c] = fmaf(h[q][k], w8[k], acc[q][c]);
+          for (int c = 0; c < DO; ++c)
+            if (c < d_out) lg[c] = acc[q][c];
         }
-      }
-    }
-    float dl[R][DO];
 #pragma unroll
-    for (int q = 0; q < R; ++q) {
-#pragma unroll
-      for (int c = 0; c < DO; ++c)
-        if (c < d_out) acc[q][c] = warp_sum(acc[q][c]) + bh[c];
-      const int r = r0 + rl0 + q;
-      float loss = 0.f;
-#pragma unroll
-      for (int c = 0; c < DO; ++c) dl[q][c] = 0.f;
-      if (r < g.B) {
-        const int32_t* idx = g.dyn ? g.dyn->idx : g.idx;
-        const void* yv = g.dyn ? g.dyn->y : g.y;
-        const int64_t row = idx ? (int64_t)idx[r] : (int64_t)r;
-        loss = row_loss<DO>(g.task, d_out, acc[q], yv, row, invB, dl[q]);
-        float z = 0.f;
-#pragma unroll
-        for (int c = 0; c < DO; ++c) if (c == lane) z = acc[q][c];
-        if (lane < d_out) g.logits[((int64_t)jb.member * g.B_cap + r) * d_out + lane] = z;
-      }
-      if (lane == 0) {
-#pragma unroll
-        for (int c = 0; c < DO; ++c) dlog[rl0 + q][c] = dl[q][c];
+        for (int c = 0; c < DOP; ++c) dlog[rl0 + q][c] = c < DO ? dl[c < DO ? c : 0] : 0.f;
         lrow[rl0 + q] = loss;
-      }
-    }
-    for (int gi = lane; gi < ng; gi += 32) {
-      float h[R][8], s[R][8];
-#pragma unroll
-      for (int q = 0; q < R; ++q) {
-        load8(H + (int64_t)(r0 + rl0 + q) * ldh + 8 * gi, h[q]);
-#pragma unroll
-        for (int k = 0; k < 8; ++k) s[q][k] = 0.f;
-      }
-#pragma unroll
-      for (int c = 0; c < DO; ++c) {
-        if (c < d_out) {
-          float w8[8];
-          load8(Wh + (int64_t)c * w + 8 * gi, w8);
-#pragma unroll
-          for (int q = 0; q < R; ++q)
-#pragma unroll
-            for (int k = 0; k < 8; ++k) s[q][k] = fmaf(dl[q][c], w8[k], s[q][k]);
-        }
-      }
-#pragma unroll
-      for (int q = 0; q < R; ++q) {
-#pragma unroll
-        for (int k = 0; k < 8; ++k) s[q][k] = h[q][k] > 0.f ? s[q][k] * md.scale : 0.f;
-        store8(dZ + (int64_t)(r0 + rl0 + q) * w + 8 * gi, s[q]);
       }
     }
   }
   __syncthreads();
-  // partial head gradients of this block: per group of G columns, all
-  // classes, rows in increasing order
-  constexpr int G = DO <= 2 ? 8 : (DO <= 16 ? 4 : 2);
+
+  const int n_cg = w / G;
+  const int S = jb.split;
+  const int rows_per_set = kHeadRows / S;
+  T* __restrict__ dZ = g.dz + jb.dz_off + (int64_t)r0 * w;
   float* part = g.head_part + jb.part_off;
-  for (int gi = threadIdx.x; gi < w / G; gi += blockDim.x) {
-    float a[DO][G];
+  for (int u = threadIdx.x; u < n_cg * S; u += blockDim.x) {
+    const int cg = u % n_cg, set = u / n_cg;
+    const int col = G * cg;
+    float Wr[DO][G], a[DO][G];
 #pragma unroll
-    for (int c = 0; c < DO; ++c)
+    for (int c = 0; c < DO; ++c) {
+      if (c < d_out) loadG<G>(Wh + (int64_t)c * w + col, Wr[c]);
+      else {
 #pragma unroll
-      for (int k = 0; k < G; ++k) a[c][k] = 0.f;
-#pragma unroll 4
-    for (int rr = 0; rr < kHeadRows; ++rr) {
-      const T* hp = H + (int64_t)(r0 + rr) * ldh + G * gi;
-      float h[G];
-      if constexpr (G == 8) {
-        load8(hp, h);
-      } else {
-#pragma unroll
-        for (int k = 0; k < G; ++k) h[k] = Elem<T>::to_f(hp[k]);
+        for (int k = 0; k < G; ++k) Wr[c][k] = 0.f;
       }
 #pragma unroll
-      for (int c = 0; c < DO; ++c)
-        if (c < d_out) {
-          const float d = dlog[rr][c];
-#pragma unroll
-          for (int k = 0; k < G; ++k) a[c][k] = fmaf(d, h[k], a[c][k]);
-        }
+      for (int k = 0; k < G; ++k) a[c][k] = 0.f;
     }
+    const int rb = set * rows_per_set;
+    // rows in batches of U (rows_per_set is a multiple of 8): the batch's
+    // loads are all issued before its products
+    constexpr int U = 8;
+    for (int rb0 = rb; rb0 < rb + rows_per_set; rb0 += U) {
+      RawG<T, G> raw[U];
 #pragma unroll
-    for (int c = 0; c < DO; ++c)
-      if (c < d_out)
+      for (int u2 = 0; u2 < U; ++u2) raw[u2].load(H + (int64_t)(rb0 + u2) * ldh + col);
 #pragma unroll
-        for (int k = 0; k < G; ++k) part[(int64_t)c * w + G * gi + k] = a[c][k];
+      for (int u2 = 0; u2 < U; ++u2) {
+      const int rr = rb0 + u2;
+      float h[G], s[G];
+      raw[u2].to_float(h);
+      float dl[DOP];
+      if constexpr (DOP % 4 == 0) {
+#pragma unroll
+        for (int c = 0; c < DOP; c += 4) {
+          const float4 v = *reinterpret_cast<const float4*>(&dlog[rr][c]);
+          dl[c] = v.x; dl[c + 1] = v.y; dl[c + 2] = v.z; dl[c + 3] = v.w;
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < DOP; ++c) dl[c] = dlog[rr][c];
+      }
+#pragma unroll
+      for (int k = 0; k < G; ++k) s[k] = 0.f;
+#pragma unroll
+      for (int c = 0; c < DO; ++c)
+#pragma unroll
+        for (int k = 0; k < G; ++k) {
+          s[k] = fmaf(dl[c], Wr[c][k], s[k]);
+          a[c][k] = fmaf(dl[c], h[k], a[c][k]);
+        }
+#pragma unroll
+      for (int k = 0; k < G; ++k) s[k] = h[k] > 0.f ? s[k] * md.scale : 0.f;
+      storeG<G>(dZ + (int64_t)rr * w + col, s);
+      }
+    }
+    if (S == 1) {
+#pragma unroll
+      for (int c = 0; c < DO; ++c)
+        if (c < d_out) storeG<G>(part + (int64_t)c * w + col, a[c]);
+    } else {  // n_cg * S <= 256: one (column group, row set) per thread
+#pragma unroll
+      for (int c = 0; c < DO; ++c)
+        if (c < d_out) storeG<G>(&red[((set * DO + c) * n_cg + cg) * G], a[c]);
+    }
   }
+  if (S > 1) {  // the block's partial: row sets added in order
+    __syncthreads();
+    for (int e = threadIdx.x; e < d_out * w; e += blockDim.x) {
+      const int c = e / w, k = e - c * w;
+      const int cg = k / G, kk = k - cg * G;
+      float v = 0.f;
+      for (int set = 0; set < S; ++set) v += red[((set * DO + c) * n_cg + cg) * G + kk];
+      part[e] = v;
+    }
+  }
+  // bias partial and loss partial of the block (rows in order)
   if (threadIdx.x < d_out) {
-    float s = 0.f;
-    for (int rr = 0; rr < kHeadRows; ++rr) s += dlog[rr][threadIdx.x];
-    part[(int64_t)d_out * w + threadIdx.x] = s;
+    float v = 0.f;
+    for (int rr = 0; rr < kHeadRows; ++rr) v += dlog[rr][threadIdx.x];
+    part[(int64_t)d_out * w + threadIdx.x] = v;
   }
   if (threadIdx.x == 0) {
     float s = 0.f;
@@ -410,6 +575,7 @@ __global__ void k_head_reduce(HeadReduceArgs g) {
   }
   for (int e = e0 + threadIdx.x; e < min(e0 + (int)blockDim.x, d_out * w + d_out); e += blockDim.x) {
     float s = 0.f;
+#pragma unroll 8
     for (int b = 0; b < n_blk; ++b) s += g.head_part[jb.part_off + b * stride + e];
     const bool is_b = e >= d_out * w;
     const int64_t o = is_b ? jb.gb_off + (e - d_out * w) : jb.gw_off + e;
@@ -536,52 +702,43 @@ __global__ void k_refresh_wq(const float* __restrict__ p, __nv_bfloat16* __restr
 // out[member, n0 + r, :] for r < rows.
 template <typename T, int DO>
 __global__ void __launch_bounds__(256) k_predict_head(PredictHeadArgs<T> g) {
+  constexpr int R = DO <= 10 ? 4 : 2;
   pdl_wait();
   const HeadJob jb = g.jobs[blockIdx.x];
   const int r0 = jb.blk * kHeadRows;
   if (r0 >= g.rows) return;
   const MemberDev md = g.mem[jb.member];
   const int w = md.w, d_out = g.d_out, ldh = jb.h_ld;
-  const T* H = g.act + jb.h_off;
+  const T* H = g.act + jb.h_off + (int64_t)r0 * ldh;
   const float* Wh = g.params + jb.w_off;
   const float* bh = g.params + jb.b_off;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int rr = warp; rr < kHeadRows; rr += 8) {
-    const int r = r0 + rr;
-    if (r >= g.rows) break;
-    float acc[DO];
+  const HeadLogits<T, DO, R> hl(w, lane);
+  for (int p0 = 0; p0 < HeadLogits<T, DO, R>::kRowsPerWarp; p0 += hl.step()) {
+    const int rl0 = warp * HeadLogits<T, DO, R>::kRowsPerWarp + p0 + hl.grp * R;
+    const bool live = hl.grp < hl.groups && r0 + rl0 < g.rows;
+    float acc[R][DO];
+    hl.run(H, ldh, Wh, bh, w, d_out, rl0, live, acc);
+    if (!live || hl.gl != 0) continue;
 #pragma unroll
-    for (int c = 0; c < DO; ++c) acc[c] = 0.f;
-    for (int gi = lane; gi < (w >> 3); gi += 32) {
-      float h[8];
-      load8(H + (int64_t)r * ldh + 8 * gi, h);
+    for (int q = 0; q < R; ++q) {
+      const int r = r0 + rl0 + q;
+      if (r >= g.rows) break;
+      float* o = g.out + ((int64_t)jb.member * g.N + g.n0 + r) * d_out;
+      if (g.task == 1) {
+        float mx = acc[q][0];
 #pragma unroll
-      for (int c = 0; c < DO; ++c) {
-        if (c < d_out) {
-          float w8[8];
-          load8(Wh + (int64_t)c * w + 8 * gi, w8);
+        for (int c = 1; c < DO; ++c) if (c < d_out) mx = fmaxf(mx, acc[q][c]);
+        float sum = 0.f;
 #pragma unroll
-          for (int k = 0; k < 8; ++k) acc[c] = fmaf(h[k], w8[k], acc[c]);
-        }
+        for (int c = 0; c < DO; ++c) if (c < d_out) sum += expf(acc[q][c] - mx);
+        const float inv = 1.f / sum;
+#pragma unroll
+        for (int c = 0; c < DO; ++c)
+          if (c < d_out) o[c] = expf(acc[q][c] - mx) * inv;
+      } else {
+        o[0] = g.task == 0 ? 1.f / (1.f + expf(-acc[q][0])) : acc[q][0];
       }
-    }
-#pragma unroll
-    for (int c = 0; c < DO; ++c)
-      if (c < d_out) acc[c] = warp_sum(acc[c]) + bh[c];
-    float* o = g.out + ((int64_t)jb.member * g.N + g.n0 + r) * d_out;
-    if (g.task == 1) {
-      float mx = acc[0];
-#pragma unroll
-      for (int c = 1; c < DO; ++c) if (c < d_out) mx = fmaxf(mx, acc[c]);
-      float s = 0.f;
-#pragma unroll
-      for (int c = 0; c < DO; ++c) if (c < d_out) s += expf(acc[c] - mx);
-      const float inv = 1.f / s;
-#pragma unroll
-      for (int c = 0; c < DO; ++c)
-        if (c < d_out && c == lane) o[c] = expf(acc[c] - mx) * inv;
-    } else if (lane == 0) {
-      o[0] = g.task == 0 ? 1.f / (1.f + expf(-acc[0])) : acc[0];
     }
   }
 }
@@ -623,14 +780,15 @@ void launch_gemm_simt(cudaStream_t st, const GemmArgs<T>& g, int tile_base, int 
 template <typename T>
 void launch_head(cudaStream_t st, const HeadArgs<T>& g, int n_jobs) {
   if (n_jobs <= 0) return;
-  // class-count buckets: the loops over classes are unrolled to the bucket size
-  if (g.d_out == 1) launch_pdl(k_head<T, 1>, dim3(n_jobs), dim3(256), 0, st, g);
-  else if (g.d_out <= 2) launch_pdl(k_head<T, 2>, dim3(n_jobs), dim3(256), 0, st, g);
-  else if (g.d_out <= 4) launch_pdl(k_head<T, 4>, dim3(n_jobs), dim3(256), 0, st, g);
-  else if (g.d_out <= 8) launch_pdl(k_head<T, 8>, dim3(n_jobs), dim3(256), 0, st, g);
-  else if (g.d_out <= 10) launch_pdl(k_head<T, 10>, dim3(n_jobs), dim3(256), 0, st, g);
-  else if (g.d_out <= 16) launch_pdl(k_head<T, 16>, dim3(n_jobs), dim3(256), 0, st, g);
-  else launch_pdl(k_head<T, kMaxDout>, dim3(n_jobs), dim3(256), 0, st, g);
+  switch (head_bucket(g.d_out)) {
+    case 1: launch_pdl(k_head<T, 1>, dim3(n_jobs), dim3(256), 0, st, g); break;
+    case 2: launch_pdl(k_head<T, 2>, dim3(n_jobs), dim3(256), 0, st, g); break;
+    case 4: launch_pdl(k_head<T, 4>, dim3(n_jobs), dim3(256), 0, st, g); break;
+    case 8: launch_pdl(k_head<T, 8>, dim3(n_jobs), dim3(256), 0, st, g); break;
+    case 10: launch_pdl(k_head<T, 10>, dim3(n_jobs), dim3(256), 0, st, g); break;
+    case 16: launch_pdl(k_head<T, 16>, dim3(n_jobs), dim3(256), 0, st, g); break;
+    default: launch_pdl(k_head<T, kMaxDout>, dim3(n_jobs), dim3(256), 0, st, g); break;
+  }
 }
 
 void launch_head_reduce(cudaStream_t st, const HeadReduceArgs& g, int m, int max_elems) {
@@ -652,11 +810,15 @@ void launch_refresh_wq(cudaStream_t st, const float* p, __nv_bfloat16* wq0, __nv
 template <typename T>
 void launch_predict_head(cudaStream_t st, const PredictHeadArgs<T>& g, int n_jobs) {
   if (n_jobs <= 0) return;
-  if (g.d_out == 1) k_predict_head<T, 1><<<n_jobs, 256, 0, st>>>(g);
-  else if (g.d_out <= 4) k_predict_head<T, 4><<<n_jobs, 256, 0, st>>>(g);
-  else if (g.d_out <= 10) k_predict_head<T, 10><<<n_jobs, 256, 0, st>>>(g);
-  else if (g.d_out <= 16) k_predict_head<T, 16><<<n_jobs, 256, 0, st>>>(g);
-  else k_predict_head<T, kMaxDout><<<n_jobs, 256, 0, st>>>(g);
+  switch (head_bucket(g.d_out)) {
+    case 1: k_predict_head<T, 1><<<n_jobs, 256, 0, st>>>(g); break;
+    case 2: k_predict_head<T, 2><<<n_jobs, 256, 0, st>>>(g); break;
+    case 4: k_predict_head<T, 4><<<n_jobs, 256, 0, st>>>(g); break;
+    case 8: k_predict_head<T, 8><<<n_jobs, 256, 0, st>>>(g); break;
+    case 10: k_predict_head<T, 10><<<n_jobs, 256, 0, st>>>(g); break;
+    case 16: k_predict_head<T, 16><<<n_jobs, 256, 0, st>>>(g); break;
+    default: k_predict_head<T, kMaxDout><<<n_jobs, 256, 0, st>>>(g); break;
+  }
 }
 
 void launch_debug_masks(cudaStream_t st, uint8_t* out, int B, int w, uint64_t seed, uint32_t member,

@@ -347,11 +347,12 @@ tp_status build_schedule(tabpack* h) {
       j.member = i;
       j.blk = b;
       j.h_ld = ldh_of(h, i);
+      j.split = head_split(h->width[i], h->cfg.d_out);
       j.h_off = h->act_off[i][L - 1];
       j.dz_off = h->dz_off[i][L - 1];
       j.w_off = h->W_off[i][L];
       j.b_off = h->b_off[i][L];
-      j.part_off = h->part_off[i] + b * h->part_stride[i];
+      j.part_off = h->part_off[i] + (int64_t)b * h->part_stride[i];
       hj.push_back(j);
     }
   }
@@ -791,6 +792,7 @@ tp_status build_predict(tabpack* h, int P_need) {
       j.member = i;
       j.blk = b;
       j.h_ld = ldh_of(h, i);
+      j.split = 1;
       j.h_off = h->p_act_off[i][L - 1];
       j.w_off = h->W_off[i][L];
       j.b_off = h->b_off[i][L];

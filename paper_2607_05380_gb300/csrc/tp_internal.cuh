@@ -30,7 +30,7 @@ namespace tp {
 constexpr int kMaxDepth = 14;   // hidden blocks per member (4-bit layer field of the Philox counter)
 constexpr int kMaxDout = 32;
 constexpr int kRowTile = 128;   // batch rows per tile; B_pad is a multiple of this
-constexpr int kHeadRows = 32;   // batch rows per head-kernel block
+constexpr int kHeadRows = 64;   // batch rows per head-kernel block
 constexpr int kSegAlign = 32;   // elements
 constexpr int kOnesCols = 16;   // the ones column plus zero padding to 16 columns
 
@@ -80,9 +80,10 @@ struct Chunk {            // element-wise work unit (init, AdamW): never crosses
   int32_t len, seg;
 };
 
-struct HeadJob {          // head forward / loss / backward of one member on one 32-row block
+struct HeadJob {          // head forward / loss / backward of one member on one 64-row block
   int32_t member, blk;
-  int32_t h_ld, _pad;     // pitch of H_L
+  int32_t h_ld;           // pitch of H_L
+  int32_t split;          // row sets of the gradient pass (head_split)
   int64_t h_off;          // H_L in act
   int64_t dz_off;         // dZ_{L-1} in dz (pitch w)
   int64_t w_off, b_off;   // head weight / bias offsets in params
@@ -204,6 +205,22 @@ inline void launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 }
 
 __host__ __device__ constexpr int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+
+// Head kernels: class-count bucket (the loops over classes are unrolled to
+// it) and columns per thread of the gradient pass for a bucket.
+__host__ __device__ constexpr int head_bucket(int d_out) {
+  return d_out <= 1 ? 1 : d_out <= 2 ? 2 : d_out <= 4 ? 4 : d_out <= 8 ? 8 : d_out <= 10 ? 10 : d_out <= 16 ? 16 : kMaxDout;
+}
+__host__ __device__ constexpr int head_cols(int DO) { return DO <= 2 ? 8 : DO <= 10 ? 4 : DO <= 16 ? 2 : 1; }
+// Row sets of a head block's gradient pass: the block's 256 threads take
+// w / head_cols column groups; narrow heads split the block's rows into up
+// to 8 sets so that more threads work.
+__host__ __device__ constexpr int head_split(int w, int d_out) {
+  const int n_cg = w / head_cols(head_bucket(d_out));
+  int S = 1;
+  while (S < 8 && n_cg * S * 2 <= 256) S *= 2;
+  return S;
+}
 __host__ __device__ constexpr int64_t ceil_div(int64_t x, int64_t a) { return (x + a - 1) / a; }
 
 }  // namespace tp
