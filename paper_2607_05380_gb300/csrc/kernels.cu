@@ -403,7 +403,7 @@ struct HeadLogits {
 //      memory, so that every block writes one partial.
 template <typename T, int DO>
 __global__ void __launch_bounds__(256, 2) k_head(HeadArgs<T> g) {
-  constexpr int R = DO <= 10 ? 4 : 2;
+  constexpr int R = DO <= 4 ? 4 : 2;
   constexpr int G = head_cols(DO);
   constexpr int DOP = DO == 1 ? 1 : (DO + 3) & ~3;  // padded row of dlogits in shared memory
   pdl_trigger();
@@ -428,28 +428,34 @@ __global__ void __launch_bounds__(256, 2) k_head(HeadArgs<T> g) {
     const bool live = hl.grp < hl.groups;
     float acc[R][DO];
     hl.run(H, ldh, Wh, bh, w, d_out, rl0, live, acc);
-    if (live && hl.gl == 0) {
+    // the group's lanes take its R rows in turn (every lane holds the sums)
+    for (int q = hl.gl; live && q < R; q += hl.lpr) {
+      float z[DO];
+#pragma unroll
+      for (int c = 0; c < DO; ++c) z[c] = acc[0][c];
+#pragma unroll
+      for (int qq = 1; qq < R; ++qq)
+        if (q == qq)
+#pragma unroll
+          for (int c = 0; c < DO; ++c) z[c] = acc[qq][c];
       const int32_t* idx = g.dyn ? g.dyn->idx : g.idx;
       const void* yv = g.dyn ? g.dyn->y : g.y;
+      const int r = r0 + rl0 + q;
+      float dl[DO];
+      float loss = 0.f;
 #pragma unroll
-      for (int q = 0; q < R; ++q) {
-        const int r = r0 + rl0 + q;
-        float dl[DO];
-        float loss = 0.f;
+      for (int c = 0; c < DO; ++c) dl[c] = 0.f;
+      if (r < g.B) {
+        const int64_t row = idx ? (int64_t)idx[r] : (int64_t)r;
+        loss = row_loss<DO>(g.task, d_out, z, yv, row, invB, dl);
+        float* lg = g.logits + ((int64_t)jb.member * g.B_cap + r) * d_out;
 #pragma unroll
-        for (int c = 0; c < DO; ++c) dl[c] = 0.f;
-        if (r < g.B) {
-          const int64_t row = idx ? (int64_t)idx[r] : (int64_t)r;
-          loss = row_loss<DO>(g.task, d_out, acc[q], yv, row, invB, dl);
-          float* lg = g.logits + ((int64_t)jb.member * g.B_cap + r) * d_out;
-#pragma unroll
-          for (int c = 0; c < DO; ++c)
-            if (c < d_out) lg[c] = acc[q][c];
-        }
-#pragma unroll
-        for (int c = 0; c < DOP; ++c) dlog[rl0 + q][c] = c < DO ? dl[c < DO ? c : 0] : 0.f;
-        lrow[rl0 + q] = loss;
+        for (int c = 0; c < DO; ++c)
+          if (c < d_out) lg[c] = z[c];
       }
+#pragma unroll
+      for (int c = 0; c < DOP; ++c) dlog[rl0 + q][c] = c < DO ? dl[c < DO ? c : 0] : 0.f;
+      lrow[rl0 + q] = loss;
     }
   }
   __syncthreads();
@@ -476,7 +482,7 @@ __global__ void __launch_bounds__(256, 2) k_head(HeadArgs<T> g) {
     const int rb = set * rows_per_set;
     // rows in batches of U (rows_per_set is a multiple of 8): the batch's
     // loads are all issued before its products
-    constexpr int U = 8;
+    constexpr int U = G * DO >= 32 ? 4 : 8;
     for (int rb0 = rb; rb0 < rb + rows_per_set; rb0 += U) {
       RawG<T, G> raw[U];
 #pragma unroll
@@ -719,25 +725,33 @@ __global__ void __launch_bounds__(256) k_predict_head(PredictHeadArgs<T> g) {
     const bool live = hl.grp < hl.groups && r0 + rl0 < g.rows;
     float acc[R][DO];
     hl.run(H, ldh, Wh, bh, w, d_out, rl0, live, acc);
-    if (!live || hl.gl != 0) continue;
-#pragma unroll
-    for (int q = 0; q < R; ++q) {
+    if (!live) continue;
+    // the group's lanes write its R rows in turn
+    for (int q = hl.gl; q < R; q += hl.lpr) {
       const int r = r0 + rl0 + q;
       if (r >= g.rows) break;
+      float z[DO];
+#pragma unroll
+      for (int c = 0; c < DO; ++c) z[c] = acc[0][c];
+#pragma unroll
+      for (int qq = 1; qq < R; ++qq)
+        if (q == qq)
+#pragma unroll
+          for (int c = 0; c < DO; ++c) z[c] = acc[qq][c];
       float* o = g.out + ((int64_t)jb.member * g.N + g.n0 + r) * d_out;
       if (g.task == 1) {
-        float mx = acc[q][0];
+        float mx = z[0];
 #pragma unroll
-        for (int c = 1; c < DO; ++c) if (c < d_out) mx = fmaxf(mx, acc[q][c]);
+        for (int c = 1; c < DO; ++c) if (c < d_out) mx = fmaxf(mx, z[c]);
         float sum = 0.f;
 #pragma unroll
-        for (int c = 0; c < DO; ++c) if (c < d_out) sum += expf(acc[q][c] - mx);
+        for (int c = 0; c < DO; ++c) if (c < d_out) sum += expf(z[c] - mx);
         const float inv = 1.f / sum;
 #pragma unroll
         for (int c = 0; c < DO; ++c)
-          if (c < d_out) o[c] = expf(acc[q][c] - mx) * inv;
+          if (c < d_out) o[c] = expf(z[c] - mx) * inv;
       } else {
-        o[0] = g.task == 0 ? 1.f / (1.f + expf(-acc[q][0])) : acc[q][0];
+        o[0] = g.task == 0 ? 1.f / (1.f + expf(-z[0])) : z[0];
       }
     }
   }
