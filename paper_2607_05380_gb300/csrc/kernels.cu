@@ -1,6 +1,7 @@
 // kernels.cu -- element-wise, reduction and CUDA-core matrix kernels of the
 // packed training step (gather, CUDA-core grouped GEMM, head + loss + head
 // AdamW, AdamW, init, predict head, mask dump).
+#include <algorithm>
 #include <type_traits>
 
 #include "kernels.cuh"
@@ -607,11 +608,17 @@ __global__ void k_head_reduce(HeadReduceArgs g) {
 }
 
 // ------------------------------------------------------------------ AdamW
-// Stand-alone AdamW over chunks of the arena (fp32 mode), with the member's
-// lr and wd and its step's bias corrections; float4 body, scalar tail.
-__global__ void __launch_bounds__(256) k_adamw(AdamArgs g) {
+// Stand-alone AdamW over chunks of the arena (unless AdamW is fused into the
+// weight-gradient epilogue), with the member's lr and wd and its step's bias
+// corrections; float4 body, scalar tail.  In bf16 mode the same threads
+// first fill the dropout mask arena for the next step.
+// Six blocks per SM: the register budget of the mask work must not cost the
+// pass its memory-level parallelism.
+__global__ void __launch_bounds__(256, 6) k_adamw(AdamArgs g) {
   pdl_trigger();
   pdl_wait();
+  // the next step's dropout masks: ALU work beside this pass's HBM streaming
+  fill_masks(g.mg, (int64_t)blockIdx.x * blockDim.x + threadIdx.x, (int64_t)gridDim.x * blockDim.x);
   const Chunk ch = g.chunks[blockIdx.x];
   const Segment s = g.segs[ch.seg];
   const MemberDev md = g.mem[s.member];
@@ -815,6 +822,18 @@ void launch_adamw(cudaStream_t st, const AdamArgs& g, int n_chunks) {
 
 void launch_init(cudaStream_t st, const InitArgs& g, int n_chunks) {
   if (n_chunks > 0) k_init<<<n_chunks, 256, 0, st>>>(g);
+}
+
+__global__ void __launch_bounds__(256) k_masks(MaskGen mg) {
+  pdl_trigger();
+  pdl_wait();
+  fill_masks(mg, (int64_t)blockIdx.x * blockDim.x + threadIdx.x, (int64_t)gridDim.x * blockDim.x);
+}
+
+void launch_masks(cudaStream_t st, const MaskGen& mg) {
+  const int64_t total = (int64_t)mg.n_chunks * mg.rows;
+  if (total <= 0) return;
+  launch_pdl(k_masks, dim3((unsigned)std::min<int64_t>(ceil_div(total, 256), 152 * 8)), dim3(256), 0, st, mg);
 }
 
 void launch_refresh_wq(cudaStream_t st, const float* p, __nv_bfloat16* wq0, __nv_bfloat16* wq1, int64_t n) {

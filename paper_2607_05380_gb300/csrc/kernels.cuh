@@ -68,6 +68,7 @@ struct AdamArgs {
   __nv_bfloat16* wq;      // NULL in fp32 mode
   float beta1, beta2, eps;
   int32_t wd_on_bias;
+  MaskGen mg;             // the next step's dropout masks, filled by the same threads
 };
 
 struct InitArgs {
@@ -107,6 +108,7 @@ void launch_head(cudaStream_t st, const HeadArgs<T>& g, int n_jobs);
 void launch_head_reduce(cudaStream_t st, const HeadReduceArgs& g, int m, int max_elems);
 void launch_adamw(cudaStream_t st, const AdamArgs& g, int n_chunks);
 void launch_init(cudaStream_t st, const InitArgs& g, int n_chunks);
+void launch_masks(cudaStream_t st, const MaskGen& mg);
 void launch_refresh_wq(cudaStream_t st, const float* p, __nv_bfloat16* wq0, __nv_bfloat16* wq1, int64_t n);
 template <typename T>
 void launch_fill_ones(cudaStream_t st, const OnesJob* jobs, int n_jobs, T* xb, T* act);

@@ -81,6 +81,19 @@ struct tabpack {
   int n_p_head = 0;
   bool p_stale = true;      // active set changed since the prediction plan was built
 
+  // Dropout keep words of one step (bf16 mode): per (member, layer) with
+  // p > 0, [ceil(w / 32), B_cap] words from mask_off[i][l] (-1: none).  The
+  // AdamW pass of a training step fills them for step + 1; masks_for is the
+  // step they hold (-1: none), and a step whose masks are not there runs
+  // k_masks first.
+  std::vector<std::array<int64_t, kMaxDepth>> mask_off;
+  int64_t mask_words = 0;
+  uint32_t* masks = nullptr;
+  MaskSeg* mseg_dev = nullptr;
+  int32_t* mchunk_dev = nullptr;
+  int n_mchunks = 0;
+  int64_t masks_for = -1;
+
   // schedule (active members)
   int n_active = 0, n_chunks = 0, n_head_jobs = 0;
   std::vector<std::pair<int, int>> fwd_rng, bwd_rng;  // CUDA-core tile ranges per depth index
@@ -255,6 +268,16 @@ tp_status build_layout(tabpack* h) {
     hoff += h->part_stride[i] * h->n_blk_cap;
   }
   h->n_params = round_up(off, kSegAlign);
+  h->mask_off.assign(m, {});
+  h->mask_words = 0;
+  for (int i = 0; i < m; ++i)
+    for (int l = 0; l < kMaxDepth; ++l) {
+      h->mask_off[i][l] = -1;
+      if (!h->bf16 || l >= h->depth[i] || h->mem[i].drop_T == 0) continue;
+      h->mask_off[i][l] = h->mask_words;
+      h->mask_words += ceil_div(h->width[i], 32) * (int64_t)h->B_cap;
+    }
+  if (h->mask_words >= (int64_t)1 << 31) return fail(h, TP_EINVAL, "dropout mask arena too large");
   h->act_elems = std::max<int64_t>(aoff, 128);
   h->dz_elems = std::max<int64_t>(zoff, 128);
   h->xb_elems = (int64_t)h->B_cap * h->ldx;
@@ -391,6 +414,25 @@ tp_status build_schedule(tabpack* h) {
   if (!ch.empty()) TP_CUDA(h, cudaMemcpy(h->chunks_dev, ch.data(), sizeof(Chunk) * ch.size(), cudaMemcpyHostToDevice));
   if (!ids.empty()) TP_CUDA(h, cudaMemcpy(h->active_ids_dev, ids.data(), sizeof(int32_t) * ids.size(), cudaMemcpyHostToDevice));
   TP_CUDA(h, cudaMemcpy(h->active_dev, h->active.data(), m, cudaMemcpyHostToDevice));
+  // dropout mask segments of the active members
+  h->n_mchunks = 0;
+  h->masks_for = -1;
+  if (h->mask_words > 0) {
+    std::vector<MaskSeg> ms;
+    std::vector<int32_t> mc;
+    for (int i : ids)
+      for (int l = 0; l < h->depth[i]; ++l) {
+        if (h->mask_off[i][l] < 0) continue;
+        const int nck = (int)ceil_div(h->width[i], 32);
+        ms.push_back(MaskSeg{h->mask_off[i][l], i, l, h->mem[i].drop_T, (int32_t)mc.size()});
+        for (int k = 0; k < nck; ++k) mc.push_back((int32_t)ms.size() - 1);
+      }
+    if (!ms.empty()) {
+      TP_CUDA(h, cudaMemcpy(h->mseg_dev, ms.data(), sizeof(MaskSeg) * ms.size(), cudaMemcpyHostToDevice));
+      TP_CUDA(h, cudaMemcpy(h->mchunk_dev, mc.data(), sizeof(int32_t) * mc.size(), cudaMemcpyHostToDevice));
+    }
+    h->n_mchunks = (int)mc.size();
+  }
   h->n_head_jobs = (int)hj.size();
   h->n_chunks = (int)ch.size();
   h->p_stale = true;
@@ -412,6 +454,7 @@ tp_status build_schedule(tabpack* h) {
     lay.xb = h->xb;
     lay.act = h->act;
     lay.dz = h->dz;
+    lay.mask_off = h->mask_words > 0 ? &h->mask_off : nullptr;
     TP_TRY(tc_build_plan(h->tc, lay, h->err));
   }
   return TP_OK;
@@ -464,6 +507,14 @@ tp_status alloc_all(tabpack* h) {
   TP_TRY(dalloc(h, &h->segs_dev, sizeof(Segment) * h->segs.size()));
   TP_TRY(dalloc(h, &h->part_stride_dev, sizeof(int64_t) * m));
   TP_TRY(dalloc(h, &h->dyn_dev, sizeof(StepDyn)));
+  if (h->mask_words > 0) {
+    int64_t n_mc = 0;
+    for (int i = 0; i < m; ++i)
+      if (h->mask_off[i][0] >= 0) n_mc += h->depth[i] * ceil_div(h->width[i], 32);
+    TP_TRY(dalloc(h, &h->masks, sizeof(uint32_t) * h->mask_words));
+    TP_TRY(dalloc(h, &h->mseg_dev, sizeof(MaskSeg) * (size_t)m * kMaxDepth));
+    TP_TRY(dalloc(h, &h->mchunk_dev, sizeof(int32_t) * n_mc));
+  }
   TP_CUDA(h, cudaHostAlloc((void**)&h->dyn_host, sizeof(StepDyn) * tabpack::kRing, cudaHostAllocDefault));
   for (int k = 0; k < tabpack::kRing; ++k) TP_CUDA(h, cudaEventCreateWithFlags(&h->dyn_ev[k], cudaEventDisableTiming));
   TP_CUDA(h, cudaStreamCreateWithFlags(&h->st_cap, cudaStreamNonBlocking));
@@ -553,7 +604,7 @@ tp_status run_forward(tabpack* h, int B, int B_pad, uint32_t step, const StepDyn
   if (h->bf16) {  // every layer in one launch
     int slot;
     prof_begin(h, train ? TP_PH_FWD : TP_PH_PREDICT, &slot);
-    TP_TRY(tc_run_fwd(h->tc, h->st, B, B_pad, h->wcur, step, dyn, train, h->cfg.seed, h->params, h->mem_dev, h->act,
+    TP_TRY(tc_run_fwd(h->tc, h->st, B, B_pad, h->wcur, train, h->masks, h->B_cap, h->params, h->mem_dev, h->act,
                       h->err));
     TP_LAUNCHED(h);
     h->launches++;
@@ -571,6 +622,21 @@ tp_status run_forward(tabpack* h, int B, int B_pad, uint32_t step, const StepDyn
     prof_end(h, slot, 1, train ? TP_PH_FWD : TP_PH_PREDICT);
   }
   return TP_OK;
+}
+
+// Filling the mask arena for a step (dyn non-NULL: dyn->step + step_add).
+MaskGen mask_gen(tabpack* h, uint32_t step, const StepDyn* dyn, uint32_t step_add) {
+  MaskGen mg{};
+  mg.masks = h->masks;
+  mg.segs = h->mseg_dev;
+  mg.chunk_seg = h->mchunk_dev;
+  mg.n_chunks = h->bf16 ? h->n_mchunks : 0;
+  mg.rows = h->B_cap;
+  mg.seed = h->cfg.seed;
+  mg.step = step;
+  mg.step_add = step_add;
+  mg.dyn = dyn;
+  return mg;
 }
 
 // One step on the pack's stream (enqueue only; the caller flips the weight
@@ -676,6 +742,7 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
     ag.beta2 = h->cfg.beta2;
     ag.eps = h->cfg.eps;
     ag.wd_on_bias = h->cfg.wd_on_bias;
+    ag.mg = mask_gen(h, step + 1u, dyn, 1u);  // the next step's dropout masks
     launch_adamw(h->st, ag, h->n_chunks);
     TP_LAUNCHED(h);
     h->launches++;
@@ -691,6 +758,14 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
 template <typename T>
 tp_status step_entry(tabpack* h, const float* X, int64_t n_rows, const int32_t* idx, const void* y, int B,
                      uint32_t step, float* loss_out, bool update) {
+  // the forward reads the step's dropout masks from the arena: fill it now
+  // unless the previous step's AdamW pass did
+  const bool masks_next = update && h->bf16 && !h->fuse_adamw && h->n_chunks > 0;
+  if (h->bf16 && h->n_mchunks > 0 && h->masks_for != (int64_t)step) {
+    launch_masks(h->st, mask_gen(h, step, nullptr, 0));
+    TP_LAUNCHED(h);
+    h->launches++;
+  }
   if (!h->use_graphs || h->profiling) {
     TP_TRY(run_step<T>(h, X, n_rows, idx, y, B, step, loss_out, update, nullptr));
   } else {
@@ -733,6 +808,7 @@ tp_status step_entry(tabpack* h, const float* X, int64_t n_rows, const int32_t* 
     h->launches += ge->n_launch;
   }
   if (update && h->bf16) h->wcur ^= 1;
+  h->masks_for = masks_next ? (int64_t)(uint32_t)(step + 1u) : (int64_t)step;
   h->last_B = B;
   return TP_OK;
 }
@@ -817,8 +893,7 @@ tp_status run_predict_tc(tabpack* h, const float* X, int64_t N, float* out) {
                                  h->ldx, (__nv_bfloat16*)h->p_xb, 0, h->t_dev, h->bias_corr, h->active_ids_dev, 0,
                                  h->cfg.beta1, h->cfg.beta2, h->tcp.cnt_dev, h->tcp.n_cnt);
     TP_LAUNCHED(h);
-    TP_TRY(tc_run_fwd(h->tcp, h->st, rows, B_pad, h->wcur, 0u, nullptr, 0, h->cfg.seed, h->params, h->mem_dev, h->p_act,
-                      h->err));
+    TP_TRY(tc_run_fwd(h->tcp, h->st, rows, B_pad, h->wcur, 0, nullptr, 0, h->params, h->mem_dev, h->p_act, h->err));
     TP_LAUNCHED(h);
     PredictHeadArgs<__nv_bfloat16> pg;
     pg.jobs = h->p_head_dev;

@@ -103,11 +103,11 @@ struct TcArgs {
   const TcTile* tiles;
   int32_t n_tiles;
   int32_t B, B_pad;
-  uint32_t step;
   int32_t train;
+  int32_t mask_rows;  // rows of a chunk of keep words in the mask arena
   int32_t w_shift;  // added to the weight-map index of kFwd / kDgrad tiles (weight copy)
   int32_t update;   // kWgrad: 1 = fused AdamW, 0 = store gradients
-  uint64_t seed;
+  const uint32_t* masks;  // dropout keep words of the step (train)
   const CUtensorMap* maps;
   const float* params;
   const MemberDev* mem;
@@ -116,7 +116,6 @@ struct TcArgs {
   float* grads;
   AdamDev adam;
   int* err;
-  const StepDyn* dyn;  // non-NULL: the dropout step counter is read from here
   int* cnt;            // row-block completion counters
   int32_t kmaj_off;    // index distance to the same matrix's map with 128-row boxes (K-major loads)
 };
@@ -562,7 +561,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
     const int q = warp & 3;             // TMEM lane quarter this warp may access
     const int half = (warp - 2) >> 2;   // 0 for warps 2-5, 1 for warps 6-9
     const int row = 32 * q + lane;
-    const uint32_t step = g.dyn ? g.dyn->step : g.step;
     uint32_t acc = 0, acc_phase = 0;
     // Fused AdamW: the parameter rows of the CTA's next weight-gradient tile
     // stream into L2 while this tile's products run and its epilogue works.
@@ -603,15 +601,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         if (c >= n_end || ncols <= 0) continue;
         if (tile.kind == kFwd) {
           if (lane < ncols) bias_l[ci] = __ldg(g.params + tile.aux_off + col0 + lane);
-          if (row_ok && g.train && md.drop_T) {
-            uint32_t keep = 0;
-#pragma unroll
-            for (int g4 = 0; g4 < 8; ++g4)
-              keep |= keep_bits4(g.seed, (uint32_t)tile.member, (uint32_t)tile.layer, step, (uint32_t)r,
-                                 (uint32_t)((col0 >> 2) + g4), md.drop_T)
-                      << (4 * g4);
-            bits[ci] = keep;
-          }
+          // tile origins and chunks are 32-column aligned for forward tiles
+          if (row_ok && g.train && tile.mask_off >= 0)
+            bits[ci] = __ldg(g.masks + tile.mask_off + (int64_t)(col0 >> 5) * g.mask_rows + r);
         } else if (tile.kind == kDgrad && row_ok) {
           const __nv_bfloat16* hm = g.act + tile.aux_off + (int64_t)r * tile.ld_aux + col0;
           uint32_t mb = 0;
@@ -847,11 +839,12 @@ bool encode_map(CUtensorMap* m, const void* base, int64_t cols, int64_t rows, in
   return true;
 }
 
-// Balanced split of n columns into tiles of at most 256 (multiples of 16).
-void split_n(int n, std::vector<std::pair<int, int>>& out) {
+// Balanced split of n columns into tiles of at most 256 (multiples of 16),
+// every tile starting at a multiple of `align` (16 or 32).
+void split_n(int n, std::vector<std::pair<int, int>>& out, int align = 16) {
   out.clear();
   const int nt = (int)ceil_div(n, 256);
-  const int len = (int)round_up(ceil_div(n, nt), 16);
+  const int len = (int)round_up(ceil_div(n, nt), align);
   for (int n0 = 0; n0 < n; n0 += len) out.push_back({n0, std::min(len, (int)round_up(n - n0, 16))});
 }
 
@@ -1022,9 +1015,10 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
     for (int i = 0; i < m; ++i) {
       if (!active[i] || depth[i] <= l) continue;
       const int w = width[i];
-      split_n(w, ns);
+      split_n(w, ns, 32);  // 32-column aligned: one keep word per chunk of the epilogue
       TcTile t{};
       t.kind = kFwd; t.member = i; t.layer = l;
+      t.mask_off = lay.mask_off ? (int32_t)(*lay.mask_off)[i][l] : -1;
       t.m_real = 0; t.n_real = w;
       t.k_len = l == 0 ? lay.d_in_pad : w;
       t.map_a = l == 0 ? 0 : plan.map_act[(size_t)i * kMaxDepth + l - 1];
@@ -1057,6 +1051,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
       if (l > 0) {
         TcTile t{};
         t.kind = kDgrad; t.member = i; t.layer = l;
+        t.mask_off = -1;
         t.m_real = 0; t.n_real = w;
         t.k_len = w;
         t.map_a = plan.map_dz[(size_t)i * kMaxDepth + l];
@@ -1075,6 +1070,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
       split_n(in_pad + 1, nw);  // weight columns plus the bias column
       TcTile t{};
       t.kind = kWgrad; t.member = i; t.layer = l;
+      t.mask_off = -1;
       t.m_real = w; t.n_real = in_pad + 1;
       t.k_len = 0;
       t.map_a = plan.map_dz[(size_t)i * kMaxDepth + l];
@@ -1174,18 +1170,16 @@ static tp_status launch(TcPlan& plan, cudaStream_t st, const std::pair<int, int>
   return TP_OK;
 }
 
-tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, uint32_t step, const StepDyn* dyn,
-                     int train, uint64_t seed, const float* params, const MemberDev* mem, void* act,
-                     std::string& err) {
+tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, int train, const uint32_t* masks,
+                     int mask_rows, const float* params, const MemberDev* mem, void* act, std::string& err) {
   TcArgs a{};
   a.B = B;
   a.B_pad = B_pad;
-  a.step = step;
-  a.dyn = dyn;
   a.train = train;
+  a.masks = masks;
+  a.mask_rows = mask_rows;
   a.w_shift = wcur ? plan.w_shift : 0;
   a.update = 0;
-  a.seed = seed;
   a.params = params;
   a.mem = mem;
   a.act = (__nv_bfloat16*)act;

@@ -33,7 +33,9 @@ struct TcTile {
   // (dep_n = 1: d = dep + mi, n = 1; dep_n = 0: d = dep, n = the step's
   // B_pad / 128); after storing its output every epilogue warp adds 1 to
   // counter sig + mi.  -1: none.
-  int32_t dep, dep_n, dep_need, sig, _pad;
+  int32_t dep, dep_n, dep_need, sig;
+  int32_t mask_off;        // kFwd of a member with dropout: word offset of its keep words in the
+                           // mask arena ([ceil(n_real / 32), mask rows]); -1: none
   int64_t c_off;           // output: act (kFwd), dz (kDgrad), weight offset in the arena (kWgrad)
   int64_t aux_off;         // kFwd: bias offset in params; kDgrad: H_l offset in act (mask);
                            // kWgrad: bias offset in the arena
@@ -74,15 +76,16 @@ struct TcLayout {          // what the plan needs to know about the pack's arena
   const void* act;
   const void* dz;
   bool fwd_only = false;   // forward tiles only (prediction): no dz maps, counters or backward tiles
+  // per (member, layer): word offset of the dropout keep words, -1 for none (NULL: no masks)
+  const std::vector<std::array<int64_t, kMaxDepth>>* mask_off = nullptr;
 };
 
 tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err);
 // Forward products of every hidden layer of every active member (one
-// launch), reading weight copy `wcur`.  The dropout step counter is `step`,
-// or dyn->step when dyn is non-NULL.
-tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, uint32_t step, const StepDyn* dyn,
-                     int train, uint64_t seed, const float* params, const MemberDev* mem, void* act,
-                     std::string& err);
+// launch), reading weight copy `wcur`.  train = 1: dropout with the keep
+// words of the step in `masks` (rows = mask_rows per 32-column chunk).
+tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, int train, const uint32_t* masks,
+                     int mask_rows, const float* params, const MemberDev* mem, void* act, std::string& err);
 // Backward products (dgrad + wgrad) of every hidden layer (one launch).
 // update = 0: the weight and bias gradients are stored in `grads`;
 // update = 1: AdamW is applied in the epilogue (adam.wq_out = the other

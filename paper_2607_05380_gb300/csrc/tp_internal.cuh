@@ -167,6 +167,55 @@ __device__ __forceinline__ uint32_t keep_bits4(uint64_t seed, uint32_t member, u
          ((uint32_t)(r.w >= T) << 3);
 }
 
+// Dropout keep bits of 32 consecutive columns of one row, word bit j =
+// keep(32 * chunk + j): the eight Philox draws of the chunk.
+__device__ __forceinline__ uint32_t keep_word(uint64_t seed, uint32_t member, uint32_t layer, uint32_t step,
+                                              uint32_t row, uint32_t chunk, uint32_t T) {
+  uint32_t keep = 0;
+#pragma unroll
+  for (int g4 = 0; g4 < 8; ++g4) keep |= keep_bits4(seed, member, layer, step, row, 8 * chunk + g4, T) << (4 * g4);
+  return keep;
+}
+
+// Precomputed dropout masks (bf16 mode).  Each (member, layer) with p > 0
+// owns [ceil(w / 32), B_cap] keep words of one step in the mask arena; the
+// forward epilogue reads its row's word of each 32-column chunk instead of
+// evaluating Philox.  The chunks of all such (member, layer) pairs are
+// numbered in one flat list for the kernels that fill the arena.
+struct MaskSeg {
+  int64_t off;            // word offset in the mask arena
+  int32_t member, layer;
+  uint32_t drop_T;
+  int32_t chunk0;         // its first chunk in the flat list
+};
+
+struct MaskGen {          // what a kernel needs to fill the mask arena for one step
+  uint32_t* masks;
+  const MaskSeg* segs;
+  const int32_t* chunk_seg;  // flat chunk -> segment
+  int32_t n_chunks;          // 0: nothing to fill
+  int32_t rows;              // B_cap
+  uint64_t seed;
+  uint32_t step;             // the step (dyn == NULL)
+  uint32_t step_add;         // dyn != NULL: the step is dyn->step + step_add
+  const StepDyn* dyn;
+};
+
+// Fill the mask arena (threads tid of nthreads; consecutive threads take
+// consecutive rows of a chunk, so the stores coalesce).
+__device__ __forceinline__ void fill_masks(const MaskGen& mg, int64_t tid, int64_t nthreads) {
+  if (mg.n_chunks == 0) return;
+  const uint32_t step = mg.dyn ? mg.dyn->step + mg.step_add : mg.step;
+  const int64_t total = (int64_t)mg.n_chunks * mg.rows;
+  for (int64_t e = tid; e < total; e += nthreads) {
+    const int gc = (int)(e / mg.rows), row = (int)(e - (int64_t)gc * mg.rows);
+    const MaskSeg s = mg.segs[mg.chunk_seg[gc]];
+    const int chunk = gc - s.chunk0;
+    mg.masks[s.off + (int64_t)chunk * mg.rows + row] =
+        keep_word(mg.seed, (uint32_t)s.member, (uint32_t)s.layer, step, (uint32_t)row, (uint32_t)chunk, s.drop_T);
+  }
+}
+
 // ---------------------------------------------------------------- element types
 template <typename T> struct Elem;
 template <> struct Elem<float> {
