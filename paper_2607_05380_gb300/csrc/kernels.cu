@@ -612,9 +612,7 @@ __global__ void k_head_reduce(HeadReduceArgs g) {
 // weight-gradient epilogue), with the member's lr and wd and its step's bias
 // corrections; float4 body, scalar tail.  In bf16 mode the same threads
 // first fill the dropout mask arena for the next step.
-// Six blocks per SM: the register budget of the mask work must not cost the
-// pass its memory-level parallelism.
-__global__ void __launch_bounds__(256, 6) k_adamw(AdamArgs g) {
+__global__ void __launch_bounds__(256) k_adamw(AdamArgs g) {
   pdl_trigger();
   pdl_wait();
   // the next step's dropout masks: ALU work beside this pass's HBM streaming

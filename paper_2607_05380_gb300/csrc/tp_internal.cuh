@@ -168,11 +168,13 @@ __device__ __forceinline__ uint32_t keep_bits4(uint64_t seed, uint32_t member, u
 }
 
 // Dropout keep bits of 32 consecutive columns of one row, word bit j =
-// keep(32 * chunk + j): the eight Philox draws of the chunk.
+// keep(32 * chunk + j): the eight Philox draws of the chunk, one after the
+// other (few registers: the kernels that fill the mask arena stream memory
+// beside it).
 __device__ __forceinline__ uint32_t keep_word(uint64_t seed, uint32_t member, uint32_t layer, uint32_t step,
                                               uint32_t row, uint32_t chunk, uint32_t T) {
   uint32_t keep = 0;
-#pragma unroll
+#pragma unroll 1
   for (int g4 = 0; g4 < 8; ++g4) keep |= keep_bits4(seed, member, layer, step, row, 8 * chunk + g4, T) << (4 * g4);
   return keep;
 }
