@@ -72,6 +72,7 @@ def lib():
                 "orc_destroy": (None, [P]),
                 "orc_init_value": (f64, [u64, u32, u32, u32, i32]),
                 "orc_train_step": (ctypes.c_int, [P, P, i64, P, P, P, i32, u32, i32, P]),
+                "orc_train_step_stacked": (ctypes.c_int, [P, P, i64, P, P, P, i32, u32, i32, P]),
                 "orc_predict": (ctypes.c_int, [P, P, i64, P]),
                 "orc_set_active": (ctypes.c_int, [P, P]),
                 "orc_adamw_apply": (None, [P, P, P, P, i64, i64, f64, f64, f64, f64, f64]),
@@ -178,15 +179,23 @@ class OraclePack:
         return n_out, n_in
 
     def train_step(self, X, idx, y, step, update=True):
+        """idx [B] (one batch for every member) or [m, B] (member i's batch in
+        row i, Sec. 3.6 stacked base batches)."""
         X = np.ascontiguousarray(X, dtype=np.float32)
         idx = np.ascontiguousarray(idx, dtype=np.int32)
         yi, yf = _labels(self.task, y)
         loss = np.zeros(self.m, dtype=np.float64)
-        rc = lib().orc_train_step(self._h, _ptr(X), X.shape[0], _ptr(idx), _ptr(yi), _ptr(yf),
-                                  len(idx), int(step), int(bool(update)), _ptr(loss))
+        if idx.ndim == 2:
+            if idx.shape[0] != self.m:
+                raise ValueError("stacked idx must have one row per member")
+            fn, B = lib().orc_train_step_stacked, idx.shape[1]
+        else:
+            fn, B = lib().orc_train_step, len(idx)
+        rc = fn(self._h, _ptr(X), X.shape[0], _ptr(idx), _ptr(yi), _ptr(yf), B, int(step), int(bool(update)),
+                _ptr(loss))
         if rc:
             raise ValueError("oracle train_step rejected its arguments")
-        self._B = len(idx)
+        self._B = B
         return loss
 
     def predict(self, X):

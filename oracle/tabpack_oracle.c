@@ -428,12 +428,20 @@ static void orc_adamw(const orc_pack* h, const orc_member* M, double* p, double*
   orc_adamw_apply(p, m, v, g, n, M->t, (double)M->lr, wd, h->cfg.beta1, h->cfg.beta2, h->cfg.eps);
 }
 
-int orc_train_step(orc_pack* h, const float* X, int64_t N, const int32_t* idx,
-                   const int32_t* y_int, const float* y_float, int32_t B,
-                   uint32_t step, int32_t update, double* loss_out) {
+/* One step of every active member; member i reads its batch rows from
+ * idx + i * idx_stride (idx_stride 0: one batch shared by all members;
+ * idx_stride B: the stacked per-member batches of Sec. 3.6).               */
+static int orc_step(orc_pack* h, const float* X, int64_t N, const int32_t* idx, int64_t idx_stride,
+                    const int32_t* y_int, const float* y_float, int32_t B,
+                    uint32_t step, int32_t update, double* loss_out) {
   if (!h || !X || !idx || B <= 0) return 1;
   if (h->cfg.task == ORC_REGRESSION ? !y_float : !y_int) return 1;
-  for (int b = 0; b < B; ++b) if (idx[b] < 0 || idx[b] >= N) return 1;
+  const int n_rows = idx_stride ? h->cfg.m : 1;
+  for (int i = 0; i < n_rows; ++i)
+    for (int b = 0; b < B; ++b) {
+      const int32_t r = idx[(int64_t)i * idx_stride + b];
+      if (r < 0 || r >= N) return 1;
+    }
   int status = 0;
 #pragma omp parallel for schedule(dynamic, 1)
   for (int i = 0; i < h->cfg.m; ++i) {
@@ -442,9 +450,10 @@ int orc_train_step(orc_pack* h, const float* X, int64_t N, const int32_t* idx,
       if (loss_out) loss_out[i] = NAN;
       continue;
     }
+    const int32_t* idx_i = idx + (int64_t)i * idx_stride;
     orc_alloc_cache(M, B, h->cfg.d_out);
-    orc_member_forward(h, M, X, idx, B, step, 1);
-    double loss = orc_member_backward(h, M, idx, y_int, y_float, B);
+    orc_member_forward(h, M, X, idx_i, B, step, 1);
+    double loss = orc_member_backward(h, M, idx_i, y_int, y_float, B);
     if (loss_out) loss_out[i] = loss;
     if (update) {
       M->t += 1;
@@ -455,6 +464,18 @@ int orc_train_step(orc_pack* h, const float* X, int64_t N, const int32_t* idx,
     }
   }
   return status;
+}
+
+int orc_train_step(orc_pack* h, const float* X, int64_t N, const int32_t* idx,
+                   const int32_t* y_int, const float* y_float, int32_t B,
+                   uint32_t step, int32_t update, double* loss_out) {
+  return orc_step(h, X, N, idx, 0, y_int, y_float, B, step, update, loss_out);
+}
+
+int orc_train_step_stacked(orc_pack* h, const float* X, int64_t N, const int32_t* idx,
+                           const int32_t* y_int, const float* y_float, int32_t B,
+                           uint32_t step, int32_t update, double* loss_out) {
+  return orc_step(h, X, N, idx, B, y_int, y_float, B, step, update, loss_out);
 }
 
 /* Per-member validation predictions (Sec. 3.5 "Online ensemble": the pool is

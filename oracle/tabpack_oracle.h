@@ -92,6 +92,14 @@ int orc_train_step(orc_pack* h, const float* X, int64_t N, const int32_t* idx,
                    const int32_t* y_int, const float* y_float, int32_t B,
                    uint32_t step, int32_t update, double* loss_out);
 
+/* The same step with a batch per member (Sec. 3.6: the base models train on
+ * different batch sequences, one training batch being m base batches of B
+ * rows stacked along the pack dimension): idx is [m, B], member i reads rows
+ * idx[i * B .. i * B + B - 1] (rows of inactive members are still checked). */
+int orc_train_step_stacked(orc_pack* h, const float* X, int64_t N, const int32_t* idx,
+                           const int32_t* y_int, const float* y_float, int32_t B,
+                           uint32_t step, int32_t update, double* loss_out);
+
 /* Forward only, no dropout: out [m, N, d_out] = probabilities (softmax /
  * sigmoid) or regression values.                                               */
 int orc_predict(orc_pack* h, const float* X, int64_t N, double* out);

@@ -220,6 +220,47 @@ def test_packed_equals_solo_members(orc, bf16):
         np.testing.assert_array_equal(Pp[i], solos[i].predict(X[:10])[0])
 
 
+@pytest.mark.parametrize("bf16", [False, True])
+def test_stacked_batches_equal_solo_members_on_their_own_batches(orc, bf16):
+    """Sec. 3.6: each base model trains on its own batch sequence; a stacked
+    step (idx [m, B]) gives member i exactly what training it alone on row i
+    of idx gives (and a shifted or transposed row would not)."""
+    m, d_in, d_out = 4, 7, 3
+    hp = random_pack(m, d_in, d_out, seed=23)
+    X, y = _make_data("multiclass", 80, d_in, d_out, seed=5)
+    packed = orc.OraclePack(d_in, d_out, "multiclass", hp["depth"], hp["width"], hp["dropout"],
+                            hp["lr"], hp["wd"], seed=9, bf16_storage=bf16)
+    solos = [orc.OraclePack(d_in, d_out, "multiclass", hp["depth"][i:i + 1], hp["width"][i:i + 1],
+                            hp["dropout"][i:i + 1], hp["lr"][i:i + 1], hp["wd"][i:i + 1], seed=9,
+                            bf16_storage=bf16, member_id=[i]) for i in range(m)]
+    rng = np.random.default_rng(1)
+    for step in range(3):
+        idx = np.stack([rng.choice(80, 16, replace=False) for _ in range(m)]).astype(np.int32)
+        lp = packed.train_step(X, idx, y, step)
+        for i in range(m):
+            assert lp[i] == solos[i].train_step(X, idx[i], y, step)[0]
+    for i in range(m):
+        for l in range(int(hp["depth"][i]) + 1):
+            np.testing.assert_array_equal(packed.get_params(i, l)[0], solos[i].get_params(0, l)[0])
+            np.testing.assert_array_equal(packed.get_params(i, l)[1], solos[i].get_params(0, l)[1])
+
+
+def test_stacked_batches_with_one_batch_equal_the_shared_step(orc):
+    m, d_in, d_out = 3, 6, 1
+    hp = random_pack(m, d_in, d_out, seed=31)
+    X, y = _make_data("regression", 50, d_in, d_out, seed=6)
+    a = orc.OraclePack(d_in, d_out, "regression", hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"], seed=4)
+    b = orc.OraclePack(d_in, d_out, "regression", hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"], seed=4)
+    rng = np.random.default_rng(2)
+    for step in range(2):
+        idx = rng.choice(50, 12, replace=False).astype(np.int32)
+        np.testing.assert_array_equal(a.train_step(X, idx, y, step), b.train_step(X, np.tile(idx, (m, 1)), y, step))
+    for i in range(m):
+        np.testing.assert_array_equal(a.get_params(i, 0)[0], b.get_params(i, 0)[0])
+    with pytest.raises(ValueError):
+        b.train_step(X, np.zeros((m + 1, 4), dtype=np.int32), y, 3)
+
+
 def _zero_head(pack, i):
     L = int(pack.depth[i])
     W, b = pack.get_params(i, L)
