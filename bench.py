@@ -192,10 +192,11 @@ def time_online_epoch(tp, torch, pack, wl, hp, d, X, y, idx_all, stream, loss, n
                     % -(-wl.n_train // B)}
 
 
-def cpu_baseline(wl, hp, data_np, B, budget_s=20.0):
+def cpu_baseline(wl, hp, data_np, B, budget_s=20.0, stacked=False):
     """The oracle as it stands, on the host cores, on a bounded sample of the
     same workload: the first k members (independent of the others), timed
-    over whole steps until about budget_s seconds of CPU work."""
+    over whole steps until about budget_s seconds of CPU work (stacked: a
+    batch per member)."""
     import oracle
     oracle.build()
     X, y = data_np
@@ -209,7 +210,10 @@ def cpu_baseline(wl, hp, data_np, B, budget_s=20.0):
     steps = 0
     t0 = time.perf_counter()
     while True:
-        idx = rng.choice(X.shape[0], B, replace=False).astype(np.int32)
+        if stacked:
+            idx = np.stack([rng.choice(X.shape[0], B, replace=False) for _ in range(k)]).astype(np.int32)
+        else:
+            idx = rng.choice(X.shape[0], B, replace=False).astype(np.int32)
         pk.train_step(X, idx, y, steps)
         steps += 1
         el = time.perf_counter() - t0
@@ -235,7 +239,7 @@ def run_reference(args, wl, rank):
         pass
     base = None
     for s in range(max(1, args.steps)):
-        base = cpu_baseline(wl, hp, data, B, budget_s=per)
+        base = cpu_baseline(wl, hp, data, B, budget_s=per, stacked=args.stacked)
         vals.append(base["value"])
     value = float(np.mean(vals))
     ms = float(1000.0 * wl.m * B / value)
@@ -263,6 +267,8 @@ def main():
                     help="train only the first N members of the workload (profiling small cases)")
     ap.add_argument("--fuse-optimizer", action="store_true", help="AdamW inside the weight-gradient epilogue")
     ap.add_argument("--no-online", action="store_true", help="skip timing the online-ensemble epoch end")
+    ap.add_argument("--stacked", action="store_true",
+                    help="a batch per member (idx [m, B], Sec. 3.6) instead of one batch shared by all members")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -297,7 +303,10 @@ def main():
     total = args.warmup + args.steps
     gen = torch.Generator(device=dev)
     gen.manual_seed(3)
-    idx_all = torch.stack([torch.randperm(n_train, generator=gen, device=dev)[:B] for _ in range(total)])
+    if args.stacked:   # [steps, m, B]: each member its own rows
+        idx_all = torch.randint(0, n_train, (total, wl.m, B), generator=gen, device=dev)
+    else:
+        idx_all = torch.stack([torch.randperm(n_train, generator=gen, device=dev)[:B] for _ in range(total)])
     idx_all = idx_all.to(torch.int32).contiguous()
 
     stream = torch.cuda.current_stream()
@@ -375,11 +384,15 @@ def main():
         Xh = X.cpu().pin_memory()
         yh = y.cpu().pin_memory()
         idx_h = idx_all.cpu()
-        xb_h = [Xh[idx_h[s].long()].pin_memory() for s in range(min(total, 64))]
-        yb_h = [yh[idx_h[s].long()].pin_memory() for s in range(min(total, 64))]
-        ident = torch.arange(B, dtype=torch.int32, device=dev)
-        xb_d = torch.empty(B, wl.d_in, dtype=torch.float32, device=dev)
-        yb_d = torch.empty(B, dtype=y.dtype, device=dev)
+        # per step the rows the step reads (stacked: m batches of B rows)
+        xb_h = [Xh[idx_h[s].reshape(-1).long()].pin_memory() for s in range(min(total, 64))]
+        yb_h = [yh[idx_h[s].reshape(-1).long()].pin_memory() for s in range(min(total, 64))]
+        n_rows_step = xb_h[0].shape[0]
+        ident = torch.arange(n_rows_step, dtype=torch.int32, device=dev)
+        if args.stacked:
+            ident = ident.view(wl.m, B)
+        xb_d = torch.empty(n_rows_step, wl.d_in, dtype=torch.float32, device=dev)
+        yb_d = torch.empty(n_rows_step, dtype=y.dtype, device=dev)
         loss_h = torch.empty(wl.m, dtype=torch.float32).pin_memory()
         n_e2e = min(args.steps, 64)
         for s in range(3):
@@ -401,7 +414,8 @@ def main():
         wall = time.perf_counter() - t0
         ms_e2e = max(e0.elapsed_time(e1), wall * 1000.0)
         e2e = {"value": world * wl.m * B * n_e2e / (ms_e2e / 1000.0), "unit": UNIT,
-               "h2d_bytes_per_step": B * wl.d_in * 4 + B * 4, "d2h_bytes_per_step": wl.m * 4, "steps": n_e2e}
+               "h2d_bytes_per_step": n_rows_step * (wl.d_in * 4 + 4), "d2h_bytes_per_step": wl.m * 4,
+               "steps": n_e2e}
 
     online = None if args.no_online else time_online_epoch(tp, torch, pack, wl, hp, d, X, y, idx_all, stream, loss)
 
@@ -409,7 +423,7 @@ def main():
     if rank == 0 and not args.no_cpu_baseline:
         n = min(n_train, 20000)
         data_np = (X[:n].cpu().numpy(), y[:n].cpu().numpy())
-        cpu = cpu_baseline(wl, hp, data_np, B, budget_s=20.0)
+        cpu = cpu_baseline(wl, hp, data_np, B, budget_s=20.0, stacked=args.stacked)
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -419,7 +433,8 @@ def main():
                            "params": n_params, "gemm_flop_per_step": flops,
                            "l2": "inputs larger than L2: each step streams ~%.2f GB of parameters and optimizer state"
                                  % (30.0 * n_params / 1e9),
-                           "parallelism": "one independent pack per GPU" if world > 1 else "single GPU"},
+                           "parallelism": "one independent pack per GPU" if world > 1 else "single GPU",
+                           "batches": "one per member (stacked)" if args.stacked else "one shared by all members"},
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches, "online_epoch": online,
                 "clocks": clk.summary(), "final_losses_mean": float(np.nanmean(lossv))}
         print(json.dumps(line), flush=True)

@@ -121,6 +121,21 @@ tp_status pack_train_step(tabpack_t* pack, const float* X, int64_t n_rows, const
 tp_status pack_forward_backward(tabpack_t* pack, const float* X, int64_t n_rows, const int32_t* idx,
                                 const void* y, int32_t B, uint32_t step, float* loss_out);
 
+/* The same steps with a batch per member (Sec. 3.6: the base models are
+ * trained on different batch sequences; one training batch is m base
+ * batches of B rows stacked along the pack dimension).
+ *   idx: device int32 [m, B]: member i's batch is rows idx[i * B .. i * B +
+ *   B - 1] of X (rows of inactive members are not read; no range check on
+ *   the device).  Everything else as pack_train_step / pack_forward_backward;
+ *   dropout masks are the same function of (seed, member, layer, step, row
+ *   position, column).  The first call allocates m gathered-batch matrices
+ *   ([max_batch rounded up to 128, d_in rounded up to 8, plus 16] each, in
+ *   the matrix-product precision) and synchronises.                         */
+tp_status pack_train_step_stacked(tabpack_t* pack, const float* X, int64_t n_rows, const int32_t* idx,
+                                  const void* y, int32_t B, uint32_t step, float* loss_out);
+tp_status pack_forward_backward_stacked(tabpack_t* pack, const float* X, int64_t n_rows, const int32_t* idx,
+                                        const void* y, int32_t B, uint32_t step, float* loss_out);
+
 /* Per-member validation predictions (Sec. 3.5 "Online ensemble"): forward
  * without dropout of every active member on all N rows of X.
  *   X: device float32 [N, d_in];  out: device float32 [m, N, d_out]:

@@ -34,7 +34,7 @@ SYMBOLS = ["pack_create", "pack_destroy", "pack_set_stream", "pack_train_step", 
            "pack_snapshot", "pack_restore", "pack_get_config", "pack_member_hparams", "pack_get_active",
            "pack_get_stream", "pack_online_create", "pack_online_destroy", "pack_online_epoch", "pack_online_info",
            "pack_online_members", "pack_online_ensemble", "pack_online_snapshot", "pack_online_predict",
-           "pack_online_last_error"]
+           "pack_online_last_error", "pack_train_step_stacked", "pack_forward_backward_stacked"]
 
 
 class TabpackError(RuntimeError):
@@ -107,6 +107,8 @@ def load_library(path: str = LIB_PATH):
         "pack_online_snapshot": (st, [P, i32, P]),
         "pack_online_predict": (st, [P, P, i64, P]),
         "pack_online_last_error": (ctypes.c_char_p, [P]),
+        "pack_train_step_stacked": (st, [P, P, i64, P, P, i32, u32, P]),
+        "pack_forward_backward_stacked": (st, [P, P, i64, P, P, i32, u32, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -187,13 +189,22 @@ class Pack:
         return self.torch.float32 if self.task == REGRESSION else self.torch.int32
 
     def train_step(self, X, idx, y, step, loss_out=None, update=True):
-        """X float32 [n, d_in], idx int32 [B], y labels [n] (CUDA tensors);
-        loss_out: optional float32 [m] CUDA tensor."""
-        fn = load_library().pack_train_step if update else load_library().pack_forward_backward
+        """X float32 [n, d_in], idx int32 [B] (one batch for every member) or
+        [m, B] (a batch per member), y labels [n] (CUDA tensors); loss_out:
+        optional float32 [m] CUDA tensor."""
+        L = load_library()
         t = self.torch
+        if idx.dim() == 2:
+            if idx.shape[0] != self.m:
+                raise ValueError("stacked idx must have one row per member")
+            fn = L.pack_train_step_stacked if update else L.pack_forward_backward_stacked
+            B = int(idx.shape[1])
+        else:
+            fn = L.pack_train_step if update else L.pack_forward_backward
+            B = int(idx.shape[0])
         _check(fn(self._h, _dptr(X, t.float32), X.shape[0], _dptr(idx, t.int32), _dptr(y, self._y_dtype()),
-                  int(idx.shape[0]), int(step), _dptr(loss_out, t.float32)), self._h)
-        self._B = int(idx.shape[0])
+                  B, int(step), _dptr(loss_out, t.float32)), self._h)
+        self._B = B
 
     def forward_backward(self, X, idx, y, step, loss_out=None):
         self.train_step(X, idx, y, step, loss_out, update=False)

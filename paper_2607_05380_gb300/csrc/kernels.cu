@@ -9,25 +9,46 @@
 namespace tp {
 
 // ------------------------------------------------------------------ gather
+// Four values at once: 8-byte bf16 / 16-byte fp32 stores.
+__device__ __forceinline__ void store4(__nv_bfloat16* p, float4 v) {
+  uint2 u;
+  __nv_bfloat162* b = reinterpret_cast<__nv_bfloat162*>(&u);
+  b[0] = __floats2bfloat162_rn(v.x, v.y);
+  b[1] = __floats2bfloat162_rn(v.z, v.w);
+  *reinterpret_cast<uint2*>(p) = u;
+}
+__device__ __forceinline__ void store4(float* p, float4 v) { *reinterpret_cast<float4*>(p) = v; }
+
 // xb[b, k] = X[idx[b], k] for b < B, k < d_in; zero for the rest of the first
 // d_in_pad columns of rows < B_pad (column d_in_pad holds the constant 1).
+// Grid: ceil(B_pad / 8) blocks of 8 warps, a row per warp.
 // Block 0 also advances the step count of every active member and stores the
 // AdamW bias corrections 1 - beta^t of the new step (when `advance`); the
 // grid clears `zero[0 .. n_zero)` (the GEMMs' row-block completion counters).
+// stacked != 0 (a batch per member, Sec. 3.6): blockIdx.y is an active
+// member's index, whose rows are idx[member * B ..] and whose batch matrix
+// starts xb_stride elements after the previous member's.
 template <typename T>
 __global__ void k_gather(const float* __restrict__ X, const int32_t* __restrict__ idx, const StepDyn* dyn,
                          int32_t B, int32_t B_pad, int32_t d_in, int32_t d_in_pad, int32_t ldx, T* __restrict__ xb,
                          int32_t advance, int32_t* __restrict__ t_dev, float2* __restrict__ bias_corr,
                          const int32_t* __restrict__ active_ids, int32_t n_active, float beta1,
-                         float beta2, int32_t* __restrict__ zero, int32_t n_zero) {
+                         float beta2, int32_t* __restrict__ zero, int32_t n_zero, int32_t stacked,
+                         int64_t xb_stride) {
   pdl_trigger();
   pdl_wait();
-  for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < n_zero; e += gridDim.x * blockDim.x) zero[e] = 0;
   if (dyn) {
     X = dyn->X;
     idx = dyn->idx;
   }
-  if (advance && blockIdx.x == 0) {
+  if (stacked) {
+    const int member = active_ids[blockIdx.y];
+    if (idx) idx += (int64_t)member * B;
+    xb += (int64_t)member * xb_stride;
+  }
+  if (blockIdx.y == 0)
+    for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < n_zero; e += gridDim.x * blockDim.x) zero[e] = 0;
+  if (advance && blockIdx.x == 0 && blockIdx.y == 0) {
     for (int a = threadIdx.x; a < n_active; a += blockDim.x) {
       int i = active_ids[a];
       int t = t_dev[i] + 1;
@@ -36,17 +57,24 @@ __global__ void k_gather(const float* __restrict__ X, const int32_t* __restrict_
                                  (float)(1.0 - pow((double)beta2, (double)t)));
     }
   }
-  const int64_t total = (int64_t)B_pad * d_in_pad;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
-       e += (int64_t)gridDim.x * blockDim.x) {
-    int b = (int)(e / d_in_pad), k = (int)(e % d_in_pad);
-    float v = 0.f;
-    if (b < B && k < d_in) {
-      int64_t row = idx ? (int64_t)idx[b] : (int64_t)b;
-      v = X[row * d_in + k];
+  // one warp per batch row: float4 reads of the source row when it is
+  // 16-byte aligned, four converted values written at once
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.x * (blockDim.x >> 5) + warp;
+  if (b >= B_pad) return;
+  T* dst = xb + (int64_t)b * ldx;
+  const bool live = b < B;
+  const int64_t row = live ? (idx ? (int64_t)idx[b] : (int64_t)b) : 0;
+  const float* src = X + row * d_in;
+  int k0 = 0;
+  if (live && (d_in & 3) == 0 && ((uintptr_t)src & 15) == 0) {
+    const float4* s4 = reinterpret_cast<const float4*>(src);
+    for (int c = lane; c < (d_in >> 2); c += 32) {
+      store4(dst + 4 * c, __ldg(s4 + c));
     }
-    xb[(int64_t)b * ldx + k] = Elem<T>::from_f(v);
+    k0 = d_in;
   }
+  for (int k = k0 + lane; k < d_in_pad; k += 32) dst[k] = Elem<T>::from_f(live && k < d_in ? src[k] : 0.f);
 }
 
 // Column `col` of the first `rows` rows := 1 (xb and every act matrix, once).
@@ -73,8 +101,10 @@ __global__ void __launch_bounds__(256) k_gemm_simt(GemmArgs<T> g, int32_t tile_b
   if (t.m0 >= M) return;
   const uint32_t step = g.dyn ? g.dyn->step : g.step;
   const T* bases[4] = {g.xb, g.act, g.dz, g.wq};
-  const T* A = bases[P.a_src] + P.a_off;
-  const T* Bm = bases[P.b_src] + P.b_off;
+  // stacked batches: the member's own batch matrix
+  const int64_t xs = (int64_t)P.member * g.xb_stride;
+  const T* A = bases[P.a_src] + P.a_off + (P.a_src == kSrcXb ? xs : 0);
+  const T* Bm = bases[P.b_src] + P.b_off + (P.b_src == kSrcXb ? xs : 0);
   int64_t a_rs, a_ks, b_rs, b_ks;
   if (P.kind == kFwd) {
     a_rs = P.lda; a_ks = 1; b_rs = P.ldb; b_ks = 1;
@@ -447,7 +477,7 @@ __global__ void __launch_bounds__(256, 2) k_head(HeadArgs<T> g) {
 #pragma unroll
       for (int c = 0; c < DO; ++c) dl[c] = 0.f;
       if (r < g.B) {
-        const int64_t row = idx ? (int64_t)idx[r] : (int64_t)r;
+        const int64_t row = idx ? (int64_t)idx[(int64_t)jb.member * g.idx_stride + r] : (int64_t)r;
         loss = row_loss<DO>(g.task, d_out, z, yv, row, invB, dl);
         float* lg = g.logits + ((int64_t)jb.member * g.B_cap + r) * d_out;
 #pragma unroll
@@ -778,12 +808,12 @@ __global__ void k_debug_masks(uint8_t* __restrict__ out, int32_t B, int32_t w, u
 template <typename T>
 void launch_gather(cudaStream_t st, const float* X, const int32_t* idx, const StepDyn* dyn, int B, int B_pad,
                    int d_in, int d_in_pad, int ldx, T* xb, int advance, int32_t* t_dev, float2* bias_corr,
-                   const int32_t* active_ids, int n_active, float beta1, float beta2, int* zero, int n_zero) {
-  int64_t total = (int64_t)B_pad * d_in_pad;
-  int blocks = (int)std::min<int64_t>(ceil_div(total, 256), 152 * 8);
-  if (blocks < 1) blocks = 1;
-  launch_pdl(k_gather<T>, dim3(blocks), dim3(256), 0, st, X, idx, dyn, B, B_pad, d_in, d_in_pad, ldx, xb, advance, t_dev, bias_corr,
-             active_ids, n_active, beta1, beta2, zero, n_zero);
+                   const int32_t* active_ids, int n_active, float beta1, float beta2, int* zero, int n_zero,
+                   int stacked, int64_t xb_stride) {
+  const int blocks = std::max(1, (int)ceil_div(B_pad, 8));  // 8 rows (warps) per block
+  const unsigned gy = stacked ? (unsigned)std::max(n_active, 1) : 1u;
+  launch_pdl(k_gather<T>, dim3(blocks, gy), dim3(256), 0, st, X, idx, dyn, B, B_pad, d_in, d_in_pad, ldx, xb, advance,
+             t_dev, bias_corr, active_ids, n_active, beta1, beta2, zero, n_zero, stacked, xb_stride);
 }
 
 template <typename T>
@@ -860,7 +890,7 @@ void launch_debug_masks(cudaStream_t st, uint8_t* out, int B, int w, uint64_t se
 #define TP_INSTANTIATE(T)                                                                              \
   template void launch_gather<T>(cudaStream_t, const float*, const int32_t*, const StepDyn*, int, int, int, int, \
                                  int, T*, int, int32_t*, float2*, const int32_t*, int, float, float,    \
-                                 int*, int);                                                           \
+                                 int*, int, int, int64_t);                                              \
   template void launch_fill_ones<T>(cudaStream_t, const OnesJob*, int, T*, T*);                         \
   template void launch_gemm_simt<T>(cudaStream_t, const GemmArgs<T>&, int, int);                       \
   template void launch_head<T>(cudaStream_t, const HeadArgs<T>&, int);                                 \

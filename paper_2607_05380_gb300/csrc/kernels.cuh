@@ -23,6 +23,7 @@ struct GemmArgs {
   int32_t train;          // 1: dropout on
   uint64_t seed;
   const StepDyn* dyn;     // non-NULL: take the step from here
+  int64_t xb_stride;      // stacked batches: elements between members' batch matrices (0: shared)
 };
 
 template <typename T>
@@ -39,6 +40,7 @@ struct HeadArgs {
   const void* y;
   int32_t B, B_pad, B_cap, d_out, task, n_blk_cap;
   const StepDyn* dyn;     // non-NULL: take idx and y from here
+  int32_t idx_stride;     // member i's rows are idx[i * idx_stride ..] (0: one shared batch)
 };
 
 struct HeadReduceArgs {
@@ -99,7 +101,7 @@ template <typename T>
 void launch_gather(cudaStream_t st, const float* X, const int32_t* idx, const StepDyn* dyn, int B, int B_pad,
                    int d_in, int d_in_pad, int ldx, T* xb, int advance, int32_t* t_dev, float2* bias_corr,
                    const int32_t* active_ids, int n_active, float beta1, float beta2, int* zero = nullptr,
-                   int n_zero = 0);
+                   int n_zero = 0, int stacked = 0, int64_t xb_stride = 0);
 template <typename T>
 void launch_gemm_simt(cudaStream_t st, const GemmArgs<T>& g, int tile_base, int n_tiles);
 template <typename T>

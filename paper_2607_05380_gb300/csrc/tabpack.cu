@@ -81,6 +81,14 @@ struct tabpack {
   int n_p_head = 0;
   bool p_stale = true;      // active set changed since the prediction plan was built
 
+  // Stacked batches (Sec. 3.6: a batch per member), built on first use:
+  // xbs holds member i's gathered batch at i * xb_elems ([B_cap, ldx] each,
+  // its column d_in_pad = 1), and tcs is the tensor-core plan whose layer-0
+  // tiles read member i's matrix.
+  void* xbs = nullptr;
+  TcPlan tcs;
+  bool s_stale = true;      // active set changed since tcs was built
+
   // Dropout keep words of one step (bf16 mode): per (member, layer) with
   // p > 0, [ceil(w / 32), B_cap] words from mask_off[i][l] (-1: none).  The
   // AdamW pass of a training step fills them for step + 1; masks_for is the
@@ -102,7 +110,7 @@ struct tabpack {
   // CUDA graphs of the training step, one per (B, update, weight copy); the
   // per-call arguments travel through dyn_dev, filled from a pinned ring
   struct GraphEntry {
-    int B, update, wcur;
+    int B, update, wcur, stacked;
     cudaGraphExec_t exec;
     int64_t n_launch;
   };
@@ -436,6 +444,7 @@ tp_status build_schedule(tabpack* h) {
   h->n_head_jobs = (int)hj.size();
   h->n_chunks = (int)ch.size();
   h->p_stale = true;
+  h->s_stale = true;
   if (h->bf16) {
     TcLayout lay;
     lay.depth = &h->depth;
@@ -557,6 +566,9 @@ void free_all(tabpack* h) {
   h->dyn_host = nullptr;
   tc_free_plan(h->tc);
   free_predict(h);
+  tc_free_plan(h->tcs);
+  if (h->xbs) cudaFree(h->xbs);
+  h->xbs = nullptr;
   for (void* p : h->allocs) cudaFree(p);
   h->allocs.clear();
   for (auto e : h->prof.pool) cudaEventDestroy(e);
@@ -564,11 +576,12 @@ void free_all(tabpack* h) {
 }
 
 template <typename T>
-GemmArgs<T> gemm_args(tabpack* h, int B, int B_pad, uint32_t step, int train) {
+GemmArgs<T> gemm_args(tabpack* h, int B, int B_pad, uint32_t step, int train, bool stacked = false) {
   GemmArgs<T> g;
   g.probs = h->probs_dev;
   g.tiles = h->tiles_dev;
-  g.xb = (const T*)h->xb;
+  g.xb = (const T*)(stacked ? h->xbs : h->xb);
+  g.xb_stride = stacked ? h->xb_elems : 0;
   g.act = (T*)h->act;
   g.dz = (T*)h->dz;
   g.wq = (const T*)h->params;  // the CUDA-core path runs in fp32 mode only
@@ -600,11 +613,12 @@ AdamDev adam_dev(tabpack* h, __nv_bfloat16* wq_out) {
 }
 
 template <typename T>
-tp_status run_forward(tabpack* h, int B, int B_pad, uint32_t step, const StepDyn* dyn, int train) {
+tp_status run_forward(tabpack* h, int B, int B_pad, uint32_t step, const StepDyn* dyn, int train,
+                      bool stacked = false) {
   if (h->bf16) {  // every layer in one launch
     int slot;
     prof_begin(h, train ? TP_PH_FWD : TP_PH_PREDICT, &slot);
-    TP_TRY(tc_run_fwd(h->tc, h->st, B, B_pad, h->wcur, train, h->masks, h->B_cap, h->params, h->mem_dev, h->act,
+    TP_TRY(tc_run_fwd(stacked ? h->tcs : h->tc, h->st, B, B_pad, h->wcur, train, h->masks, h->B_cap, h->params, h->mem_dev, h->act,
                       h->err));
     TP_LAUNCHED(h);
     h->launches++;
@@ -614,7 +628,7 @@ tp_status run_forward(tabpack* h, int B, int B_pad, uint32_t step, const StepDyn
   for (int l = 0; l < h->Lmax; ++l) {  // CUDA-core path: one launch per depth
     int slot;
     prof_begin(h, train ? TP_PH_FWD : TP_PH_PREDICT, &slot);
-    auto g = gemm_args<T>(h, B, B_pad, step, train);
+    auto g = gemm_args<T>(h, B, B_pad, step, train, stacked);
     g.dyn = dyn;
     launch_gemm_simt<T>(h->st, g, h->fwd_rng[l].first, h->fwd_rng[l].second);
     TP_LAUNCHED(h);
@@ -647,19 +661,20 @@ MaskGen mask_gen(tabpack* h, uint32_t step, const StepDyn* dyn, uint32_t step_ad
 // dyn non-NULL: X, idx, y, loss_out and step are read from it on the device.
 template <typename T>
 tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* idx, const void* y, int B,
-                   uint32_t step, float* loss_out, bool update, const StepDyn* dyn) {
+                   uint32_t step, float* loss_out, bool update, const StepDyn* dyn, bool stacked) {
+  TcPlan& plan = stacked ? h->tcs : h->tc;
   const int B_pad = (int)round_up(B, kRowTile);
   const bool fused = update && h->bf16 && h->fuse_adamw;
   __nv_bfloat16* wq_next = h->bf16 ? h->wq[h->wcur ^ 1] : nullptr;
   int slot;
   prof_begin(h, TP_PH_GATHER, &slot);
-  launch_gather<T>(h->st, X, idx, dyn, B, B_pad, h->cfg.d_in, h->d_in_pad, h->ldx, (T*)h->xb, update ? 1 : 0,
-                   h->t_dev, h->bias_corr, h->active_ids_dev, h->n_active, h->cfg.beta1, h->cfg.beta2,
-                   h->tc.cnt_dev, h->tc.n_cnt);
+  launch_gather<T>(h->st, X, idx, dyn, B, B_pad, h->cfg.d_in, h->d_in_pad, h->ldx, (T*)(stacked ? h->xbs : h->xb),
+                   update ? 1 : 0, h->t_dev, h->bias_corr, h->active_ids_dev, h->n_active, h->cfg.beta1, h->cfg.beta2,
+                   plan.cnt_dev, plan.n_cnt, stacked ? 1 : 0, h->xb_elems);
   TP_LAUNCHED(h);
   h->launches++;
   prof_end(h, slot, 1, TP_PH_GATHER);
-  TP_TRY(run_forward<T>(h, B, B_pad, step, dyn, 1));
+  TP_TRY(run_forward<T>(h, B, B_pad, step, dyn, 1, stacked));
   // head + loss
   prof_begin(h, TP_PH_HEAD, &slot);
   HeadArgs<T> hg;
@@ -680,6 +695,7 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
   hg.task = h->cfg.task;
   hg.n_blk_cap = h->n_blk_cap;
   hg.dyn = dyn;
+  hg.idx_stride = stacked ? B : 0;
   launch_head<T>(h->st, hg, h->n_head_jobs);
   TP_LAUNCHED(h);
   h->launches++;
@@ -711,7 +727,7 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
   const AdamDev ad = adam_dev(h, wq_next);
   if (h->bf16) {
     prof_begin(h, TP_PH_BWD, &slot);
-    TP_TRY(tc_run_bwd(h->tc, h->st, B, B_pad, h->wcur, h->mem_dev, h->act, h->dz, h->grads, fused ? 1 : 0, ad,
+    TP_TRY(tc_run_bwd(plan, h->st, B, B_pad, h->wcur, h->mem_dev, h->act, h->dz, h->grads, fused ? 1 : 0, ad,
                       h->err));
     TP_LAUNCHED(h);
     h->launches++;
@@ -719,7 +735,7 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
   } else {
     for (int l = h->Lmax - 1; l >= 0; --l) {
       prof_begin(h, TP_PH_BWD, &slot);
-      auto g = gemm_args<T>(h, B, B_pad, step, 1);
+      auto g = gemm_args<T>(h, B, B_pad, step, 1, stacked);
       launch_gemm_simt<T>(h->st, g, h->bwd_rng[l].first, h->bwd_rng[l].second);
       TP_LAUNCHED(h);
       h->launches++;
@@ -757,7 +773,7 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
 // the device, or launch the kernels directly while profiling.
 template <typename T>
 tp_status step_entry(tabpack* h, const float* X, int64_t n_rows, const int32_t* idx, const void* y, int B,
-                     uint32_t step, float* loss_out, bool update) {
+                     uint32_t step, float* loss_out, bool update, bool stacked = false) {
   // the forward reads the step's dropout masks from the arena: fill it now
   // unless the previous step's AdamW pass did
   const bool masks_next = update && h->bf16 && !h->fuse_adamw && h->n_chunks > 0;
@@ -767,7 +783,7 @@ tp_status step_entry(tabpack* h, const float* X, int64_t n_rows, const int32_t* 
     h->launches++;
   }
   if (!h->use_graphs || h->profiling) {
-    TP_TRY(run_step<T>(h, X, n_rows, idx, y, B, step, loss_out, update, nullptr));
+    TP_TRY(run_step<T>(h, X, n_rows, idx, y, B, step, loss_out, update, nullptr, stacked));
   } else {
     // per-call arguments: pinned ring slot -> dyn_dev, ordered before the graph
     const int k = h->dyn_next;
@@ -779,13 +795,13 @@ tp_status step_entry(tabpack* h, const float* X, int64_t n_rows, const int32_t* 
     h->dyn_used[k] = true;
     tabpack::GraphEntry* ge = nullptr;
     for (auto& e : h->graphs)
-      if (e.B == B && e.update == (int)update && e.wcur == h->wcur) ge = &e;
+      if (e.B == B && e.update == (int)update && e.wcur == h->wcur && e.stacked == (int)stacked) ge = &e;
     if (!ge) {
       cudaStream_t user = h->st;
       h->st = h->st_cap;
       const int64_t l0 = h->launches;
       cudaError_t e = cudaStreamBeginCapture(h->st, cudaStreamCaptureModeThreadLocal);
-      tp_status s = e == cudaSuccess ? run_step<T>(h, X, n_rows, idx, y, B, step, loss_out, update, h->dyn_dev)
+      tp_status s = e == cudaSuccess ? run_step<T>(h, X, n_rows, idx, y, B, step, loss_out, update, h->dyn_dev, stacked)
                                      : fail(h, TP_ECUDA, "cudaStreamBeginCapture: %s", cudaGetErrorString(e));
       cudaGraph_t graph = nullptr;
       cudaError_t e2 = e == cudaSuccess ? cudaStreamEndCapture(h->st, &graph) : cudaSuccess;
@@ -801,7 +817,7 @@ tp_status step_entry(tabpack* h, const float* X, int64_t n_rows, const int32_t* 
       e = cudaGraphInstantiate(&exec, graph, 0);
       cudaGraphDestroy(graph);
       if (e != cudaSuccess) return fail(h, TP_ECUDA, "cudaGraphInstantiate: %s", cudaGetErrorString(e));
-      h->graphs.push_back(tabpack::GraphEntry{B, (int)update, h->wcur, exec, n_launch});
+      h->graphs.push_back(tabpack::GraphEntry{B, (int)update, h->wcur, (int)stacked, exec, n_launch});
       ge = &h->graphs.back();
     }
     TP_CUDA(h, cudaGraphLaunch(ge->exec, h->st));
@@ -810,6 +826,58 @@ tp_status step_entry(tabpack* h, const float* X, int64_t n_rows, const int32_t* 
   if (update && h->bf16) h->wcur ^= 1;
   h->masks_for = masks_next ? (int64_t)(uint32_t)(step + 1u) : (int64_t)step;
   h->last_B = B;
+  return TP_OK;
+}
+
+// The stacked-batch arena and (bf16) its tile plan, on first use and after an
+// active-set change.
+template <typename T>
+tp_status ensure_stacked(tabpack* h) {
+  const int m = h->cfg.m;
+  if (!h->xbs) {
+    TP_CUDA(h, cudaStreamSynchronize(h->st));
+    const size_t bytes = h->elem * (size_t)m * h->xb_elems;
+    TP_CUDA(h, cudaMalloc(&h->xbs, bytes));
+    TP_CUDA(h, cudaMemset(h->xbs, 0, bytes));
+    std::vector<OnesJob> jobs;
+    for (int i = 0; i < m; ++i) jobs.push_back(OnesJob{(int64_t)i * h->xb_elems, h->ldx, h->d_in_pad, h->B_cap, 0});
+    OnesJob* d = nullptr;
+    TP_CUDA(h, cudaMalloc(&d, sizeof(OnesJob) * jobs.size()));
+    cudaError_t e = cudaMemcpy(d, jobs.data(), sizeof(OnesJob) * jobs.size(), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) {
+      launch_fill_ones<T>(h->st, d, (int)jobs.size(), (T*)h->xbs, (T*)h->act);
+      h->launches++;
+      e = cudaGetLastError();
+    }
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+    cudaFree(d);
+    if (e != cudaSuccess) return fail(h, TP_ECUDA, "stacked batch arena: %s", cudaGetErrorString(e));
+    h->s_stale = true;
+  }
+  if (h->bf16 && h->s_stale) {
+    TcLayout lay;
+    lay.depth = &h->depth;
+    lay.width = &h->width;
+    lay.active = &h->active;
+    lay.W_off = &h->W_off;
+    lay.b_off = &h->b_off;
+    lay.act_off = &h->act_off;
+    lay.dz_off = &h->dz_off;
+    lay.m = m;
+    lay.d_in_pad = h->d_in_pad;
+    lay.ldx = h->ldx;
+    lay.B_cap = h->B_cap;
+    lay.wq[0] = h->wq[0];
+    lay.wq[1] = h->wq[1];
+    lay.xb = h->xbs;
+    lay.act = h->act;
+    lay.dz = h->dz;
+    lay.mask_off = h->mask_words > 0 ? &h->mask_off : nullptr;
+    lay.xb_stride = h->xb_elems;
+    TP_CUDA(h, cudaStreamSynchronize(h->st));
+    TP_TRY(tc_build_plan(h->tcs, lay, h->err));
+  }
+  h->s_stale = false;
   return TP_OK;
 }
 
@@ -989,6 +1057,7 @@ tp_status sync_check(tabpack* h) {
   TP_CUDA(h, cudaStreamSynchronize(h->st));
   if (h->bf16 && h->tc.enabled) TP_TRY(tc_check(h->tc, h->st, h->err));
   if (h->bf16 && h->tcp.enabled) TP_TRY(tc_check(h->tcp, h->st, h->err));
+  if (h->bf16 && h->tcs.enabled) TP_TRY(tc_check(h->tcs, h->st, h->err));
   return TP_OK;
 }
 
@@ -1088,6 +1157,30 @@ tp_status pack_forward_backward(tabpack_t* h, const float* X, int64_t n_rows, co
   if (h->n_active == 0) return fail(h, TP_ESTATE, "no active member");
   return h->bf16 ? step_entry<__nv_bfloat16>(h, X, n_rows, idx, y, B, step, loss_out, false)
                  : step_entry<float>(h, X, n_rows, idx, y, B, step, loss_out, false);
+}
+
+tp_status pack_train_step_stacked(tabpack_t* h, const float* X, int64_t n_rows, const int32_t* idx, const void* y,
+                                  int32_t B, uint32_t step, float* loss_out) {
+  TP_TRY(check_step_args(h, X, n_rows, idx, y, B));
+  if (h->n_active == 0) return fail(h, TP_ESTATE, "no active member");
+  if (h->bf16) {
+    TP_TRY(ensure_stacked<__nv_bfloat16>(h));
+    return step_entry<__nv_bfloat16>(h, X, n_rows, idx, y, B, step, loss_out, true, true);
+  }
+  TP_TRY(ensure_stacked<float>(h));
+  return step_entry<float>(h, X, n_rows, idx, y, B, step, loss_out, true, true);
+}
+
+tp_status pack_forward_backward_stacked(tabpack_t* h, const float* X, int64_t n_rows, const int32_t* idx,
+                                        const void* y, int32_t B, uint32_t step, float* loss_out) {
+  TP_TRY(check_step_args(h, X, n_rows, idx, y, B));
+  if (h->n_active == 0) return fail(h, TP_ESTATE, "no active member");
+  if (h->bf16) {
+    TP_TRY(ensure_stacked<__nv_bfloat16>(h));
+    return step_entry<__nv_bfloat16>(h, X, n_rows, idx, y, B, step, loss_out, false, true);
+  }
+  TP_TRY(ensure_stacked<float>(h));
+  return step_entry<float>(h, X, n_rows, idx, y, B, step, loss_out, false, true);
 }
 
 tp_status pack_predict(tabpack_t* h, const float* X, int64_t N, float* out) {

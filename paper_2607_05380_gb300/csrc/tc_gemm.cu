@@ -871,8 +871,12 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
     for (int set = 0; set < 2; ++set) {
       const int br = set ? 128 : 64;
       const int base = (int)maps.size();
-      if (!encode_map(&mp, lay.xb, lay.ldx, lay.B_cap, lay.ldx, br, err)) return TP_ECUDA;
-      maps.push_back(mp);
+      // the batch matrix: one, or one per member (stacked batches: map index = member)
+      for (int i = 0; i < (lay.xb_stride ? m : 1); ++i) {
+        const __nv_bfloat16* xbi = (const __nv_bfloat16*)lay.xb + (int64_t)i * lay.xb_stride;
+        if (!encode_map(&mp, xbi, lay.ldx, lay.B_cap, lay.ldx, br, err)) return TP_ECUDA;
+        maps.push_back(mp);
+      }
       for (int i = 0; i < m; ++i)
         for (int l = 0; l < depth[i]; ++l) {
           const int w = width[i];
@@ -1021,7 +1025,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
       t.mask_off = lay.mask_off ? (int32_t)(*lay.mask_off)[i][l] : -1;
       t.m_real = 0; t.n_real = w;
       t.k_len = l == 0 ? lay.d_in_pad : w;
-      t.map_a = l == 0 ? 0 : plan.map_act[(size_t)i * kMaxDepth + l - 1];
+      t.map_a = l == 0 ? (lay.xb_stride ? i : 0) : plan.map_act[(size_t)i * kMaxDepth + l - 1];
       t.map_b = plan.map_w[(size_t)i * kMaxDepth + l];
       t.ldc = w + kOnesCols;
       t.ld_aux = 0;
@@ -1074,7 +1078,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
       t.m_real = w; t.n_real = in_pad + 1;
       t.k_len = 0;
       t.map_a = plan.map_dz[(size_t)i * kMaxDepth + l];
-      t.map_b = l == 0 ? 0 : plan.map_act[(size_t)i * kMaxDepth + l - 1];
+      t.map_b = l == 0 ? (lay.xb_stride ? i : 0) : plan.map_act[(size_t)i * kMaxDepth + l - 1];
       t.ldc = in_pad;
       t.ld_aux = 0;
       t.dep = from_head ? -1 : cnt_dz(i, l);  // every row block of dz_l

@@ -76,6 +76,7 @@ struct TcLayout {          // what the plan needs to know about the pack's arena
   const void* act;
   const void* dz;
   bool fwd_only = false;   // forward tiles only (prediction): no dz maps, counters or backward tiles
+  int64_t xb_stride = 0;   // > 0: a batch matrix per member (stacked batches), this many elements apart
   // per (member, layer): word offset of the dropout keep words, -1 for none (NULL: no masks)
   const std::vector<std::array<int64_t, kMaxDepth>>* mask_off = nullptr;
 };

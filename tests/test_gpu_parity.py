@@ -192,6 +192,76 @@ def test_one_step_logits_losses_grads(tp, prec, task, d_out, B):
     assert not problems, problems
 
 
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+@pytest.mark.parametrize("task,d_out", [("binary", 1), ("multiclass", 7), ("regression", 1)])
+@pytest.mark.parametrize("B", [256, 200])
+def test_stacked_batches_one_step(tp, prec, task, d_out, B):
+    """A batch per member (Sec. 3.6, idx [m, B]): every member's logits, loss
+    and gradients against the oracle's stacked step, and member 3's equal to
+    the shared-batch step on its own batch (bit-exact)."""
+    d_in, m = 37, 6
+    hp = random_pack(m, d_in, d_out, seed=40 + d_out, width=(16, 160, 16), depth=(1, 4))
+    pk, orc = pair(tp, task, d_in, d_out, hp, prec, 256)
+    X, y = make_data(task, 400, d_in, d_out, 1)
+    rng = np.random.default_rng(3)
+    idx = np.stack([rng.choice(400, B, replace=False) for _ in range(m)]).astype(np.int32)
+    Xd, yd, idxd = to_dev(X, y, idx)
+    loss = torch.zeros(m, dtype=torch.float32, device=DEV)
+    pk.forward_backward(Xd, idxd, yd, 5, loss)
+    lo = orc.train_step(X, idx, y, 5, update=False)
+    problems = _compare_step(pk, orc, hp, prec, loss.cpu().numpy(), lo)
+    assert not problems, problems
+    # the shared-batch step on row 3 gives member 3 the same result
+    pk2, _ = pair(tp, task, d_in, d_out, hp, prec, 256)
+    (idx3,) = to_dev(idx[3].copy())
+    loss2 = torch.zeros(m, dtype=torch.float32, device=DEV)
+    pk2.forward_backward(Xd, idx3, yd, 5, loss2)
+    assert loss2.cpu().numpy()[3] == loss.cpu().numpy()[3]
+    for l in range(int(hp["depth"][3]) + 1):
+        np.testing.assert_array_equal(pk2.get_grads(3, l)[0], pk.get_grads(3, l)[0])
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_stacked_batches_ten_steps(tp, prec):
+    """Ten AdamW steps on stacked batches (graph replay after the first
+    step), with a shared-batch step in the middle (the two plans alternate),
+    against the oracle."""
+    d_in, m, B, d_out = 24, 8, 192, 5
+    hp = random_pack(m, d_in, d_out, seed=52, width=(16, 128, 16), depth=(1, 3))
+    pk, orc = pair(tp, "multiclass", d_in, d_out, hp, prec, 256)
+    X, y = make_data("multiclass", 600, d_in, d_out, 3)
+    Xd, yd = to_dev(X, y)
+    rng = np.random.default_rng(9)
+    loss = torch.zeros(m, dtype=torch.float32, device=DEV)
+    margin = np.full(m, np.inf)
+    for step in range(10):
+        if step == 5:
+            idx = rng.choice(600, B, replace=False).astype(np.int32)
+        else:
+            idx = np.stack([rng.choice(600, B, replace=False) for _ in range(m)]).astype(np.int32)
+        (idxd,) = to_dev(idx)
+        pk.train_step(Xd, idxd, yd, step, loss)
+        lo = orc.train_step(X, idx, y, step)
+        margin = np.minimum(margin, [orc.margin(i) for i in range(m)])
+        lg = loss.cpu().numpy()
+        for i in range(m):
+            assert abs(lg[i] - lo[i]) <= TOL["bf16"] * max(1.0, abs(lo[i])), (step, i, lg[i], lo[i])
+    errs = {}
+    for i in range(m):
+        e = 0.0
+        for l in range(int(hp["depth"][i]) + 1):
+            W, b = pk.get_params(i, l)
+            Wo, bo = orc.get_params(i, l)
+            e = max(e, rel_err(W, Wo), rel_err(b, bo))
+        errs[i] = e
+    bad = {i: e for i, e in errs.items() if e > TOL[prec]}
+    if prec == "fp32":
+        ties = {i for i in bad if margin[i] < 1e-5}
+        assert all(errs[i] <= TOL["bf16"] for i in ties), (errs, margin)
+        bad = {i: e for i, e in bad.items() if i not in ties}
+    assert not bad, (errs, margin)
+
+
 @pytest.mark.parametrize("prec,fuse", [("fp32", False), ("bf16", False), ("bf16", True)])
 @pytest.mark.parametrize("task,d_out", [("binary", 1), ("multiclass", 5), ("regression", 1)])
 def test_ten_steps_params(tp, prec, fuse, task, d_out):
