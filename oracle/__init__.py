@@ -73,6 +73,9 @@ def lib():
                 "orc_init_value": (f64, [u64, u32, u32, u32, i32]),
                 "orc_train_step": (ctypes.c_int, [P, P, i64, P, P, P, i32, u32, i32, P]),
                 "orc_train_step_stacked": (ctypes.c_int, [P, P, i64, P, P, P, i32, u32, i32, P]),
+                "orc_set_muon": (ctypes.c_int, [P, P, ctypes.c_double, i32]),
+                "orc_newton_schulz": (None, [P, i32, i32, i32, i32, P]),
+                "orc_get_muon_dir": (ctypes.c_int, [P, i32, i32, P]),
                 "orc_predict": (ctypes.c_int, [P, P, i64, P]),
                 "orc_set_active": (ctypes.c_int, [P, P]),
                 "orc_adamw_apply": (None, [P, P, P, P, i64, i64, f64, f64, f64, f64, f64]),
@@ -209,6 +212,19 @@ class OraclePack:
         a = np.ascontiguousarray(active, dtype=np.uint8)
         lib().orc_set_active(self._h, _ptr(a))
 
+    def set_muon(self, lr_muon, momentum=0.95, ns_steps=5):
+        """Muon for the hidden-layer weights from now on (Sec. 3.4)."""
+        lr = np.ascontiguousarray(lr_muon, dtype=np.float64)
+        if lib().orc_set_muon(self._h, _ptr(lr), float(momentum), int(ns_steps)):
+            raise ValueError("oracle set_muon rejected its arguments")
+
+    def muon_dir(self, member, layer):
+        n_out, n_in = self.layer_shape(member, layer)
+        out = np.zeros((n_out, n_in), dtype=np.float64)
+        if lib().orc_get_muon_dir(self._h, int(member), int(layer), _ptr(out)):
+            raise ValueError("no Muon direction for this layer")
+        return out
+
     def _two(self, fn, member, layer):
         n_out, n_in = self.layer_shape(member, layer)
         W = np.zeros((n_out, n_in), dtype=np.float64)
@@ -261,6 +277,14 @@ class OraclePack:
 
     def member_steps(self, member):
         return int(lib().orc_member_steps(self._h, member))
+
+
+def newton_schulz(U, steps=5, bf16=False):
+    """Muon's orthogonalized direction of U (oracle; see tabpack_oracle.c)."""
+    U = np.ascontiguousarray(U, dtype=np.float64)
+    O = np.zeros_like(U)
+    lib().orc_newton_schulz(_ptr(U), U.shape[0], U.shape[1], int(steps), int(bool(bf16)), _ptr(O))
+    return O
 
 
 def greedy(preds, y, task, score="loss", m_ens=32, fp32_terms=False):

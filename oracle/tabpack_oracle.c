@@ -123,11 +123,16 @@ typedef struct {
   uint8_t **keep;     /* [L]: dropout keep decisions, B x w                */
   double *logits;     /* B x d_out                                          */
   double margin;      /* min |Z| / rms(Z) of the last forward               */
+  double lr_muon;     /* Muon learning rate (when the pack uses Muon)       */
+  double **dir;       /* [L]: the last Muon direction O of each hidden W    */
 } orc_member;
 
 struct orc_pack {
   orc_config cfg;
   orc_member* mem;
+  int32_t muon;       /* 1: hidden-layer weights take Muon steps (Sec. 3.4) */
+  double momentum;    /* Muon momentum mu                                   */
+  int32_t ns_steps;   /* Newton-Schulz iterations                           */
 };
 
 static double* orc_zeros(int64_t n) { return (double*)calloc((size_t)(n > 0 ? n : 1), sizeof(double)); }
@@ -177,6 +182,10 @@ void orc_destroy(orc_pack* h) {
     }
     free(M->W); free(M->b); free(M->gW); free(M->gb);
     free(M->mW); free(M->vW); free(M->mb); free(M->vb);
+    if (M->dir) {
+      for (int l = 0; l < M->L; ++l) free(M->dir[l]);
+      free(M->dir);
+    }
     free(M->in_dim); free(M->out_dim);
   }
   free(h->mem);
@@ -428,6 +437,109 @@ static void orc_adamw(const orc_pack* h, const orc_member* M, double* p, double*
   orc_adamw_apply(p, m, v, g, n, M->t, (double)M->lr, wd, h->cfg.beta1, h->cfg.beta2, h->cfg.eps);
 }
 
+/* ------------------------------------------------------------------------ */
+/* Muon (Sec. 3.4 and App. F.1: Muon for the weight matrices of the hidden  */
+/* layers, AdamW for biases and the head), after Jordan et al. (2024):       */
+/*   M <- mu M + (1 - mu) G;  U = (1 - mu) G + mu M (Nesterov);              */
+/*   X = U / max(||U||_F, 1e-7), taken transposed when U has more rows than  */
+/*   columns;                                                                */
+/*   ns_steps times: A = X X^T, Bm = b A + c A A, X = a X + Bm X with        */
+/*   (a, b, c) = (3.4445, -4.7750, 2.0315);  O = X (transposed back);        */
+/*   W <- W - lr wd W;  W <- W - lr max(1, rows / cols)^(1/2) O.             */
+/* In bf16-storage mode X, A and Bm are rounded to bf16 where the GPU       */
+/* stores them.                                                              */
+/* ------------------------------------------------------------------------ */
+static const double ORC_NS_A = 3.4445, ORC_NS_B = -4.7750, ORC_NS_C = 2.0315;
+
+/* The orthogonalized direction O [rows, cols] of U [rows, cols].            */
+void orc_newton_schulz(const double* U, int32_t rows, int32_t cols, int32_t steps, int32_t bf16, double* O) {
+  const int tr = rows > cols;
+  const int r = tr ? cols : rows, c = tr ? rows : cols;
+  double* X = orc_zeros((int64_t)r * c);
+  double* A = orc_zeros((int64_t)r * r);
+  double* Bm = orc_zeros((int64_t)r * r);
+  double* Xn = orc_zeros((int64_t)r * c);
+  double nrm = 0.0;
+  for (int64_t e = 0; e < (int64_t)rows * cols; ++e) nrm += U[e] * U[e];
+  nrm = sqrt(nrm);
+  if (nrm < 1e-7) nrm = 1e-7;
+  for (int i = 0; i < rows; ++i)
+    for (int j = 0; j < cols; ++j) {
+      const double x = U[(int64_t)i * cols + j] / nrm;
+      X[tr ? (int64_t)j * c + i : (int64_t)i * c + j] = bf16 ? orc_round_bf16(x) : x;
+    }
+  for (int it = 0; it < steps; ++it) {
+    for (int i = 0; i < r; ++i)          /* A = X X^T */
+      for (int j = 0; j < r; ++j) {
+        double s = 0.0;
+        for (int k = 0; k < c; ++k) s += X[(int64_t)i * c + k] * X[(int64_t)j * c + k];
+        A[(int64_t)i * r + j] = bf16 ? orc_round_bf16(s) : s;
+      }
+    for (int i = 0; i < r; ++i)          /* Bm = b A + c A A */
+      for (int j = 0; j < r; ++j) {
+        double s = 0.0;
+        for (int k = 0; k < r; ++k) s += A[(int64_t)i * r + k] * A[(int64_t)k * r + j];
+        const double v = ORC_NS_B * A[(int64_t)i * r + j] + ORC_NS_C * s;
+        Bm[(int64_t)i * r + j] = bf16 ? orc_round_bf16(v) : v;
+      }
+    for (int i = 0; i < r; ++i)          /* X = a X + Bm X */
+      for (int j = 0; j < c; ++j) {
+        double s = 0.0;
+        for (int k = 0; k < r; ++k) s += Bm[(int64_t)i * r + k] * X[(int64_t)k * c + j];
+        const double v = ORC_NS_A * X[(int64_t)i * c + j] + s;
+        Xn[(int64_t)i * c + j] = bf16 ? orc_round_bf16(v) : v;
+      }
+    double* t = X;
+    X = Xn;
+    Xn = t;
+  }
+  for (int i = 0; i < rows; ++i)
+    for (int j = 0; j < cols; ++j) O[(int64_t)i * cols + j] = X[tr ? (int64_t)j * c + i : (int64_t)i * c + j];
+  free(X); free(A); free(Bm); free(Xn);
+}
+
+static void orc_muon(const orc_pack* h, orc_member* M, int l) {
+  const int rows = M->out_dim[l], cols = M->in_dim[l];
+  const int64_t n = (int64_t)rows * cols;
+  double* U = orc_zeros(n);
+  const double mu = h->momentum;
+  for (int64_t e = 0; e < n; ++e) {
+    M->mW[l][e] = mu * M->mW[l][e] + (1.0 - mu) * M->gW[l][e];
+    U[e] = (1.0 - mu) * M->gW[l][e] + mu * M->mW[l][e];
+  }
+  if (!M->dir[l]) M->dir[l] = orc_zeros(n);
+  orc_newton_schulz(U, rows, cols, h->ns_steps, h->cfg.bf16_storage, M->dir[l]);
+  const double lr = M->lr_muon, wd = (double)M->wd;
+  const double scale = sqrt(rows > cols ? (double)rows / (double)cols : 1.0);
+  for (int64_t e = 0; e < n; ++e) {
+    M->W[l][e] = M->W[l][e] - lr * wd * M->W[l][e];
+    M->W[l][e] = M->W[l][e] - lr * scale * M->dir[l][e];
+  }
+  free(U);
+}
+
+int orc_set_muon(orc_pack* h, const double* lr_muon, double momentum, int32_t ns_steps) {
+  if (!h || !lr_muon || !(momentum >= 0.0 && momentum < 1.0) || ns_steps < 1) return 1;
+  for (int i = 0; i < h->cfg.m; ++i) if (!(lr_muon[i] >= 0.0)) return 1;
+  h->muon = 1;
+  h->momentum = momentum;
+  h->ns_steps = ns_steps;
+  for (int i = 0; i < h->cfg.m; ++i) {
+    orc_member* M = &h->mem[i];
+    M->lr_muon = lr_muon[i];
+    if (!M->dir) M->dir = (double**)calloc((size_t)M->L, sizeof(double*));
+  }
+  return 0;
+}
+
+int orc_get_muon_dir(const orc_pack* h, int32_t member, int32_t layer, double* out) {
+  if (!h || !h->muon || member < 0 || member >= h->cfg.m) return 1;
+  const orc_member* M = &h->mem[member];
+  if (layer < 0 || layer >= M->L || !M->dir[layer]) return 1;
+  memcpy(out, M->dir[layer], sizeof(double) * (size_t)M->out_dim[layer] * (size_t)M->in_dim[layer]);
+  return 0;
+}
+
 /* One step of every active member; member i reads its batch rows from
  * idx + i * idx_stride (idx_stride 0: one batch shared by all members;
  * idx_stride B: the stacked per-member batches of Sec. 3.6).               */
@@ -458,7 +570,8 @@ static int orc_step(orc_pack* h, const float* X, int64_t N, const int32_t* idx, 
     if (update) {
       M->t += 1;
       for (int l = 0; l <= M->L; ++l) {
-        orc_adamw(h, M, M->W[l], M->mW[l], M->vW[l], M->gW[l], (int64_t)M->out_dim[l] * M->in_dim[l], 0);
+        if (h->muon && l < M->L) orc_muon(h, M, l);
+        else orc_adamw(h, M, M->W[l], M->mW[l], M->vW[l], M->gW[l], (int64_t)M->out_dim[l] * M->in_dim[l], 0);
         orc_adamw(h, M, M->b[l], M->mb[l], M->vb[l], M->gb[l], M->out_dim[l], 1);
       }
     }

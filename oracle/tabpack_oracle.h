@@ -106,6 +106,17 @@ int orc_predict(orc_pack* h, const float* X, int64_t N, double* out);
 
 int orc_set_active(orc_pack* h, const uint8_t* active);
 
+/* Muon for the hidden-layer weight matrices (the paper's default optimizer,
+ * Sec. 3.4 / App. F.1; AdamW stays on biases and the head): member i with
+ * learning rate lr_muon[i], momentum mu (Nesterov), ns_steps Newton-Schulz
+ * iterations; see tabpack_oracle.c for the steps.  Returns 0 on success.     */
+int orc_set_muon(orc_pack* h, const double* lr_muon, double momentum, int32_t ns_steps);
+/* The orthogonalized direction O of U [rows, cols] (bf16 != 0: rounding of
+ * X, A and Bm to bf16 where the GPU stores them).                            */
+void orc_newton_schulz(const double* U, int32_t rows, int32_t cols, int32_t steps, int32_t bf16, double* O);
+/* The direction O [out, in] of the last Muon step of hidden layer `layer`.  */
+int orc_get_muon_dir(const orc_pack* h, int32_t member, int32_t layer, double* out);
+
 /* One AdamW step (PyTorch semantics, the update the training step applies to
  * every parameter; Sec. 3.4) on n elements in place: decoupled decay
  * p <- p - lr wd p, moments m, v, then the step bias-corrected for step
