@@ -267,6 +267,8 @@ def main():
                     help="train only the first N members of the workload (profiling small cases)")
     ap.add_argument("--fuse-optimizer", action="store_true", help="AdamW inside the weight-gradient epilogue")
     ap.add_argument("--no-online", action="store_true", help="skip timing the online-ensemble epoch end")
+    ap.add_argument("--muon", action="store_true",
+                    help="Muon for the hidden-layer weights (the paper's default optimizer), AdamW for the rest")
     ap.add_argument("--stacked", action="store_true",
                     help="a batch per member (idx [m, B], Sec. 3.6) instead of one batch shared by all members")
     args = ap.parse_args()
@@ -314,6 +316,11 @@ def main():
                    max_batch=B, seed=SEED_INIT, precision=args.precision, stream=stream,
                    fuse_optimizer=args.fuse_optimizer)
     loss = torch.zeros(wl.m, dtype=torch.float32, device=dev)
+    lr_muon = None
+    if args.muon:   # Muon lr LogUniform[1e-3, 1e-1] per member
+        rng_m = np.random.default_rng(SEED_HP + 100)
+        lr_muon = np.exp(rng_m.uniform(math.log(1e-3), math.log(1e-1), wl.m)).astype(np.float32)
+        pack.set_muon(lr_muon)
 
     for s in range(args.warmup):
         pack.train_step(X, idx_all[s], y, s, loss)
@@ -376,6 +383,17 @@ def main():
     roof = dict(gemm if gemm_ms >= adam_ms else mem)
     roof["other"] = mem if gemm_ms >= adam_ms else gemm
     roof["shares"] = shares
+    if args.muon:   # the Newton-Schulz products: 5 x (4 r^2 c + 2 r^3) per matrix
+        ns_flops = 0.0
+        for L_, w_ in zip(hp["depth"], hp["width"]):
+            for l in range(int(L_)):
+                cols = wl.d_in if l == 0 else int(w_)
+                r_, c_ = min(int(w_), cols), max(int(w_), cols)
+                ns_flops += 5 * (4.0 * r_ * r_ * c_ + 2.0 * r_ ** 3)
+        muon_ms = prof["muon"][0] / n_prof
+        roof["muon"] = {"kernels": "k_muon_* + k_tc_gemm Newton-Schulz launches", "ms_per_step": muon_ms,
+                        "ns_flop_per_step": ns_flops, "achieved": ns_flops / (muon_ms / 1e3) / 1e12,
+                        "unit": "TFLOP/s", "peak": pk["bf16_sus"], "frac": ns_flops / (muon_ms / 1e3) / 1e12 / pk["bf16_sus"]}
 
     # end to end through the public API with host buffers: per step the batch
     # rows and labels go host -> device (pinned), the member losses come back
@@ -434,7 +452,9 @@ def main():
                            "l2": "inputs larger than L2: each step streams ~%.2f GB of parameters and optimizer state"
                                  % (30.0 * n_params / 1e9),
                            "parallelism": "one independent pack per GPU" if world > 1 else "single GPU",
-                           "batches": "one per member (stacked)" if args.stacked else "one shared by all members"},
+                           "batches": "one per member (stacked)" if args.stacked else "one shared by all members",
+                           "optimizer": "Muon (hidden weights, lr LogUniform[1e-3, 1e-1]) + AdamW" if args.muon
+                                        else "AdamW"},
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches, "online_epoch": online,
                 "clocks": clk.summary(), "final_losses_mean": float(np.nanmean(lossv))}
         print(json.dumps(line), flush=True)

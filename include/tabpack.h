@@ -136,6 +136,29 @@ tp_status pack_train_step_stacked(tabpack_t* pack, const float* X, int64_t n_row
 tp_status pack_forward_backward_stacked(tabpack_t* pack, const float* X, int64_t n_rows, const int32_t* idx,
                                         const void* y, int32_t B, uint32_t step, float* loss_out);
 
+/* Muon for the hidden-layer weight matrices (the paper's default optimizer:
+ * Muon for the weights of the hidden linear layers, AdamW for biases and the
+ * head; Sec. 3.4, App. F.1; Jordan et al. 2024), from the next step on.
+ * Per step and matrix W [out, in] with gradient G:
+ *   M <- mu M + (1 - mu) G;  U = (1 - mu) G + mu M (Nesterov);
+ *   X = U / max(||U||_F, 1e-7), transposed when out > in;
+ *   ns_steps times: A = X X^T; Bm = b A + c A A; X = a X + Bm X,
+ *   (a, b, c) = (3.4445, -4.7750, 2.0315) (on the tensor cores in bf16 mode,
+ *   X, A and Bm stored in bf16; on CUDA cores in fp32 mode);
+ *   W <- W - lr_muon wd W;  W <- W - lr_muon max(1, out / in)^(1/2) X
+ * (in = the real input width).  lr_muon: host [m]; wd: the member's weight
+ * decay; momentum in [0, 1); ns_steps in 1..32 (5 in the paper's Muon).  The
+ * momentum buffers start at zero; AdamW in the weight-gradient epilogue
+ * (fuse_optimizer) is turned off.  Allocates the Newton-Schulz buffers
+ * (2 r c + 2 r^2 elements per matrix, r = min(out, in), c = max) on the
+ * first call; synchronises.                                                  */
+tp_status pack_set_muon(tabpack_t* pack, const float* lr_muon, float momentum, int32_t ns_steps);
+
+/* The direction X of the last Muon step of hidden layer `layer` of `member`
+ * (the orthogonalised momentum, [out, in] with the real input width):
+ * host float32.  For tests and diagnostics; synchronises.                    */
+tp_status pack_debug_muon_dir(tabpack_t* pack, int32_t member, int32_t layer, float* out);
+
 /* Per-member validation predictions (Sec. 3.5 "Online ensemble"): forward
  * without dropout of every active member on all N rows of X.
  *   X: device float32 [N, d_in];  out: device float32 [m, N, d_out]:
@@ -251,7 +274,7 @@ tp_status pack_debug_activations(tabpack_t* pack, int32_t member, int32_t layer,
  * (synchronises).  Families: see tp_phase.                                  */
 typedef enum {
   TP_PH_GATHER = 0, TP_PH_FWD = 1, TP_PH_HEAD = 2, TP_PH_BWD = 3, TP_PH_BIAS = 4,
-  TP_PH_ADAMW = 5, TP_PH_PREDICT = 6, TP_PH_COUNT = 7
+  TP_PH_ADAMW = 5, TP_PH_PREDICT = 6, TP_PH_MUON = 7, TP_PH_COUNT = 8
 } tp_phase;
 tp_status pack_profile_enable(tabpack_t* pack, int32_t enable);
 tp_status pack_profile_read(tabpack_t* pack, double* ms /* [TP_PH_COUNT] */,

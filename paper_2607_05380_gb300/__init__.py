@@ -24,7 +24,7 @@ SCORE_LOSS, SCORE_ACCURACY, SCORE_RMSE = 0, 1, 2
 TASKS = {"binary": BINARY, "multiclass": MULTICLASS, "regression": REGRESSION}
 PRECISIONS = {"bf16": BF16, "fp32": FP32}
 SCORES = {"loss": SCORE_LOSS, "accuracy": SCORE_ACCURACY, "rmse": SCORE_RMSE}
-PHASES = ["gather", "fwd", "head", "bwd", "bias", "adamw", "predict"]
+PHASES = ["gather", "fwd", "head", "bwd", "bias", "adamw", "predict", "muon"]
 
 # every entry point declared in include/tabpack.h
 SYMBOLS = ["pack_create", "pack_destroy", "pack_set_stream", "pack_train_step", "pack_forward_backward",
@@ -34,7 +34,8 @@ SYMBOLS = ["pack_create", "pack_destroy", "pack_set_stream", "pack_train_step", 
            "pack_snapshot", "pack_restore", "pack_get_config", "pack_member_hparams", "pack_get_active",
            "pack_get_stream", "pack_online_create", "pack_online_destroy", "pack_online_epoch", "pack_online_info",
            "pack_online_members", "pack_online_ensemble", "pack_online_snapshot", "pack_online_predict",
-           "pack_online_last_error", "pack_train_step_stacked", "pack_forward_backward_stacked"]
+           "pack_online_last_error", "pack_train_step_stacked", "pack_forward_backward_stacked", "pack_set_muon",
+           "pack_debug_muon_dir"]
 
 
 class TabpackError(RuntimeError):
@@ -108,6 +109,8 @@ def load_library(path: str = LIB_PATH):
         "pack_online_predict": (st, [P, P, i64, P]),
         "pack_online_last_error": (ctypes.c_char_p, [P]),
         "pack_train_step_stacked": (st, [P, P, i64, P, P, i32, u32, P]),
+        "pack_set_muon": (st, [P, P, ctypes.c_float, i32]),
+        "pack_debug_muon_dir": (st, [P, i32, i32, P]),
         "pack_forward_backward_stacked": (st, [P, P, i64, P, P, i32, u32, P]),
     }
     for name, (res, args) in sig.items():
@@ -219,6 +222,17 @@ class Pack:
     def set_active(self, active):
         a = np.ascontiguousarray(active, dtype=np.uint8)
         _check(load_library().pack_set_active(self._h, _hptr(a)), self._h)
+
+    def set_muon(self, lr_muon, momentum=0.95, ns_steps=5):
+        """Muon for the hidden-layer weights from the next step on."""
+        lr = np.ascontiguousarray(lr_muon, dtype=np.float32)
+        _check(load_library().pack_set_muon(self._h, _hptr(lr), float(momentum), int(ns_steps)), self._h)
+
+    def muon_dir(self, member, layer):
+        o, i = self.layer_shape(member, layer)
+        out = np.zeros((o, i), dtype=np.float32)
+        _check(load_library().pack_debug_muon_dir(self._h, int(member), int(layer), _hptr(out)), self._h)
+        return out
 
     def get_active(self):
         a = np.zeros(self.m, dtype=np.uint8)

@@ -100,15 +100,15 @@ __global__ void __launch_bounds__(256) k_gemm_simt(GemmArgs<T> g, int32_t tile_b
   const int K = P.K ? P.K : g.B_pad;
   if (t.m0 >= M) return;
   const uint32_t step = g.dyn ? g.dyn->step : g.step;
-  const T* bases[4] = {g.xb, g.act, g.dz, g.wq};
+  const T* bases[5] = {g.xb, g.act, g.dz, g.wq, g.ns};
   // stacked batches: the member's own batch matrix
   const int64_t xs = (int64_t)P.member * g.xb_stride;
   const T* A = bases[P.a_src] + P.a_off + (P.a_src == kSrcXb ? xs : 0);
   const T* Bm = bases[P.b_src] + P.b_off + (P.b_src == kSrcXb ? xs : 0);
   int64_t a_rs, a_ks, b_rs, b_ks;
-  if (P.kind == kFwd) {
+  if (P.kind == kFwd || P.kind == kNsGram || P.kind == kNsPoly) {
     a_rs = P.lda; a_ks = 1; b_rs = P.ldb; b_ks = 1;
-  } else if (P.kind == kDgrad) {
+  } else if (P.kind == kDgrad || P.kind == kNsApply) {
     a_rs = P.lda; a_ks = 1; b_rs = 1; b_ks = P.ldb;
   } else {
     a_rs = 1; a_ks = P.lda; b_rs = 1; b_ks = P.ldb;
@@ -160,7 +160,18 @@ __global__ void __launch_bounds__(256) k_gemm_simt(GemmArgs<T> g, int32_t tile_b
   for (int i = 0; i < 4; ++i) {
     const int r = t.m0 + ty + 16 * i;
     if (r >= M) continue;
-    if (P.kind == kFwd) {  // N = w, a multiple of 16
+    if (P.kind >= kNsGram) {  // Newton-Schulz: alpha acc + beta aux (N a multiple of 8)
+      const float al = P.kind == kNsPoly ? kNsC : 1.f;
+      const float be = P.kind == kNsPoly ? kNsB : (P.kind == kNsApply ? kNsA : 0.f);
+      T* C = g.ns + P.c_off;
+      const T* Aux = g.ns + P.aux_off;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        float v = al * acc[i][j];
+        if (P.kind != kNsGram) v += be * Elem<T>::to_f(Aux[(int64_t)r * P.ld_aux + c0 + j]);
+        C[(int64_t)r * P.ldc + c0 + j] = Elem<T>::from_f(v);
+      }
+    } else if (P.kind == kFwd) {  // N = w, a multiple of 16
       uint32_t keep = g.train ? keep_bits4(g.seed, (uint32_t)P.member, (uint32_t)P.layer, step,
                                            (uint32_t)r, (uint32_t)(c0 >> 2), md.drop_T)
                               : 0xFu;
@@ -852,6 +863,100 @@ void launch_init(cudaStream_t st, const InitArgs& g, int n_chunks) {
   if (n_chunks > 0) k_init<<<n_chunks, 256, 0, st>>>(g);
 }
 
+// ------------------------------------------------------------------ Muon
+// One block per chunk of kMuonChunk elements of a Muon matrix (row-major
+// [rows, cols] in the arena).
+template <typename T>
+struct MuonChunk {
+  MuonMat mt;
+  int64_t e0, e1;  // element range of the chunk
+  __device__ __forceinline__ MuonChunk(const MuonArgs<T>& a) {
+    mt = a.mats[a.chunk_mat[blockIdx.x]];
+    e0 = (int64_t)(blockIdx.x - mt.chunk0) * kMuonChunk;
+    e1 = min(e0 + kMuonChunk, (int64_t)mt.rows * mt.cols);
+  }
+  // index of element e of W in X (transposed when tr)
+  __device__ __forceinline__ int64_t xi(int64_t e) const {
+    const int64_t i = e / mt.cols, j = e - i * mt.cols;
+    return mt.tr ? j * mt.c + i : i * mt.c + j;
+  }
+};
+
+// momentum M <- mu M + (1 - mu) G; U = (1 - mu) G + mu M; the chunk's sum of
+// squares of U (per-thread partials, then a fixed-order tree)
+template <typename T>
+__global__ void __launch_bounds__(256) k_muon_momentum(MuonArgs<T> a) {
+  pdl_trigger();
+  pdl_wait();
+  const MuonChunk<T> ck(a);
+  const float mu = a.mu;
+  double ss = 0.0;
+  for (int64_t e = ck.e0 + threadIdx.x; e < ck.e1; e += blockDim.x) {
+    const int64_t o = ck.mt.w_off + e;
+    const float g = a.grads[o];
+    const float m = mu * a.mom[o] + (1.f - mu) * g;
+    a.mom[o] = m;
+    const float u = (1.f - mu) * g + mu * m;
+    ss += (double)u * (double)u;
+  }
+  __shared__ double red[256];
+  red[threadIdx.x] = ss;
+  __syncthreads();
+  for (int s = 128; s > 0; s >>= 1) {
+    if (threadIdx.x < s) red[threadIdx.x] += red[threadIdx.x + s];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) a.part[blockIdx.x] = red[0];
+}
+
+// X0 = U / max(||U||_F, 1e-7), transposed when rows > cols
+template <typename T>
+__global__ void __launch_bounds__(256) k_muon_x0(MuonArgs<T> a) {
+  pdl_trigger();
+  pdl_wait();
+  const MuonChunk<T> ck(a);
+  __shared__ float inv_s;
+  if (threadIdx.x == 0) {
+    double ss = 0.0;
+    for (int k = 0; k < ck.mt.n_chunks; ++k) ss += a.part[ck.mt.chunk0 + k];
+    inv_s = (float)(1.0 / fmax(sqrt(ss), 1e-7));
+  }
+  __syncthreads();
+  const float inv = inv_s, mu = a.mu;
+  T* X = a.ns + ck.mt.x_off[0];
+  for (int64_t e = ck.e0 + threadIdx.x; e < ck.e1; e += blockDim.x) {
+    const int64_t o = ck.mt.w_off + e;
+    const float u = (1.f - mu) * a.grads[o] + mu * a.mom[o];
+    X[ck.xi(e)] = Elem<T>::from_f(u * inv);
+  }
+}
+
+// W <- W - lr wd W; W <- W - lr scale O, O = the final X (transposed back)
+template <typename T>
+__global__ void __launch_bounds__(256) k_muon_apply(MuonArgs<T> a) {
+  pdl_trigger();
+  pdl_wait();
+  const MuonChunk<T> ck(a);
+  const float lr = ck.mt.lr, wd = a.mem[ck.mt.member].wd, sc = ck.mt.scale;
+  const T* X = a.ns + ck.mt.x_off[a.x_final];
+  for (int64_t e = ck.e0 + threadIdx.x; e < ck.e1; e += blockDim.x) {
+    const int64_t o = ck.mt.w_off + e;
+    float p = a.params[o];
+    p = p - lr * wd * p;
+    p = p - lr * sc * Elem<T>::to_f(X[ck.xi(e)]);
+    a.params[o] = p;
+    if (a.wq_out) a.wq_out[o] = __float2bfloat16_rn(p);
+  }
+}
+
+template <typename T>
+void launch_muon(cudaStream_t st, const MuonArgs<T>& a, int n_chunks, int phase) {
+  if (n_chunks <= 0) return;
+  if (phase == 0) launch_pdl(k_muon_momentum<T>, dim3(n_chunks), dim3(256), 0, st, a);
+  else if (phase == 1) launch_pdl(k_muon_x0<T>, dim3(n_chunks), dim3(256), 0, st, a);
+  else launch_pdl(k_muon_apply<T>, dim3(n_chunks), dim3(256), 0, st, a);
+}
+
 __global__ void __launch_bounds__(256) k_masks(MaskGen mg) {
   pdl_trigger();
   pdl_wait();
@@ -894,7 +999,8 @@ void launch_debug_masks(cudaStream_t st, uint8_t* out, int B, int w, uint64_t se
   template void launch_fill_ones<T>(cudaStream_t, const OnesJob*, int, T*, T*);                         \
   template void launch_gemm_simt<T>(cudaStream_t, const GemmArgs<T>&, int, int);                       \
   template void launch_head<T>(cudaStream_t, const HeadArgs<T>&, int);                                 \
-  template void launch_predict_head<T>(cudaStream_t, const PredictHeadArgs<T>&, int);
+  template void launch_predict_head<T>(cudaStream_t, const PredictHeadArgs<T>&, int);           \
+  template void launch_muon<T>(cudaStream_t, const MuonArgs<T>&, int, int);
 
 TP_INSTANTIATE(float)
 TP_INSTANTIATE(__nv_bfloat16)

@@ -24,6 +24,23 @@ struct GemmArgs {
   uint64_t seed;
   const StepDyn* dyn;     // non-NULL: take the step from here
   int64_t xb_stride;      // stacked batches: elements between members' batch matrices (0: shared)
+  T* ns;                  // Muon's Newton-Schulz arena (kNs* problems)
+};
+
+// Muon steps around the Newton-Schulz products (see MuonMat).
+template <typename T>
+struct MuonArgs {
+  const MuonMat* mats;
+  const int32_t* chunk_mat;  // flat chunk -> matrix
+  const float* grads;
+  float* mom;                // momentum buffers (the AdamW first-moment arena)
+  float* params;
+  T* ns;
+  double* part;              // per flat chunk: sum of squares of U
+  __nv_bfloat16* wq_out;     // bf16 copy to refresh (NULL in fp32 mode)
+  const MemberDev* mem;
+  float mu;
+  int32_t x_final;           // the X buffer that holds the result
 };
 
 template <typename T>
@@ -111,6 +128,8 @@ void launch_head_reduce(cudaStream_t st, const HeadReduceArgs& g, int m, int max
 void launch_adamw(cudaStream_t st, const AdamArgs& g, int n_chunks);
 void launch_init(cudaStream_t st, const InitArgs& g, int n_chunks);
 void launch_masks(cudaStream_t st, const MaskGen& mg);
+template <typename T>
+void launch_muon(cudaStream_t st, const MuonArgs<T>& a, int n_chunks, int phase);  // 0 momentum, 1 X0, 2 apply
 void launch_refresh_wq(cudaStream_t st, const float* p, __nv_bfloat16* wq0, __nv_bfloat16* wq1, int64_t n);
 template <typename T>
 void launch_fill_ones(cudaStream_t st, const OnesJob* jobs, int n_jobs, T* xb, T* act);

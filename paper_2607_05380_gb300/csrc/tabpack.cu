@@ -81,6 +81,23 @@ struct tabpack {
   int n_p_head = 0;
   bool p_stale = true;      // active set changed since the prediction plan was built
 
+  // Muon for the hidden-layer weights (pack_set_muon): one MuonMat per (member,
+  // hidden layer), its X0, X1, A, Bm in the Newton-Schulz arena `ns` (the
+  // product precision), the flat list of kMuonChunk-element chunks of the
+  // active members' matrices and a sum-of-squares partial per chunk.  The
+  // momentum buffers are the AdamW first-moment arena (AdamW skips these
+  // matrices).
+  bool muon = false;
+  float muon_mu = 0.95f;
+  int ns_steps = 5;
+  std::vector<MuonMat> mmats;
+  void* ns = nullptr;
+  MuonMat* mmats_dev = nullptr;
+  int32_t* mchunk_mat_dev = nullptr;
+  double* mpart_dev = nullptr;
+  int n_muon_chunks = 0;
+  std::pair<int, int> ns_simt_rng[5] = {};  // CUDA-core Newton-Schulz tiles (fp32 mode)
+
   // Stacked batches (Sec. 3.6: a batch per member), built on first use:
   // xbs holds member i's gathered batch at i * xb_elems ([B_cap, ldx] each,
   // its column d_in_pad = 1), and tcs is the tensor-core plan whose layer-0
@@ -363,6 +380,38 @@ tp_status build_schedule(tabpack* h) {
       }
       h->bwd_rng[l] = {base, (int)tiles.size() - base};
     }
+    for (auto& r : h->ns_simt_rng) r = {(int)tiles.size(), 0};
+    if (h->muon)
+      for (int which = 0; which < 5; ++which) {
+        const int base = (int)tiles.size();
+        const int p = which == 0 || which == 3 ? 0 : 1;
+        for (const MuonMat& mt : h->mmats) {
+          if (!h->active[mt.member]) continue;
+          GemmProblem P{};
+          P.member = mt.member; P.layer = mt.layer;
+          P.M = mt.r;
+          P.a_src = kSrcNs; P.b_src = kSrcNs;
+          if (which < 2) {
+            P.kind = kNsGram; P.N = mt.r; P.K = mt.c;
+            P.a_off = P.b_off = mt.x_off[p]; P.lda = P.ldb = mt.c;
+            P.c_off = mt.a_off; P.ldc = mt.r;
+          } else if (which == 2) {
+            P.kind = kNsPoly; P.N = mt.r; P.K = mt.r;
+            P.a_off = P.b_off = mt.a_off; P.lda = P.ldb = mt.r;
+            P.c_off = mt.bm_off; P.ldc = mt.r;
+            P.aux_off = mt.a_off; P.ld_aux = mt.r;
+          } else {
+            P.kind = kNsApply; P.N = mt.c; P.K = mt.r;
+            P.a_off = mt.bm_off; P.lda = mt.r;
+            P.b_off = mt.x_off[p]; P.ldb = mt.c;
+            P.c_off = mt.x_off[1 - p]; P.ldc = mt.c;
+            P.aux_off = mt.x_off[p]; P.ld_aux = mt.c;
+          }
+          probs.push_back(P);
+          add_tiles((int)probs.size() - 1, mt.r, P.N);
+        }
+        h->ns_simt_rng[which] = {base, (int)tiles.size() - base};
+      }
   }
 
   std::vector<HeadJob> hj;
@@ -392,6 +441,7 @@ tp_status build_schedule(tabpack* h) {
   for (int s = 0; s < (int)h->segs.size(); ++s) {
     const Segment& S = h->segs[s];
     if (!h->active[S.member]) continue;
+    if (h->muon && !S.is_bias && S.layer < h->depth[S.member]) continue;  // Muon's
     const int64_t len = S.is_bias ? S.rows : (int64_t)S.rows * S.cols_pad;
     for (int64_t o = 0; o < len; o += 4096)
       ch.push_back(Chunk{S.off + o, (int32_t)std::min<int64_t>(4096, len - o), s});
@@ -409,6 +459,15 @@ tp_status build_schedule(tabpack* h) {
     TP_TRY(dalloc(h, &h->hred_dev, sizeof(HeadReduceJob) * m));
     TP_TRY(dalloc(h, &h->chunks_dev, sizeof(Chunk) * h->cap_chunks));
     TP_TRY(dalloc(h, &h->active_ids_dev, sizeof(int32_t) * m));
+  }
+  // Muon adds Newton-Schulz problems: grow those two lists once
+  if ((int)probs.size() > h->cap_probs) {
+    h->cap_probs = (int)probs.size() + 1;
+    TP_TRY(dalloc(h, &h->probs_dev, sizeof(GemmProblem) * h->cap_probs));
+  }
+  if ((int)tiles.size() > h->cap_tiles) {
+    h->cap_tiles = (int)tiles.size() + 1;
+    TP_TRY(dalloc(h, &h->tiles_dev, sizeof(GemmTile) * h->cap_tiles));
   }
   if ((int)probs.size() > h->cap_probs || (int)tiles.size() > h->cap_tiles || (int)hj.size() > h->cap_head ||
       (int)ch.size() > h->cap_chunks)
@@ -441,6 +500,21 @@ tp_status build_schedule(tabpack* h) {
     }
     h->n_mchunks = (int)mc.size();
   }
+  // Muon: flat chunk list of the active members' matrices
+  h->n_muon_chunks = 0;
+  if (h->muon) {
+    std::vector<int32_t> cm;
+    for (size_t j = 0; j < h->mmats.size(); ++j) {
+      MuonMat& mt = h->mmats[j];
+      mt.chunk0 = (int32_t)cm.size();
+      mt.n_chunks = h->active[mt.member] ? (int32_t)ceil_div((int64_t)mt.rows * mt.cols, kMuonChunk) : 0;
+      for (int k = 0; k < mt.n_chunks; ++k) cm.push_back((int32_t)j);
+    }
+    TP_CUDA(h, cudaMemcpy(h->mmats_dev, h->mmats.data(), sizeof(MuonMat) * h->mmats.size(), cudaMemcpyHostToDevice));
+    if (!cm.empty())
+      TP_CUDA(h, cudaMemcpy(h->mchunk_mat_dev, cm.data(), sizeof(int32_t) * cm.size(), cudaMemcpyHostToDevice));
+    h->n_muon_chunks = (int)cm.size();
+  }
   h->n_head_jobs = (int)hj.size();
   h->n_chunks = (int)ch.size();
   h->p_stale = true;
@@ -464,6 +538,8 @@ tp_status build_schedule(tabpack* h) {
     lay.act = h->act;
     lay.dz = h->dz;
     lay.mask_off = h->mask_words > 0 ? &h->mask_off : nullptr;
+    lay.muon = h->muon ? &h->mmats : nullptr;
+    lay.ns = h->ns;
     TP_TRY(tc_build_plan(h->tc, lay, h->err));
   }
   return TP_OK;
@@ -569,6 +645,12 @@ void free_all(tabpack* h) {
   tc_free_plan(h->tcs);
   if (h->xbs) cudaFree(h->xbs);
   h->xbs = nullptr;
+  for (void* p : {h->ns, (void*)h->mmats_dev, (void*)h->mchunk_mat_dev, (void*)h->mpart_dev})
+    if (p) cudaFree(p);
+  h->ns = nullptr;
+  h->mmats_dev = nullptr;
+  h->mchunk_mat_dev = nullptr;
+  h->mpart_dev = nullptr;
   for (void* p : h->allocs) cudaFree(p);
   h->allocs.clear();
   for (auto e : h->prof.pool) cudaEventDestroy(e);
@@ -594,6 +676,7 @@ GemmArgs<T> gemm_args(tabpack* h, int B, int B_pad, uint32_t step, int train, bo
   g.train = train;
   g.seed = h->cfg.seed;
   g.dyn = nullptr;
+  g.ns = (T*)h->ns;
   return g;
 }
 
@@ -741,6 +824,48 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
       h->launches++;
       prof_end(h, slot, 1, TP_PH_BWD);
     }
+  }
+  if (update && h->muon && h->n_muon_chunks > 0) {
+    // Muon on the hidden-layer weights: momentum and |U|, X0, the
+    // Newton-Schulz iterations, the update (and the bf16 copy for the next step)
+    prof_begin(h, TP_PH_MUON, &slot);
+    MuonArgs<T> ma;
+    ma.mats = h->mmats_dev;
+    ma.chunk_mat = h->mchunk_mat_dev;
+    ma.grads = h->grads;
+    ma.mom = h->adam_m;
+    ma.params = h->params;
+    ma.ns = (T*)h->ns;
+    ma.part = h->mpart_dev;
+    ma.wq_out = wq_next;
+    ma.mem = h->mem_dev;
+    ma.mu = h->muon_mu;
+    ma.x_final = h->ns_steps & 1;
+    int nl = 0;
+    for (int phase = 0; phase < 2; ++phase) {
+      launch_muon<T>(h->st, ma, h->n_muon_chunks, phase);
+      TP_LAUNCHED(h);
+      ++nl;
+    }
+    for (int it = 0; it < h->ns_steps; ++it) {
+      const int p = it & 1;
+      const int which[3] = {p, 2, 3 + p};
+      for (int q = 0; q < 3; ++q) {
+        if (h->bf16) {
+          TP_TRY(tc_run_ns(h->tc, h->st, which[q], h->ns, h->mem_dev, h->err));
+        } else {
+          auto g = gemm_args<T>(h, B, B_pad, step, 0);
+          launch_gemm_simt<T>(h->st, g, h->ns_simt_rng[which[q]].first, h->ns_simt_rng[which[q]].second);
+        }
+        TP_LAUNCHED(h);
+        ++nl;
+      }
+    }
+    launch_muon<T>(h->st, ma, h->n_muon_chunks, 2);
+    TP_LAUNCHED(h);
+    ++nl;
+    h->launches += nl;
+    prof_end(h, slot, nl, TP_PH_MUON);
   }
   if (update && !fused && h->n_chunks > 0) {
     prof_begin(h, TP_PH_ADAMW, &slot);
@@ -1181,6 +1306,82 @@ tp_status pack_forward_backward_stacked(tabpack_t* h, const float* X, int64_t n_
   }
   TP_TRY(ensure_stacked<float>(h));
   return step_entry<float>(h, X, n_rows, idx, y, B, step, loss_out, false, true);
+}
+
+tp_status pack_set_muon(tabpack_t* h, const float* lr_muon, float momentum, int32_t ns_steps) {
+  if (!h || !lr_muon) return fail(h, TP_EINVAL, "null argument");
+  if (!(momentum >= 0.f && momentum < 1.f) || ns_steps < 1 || ns_steps > 32)
+    return fail(h, TP_EINVAL, "momentum must be in [0, 1) and ns_steps in 1..32");
+  for (int i = 0; i < h->cfg.m; ++i)
+    if (!(lr_muon[i] >= 0.f)) return fail(h, TP_EINVAL, "lr_muon[%d] must be >= 0", i);
+  TP_TRY(sync_check(h));
+  const int m = h->cfg.m;
+  if (!h->muon) {
+    // the matrices and their Newton-Schulz buffers (128-element aligned)
+    int64_t off = 0, n_chunks = 0;
+    for (int i = 0; i < m; ++i)
+      for (int l = 0; l < h->depth[i]; ++l) {
+        MuonMat mt{};
+        mt.member = i;
+        mt.layer = l;
+        mt.rows = h->width[i];
+        mt.cols = l == 0 ? h->d_in_pad : h->width[i];
+        const int real_cols = l == 0 ? h->cfg.d_in : h->width[i];
+        mt.tr = mt.rows > mt.cols;
+        mt.r = std::min(mt.rows, mt.cols);
+        mt.c = std::max(mt.rows, mt.cols);
+        mt.w_off = h->W_off[i][l];
+        auto take = [&](int64_t n) { const int64_t o = off; off = round_up(off + n, 128); return o; };
+        mt.x_off[0] = take((int64_t)mt.r * mt.c);
+        mt.x_off[1] = take((int64_t)mt.r * mt.c);
+        mt.a_off = take((int64_t)mt.r * mt.r);
+        mt.bm_off = take((int64_t)mt.r * mt.r);
+        mt.scale = (float)std::sqrt(std::max(1.0, (double)mt.rows / (double)real_cols));
+        n_chunks += ceil_div((int64_t)mt.rows * mt.cols, kMuonChunk);
+        h->mmats.push_back(mt);
+      }
+    TP_CUDA(h, cudaMalloc(&h->ns, h->elem * (size_t)std::max<int64_t>(off, 128)));
+    TP_CUDA(h, cudaMemset(h->ns, 0, h->elem * (size_t)std::max<int64_t>(off, 128)));
+    TP_CUDA(h, cudaMalloc((void**)&h->mmats_dev, sizeof(MuonMat) * h->mmats.size()));
+    TP_CUDA(h, cudaMalloc((void**)&h->mchunk_mat_dev, sizeof(int32_t) * std::max<int64_t>(n_chunks, 1)));
+    TP_CUDA(h, cudaMalloc((void**)&h->mpart_dev, sizeof(double) * std::max<int64_t>(n_chunks, 1)));
+    // Muon's momentum starts at zero in the first-moment arena
+    for (const MuonMat& mt : h->mmats)
+      TP_CUDA(h, cudaMemset(h->adam_m + mt.w_off, 0, sizeof(float) * (size_t)mt.rows * mt.cols));
+  }
+  for (MuonMat& mt : h->mmats) mt.lr = lr_muon[mt.member];
+  h->muon = true;
+  h->muon_mu = momentum;
+  h->ns_steps = ns_steps;
+  h->fuse_adamw = false;   // the weight-gradient epilogue would apply AdamW to Muon's matrices
+  // the tensor-core plan's map table gains the Newton-Schulz buffers
+  tc_free_plan(h->tc);
+  drop_graphs(h);
+  TP_TRY(build_schedule(h));
+  return sync_check(h);
+}
+
+tp_status pack_debug_muon_dir(tabpack_t* h, int32_t member, int32_t layer, float* out) {
+  TP_TRY(check_ml(h, member, layer));
+  if (!h->muon || layer >= h->depth[member] || !out) return fail(h, TP_EINVAL, "no Muon matrix there");
+  TP_TRY(sync_check(h));
+  const MuonMat* mt = nullptr;
+  for (const MuonMat& x : h->mmats)
+    if (x.member == member && x.layer == layer) mt = &x;
+  const int64_t n = (int64_t)mt->r * mt->c;
+  const int xf = h->ns_steps & 1;
+  std::vector<float> X(n);
+  if (h->bf16) {
+    std::vector<__nv_bfloat16> xb(n);
+    TP_CUDA(h, cudaMemcpy(xb.data(), (__nv_bfloat16*)h->ns + mt->x_off[xf], n * 2, cudaMemcpyDeviceToHost));
+    for (int64_t e = 0; e < n; ++e) X[e] = __bfloat162float(xb[e]);
+  } else {
+    TP_CUDA(h, cudaMemcpy(X.data(), (float*)h->ns + mt->x_off[xf], n * 4, cudaMemcpyDeviceToHost));
+  }
+  const int in = layer == 0 ? h->cfg.d_in : h->width[member];
+  for (int i = 0; i < mt->rows; ++i)
+    for (int j = 0; j < in; ++j) out[(int64_t)i * in + j] = X[mt->tr ? (int64_t)j * mt->c + i : (int64_t)i * mt->c + j];
+  return TP_OK;
 }
 
 tp_status pack_predict(tabpack_t* h, const float* X, int64_t N, float* out) {

@@ -118,6 +118,7 @@ struct TcArgs {
   int* err;
   int* cnt;            // row-block completion counters
   int32_t kmaj_off;    // index distance to the same matrix's map with 128-row boxes (K-major loads)
+  __nv_bfloat16* ns;   // Newton-Schulz arena (kNs launches)
 };
 
 // ------------------------------------------------------------ PTX helpers
@@ -321,7 +322,14 @@ __device__ __forceinline__ V pick(const V (&a)[N], int i) {
   return r;
 }
 
-__device__ __forceinline__ bool tile_live(const TcTile& t, int B_pad) { return t.kind == kWgrad || t.m0 < B_pad; }
+__device__ __forceinline__ bool tile_live(const TcTile& t, int B_pad) {
+  return t.kind == kWgrad || t.kind >= kNsGram || t.m0 < B_pad;
+}
+// Operand major-ness of a product kind: A is MN-major only for kWgrad; B is
+// K-major for kFwd, kNsGram and kNsPoly.  Only kFwd and kDgrad read the
+// weight copies (w_shift applies to their B maps).
+__device__ __forceinline__ bool b_kmajor(int kind) { return kind == kFwd || kind == kNsGram || kind == kNsPoly; }
+__device__ __forceinline__ bool reads_weights(int kind) { return kind == kFwd || kind == kDgrad; }
 
 // This CTA's rows of a tile: row block `mi` of the tile (rows m0 .. m0 + 127).
 // Rows beyond the product still load their share of the operands for the
@@ -358,14 +366,16 @@ __device__ __forceinline__ void prefetch_adam_rows(const TcArgs& g, const TcTile
 // Prefetch of the tensor map of a tile's A (which = 0) or B (which = 1)
 // operand, as the producer selects it below.
 __device__ __forceinline__ void prefetch_tile_map(const TcArgs& g, const TcTile& t, int which) {
-  const bool a_k = t.kind != kWgrad, b_k = t.kind == kFwd;
+  const bool a_k = t.kind != kWgrad, b_k = b_kmajor(t.kind);
   const CUtensorMap* m = which == 0 ? g.maps + t.map_a + (a_k ? g.kmaj_off : 0)
-                                    : g.maps + t.map_b + (t.kind == kWgrad ? 0 : g.w_shift) + (b_k ? g.kmaj_off : 0);
+                                    : g.maps + t.map_b + (reads_weights(t.kind) ? g.w_shift : 0) + (b_k ? g.kmaj_off : 0);
   asm volatile("prefetch.tensormap [%0];" ::"l"(m) : "memory");
 }
 
 // ------------------------------------------------------------------ kernel
-template <int kCta>
+// kNs: the Newton-Schulz products of Muon (their own instantiation, so that
+// their epilogue adds nothing to the training products' registers).
+template <int kCta, bool kNs>
 __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
   using G = Geo<kCta>;
   constexpr int kStages = G::kStages;
@@ -438,7 +448,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       // K-major operands (A of kFwd / kDgrad, B of kFwd) load 128-row boxes,
       // MN-major ones 64 x 64 boxes.  This CTA's B: all n_len rows / columns
       // (kCta 1) or its half of them (kCta 2).
-      const bool a_k = tile.kind != kWgrad, b_k = tile.kind == kFwd;
+      const bool a_k = tile.kind != kWgrad, b_k = b_kmajor(tile.kind);
       const int nbA = a_k ? 1 : 2;
       const int nh = tile.n_len / kCta;
       const int bn0 = tile.n0 + rank * nh;
@@ -452,7 +462,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       const bool mine = is_a || qb < nbB;
       const CUtensorMap* map =
           is_a ? g.maps + tile.map_a + (a_k ? g.kmaj_off : 0)
-               : g.maps + tile.map_b + (tile.kind == kWgrad ? 0 : g.w_shift) + (b_k ? g.kmaj_off : 0);
+               : g.maps + tile.map_b + (reads_weights(tile.kind) ? g.w_shift : 0) + (b_k ? g.kmaj_off : 0);
       const bool mn = is_a ? !a_k : !b_k;  // MN-major box: x = row / column, y = k
       const int xy0 = is_a ? u.m0 + 64 * bl : bn0 + (b_k ? 128 : 64) * qb;
       const uint32_t off = is_a ? (uint32_t)bl * kBoxBytes : (uint32_t)kABytes + (uint32_t)qb * boxB;
@@ -519,7 +529,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         if (!mbar_wait(&tl->tempty[acc], acc_phase ^ 1u, abort_flag, g.err, kWaitNs, 5)) break;
         tc_fence_after();
         const uint32_t d = tmem + acc * kAccCols;
-        const int a_mn = tile.kind == kWgrad, b_mn = tile.kind != kFwd;
+        const int a_mn = tile.kind == kWgrad, b_mn = !b_kmajor(tile.kind);
         const uint32_t idesc = instr_desc(128 * kCta, tile.n_len, a_mn, b_mn);
         const uint64_t ta = a_mn ? dA_mn : dA_k, tb = b_mn ? dB_mn : dB_k;
         const uint32_t ka = a_mn ? 2048 >> 4 : 32 >> 4, kb = b_mn ? 2048 >> 4 : 32 >> 4;
@@ -639,7 +649,36 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         const bool live = row_ok && ncols > 0;
         uint32_t v[32];
         tmem_ld32(taddr + c, v);
-        if (tile.kind == kWgrad) {
+        if constexpr (kNs) {
+          // Newton-Schulz: out = alpha acc + beta aux, bf16 (kNsGram: A;
+          // kNsPoly: Bm = c (A A) + b A; kNsApply: X' = (Bm X) + a X)
+          if (!live) continue;
+          const float al = tile.kind == kNsPoly ? kNsC : 1.f;
+          const float be = tile.kind == kNsPoly ? kNsB : (tile.kind == kNsApply ? kNsA : 0.f);
+          __nv_bfloat16* out = g.ns + tile.c_off + (int64_t)r * tile.ldc + col0;
+          const __nv_bfloat16* aux = g.ns + tile.aux_off + (int64_t)r * tile.ld_aux + col0;
+#pragma unroll
+          for (int s = 0; s < 4; ++s) {
+            if (8 * s >= ncols) break;
+            float ax[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) ax[e] = 0.f;
+            if (tile.kind != kNsGram) {
+              const uint4 av = *reinterpret_cast<const uint4*>(aux + 8 * s);
+              const __nv_bfloat16* ab = reinterpret_cast<const __nv_bfloat16*>(&av);
+#pragma unroll
+              for (int e = 0; e < 8; ++e) ax[e] = __bfloat162float(ab[e]);
+            }
+            uint32_t pk[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const int j = 8 * s + 2 * e;
+              pk[e] = pack_bf16x2(al * __uint_as_float(v[j]) + be * ax[2 * e],
+                                  al * __uint_as_float(v[j + 1]) + be * ax[2 * e + 1]);
+            }
+            *reinterpret_cast<uint4*>(out + 8 * s) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          }
+        } else if (tile.kind == kWgrad) {
           // Transpose the warp's 32 rows x 32 columns through shared memory
           // (float4 groups XOR-swizzled by row, so that both the row-wise
           // write and the group-wise read are free of bank conflicts).  Then
@@ -900,6 +939,22 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
           }
       plan.w_shift = ((int)maps.size() - w_base) / 2;
       if (set == 1) plan.kmaj_off = base;
+      // Muon: X0, X1 [r, c] and A, Bm [r, r] of every Muon matrix
+      if (lay.muon && lay.ns) {
+        const __nv_bfloat16* nsb = (const __nv_bfloat16*)lay.ns;
+        if (set == 0) plan.map_ns.assign(lay.muon->size() * 4, -1);
+        for (size_t j = 0; j < lay.muon->size(); ++j) {
+          const MuonMat& mt = (*lay.muon)[j];
+          const int64_t offs[4] = {mt.x_off[0], mt.x_off[1], mt.a_off, mt.bm_off};
+          for (int q = 0; q < 4; ++q) {
+            const int cols = q < 2 ? mt.c : mt.r;
+            if (!encode_map(&mp, nsb + offs[q], cols, mt.r, cols, br, err)) return TP_ECUDA;
+            if (set == 0) plan.map_ns[j * 4 + q] = (int)maps.size();
+            maps.push_back(mp);
+          }
+        }
+        plan.ns_maps = true;
+      }
     }
     plan.n_maps = (int)maps.size();
     if (cudaMalloc(&plan.maps_dev, sizeof(CUtensorMap) * maps.size()) != cudaSuccess) {
@@ -918,9 +973,13 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
     int dev = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&plan.n_sm, cudaDevAttrMultiProcessorCount, dev);
-    if (cudaFuncSetAttribute(k_tc_gemm<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<1>()) !=
+    if (cudaFuncSetAttribute(k_tc_gemm<1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<1>()) !=
             cudaSuccess ||
-        cudaFuncSetAttribute(k_tc_gemm<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<2>()) !=
+        cudaFuncSetAttribute(k_tc_gemm<2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<2>()) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(k_tc_gemm<1, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<1>()) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(k_tc_gemm<2, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<2>()) !=
             cudaSuccess) {
       err = "cudaFuncSetAttribute(smem) failed";
       return TP_ECUDA;
@@ -955,7 +1014,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
       cfg.attrs = attr;
       cfg.numAttrs = 1;
       int n = 0;
-      if (cudaOccupancyMaxActiveClusters(&n, (void*)k_tc_gemm<2>, &cfg) == cudaSuccess && n >= 1) {
+      if (cudaOccupancyMaxActiveClusters(&n, (void*)k_tc_gemm<2, false>, &cfg) == cudaSuccess && n >= 1) {
         plan.max_clusters = n;
       } else {
         cudaGetLastError();
@@ -1121,6 +1180,61 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
     all.insert(all.end(), VW[Lmax - 1].begin(), VW[Lmax - 1].end());
   }
   plan.bwd_rng = {plan.fwd_rng.second, (int)all.size() - plan.fwd_rng.second};
+  // Muon: the Newton-Schulz products of the active members' matrices, one
+  // launch per product kind (and X buffer), costliest tiles first
+  for (auto& r : plan.ns_rng) r = {(int)all.size(), 0};
+  if (lay.muon && plan.ns_maps) {
+    for (int which = 0; which < 5; ++which) {
+      std::vector<TcTile> v;
+      for (size_t j = 0; j < lay.muon->size(); ++j) {
+        const MuonMat& mt = (*lay.muon)[j];
+        if (!active[mt.member]) continue;
+        const int p = which == 0 || which == 3 ? 0 : 1;  // the X buffer read
+        TcTile t{};
+        t.member = mt.member;
+        t.layer = mt.layer;
+        t.m0 = 0;
+        t.m_real = mt.r;
+        t.dep = -1;
+        t.sig = -1;
+        t.mask_off = -1;
+        if (which < 2) {          // A = X X^T
+          t.kind = kNsGram;
+          t.n_real = mt.r;
+          t.k_len = mt.c;
+          t.map_a = t.map_b = plan.map_ns[j * 4 + p];
+          t.c_off = mt.a_off;
+          t.ldc = mt.r;
+        } else if (which == 2) {  // Bm = b A + c A A
+          t.kind = kNsPoly;
+          t.n_real = mt.r;
+          t.k_len = mt.r;
+          t.map_a = t.map_b = plan.map_ns[j * 4 + 2];
+          t.c_off = mt.bm_off;
+          t.ldc = mt.r;
+          t.aux_off = mt.a_off;
+          t.ld_aux = mt.r;
+        } else {                  // X' = a X + Bm X
+          t.kind = kNsApply;
+          t.n_real = mt.c;
+          t.k_len = mt.r;
+          t.map_a = plan.map_ns[j * 4 + 3];
+          t.map_b = plan.map_ns[j * 4 + p];
+          t.c_off = mt.x_off[1 - p];
+          t.ldc = mt.c;
+          t.aux_off = mt.x_off[p];
+          t.ld_aux = mt.c;
+        }
+        split_n(t.n_real, ns, 32);
+        emit(v, t, (int)ceil_div(mt.r, kRowTile), ns);
+      }
+      std::stable_sort(v.begin(), v.end(), [](const TcTile& a, const TcTile& b) {
+        return (int64_t)a.k_len * a.n_len > (int64_t)b.k_len * b.n_len;
+      });
+      plan.ns_rng[which] = {(int)all.size(), (int)v.size()};
+      all.insert(all.end(), v.begin(), v.end());
+    }
+  }
   if ((int)all.size() + 1 > plan.cap_tiles) {
     if (plan.tiles_dev) cudaFree(plan.tiles_dev);
     plan.cap_tiles = (int)all.size() + 1;
@@ -1139,7 +1253,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
 }
 
 static tp_status launch(TcPlan& plan, cudaStream_t st, const std::pair<int, int>& rng, const TcArgs& base,
-                        std::string& err) {
+                        std::string& err, bool ns = false) {
   if (rng.second <= 0) return TP_OK;
   TcArgs a = base;
   a.tiles = plan.tiles_dev + rng.first;
@@ -1165,7 +1279,10 @@ static tp_status launch(TcPlan& plan, cudaStream_t st, const std::pair<int, int>
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = cta == 2 ? 2 : 1;
-  cudaError_t e = cta == 2 ? cudaLaunchKernelEx(&cfg, k_tc_gemm<2>, a) : cudaLaunchKernelEx(&cfg, k_tc_gemm<1>, a);
+  cudaError_t e = ns ? (cta == 2 ? cudaLaunchKernelEx(&cfg, k_tc_gemm<2, true>, a)
+                                 : cudaLaunchKernelEx(&cfg, k_tc_gemm<1, true>, a))
+                     : (cta == 2 ? cudaLaunchKernelEx(&cfg, k_tc_gemm<2, false>, a)
+                                 : cudaLaunchKernelEx(&cfg, k_tc_gemm<1, false>, a));
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) {
     err = std::string("tcgen05 GEMM launch: ") + cudaGetErrorString(e);
@@ -1205,6 +1322,15 @@ tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, 
   return launch(plan, st, plan.bwd_rng, a, err);
 }
 
+tp_status tc_run_ns(TcPlan& plan, cudaStream_t st, int which, void* ns, const MemberDev* mem, std::string& err) {
+  TcArgs a{};
+  a.B = 0;
+  a.B_pad = 0;
+  a.mem = mem;  // the epilogue reads every tile's member record
+  a.ns = (__nv_bfloat16*)ns;
+  return launch(plan, st, plan.ns_rng[which], a, err, true);
+}
+
 tp_status tc_check(TcPlan& plan, cudaStream_t st, std::string& err) {
   if (!plan.err_dev) return TP_OK;
   int v = 0;
@@ -1230,8 +1356,11 @@ void tc_free_plan(TcPlan& plan) {
   plan.n_cnt = 0;
   plan.maps_dev = nullptr;
   plan.tiles_dev = nullptr;
+  plan.cap_tiles = 0;
   plan.err_dev = nullptr;
   plan.enabled = false;
+  plan.ns_maps = false;
+  plan.map_ns.clear();
 }
 
 }  // namespace tp

@@ -51,6 +51,10 @@ struct TcPlan {
   TcTile* tiles_dev = nullptr;
   int cap_tiles = 0;
   std::pair<int, int> fwd_rng, bwd_rng;  // tile ranges of the forward / backward launch
+  // Newton-Schulz launches: kNsGram reading X0 / X1, kNsPoly, kNsApply
+  // reading X0 / X1 (writing the other)
+  std::pair<int, int> ns_rng[5] = {};
+  bool ns_maps = false;    // the map table holds the Muon matrices' maps
   // Row-block completion counters: act of (member, layer) then dz of
   // (member, layer), B_cap / 128 each.  They must be zero before a launch
   // (the gather kernel that precedes every forward clears them).
@@ -60,6 +64,7 @@ struct TcPlan {
   int max_clusters = 0;    // tiles in flight at once (resident CTAs / cta)
   int* err_dev = nullptr;  // device error word (bounded waits that gave up)
   std::vector<int> map_act, map_dz, map_w;  // per (member * kMaxDepth + layer)
+  std::vector<int> map_ns;                  // per Muon matrix: X0, X1, A, Bm
 };
 
 struct TcLayout {          // what the plan needs to know about the pack's arenas
@@ -76,6 +81,10 @@ struct TcLayout {          // what the plan needs to know about the pack's arena
   const void* act;
   const void* dz;
   bool fwd_only = false;   // forward tiles only (prediction): no dz maps, counters or backward tiles
+  // Muon: the matrices whose Newton-Schulz products get tiles (NULL: none)
+  // and the bf16 arena holding their X, A and Bm buffers
+  const std::vector<MuonMat>* muon = nullptr;
+  const void* ns = nullptr;
   int64_t xb_stride = 0;   // > 0: a batch matrix per member (stacked batches), this many elements apart
   // per (member, layer): word offset of the dropout keep words, -1 for none (NULL: no masks)
   const std::vector<std::array<int64_t, kMaxDepth>>* mask_off = nullptr;
@@ -93,6 +102,9 @@ tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, 
 // weight copy).
 tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, const MemberDev* mem, void* act,
                      void* dz, float* grads, int update, const AdamDev& adam, std::string& err);
+// One Newton-Schulz product launch over every Muon matrix: which = 0 / 1
+// kNsGram of X0 / X1, 2 kNsPoly, 3 / 4 kNsApply of X0 / X1.
+tp_status tc_run_ns(TcPlan& plan, cudaStream_t st, int which, void* ns, const MemberDev* mem, std::string& err);
 // Reads and clears the device error word (synchronises the stream).
 tp_status tc_check(TcPlan& plan, cudaStream_t st, std::string& err);
 void tc_free_plan(TcPlan& plan);

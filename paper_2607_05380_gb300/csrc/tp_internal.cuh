@@ -34,8 +34,30 @@ constexpr int kHeadRows = 64;   // batch rows per head-kernel block
 constexpr int kSegAlign = 32;   // elements
 constexpr int kOnesCols = 16;   // the ones column plus zero padding to 16 columns
 
-enum GemmKind : int32_t { kFwd = 0, kDgrad = 1, kWgrad = 2 };
-enum Src : int32_t { kSrcXb = 0, kSrcAct = 1, kSrcDz = 2, kSrcWq = 3 };
+enum GemmKind : int32_t { kFwd = 0, kDgrad = 1, kWgrad = 2, kNsGram = 3, kNsPoly = 4, kNsApply = 5 };
+enum Src : int32_t { kSrcXb = 0, kSrcAct = 1, kSrcDz = 2, kSrcWq = 3, kSrcNs = 4 };
+
+// Muon (Sec. 3.4; Jordan et al. 2024) on the hidden-layer weight matrices:
+// the products of one Newton-Schulz iteration over the normalised momentum
+// X [r, c] (r <= c; the transposed gradient when W has more rows than
+// columns), all members and layers at once:
+//   kNsGram  A  = X X^T            (A, B operands: X, K-major)
+//   kNsPoly  Bm = b A + c A A      (A, B operands: A, K-major; A symmetric)
+//   kNsApply X' = a X + Bm X       (A: Bm K-major, B: X MN-major)
+// Coefficients (a, b, c) = (3.4445, -4.7750, 2.0315).
+constexpr float kNsA = 3.4445f, kNsB = -4.7750f, kNsC = 2.0315f;
+
+struct MuonMat {          // one Muon matrix: W_l of a member, [rows, cols] in the arena
+  int64_t w_off;          // weight block offset in the parameter arena (pitch cols)
+  int64_t x_off[2];       // X ping-pong buffers [r, c] in the Newton-Schulz arena
+  int64_t a_off, bm_off;  // A and Bm [r, r]
+  int32_t member, layer;
+  int32_t rows, cols;     // w and in_pad
+  int32_t r, c, tr;       // tr = 1: X = U^T (rows > cols)
+  float scale, lr;        // max(1, rows / real columns)^(1/2); the member's Muon lr
+  int32_t chunk0, n_chunks;  // its element chunks (of kMuonChunk) in the flat list
+};
+constexpr int kMuonChunk = 4096;
 
 // One matrix product of one member and layer (CUDA-core path).
 // Output C[r, c] = sum_k A(r, k) B(c, k).
