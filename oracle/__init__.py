@@ -25,9 +25,9 @@ _HDR = os.path.join(_HERE, "tabpack_oracle.h")
 LIB_PATH = os.path.join(_HERE, "liboracle.so")
 
 BINARY, MULTICLASS, REGRESSION = 0, 1, 2
-SCORE_LOSS, SCORE_ACCURACY, SCORE_RMSE = 0, 1, 2
+SCORE_LOSS, SCORE_ACCURACY, SCORE_RMSE, SCORE_AUC = 0, 1, 2, 3
 TASKS = {"binary": BINARY, "multiclass": MULTICLASS, "regression": REGRESSION}
-SCORES = {"loss": SCORE_LOSS, "accuracy": SCORE_ACCURACY, "rmse": SCORE_RMSE}
+SCORES = {"loss": SCORE_LOSS, "accuracy": SCORE_ACCURACY, "rmse": SCORE_RMSE, "auc": SCORE_AUC}
 
 _lock = threading.Lock()
 _lib = None
@@ -74,6 +74,7 @@ def lib():
                 "orc_train_step": (ctypes.c_int, [P, P, i64, P, P, P, i32, u32, i32, P]),
                 "orc_train_step_stacked": (ctypes.c_int, [P, P, i64, P, P, P, i32, u32, i32, P]),
                 "orc_set_muon": (ctypes.c_int, [P, P, ctypes.c_double, i32]),
+                "orc_auc": (ctypes.c_double, [P, P, i64]),
                 "orc_newton_schulz": (None, [P, i32, i32, i32, i32, P]),
                 "orc_get_muon_dir": (ctypes.c_int, [P, i32, i32, P]),
                 "orc_predict": (ctypes.c_int, [P, P, i64, P]),
@@ -277,6 +278,13 @@ class OraclePack:
 
     def member_steps(self, member):
         return int(lib().orc_member_steps(self._h, member))
+
+
+def auc(e, y):
+    """ROC-AUC of scores e for 0/1 labels y (ranked in fp32, midranks for ties)."""
+    e = np.ascontiguousarray(e, dtype=np.float64)
+    y = np.ascontiguousarray(y, dtype=np.int32)
+    return float(lib().orc_auc(_ptr(e), _ptr(y), len(e)))
 
 
 def newton_schulz(U, steps=5, bf16=False):

@@ -721,8 +721,42 @@ int64_t orc_member_steps(const orc_pack* h, int32_t member) {
 #define ORC_CLIP_HI (1.0 - 1e-7)
 
 /* plain fp64 score of the ensemble whose row predictions are ens[N, d_out] */
+typedef struct { float key; int32_t y; } orc_ranked;
+static int orc_cmp_ranked(const void* a, const void* b) {
+  const float x = ((const orc_ranked*)a)->key, z = ((const orc_ranked*)b)->key;
+  return x < z ? -1 : (x > z ? 1 : 0);
+}
+
+double orc_auc(const double* e, const int32_t* y, int64_t N) {
+  orc_ranked* v = (orc_ranked*)malloc(sizeof(orc_ranked) * (size_t)(N > 0 ? N : 1));
+  int64_t n_pos = 0;
+  for (int64_t b = 0; b < N; ++b) {
+    v[b].key = (float)e[b];
+    v[b].y = y[b] == 1;
+    n_pos += v[b].y;
+  }
+  const int64_t n_neg = N - n_pos;
+  if (n_pos == 0 || n_neg == 0) {
+    free(v);
+    return NAN;
+  }
+  qsort(v, (size_t)N, sizeof(orc_ranked), orc_cmp_ranked);
+  double rank_sum = 0.0;  /* ranks 1..N; a tie group [i, j) shares (i + 1 + j) / 2 */
+  for (int64_t i = 0; i < N;) {
+    int64_t j = i + 1;
+    while (j < N && v[j].key == v[i].key) ++j;
+    int64_t pos = 0;
+    for (int64_t k = i; k < j; ++k) pos += v[k].y;
+    rank_sum += (double)pos * 0.5 * (double)(i + 1 + j);
+    i = j;
+  }
+  free(v);
+  return (rank_sum - 0.5 * (double)n_pos * (double)(n_pos + 1)) / ((double)n_pos * (double)n_neg);
+}
+
 static double orc_score_rows(const double* ens, int64_t N, int32_t d_out, const int32_t* y_int,
                              const float* y_float, int32_t task, int32_t score) {
+  if (score == ORC_SCORE_AUC) return -orc_auc(ens, y_int, N);
   double acc = 0.0;
   for (int64_t b = 0; b < N; ++b) {
     const double* e = &ens[b * d_out];
@@ -758,6 +792,13 @@ static double orc_score_rows(const double* ens, int64_t N, int32_t d_out, const 
 static double orc_score_fp32_terms(const double* S, const float* p, int32_t n, int64_t N, int32_t d_out,
                                    const int32_t* y_int, const float* y_float, int32_t task, int32_t score) {
   const double inv = 1.0 / (double)(n + 1);
+  if (score == ORC_SCORE_AUC) {  /* the fp64 ensemble values; orc_auc ranks them in fp32 */
+    double* e = orc_zeros(N);
+    for (int64_t b = 0; b < N; ++b) e[b] = (S[b] + (double)p[b]) * inv;
+    const double r = -orc_auc(e, y_int, N);
+    free(e);
+    return r;
+  }
   double acc = 0.0;
   for (int64_t b = 0; b < N; ++b) {
     const double* s = &S[b * d_out];
@@ -794,7 +835,8 @@ static double orc_score_fp32_terms(const double* S, const float* p, int32_t n, i
 }
 
 static int orc_score_valid(int32_t task, int32_t score, int32_t d_out) {
-  if (score < 0 || score > 2) return 0;
+  if (score < 0 || score > 3) return 0;
+  if (score == ORC_SCORE_AUC && task != ORC_BINARY) return 0;
   if (score == ORC_SCORE_ACCURACY && task == ORC_REGRESSION) return 0;
   if (score == ORC_SCORE_RMSE && task != ORC_REGRESSION) return 0;
   if (task != ORC_MULTICLASS && d_out != 1) return 0;

@@ -46,7 +46,15 @@ extern "C" {
 #endif
 
 enum { ORC_BINARY = 0, ORC_MULTICLASS = 1, ORC_REGRESSION = 2 };
-enum { ORC_SCORE_LOSS = 0, ORC_SCORE_ACCURACY = 1, ORC_SCORE_RMSE = 2 };
+enum { ORC_SCORE_LOSS = 0, ORC_SCORE_ACCURACY = 1, ORC_SCORE_RMSE = 2, ORC_SCORE_AUC = 3 };
+
+/* ROC-AUC of scores e [N] (probability of class 1) for labels y [N] (0 / 1):
+ * the scores are rounded to fp32 (the decision precision of the GPU scorer)
+ * and ranked, tied scores sharing the mean of their ranks; AUC = (sum of the
+ * positives' ranks - n_pos (n_pos + 1) / 2) / (n_pos n_neg) (Mann-Whitney).
+ * NaN when one class is absent.  As an ensemble score (ORC_SCORE_AUC,
+ * binary tasks) the greedy selection minimises -AUC.                        */
+double orc_auc(const double* e, const int32_t* y, int64_t N);
 
 typedef struct {
   int32_t m;            /* number of base models in the pack (the paper's m) */

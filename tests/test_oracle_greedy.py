@@ -20,6 +20,11 @@ GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
 def np_score(preds, subset, y, task, score):
     """Independent scorer: mean of the subset's predictions, then the metric."""
     ens = np.mean([preds[c].astype(np.float64) for c in subset], axis=0)
+    if score == "auc":   # Mann-Whitney by pairs, on the fp32-rounded scores
+        s32 = ens[:, 0].astype(np.float32)
+        pos, neg = s32[y == 1], s32[y == 0]
+        gt = (pos[:, None] > neg[None, :]).sum() + 0.5 * (pos[:, None] == neg[None, :]).sum()
+        return -gt / (len(pos) * len(neg))
     if score == "accuracy":
         pred = np.argmax(ens, axis=1) if task == "multiclass" else (ens[:, 0] > 0.5).astype(int)
         return -np.mean(pred == y)
@@ -49,7 +54,7 @@ def make_pool(task, P, N, C, seed):
 
 
 CASES = [("multiclass", "loss"), ("multiclass", "accuracy"), ("binary", "loss"),
-         ("binary", "accuracy"), ("regression", "loss"), ("regression", "rmse")]
+         ("binary", "accuracy"), ("binary", "auc"), ("regression", "loss"), ("regression", "rmse")]
 
 
 def test_worked_example(orc):
