@@ -149,7 +149,7 @@ def predict_flops(wl, hp, n_rows):
 
 
 def time_online_epoch(tp, torch, pack, wl, hp, d, X, y, idx_all, stream, loss, n_epochs=6, steps_between=8,
-                      m_ens=32, p_base=16, p_ens=32):
+                      m_ens=32, p_base=16, p_ens=32, score="loss"):
     """Wall time of the online ensemble's epoch end (Sec. 3.5: predict the
     members on the validation rows, greedy selection over the pool, member
     snapshots, patience bookkeeping) on the workload's full validation set,
@@ -157,7 +157,7 @@ def time_online_epoch(tp, torch, pack, wl, hp, d, X, y, idx_all, stream, loss, n
     call synchronises, so it is timed on the host around a synchronised
     stream; the prediction share comes from the pack's CUDA-event profile."""
     X_val, y_val = d["X_val"], d["y_val"]
-    on = tp.OnlineEnsemble(pack, X_val.shape[0], "loss", m_ens, p_base, p_ens)
+    on = tp.OnlineEnsemble(pack, X_val.shape[0], score, m_ens, p_base, p_ens)
     B = wl.batch
     times, pred_ms = [], []
     s_next = 50_000
@@ -184,7 +184,7 @@ def time_online_epoch(tp, torch, pack, wl, hp, d, X, y, idx_all, stream, loss, n
     n_val = int(X_val.shape[0])
     pool = info["n_pool"]
     sel_bytes = m_ens * pool * n_val * wl.d_out * 4.0
-    return {"ms": ms, "predict_ms": pm, "select_and_rest_ms": ms - pm, "n_val": n_val, "m_ens": m_ens,
+    return {"ms": ms, "predict_ms": pm, "select_and_rest_ms": ms - pm, "n_val": n_val, "m_ens": m_ens, "score": score,
             "pool": pool, "n_best": info["n_best"], "epochs_timed": len(times),
             "predict_tflops": predict_flops(wl, hp, n_val) / (pm / 1e3) / 1e12,
             "select_candidate_bytes": sel_bytes,
@@ -267,6 +267,8 @@ def main():
                     help="train only the first N members of the workload (profiling small cases)")
     ap.add_argument("--fuse-optimizer", action="store_true", help="AdamW inside the weight-gradient epilogue")
     ap.add_argument("--no-online", action="store_true", help="skip timing the online-ensemble epoch end")
+    ap.add_argument("--online-score", default="loss", choices=["loss", "accuracy", "rmse", "auc"],
+                    help="ensemble score of the timed online epoch end (auc: binary workloads)")
     ap.add_argument("--muon", action="store_true",
                     help="Muon for the hidden-layer weights (the paper's default optimizer), AdamW for the rest")
     ap.add_argument("--stacked", action="store_true",
@@ -435,7 +437,8 @@ def main():
                "h2d_bytes_per_step": n_rows_step * (wl.d_in * 4 + 4), "d2h_bytes_per_step": wl.m * 4,
                "steps": n_e2e}
 
-    online = None if args.no_online else time_online_epoch(tp, torch, pack, wl, hp, d, X, y, idx_all, stream, loss)
+    online = None if args.no_online else time_online_epoch(tp, torch, pack, wl, hp, d, X, y, idx_all, stream, loss,
+                                                           score=args.online_score)
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:

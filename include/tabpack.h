@@ -54,7 +54,7 @@ typedef enum {
 
 typedef enum { TP_BINARY = 0, TP_MULTICLASS = 1, TP_REGRESSION = 2 } tp_task;
 typedef enum { TP_BF16 = 0, TP_FP32 = 1 } tp_precision;
-typedef enum { TP_SCORE_LOSS = 0, TP_SCORE_ACCURACY = 1, TP_SCORE_RMSE = 2 } tp_score;
+typedef enum { TP_SCORE_LOSS = 0, TP_SCORE_ACCURACY = 1, TP_SCORE_RMSE = 2, TP_SCORE_AUC = 3 } tp_score;
 
 typedef struct {
   int32_t m;          /* number of base models in the pack, >= 1                        */
@@ -175,8 +175,12 @@ tp_status pack_predict(tabpack_t* pack, const float* X, int64_t N, float* out);
  * candidate index.  Scores (lower is better): TP_SCORE_LOSS = mean CE / BCE
  * of the averaged probabilities clipped to [1e-7, 1 - 1e-7], or MSE;
  * TP_SCORE_ACCURACY = minus the accuracy (classification);
- * TP_SCORE_RMSE = root MSE (regression).  Per-row terms are taken in fp32
- * and summed in fp64 in a fixed order; the running ensemble sum is fp64.
+ * TP_SCORE_RMSE = root MSE (regression); TP_SCORE_AUC = minus the ROC-AUC
+ * (binary): the ensemble's scores rounded to fp32 are ranked (stable radix
+ * sort on the device), tied scores share their mean rank, and AUC = (sum of
+ * the positives' ranks - n_pos (n_pos + 1) / 2) / (n_pos n_neg) (NaN, never
+ * selected, when a class is absent).  Per-row terms are taken in fp32 and
+ * summed in fp64 in a fixed order; the running ensemble sum is fp64.
  *   preds: device float32 [P, N, d_out] (probabilities or values as written
  *   by pack_predict);  y: device labels [N];  cuda_stream: stream to run on;
  *   selected: host int32 [m_ens] receives the selection order;

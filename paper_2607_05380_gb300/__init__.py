@@ -20,10 +20,10 @@ LIB_PATH = _build.LIB
 TP_OK, TP_EINVAL, TP_ENOMEM, TP_ECUDA, TP_ESTATE, TP_ETIMEOUT, TP_ENOTSUP = range(7)
 BINARY, MULTICLASS, REGRESSION = 0, 1, 2
 BF16, FP32 = 0, 1
-SCORE_LOSS, SCORE_ACCURACY, SCORE_RMSE = 0, 1, 2
+SCORE_LOSS, SCORE_ACCURACY, SCORE_RMSE, SCORE_AUC = 0, 1, 2, 3
 TASKS = {"binary": BINARY, "multiclass": MULTICLASS, "regression": REGRESSION}
 PRECISIONS = {"bf16": BF16, "fp32": FP32}
-SCORES = {"loss": SCORE_LOSS, "accuracy": SCORE_ACCURACY, "rmse": SCORE_RMSE}
+SCORES = {"loss": SCORE_LOSS, "accuracy": SCORE_ACCURACY, "rmse": SCORE_RMSE, "auc": SCORE_AUC}
 PHASES = ["gather", "fwd", "head", "bwd", "bias", "adamw", "predict", "muon"]
 
 # every entry point declared in include/tabpack.h

@@ -147,9 +147,12 @@ struct SelectScratch {
   double* partial;        // [P, n_blk]
   int32_t* state;         // [4 + m_ens + P]: n, done, last, pad | selected | used
   double* cur;            // [1]: current score
+  uint32_t* keys;         // ROC-AUC score: sort keys, two buffers of N per candidate
+  uint8_t* lab;           // and their labels
 };
-int64_t select_scratch_bytes(int32_t P, int64_t N, int32_t d_out, int32_t m_ens);
-SelectScratch select_carve(void* base, int32_t P, int64_t N, int32_t d_out, int32_t m_ens);
+// score: scratch for the ROC-AUC score's sorts only when score == TP_SCORE_AUC
+int64_t select_scratch_bytes(int32_t P, int64_t N, int32_t d_out, int32_t m_ens, int32_t score);
+SelectScratch select_carve(void* base, int32_t P, int64_t N, int32_t d_out, int32_t m_ens, int32_t score);
 // excl: device uint8 [P] or NULL; candidates with excl[c] != 0 take no part.
 // solo: device double [P] or NULL; receives every candidate's score on its
 // own (the first iteration's values; NaN for excluded candidates).

@@ -158,7 +158,8 @@ tp_status pack_online_create(tabpack_t* pack, int64_t n_val, int32_t score, int3
   if (pack_get_config(pack, &cfg) != TP_OK) return ofail(nullptr, TP_EINVAL, "bad pack");
   if (n_val < 1 || m_ens < 1 || p_base < 0 || p_ens < 0)
     return ofail(nullptr, TP_EINVAL, "n_val, m_ens must be >= 1 and p_base, p_ens >= 0");
-  if (score < 0 || score > 2) return ofail(nullptr, TP_EINVAL, "unknown score %d", score);
+  if (score < 0 || score > 3) return ofail(nullptr, TP_EINVAL, "unknown score %d", score);
+  if (score == TP_SCORE_AUC && cfg.task != TP_BINARY) return ofail(nullptr, TP_EINVAL, "auc needs a binary task");
   if (score == TP_SCORE_ACCURACY && cfg.task == TP_REGRESSION) return ofail(nullptr, TP_EINVAL, "accuracy needs classification");
   if (score == TP_SCORE_RMSE && cfg.task != TP_REGRESSION) return ofail(nullptr, TP_EINVAL, "rmse needs regression");
   const int64_t P_max = (int64_t)cfg.m + m_ens;
@@ -195,7 +196,7 @@ tp_status pack_online_create(tabpack_t* pack, int64_t n_val, int32_t score, int3
   tp_status s = alloc((void**)&o->pool, (size_t)(P_max * o->row_elems) * 4);
   if (s == TP_OK) s = alloc((void**)&o->tmp, (size_t)((int64_t)m_ens * o->row_elems) * 4);
   if (s == TP_OK) s = alloc((void**)&o->slots, (size_t)((int64_t)o->n_slots * o->slot_elems) * 4);
-  if (s == TP_OK) s = alloc(&o->scratch, (size_t)select_scratch_bytes((int32_t)P_max, n_val, cfg.d_out, m_ens));
+  if (s == TP_OK) s = alloc(&o->scratch, (size_t)select_scratch_bytes((int32_t)P_max, n_val, cfg.d_out, m_ens, score));
   if (s == TP_OK) s = alloc((void**)&o->excl_dev, (size_t)P_max);
   if (s == TP_OK) s = alloc((void**)&o->solo_dev, (size_t)P_max * 8);
   if (s != TP_OK) {
@@ -239,7 +240,7 @@ tp_status pack_online_epoch(tabpack_online_t* o, const float* X_val, const void*
   }
   O_CUDA(o, cudaMemcpyAsync(o->excl_dev, excl.data(), (size_t)P, cudaMemcpyHostToDevice, st));
   // 3. greedy selection, with every candidate's own score on the side
-  SelectScratch ss = select_carve(o->scratch, P, o->n_val, o->cfg.d_out, o->m_ens);
+  SelectScratch ss = select_carve(o->scratch, P, o->n_val, o->cfg.d_out, o->m_ens, o->score);
   const int n_words = select_enqueue(st, ss, o->pool, P, o->n_val, o->cfg.d_out, y_val, o->cfg.task, o->score,
                                      o->m_ens, o->excl_dev, o->solo_dev, nullptr);
   O_CUDA(o, cudaGetLastError());

@@ -16,6 +16,8 @@ constexpr int kSelRowsPerThread = 4;
 constexpr int kSelRowsPerBlock = kSelThreads * kSelRowsPerThread;
 
 enum { kStN = 0, kStDone = 1, kStLast = 2, kStHdr = 4 };
+constexpr int kScoreAuc = 3;      // TP_SCORE_AUC
+constexpr int kAucThreads = 1024;
 
 __device__ __forceinline__ double warp_sum_d(double v) {
 #pragma unroll
@@ -99,9 +101,11 @@ __global__ void __launch_bounds__(kSelThreads) k_sel_score(const double* __restr
 }
 
 // Score of candidate c from its per-block partial sums: blocks in index
-// order, then the mean over N rows and the score's transform.
+// order, then the mean over N rows and the score's transform (the ROC-AUC
+// kernel writes the candidate's score itself, -AUC, as its first partial).
 __device__ __forceinline__ double cand_score(const double* __restrict__ partial, int c, int32_t n_blk, int64_t N,
                                              int32_t score) {
+  if (score == kScoreAuc) return partial[(int64_t)c * n_blk];
   double s = 0.0;
   for (int b = 0; b < n_blk; ++b) s += partial[(int64_t)c * n_blk + b];
   const double mean = s / (double)N;
@@ -115,6 +119,142 @@ __global__ void k_sel_solo(const double* __restrict__ partial, int32_t P, int32_
   if (c >= P) return;
   const int32_t* used = state + kStHdr + m_ens;
   solo[c] = used[c] ? __longlong_as_double(0x7ff8000000000000LL) : cand_score(partial, c, n_blk, N, score);
+}
+
+// ROC-AUC score of candidate c (one block per candidate): the ensemble's
+// scores (S + p_c) / (n + 1), rounded to fp32, sorted with their labels by a
+// stable 4-pass radix sort of order-preserving keys (8-bit digits; within a
+// 1024-key tile a key's place among equal digits comes from its warp's
+// match mask and the warps before it), then each positive's mid-rank among
+// equal scores by binary search: AUC = (sum of the positives' ranks -
+// n_pos (n_pos + 1) / 2) / (n_pos n_neg).  Rank sums are half-integers, exact
+// in fp64, so the result does not depend on the order of the sum.
+__global__ void __launch_bounds__(kAucThreads) k_sel_auc(const double* __restrict__ S,
+                                                         const float* __restrict__ preds,
+                                                         const int32_t* __restrict__ y, int64_t N,
+                                                         const int32_t* __restrict__ state,
+                                                         double* __restrict__ partial, int32_t n_blk,
+                                                         int32_t m_ens, uint32_t* __restrict__ keys,
+                                                         uint8_t* __restrict__ lab) {
+  const int c = blockIdx.x;
+  const int32_t* used = state + kStHdr + m_ens;
+  if (state[kStDone] || used[c]) return;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const double inv = 1.0 / (double)(state[kStN] + 1);
+  const float* p = preds + (int64_t)c * N;
+  uint32_t* const k0 = keys + (int64_t)(2 * c) * N;
+  uint32_t* const k1 = k0 + N;
+  uint8_t* const l0 = lab + (int64_t)(2 * c) * N;
+  uint8_t* const l1 = l0 + N;
+  for (int64_t b = tid; b < N; b += kAucThreads) {
+    const float f = (float)((S[b] + (double)p[b]) * inv);
+    const uint32_t u = __float_as_uint(f);
+    k0[b] = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+    l0[b] = y[b] == 1 ? 1 : 0;
+  }
+  __shared__ uint32_t hist[256], base[256], tot[256];
+  __shared__ uint32_t wcnt[kAucThreads / 32][256];
+  for (int e = tid; e < (kAucThreads / 32) * 256; e += kAucThreads) (&wcnt[0][0])[e] = 0;
+  __syncthreads();
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 8 * pass;
+    const bool odd = pass & 1;
+    const uint32_t* src = odd ? k1 : k0;
+    const uint8_t* srcl = odd ? l1 : l0;
+    uint32_t* dst = odd ? k0 : k1;
+    uint8_t* dstl = odd ? l0 : l1;
+    if (tid < 256) hist[tid] = 0;
+    __syncthreads();
+    for (int64_t b = tid; b < N; b += kAucThreads) atomicAdd(&hist[(src[b] >> shift) & 255u], 1u);
+    __syncthreads();
+    if (tid == 0) {
+      uint32_t run = 0;
+      for (int d = 0; d < 256; ++d) {
+        base[d] = run;
+        run += hist[d];
+      }
+    }
+    __syncthreads();
+    for (int64_t t0 = 0; t0 < N; t0 += kAucThreads) {
+      const int64_t b = t0 + tid;
+      const bool valid = b < N;
+      const uint32_t key = valid ? src[b] : 0u;
+      const uint8_t l = valid ? srcl[b] : 0;
+      const int d = valid ? (int)((key >> shift) & 255u) : 256;
+      const uint32_t peers = __match_any_sync(0xffffffffu, d);
+      const int rank = __popc(peers & ((1u << lane) - 1u));
+      if (valid && rank == 0) wcnt[warp][d] = __popc(peers);
+      __syncthreads();
+      if (tid < 256) {   // per digit: exclusive prefix over warps, then the tile's total
+        uint32_t run = 0;
+        for (int w = 0; w < kAucThreads / 32; ++w) {
+          const uint32_t v = wcnt[w][tid];
+          wcnt[w][tid] = run;
+          run += v;
+        }
+        tot[tid] = run;
+      }
+      __syncthreads();
+      if (valid) {
+        const uint32_t off = base[d] + wcnt[warp][d] + (uint32_t)rank;
+        dst[off] = key;
+        dstl[off] = l;
+      }
+      __syncthreads();
+      if (tid < 256) {
+        base[tid] += tot[tid];
+        for (int w = 0; w < kAucThreads / 32; ++w) wcnt[w][tid] = 0;
+      }
+      __syncthreads();
+    }
+  }
+  // sorted: k0, l0 (four passes).  Mid-ranks of the positives.
+  const uint32_t* sk = k0;
+  const uint8_t* sl = l0;
+  double rs = 0.0;
+  int64_t np = 0;
+  for (int64_t i = tid; i < N; i += kAucThreads) {
+    if (!sl[i]) continue;
+    const uint32_t key = sk[i];
+    int64_t lo = 0, hi = i;              // first index with this key
+    while (lo < hi) {
+      const int64_t mid = (lo + hi) >> 1;
+      if (sk[mid] < key) lo = mid + 1; else hi = mid;
+    }
+    const int64_t first = lo;
+    lo = i + 1;
+    hi = N;                              // one past the last index with this key
+    while (lo < hi) {
+      const int64_t mid = (lo + hi) >> 1;
+      if (sk[mid] <= key) lo = mid + 1; else hi = mid;
+    }
+    rs += 0.5 * (double)(first + 1 + lo);
+    ++np;
+  }
+  __shared__ double rsum[kAucThreads / 32];
+  __shared__ long long pcnt[kAucThreads / 32];
+  for (int o = 16; o > 0; o >>= 1) {
+    rs += __shfl_xor_sync(0xffffffffu, rs, o);
+    np += __shfl_xor_sync(0xffffffffu, np, o);
+  }
+  if (lane == 0) {
+    rsum[warp] = rs;
+    pcnt[warp] = np;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    double r = 0.0;
+    long long n_pos = 0;
+    for (int w = 0; w < kAucThreads / 32; ++w) {
+      r += rsum[w];
+      n_pos += pcnt[w];
+    }
+    const long long n_neg = (long long)N - n_pos;
+    double auc = __longlong_as_double(0x7ff8000000000000LL);
+    if (n_pos > 0 && n_neg > 0)
+      auc = (r - 0.5 * (double)n_pos * (double)(n_pos + 1)) / ((double)n_pos * (double)n_neg);
+    partial[(int64_t)c * n_blk] = -auc;
+  }
 }
 
 __global__ void __launch_bounds__(1024) k_sel_pick(const double* __restrict__ partial, int32_t P, int32_t n_blk,
@@ -177,14 +317,15 @@ __global__ void k_sel_add(double* __restrict__ S, const float* __restrict__ pred
     S[e] += (double)p[e];
 }
 
-int64_t select_scratch_bytes(int32_t P, int64_t N, int32_t d_out, int32_t m_ens) {
+int64_t select_scratch_bytes(int32_t P, int64_t N, int32_t d_out, int32_t m_ens, int32_t score) {
   const int64_t n_blk = ceil_div(N, kSelRowsPerBlock);
   int64_t bytes = round_up(N * d_out * 8, 256) + round_up((int64_t)P * n_blk * 8, 256) + 256 +
                   round_up((int64_t)(kStHdr + m_ens + P) * 4, 256);
+  if (score == kScoreAuc) bytes += round_up((int64_t)P * 2 * N * 4, 256) + round_up((int64_t)P * 2 * N, 256);
   return bytes;
 }
 
-SelectScratch select_carve(void* base, int32_t P, int64_t N, int32_t d_out, int32_t m_ens) {
+SelectScratch select_carve(void* base, int32_t P, int64_t N, int32_t d_out, int32_t m_ens, int32_t score) {
   const int64_t n_blk = ceil_div(N, kSelRowsPerBlock);
   char* p = (char*)base;
   SelectScratch s;
@@ -195,6 +336,14 @@ SelectScratch select_carve(void* base, int32_t P, int64_t N, int32_t d_out, int3
   s.cur = (double*)p;
   p += 256;
   s.state = (int32_t*)p;
+  p += round_up((int64_t)(kStHdr + m_ens + P) * 4, 256);
+  s.keys = nullptr;
+  s.lab = nullptr;
+  if (score == kScoreAuc) {
+    s.keys = (uint32_t*)p;
+    p += round_up((int64_t)P * 2 * N * 4, 256);
+    s.lab = (uint8_t*)p;
+  }
   return s;
 }
 
@@ -210,8 +359,12 @@ int select_enqueue(cudaStream_t st, const SelectScratch& s, const float* preds, 
   k_sel_init<<<add_blocks, 256, 0, st>>>(s.S, n_S, s.state, n_state, s.cur, excl, m_ens);
   int64_t nl = 1;
   for (int it = 0; it < m_ens; ++it) {
-    k_sel_score<<<dim3(n_blk, P), kSelThreads, 0, st>>>(s.S, preds, y, N, d_out, task, score, s.state,
-                                                        s.partial, n_blk, m_ens);
+    if (score == kScoreAuc)
+      k_sel_auc<<<P, kAucThreads, 0, st>>>(s.S, preds, (const int32_t*)y, N, s.state, s.partial, n_blk, m_ens,
+                                           s.keys, s.lab);
+    else
+      k_sel_score<<<dim3(n_blk, P), kSelThreads, 0, st>>>(s.S, preds, y, N, d_out, task, score, s.state,
+                                                          s.partial, n_blk, m_ens);
     if (it == 0 && solo != nullptr) {
       k_sel_solo<<<(int)ceil_div(P, 256), 256, 0, st>>>(s.partial, P, n_blk, N, score, s.state, m_ens, solo);
       ++nl;

@@ -70,13 +70,14 @@ tp_status pack_select_greedy_static(const float* preds, int32_t P, int64_t N, in
                                     int32_t* selected, int32_t* n_selected, double* final_score) {
   if (!preds || !y || !selected || !n_selected) return static_fail(TP_EINVAL, "null argument");
   if (P < 1 || N < 1 || m_ens < 1) return static_fail(TP_EINVAL, "P, N, m_ens must be >= 1");
-  if (task < 0 || task > 2 || score < 0 || score > 2) return static_fail(TP_EINVAL, "unknown task/score");
+  if (task < 0 || task > 2 || score < 0 || score > 3) return static_fail(TP_EINVAL, "unknown task/score");
+  if (score == TP_SCORE_AUC && task != TP_BINARY) return static_fail(TP_EINVAL, "auc needs a binary task");
   if (score == TP_SCORE_ACCURACY && task == TP_REGRESSION)
     return static_fail(TP_EINVAL, "accuracy needs classification");
   if (score == TP_SCORE_RMSE && task != TP_REGRESSION) return static_fail(TP_EINVAL, "rmse needs regression");
   if (task == TP_MULTICLASS ? (d_out < 2 || d_out > kMaxDout) : d_out != 1) return static_fail(TP_EINVAL, "bad d_out");
   if (P > 65535) return static_fail(TP_EINVAL, "P > 65535");
-  const int64_t need = select_scratch_bytes(P, N, d_out, m_ens);
+  const int64_t need = select_scratch_bytes(P, N, d_out, m_ens, score);
   if (need > kStaticScratchBytes) {
     char buf[256];
     snprintf(buf, sizeof buf,
@@ -89,7 +90,7 @@ tp_status pack_select_greedy_static(const float* preds, int32_t P, int64_t N, in
   cudaError_t e = scratch_address(&base);
   if (e != cudaSuccess) return static_fail(TP_ECUDA, "cudaGetSymbolAddress(scratch)", e);
   cudaStream_t st = (cudaStream_t)cuda_stream;
-  SelectScratch s = select_carve(base, P, N, d_out, m_ens);
+  SelectScratch s = select_carve(base, P, N, d_out, m_ens, score);
   // select_enqueue's first kernel zeroes the running sum and the state, so the
   // previous call's contents do not leak into this one.
   select_enqueue(st, s, preds, P, N, d_out, y, task, score, m_ens, nullptr, nullptr, nullptr);

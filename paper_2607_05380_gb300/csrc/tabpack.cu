@@ -1542,17 +1542,18 @@ tp_status pack_select_greedy(const float* preds, int32_t P, int64_t N, int32_t d
                              int32_t* n_selected, double* final_score) {
   if (!preds || !y || !selected || !n_selected) return fail(nullptr, TP_EINVAL, "null argument");
   if (P < 1 || N < 1 || m_ens < 1) return fail(nullptr, TP_EINVAL, "P, N, m_ens must be >= 1");
-  if (task < 0 || task > 2 || score < 0 || score > 2) return fail(nullptr, TP_EINVAL, "unknown task/score");
+  if (task < 0 || task > 2 || score < 0 || score > 3) return fail(nullptr, TP_EINVAL, "unknown task/score");
+  if (score == TP_SCORE_AUC && task != TP_BINARY) return fail(nullptr, TP_EINVAL, "auc needs a binary task");
   if (score == TP_SCORE_ACCURACY && task == TP_REGRESSION) return fail(nullptr, TP_EINVAL, "accuracy needs classification");
   if (score == TP_SCORE_RMSE && task != TP_REGRESSION) return fail(nullptr, TP_EINVAL, "rmse needs regression");
   if (task == TP_MULTICLASS ? (d_out < 2 || d_out > kMaxDout) : d_out != 1) return fail(nullptr, TP_EINVAL, "bad d_out");
   if (P > 65535) return fail(nullptr, TP_EINVAL, "P > 65535");
   cudaStream_t st = (cudaStream_t)cuda_stream;
-  const int64_t bytes = select_scratch_bytes(P, N, d_out, m_ens);
+  const int64_t bytes = select_scratch_bytes(P, N, d_out, m_ens, score);
   void* scratch = nullptr;
   cudaError_t e = cudaMallocAsync(&scratch, (size_t)bytes, st);
   if (e != cudaSuccess) return fail(nullptr, TP_ENOMEM, "cudaMallocAsync(%lld): %s", (long long)bytes, cudaGetErrorString(e));
-  SelectScratch s = select_carve(scratch, P, N, d_out, m_ens);
+  SelectScratch s = select_carve(scratch, P, N, d_out, m_ens, score);
   const int n_words = select_enqueue(st, s, preds, P, N, d_out, y, task, score, m_ens, nullptr, nullptr, nullptr);
   std::vector<int32_t> host(n_words);
   double cur = 0.0;

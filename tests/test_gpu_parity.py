@@ -486,7 +486,7 @@ def test_inactive_members(tp, prec, fuse):
 
 
 @pytest.mark.parametrize("task,score,d_out", [("multiclass", "loss", 10), ("multiclass", "accuracy", 10),
-                                              ("binary", "loss", 1), ("binary", "accuracy", 1),
+                                              ("binary", "loss", 1), ("binary", "accuracy", 1), ("binary", "auc", 1),
                                               ("regression", "loss", 1), ("regression", "rmse", 1)])
 def test_select_greedy_indices_bit_exact(tp, task, score, d_out):
     """Oracle greedy (fp32 terms, the kernel's decision precision) on the
@@ -517,6 +517,30 @@ def test_select_greedy_indices_bit_exact(tp, task, score, d_out):
     else:
         # per-row terms are fp32: the score is defined to fp32 term rounding
         assert abs(fin - ofin) <= 1e-6 * max(1.0, abs(ofin))
+
+
+@pytest.mark.parametrize("N", [1, 2, 1023, 1024, 1025, 4096 + 77, 70000])
+def test_auc_score_bit_exact(tp, N):
+    """The device's ROC-AUC (radix sort, mid-ranks) equals the oracle's on
+    the same fp32 scores: every candidate's own score, through a one-member
+    selection, on ragged sizes around the 1024-key sort tile and with many
+    ties (scores rounded to 1/64)."""
+    rng = np.random.default_rng(N)
+    P = 6
+    preds = np.round(rng.uniform(0, 1, (P, N, 1)) * 64) / 64
+    preds[5] = rng.uniform(0, 1, (N, 1))                         # no ties
+    preds = preds.astype(np.float32)
+    y = rng.integers(0, 2, N).astype(np.int32)
+    if N >= 2:
+        y[0], y[1] = 0, 1
+    pd, yd = to_dev(preds, y)
+    for c in range(P):
+        sel, fin = tp.select_greedy(pd[c:c + 1].contiguous(), yd, "binary", "auc", m_ens=1)
+        ref = oracle.auc(preds[c, :, 0].astype(np.float64), y)
+        if np.isnan(ref):
+            assert len(sel) == 0
+        else:
+            assert list(sel) == [0] and fin == -ref, (c, fin, ref)
 
 
 def test_select_greedy_worked_example(tp):
