@@ -75,6 +75,9 @@ def lib():
                 "orc_train_step_stacked": (ctypes.c_int, [P, P, i64, P, P, P, i32, u32, i32, P]),
                 "orc_set_muon": (ctypes.c_int, [P, P, ctypes.c_double, i32]),
                 "orc_auc": (ctypes.c_double, [P, P, i64]),
+                "orc_create_emb": (P, [ctypes.POINTER(_Config), P, P, P, P, P, P, P, P]),
+                "orc_get_emb": (ctypes.c_int, [P, i32, i32, P]),
+                "orc_set_emb": (ctypes.c_int, [P, i32, P]),
                 "orc_newton_schulz": (None, [P, i32, i32, i32, i32, P]),
                 "orc_get_muon_dir": (ctypes.c_int, [P, i32, i32, P]),
                 "orc_predict": (ctypes.c_int, [P, P, i64, P]),
@@ -151,7 +154,9 @@ class OraclePack:
 
     def __init__(self, d_in, d_out, task, depth, width, dropout, lr, wd, seed,
                  beta1=0.9, beta2=0.999, eps=1e-8, wd_on_bias=True, bf16_storage=False,
-                 member_id=None):
+                 member_id=None, d_emb=None, freq=None):
+        """d_emb [m] and freq (the members' initial embedding frequencies,
+        d_in x (d_emb[i] - 1) each, concatenated): periodic embeddings."""
         self.task = TASKS[task] if isinstance(task, str) else int(task)
         self.depth = np.ascontiguousarray(depth, dtype=np.int32)
         self.width = np.ascontiguousarray(width, dtype=np.int32)
@@ -163,8 +168,17 @@ class OraclePack:
         lr_ = np.ascontiguousarray(lr, dtype=np.float32)
         wd_ = np.ascontiguousarray(wd, dtype=np.float32)
         mid = None if member_id is None else np.ascontiguousarray(member_id, dtype=np.int32)
-        h = lib().orc_create(ctypes.byref(cfg), _ptr(self.depth), _ptr(self.width), _ptr(drop),
-                             _ptr(lr_), _ptr(wd_), _ptr(mid))
+        self.d_emb = None
+        if d_emb is None:
+            h = lib().orc_create(ctypes.byref(cfg), _ptr(self.depth), _ptr(self.width), _ptr(drop),
+                                 _ptr(lr_), _ptr(wd_), _ptr(mid))
+        else:
+            self.d_emb = np.ascontiguousarray(d_emb, dtype=np.int32)
+            fr = np.ascontiguousarray(freq, dtype=np.float64).ravel()
+            if fr.size != int(np.sum(self.d_in * (self.d_emb - 1))) or np.any(self.d_emb < 1):
+                raise ValueError("freq must hold d_in x (d_emb - 1) values per member; d_emb >= 1")
+            h = lib().orc_create_emb(ctypes.byref(cfg), _ptr(self.depth), _ptr(self.width), _ptr(drop),
+                                     _ptr(lr_), _ptr(wd_), _ptr(mid), _ptr(self.d_emb), _ptr(fr))
         if not h:
             raise ValueError("oracle rejected the pack configuration")
         self._h = ctypes.c_void_p(h)
@@ -178,7 +192,7 @@ class OraclePack:
 
     def layer_shape(self, member, layer):
         L, w = int(self.depth[member]), int(self.width[member])
-        n_in = self.d_in if layer == 0 else w
+        n_in = (self.d_in * (int(self.d_emb[member]) if self.d_emb is not None else 1)) if layer == 0 else w
         n_out = self.d_out if layer == L else w
         return n_out, n_in
 
@@ -212,6 +226,21 @@ class OraclePack:
     def set_active(self, active):
         a = np.ascontiguousarray(active, dtype=np.uint8)
         lib().orc_set_active(self._h, _ptr(a))
+
+    def emb(self, member, grads=False):
+        """(w, b, alpha, beta) of a member's embeddings (or their gradients)."""
+        d, n = int(self.d_emb[member]), self.d_in
+        out = np.zeros(n * (4 * d - 2), dtype=np.float64)
+        if lib().orc_get_emb(self._h, int(member), int(bool(grads)), _ptr(out)):
+            raise ValueError("no embeddings")
+        k = n * (d - 1)
+        return (out[:k].reshape(n, d - 1), out[k:2 * k].reshape(n, d - 1), out[2 * k:2 * k + n * d].reshape(n, d),
+                out[2 * k + n * d:].reshape(n, d))
+
+    def set_emb(self, member, w, b, alpha, beta):
+        flat = np.concatenate([np.ravel(w), np.ravel(b), np.ravel(alpha), np.ravel(beta)]).astype(np.float64)
+        if lib().orc_set_emb(self._h, int(member), _ptr(flat)):
+            raise ValueError("no embeddings")
 
     def set_muon(self, lr_muon, momentum=0.95, ns_steps=5):
         """Muon for the hidden-layer weights from now on (Sec. 3.4)."""

@@ -125,6 +125,15 @@ typedef struct {
   double margin;      /* min |Z| / rms(Z) of the last forward               */
   double lr_muon;     /* Muon learning rate (when the pack uses Muon)       */
   double **dir;       /* [L]: the last Muon direction O of each hidden W    */
+  /* periodic feature embeddings (App. "Feature Embeddings"; d_emb 0: none):
+   * emb = [w: d_in x (d_emb - 1)] [b: d_in x (d_emb - 1)] [alpha: d_in x
+   * d_emb] [beta: d_in x d_emb]; feature j becomes
+   * alpha_j * [x_j, cos(w_j x_j + b_j)] + beta_j, layer 1 reads the d_in
+   * embeddings side by side (in_dim[0] = d_in d_emb).                      */
+  int32_t d_emb;
+  int64_t n_emb;
+  double *emb, *gemb, *memb, *vemb;
+  double *xraw;       /* the last batch's inputs, B x d_in                  */
 } orc_member;
 
 struct orc_pack {
@@ -149,6 +158,8 @@ static double* orc_transpose(const double* a, int64_t rows, int64_t cols) {
 }
 
 static void orc_free_cache(orc_member* M) {
+  free(M->xraw);
+  M->xraw = NULL;
   if (M->Hin) for (int l = 0; l <= M->L; ++l) free(M->Hin[l]);
   if (M->Z) for (int l = 0; l < M->L; ++l) free(M->Z[l]);
   if (M->keep) for (int l = 0; l < M->L; ++l) free(M->keep[l]);
@@ -169,6 +180,7 @@ static void orc_alloc_cache(orc_member* M, int32_t B, int32_t d_out) {
     M->keep[l] = (uint8_t*)calloc((size_t)B * M->w + 1, 1);
   }
   M->logits = orc_zeros((int64_t)B * d_out);
+  M->xraw = orc_zeros((int64_t)B * (M->d_emb ? M->in_dim[0] / M->d_emb : M->in_dim[0]));
 }
 
 void orc_destroy(orc_pack* h) {
@@ -186,15 +198,16 @@ void orc_destroy(orc_pack* h) {
       for (int l = 0; l < M->L; ++l) free(M->dir[l]);
       free(M->dir);
     }
+    free(M->emb); free(M->gemb); free(M->memb); free(M->vemb);
     free(M->in_dim); free(M->out_dim);
   }
   free(h->mem);
   free(h);
 }
 
-orc_pack* orc_create(const orc_config* cfg, const int32_t* depth, const int32_t* width,
-                     const float* dropout, const float* lr, const float* wd,
-                     const int32_t* member_id) {
+orc_pack* orc_create_emb(const orc_config* cfg, const int32_t* depth, const int32_t* width,
+                         const float* dropout, const float* lr, const float* wd,
+                         const int32_t* member_id, const int32_t* d_emb, const double* freq) {
   if (!cfg || cfg->m <= 0 || cfg->d_in <= 0 || cfg->d_out <= 0) return NULL;
   if (cfg->task < 0 || cfg->task > 2) return NULL;
   if (cfg->task != ORC_MULTICLASS && cfg->d_out != 1) return NULL;
@@ -218,9 +231,19 @@ orc_pack* orc_create(const orc_config* cfg, const int32_t* depth, const int32_t*
     M->active = 1;
     M->in_dim = (int32_t*)calloc((size_t)M->L + 1, sizeof(int32_t));
     M->out_dim = (int32_t*)calloc((size_t)M->L + 1, sizeof(int32_t));
+    M->d_emb = d_emb ? d_emb[i] : 0;
     for (int l = 0; l <= M->L; ++l) {
-      M->in_dim[l] = (l == 0) ? cfg->d_in : M->w;
+      M->in_dim[l] = (l == 0) ? cfg->d_in * (M->d_emb ? M->d_emb : 1) : M->w;
       M->out_dim[l] = (l == M->L) ? cfg->d_out : M->w;
+    }
+    if (M->d_emb > 0) {  /* frequencies from the caller, phases and scales zero */
+      M->n_emb = (int64_t)cfg->d_in * (4 * M->d_emb - 2);
+      M->emb = orc_zeros(M->n_emb);
+      M->gemb = orc_zeros(M->n_emb);
+      M->memb = orc_zeros(M->n_emb);
+      M->vemb = orc_zeros(M->n_emb);
+      const int64_t nf = (int64_t)cfg->d_in * (M->d_emb - 1);
+      for (int64_t e = 0; e < nf; ++e) M->emb[e] = *freq++;
     }
     int nl = M->L + 1;
     M->W = (double**)calloc((size_t)nl, sizeof(double*));
@@ -247,6 +270,26 @@ orc_pack* orc_create(const orc_config* cfg, const int32_t* depth, const int32_t*
   return h;
 }
 
+orc_pack* orc_create(const orc_config* cfg, const int32_t* depth, const int32_t* width,
+                     const float* dropout, const float* lr, const float* wd,
+                     const int32_t* member_id) {
+  return orc_create_emb(cfg, depth, width, dropout, lr, wd, member_id, NULL, NULL);
+}
+
+int orc_get_emb(const orc_pack* h, int32_t member, int32_t grads, double* out) {
+  if (!h || member < 0 || member >= h->cfg.m || !h->mem[member].d_emb) return 1;
+  const orc_member* M = &h->mem[member];
+  memcpy(out, grads ? M->gemb : M->emb, sizeof(double) * (size_t)M->n_emb);
+  return 0;
+}
+
+int orc_set_emb(orc_pack* h, int32_t member, const double* in) {
+  if (!h || member < 0 || member >= h->cfg.m || !h->mem[member].d_emb) return 1;
+  orc_member* M = &h->mem[member];
+  memcpy(M->emb, in, sizeof(double) * (size_t)M->n_emb);
+  return 0;
+}
+
 /* value as stored between kernels: bf16 in bf16 mode, exact otherwise */
 static double orc_st(const orc_pack* h, double x) { return h->cfg.bf16_storage ? orc_round_bf16(x) : x; }
 
@@ -261,7 +304,23 @@ static void orc_member_forward(const orc_pack* h, orc_member* M, const float* X,
   const int d_in = h->cfg.d_in, d_out = h->cfg.d_out;
   for (int b = 0; b < B; ++b) {
     int64_t row = idx ? idx[b] : b;
-    for (int k = 0; k < d_in; ++k) M->Hin[0][(int64_t)b * d_in + k] = orc_st(h, (double)X[row * d_in + k]);
+    for (int k = 0; k < d_in; ++k) M->xraw[(int64_t)b * d_in + k] = (double)X[row * d_in + k];
+  }
+  if (M->d_emb == 0) {
+    for (int64_t e = 0; e < (int64_t)B * d_in; ++e) M->Hin[0][e] = orc_st(h, M->xraw[e]);
+  } else {  /* periodic embeddings */
+    const int d = M->d_emb, in0 = d_in * d;
+    const double *ew = M->emb, *eb = ew + (int64_t)d_in * (d - 1), *ea = eb + (int64_t)d_in * (d - 1),
+                 *ebt = ea + (int64_t)d_in * d;
+    for (int b = 0; b < B; ++b)
+      for (int j = 0; j < d_in; ++j) {
+        const double x = M->xraw[(int64_t)b * d_in + j];
+        for (int k = 0; k < d; ++k) {
+          const double f = k == 0 ? x : cos(ew[(int64_t)j * (d - 1) + k - 1] * x + eb[(int64_t)j * (d - 1) + k - 1]);
+          M->Hin[0][(int64_t)b * in0 + j * d + k] =
+              orc_st(h, ea[(int64_t)j * d + k] * f + ebt[(int64_t)j * d + k]);
+        }
+      }
   }
   double margin = INFINITY;
   for (int l = 0; l < M->L; ++l) {
@@ -394,6 +453,45 @@ static double orc_member_backward(const orc_pack* h, orc_member* M, const int32_
     free(HT_l);
     free(dH);
     dH = NULL;
+    if (l == 0 && M->d_emb > 0) {
+      /* dE[b, q] = sum_j dZ[b, j] W_0[j, q] (W as stored; dE stored like dZ),
+       * then the embedding parameters' gradients, rows b increasing */
+      const int d = M->d_emb, d_in = h->cfg.d_in;
+      double* dE = orc_zeros((int64_t)B * in);
+      for (int b = 0; b < B; ++b)
+        for (int q = 0; q < in; ++q) {
+          double s = 0.0;
+          for (int j = 0; j < w; ++j) s += dZ[(int64_t)b * w + j] * orc_st(h, M->W[0][(int64_t)j * in + q]);
+          dE[(int64_t)b * in + q] = orc_st(h, s);
+        }
+      const double *ew = M->emb, *eb = ew + (int64_t)d_in * (d - 1), *ea = eb + (int64_t)d_in * (d - 1);
+      double *gw = M->gemb, *gbb = gw + (int64_t)d_in * (d - 1), *ga = gbb + (int64_t)d_in * (d - 1),
+             *gbt = ga + (int64_t)d_in * d;
+      for (int j = 0; j < d_in; ++j)
+        for (int k = 0; k < d; ++k) {
+          double sa = 0.0, sbt = 0.0, sw = 0.0, sb = 0.0;
+          const double a = ea[(int64_t)j * d + k];
+          for (int b = 0; b < B; ++b) {
+            const double g = dE[(int64_t)b * in + j * d + k], x = M->xraw[(int64_t)b * d_in + j];
+            sbt += g;
+            if (k == 0) {
+              sa += g * x;
+            } else {
+              const double u = ew[(int64_t)j * (d - 1) + k - 1] * x + eb[(int64_t)j * (d - 1) + k - 1];
+              sa += g * cos(u);
+              sw += g * a * (-sin(u)) * x;
+              sb += g * a * (-sin(u));
+            }
+          }
+          ga[(int64_t)j * d + k] = sa;
+          gbt[(int64_t)j * d + k] = sbt;
+          if (k > 0) {
+            gw[(int64_t)j * (d - 1) + k - 1] = sw;
+            gbb[(int64_t)j * (d - 1) + k - 1] = sb;
+          }
+        }
+      free(dE);
+    }
     if (l > 0) {
       /* dH_l[b, k] = sum_j dZ[b, j] W_l[j, k] (j increasing), W as stored */
       double* WT = orc_zeros((int64_t)in * w);
@@ -574,6 +672,7 @@ static int orc_step(orc_pack* h, const float* X, int64_t N, const int32_t* idx, 
         else orc_adamw(h, M, M->W[l], M->mW[l], M->vW[l], M->gW[l], (int64_t)M->out_dim[l] * M->in_dim[l], 0);
         orc_adamw(h, M, M->b[l], M->mb[l], M->vb[l], M->gb[l], M->out_dim[l], 1);
       }
+      if (M->d_emb > 0) orc_adamw(h, M, M->emb, M->memb, M->vemb, M->gemb, M->n_emb, 1);
     }
   }
   return status;
@@ -603,7 +702,7 @@ int orc_predict(orc_pack* h, const float* X, int64_t N, double* out) {
     if (!M->active) continue;
     /* a private cache sized for the validation rows */
     orc_member V = *M;
-    V.Hin = NULL; V.Z = NULL; V.keep = NULL; V.logits = NULL; V.B = 0;
+    V.Hin = NULL; V.Z = NULL; V.keep = NULL; V.logits = NULL; V.xraw = NULL; V.B = 0;
     orc_alloc_cache(&V, (int32_t)N, d_out);
     orc_member_forward(h, &V, X, NULL, (int32_t)N, 0u, 0);
     for (int64_t b = 0; b < N; ++b) {

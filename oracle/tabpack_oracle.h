@@ -88,6 +88,22 @@ orc_pack* orc_create(const orc_config* cfg, const int32_t* depth, const int32_t*
                      const int32_t* member_id);
 void orc_destroy(orc_pack* h);
 
+/* The same pack with periodic feature embeddings (App. "Feature Embeddings"):
+ * member i (d_emb[i] >= 1) maps feature j to alpha_j * [x_j, cos(w_j x_j +
+ * b_j)] + beta_j in R^d_emb (w_j, b_j in R^(d_emb - 1); alpha_j, beta_j in
+ * R^d_emb), and its first layer reads the d_in embeddings side by side
+ * (d_in d_emb inputs, initialised like any layer of that fan-in).  freq: the
+ * initial w of every member in turn, d_in x (d_emb[i] - 1) values each (the
+ * caller draws them from N(0, sigma_i^2)); b, alpha, beta start at zero.
+ * The embedding parameters take AdamW steps like biases.                     */
+orc_pack* orc_create_emb(const orc_config* cfg, const int32_t* depth, const int32_t* width,
+                         const float* dropout, const float* lr, const float* wd,
+                         const int32_t* member_id, const int32_t* d_emb, const double* freq);
+/* A member's embedding parameters (grads 0) or their last gradients
+ * (grads 1): [w, b, alpha, beta] as above, d_in (4 d_emb - 2) values.        */
+int orc_get_emb(const orc_pack* h, int32_t member, int32_t grads, double* out);
+int orc_set_emb(orc_pack* h, int32_t member, const double* in);
+
 /* Initial value of element e of layer `layer` (0-based; layer == depth is the
  * head) of a member, as stored (fp32-representable).                          */
 double orc_init_value(uint64_t seed, uint32_t member_id, uint32_t layer, uint32_t e, int32_t fan_in);
