@@ -28,7 +28,7 @@ import numpy as np
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-from workloads import SEED_HP, SEED_INIT, WORKLOADS, make_data, sample_hparams  # noqa: E402
+from workloads import SEED_HP, SEED_INIT, WORKLOADS, make_data, sample_emb, sample_hparams  # noqa: E402
 
 METRIC = "member-samples/sec (fwd+bwd+AdamW)"
 
@@ -52,18 +52,28 @@ def peaks():
     return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
 
 
-def work_per_step(wl, hp, B):
+def in0_of(wl, emb, i):
+    """Member i's first-layer input width (d_in d_emb with embeddings)."""
+    return wl.d_in * (int(emb["d_emb"][i]) if emb is not None else 1)
+
+
+def work_per_step(wl, hp, B, emb=None):
     """Algorithmic work of one step, from the shapes (no padding):
-    matrix-product flops (forward 2, dgrad 2 except layer 0, wgrad 2 per MAC)
-    and AdamW bytes (read p, g, m, v; write p, m, v fp32 + the bf16 copy)."""
+    matrix-product flops (forward 2, dgrad 2 except layer 0 -- with
+    embeddings layer 0 too, for dE --, wgrad 2 per MAC) and the parameter
+    count of the AdamW bytes (read p, g, m, v; write p, m, v fp32 + the bf16
+    copy), embeddings included."""
     flops = 0.0
     n_params = 0
-    for L, w in zip(hp["depth"], hp["width"]):
+    for i, (L, w) in enumerate(zip(hp["depth"], hp["width"])):
         L, w = int(L), int(w)
-        macs_fwd = wl.d_in * w + (L - 1) * w * w
-        macs_dgrad = (L - 1) * w * w
+        in0 = in0_of(wl, emb, i)
+        macs_fwd = in0 * w + (L - 1) * w * w
+        macs_dgrad = (L - 1) * w * w + (in0 * w if emb is not None else 0)
         flops += 2.0 * B * (2 * macs_fwd + macs_dgrad)
-        n_params += wl.d_in * w + w + (L - 1) * (w * w + w) + wl.d_out * w + wl.d_out
+        n_params += in0 * w + w + (L - 1) * (w * w + w) + wl.d_out * w + wl.d_out
+        if emb is not None:
+            n_params += wl.d_in * (4 * int(emb["d_emb"][i]) - 2)
     return flops, n_params
 
 
@@ -138,18 +148,18 @@ class ClockSampler:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
-def predict_flops(wl, hp, n_rows):
+def predict_flops(wl, hp, n_rows, emb=None):
     """Matrix-product flops of one forward without dropout of every member
     over n_rows rows (hidden layers and head)."""
     f = 0
-    for L, w in zip(hp["depth"], hp["width"]):
+    for i, (L, w) in enumerate(zip(hp["depth"], hp["width"])):
         L, w = int(L), int(w)
-        f += wl.d_in * w + (L - 1) * w * w + w * wl.d_out
+        f += in0_of(wl, emb, i) * w + (L - 1) * w * w + w * wl.d_out
     return 2.0 * n_rows * f
 
 
 def time_online_epoch(tp, torch, pack, wl, hp, d, X, y, idx_all, stream, loss, n_epochs=6, steps_between=8,
-                      m_ens=32, p_base=16, p_ens=32, score="loss"):
+                      m_ens=32, p_base=16, p_ens=32, score="loss", emb=None):
     """Wall time of the online ensemble's epoch end (Sec. 3.5: predict the
     members on the validation rows, greedy selection over the pool, member
     snapshots, patience bookkeeping) on the workload's full validation set,
@@ -186,17 +196,17 @@ def time_online_epoch(tp, torch, pack, wl, hp, d, X, y, idx_all, stream, loss, n
     sel_bytes = m_ens * pool * n_val * wl.d_out * 4.0
     return {"ms": ms, "predict_ms": pm, "select_and_rest_ms": ms - pm, "n_val": n_val, "m_ens": m_ens, "score": score,
             "pool": pool, "n_best": info["n_best"], "epochs_timed": len(times),
-            "predict_tflops": predict_flops(wl, hp, n_val) / (pm / 1e3) / 1e12,
+            "predict_tflops": predict_flops(wl, hp, n_val, emb) / (pm / 1e3) / 1e12,
             "select_candidate_bytes": sel_bytes,
             "note": "epoch-end cost once per epoch of %d steps; predictions on the full validation set"
                     % -(-wl.n_train // B)}
 
 
-def cpu_baseline(wl, hp, data_np, B, budget_s=20.0, stacked=False):
+def cpu_baseline(wl, hp, data_np, B, budget_s=20.0, stacked=False, emb=None):
     """The oracle as it stands, on the host cores, on a bounded sample of the
     same workload: the first k members (independent of the others), timed
     over whole steps until about budget_s seconds of CPU work (stacked: a
-    batch per member)."""
+    batch per member; emb: the members' periodic embeddings)."""
     import oracle
     oracle.build()
     X, y = data_np
@@ -204,9 +214,13 @@ def cpu_baseline(wl, hp, data_np, B, budget_s=20.0, stacked=False):
     k = min(wl.m, max(1, cores))
     rng = np.random.default_rng(3)
     members = list(range(k))
+    kw = {}
+    if emb is not None:   # the first k members' sizes and frequencies (stored member after member)
+        n_f = wl.d_in * int(np.sum(emb["d_emb"][:k] - 1))
+        kw = dict(d_emb=emb["d_emb"][:k], freq=emb["freq"][:n_f].astype(np.float64))
     pk = oracle.OraclePack(wl.d_in, wl.d_out, wl.task, hp["depth"][members], hp["width"][members],
                            hp["dropout"][members], hp["lr"][members], hp["wd"][members], seed=SEED_INIT,
-                           member_id=members)
+                           member_id=members, **kw)
     steps = 0
     t0 = time.perf_counter()
     while True:
@@ -224,6 +238,13 @@ def cpu_baseline(wl, hp, data_np, B, budget_s=20.0, stacked=False):
             "sample": f"members 0..{k - 1} of {wl.m} (independent), {steps} full steps of batch {B}, {el:.1f} s"}
 
 
+def emb_desc(emb):
+    if emb is None:
+        return "none (raw features)"
+    return ("periodic (App. Feature Embeddings), d_emb UniformInt[8,32] step 4 (sampled %s), sigma "
+            "LogUniform[1e-2,10]" % ",".join(str(int(x)) for x in emb["d_emb"]))
+
+
 def run_reference(args, wl, rank):
     """Reference arm: the CPU fp64 oracle timed on the host cores (rank 0)."""
     if rank != 0:
@@ -238,15 +259,16 @@ def run_reference(args, wl, rank):
     for _ in range(args.warmup if args.warmup < 1 else 1):
         pass
     base = None
+    emb = sample_emb(wl.m, wl.d_in, seed=SEED_HP + 200) if args.emb else None
     for s in range(max(1, args.steps)):
-        base = cpu_baseline(wl, hp, data, B, budget_s=per, stacked=args.stacked)
+        base = cpu_baseline(wl, hp, data, B, budget_s=per, stacked=args.stacked, emb=emb)
         vals.append(base["value"])
     value = float(np.mean(vals))
     ms = float(1000.0 * wl.m * B / value)
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": workload_desc(wl, B)},
+            "config": {"workload": workload_desc(wl, B), "embeddings": emb_desc(emb)},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": base["cores"], "kind": "oracle",
                              "sample": base["sample"]},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -273,6 +295,9 @@ def main():
                     help="Muon for the hidden-layer weights (the paper's default optimizer), AdamW for the rest")
     ap.add_argument("--stacked", action="store_true",
                     help="a batch per member (idx [m, B], Sec. 3.6) instead of one batch shared by all members")
+    ap.add_argument("--emb", action="store_true",
+                    help="periodic feature embeddings (App. Feature Embeddings), d_emb and sigma per member "
+                         "from the paper's sampling space")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -314,9 +339,11 @@ def main():
     idx_all = idx_all.to(torch.int32).contiguous()
 
     stream = torch.cuda.current_stream()
+    emb = sample_emb(wl.m, wl.d_in, seed=SEED_HP + 200) if args.emb else None
     pack = tp.Pack(wl.d_in, wl.d_out, wl.task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
                    max_batch=B, seed=SEED_INIT, precision=args.precision, stream=stream,
-                   fuse_optimizer=args.fuse_optimizer)
+                   fuse_optimizer=args.fuse_optimizer, d_emb=None if emb is None else emb["d_emb"],
+                   freq=None if emb is None else emb["freq"])
     loss = torch.zeros(wl.m, dtype=torch.float32, device=dev)
     lr_muon = None
     if args.muon:   # Muon lr LogUniform[1e-3, 1e-1] per member
@@ -358,7 +385,9 @@ def main():
         pack.train_step(X, idx_all[args.warmup + s], y, total + s, loss)
     prof = pack.profile_read(reset=True)
     pack.profile_enable(False)
-    flops, n_params = work_per_step(wl, hp, B)
+    flops, n_params = work_per_step(wl, hp, B, emb)
+    # the DRAM captures are of the default configuration (shared batch, AdamW, raw features)
+    plain = args.members == 0 and not (args.emb or args.muon or args.stacked)
     pk = peaks()
     fam = {k: v for k, v in prof.items() if v[1] > 0}
     dominant = max(fam, key=lambda k: fam[k][0])
@@ -369,7 +398,7 @@ def main():
     gemm_ms = fwd_ms + bwd_ms
     gemm = {"kernel": "k_tc_gemm (grouped fwd + dgrad + wgrad launches of one step)", "bound": "tensor",
             "achieved": flops / (gemm_ms / 1e3) / 1e12, "peak": pk["bf16_sus"], "unit": "TFLOP/s",
-            "traffic": DRAM_TRAFFIC.get((args.workload, "k_tc_gemm")) if args.members == 0 else None,
+            "traffic": DRAM_TRAFFIC.get((args.workload, "k_tc_gemm")) if plain else None,
             "ms_per_step": gemm_ms, "peak_source": pk["source"] + " sustained bf16"}
     gemm["frac"] = gemm["achieved"] / gemm["peak"]
     if adam_ms > 0:   # AdamW as a separate pass (the default): 30 B per parameter
@@ -380,16 +409,16 @@ def main():
                "bound": "hbm", "achieved": 26.0 * n_params / (bwd_ms / 1e3) / 1e9, "ms_per_step": bwd_ms,
                "bytes_per_step": 26.0 * n_params}
     mem.update({"peak": pk["hbm"], "unit": "GB/s", "peak_source": pk["source"] + " HBM copy",
-                "traffic": DRAM_TRAFFIC.get((args.workload, "k_adamw")) if args.members == 0 and adam_ms > 0 else None})
+                "traffic": DRAM_TRAFFIC.get((args.workload, "k_adamw")) if plain and adam_ms > 0 else None})
     mem["frac"] = mem["achieved"] / mem["peak"]
     roof = dict(gemm if gemm_ms >= adam_ms else mem)
     roof["other"] = mem if gemm_ms >= adam_ms else gemm
     roof["shares"] = shares
     if args.muon:   # the Newton-Schulz products: 5 x (4 r^2 c + 2 r^3) per matrix
         ns_flops = 0.0
-        for L_, w_ in zip(hp["depth"], hp["width"]):
+        for i_, (L_, w_) in enumerate(zip(hp["depth"], hp["width"])):
             for l in range(int(L_)):
-                cols = wl.d_in if l == 0 else int(w_)
+                cols = in0_of(wl, emb, i_) if l == 0 else int(w_)
                 r_, c_ = min(int(w_), cols), max(int(w_), cols)
                 ns_flops += 5 * (4.0 * r_ * r_ * c_ + 2.0 * r_ ** 3)
         muon_ms = prof["muon"][0] / n_prof
@@ -438,13 +467,13 @@ def main():
                "steps": n_e2e}
 
     online = None if args.no_online else time_online_epoch(tp, torch, pack, wl, hp, d, X, y, idx_all, stream, loss,
-                                                           score=args.online_score)
+                                                           score=args.online_score, emb=emb)
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         n = min(n_train, 20000)
         data_np = (X[:n].cpu().numpy(), y[:n].cpu().numpy())
-        cpu = cpu_baseline(wl, hp, data_np, B, budget_s=20.0, stacked=args.stacked)
+        cpu = cpu_baseline(wl, hp, data_np, B, budget_s=20.0, stacked=args.stacked, emb=emb)
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -457,7 +486,8 @@ def main():
                            "parallelism": "one independent pack per GPU" if world > 1 else "single GPU",
                            "batches": "one per member (stacked)" if args.stacked else "one shared by all members",
                            "optimizer": "Muon (hidden weights, lr LogUniform[1e-3, 1e-1]) + AdamW" if args.muon
-                                        else "AdamW"},
+                                        else "AdamW",
+                           "embeddings": emb_desc(emb)},
                 "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches, "online_epoch": online,
                 "clocks": clk.summary(), "final_losses_mean": float(np.nanmean(lossv))}
         print(json.dumps(line), flush=True)

@@ -91,6 +91,42 @@ tp_status pack_create(const tp_config* cfg, const int32_t* depth, const int32_t*
                       const float* dropout, const float* lr, const float* wd,
                       void* cuda_stream, tabpack_t** out);
 
+/* Create a pack whose members read periodic feature embeddings (App.
+ * "Feature Embeddings"): feature j of member i becomes the d = d_emb[i]
+ * values  alpha_j (.) [x_j, cos(w_j x_j + b_j)] + beta_j  (w_j, b_j of
+ * length d - 1; alpha_j, beta_j of length d; (.) elementwise), and the
+ * first hidden layer reads the d_in embeddings side by side (column j d + k
+ * is component k of feature j), so its input width is d_in d.
+ * Arguments as pack_create, plus d_emb: host [m], each in 1..64; freq: host
+ * array holding, member after member, the d_in (d_emb[i] - 1) initial
+ * frequencies w of member i (row-major [d_in, d_emb[i] - 1]; the paper
+ * draws them from N(0, sigma), sigma a per-member hyperparameter, so the
+ * caller draws them); b, alpha and beta start at zero.  The embedding
+ * parameters are trained by AdamW with the member's lr, as the biases are
+ * (weight decay on them only when cfg->wd_on_bias), also under Muon;
+ * fuse_optimizer is turned off.  The embedding kernels compute in fp32
+ * (cosf) and store E in the matrix-product precision; their gradients
+ * are accumulated in fp64 over the batch rows in order.  Memory: an
+ * embedding matrix [max_batch rounded up to 128, d_in d rounded up to 8,
+ * plus 16] per member, its input gradient, and, while predicting, the
+ * same for a chunk of at most 8192 rows, fewer where the chunk's
+ * embedding matrices of all members would pass 1 GiB.                    */
+tp_status pack_create_emb(const tp_config* cfg, const int32_t* depth, const int32_t* width,
+                          const float* dropout, const float* lr, const float* wd, const int32_t* d_emb,
+                          const float* freq, void* cuda_stream, tabpack_t** out);
+
+/* Member `member`'s embedding parameters (grads = 1: their gradients from
+ * the last step without update), copied to the host array out of
+ * d_in (4 d - 2) floats: w [d_in, d - 1], b [d_in, d - 1], alpha [d_in, d],
+ * beta [d_in, d], d = its d_emb.  TP_EINVAL for a pack without
+ * embeddings.  Synchronises.                                                */
+tp_status pack_get_emb(tabpack_t* pack, int32_t member, int32_t grads, float* out);
+/* Overwrite member `member`'s embedding parameters from the host array in
+ * (layout of pack_get_emb).  Synchronises.                                 */
+tp_status pack_set_emb(tabpack_t* pack, int32_t member, const float* in);
+/* *d_emb = member `member`'s embedding size (0 for a pack without). */
+tp_status pack_member_emb(const tabpack_t* pack, int32_t member, int32_t* d_emb);
+
 /* Free the pack and its device memory (waits for the pack's stream). NULL ok. */
 void pack_destroy(tabpack_t* pack);
 

@@ -35,7 +35,7 @@ SYMBOLS = ["pack_create", "pack_destroy", "pack_set_stream", "pack_train_step", 
            "pack_get_stream", "pack_online_create", "pack_online_destroy", "pack_online_epoch", "pack_online_info",
            "pack_online_members", "pack_online_ensemble", "pack_online_snapshot", "pack_online_predict",
            "pack_online_last_error", "pack_train_step_stacked", "pack_forward_backward_stacked", "pack_set_muon",
-           "pack_debug_muon_dir"]
+           "pack_debug_muon_dir", "pack_create_emb", "pack_get_emb", "pack_set_emb", "pack_member_emb"]
 
 
 class TabpackError(RuntimeError):
@@ -112,6 +112,10 @@ def load_library(path: str = LIB_PATH):
         "pack_set_muon": (st, [P, P, ctypes.c_float, i32]),
         "pack_debug_muon_dir": (st, [P, i32, i32, P]),
         "pack_forward_backward_stacked": (st, [P, P, i64, P, P, i32, u32, P]),
+        "pack_create_emb": (st, [ctypes.POINTER(Config), P, P, P, P, P, P, P, P, ctypes.POINTER(P)]),
+        "pack_get_emb": (st, [P, i32, i32, P]),
+        "pack_set_emb": (st, [P, i32, P]),
+        "pack_member_emb": (st, [P, i32, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -156,7 +160,10 @@ class Pack:
 
     def __init__(self, d_in, d_out, task, depth, width, dropout, lr, wd, max_batch, seed=2,
                  precision="bf16", beta1=0.9, beta2=0.999, eps=1e-8, wd_on_bias=True, stream=None,
-                 fuse_optimizer=False):
+                 fuse_optimizer=False, d_emb=None, freq=None):
+        """d_emb: per-member periodic embedding sizes (None: the members read
+        the raw features); freq: their initial frequencies w, member after
+        member [d_in, d_emb[i] - 1] (App. "Feature Embeddings")."""
         import torch
         L = load_library()
         self.torch = torch
@@ -172,8 +179,18 @@ class Pack:
         lr_ = np.ascontiguousarray(lr, dtype=np.float32)
         wd_ = np.ascontiguousarray(wd, dtype=np.float32)
         h = ctypes.c_void_p()
-        _check(L.pack_create(ctypes.byref(cfg), _hptr(self.depth), _hptr(self.width), _hptr(drop), _hptr(lr_),
-                             _hptr(wd_), _stream_ptr(stream), ctypes.byref(h)))
+        self.d_emb = None
+        if d_emb is None:
+            _check(L.pack_create(ctypes.byref(cfg), _hptr(self.depth), _hptr(self.width), _hptr(drop), _hptr(lr_),
+                                 _hptr(wd_), _stream_ptr(stream), ctypes.byref(h)))
+        else:
+            self.d_emb = np.ascontiguousarray(d_emb, dtype=np.int32)
+            fr = np.ascontiguousarray(freq, dtype=np.float32)
+            if self.d_emb.shape != (self.m,) or fr.size != self.d_in * int(np.sum(self.d_emb - 1)):
+                raise ValueError("d_emb must hold m sizes and freq d_in (d_emb[i] - 1) values per member")
+            _check(L.pack_create_emb(ctypes.byref(cfg), _hptr(self.depth), _hptr(self.width), _hptr(drop),
+                                     _hptr(lr_), _hptr(wd_), _hptr(self.d_emb), _hptr(fr), _stream_ptr(stream),
+                                     ctypes.byref(h)))
         self._h = h
         self._B = 0
 
@@ -259,7 +276,30 @@ class Pack:
 
     def layer_shape(self, member, layer):
         L, w = int(self.depth[member]), int(self.width[member])
-        return (self.d_out if layer == L else w), (self.d_in if layer == 0 else w)
+        d0 = self.d_in * (int(self.d_emb[member]) if self.d_emb is not None else 1)
+        return (self.d_out if layer == L else w), (d0 if layer == 0 else w)
+
+    def emb(self, member, grads=False):
+        """(w, b, alpha, beta) of a member's embeddings, or their gradients
+        from the last step without update."""
+        if self.d_emb is None:
+            _check(load_library().pack_get_emb(self._h, 0, 0, None), self._h)
+        d, n = int(self.d_emb[member]), self.d_in
+        out = np.zeros(n * (4 * d - 2), dtype=np.float32)
+        _check(load_library().pack_get_emb(self._h, int(member), int(bool(grads)), _hptr(out)), self._h)
+        k = n * (d - 1)
+        return (out[:k].reshape(n, d - 1), out[k:2 * k].reshape(n, d - 1), out[2 * k:2 * k + n * d].reshape(n, d),
+                out[2 * k + n * d:].reshape(n, d))
+
+    def set_emb(self, member, w, b, alpha, beta):
+        if self.d_emb is None:
+            _check(load_library().pack_set_emb(self._h, 0, None), self._h)
+        d, n = int(self.d_emb[member]), self.d_in
+        parts = [np.asarray(a, dtype=np.float32) for a in (w, b, alpha, beta)]
+        if [p.size for p in parts] != [n * (d - 1), n * (d - 1), n * d, n * d]:
+            raise ValueError("shape mismatch")
+        flat = np.ascontiguousarray(np.concatenate([p.ravel() for p in parts]))
+        _check(load_library().pack_set_emb(self._h, int(member), _hptr(flat)), self._h)
 
     def _valid(self, member, layer):
         return 0 <= member < self.m and 0 <= layer <= int(self.depth[member])

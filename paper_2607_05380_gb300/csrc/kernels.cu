@@ -79,9 +79,10 @@ __global__ void k_gather(const float* __restrict__ X, const int32_t* __restrict_
 
 // Column `col` of the first `rows` rows := 1 (xb and every act matrix, once).
 template <typename T>
-__global__ void k_fill_ones(const OnesJob* __restrict__ jobs, T* __restrict__ xb, T* __restrict__ act) {
+__global__ void k_fill_ones(const OnesJob* __restrict__ jobs, T* __restrict__ xb, T* __restrict__ act,
+                            T* __restrict__ ex) {
   const OnesJob jb = jobs[blockIdx.x];
-  T* base = (jb.arena == 0 ? xb : act) + jb.off;
+  T* base = (jb.arena == 0 ? xb : jb.arena == 1 ? act : ex) + jb.off;
   for (int r = threadIdx.x; r < jb.rows; r += blockDim.x) base[(int64_t)r * jb.ld + jb.col] = Elem<T>::from_f(1.f);
 }
 
@@ -100,7 +101,7 @@ __global__ void __launch_bounds__(256) k_gemm_simt(GemmArgs<T> g, int32_t tile_b
   const int K = P.K ? P.K : g.B_pad;
   if (t.m0 >= M) return;
   const uint32_t step = g.dyn ? g.dyn->step : g.step;
-  const T* bases[5] = {g.xb, g.act, g.dz, g.wq, g.ns};
+  const T* bases[6] = {g.xb, g.act, g.dz, g.wq, g.ns, g.ex};
   // stacked batches: the member's own batch matrix
   const int64_t xs = (int64_t)P.member * g.xb_stride;
   const T* A = bases[P.a_src] + P.a_off + (P.a_src == kSrcXb ? xs : 0);
@@ -184,13 +185,18 @@ __global__ void __launch_bounds__(256) k_gemm_simt(GemmArgs<T> g, int32_t tile_b
         float h = ((keep >> j) & 1u) ? a * sc : 0.f;
         C[(int64_t)r * P.ldc + c0 + j] = Elem<T>::from_f(h);
       }
-    } else if (P.kind == kDgrad) {  // N = w
-      const T* Hm = g.act + P.aux_off;
+    } else if (P.kind == kDgrad) {  // N = w (the first layer's input gradient: no mask, aux_off < 0)
       T* C = g.dz + P.c_off;
+      if (P.aux_off < 0) {
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        float h = Elem<T>::to_f(Hm[(int64_t)r * P.ld_aux + c0 + j]);
-        C[(int64_t)r * P.ldc + c0 + j] = Elem<T>::from_f(h > 0.f ? acc[i][j] * md.scale : 0.f);
+        for (int j = 0; j < 4; ++j) C[(int64_t)r * P.ldc + c0 + j] = Elem<T>::from_f(acc[i][j]);
+      } else {
+        const T* Hm = g.act + P.aux_off;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          float h = Elem<T>::to_f(Hm[(int64_t)r * P.ld_aux + c0 + j]);
+          C[(int64_t)r * P.ldc + c0 + j] = Elem<T>::from_f(h > 0.f ? acc[i][j] * md.scale : 0.f);
+        }
       }
     } else {  // N = in_pad + 1: the last column is the bias gradient
       float* C = g.grads + P.c_off;
@@ -828,8 +834,8 @@ void launch_gather(cudaStream_t st, const float* X, const int32_t* idx, const St
 }
 
 template <typename T>
-void launch_fill_ones(cudaStream_t st, const OnesJob* jobs, int n_jobs, T* xb, T* act) {
-  if (n_jobs > 0) k_fill_ones<T><<<n_jobs, 256, 0, st>>>(jobs, xb, act);
+void launch_fill_ones(cudaStream_t st, const OnesJob* jobs, int n_jobs, T* xb, T* act, T* ex) {
+  if (n_jobs > 0) k_fill_ones<T><<<n_jobs, 256, 0, st>>>(jobs, xb, act, ex);
 }
 
 template <typename T>
@@ -861,6 +867,148 @@ void launch_adamw(cudaStream_t st, const AdamArgs& g, int n_chunks) {
 
 void launch_init(cudaStream_t st, const InitArgs& g, int n_chunks) {
   if (n_chunks > 0) k_init<<<n_chunks, 256, 0, st>>>(g);
+}
+
+// ---------------------------------------------------- periodic embeddings
+// E_i[b, q] (q = j d + k) = alpha_q f_q(x_bj) + beta_q with f_0(x) = x and
+// f_k(x) = cos(w_j,k-1 x + b_j,k-1).  Both kernels tile a member's columns
+// in groups of 32 (lane = column: each thread keeps its column's feature,
+// component and parameters in registers) and spread the rows over the
+// block's 8 warps.
+constexpr int kEmbRows = 64;   // rows per forward block
+
+struct EmbCol {
+  int j, k;
+  float w, b, alpha, beta;
+};
+
+__device__ __forceinline__ EmbCol emb_col(const EmbMember& em, const float* params, int d_in, int q) {
+  const int d = em.d, dm = d - 1;
+  const float* w = params + em.p_off;
+  const float* bb = w + (int64_t)d_in * dm;
+  const float* al = bb + (int64_t)d_in * dm;
+  const float* be = al + (int64_t)d_in * d;
+  EmbCol c;
+  c.j = q / d;
+  c.k = q - c.j * d;
+  c.alpha = al[q];
+  c.beta = be[q];
+  c.w = c.k ? w[c.j * dm + c.k - 1] : 0.f;
+  c.b = c.k ? bb[c.j * dm + c.k - 1] : 0.f;
+  return c;
+}
+
+// Forward: block (32-column group, 64-row group, active member); rows >= B
+// and the pad columns up to in0_pad are written as zero.
+template <typename T>
+__global__ void __launch_bounds__(256) k_emb_fwd(EmbArgs<T> a) {
+  pdl_trigger();
+  pdl_wait();
+  const int member = a.active_ids[blockIdx.z];
+  const EmbMember em = a.em[member];
+  const int q = blockIdx.x * 32 + (threadIdx.x & 31);
+  if (q >= em.in0_pad) return;
+  const float* X = a.dyn ? a.dyn->X : a.X;
+  const int32_t* idx = a.dyn ? a.dyn->idx : a.idx;
+  if (idx) idx += (int64_t)member * a.idx_stride;
+  const bool col = q < em.in0;
+  const EmbCol c = col ? emb_col(em, a.params, a.d_in, q) : EmbCol{0, 0, 0.f, 0.f, 0.f, 0.f};
+  const int64_t ld = em.in0_pad + kOnesCols;
+  T* E = a.ex + em.e_off + q;
+  const int r1 = min(a.B_pad, (int)(blockIdx.y + 1) * kEmbRows);
+  for (int b = blockIdx.y * kEmbRows + (threadIdx.x >> 5); b < r1; b += 8) {
+    float e = 0.f;
+    if (col && b < a.B) {
+      const int64_t row = idx ? (int64_t)idx[b] : (int64_t)b;
+      const float x = X[row * a.d_in + c.j];
+      const float f = c.k == 0 ? x : cosf(fmaf(c.w, x, c.b));
+      e = fmaf(c.alpha, f, c.beta);
+    }
+    E[(int64_t)b * ld] = Elem<T>::from_f(e);
+  }
+}
+
+// Backward: block (32-column group, active member), warp r takes rows r,
+// r + 8, ...; with dE = the first layer's input gradient,
+//   d alpha_q = sum_b dE f_q,  d beta_q = sum_b dE,
+//   d w = -alpha_q sum_b dE sin(u) x,  d b = -alpha_q sum_b dE sin(u)
+// (u = w x + b, cosine components).  Each thread sums up to 32 of its rows
+// in fp32 and adds that partial to fp64 sums; the 8 warps' fp64 sums are
+// added in warp order.
+template <typename T>
+__global__ void __launch_bounds__(256) k_emb_bwd(EmbArgs<T> a) {
+  pdl_trigger();
+  pdl_wait();
+  const int member = a.active_ids[blockIdx.y];
+  const EmbMember em = a.em[member];
+  if ((int)blockIdx.x * 32 >= em.in0) return;   // block-uniform
+  const int lane = threadIdx.x & 31, wp = threadIdx.x >> 5;
+  const int q = blockIdx.x * 32 + lane;
+  const bool col = q < em.in0;
+  const int qc = col ? q : em.in0 - 1;          // in-range column for the loads of idle lanes
+  const float* X = a.dyn ? a.dyn->X : a.X;
+  const int32_t* idx = a.dyn ? a.dyn->idx : a.idx;
+  if (idx) idx += (int64_t)member * a.idx_stride;
+  const EmbCol c = emb_col(em, a.params, a.d_in, qc);
+  const T* dE = a.dz + em.de_off + qc;
+  double s_a = 0.0, s_be = 0.0, s_w = 0.0, s_b = 0.0;
+  for (int b0 = wp; b0 < a.B; b0 += 8 * 32) {
+    float p_a = 0.f, p_be = 0.f, p_w = 0.f, p_b = 0.f;
+    const int b1 = min(a.B, b0 + 8 * 32);
+    for (int b = b0; b < b1; b += 8) {
+      const float g = Elem<T>::to_f(dE[(int64_t)b * em.in0_pad]);
+      const int64_t row = idx ? (int64_t)idx[b] : (int64_t)b;
+      const float x = X[row * a.d_in + c.j];
+      p_be += g;
+      if (c.k == 0) {
+        p_a = fmaf(g, x, p_a);
+      } else {
+        float sn, cs;
+        sincosf(fmaf(c.w, x, c.b), &sn, &cs);
+        p_a = fmaf(g, cs, p_a);
+        const float gs = g * sn;
+        p_w = fmaf(gs, x, p_w);
+        p_b += gs;
+      }
+    }
+    s_a += p_a;
+    s_be += p_be;
+    s_w += p_w;
+    s_b += p_b;
+  }
+  __shared__ double red[4][8][32];
+  red[0][wp][lane] = s_a;
+  red[1][wp][lane] = s_be;
+  red[2][wp][lane] = s_w;
+  red[3][wp][lane] = s_b;
+  __syncthreads();
+  if (wp != 0 || !col) return;
+  double t[4] = {0.0, 0.0, 0.0, 0.0};
+  for (int r = 0; r < 8; ++r)
+    for (int u = 0; u < 4; ++u) t[u] += red[u][r][lane];
+  const int d = em.d, dm = d - 1;
+  float* gw = a.grads + em.p_off;
+  float* gb = gw + (int64_t)a.d_in * dm;
+  float* ga = gb + (int64_t)a.d_in * dm;
+  float* gbt = ga + (int64_t)a.d_in * d;
+  ga[q] = (float)t[0];
+  gbt[q] = (float)t[1];
+  if (c.k) {
+    gw[c.j * dm + c.k - 1] = (float)(-(double)c.alpha * t[2]);
+    gb[c.j * dm + c.k - 1] = (float)(-(double)c.alpha * t[3]);
+  }
+}
+
+template <typename T>
+void launch_emb_fwd(cudaStream_t st, const EmbArgs<T>& a, int n_active, int cols_max) {
+  if (n_active > 0 && a.B_pad > 0)
+    launch_pdl(k_emb_fwd<T>, dim3((unsigned)ceil_div(cols_max, 32), (unsigned)ceil_div(a.B_pad, kEmbRows),
+                                  (unsigned)n_active), dim3(256), 0, st, a);
+}
+template <typename T>
+void launch_emb_bwd(cudaStream_t st, const EmbArgs<T>& a, int n_active, int cols_max) {
+  if (n_active > 0)
+    launch_pdl(k_emb_bwd<T>, dim3((unsigned)ceil_div(cols_max, 32), (unsigned)n_active), dim3(256), 0, st, a);
 }
 
 // ------------------------------------------------------------------ Muon
@@ -996,11 +1144,13 @@ void launch_debug_masks(cudaStream_t st, uint8_t* out, int B, int w, uint64_t se
   template void launch_gather<T>(cudaStream_t, const float*, const int32_t*, const StepDyn*, int, int, int, int, \
                                  int, T*, int, int32_t*, float2*, const int32_t*, int, float, float,    \
                                  int*, int, int, int64_t);                                              \
-  template void launch_fill_ones<T>(cudaStream_t, const OnesJob*, int, T*, T*);                         \
+  template void launch_fill_ones<T>(cudaStream_t, const OnesJob*, int, T*, T*, T*);                    \
   template void launch_gemm_simt<T>(cudaStream_t, const GemmArgs<T>&, int, int);                       \
   template void launch_head<T>(cudaStream_t, const HeadArgs<T>&, int);                                 \
   template void launch_predict_head<T>(cudaStream_t, const PredictHeadArgs<T>&, int);           \
-  template void launch_muon<T>(cudaStream_t, const MuonArgs<T>&, int, int);
+  template void launch_muon<T>(cudaStream_t, const MuonArgs<T>&, int, int);                      \
+  template void launch_emb_fwd<T>(cudaStream_t, const EmbArgs<T>&, int, int);                     \
+  template void launch_emb_bwd<T>(cudaStream_t, const EmbArgs<T>&, int, int);
 
 TP_INSTANTIATE(float)
 TP_INSTANTIATE(__nv_bfloat16)

@@ -25,6 +25,7 @@ struct GemmArgs {
   const StepDyn* dyn;     // non-NULL: take the step from here
   int64_t xb_stride;      // stacked batches: elements between members' batch matrices (0: shared)
   T* ns;                  // Muon's Newton-Schulz arena (kNs* problems)
+  const T* ex;            // the embedding matrices (kSrcEmb)
 };
 
 // Muon steps around the Newton-Schulz products (see MuonMat).
@@ -128,11 +129,33 @@ void launch_head_reduce(cudaStream_t st, const HeadReduceArgs& g, int m, int max
 void launch_adamw(cudaStream_t st, const AdamArgs& g, int n_chunks);
 void launch_init(cudaStream_t st, const InitArgs& g, int n_chunks);
 void launch_masks(cudaStream_t st, const MaskGen& mg);
+
+// Periodic embeddings: E of every active member from the rows idx (NULL:
+// rows 0..) of X (member i's rows at idx + i * idx_stride), rows >= B zero;
+// and the gradients of their parameters from dE.
+template <typename T>
+struct EmbArgs {
+  const EmbMember* em;
+  const int32_t* active_ids;
+  const float* X;
+  const int32_t* idx;
+  const StepDyn* dyn;       // non-NULL: X and idx from here
+  const float* params;
+  float* grads;
+  T* ex;                    // embedding arena (forward: written)
+  const T* dz;              // dz arena (backward: dE read)
+  int32_t idx_stride, B, B_pad, d_in;
+};
+// cols_max: the largest in0_pad of the members
+template <typename T>
+void launch_emb_fwd(cudaStream_t st, const EmbArgs<T>& a, int n_active, int cols_max);
+template <typename T>
+void launch_emb_bwd(cudaStream_t st, const EmbArgs<T>& a, int n_active, int cols_max);
 template <typename T>
 void launch_muon(cudaStream_t st, const MuonArgs<T>& a, int n_chunks, int phase);  // 0 momentum, 1 X0, 2 apply
 void launch_refresh_wq(cudaStream_t st, const float* p, __nv_bfloat16* wq0, __nv_bfloat16* wq1, int64_t n);
 template <typename T>
-void launch_fill_ones(cudaStream_t st, const OnesJob* jobs, int n_jobs, T* xb, T* act);
+void launch_fill_ones(cudaStream_t st, const OnesJob* jobs, int n_jobs, T* xb, T* act, T* ex);
 template <typename T>
 void launch_predict_head(cudaStream_t st, const PredictHeadArgs<T>& g, int n_jobs);
 void launch_debug_masks(cudaStream_t st, uint8_t* out, int B, int w, uint64_t seed, uint32_t member,

@@ -136,8 +136,23 @@ tp_status build_ens_pack(tabpack_online* o) {
   tp_config c = o->cfg;
   c.m = n;
   c.fuse_optimizer = 0;
+  // members with periodic embeddings: the same sizes (the frequencies are
+  // placeholders, every parameter comes from the snapshot)
+  std::vector<int32_t> d_emb(n);
+  int64_t n_freq = 0;
+  for (int j = 0; j < n; ++j) {
+    O_PACK(o, o->pack, pack_member_emb(o->pack, o->best[j].member, &d_emb[j]), "pack_member_emb");
+    n_freq += (int64_t)c.d_in * std::max(d_emb[j] - 1, 0);
+  }
   tabpack_t* ep = nullptr;
-  tp_status s = pack_create(&c, depth.data(), width.data(), drop.data(), lr.data(), wd.data(), pack_get_stream(o->pack), &ep);
+  tp_status s;
+  if (n > 0 && d_emb[0] > 0) {
+    std::vector<float> freq((size_t)std::max<int64_t>(n_freq, 1), 0.f);
+    s = pack_create_emb(&c, depth.data(), width.data(), drop.data(), lr.data(), wd.data(), d_emb.data(), freq.data(),
+                        pack_get_stream(o->pack), &ep);
+  } else {
+    s = pack_create(&c, depth.data(), width.data(), drop.data(), lr.data(), wd.data(), pack_get_stream(o->pack), &ep);
+  }
   if (s != TP_OK) return pack_fail(o, nullptr, s, "pack_create (ensemble)");
   o->ens_pack = ep;
   for (int j = 0; j < n; ++j)

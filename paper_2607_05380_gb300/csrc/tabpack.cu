@@ -98,6 +98,26 @@ struct tabpack {
   int n_muon_chunks = 0;
   std::pair<int, int> ns_simt_rng[5] = {};  // CUDA-core Newton-Schulz tiles (fp32 mode)
 
+  // Periodic feature embeddings (pack_create_emb; App. "Feature Embeddings"):
+  // member i's first layer reads E_i [B_cap, in0_pad[i] + 16] (bf16 / fp32,
+  // column in0_pad[i] = 1) in the `ex` arena at e_off[i], E_i[b, j d + k] =
+  // alpha_jk [x_bj, cos(w_j x_bj + b_j)]_k + beta_jk; the first layer's
+  // input gradient dE_i [B_cap, in0_pad[i]] lives in the dz arena at
+  // de_off[i]; the embedding parameters [w, b, alpha, beta]
+  // (d_in (4 d_emb - 2) values) follow the member's head in its run at
+  // emb_off[i].  Without embeddings in0 = d_in and in0_pad = d_in_pad.
+  bool emb = false;
+  std::vector<int32_t> d_emb, in0, in0_pad;
+  std::vector<int64_t> e_off, de_off, emb_off, n_emb;
+  int64_t ex_elems = 0;
+  void* ex = nullptr;
+  int emb_cols_max = 0;     // max in0 over members (grid of the embedding kernels)
+  EmbMember* embm_dev = nullptr;
+  // the prediction arena's embedding matrices (bf16 prediction plan)
+  void* p_ex = nullptr;
+  std::vector<int64_t> p_e_off;
+  EmbMember* embm_p_dev = nullptr;
+
   // Stacked batches (Sec. 3.6: a batch per member), built on first use:
   // xbs holds member i's gathered batch at i * xb_elems ([B_cap, ldx] each,
   // its column d_in_pad = 1), and tcs is the tensor-core plan whose layer-0
@@ -243,6 +263,19 @@ tp_status build_layout(tabpack* h) {
   const int m = c.m;
   h->d_in_pad = (int)round_up(c.d_in, 8);
   h->ldx = h->d_in_pad + kOnesCols;
+  h->in0.assign(m, c.d_in);
+  h->in0_pad.assign(m, h->d_in_pad);
+  h->e_off.assign(m, 0);
+  h->de_off.assign(m, 0);
+  h->emb_off.assign(m, 0);
+  h->n_emb.assign(m, 0);
+  if (h->emb)
+    for (int i = 0; i < m; ++i) {
+      h->in0[i] = c.d_in * h->d_emb[i];
+      h->in0_pad[i] = (int)round_up(h->in0[i], 8);
+      h->n_emb[i] = (int64_t)c.d_in * (4 * h->d_emb[i] - 2);
+      h->emb_cols_max = std::max(h->emb_cols_max, h->in0_pad[i]);
+    }
   h->B_cap = (int)round_up(c.max_batch, kRowTile);
   h->n_blk_cap = h->B_cap / kHeadRows;
   h->W_off.resize(m);
@@ -258,7 +291,7 @@ tp_status build_layout(tabpack* h) {
     const int L = h->depth[i], w = h->width[i];
     h->Lmax = std::max(h->Lmax, L);
     for (int l = 0; l <= L; ++l) {
-      const int in = l == 0 ? c.d_in : w, in_pad = l == 0 ? h->d_in_pad : w;
+      const int in = l == 0 ? h->in0[i] : w, in_pad = l == 0 ? h->in0_pad[i] : w;
       const int out = l == L ? c.d_out : w;
       off = round_up(off, kSegAlign);
       h->W_off[i][l] = off;
@@ -269,11 +302,23 @@ tp_status build_layout(tabpack* h) {
       h->segs.push_back(Segment{off, i, l, out, 1, 1, 1, in, out * in});
       off += out;
     }
+    if (h->emb) {  // the embedding parameters, stepped by AdamW like biases
+      off = round_up(off, kSegAlign);
+      h->emb_off[i] = off;
+      h->segs.push_back(Segment{off, i, L + 1, (int32_t)h->n_emb[i], 1, 1, 1, c.d_in, 0});
+      off += h->n_emb[i];
+    }
     for (int l = 0; l < L; ++l) {
       h->act_off[i][l] = aoff;
       aoff += round_up((int64_t)h->B_cap * ldh_of(h, i), 128);
       h->dz_off[i][l] = zoff;
       zoff += round_up((int64_t)h->B_cap * w, 128);
+    }
+    if (h->emb) {
+      h->de_off[i] = zoff;
+      zoff += round_up((int64_t)h->B_cap * h->in0_pad[i], 128);
+      h->e_off[i] = h->ex_elems;
+      h->ex_elems += round_up((int64_t)h->B_cap * (h->in0_pad[i] + kOnesCols), 128);
     }
     const float p = h->dropout[i];
     double T = std::floor((double)p * 4294967296.0);
@@ -338,10 +383,10 @@ tp_status build_schedule(tabpack* h) {
         const int w = h->width[i];
         GemmProblem P{};
         P.kind = kFwd; P.member = i; P.layer = l;
-        P.M = 0; P.N = w; P.K = l == 0 ? h->d_in_pad : w;
-        P.a_src = l == 0 ? kSrcXb : kSrcAct;
-        P.a_off = l == 0 ? 0 : h->act_off[i][l - 1];
-        P.lda = l == 0 ? h->ldx : ldh_of(h, i);
+        P.M = 0; P.N = w; P.K = l == 0 ? h->in0_pad[i] : w;
+        P.a_src = l == 0 ? (h->emb ? kSrcEmb : kSrcXb) : kSrcAct;
+        P.a_off = l == 0 ? (h->emb ? h->e_off[i] : 0) : h->act_off[i][l - 1];
+        P.lda = l == 0 ? (h->emb ? h->in0_pad[i] + kOnesCols : h->ldx) : ldh_of(h, i);
         P.b_src = kSrcWq; P.b_off = h->W_off[i][l]; P.ldb = P.K;
         P.c_off = h->act_off[i][l]; P.ldc = ldh_of(h, i);
         P.aux_off = h->b_off[i][l];
@@ -355,7 +400,18 @@ tp_status build_schedule(tabpack* h) {
       for (int i : ids) {
         if (h->depth[i] <= l) continue;
         const int w = h->width[i];
-        const int in_pad = l == 0 ? h->d_in_pad : w;
+        const int in_pad = l == 0 ? h->in0_pad[i] : w;
+        if (l == 0 && h->emb) {   // the input gradient of the first layer, for the embeddings
+          GemmProblem P{};
+          P.kind = kDgrad; P.member = i; P.layer = 0;
+          P.M = 0; P.N = in_pad; P.K = w;
+          P.a_src = kSrcDz; P.a_off = h->dz_off[i][0]; P.lda = w;
+          P.b_src = kSrcWq; P.b_off = h->W_off[i][0]; P.ldb = in_pad;
+          P.c_off = h->de_off[i]; P.ldc = in_pad;
+          P.aux_off = -1;
+          probs.push_back(P);
+          add_tiles((int)probs.size() - 1, h->B_cap, in_pad);
+        }
         if (l > 0) {
           GemmProblem P{};
           P.kind = kDgrad; P.member = i; P.layer = l;
@@ -371,8 +427,9 @@ tp_status build_schedule(tabpack* h) {
         Q.kind = kWgrad; Q.member = i; Q.layer = l;
         Q.M = w; Q.N = in_pad + 1; Q.K = 0;  // the last column is the bias gradient
         Q.a_src = kSrcDz; Q.a_off = h->dz_off[i][l]; Q.lda = w;
-        Q.b_src = l == 0 ? kSrcXb : kSrcAct; Q.b_off = l == 0 ? 0 : h->act_off[i][l - 1];
-        Q.ldb = l == 0 ? h->ldx : ldh_of(h, i);
+        Q.b_src = l == 0 ? (h->emb ? kSrcEmb : kSrcXb) : kSrcAct;
+        Q.b_off = l == 0 ? (h->emb ? h->e_off[i] : 0) : h->act_off[i][l - 1];
+        Q.ldb = l == 0 ? (h->emb ? h->in0_pad[i] + kOnesCols : h->ldx) : ldh_of(h, i);
         Q.c_off = h->W_off[i][l]; Q.ldc = in_pad;
         Q.aux_off = h->b_off[i][l];
         probs.push_back(Q);
@@ -540,6 +597,12 @@ tp_status build_schedule(tabpack* h) {
     lay.mask_off = h->mask_words > 0 ? &h->mask_off : nullptr;
     lay.muon = h->muon ? &h->mmats : nullptr;
     lay.ns = h->ns;
+    lay.in0_pad = &h->in0_pad;
+    if (h->emb) {
+      lay.xb = h->ex;
+      lay.x0_off = &h->e_off;
+      lay.de_off = &h->de_off;
+    }
     TP_TRY(tc_build_plan(h->tc, lay, h->err));
   }
   return TP_OK;
@@ -550,6 +613,8 @@ template <typename T>
 tp_status fill_ones(tabpack* h) {
   std::vector<OnesJob> jobs;
   jobs.push_back(OnesJob{0, h->ldx, h->d_in_pad, h->B_cap, 0});
+  if (h->emb)
+    for (int i = 0; i < h->cfg.m; ++i) jobs.push_back(OnesJob{h->e_off[i], h->in0_pad[i] + kOnesCols, h->in0_pad[i], h->B_cap, 2});
   for (int i = 0; i < h->cfg.m; ++i)
     for (int l = 0; l < h->depth[i]; ++l)
       jobs.push_back(OnesJob{h->act_off[i][l], ldh_of(h, i), h->width[i], h->B_cap, 1});
@@ -557,7 +622,7 @@ tp_status fill_ones(tabpack* h) {
   TP_CUDA(h, cudaMalloc(&d, sizeof(OnesJob) * jobs.size()));
   cudaError_t e = cudaMemcpy(d, jobs.data(), sizeof(OnesJob) * jobs.size(), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) {
-    launch_fill_ones<T>(h->st, d, (int)jobs.size(), (T*)h->xb, (T*)h->act);
+    launch_fill_ones<T>(h->st, d, (int)jobs.size(), (T*)h->xb, (T*)h->act, (T*)h->ex);
     h->launches++;
     e = cudaGetLastError();
   }
@@ -606,6 +671,10 @@ tp_status alloc_all(tabpack* h) {
   TP_CUDA(h, cudaMemset(h->t_dev, 0, sizeof(int32_t) * m));
   TP_CUDA(h, cudaMemset(h->bias_corr, 0, sizeof(float2) * m));
   TP_CUDA(h, cudaMemset(h->xb, 0, h->elem * h->xb_elems));
+  if (h->emb) {
+    TP_CUDA(h, cudaMalloc(&h->ex, h->elem * (size_t)h->ex_elems));
+    TP_CUDA(h, cudaMemset(h->ex, 0, h->elem * (size_t)h->ex_elems));
+  }
   TP_CUDA(h, cudaMemset(h->act, 0, h->elem * h->act_elems));
   TP_CUDA(h, cudaMemset(h->dz, 0, h->elem * h->dz_elems));
   TP_CUDA(h, cudaMemset(h->logits, 0, sizeof(float) * (size_t)m * h->B_cap * h->cfg.d_out));
@@ -617,10 +686,11 @@ tp_status alloc_all(tabpack* h) {
 
 void free_predict(tabpack* h) {
   tc_free_plan(h->tcp);
-  for (void* p : {h->p_xb, h->p_act, (void*)h->p_head_dev})
+  for (void* p : {h->p_xb, h->p_act, (void*)h->p_head_dev, h->p_ex, (void*)h->embm_p_dev})
     if (p) cudaFree(p);
-  h->p_xb = h->p_act = nullptr;
+  h->p_xb = h->p_act = h->p_ex = nullptr;
   h->p_head_dev = nullptr;
+  h->embm_p_dev = nullptr;
   h->P_cap = 0;
   h->n_p_head = 0;
   h->p_stale = true;
@@ -645,6 +715,10 @@ void free_all(tabpack* h) {
   tc_free_plan(h->tcs);
   if (h->xbs) cudaFree(h->xbs);
   h->xbs = nullptr;
+  if (h->ex) cudaFree(h->ex);
+  h->ex = nullptr;
+  if (h->embm_dev) cudaFree(h->embm_dev);
+  h->embm_dev = nullptr;
   for (void* p : {h->ns, (void*)h->mmats_dev, (void*)h->mchunk_mat_dev, (void*)h->mpart_dev})
     if (p) cudaFree(p);
   h->ns = nullptr;
@@ -677,6 +751,7 @@ GemmArgs<T> gemm_args(tabpack* h, int B, int B_pad, uint32_t step, int train, bo
   g.seed = h->cfg.seed;
   g.dyn = nullptr;
   g.ns = (T*)h->ns;
+  g.ex = (const T*)h->ex;
   return g;
 }
 
@@ -721,6 +796,26 @@ tp_status run_forward(tabpack* h, int B, int B_pad, uint32_t step, const StepDyn
   return TP_OK;
 }
 
+template <typename T>
+EmbArgs<T> emb_args(tabpack* h, const float* X, const int32_t* idx, const StepDyn* dyn, bool stacked, int B,
+                    int B_pad) {
+  EmbArgs<T> a;
+  a.em = h->embm_dev;
+  a.active_ids = h->active_ids_dev;
+  a.X = X;
+  a.idx = idx;
+  a.dyn = dyn;
+  a.params = h->params;
+  a.grads = h->grads;
+  a.ex = (T*)h->ex;
+  a.dz = (const T*)h->dz;
+  a.idx_stride = stacked ? B : 0;
+  a.B = B;
+  a.B_pad = B_pad;
+  a.d_in = h->cfg.d_in;
+  return a;
+}
+
 // Filling the mask arena for a step (dyn non-NULL: dyn->step + step_add).
 MaskGen mask_gen(tabpack* h, uint32_t step, const StepDyn* dyn, uint32_t step_add) {
   MaskGen mg{};
@@ -745,19 +840,27 @@ MaskGen mask_gen(tabpack* h, uint32_t step, const StepDyn* dyn, uint32_t step_ad
 template <typename T>
 tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* idx, const void* y, int B,
                    uint32_t step, float* loss_out, bool update, const StepDyn* dyn, bool stacked) {
-  TcPlan& plan = stacked ? h->tcs : h->tc;
+  // with embeddings every member has its own first-layer matrix already: the
+  // main plan serves stacked batches too (the rows enter through idx)
+  const bool st_x = stacked && !h->emb;
+  TcPlan& plan = st_x ? h->tcs : h->tc;
   const int B_pad = (int)round_up(B, kRowTile);
   const bool fused = update && h->bf16 && h->fuse_adamw;
   __nv_bfloat16* wq_next = h->bf16 ? h->wq[h->wcur ^ 1] : nullptr;
   int slot;
   prof_begin(h, TP_PH_GATHER, &slot);
-  launch_gather<T>(h->st, X, idx, dyn, B, B_pad, h->cfg.d_in, h->d_in_pad, h->ldx, (T*)(stacked ? h->xbs : h->xb),
+  launch_gather<T>(h->st, X, idx, dyn, B, B_pad, h->cfg.d_in, h->d_in_pad, h->ldx, (T*)(st_x ? h->xbs : h->xb),
                    update ? 1 : 0, h->t_dev, h->bias_corr, h->active_ids_dev, h->n_active, h->cfg.beta1, h->cfg.beta2,
-                   plan.cnt_dev, plan.n_cnt, stacked ? 1 : 0, h->xb_elems);
+                   plan.cnt_dev, plan.n_cnt, st_x ? 1 : 0, h->xb_elems);
+  if (h->emb) {   // the members' first-layer inputs: their periodic embeddings
+    launch_emb_fwd<T>(h->st, emb_args<T>(h, X, idx, dyn, stacked, B, B_pad), h->n_active, h->emb_cols_max);
+    TP_LAUNCHED(h);
+    h->launches++;
+  }
   TP_LAUNCHED(h);
   h->launches++;
-  prof_end(h, slot, 1, TP_PH_GATHER);
-  TP_TRY(run_forward<T>(h, B, B_pad, step, dyn, 1, stacked));
+  prof_end(h, slot, h->emb ? 2 : 1, TP_PH_GATHER);
+  TP_TRY(run_forward<T>(h, B, B_pad, step, dyn, 1, st_x));
   // head + loss
   prof_begin(h, TP_PH_HEAD, &slot);
   HeadArgs<T> hg;
@@ -818,12 +921,19 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
   } else {
     for (int l = h->Lmax - 1; l >= 0; --l) {
       prof_begin(h, TP_PH_BWD, &slot);
-      auto g = gemm_args<T>(h, B, B_pad, step, 1, stacked);
+      auto g = gemm_args<T>(h, B, B_pad, step, 1, st_x);
       launch_gemm_simt<T>(h->st, g, h->bwd_rng[l].first, h->bwd_rng[l].second);
       TP_LAUNCHED(h);
       h->launches++;
       prof_end(h, slot, 1, TP_PH_BWD);
     }
+  }
+  if (h->emb) {   // the embedding parameters' gradients from the first layer's input gradient
+    prof_begin(h, TP_PH_BWD, &slot);
+    launch_emb_bwd<T>(h->st, emb_args<T>(h, X, idx, dyn, stacked, B, B_pad), h->n_active, h->emb_cols_max);
+    TP_LAUNCHED(h);
+    h->launches++;
+    prof_end(h, slot, 1, TP_PH_BWD);
   }
   if (update && h->muon && h->n_muon_chunks > 0) {
     // Muon on the hidden-layer weights: momentum and |U|, X0, the
@@ -970,7 +1080,7 @@ tp_status ensure_stacked(tabpack* h) {
     TP_CUDA(h, cudaMalloc(&d, sizeof(OnesJob) * jobs.size()));
     cudaError_t e = cudaMemcpy(d, jobs.data(), sizeof(OnesJob) * jobs.size(), cudaMemcpyHostToDevice);
     if (e == cudaSuccess) {
-      launch_fill_ones<T>(h->st, d, (int)jobs.size(), (T*)h->xbs, (T*)h->act);
+      launch_fill_ones<T>(h->st, d, (int)jobs.size(), (T*)h->xbs, (T*)h->act, nullptr);
       h->launches++;
       e = cudaGetLastError();
     }
@@ -1007,6 +1117,20 @@ tp_status ensure_stacked(tabpack* h) {
 }
 
 constexpr int kPredictRows = 8192;
+constexpr int64_t kPredictEmbBytes = int64_t(1) << 30;   // cap of the prediction embedding arena
+
+// Rows of one prediction chunk for N rows: at most kPredictRows, and with
+// embeddings at most what keeps the embedding arena under kPredictEmbBytes.
+int predict_rows(const tabpack* h, int64_t N) {
+  int64_t rows = std::min<int64_t>(round_up(N, kRowTile), kPredictRows);
+  if (h->emb) {
+    int64_t per_row = 0;
+    for (int i = 0; i < h->cfg.m; ++i) per_row += h->in0_pad[i] + kOnesCols;
+    const int64_t fit = kPredictEmbBytes / ((int64_t)sizeof(__nv_bfloat16) * per_row) / kRowTile * kRowTile;
+    rows = std::min(rows, std::max<int64_t>(fit, kRowTile));
+  }
+  return (int)rows;
+}
 
 // (Re)build the bf16 prediction plan for chunks of at least P_need rows.
 tp_status build_predict(tabpack* h, int P_need) {
@@ -1031,6 +1155,36 @@ tp_status build_predict(tabpack* h, int P_need) {
     // columns the forward never writes (ones / pad columns) stay zero
     TP_CUDA(h, cudaMemset(h->p_xb, 0, xb_bytes));
     TP_CUDA(h, cudaMemset(h->p_act, 0, act_bytes));
+    if (h->emb) {
+      // the members' embedding matrices for a chunk, with their ones column
+      h->p_e_off.assign(m, 0);
+      int64_t eoff = 0;
+      for (int i = 0; i < m; ++i) {
+        h->p_e_off[i] = eoff;
+        eoff += round_up((int64_t)h->P_cap * (h->in0_pad[i] + kOnesCols), 128);
+      }
+      TP_CUDA(h, cudaMalloc(&h->p_ex, sizeof(__nv_bfloat16) * (size_t)eoff));
+      TP_CUDA(h, cudaMemset(h->p_ex, 0, sizeof(__nv_bfloat16) * (size_t)eoff));
+      std::vector<EmbMember> em(m);
+      std::vector<OnesJob> jobs;
+      for (int i = 0; i < m; ++i) {
+        em[i] = EmbMember{h->d_emb[i], h->in0[i], h->in0_pad[i], 0, h->p_e_off[i], 0, h->emb_off[i]};
+        jobs.push_back(OnesJob{h->p_e_off[i], h->in0_pad[i] + kOnesCols, h->in0_pad[i], h->P_cap, 2});
+      }
+      TP_CUDA(h, cudaMalloc((void**)&h->embm_p_dev, sizeof(EmbMember) * m));
+      TP_CUDA(h, cudaMemcpy(h->embm_p_dev, em.data(), sizeof(EmbMember) * m, cudaMemcpyHostToDevice));
+      OnesJob* d = nullptr;
+      TP_CUDA(h, cudaMalloc(&d, sizeof(OnesJob) * jobs.size()));
+      cudaError_t e = cudaMemcpy(d, jobs.data(), sizeof(OnesJob) * jobs.size(), cudaMemcpyHostToDevice);
+      if (e == cudaSuccess) {
+        launch_fill_ones<__nv_bfloat16>(h->st, d, (int)jobs.size(), nullptr, nullptr, (__nv_bfloat16*)h->p_ex);
+        h->launches++;
+        e = cudaGetLastError();
+      }
+      if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+      cudaFree(d);
+      if (e != cudaSuccess) return fail(h, TP_ECUDA, "prediction embedding arena: %s", cudaGetErrorString(e));
+    }
   }
   TcLayout lay;
   lay.depth = &h->depth;
@@ -1050,6 +1204,11 @@ tp_status build_predict(tabpack* h, int P_need) {
   lay.act = h->p_act;
   lay.dz = nullptr;
   lay.fwd_only = true;
+  lay.in0_pad = &h->in0_pad;
+  if (h->emb) {
+    lay.xb = h->p_ex;
+    lay.x0_off = &h->p_e_off;
+  }
   TP_CUDA(h, cudaStreamSynchronize(h->st));
   TP_TRY(tc_build_plan(h->tcp, lay, h->err));
   std::vector<HeadJob> hj;
@@ -1076,7 +1235,7 @@ tp_status build_predict(tabpack* h, int P_need) {
 
 // bf16 prediction: chunks of P_cap rows through the forward-only plan.
 tp_status run_predict_tc(tabpack* h, const float* X, int64_t N, float* out) {
-  TP_TRY(build_predict(h, (int)std::min<int64_t>(round_up(N, kRowTile), kPredictRows)));
+  TP_TRY(build_predict(h, predict_rows(h, N)));
   for (int64_t n0 = 0; n0 < N; n0 += h->P_cap) {
     const int rows = (int)std::min<int64_t>(h->P_cap, N - n0);
     const int B_pad = (int)round_up(rows, kRowTile);
@@ -1086,6 +1245,15 @@ tp_status run_predict_tc(tabpack* h, const float* X, int64_t N, float* out) {
                                  h->ldx, (__nv_bfloat16*)h->p_xb, 0, h->t_dev, h->bias_corr, h->active_ids_dev, 0,
                                  h->cfg.beta1, h->cfg.beta2, h->tcp.cnt_dev, h->tcp.n_cnt);
     TP_LAUNCHED(h);
+    int nl = 3;
+    if (h->emb) {
+      EmbArgs<__nv_bfloat16> ea = emb_args<__nv_bfloat16>(h, X + n0 * h->cfg.d_in, nullptr, nullptr, false, rows, B_pad);
+      ea.em = h->embm_p_dev;
+      ea.ex = (__nv_bfloat16*)h->p_ex;
+      launch_emb_fwd<__nv_bfloat16>(h->st, ea, h->n_active, h->emb_cols_max);
+      TP_LAUNCHED(h);
+      ++nl;
+    }
     TP_TRY(tc_run_fwd(h->tcp, h->st, rows, B_pad, h->wcur, 0, nullptr, 0, h->params, h->mem_dev, h->p_act, h->err));
     TP_LAUNCHED(h);
     PredictHeadArgs<__nv_bfloat16> pg;
@@ -1102,8 +1270,8 @@ tp_status run_predict_tc(tabpack* h, const float* X, int64_t N, float* out) {
     pg._pad = 0;
     launch_predict_head<__nv_bfloat16>(h->st, pg, h->n_p_head);
     TP_LAUNCHED(h);
-    h->launches += 3;
-    prof_end(h, slot, 3, TP_PH_PREDICT);
+    h->launches += nl;
+    prof_end(h, slot, nl, TP_PH_PREDICT);
   }
   return TP_OK;
 }
@@ -1122,7 +1290,13 @@ tp_status run_predict(tabpack* h, const float* X, int64_t N, float* out) {
                      h->tc.n_cnt);
     TP_LAUNCHED(h);
     h->launches++;
-    prof_end(h, slot, 1, TP_PH_PREDICT);
+    if (h->emb) {
+      launch_emb_fwd<T>(h->st, emb_args<T>(h, X + n0 * h->cfg.d_in, nullptr, nullptr, false, rows, B_pad),
+                        h->n_active, h->emb_cols_max);
+      TP_LAUNCHED(h);
+      h->launches++;
+    }
+    prof_end(h, slot, h->emb ? 2 : 1, TP_PH_PREDICT);
     TP_TRY(run_forward<T>(h, rows, B_pad, 0u, nullptr, 0));
     prof_begin(h, TP_PH_PREDICT, &slot);
     PredictHeadArgs<T> pg;
@@ -1167,7 +1341,8 @@ tp_status check_step_args(tabpack* h, const float* X, int64_t n_rows, const int3
 std::pair<int64_t, int64_t> member_run(const tabpack* h, int i) {
   const int L = h->depth[i];
   const int64_t first = h->W_off[i][0];
-  return {first, h->b_off[i][L] + h->cfg.d_out - first};
+  const int64_t last = h->emb ? h->emb_off[i] + h->n_emb[i] : h->b_off[i][L] + h->cfg.d_out;
+  return {first, last - first};
 }
 
 tp_status check_ml(tabpack* h, int member, int layer) {
@@ -1193,8 +1368,9 @@ void tp::record_thread_error(const char* msg) { g_thread_error = msg; }
 // ====================================================================== ABI
 extern "C" {
 
-tp_status pack_create(const tp_config* cfg, const int32_t* depth, const int32_t* width, const float* dropout,
-                      const float* lr, const float* wd, void* cuda_stream, tabpack_t** out) {
+static tp_status create_impl(const tp_config* cfg, const int32_t* depth, const int32_t* width, const float* dropout,
+                             const float* lr, const float* wd, const int32_t* d_emb, const float* freq,
+                             void* cuda_stream, tabpack_t** out) {
   if (out) *out = nullptr;
   if (!cfg || !depth || !width || !dropout || !lr || !wd || !out)
     return fail(nullptr, TP_EINVAL, "null argument");
@@ -1232,6 +1408,11 @@ tp_status pack_create(const tp_config* cfg, const int32_t* depth, const int32_t*
   h->lr.assign(lr, lr + cfg->m);
   h->wd.assign(wd, wd + cfg->m);
   h->active.assign(cfg->m, 1);
+  if (d_emb) {
+    h->emb = true;
+    h->d_emb.assign(d_emb, d_emb + cfg->m);
+    h->fuse_adamw = false;   // the embedding parameters take the stand-alone AdamW pass
+  }
   tp_status s = build_layout(h);
   if (s == TP_OK) s = alloc_all(h);
   if (s == TP_OK) s = build_schedule(h);
@@ -1245,6 +1426,25 @@ tp_status pack_create(const tp_config* cfg, const int32_t* depth, const int32_t*
     if (le == cudaSuccess) le = cudaStreamSynchronize(h->st);
     if (le != cudaSuccess) s = fail(h, TP_ECUDA, "init: %s", cudaGetErrorString(le));
   }
+  if (s == TP_OK && h->emb) {
+    // embedding parameters: the caller's frequencies, zero phases and scales
+    std::vector<EmbMember> em(cfg->m);
+    const float* fr = freq;
+    for (int i = 0; i < cfg->m && s == TP_OK; ++i) {
+      std::vector<float> v((size_t)h->n_emb[i], 0.f);
+      const int64_t nf = (int64_t)cfg->d_in * (h->d_emb[i] - 1);
+      std::copy(fr, fr + nf, v.begin());
+      fr += nf;
+      if (cudaMemcpy(h->params + h->emb_off[i], v.data(), v.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+        s = fail(h, TP_ECUDA, "embedding init copy failed");
+      em[i] = EmbMember{h->d_emb[i], h->in0[i], h->in0_pad[i], 0, h->e_off[i], h->de_off[i], h->emb_off[i]};
+    }
+    if (s == TP_OK && cudaMalloc((void**)&h->embm_dev, sizeof(EmbMember) * cfg->m) != cudaSuccess)
+      s = fail(h, TP_ENOMEM, "cudaMalloc(embedding records) failed");
+    if (s == TP_OK &&
+        cudaMemcpy(h->embm_dev, em.data(), sizeof(EmbMember) * cfg->m, cudaMemcpyHostToDevice) != cudaSuccess)
+      s = fail(h, TP_ECUDA, "embedding records copy failed");
+  }
   if (s != TP_OK) {
     g_thread_error = h->err;
     free_all(h);
@@ -1252,6 +1452,45 @@ tp_status pack_create(const tp_config* cfg, const int32_t* depth, const int32_t*
     return s;
   }
   *out = h;
+  return TP_OK;
+}
+
+tp_status pack_create(const tp_config* cfg, const int32_t* depth, const int32_t* width, const float* dropout,
+                      const float* lr, const float* wd, void* cuda_stream, tabpack_t** out) {
+  return create_impl(cfg, depth, width, dropout, lr, wd, nullptr, nullptr, cuda_stream, out);
+}
+
+tp_status pack_create_emb(const tp_config* cfg, const int32_t* depth, const int32_t* width, const float* dropout,
+                          const float* lr, const float* wd, const int32_t* d_emb, const float* freq,
+                          void* cuda_stream, tabpack_t** out) {
+  if (out) *out = nullptr;
+  if (!cfg || !d_emb || !freq) return fail(nullptr, TP_EINVAL, "null argument");
+  for (int i = 0; i < cfg->m; ++i)
+    if (d_emb[i] < 1 || d_emb[i] > 64) return fail(nullptr, TP_EINVAL, "d_emb[%d]=%d not in 1..64", i, d_emb[i]);
+  return create_impl(cfg, depth, width, dropout, lr, wd, d_emb, freq, cuda_stream, out);
+}
+
+tp_status pack_get_emb(tabpack_t* h, int32_t member, int32_t grads, float* out) {
+  TP_TRY(check_ml(h, member, 0));
+  if (!h->emb || !out) return fail(h, TP_EINVAL, "the pack has no embeddings");
+  TP_TRY(sync_check(h));
+  TP_CUDA(h, cudaMemcpy(out, (grads ? h->grads : h->params) + h->emb_off[member], h->n_emb[member] * 4,
+                        cudaMemcpyDeviceToHost));
+  return TP_OK;
+}
+
+tp_status pack_set_emb(tabpack_t* h, int32_t member, const float* in) {
+  TP_TRY(check_ml(h, member, 0));
+  if (!h->emb || !in) return fail(h, TP_EINVAL, "the pack has no embeddings");
+  TP_TRY(sync_check(h));
+  TP_CUDA(h, cudaMemcpy(h->params + h->emb_off[member], in, h->n_emb[member] * 4, cudaMemcpyHostToDevice));
+  return TP_OK;
+}
+
+tp_status pack_member_emb(const tabpack_t* h, int32_t member, int32_t* d_emb) {
+  if (!h || !d_emb) return fail(const_cast<tabpack_t*>(h), TP_EINVAL, "null argument");
+  if (member < 0 || member >= h->cfg.m) return fail(const_cast<tabpack_t*>(h), TP_EINVAL, "member %d out of range", member);
+  *d_emb = h->emb ? h->d_emb[member] : 0;
   return TP_OK;
 }
 
@@ -1289,10 +1528,10 @@ tp_status pack_train_step_stacked(tabpack_t* h, const float* X, int64_t n_rows, 
   TP_TRY(check_step_args(h, X, n_rows, idx, y, B));
   if (h->n_active == 0) return fail(h, TP_ESTATE, "no active member");
   if (h->bf16) {
-    TP_TRY(ensure_stacked<__nv_bfloat16>(h));
+    if (!h->emb) TP_TRY(ensure_stacked<__nv_bfloat16>(h));
     return step_entry<__nv_bfloat16>(h, X, n_rows, idx, y, B, step, loss_out, true, true);
   }
-  TP_TRY(ensure_stacked<float>(h));
+  if (!h->emb) TP_TRY(ensure_stacked<float>(h));
   return step_entry<float>(h, X, n_rows, idx, y, B, step, loss_out, true, true);
 }
 
@@ -1301,10 +1540,10 @@ tp_status pack_forward_backward_stacked(tabpack_t* h, const float* X, int64_t n_
   TP_TRY(check_step_args(h, X, n_rows, idx, y, B));
   if (h->n_active == 0) return fail(h, TP_ESTATE, "no active member");
   if (h->bf16) {
-    TP_TRY(ensure_stacked<__nv_bfloat16>(h));
+    if (!h->emb) TP_TRY(ensure_stacked<__nv_bfloat16>(h));
     return step_entry<__nv_bfloat16>(h, X, n_rows, idx, y, B, step, loss_out, false, true);
   }
-  TP_TRY(ensure_stacked<float>(h));
+  if (!h->emb) TP_TRY(ensure_stacked<float>(h));
   return step_entry<float>(h, X, n_rows, idx, y, B, step, loss_out, false, true);
 }
 
@@ -1325,8 +1564,8 @@ tp_status pack_set_muon(tabpack_t* h, const float* lr_muon, float momentum, int3
         mt.member = i;
         mt.layer = l;
         mt.rows = h->width[i];
-        mt.cols = l == 0 ? h->d_in_pad : h->width[i];
-        const int real_cols = l == 0 ? h->cfg.d_in : h->width[i];
+        mt.cols = l == 0 ? h->in0_pad[i] : h->width[i];
+        const int real_cols = l == 0 ? h->in0[i] : h->width[i];
         mt.tr = mt.rows > mt.cols;
         mt.r = std::min(mt.rows, mt.cols);
         mt.c = std::max(mt.rows, mt.cols);
@@ -1378,7 +1617,7 @@ tp_status pack_debug_muon_dir(tabpack_t* h, int32_t member, int32_t layer, float
   } else {
     TP_CUDA(h, cudaMemcpy(X.data(), (float*)h->ns + mt->x_off[xf], n * 4, cudaMemcpyDeviceToHost));
   }
-  const int in = layer == 0 ? h->cfg.d_in : h->width[member];
+  const int in = layer == 0 ? h->in0[member] : h->width[member];
   for (int i = 0; i < mt->rows; ++i)
     for (int j = 0; j < in; ++j) out[(int64_t)i * in + j] = X[mt->tr ? (int64_t)j * mt->c + i : (int64_t)i * mt->c + j];
   return TP_OK;
@@ -1404,7 +1643,7 @@ static tp_status copy_layer(tabpack_t* h, int member, int layer, float* W, float
   TP_TRY(check_ml(h, member, layer));
   TP_TRY(sync_check(h));
   const int L = h->depth[member], w = h->width[member];
-  const int in = layer == 0 ? h->cfg.d_in : w, in_pad = layer == 0 ? h->d_in_pad : w;
+  const int in = layer == 0 ? h->in0[member] : w, in_pad = layer == 0 ? h->in0_pad[member] : w;
   const int out = layer == L ? h->cfg.d_out : w;
   if (W) {
     std::vector<float> tmp((size_t)out * in_pad);
@@ -1429,7 +1668,7 @@ tp_status pack_set_params(tabpack_t* h, int32_t member, int32_t layer, const flo
   TP_TRY(check_ml(h, member, layer));
   TP_TRY(sync_check(h));
   const int L = h->depth[member], w = h->width[member];
-  const int in = layer == 0 ? h->cfg.d_in : w, in_pad = layer == 0 ? h->d_in_pad : w;
+  const int in = layer == 0 ? h->in0[member] : w, in_pad = layer == 0 ? h->in0_pad[member] : w;
   const int out = layer == L ? h->cfg.d_out : w;
   if (W) {
     std::vector<float> tmp((size_t)out * in_pad, 0.f);

@@ -614,7 +614,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           // tile origins and chunks are 32-column aligned for forward tiles
           if (row_ok && g.train && tile.mask_off >= 0)
             bits[ci] = __ldg(g.masks + tile.mask_off + (int64_t)(col0 >> 5) * g.mask_rows + r);
-        } else if (tile.kind == kDgrad && row_ok) {
+        } else if (tile.kind == kDgrad && row_ok && tile.aux_off >= 0) {
           const __nv_bfloat16* hm = g.act + tile.aux_off + (int64_t)r * tile.ld_aux + col0;
           uint32_t mb = 0;
 #pragma unroll
@@ -793,6 +793,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         } else if (tile.kind == kDgrad) {
           if (!live) continue;
           const uint32_t mb = pick(bits, ci);
+          const float dsc = tile.aux_off >= 0 ? md.scale : 1.f;   // the first layer's input gradient: 1
           __nv_bfloat16* out = g.dz + tile.c_off + (int64_t)r * tile.ldc + col0;
 #pragma unroll
           for (int s = 0; s < 4; ++s) {
@@ -801,8 +802,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
               const int j = 8 * s + 2 * e;
-              const float x0 = ((mb >> j) & 1u) ? __uint_as_float(v[j]) * md.scale : 0.f;
-              const float x1 = ((mb >> (j + 1)) & 1u) ? __uint_as_float(v[j + 1]) * md.scale : 0.f;
+              const float x0 = ((mb >> j) & 1u) ? __uint_as_float(v[j]) * dsc : 0.f;
+              const float x1 = ((mb >> (j + 1)) & 1u) ? __uint_as_float(v[j + 1]) * dsc : 0.f;
               pk[e] = pack_bf16x2(x0, x1);
             }
             *reinterpret_cast<uint4*>(out + 8 * s) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
@@ -891,6 +892,7 @@ void split_n(int n, std::vector<std::pair<int, int>>& out, int align = 16) {
 
 tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
   const int m = lay.m;
+  auto in0p = [&](int i) { return lay.in0_pad ? (*lay.in0_pad)[i] : lay.d_in_pad; };
   const auto& depth = *lay.depth;
   const auto& width = *lay.width;
   const auto& active = *lay.active;
@@ -910,10 +912,17 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
     for (int set = 0; set < 2; ++set) {
       const int br = set ? 128 : 64;
       const int base = (int)maps.size();
-      // the batch matrix: one, or one per member (stacked batches: map index = member)
-      for (int i = 0; i < (lay.xb_stride ? m : 1); ++i) {
-        const __nv_bfloat16* xbi = (const __nv_bfloat16*)lay.xb + (int64_t)i * lay.xb_stride;
-        if (!encode_map(&mp, xbi, lay.ldx, lay.B_cap, lay.ldx, br, err)) return TP_ECUDA;
+      // the first layer's input: one batch matrix, or one per member
+      // (stacked batches, embeddings: map index = member)
+      for (int i = 0; i < (lay.xb_stride || lay.x0_off ? m : 1); ++i) {
+        if (lay.x0_off) {
+          const int ld = (*lay.in0_pad)[i] + kOnesCols;
+          if (!encode_map(&mp, (const __nv_bfloat16*)lay.xb + (*lay.x0_off)[i], ld, lay.B_cap, ld, br, err))
+            return TP_ECUDA;
+        } else {
+          const __nv_bfloat16* xbi = (const __nv_bfloat16*)lay.xb + (int64_t)i * lay.xb_stride;
+          if (!encode_map(&mp, xbi, lay.ldx, lay.B_cap, lay.ldx, br, err)) return TP_ECUDA;
+        }
         maps.push_back(mp);
       }
       for (int i = 0; i < m; ++i)
@@ -932,7 +941,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
       for (int copy = 0; copy < 2; ++copy)
         for (int i = 0; i < m; ++i)
           for (int l = 0; l < depth[i]; ++l) {
-            const int w = width[i], in_pad = l == 0 ? lay.d_in_pad : w;
+            const int w = width[i], in_pad = l == 0 ? in0p(i) : w;
             if (!encode_map(&mp, lay.wq[copy] + (*lay.W_off)[i][l], in_pad, w, in_pad, br, err)) return TP_ECUDA;
             if (set == 0 && copy == 0) plan.map_w[(size_t)i * kMaxDepth + l] = (int)maps.size();
             maps.push_back(mp);
@@ -992,7 +1001,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
     int64_t fwd_kblocks = 0;
     for (int i = 0; i < m; ++i)
       for (int l = 0; l < depth[i]; ++l) {
-        const int in_pad = l == 0 ? lay.d_in_pad : width[i];
+        const int in_pad = l == 0 ? in0p(i) : width[i];
         fwd_kblocks += (lay.B_cap / kRowTile) * ceil_div(width[i], 256) * ceil_div(in_pad, 64);
       }
     plan.cta = fwd_kblocks >= 100 * (int64_t)plan.n_sm ? 2 : 1;
@@ -1083,8 +1092,8 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
       t.kind = kFwd; t.member = i; t.layer = l;
       t.mask_off = lay.mask_off ? (int32_t)(*lay.mask_off)[i][l] : -1;
       t.m_real = 0; t.n_real = w;
-      t.k_len = l == 0 ? lay.d_in_pad : w;
-      t.map_a = l == 0 ? (lay.xb_stride ? i : 0) : plan.map_act[(size_t)i * kMaxDepth + l - 1];
+      t.k_len = l == 0 ? in0p(i) : w;
+      t.map_a = l == 0 ? (lay.xb_stride || lay.x0_off ? i : 0) : plan.map_act[(size_t)i * kMaxDepth + l - 1];
       t.map_b = plan.map_w[(size_t)i * kMaxDepth + l];
       t.ldc = w + kOnesCols;
       t.ld_aux = 0;
@@ -1107,10 +1116,30 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
     for (int i = 0; i < m; ++i) {
       if (!active[i] || depth[i] <= lev) continue;
       const int l = depth[i] - 1 - lev;
-      const int w = width[i], in_pad = l == 0 ? lay.d_in_pad : w;
+      const int w = width[i], in_pad = l == 0 ? in0p(i) : w;
       split_n(w, ns);
       const int need = kEpiWarps * (int)ns.size();  // dgrad column tiles of layer l + 1 per row block of dz_l
       const bool from_head = l == depth[i] - 1;
+      if (l == 0 && lay.de_off) {   // the first layer's input gradient (embeddings): no mask, no scale
+        std::vector<std::pair<int, int>> ne;
+        split_n(in_pad, ne);
+        TcTile t{};
+        t.kind = kDgrad; t.member = i; t.layer = 0;
+        t.mask_off = -1;
+        t.m_real = 0; t.n_real = in_pad;
+        t.k_len = w;
+        t.map_a = plan.map_dz[(size_t)i * kMaxDepth + 0];
+        t.map_b = plan.map_w[(size_t)i * kMaxDepth + 0];
+        t.ldc = in_pad;
+        t.ld_aux = 0;
+        t.dep = from_head ? -1 : cnt_dz(i, 0);
+        t.dep_n = 1;
+        t.dep_need = need;
+        t.sig = -1;
+        t.c_off = (*lay.de_off)[i];
+        t.aux_off = -1;
+        emit(vd, t, lay.B_cap / kRowTile, ne);
+      }
       if (l > 0) {
         TcTile t{};
         t.kind = kDgrad; t.member = i; t.layer = l;
@@ -1137,7 +1166,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
       t.m_real = w; t.n_real = in_pad + 1;
       t.k_len = 0;
       t.map_a = plan.map_dz[(size_t)i * kMaxDepth + l];
-      t.map_b = l == 0 ? (lay.xb_stride ? i : 0) : plan.map_act[(size_t)i * kMaxDepth + l - 1];
+      t.map_b = l == 0 ? (lay.xb_stride || lay.x0_off ? i : 0) : plan.map_act[(size_t)i * kMaxDepth + l - 1];
       t.ldc = in_pad;
       t.ld_aux = 0;
       t.dep = from_head ? -1 : cnt_dz(i, l);  // every row block of dz_l

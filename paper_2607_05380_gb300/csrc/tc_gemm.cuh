@@ -86,6 +86,12 @@ struct TcLayout {          // what the plan needs to know about the pack's arena
   const std::vector<MuonMat>* muon = nullptr;
   const void* ns = nullptr;
   int64_t xb_stride = 0;   // > 0: a batch matrix per member (stacked batches), this many elements apart
+  // Periodic embeddings: member i's first layer reads the matrix at xb +
+  // x0_off[i] ([B_cap, in0_pad[i] + 16]) and, with de_off, its input gradient
+  // dE_i [B_cap, in0_pad[i]] is written to dz + de_off[i] (NULL: none)
+  const std::vector<int32_t>* in0_pad = nullptr;
+  const std::vector<int64_t>* x0_off = nullptr;
+  const std::vector<int64_t>* de_off = nullptr;
   // per (member, layer): word offset of the dropout keep words, -1 for none (NULL: no masks)
   const std::vector<std::array<int64_t, kMaxDepth>>* mask_off = nullptr;
 };

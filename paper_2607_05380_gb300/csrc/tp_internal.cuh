@@ -35,7 +35,7 @@ constexpr int kSegAlign = 32;   // elements
 constexpr int kOnesCols = 16;   // the ones column plus zero padding to 16 columns
 
 enum GemmKind : int32_t { kFwd = 0, kDgrad = 1, kWgrad = 2, kNsGram = 3, kNsPoly = 4, kNsApply = 5 };
-enum Src : int32_t { kSrcXb = 0, kSrcAct = 1, kSrcDz = 2, kSrcWq = 3, kSrcNs = 4 };
+enum Src : int32_t { kSrcXb = 0, kSrcAct = 1, kSrcDz = 2, kSrcWq = 3, kSrcNs = 4, kSrcEmb = 5 };
 
 // Muon (Sec. 3.4; Jordan et al. 2024) on the hidden-layer weight matrices:
 // the products of one Newton-Schulz iteration over the normalised momentum
@@ -122,7 +122,7 @@ struct HeadReduceJob {
 struct OnesJob {          // column `col` of rows 0..rows-1 of a matrix with pitch `ld` := 1
   int64_t off;
   int32_t ld, col, rows;
-  int32_t arena;          // 0: xb, 1: act
+  int32_t arena;          // 0: xb, 1: act, 2: the embedding matrices
 };
 
 // The per-call arguments of a training step, read from device memory by the
@@ -188,6 +188,17 @@ __device__ __forceinline__ uint32_t keep_bits4(uint64_t seed, uint32_t member, u
   return (uint32_t)(r.x >= T) | ((uint32_t)(r.y >= T) << 1) | ((uint32_t)(r.z >= T) << 2) |
          ((uint32_t)(r.w >= T) << 3);
 }
+
+// Periodic feature embeddings of one member (App. "Feature Embeddings"):
+// E[b, j d + k] = alpha_jk f_k + beta_jk with f_0 = x_bj and f_k =
+// cos(w_j,k-1 x_bj + b_j,k-1); the parameters [w, b, alpha, beta] at p_off
+// in the parameter (and gradient) arena.
+struct EmbMember {
+  int32_t d, in0, in0_pad, _pad;
+  int64_t e_off;          // E in the embedding arena, pitch in0_pad + 16
+  int64_t de_off;         // dE in the dz arena, pitch in0_pad
+  int64_t p_off;
+};
 
 // Dropout keep bits of 32 consecutive columns of one row, word bit j =
 // keep(32 * chunk + j): the eight Philox draws of the chunk, one after the

@@ -1,0 +1,333 @@
+"""Periodic feature embeddings on the GPU (App. "Feature Embeddings") against
+the oracle's (pinned in tests/test_oracle_emb.py by finite differences and by
+reduction to a plain pack).
+
+Bars as in tests/test_gpu_parity.py: floats within 1e-4 (fp32 mode) and
+2e-2 (bf16 mode, against the oracle's bf16-storage mode, where E and dE are
+stored in bf16 as on the GPU) in the relative error |g - o| / max(|o|,
+rms(o)); initial values bit-exact.  The embedding parameters' gradients are
+compared like the other gradients: elementwise for members without flipped
+ReLU decisions, norm-wise for members with flips at near-ties.
+"""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+import oracle  # noqa: E402
+from workloads import random_pack, sample_emb  # noqa: E402
+from test_gpu_parity import TOL, _compare_step, make_data, rel_err, to_dev  # noqa: E402
+from test_gpu_online import ens_mean  # noqa: E402
+
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module")
+def tp():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    from paper_2607_05380_gb300 import build
+    build.build()
+    import paper_2607_05380_gb300 as tpm
+    tpm.load_library()
+    return tpm
+
+
+def emb_pair(tp, task, d_in, d_out, hp, em, prec, max_batch, seed=2):
+    pk = tp.Pack(d_in, d_out, task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
+                 max_batch=max_batch, seed=seed, precision=prec, d_emb=em["d_emb"], freq=em["freq"])
+    orc = oracle.OraclePack(d_in, d_out, task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
+                            seed=seed, bf16_storage=(prec == "bf16"), d_emb=em["d_emb"],
+                            freq=em["freq"].astype(np.float64))
+    return pk, orc
+
+
+def randomise_emb(pk, orc, em, d_in, seed):
+    """Non-zero b, alpha and beta (from the zero start the cosine parts get
+    no gradient), the same fp32 values on both sides."""
+    rng = np.random.default_rng(seed)
+    for i, d in enumerate(em["d_emb"]):
+        d = int(d)
+        w, _, _, _ = orc.emb(i)
+        parts = [w, rng.uniform(-np.pi, np.pi, (d_in, d - 1)), rng.standard_normal((d_in, d)) * 0.7,
+                 rng.standard_normal((d_in, d)) * 0.2]
+        parts = [np.asarray(p, dtype=np.float32) for p in parts]
+        pk.set_emb(i, *parts)
+        orc.set_emb(i, *[p.astype(np.float64) for p in parts])
+
+
+def emb_errs(pk, orc, members, flips_ok=()):
+    """Largest relative error of each member's embedding gradients."""
+    out = {}
+    for i in members:
+        e = 0.0
+        for g, o in zip(pk.emb(i, grads=True), orc.emb(i, grads=True)):
+            if g.size == 0:
+                continue
+            if i in flips_ok:
+                e = max(e, float(np.linalg.norm(g - o) / max(np.linalg.norm(o), 1e-30)))
+            else:
+                e = max(e, rel_err(g, o))
+        out[i] = e
+    return out
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_emb_init_bit_exact(tp, prec):
+    """The first layer's init over fan-in d_in d_emb, and the embedding
+    parameters as given (w = freq, b = alpha = beta = 0)."""
+    d_in, d_out, m = 11, 3, 4
+    hp = random_pack(m, d_in, d_out, seed=3)
+    em = sample_emb(m, d_in, seed=3)
+    pk, orc = emb_pair(tp, "multiclass", d_in, d_out, hp, em, prec, 64)
+    off = 0
+    for i in range(m):
+        d = int(em["d_emb"][i])
+        for l in range(int(hp["depth"][i]) + 1):
+            W, b = pk.get_params(i, l)
+            Wo, bo = orc.get_params(i, l)
+            np.testing.assert_array_equal(W, Wo.astype(np.float32))
+            np.testing.assert_array_equal(b, bo.astype(np.float32))
+        w, bb, a, be = pk.emb(i)
+        np.testing.assert_array_equal(w.ravel(), em["freq"][off:off + d_in * (d - 1)])
+        off += d_in * (d - 1)
+        assert not bb.any() and not a.any() and not be.any()
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+@pytest.mark.parametrize("task,d_out", [("binary", 1), ("multiclass", 7), ("regression", 1)])
+@pytest.mark.parametrize("B", [200, 1])
+def test_emb_one_step(tp, prec, task, d_out, B):
+    """Logits, losses, every gradient (weights, biases, embeddings) of one
+    step; d_emb from the paper's range 8..32 plus 1 and 3 (the x component
+    alone; an input width that is not a multiple of 8), several 128-row
+    tiles and a ragged tail (B = 200), and B = 1."""
+    d_in, m = 13, 6
+    hp = random_pack(m, d_in, d_out, seed=80 + d_out, width=(16, 128, 16), depth=(1, 3))
+    em = sample_emb_fixed(m, d_in, [1, 3, 8, 16, 24, 32], seed=4)
+    pk, orc = emb_pair(tp, task, d_in, d_out, hp, em, prec, 256)
+    randomise_emb(pk, orc, em, d_in, seed=5)
+    X, y = make_data(task, 400, d_in, d_out, 1)
+    idx = np.random.default_rng(2).choice(400, B, replace=False).astype(np.int32)
+    Xd, yd, idxd = to_dev(X, y, idx)
+    loss = torch.zeros(m, dtype=torch.float32, device=DEV)
+    pk.forward_backward(Xd, idxd, yd, 5, loss)
+    lo = orc.train_step(X, idx, y, 5, update=False)
+    problems = _compare_step(pk, orc, hp, prec, loss.cpu().numpy(), lo)
+    assert not problems, problems
+    errs = emb_errs(pk, orc, range(m), flips_ok=flipped(pk, orc, hp))
+    bad = {i: e for i, e in errs.items() if e > TOL[prec]}
+    assert not bad, errs
+
+
+def sample_emb_fixed(m, d_in, d_emb, seed):
+    """Frequencies ~ N(0, 1) for given embedding sizes."""
+    rng = np.random.default_rng([seed, 11])
+    freq = np.concatenate([rng.standard_normal(d_in * (int(d) - 1)) for d in d_emb] + [np.zeros(0)])
+    return dict(d_emb=np.asarray(d_emb, dtype=np.int32), freq=freq.astype(np.float32))
+
+
+def flipped(pk, orc, hp):
+    """Members with any ReLU / dropout decision that differs between the GPU
+    and the oracle (their gradients are compared norm-wise)."""
+    out = set()
+    for i in range(len(hp["depth"])):
+        for l in range(int(hp["depth"][i])):
+            Hg = pk.debug_activations(i, l)
+            mo = (orc.preact(i, l) > 0) & (orc.keep(i, l) > 0)
+            if ((Hg > 0) != mo).any():
+                out.add(i)
+    return out
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_emb_stacked_one_step(tp, prec):
+    """A batch per member (idx [m, B]): each member's embeddings read its own
+    rows."""
+    d_in, m, B, d_out = 13, 5, 160, 4
+    hp = random_pack(m, d_in, d_out, seed=91, width=(16, 96, 16), depth=(1, 3))
+    em = sample_emb(m, d_in, seed=6)
+    pk, orc = emb_pair(tp, "multiclass", d_in, d_out, hp, em, prec, 256)
+    randomise_emb(pk, orc, em, d_in, seed=7)
+    X, y = make_data("multiclass", 400, d_in, d_out, 2)
+    rng = np.random.default_rng(3)
+    idx = np.stack([rng.choice(400, B, replace=False) for _ in range(m)]).astype(np.int32)
+    Xd, yd, idxd = to_dev(X, y, idx)
+    loss = torch.zeros(m, dtype=torch.float32, device=DEV)
+    pk.forward_backward(Xd, idxd, yd, 2, loss)
+    lo = orc.train_step(X, idx, y, 2, update=False)
+    problems = _compare_step(pk, orc, hp, prec, loss.cpu().numpy(), lo)
+    assert not problems, problems
+    errs = emb_errs(pk, orc, range(m), flips_ok=flipped(pk, orc, hp))
+    assert all(e <= TOL[prec] for e in errs.values()), errs
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_emb_eight_steps(tp, prec):
+    """AdamW on every parameter including the embeddings over eight steps
+    from the paper's zero start of b, alpha and beta (graph replay after the
+    first step; a stacked step in the middle).
+
+    bf16: Adam's first updates are about lr times the sign of the gradient,
+    so a parameter that starts at zero (b, alpha, beta) and a gradient within
+    bf16 rounding of zero move by +-lr on one side and -+lr on the other: the
+    elementwise bar does not apply to them.  As in the Muon test, an
+    exact-arithmetic oracle runs beside the bf16 one, and a tensor that
+    misses the elementwise bar must be no further from the bf16 oracle than
+    three times the distance between the bf16 and the exact oracle
+    (norm-wise)."""
+    d_in, m, B, d_out = 9, 6, 192, 3
+    hp = random_pack(m, d_in, d_out, seed=93, width=(16, 96, 16), depth=(1, 3))
+    em = sample_emb(m, d_in, seed=8, sigma=(0.1, 1.0))
+    pk, orc = emb_pair(tp, "multiclass", d_in, d_out, hp, em, prec, 256)
+    exact = None
+    if prec == "bf16":
+        exact = oracle.OraclePack(d_in, d_out, "multiclass", hp["depth"], hp["width"], hp["dropout"], hp["lr"],
+                                  hp["wd"], seed=2, bf16_storage=False, d_emb=em["d_emb"],
+                                  freq=em["freq"].astype(np.float64))
+    X, y = make_data("multiclass", 600, d_in, d_out, 3)
+    Xd, yd = to_dev(X, y)
+    rng = np.random.default_rng(5)
+    loss = torch.zeros(m, dtype=torch.float32, device=DEV)
+    margin = np.full(m, np.inf)
+    for step in range(8):
+        if step == 4:
+            idx = np.stack([rng.choice(600, B, replace=False) for _ in range(m)]).astype(np.int32)
+        else:
+            idx = rng.choice(600, B, replace=False).astype(np.int32)
+        (idxd,) = to_dev(idx)
+        pk.train_step(Xd, idxd, yd, step, loss)
+        lo = orc.train_step(X, idx, y, step)
+        if exact is not None:
+            exact.train_step(X, idx, y, step)
+        margin = np.minimum(margin, [orc.margin(i) for i in range(m)])
+        lg = loss.cpu().numpy()
+        for i in range(m):
+            assert abs(lg[i] - lo[i]) <= TOL["bf16"] * max(1.0, abs(lo[i])), (step, i, lg[i], lo[i])
+
+    def tensors(p, i):
+        out = {}
+        for l in range(int(hp["depth"][i]) + 1):
+            W, b = p.get_params(i, l)
+            out[f"W{l}"], out[f"b{l}"] = W, b
+        for name, t in zip(("w", "b", "alpha", "beta"), p.emb(i)):
+            if t.size:
+                out["emb_" + name] = t
+        return out
+
+    errs = {}
+    for i in range(m):
+        g_t, o_t = tensors(pk, i), tensors(orc, i)
+        e_t = tensors(exact, i) if exact is not None else None
+        for name in g_t:
+            e = rel_err(g_t[name], o_t[name])
+            if e > TOL[prec] and e_t is not None:
+                d_gpu = np.linalg.norm(g_t[name] - o_t[name]) / max(np.linalg.norm(o_t[name]), 1e-30)
+                d_ref = np.linalg.norm(o_t[name] - e_t[name]) / max(np.linalg.norm(e_t[name]), 1e-30)
+                e = 0.0 if d_gpu <= max(3.0 * d_ref, 1e-3) else e
+            errs[(i, name)] = e
+    bad = {k: e for k, e in errs.items() if e > TOL[prec]}
+    if prec == "fp32":
+        ties = {k for k in bad if margin[k[0]] < 1e-5}
+        assert all(errs[k] <= TOL["bf16"] for k in ties), (bad, margin)
+        bad = {k: e for k, e in bad.items() if k not in ties}
+    assert not bad, (bad, margin)
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_emb_muon_one_step(tp, prec):
+    """Muon on the first layer's [width, d_in d_emb] matrix (AdamW on the
+    embeddings): parameters after one step (fp32 against the oracle; bf16
+    within the bf16 bar)."""
+    d_in, m, B, d_out = 7, 4, 160, 3
+    hp = random_pack(m, d_in, d_out, seed=95, width=(16, 96, 16), depth=(1, 2), dropout=(0.0, 0.0))
+    em = sample_emb(m, d_in, seed=9)
+    pk, orc = emb_pair(tp, "multiclass", d_in, d_out, hp, em, prec, 256)
+    randomise_emb(pk, orc, em, d_in, seed=10)
+    lr_m = np.full(m, 0.02, dtype=np.float32)
+    pk.set_muon(lr_m)
+    orc.set_muon(lr_m.astype(np.float64))
+    X, y = make_data("multiclass", 300, d_in, d_out, 4)
+    idx = np.random.default_rng(6).choice(300, B, replace=False).astype(np.int32)
+    Xd, yd, idxd = to_dev(X, y, idx)
+    pk.train_step(Xd, idxd, yd, 0)
+    orc.train_step(X, idx, y, 0)
+    errs = {}
+    for i in range(m):
+        for l in range(int(hp["depth"][i]) + 1):
+            W, b = pk.get_params(i, l)
+            Wo, bo = orc.get_params(i, l)
+            errs[(i, l)] = max(rel_err(W, Wo), rel_err(b, bo))
+        for g, o in zip(pk.emb(i), orc.emb(i)):
+            errs[(i, "emb")] = max(errs.get((i, "emb"), 0.0), rel_err(g, o))
+    bad = {k: e for k, e in errs.items() if e > TOL[prec]}
+    assert not bad, errs
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_emb_predict(tp, prec):
+    """Predictions (fp32: chunks of max_batch rows, ragged tail; bf16: one
+    chunk) against the oracle."""
+    d_in, d_out, m = 10, 5, 5
+    hp = random_pack(m, d_in, d_out, seed=97, width=(16, 96, 16))
+    em = sample_emb(m, d_in, seed=11)
+    pk, orc = emb_pair(tp, "multiclass", d_in, d_out, hp, em, prec, 128)
+    randomise_emb(pk, orc, em, d_in, seed=12)
+    X, _ = make_data("multiclass", 333, d_in, d_out, 5)
+    (Xd,) = to_dev(X)
+    out = pk.predict(Xd).cpu().numpy()
+    ref = orc.predict(X)
+    for i in range(m):
+        assert rel_err(out[i], ref[i]) <= TOL[prec], i
+
+
+def test_emb_predict_chunk_cap(tp):
+    """Wide embeddings (4 members x 1024 features x d_emb 16): the chunk's
+    embedding matrices would pass 1 GiB at 8192 rows, so bf16 prediction
+    runs in smaller chunks (8064 rows).  Rows of the second chunk predict
+    the same alone (bit-exact), and sampled rows of both chunks match the
+    oracle."""
+    d_in, d_out, m, N = 1024, 2, 4, 8200
+    hp = random_pack(m, d_in, d_out, seed=99, width=(16, 48, 16), depth=(1, 2))
+    em = sample_emb_fixed(m, d_in, [16] * m, seed=13)
+    pk, orc = emb_pair(tp, "multiclass", d_in, d_out, hp, em, "bf16", 64)
+    randomise_emb(pk, orc, em, d_in, seed=14)
+    X, _ = make_data("multiclass", N, d_in, d_out, 6)
+    (Xd,) = to_dev(X)
+    full = pk.predict(Xd).cpu().numpy()
+    np.testing.assert_array_equal(pk.predict(Xd[8064:].contiguous()).cpu().numpy(), full[:, 8064:])
+    rows = np.r_[0:40, 8040:8100, 8160:8200]
+    ref = orc.predict(X[rows])
+    for i in range(m):
+        assert rel_err(full[i][rows], ref[i]) <= TOL["bf16"], i
+
+
+def test_emb_online_ensemble(tp):
+    """The online ensemble of a pack with embeddings: its prediction is the
+    fp64 mean of the pack's predictions of the selected members at the
+    epoch they were recorded (the ensemble pack is rebuilt with the same
+    embedding sizes from the snapshots)."""
+    d_in, d_out, m, n_val = 8, 3, 6, 300
+    hp = random_pack(m, d_in, d_out, seed=101, width=(16, 64, 16))
+    em = sample_emb(m, d_in, seed=15)
+    pk, _ = emb_pair(tp, "multiclass", d_in, d_out, hp, em, "bf16", 128)
+    X, y = make_data("multiclass", 800, d_in, d_out, 7)
+    Xd, yd = to_dev(X, y)
+    Xv, yv = Xd[:n_val].contiguous(), yd[:n_val].contiguous()
+    Xt = Xd[n_val:].contiguous()
+    on = tp.OnlineEnsemble(pk, n_val, score="loss", m_ens=4, p_base=4, p_ens=4)
+    rec = {}
+    rng = np.random.default_rng(8)
+    for ep in range(1, 4):   # the online ensemble numbers epochs from 1
+        for s in range(4):
+            idx = (n_val + rng.choice(500, 128, replace=False)).astype(np.int32)
+            (idxd,) = to_dev(idx)
+            pk.train_step(Xd, idxd, yd, ep * 4 + s)
+        pt = pk.predict(Xt).cpu().numpy()
+        for i in range(m):
+            rec[(i, ep)] = pt[i]
+        on.epoch(Xv, yv)
+    mem, eps, _ = on.ensemble("best")
+    got = on.predict(Xt).cpu().numpy()
+    assert np.array_equal(got, ens_mean([rec[(int(a), int(b))] for a, b in zip(mem, eps)]))

@@ -145,3 +145,17 @@ def random_pack(m, d_in, d_out, seed, depth=(1, 3), width=(16, 96, 16), dropout=
     """Small random pack shapes for tests."""
     wl = Workload("test", "binary", 0, 0, d_in, d_out, m, depth, width, dropout, lr, wd)
     return sample_hparams(wl, seed=seed, m=m)
+
+
+def sample_emb(m, d_in, seed, d_emb=(8, 32, 4), sigma=(1e-2, 10.0)) -> dict:
+    """Periodic-embedding hyperparameters of m members (App. "Feature
+    Embeddings", TabPack-with-embeddings sampling space: d_emb UniformInt
+    [8, 32] step 4, sigma LogUniform[1e-2, 10]) and the initial frequencies
+    w ~ N(0, sigma) of each member, [d_in, d_emb - 1] row-major, member after
+    member (float32 values, as the library takes them)."""
+    rng = np.random.default_rng([seed, 7])
+    lo, hi, step = d_emb
+    d = rng.integers(0, (hi - lo) // step + 1, m) * step + lo
+    s = np.exp(rng.uniform(np.log(sigma[0]), np.log(sigma[1]), m))
+    freq = np.concatenate([rng.normal(0.0, s[i], d_in * (int(d[i]) - 1)) for i in range(m)] + [np.zeros(0)])
+    return dict(d_emb=d.astype(np.int32), sigma=s, freq=freq.astype(np.float32))
