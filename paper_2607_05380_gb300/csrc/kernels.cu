@@ -875,7 +875,7 @@ void launch_init(cudaStream_t st, const InitArgs& g, int n_chunks) {
 // in groups of 32 (lane = column: each thread keeps its column's feature,
 // component and parameters in registers) and spread the rows over the
 // block's 8 warps.
-constexpr int kEmbRows = 64;   // rows per forward block
+constexpr int kEmbRows = 128;  // rows per forward block
 
 struct EmbCol {
   int j, k;
@@ -898,7 +898,7 @@ __device__ __forceinline__ EmbCol emb_col(const EmbMember& em, const float* para
   return c;
 }
 
-// Forward: block (32-column group, 64-row group, active member); rows >= B
+// Forward: block (32-column group, 128-row group, active member); rows >= B
 // and the pad columns up to in0_pad are written as zero.
 template <typename T>
 __global__ void __launch_bounds__(256) k_emb_fwd(EmbArgs<T> a) {
@@ -936,7 +936,7 @@ __global__ void __launch_bounds__(256) k_emb_fwd(EmbArgs<T> a) {
 // in fp32 and adds that partial to fp64 sums; the 8 warps' fp64 sums are
 // added in warp order.
 template <typename T>
-__global__ void __launch_bounds__(256) k_emb_bwd(EmbArgs<T> a) {
+__global__ void __launch_bounds__(256, 6) k_emb_bwd(EmbArgs<T> a) {
   pdl_trigger();
   pdl_wait();
   const int member = a.active_ids[blockIdx.y];
@@ -955,6 +955,7 @@ __global__ void __launch_bounds__(256) k_emb_bwd(EmbArgs<T> a) {
   for (int b0 = wp; b0 < a.B; b0 += 8 * 32) {
     float p_a = 0.f, p_be = 0.f, p_w = 0.f, p_b = 0.f;
     const int b1 = min(a.B, b0 + 8 * 32);
+#pragma unroll 4
     for (int b = b0; b < b1; b += 8) {
       const float g = Elem<T>::to_f(dE[(int64_t)b * em.in0_pad]);
       const int64_t row = idx ? (int64_t)idx[b] : (int64_t)b;

@@ -331,3 +331,54 @@ def test_emb_online_ensemble(tp):
     mem, eps, _ = on.ensemble("best")
     got = on.predict(Xt).cpu().numpy()
     assert np.array_equal(got, ens_mean([rec[(int(a), int(b))] for a, b in zip(mem, eps)]))
+
+
+def test_emb_full_size_sampled_members(tp):
+    """The medium workload with embeddings as `bench.py --emb` runs it (the
+    whole pack of 32 members, batch 512, bf16, the embedding sizes and
+    frequencies the bench samples): for the cheapest member of each depth
+    (embedding parameters set to random values on both sides: from the
+    paper's zero start E is zero), losses, logits, every gradient and the
+    embedding gradients against the oracle run on those members alone
+    (members are independent, Sec. 3.6)."""
+    from workloads import SEED_HP, SEED_INIT, WORKLOADS, make_data as wl_data, sample_hparams
+    from test_gpu_parity import _sample_members
+    wl = WORKLOADS["medium"]
+    hp = sample_hparams(wl, seed=SEED_HP)
+    em = sample_emb(wl.m, wl.d_in, seed=SEED_HP + 200)
+    B = wl.batch
+    d = wl_data(wl, device="cpu", n_train=3 * B, n_val=0)
+    X, y = d["X_train"].numpy(), d["y_train"].numpy()
+    Xd, yd = to_dev(X, y)
+    idx = np.random.default_rng(3).permutation(3 * B)[:B].astype(np.int32)
+    (idxd,) = to_dev(idx)
+    sample = _sample_members(wl, hp)
+    sub = {k: v[sample] for k, v in hp.items()}
+    starts = np.concatenate([[0], np.cumsum(wl.d_in * (em["d_emb"] - 1))])
+    freq_sub = np.concatenate([em["freq"][starts[i]:starts[i + 1]] for i in sample])
+    pk = tp.Pack(wl.d_in, wl.d_out, wl.task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
+                 max_batch=B, seed=SEED_INIT, precision="bf16", d_emb=em["d_emb"], freq=em["freq"])
+    orc = oracle.OraclePack(wl.d_in, wl.d_out, wl.task, sub["depth"], sub["width"], sub["dropout"], sub["lr"],
+                            sub["wd"], seed=SEED_INIT, bf16_storage=True, member_id=sample,
+                            d_emb=em["d_emb"][sample], freq=freq_sub.astype(np.float64))
+    rng = np.random.default_rng(21)
+    for oi, i in enumerate(sample):
+        dm = int(em["d_emb"][i])
+        parts = [np.asarray(p, dtype=np.float32) for p in (
+            pk.emb(i)[0], rng.uniform(-np.pi, np.pi, (wl.d_in, dm - 1)), rng.standard_normal((wl.d_in, dm)) * 0.7,
+            rng.standard_normal((wl.d_in, dm)) * 0.2)]
+        pk.set_emb(i, *parts)
+        orc.set_emb(oi, *[p.astype(np.float64) for p in parts])
+    loss = torch.zeros(wl.m, dtype=torch.float32, device=DEV)
+    pk.forward_backward(Xd, idxd, yd, 0, loss)
+    lo = orc.train_step(X, idx, y, 0, update=False)
+    problems = _compare_step(pk, orc, hp, "bf16", loss.cpu().numpy(), lo, members=sample,
+                             max_flip_members=len(sample))
+    assert not problems, problems
+    errs = {}
+    for oi, i in enumerate(sample):
+        for g, o in zip(pk.emb(i, grads=True), orc.emb(oi, grads=True)):
+            if g.size:   # norm-wise: a full-size member may carry flipped ReLU decisions at near-ties
+                e = float(np.linalg.norm(g - o) / max(np.linalg.norm(o), 1e-30))
+                errs[i] = max(errs.get(i, 0.0), e)
+    assert all(e <= TOL["bf16"] for e in errs.values()), errs

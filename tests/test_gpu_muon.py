@@ -161,3 +161,58 @@ def test_muon_argument_checks(tp):
         pk.set_muon(np.array([0.01, 0.01], dtype=np.float32), momentum=1.0)
     with pytest.raises(tp.TabpackError):
         pk.muon_dir(0, 0)   # Muon not on yet
+
+
+def test_muon_full_size_sampled_members(tp):
+    """The medium workload with Muon as `bench.py --muon` runs it (the whole
+    pack, batch 512, bf16, the bench's per-member Muon learning rates): one
+    step; for the cheapest member of each depth, the Newton-Schulz direction
+    of every hidden layer from the GPU's own gradient within twice the error
+    of the oracle's bf16 model of the iteration (norm-wise, against the exact
+    iteration), and the parameters after the step within 2e-2 elementwise of
+    the bf16 oracle run on those members alone, or no further from it than
+    three times the distance between the bf16 and the exact oracle."""
+    import math
+    from workloads import SEED_HP, SEED_INIT, WORKLOADS, make_data as wl_data, sample_hparams
+    from test_gpu_parity import _sample_members
+    wl = WORKLOADS["medium"]
+    hp = sample_hparams(wl, seed=SEED_HP)
+    rng_m = np.random.default_rng(SEED_HP + 100)
+    lr_m = np.exp(rng_m.uniform(math.log(1e-3), math.log(1e-1), wl.m)).astype(np.float32)
+    B = wl.batch
+    d = wl_data(wl, device="cpu", n_train=3 * B, n_val=0)
+    X, y = d["X_train"].numpy(), d["y_train"].numpy()
+    Xd, yd = (torch.from_numpy(a).to(DEV) for a in (X, y))
+    idx = np.random.default_rng(3).permutation(3 * B)[:B].astype(np.int32)
+    sample = _sample_members(wl, hp)
+    sub = {k: v[sample] for k, v in hp.items()}
+    pk = tp.Pack(wl.d_in, wl.d_out, wl.task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
+                 max_batch=B, seed=SEED_INIT, precision="bf16")
+    pk.set_muon(lr_m)
+    orcs = []
+    for bf in (True, False):
+        o = oracle.OraclePack(wl.d_in, wl.d_out, wl.task, sub["depth"], sub["width"], sub["dropout"], sub["lr"],
+                              sub["wd"], seed=SEED_INIT, bf16_storage=bf, member_id=sample)
+        o.set_muon(lr_m[sample].astype(np.float64))
+        o.train_step(X, idx, y, 0)
+        orcs.append(o)
+    orc, exact = orcs
+    pk.train_step(Xd, torch.from_numpy(idx).to(DEV), yd, 0)
+    errs = {}
+    for oi, i in enumerate(sample):
+        for l in range(int(hp["depth"][i])):
+            G = pk.get_grads(i, l)[0].astype(np.float64)
+            O_ref = oracle.newton_schulz(G)
+            e_orc = np.linalg.norm(oracle.newton_schulz(G, bf16=True) - O_ref) / np.linalg.norm(O_ref)
+            e_gpu = np.linalg.norm(pk.muon_dir(i, l) - O_ref) / np.linalg.norm(O_ref)
+            errs[(i, l, "dir")] = 0.0 if e_gpu <= max(2.0 * e_orc, 5e-3) else e_gpu
+        for l in range(int(hp["depth"][i]) + 1):
+            for g_, o_, e_ in zip(pk.get_params(i, l), orc.get_params(oi, l), exact.get_params(oi, l)):
+                e = rel_err(g_, o_)
+                if e > TOL["bf16"]:
+                    d_gpu = np.linalg.norm(g_ - o_) / max(np.linalg.norm(o_), 1e-30)
+                    d_ref = np.linalg.norm(o_ - e_) / max(np.linalg.norm(e_), 1e-30)
+                    e = 0.0 if d_gpu <= max(3.0 * d_ref, 1e-3) else e
+                errs[(i, l, len(g_.shape))] = max(errs.get((i, l, len(g_.shape)), 0.0), e)
+    bad = {k: e for k, e in errs.items() if e > TOL["bf16"]}
+    assert not bad, bad
