@@ -89,3 +89,34 @@ def test_invalid_configs_rejected_before_any_gpu_call(lib_path):
                            tp._hptr(arr([0.0], np.float32)), None, ctypes.byref(h))
         assert st == tp.TP_EINVAL, (cfg.m, d, w, p)
         assert not h.value
+
+
+def test_embedding_entry_points_reject_bad_arguments_without_a_gpu(lib_path):
+    """pack_create_emb checks the embedding sizes and pointers before any GPU
+    call; the embedding accessors reject a NULL pack."""
+    import numpy as np
+    import paper_2607_05380_gb300 as tp
+    L = tp.load_library()
+    arr = lambda v, dt: np.array(v, dtype=dt)
+    cfg = tp.Config(2, 4, 1, 16, 0, 0, 1, 0.9, 0.999, 1e-8, 1)
+    d, w, p = arr([1, 2], np.int32), arr([16, 32], np.int32), arr([0.1, 0.0], np.float32)
+    lr, wd = arr([1e-3, 1e-3], np.float32), arr([0.0, 0.0], np.float32)
+    freq = arr(np.zeros(4 * 70), np.float32)
+    for d_emb, fr in (([0, 4], freq), ([4, 65], freq), ([4, 4], None), (None, freq)):
+        h = ctypes.c_void_p()
+        de = None if d_emb is None else tp._hptr(arr(d_emb, np.int32))
+        st = L.pack_create_emb(ctypes.byref(cfg), tp._hptr(d), tp._hptr(w), tp._hptr(p), tp._hptr(lr), tp._hptr(wd),
+                               de, None if fr is None else tp._hptr(fr), None, ctypes.byref(h))
+        assert st == tp.TP_EINVAL, d_emb
+        assert not h.value
+    # a bad width is still caught with valid embedding sizes
+    h = ctypes.c_void_p()
+    st = L.pack_create_emb(ctypes.byref(cfg), tp._hptr(d), tp._hptr(arr([16, 24], np.int32)), tp._hptr(p),
+                           tp._hptr(lr), tp._hptr(wd), tp._hptr(arr([4, 4], np.int32)), tp._hptr(freq), None,
+                           ctypes.byref(h))
+    assert st == tp.TP_EINVAL and not h.value
+    out = arr(np.zeros(64), np.float32)
+    n = ctypes.c_int32()
+    assert L.pack_get_emb(None, 0, 0, tp._hptr(out)) == tp.TP_EINVAL
+    assert L.pack_set_emb(None, 0, tp._hptr(out)) == tp.TP_EINVAL
+    assert L.pack_member_emb(None, 0, ctypes.byref(n)) == tp.TP_EINVAL
