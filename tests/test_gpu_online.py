@@ -150,7 +150,7 @@ def check_best(on, orc, data, X_test, rec_val, rec_test, rec_snap):
     assert np.array_equal(pt, ens_mean([rec_test[i] for i in best]))
 
 
-@pytest.mark.parametrize("prec,score", [("bf16", "loss"), ("fp32", "accuracy"), ("bf16", "accuracy")])
+@pytest.mark.parametrize("prec,score", [("bf16", "loss"), ("fp32", "accuracy"), ("bf16", "accuracy"), ("bf16", "auc")])
 def test_online_tiny_matches_oracle(tp, prec, score):
     """Tiny binary workload, 10 epochs; members 1 and 5 have lr = 0, so their
     predictions never change and p_base = 1 removes them after epoch 3."""

@@ -114,3 +114,26 @@ def test_accuracy_score_multiclass_pool():
     assert r2["selected"] == [(0, 2)] and not r2["improved"] and o.best == [(0, 1)]
     # model 0 did not improve (equal), model 1 did
     assert o.member_bad.tolist() == [1, 0]
+
+
+def test_auc_score_binary_pool():
+    """ROC-AUC (score = -AUC): two models that each rank 3 of the 4
+    positive-negative pairs right (AUC 3/4) but whose mean ranks all four
+    right (AUC 1).  The first pick is the lower index among the tied
+    singletons, the second model's addition strictly improves, and the base
+    models' own scores are their single-model AUCs."""
+    y = np.array([0, 0, 1, 1], dtype=np.int32)
+    a = np.array([0.1, 0.5, 0.4, 0.9], dtype=np.float32)[:, None]   # 0.4 < 0.5: one pair wrong
+    b = np.array([0.5, 0.1, 0.9, 0.4], dtype=np.float32)[:, None]   # 0.4 < 0.5: one pair wrong
+    o = OnlineEnsemble(2, "binary", "auc", m_ens=4, p_base=3, p_ens=3)
+    r = o.epoch_end(np.stack([a, b]), y)
+    assert r["selected"] == [(0, 1), (1, 1)]
+    assert r["score"] == -1.0 and r["improved"]
+    assert o.member_best.tolist() == [-0.75, -0.75]
+    # a model that ranks every pair right scores -1 alone and is picked first
+    # (lowest pool index); nothing improves on -1, and a tie with the previous
+    # ensemble's score is no improvement, so the best ensemble stays the first
+    c = np.array([0.2, 0.3, 0.6, 0.7], dtype=np.float32)[:, None]
+    r2 = o.epoch_end(np.stack([c, b]), y)
+    assert r2["selected"][0] == (0, 2) and r2["score"] == -1.0 and not r2["improved"]
+    assert o.best == [(0, 1), (1, 1)]
