@@ -52,6 +52,12 @@ def peaks():
     return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
 
 
+def muon_lrs(m):
+    """Per-member Muon learning rates, LogUniform[1e-3, 1e-1] (seed 101)."""
+    rng_m = np.random.default_rng(SEED_HP + 100)
+    return np.exp(rng_m.uniform(math.log(1e-3), math.log(1e-1), m)).astype(np.float32)
+
+
 def in0_of(wl, emb, i):
     """Member i's first-layer input width (d_in d_emb with embeddings)."""
     return wl.d_in * (int(emb["d_emb"][i]) if emb is not None else 1)
@@ -202,11 +208,12 @@ def time_online_epoch(tp, torch, pack, wl, hp, d, X, y, idx_all, stream, loss, n
                     % -(-wl.n_train // B)}
 
 
-def cpu_baseline(wl, hp, data_np, B, budget_s=20.0, stacked=False, emb=None):
+def cpu_baseline(wl, hp, data_np, B, budget_s=20.0, stacked=False, emb=None, lr_muon=None):
     """The oracle as it stands, on the host cores, on a bounded sample of the
     same workload: the first k members (independent of the others), timed
     over whole steps until about budget_s seconds of CPU work (stacked: a
-    batch per member; emb: the members' periodic embeddings)."""
+    batch per member; emb: the members' periodic embeddings; lr_muon: Muon
+    for the hidden weights with these per-member learning rates)."""
     import oracle
     oracle.build()
     X, y = data_np
@@ -221,6 +228,8 @@ def cpu_baseline(wl, hp, data_np, B, budget_s=20.0, stacked=False, emb=None):
     pk = oracle.OraclePack(wl.d_in, wl.d_out, wl.task, hp["depth"][members], hp["width"][members],
                            hp["dropout"][members], hp["lr"][members], hp["wd"][members], seed=SEED_INIT,
                            member_id=members, **kw)
+    if lr_muon is not None:
+        pk.set_muon(np.asarray(lr_muon[:k], dtype=np.float64))
     steps = 0
     t0 = time.perf_counter()
     while True:
@@ -261,14 +270,16 @@ def run_reference(args, wl, rank):
     base = None
     emb = sample_emb(wl.m, wl.d_in, seed=SEED_HP + 200) if args.emb else None
     for s in range(max(1, args.steps)):
-        base = cpu_baseline(wl, hp, data, B, budget_s=per, stacked=args.stacked, emb=emb)
+        base = cpu_baseline(wl, hp, data, B, budget_s=per, stacked=args.stacked, emb=emb,
+                            lr_muon=muon_lrs(wl.m) if args.muon else None)
         vals.append(base["value"])
     value = float(np.mean(vals))
     ms = float(1000.0 * wl.m * B / value)
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": workload_desc(wl, B), "embeddings": emb_desc(emb)},
+            "config": {"workload": workload_desc(wl, B), "embeddings": emb_desc(emb),
+                       "optimizer": "Muon (hidden weights) + AdamW" if args.muon else "AdamW"},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": base["cores"], "kind": "oracle",
                              "sample": base["sample"]},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -346,9 +357,8 @@ def main():
                    freq=None if emb is None else emb["freq"])
     loss = torch.zeros(wl.m, dtype=torch.float32, device=dev)
     lr_muon = None
-    if args.muon:   # Muon lr LogUniform[1e-3, 1e-1] per member
-        rng_m = np.random.default_rng(SEED_HP + 100)
-        lr_muon = np.exp(rng_m.uniform(math.log(1e-3), math.log(1e-1), wl.m)).astype(np.float32)
+    if args.muon:
+        lr_muon = muon_lrs(wl.m)
         pack.set_muon(lr_muon)
 
     for s in range(args.warmup):
@@ -473,7 +483,7 @@ def main():
     if rank == 0 and not args.no_cpu_baseline:
         n = min(n_train, 20000)
         data_np = (X[:n].cpu().numpy(), y[:n].cpu().numpy())
-        cpu = cpu_baseline(wl, hp, data_np, B, budget_s=20.0, stacked=args.stacked, emb=emb)
+        cpu = cpu_baseline(wl, hp, data_np, B, budget_s=20.0, stacked=args.stacked, emb=emb, lr_muon=lr_muon)
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
