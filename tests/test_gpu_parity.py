@@ -414,6 +414,38 @@ def test_full_size_sampled_members(tp, name):
         pk_s.close()
 
 
+def test_full_size_stacked_sampled_members(tp):
+    """The medium workload with a batch per member, as `bench.py --stacked`
+    runs it (idx [32, 512] drawn with replacement, bf16, the second tile plan
+    whose layer-1 tiles read each member's own batch matrix): for the
+    cheapest member of each depth, dropout masks bit-exact and losses,
+    logits and every gradient against the oracle's stacked step on those
+    members' rows alone."""
+    from workloads import SEED_HP, SEED_INIT, WORKLOADS, make_data as wl_data, sample_hparams
+    wl = WORKLOADS["medium"]
+    hp = sample_hparams(wl, seed=SEED_HP)
+    B = wl.batch
+    d = wl_data(wl, device="cpu", n_train=3 * B, n_val=0)
+    X, y = d["X_train"].numpy(), d["y_train"].numpy()
+    idx = np.random.default_rng(4).integers(0, 3 * B, (wl.m, B)).astype(np.int32)
+    Xd, yd, idxd = to_dev(X, y, idx)
+    sample = _sample_members(wl, hp)
+    sub = {k: v[sample] for k, v in hp.items()}
+    pk = tp.Pack(wl.d_in, wl.d_out, wl.task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
+                 max_batch=B, seed=SEED_INIT, precision="bf16")
+    loss = torch.zeros(wl.m, dtype=torch.float32, device=DEV)
+    pk.forward_backward(Xd, idxd, yd, 0, loss)
+    orc = oracle.OraclePack(wl.d_in, wl.d_out, wl.task, sub["depth"], sub["width"], sub["dropout"], sub["lr"],
+                            sub["wd"], seed=SEED_INIT, bf16_storage=True, member_id=sample)
+    lo = orc.train_step(X, idx[sample], y, 0, update=False)
+    for oi, i in enumerate(sample):
+        for l in range(int(hp["depth"][i])):
+            np.testing.assert_array_equal(pk.debug_masks(i, l, 0, B), orc.keep(oi, l))
+    problems = _compare_step(pk, orc, hp, "bf16", loss.cpu().numpy(), lo, members=sample,
+                             max_flip_members=len(sample))
+    assert not problems, problems
+
+
 @pytest.mark.parametrize("prec", ["fp32", "bf16"])
 @pytest.mark.parametrize("task,d_out", [("binary", 1), ("multiclass", 6), ("regression", 1)])
 def test_predict(tp, prec, task, d_out):
