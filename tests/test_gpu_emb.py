@@ -382,3 +382,30 @@ def test_emb_full_size_sampled_members(tp):
                 e = float(np.linalg.norm(g - o) / max(np.linalg.norm(o), 1e-30))
                 errs[i] = max(errs.get(i, 0.0), e)
     assert all(e <= TOL["bf16"] for e in errs.values()), errs
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+@pytest.mark.parametrize("wd_on_bias", [False, True])
+def test_emb_weight_decay_follows_the_bias_flag(tp, prec, wd_on_bias):
+    """From the paper's zero start (alpha = 0) w and b get a zero gradient:
+    with wd_on_bias off one AdamW step leaves w bit-identical, with it on w
+    shrinks by lr wd w (fp32 arithmetic); b stays zero; alpha moves."""
+    d_in, d_out, m = 6, 3, 3
+    hp = random_pack(m, d_in, d_out, seed=103, width=(16, 64, 16))
+    em = sample_emb(m, d_in, seed=16)
+    pk = tp.Pack(d_in, d_out, "multiclass", hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
+                 max_batch=128, seed=2, precision=prec, wd_on_bias=wd_on_bias, d_emb=em["d_emb"], freq=em["freq"])
+    X, y = make_data("multiclass", 200, d_in, d_out, 9)
+    Xd, yd = to_dev(X, y)
+    before = [pk.emb(i) for i in range(m)]
+    (idxd,) = to_dev(np.arange(128, dtype=np.int32))
+    pk.train_step(Xd, idxd, yd, 0)
+    for i in range(m):
+        w0 = before[i][0]
+        w1, b1, a1, _ = pk.emb(i)
+        if wd_on_bias:
+            expect = w0.astype(np.float64) * (1.0 - float(np.float32(hp["lr"][i])) * float(np.float32(hp["wd"][i])))
+            np.testing.assert_allclose(w1, expect, rtol=1e-6, atol=0)
+        else:
+            np.testing.assert_array_equal(w1, w0)
+        assert not b1.any() and np.abs(a1).max() > 0

@@ -127,3 +127,21 @@ def test_embeddings_train_with_adamw():
     # zero gradient while alpha is zero: only the decoupled weight decay acts on w
     np.testing.assert_allclose(w1, w0 - float(hp["lr"][1]) * float(hp["wd"][1]) * w0, rtol=1e-15, atol=0)
     assert not b1.any()
+
+
+def test_embedding_weight_decay_follows_the_bias_flag():
+    """The embedding parameters take weight decay as the biases do: with
+    wd_on_bias off, a step from alpha = 0 (zero gradient for w and b) leaves
+    w exactly in place; with it on, w shrinks by lr wd w."""
+    d_in, d_out, d = 3, 2, 4
+    hp = random_pack(1, d_in, d_out, seed=13, dropout=(0.0, 0.0))
+    freq = np.random.default_rng(4).standard_normal(d_in * (d - 1))
+    X, y = data(30, d_in, d_out, 10)
+    for on in (False, True):
+        e = oracle.OraclePack(d_in, d_out, "multiclass", hp["depth"], hp["width"], hp["dropout"], hp["lr"],
+                              hp["wd"], seed=2, wd_on_bias=on, d_emb=[d], freq=freq)
+        w0 = e.emb(0)[0].copy()
+        e.train_step(X, np.arange(30, dtype=np.int32), y, 0)
+        w1 = e.emb(0)[0]
+        expect = w0 - float(hp["lr"][0]) * float(hp["wd"][0]) * w0 if on else w0
+        np.testing.assert_allclose(w1, expect, rtol=1e-15, atol=0)
