@@ -145,3 +145,38 @@ def test_embedding_weight_decay_follows_the_bias_flag():
         w1 = e.emb(0)[0]
         expect = w0 - float(hp["lr"][0]) * float(hp["wd"][0]) * w0 if on else w0
         np.testing.assert_allclose(w1, expect, rtol=1e-15, atol=0)
+
+
+@pytest.mark.parametrize("bf16", [False, True])
+def test_packed_embedding_members_equal_solo_members(bf16):
+    """Members with periodic embeddings of different sizes are independent
+    (Sec. 3.6): three AdamW steps of the pack give each member exactly what
+    training it alone gives (losses, every parameter, embeddings included,
+    and predictions), with the frequencies split member by member."""
+    m, d_in, d_out = 4, 5, 3
+    hp = random_pack(m, d_in, d_out, seed=19)
+    d_emb = np.array([1, 3, 8, 5], dtype=np.int32)
+    freq = np.random.default_rng(7).standard_normal(d_in * int(np.sum(d_emb - 1)))
+    starts = np.concatenate([[0], np.cumsum(d_in * (d_emb - 1))])
+    X, y = data(64, d_in, d_out, 3)
+    kw = dict(seed=8, bf16_storage=bf16)
+    packed = oracle.OraclePack(d_in, d_out, "multiclass", hp["depth"], hp["width"], hp["dropout"], hp["lr"],
+                               hp["wd"], d_emb=d_emb, freq=freq, **kw)
+    solos = [oracle.OraclePack(d_in, d_out, "multiclass", hp["depth"][i:i + 1], hp["width"][i:i + 1],
+                               hp["dropout"][i:i + 1], hp["lr"][i:i + 1], hp["wd"][i:i + 1], member_id=[i],
+                               d_emb=d_emb[i:i + 1], freq=freq[starts[i]:starts[i + 1]], **kw) for i in range(m)]
+    rng = np.random.default_rng(1)
+    for step in range(3):
+        idx = rng.choice(64, 24, replace=False).astype(np.int32)
+        lp = packed.train_step(X, idx, y, step)
+        for i in range(m):
+            assert lp[i] == solos[i].train_step(X, idx, y, step)[0]
+    for i in range(m):
+        for l in range(int(hp["depth"][i]) + 1):
+            for a, b in zip(packed.get_params(i, l), solos[i].get_params(0, l)):
+                np.testing.assert_array_equal(a, b)
+        for a, b in zip(packed.emb(i), solos[i].emb(0)):
+            np.testing.assert_array_equal(a, b)
+    Pp = packed.predict(X[:10])
+    for i in range(m):
+        np.testing.assert_array_equal(Pp[i], solos[i].predict(X[:10])[0])
