@@ -409,3 +409,25 @@ def test_emb_weight_decay_follows_the_bias_flag(tp, prec, wd_on_bias):
         else:
             np.testing.assert_array_equal(w1, w0)
         assert not b1.any() and np.abs(a1).max() > 0
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_emb_maximum_size(tp, prec):
+    """The largest embedding the library takes (d_emb = 64) on 40 features:
+    a first layer of 2560 inputs (40 K blocks), next to a d_emb = 2 member;
+    one step's logits, losses and every gradient against the oracle."""
+    d_in, d_out, m = 40, 4, 2
+    hp = random_pack(m, d_in, d_out, seed=107, width=(32, 96, 16), depth=(1, 2))
+    em = sample_emb_fixed(m, d_in, [64, 2], seed=17)
+    pk, orc = emb_pair(tp, "multiclass", d_in, d_out, hp, em, prec, 128)
+    randomise_emb(pk, orc, em, d_in, seed=18)
+    X, y = make_data("multiclass", 300, d_in, d_out, 11)
+    idx = np.random.default_rng(12).choice(300, 130, replace=False).astype(np.int32)
+    Xd, yd, idxd = to_dev(X, y, idx)
+    loss = torch.zeros(m, dtype=torch.float32, device=DEV)
+    pk.forward_backward(Xd, idxd, yd, 3, loss)
+    lo = orc.train_step(X, idx, y, 3, update=False)
+    problems = _compare_step(pk, orc, hp, prec, loss.cpu().numpy(), lo, max_flip_members=m)
+    assert not problems, problems
+    errs = emb_errs(pk, orc, range(m), flips_ok=flipped(pk, orc, hp))
+    assert all(e <= TOL[prec] for e in errs.values()), errs
