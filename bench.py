@@ -255,33 +255,72 @@ def emb_desc(emb):
 
 
 def run_reference(args, wl, rank):
-    """Reference arm: the CPU fp64 oracle timed on the host cores (rank 0)."""
+    """Reference arm: the CPU fp64 oracle, as it stands, timed on the host
+    cores (rank 0 only) over exactly W untimed and K timed steps.  Each step
+    is a bounded sample of the workload: the first min(m, cores) members
+    (independent of the others, one OpenMP thread each) on a batch whose rows
+    are cut, when needed, so that the W + K steps fit in about
+    --reference-seconds: a full-batch step and a one-row step calibrate the
+    step time as a fixed cost (the optimizer pass over every parameter,
+    operand copies) plus a cost per row."""
     if rank != 0:
         return
+    import oracle
+    oracle.build()
     hp = sample_hparams(wl, seed=SEED_HP)
     B = wl.batch
     n = min(wl.n_train, 20000)
     d = make_data(wl, device="cpu", n_train=n, n_val=0)
-    data = (d["X_train"].numpy(), d["y_train"].numpy())
-    per = max(3.0, min(30.0, 120.0 / max(1, args.steps)))
-    vals = []
-    for _ in range(args.warmup if args.warmup < 1 else 1):
-        pass
-    base = None
+    X, y = d["X_train"].numpy(), d["y_train"].numpy()
     emb = sample_emb(wl.m, wl.d_in, seed=SEED_HP + 200) if args.emb else None
-    for s in range(max(1, args.steps)):
-        base = cpu_baseline(wl, hp, data, B, budget_s=per, stacked=args.stacked, emb=emb,
-                            lr_muon=muon_lrs(wl.m) if args.muon else None)
-        vals.append(base["value"])
-    value = float(np.mean(vals))
-    ms = float(1000.0 * wl.m * B / value)
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    k = min(wl.m, max(1, cores))
+    members = list(range(k))
+    kw = {}
+    if emb is not None:
+        n_f = wl.d_in * int(np.sum(emb["d_emb"][:k] - 1))
+        kw = dict(d_emb=emb["d_emb"][:k], freq=emb["freq"][:n_f].astype(np.float64))
+    pk = oracle.OraclePack(wl.d_in, wl.d_out, wl.task, hp["depth"][members], hp["width"][members],
+                           hp["dropout"][members], hp["lr"][members], hp["wd"][members], seed=SEED_INIT,
+                           member_id=members, **kw)
+    if args.muon:
+        pk.set_muon(muon_lrs(wl.m)[:k].astype(np.float64))
+    rng = np.random.default_rng(3)
+
+    def step(rows, s):
+        if args.stacked:
+            idx = np.stack([rng.choice(n, rows, replace=False) for _ in range(k)]).astype(np.int32)
+        else:
+            idx = rng.choice(n, rows, replace=False).astype(np.int32)
+        pk.train_step(X, idx, y, s)
+
+    t0 = time.perf_counter()
+    step(B, 0)                                   # calibration steps (they count as warm-up)
+    t_full = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    step(1, 1)
+    t_one = time.perf_counter() - t0
+    per_row = max(t_full - t_one, 1e-9) / max(B - 1, 1)
+    budget = float(args.reference_seconds) / max(1, args.steps + args.warmup)
+    rows = B if t_full <= budget else max(1, min(B, int((budget - t_one) / per_row)))
+    for s in range(2, args.warmup):
+        step(rows, s)
+    t0 = time.perf_counter()
+    for s in range(args.steps):
+        step(rows, args.warmup + s)
+    el = time.perf_counter() - t0
+    value = k * rows * args.steps / el
+    sample = (f"members 0..{k - 1} of {wl.m} (independent, one thread each), {args.steps} timed steps of "
+              f"{rows} row{'s' if rows != 1 else ''} each" + (f" (batch {B} cut to fit {args.reference_seconds:.0f} s; a full-batch step "
+                                     f"took {t_full:.2f} s, a one-row step {t_one:.3f} s)" if rows < B
+                                     else " (the full batch)") + f", {el:.1f} s")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * el / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": workload_desc(wl, B), "embeddings": emb_desc(emb),
-                       "optimizer": "Muon (hidden weights) + AdamW" if args.muon else "AdamW"},
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": base["cores"], "kind": "oracle",
-                             "sample": base["sample"]},
+                       "optimizer": "Muon (hidden weights) + AdamW" if args.muon else "AdamW",
+                       "batches": "one per member (stacked)" if args.stacked else "one shared by all members"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": k, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -306,6 +345,8 @@ def main():
                     help="Muon for the hidden-layer weights (the paper's default optimizer), AdamW for the rest")
     ap.add_argument("--stacked", action="store_true",
                     help="a batch per member (idx [m, B], Sec. 3.6) instead of one batch shared by all members")
+    ap.add_argument("--reference-seconds", type=float, default=120.0,
+                    help="--impl reference: CPU seconds the W + K oracle steps are sized to")
     ap.add_argument("--emb", action="store_true",
                     help="periodic feature embeddings (App. Feature Embeddings), d_emb and sigma per member "
                          "from the paper's sampling space")
