@@ -61,3 +61,25 @@ def test_reference_arm_prints_from_rank_zero_only():
     import json
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
+
+
+def test_reference_arm_fits_its_time_budget():
+    """`bench.py --impl reference` times exactly K oracle steps and sizes
+    each step's rows so that W + K steps fit the budget: with K = 400 and a
+    4 s budget on the tiny workload the rows are cut below the batch (on a
+    host fast enough for 400 full steps in 4 s they are not) and the run ends
+    in seconds."""
+    import json
+    import time
+    cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "400", "--warmup", "3",
+           "--workload", "tiny", "--reference-seconds", "4"]
+    t0 = time.perf_counter()
+    r = subprocess.run(cmd, capture_output=True, text=True, timeout=300, cwd=ROOT)
+    wall = time.perf_counter() - t0
+    assert r.returncode == 0, r.stderr[-2000:]
+    d = json.loads(r.stdout.strip().splitlines()[-1])
+    assert d["impl"] == "reference" and d["steps"] == 400 and d["value"] > 0
+    sample = d["cpu_baseline"]["sample"]
+    assert "400 timed steps of" in sample and ("cut to fit" in sample or "the full batch" in sample)
+    assert d["e2e"]["h2d_bytes_per_step"] == 0
+    assert wall < 120, wall
