@@ -419,7 +419,7 @@ def test_emb_maximum_size(tp, prec):
     d_in, d_out, m = 40, 4, 2
     hp = random_pack(m, d_in, d_out, seed=107, width=(32, 96, 16), depth=(1, 2))
     em = sample_emb_fixed(m, d_in, [64, 2], seed=17)
-    pk, orc = emb_pair(tp, "multiclass", d_in, d_out, hp, em, prec, 128)
+    pk, orc = emb_pair(tp, "multiclass", d_in, d_out, hp, em, prec, 256)
     randomise_emb(pk, orc, em, d_in, seed=18)
     X, y = make_data("multiclass", 300, d_in, d_out, 11)
     idx = np.random.default_rng(12).choice(300, 130, replace=False).astype(np.int32)
