@@ -116,7 +116,8 @@ tp_status pack_create_emb(const tp_config* cfg, const int32_t* depth, const int3
                           const float* freq, void* cuda_stream, tabpack_t** out);
 
 /* Member `member`'s embedding parameters (grads = 1: their gradients from
- * the last step without update), copied to the host array out of
+ * the last step; a pack with embeddings stores them on every step, since
+ * its optimizer runs as a separate pass), copied to the host array out of
  * d_in (4 d - 2) floats: w [d_in, d - 1], b [d_in, d - 1], alpha [d_in, d],
  * beta [d_in, d], d = its d_emb.  TP_EINVAL for a pack without
  * embeddings.  Synchronises.                                                */
