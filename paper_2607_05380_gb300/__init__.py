@@ -281,7 +281,7 @@ class Pack:
 
     def emb(self, member, grads=False):
         """(w, b, alpha, beta) of a member's embeddings, or their gradients
-        from the last step without update."""
+        from the last step."""
         if self.d_emb is None:
             _check(load_library().pack_get_emb(self._h, 0, 0, None), self._h)
         d, n = int(self.d_emb[member]), self.d_in
