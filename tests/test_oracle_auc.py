@@ -45,3 +45,19 @@ def test_monotone_transform_invariance():
     s = rng.uniform(-1, 1, 200)
     y = (rng.uniform(0, 1, 200) < 0.4).astype(np.int32)
     assert oracle.auc(s, y) == oracle.auc(s ** 3 + 2 * s, y)
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_matches_scikit_learn(seed):
+    """Against scikit-learn's roc_auc_score (an independent implementation,
+    trapezoidal area under the ROC curve, which counts ties as 1/2), on
+    fp32 scores with and without ties."""
+    metrics = pytest.importorskip("sklearn.metrics")
+    rng = np.random.default_rng(100 + seed)
+    n = int(rng.integers(5, 400))
+    s = rng.uniform(0, 1, n).astype(np.float32)
+    if seed % 2:
+        s = (np.round(s * 16) / 16).astype(np.float32)
+    y = rng.integers(0, 2, n).astype(np.int32)
+    y[0], y[1] = 0, 1
+    assert oracle.auc(s, y) == pytest.approx(metrics.roc_auc_score(y, s.astype(np.float64)), abs=1e-12)
