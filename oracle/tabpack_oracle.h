@@ -31,10 +31,10 @@
  *     the precision in which the GPU scorer takes the same decision.
  *
  * Parity status: every function here is pinned by tests in tests/ against
- * closed forms, finite differences, torch CPU fp64 library routines or brute
- * force, except the Philox word values, which are pinned only structurally
- * (Weyl key constants from their closed forms, round invertibility) and
- * statistically -- "parity unpinned" at the level of individual words.
+ * closed forms, finite differences, torch CPU fp64 library routines, brute
+ * force or published values; Philox4x32-10 word by word by the known-answer
+ * vectors published with Random123 (Salmon et al., SC'11), and structurally
+ * (Weyl key constants from their closed forms, round invertibility).
  */
 #ifndef TABPACK_ORACLE_H
 #define TABPACK_ORACLE_H

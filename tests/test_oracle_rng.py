@@ -1,10 +1,13 @@
 """Pins for the oracle's random streams and number formats (CPU only).
 
-Philox4x32-10 is pinned by inverting it: the inverse below is derived from
-the round definition in Salmon et al. (SC'11) with the Weyl key increments
-computed here from their closed forms, 2^32 (golden ratio - 1) and
-2^32 (sqrt(3) - 1).  Word values beyond that are pinned only statistically.
+Philox4x32-10 is pinned word by word by the known-answer vectors published
+with Random123 (Salmon et al., SC'11; tests/golden/philox4x32_10_kat.json),
+and structurally by inverting it: the inverse below is derived from the
+round definition with the Weyl key increments computed here from their
+closed forms, 2^32 (golden ratio - 1) and 2^32 (sqrt(3) - 1).
 """
+import json
+import os
 from decimal import Decimal, getcontext
 
 import numpy as np
@@ -38,6 +41,20 @@ def _philox_inverse(out, key):
         c3 = n2 ^ hi0 ^ k1
         n0, n1, n2, n3 = c0, c1, c2, c3
     return [n0, n1, n2, n3]
+
+
+def _kat():
+    with open(os.path.join(os.path.dirname(__file__), "golden", "philox4x32_10_kat.json")) as f:
+        g = json.load(f)
+    return [([int(x, 16) for x in v["ctr"]], [int(x, 16) for x in v["key"]], [int(x, 16) for x in v["out"]])
+            for v in g["vectors"]]
+
+
+@pytest.mark.parametrize("k", range(3))
+def test_philox_known_answer_vectors(orc, k):
+    """The three published philox4x32 10-round vectors, word for word."""
+    ctr, key, out = _kat()[k]
+    assert [int(w) for w in orc.philox4x32_10(ctr, key)] == out
 
 
 def test_weyl_constants_closed_form():
