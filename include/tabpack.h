@@ -310,6 +310,25 @@ tp_status pack_debug_masks(tabpack_t* pack, int32_t member, int32_t layer, uint3
  * [B, width] with B the last step's batch size.  For tests and diagnostics. */
 tp_status pack_debug_activations(tabpack_t* pack, int32_t member, int32_t layer, float* out);
 
+/* The dropout keep mask held in the pack's mask arena for hidden layer
+ * `layer` of `member` (bf16 mode): the words the forward epilogue reads
+ * (Sec. 3.3, one mask per member at its own rate), decoded to host uint8
+ * keep [B, width] (1 keep, 0 drop) for rows 0 .. B-1 (B <= max_batch).
+ * *step_held receives the step whose masks the arena holds (-1: none yet).
+ * After a training step t the arena holds step t + 1's masks (the optimizer
+ * pass fills them), which the forward of step t + 1 then reads unchanged;
+ * after pack_forward_backward(t) it holds step t's, the ones that forward
+ * applied.  Layers with rate 0 report all ones.  TP_ESTATE in fp32 mode,
+ * whose epilogue evaluates the keep bits itself.  Synchronises.            */
+tp_status pack_debug_mask_arena(tabpack_t* pack, int32_t member, int32_t layer, int32_t B, uint8_t* keep,
+                                int64_t* step_held);
+
+/* Philox4x32-10 (Salmon et al., SC'11) as the device evaluates it for the
+ * dropout masks and the initial values: out[i] = the four words of counter
+ * ctr[i] (host uint32 [n, 4]) under key key[i] (host uint32 [n, 2]).  Runs
+ * on the current device's default stream and synchronises; for tests.     */
+tp_status pack_debug_philox(const uint32_t* ctr, const uint32_t* key, int32_t n, uint32_t* out);
+
 /* Per-kernel-family timing with CUDA events recorded on the pack's stream.
  * Enable, run work, then read the accumulated milliseconds and launch counts
  * (synchronises).  Families: see tp_phase.                                  */

@@ -68,6 +68,7 @@ def lib():
                 "orc_philox4x32_10": (None, [P, P, P]),
                 "orc_dropout_keep": (ctypes.c_int, [u64, u32, u32, u32, u32, u32, ctypes.c_float]),
                 "orc_round_bf16": (f64, [f64]),
+                "orc_dropout_mask": (None, [u64, u32, u32, u32, i32, i32, ctypes.c_float, P]),
                 "orc_create": (P, [ctypes.POINTER(_Config), P, P, P, P, P, P]),
                 "orc_destroy": (None, [P]),
                 "orc_init_value": (f64, [u64, u32, u32, u32, i32]),
@@ -118,6 +119,13 @@ def philox4x32_10(ctr, key):
 
 def dropout_keep(seed, member_id, layer, step, row, col, p) -> int:
     return int(lib().orc_dropout_keep(seed, member_id, layer, step, row, col, float(p)))
+
+
+def dropout_mask(seed, member_id, layer, step, B, w, p):
+    """Keep mask [B, w] (uint8, 1 = keep) of one hidden layer at one step."""
+    out = np.zeros((int(B), int(w)), dtype=np.uint8)
+    lib().orc_dropout_mask(int(seed), int(member_id), int(layer), int(step), int(B), int(w), float(p), _ptr(out))
+    return out
 
 
 def round_bf16(x: float) -> float:

@@ -75,6 +75,23 @@ int orc_dropout_keep(uint64_t seed, uint32_t member_id, uint32_t layer, uint32_t
   return r >= T ? 1 : 0;
 }
 
+/* The keep mask of rows 0..B-1 and columns 0..w-1 of one hidden layer at one
+ * step (out [B, w], 1 = keep): orc_dropout_keep element by element.        */
+void orc_dropout_mask(uint64_t seed, uint32_t member_id, uint32_t layer, uint32_t step,
+                      int32_t B, int32_t w, float p, uint8_t* out) {
+  const uint32_t T = orc_drop_threshold(p);
+  #pragma omp parallel for schedule(static)
+  for (int32_t r = 0; r < B; ++r)
+    for (int32_t c4 = 0; c4 < w; c4 += 4) {   /* one counter gives columns c4 .. c4 + 3 */
+      const uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+      const uint32_t ctr[4] = {(uint32_t)r, (uint32_t)c4 >> 2, step, (member_id << 4) | layer};
+      uint32_t word[4];
+      orc_philox4x32_10(ctr, key, word);
+      for (int32_t k = 0; k < 4 && c4 + k < w; ++k)
+        out[(int64_t)r * w + c4 + k] = (uint8_t)(T == 0 || word[k] >= T);
+    }
+}
+
 /* bfloat16 storage rounding.  A value stored in bf16 is first an fp32 value
  * (the GPU computes in fp32), so x is rounded to fp32 and then to bf16: 8
  * significant bits, fp32 exponent range, subnormal ulp 2^-133, round to

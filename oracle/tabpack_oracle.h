@@ -77,6 +77,10 @@ void orc_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t ou
 int orc_dropout_keep(uint64_t seed, uint32_t member_id, uint32_t layer, uint32_t step,
                      uint32_t row, uint32_t col, float p);
 
+/* orc_dropout_keep for rows 0..B-1, columns 0..w-1: out [B, w] uint8.   */
+void orc_dropout_mask(uint64_t seed, uint32_t member_id, uint32_t layer, uint32_t step,
+                      int32_t B, int32_t w, float p, uint8_t* out);
+
 /* Round-to-nearest-even to bfloat16, result returned as a double. */
 double orc_round_bf16(double x);
 

@@ -35,7 +35,8 @@ SYMBOLS = ["pack_create", "pack_destroy", "pack_set_stream", "pack_train_step", 
            "pack_get_stream", "pack_online_create", "pack_online_destroy", "pack_online_epoch", "pack_online_info",
            "pack_online_members", "pack_online_ensemble", "pack_online_snapshot", "pack_online_predict",
            "pack_online_last_error", "pack_train_step_stacked", "pack_forward_backward_stacked", "pack_set_muon",
-           "pack_debug_muon_dir", "pack_create_emb", "pack_get_emb", "pack_set_emb", "pack_member_emb"]
+           "pack_debug_muon_dir", "pack_create_emb", "pack_get_emb", "pack_set_emb", "pack_member_emb",
+           "pack_debug_mask_arena", "pack_debug_philox"]
 
 
 class TabpackError(RuntimeError):
@@ -116,6 +117,8 @@ def load_library(path: str = LIB_PATH):
         "pack_get_emb": (st, [P, i32, i32, P]),
         "pack_set_emb": (st, [P, i32, P]),
         "pack_member_emb": (st, [P, i32, P]),
+        "pack_debug_mask_arena": (st, [P, i32, i32, i32, P, P]),
+        "pack_debug_philox": (st, [P, P, i32, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -338,6 +341,14 @@ class Pack:
         _check(load_library().pack_debug_masks(self._h, member, layer, int(step), int(B), _hptr(out)), self._h)
         return out
 
+    def debug_mask_arena(self, member, layer, B):
+        """(keep [B, width] uint8, step) held in the bf16 mask arena."""
+        out = np.zeros((B, int(self.width[member])), dtype=np.uint8)
+        held = ctypes.c_int64(0)
+        _check(load_library().pack_debug_mask_arena(self._h, member, layer, int(B), _hptr(out), ctypes.byref(held)),
+               self._h)
+        return out, held.value
+
     def debug_activations(self, member, layer):
         out = np.zeros((self._B, int(self.width[member])), dtype=np.float32)
         _check(load_library().pack_debug_activations(self._h, member, layer, _hptr(out)), self._h)
@@ -360,6 +371,17 @@ class Pack:
         b = ctypes.c_int64()
         _check(load_library().pack_sizes(self._h, ctypes.byref(n), ctypes.byref(b)), self._h)
         return n.value, b.value
+
+
+def debug_philox(ctr, key):
+    """The device's Philox4x32-10 words [n, 4] for counters [n, 4], keys [n, 2]."""
+    c = np.ascontiguousarray(np.atleast_2d(ctr), dtype=np.uint32)
+    k = np.ascontiguousarray(np.atleast_2d(key), dtype=np.uint32)
+    if c.shape[1] != 4 or k.shape != (c.shape[0], 2):
+        raise ValueError("ctr must be [n, 4] and key [n, 2]")
+    out = np.zeros((c.shape[0], 4), dtype=np.uint32)
+    _check(load_library().pack_debug_philox(_hptr(c), _hptr(k), c.shape[0], _hptr(out)))
+    return out
 
 
 def select_greedy(preds, y, task, score="loss", m_ens=32, stream=None, static_scratch=False):

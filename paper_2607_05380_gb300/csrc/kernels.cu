@@ -821,6 +821,20 @@ __global__ void k_debug_masks(uint8_t* __restrict__ out, int32_t B, int32_t w, u
   }
 }
 
+// ------------------------------------------------------------- Philox words
+// in [n, 6]: counter c0..c3 then key k0, k1; out [n, 4]: the four words.
+__global__ void k_debug_philox(const uint32_t* __restrict__ in, uint32_t* __restrict__ out, int32_t n) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const uint32_t* c = in + (int64_t)i * 6;
+  const U4 r = philox10(c[0], c[1], c[2], c[3], c[4], c[5]);
+  uint32_t* o = out + (int64_t)i * 4;
+  o[0] = r.x;
+  o[1] = r.y;
+  o[2] = r.z;
+  o[3] = r.w;
+}
+
 // ------------------------------------------------------------- launchers
 template <typename T>
 void launch_gather(cudaStream_t st, const float* X, const int32_t* idx, const StepDyn* dyn, int B, int B_pad,
@@ -1139,6 +1153,10 @@ void launch_predict_head(cudaStream_t st, const PredictHeadArgs<T>& g, int n_job
 void launch_debug_masks(cudaStream_t st, uint8_t* out, int B, int w, uint64_t seed, uint32_t member,
                         uint32_t layer, uint32_t step, uint32_t T) {
   k_debug_masks<<<64, 256, 0, st>>>(out, B, w, seed, member, layer, step, T);
+}
+
+void launch_debug_philox(cudaStream_t st, const uint32_t* in, uint32_t* out, int n) {
+  k_debug_philox<<<(int)ceil_div(n, 128), 128, 0, st>>>(in, out, n);
 }
 
 #define TP_INSTANTIATE(T)                                                                              \

@@ -160,6 +160,7 @@ template <typename T>
 void launch_predict_head(cudaStream_t st, const PredictHeadArgs<T>& g, int n_jobs);
 void launch_debug_masks(cudaStream_t st, uint8_t* out, int B, int w, uint64_t seed, uint32_t member,
                         uint32_t layer, uint32_t step, uint32_t T);
+void launch_debug_philox(cudaStream_t st, const uint32_t* in, uint32_t* out, int n);
 
 // Sets the per-thread message pack_last_error(NULL) returns (tabpack.cu).
 void record_thread_error(const char* msg);

@@ -1755,6 +1755,51 @@ tp_status pack_debug_masks(tabpack_t* h, int32_t member, int32_t layer, uint32_t
   return TP_OK;
 }
 
+tp_status pack_debug_mask_arena(tabpack_t* h, int32_t member, int32_t layer, int32_t B, uint8_t* keep,
+                                int64_t* step_held) {
+  TP_TRY(check_ml(h, member, layer));
+  if (layer >= h->depth[member]) return fail(h, TP_EINVAL, "layer %d is the head", layer);
+  if (B < 1 || B > h->B_cap || !keep || !step_held) return fail(h, TP_EINVAL, "bad B or null output");
+  if (!h->bf16) return fail(h, TP_ESTATE, "fp32 mode evaluates dropout in the epilogue: no mask arena");
+  TP_TRY(sync_check(h));
+  const int w = h->width[member];
+  *step_held = h->masks_for;
+  const int64_t off = h->mask_off[member][layer];
+  if (off < 0) {  // p = 0: the forward applies no mask
+    memset(keep, 1, (size_t)B * w);
+    return TP_OK;
+  }
+  const int n_chunk = (int)ceil_div(w, 32);
+  std::vector<uint32_t> words((size_t)n_chunk * h->B_cap);
+  TP_CUDA(h, cudaMemcpy(words.data(), h->masks + off, sizeof(uint32_t) * words.size(), cudaMemcpyDeviceToHost));
+  for (int r = 0; r < B; ++r)
+    for (int c = 0; c < w; ++c)
+      keep[(size_t)r * w + c] = (uint8_t)((words[(size_t)(c >> 5) * h->B_cap + r] >> (c & 31)) & 1u);
+  return TP_OK;
+}
+
+tp_status pack_debug_philox(const uint32_t* ctr, const uint32_t* key, int32_t n, uint32_t* out) {
+  if (n < 1 || !ctr || !key || !out) return fail(nullptr, TP_EINVAL, "bad n or null pointer");
+  std::vector<uint32_t> in((size_t)n * 6);
+  for (int32_t i = 0; i < n; ++i) {
+    for (int q = 0; q < 4; ++q) in[(size_t)i * 6 + q] = ctr[(size_t)i * 4 + q];
+    in[(size_t)i * 6 + 4] = key[(size_t)i * 2];
+    in[(size_t)i * 6 + 5] = key[(size_t)i * 2 + 1];
+  }
+  uint32_t* d = nullptr;
+  cudaError_t e = cudaMalloc(&d, sizeof(uint32_t) * (size_t)n * 10);
+  if (e != cudaSuccess) return fail(nullptr, TP_ECUDA, "debug philox: %s", cudaGetErrorString(e));
+  e = cudaMemcpy(d, in.data(), sizeof(uint32_t) * in.size(), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) {
+    tp::launch_debug_philox(0, d, d + (size_t)n * 6, n);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) e = cudaMemcpy(out, d + (size_t)n * 6, sizeof(uint32_t) * (size_t)n * 4, cudaMemcpyDeviceToHost);
+  cudaFree(d);
+  if (e != cudaSuccess) return fail(nullptr, TP_ECUDA, "debug philox: %s", cudaGetErrorString(e));
+  return TP_OK;
+}
+
 tp_status pack_debug_activations(tabpack_t* h, int32_t member, int32_t layer, float* out) {
   TP_TRY(check_ml(h, member, layer));
   if (layer >= h->depth[member]) return fail(h, TP_EINVAL, "layer %d is the head", layer);

@@ -1,15 +1,14 @@
 """GPU path versus the CPU oracle, element by element, through the C ABI.
 
 Bars: dropout masks, init values and selected indices bit-exact; floats
-within max relative error 1e-4 (fp32 mode, vs the fp64 oracle) and 2e-2
-(bf16 mode, vs the oracle's bf16-storage mode), where the relative error of
-an entry is |g - o| / max(|o|, rms(o)) -- the tensor's rms is the floor for
-entries near zero.
-
-A ReLU pre-activation within rounding of zero makes both masks valid
-subgradients; in fp32 mode a member whose oracle pre-activations came within
-1e-5 rms of zero in any compared step is checked at the bf16 bar instead and
-counted (the test requires most members to meet the strict bar).
+within max relative error 1e-4 (fp32 mode) and 2e-2 (bf16 mode) of the fp64
+oracle run in exact arithmetic, with the rules of tests/parity.py: the
+relative error of an entry is |g - o| / max(|o|, rms(o)); where the
+oracle's own bf16-storage model of the method is further than 2e-2 from its
+exact result (shown by the oracle alone), the GPU is held within twice that
+distance; ReLU decisions may differ only at oracle near-ties; the
+bf16-storage oracle (the same storage points) is a second comparison at
+2e-2.
 """
 import numpy as np
 import pytest
@@ -18,6 +17,7 @@ torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
 import oracle  # noqa: E402
+from parity import TOL, Oracles, check_bf16_vs_exact, compare_params, compare_step, rel_err  # noqa: E402
 from workloads import random_pack  # noqa: E402
 
 
@@ -33,17 +33,6 @@ def tp():
 
 
 DEV = "cuda"
-TOL = {"fp32": 1e-4, "bf16": 2e-2}
-
-
-def rel_err(got, ref):
-    got = np.asarray(got, dtype=np.float64)
-    ref = np.asarray(ref, dtype=np.float64)
-    if ref.size == 0:
-        return 0.0
-    rms = np.sqrt(np.mean(ref ** 2))
-    floor = np.maximum(np.abs(ref), rms if rms > 0 else 1e-30)
-    return float(np.max(np.abs(got - ref) / floor))
 
 
 def make_data(task, n, d_in, d_out, seed):
@@ -61,8 +50,7 @@ def make_data(task, n, d_in, d_out, seed):
 def pair(tp, task, d_in, d_out, hp, prec, max_batch, seed=2, fuse=False):
     pk = tp.Pack(d_in, d_out, task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
                  max_batch=max_batch, seed=seed, precision=prec, fuse_optimizer=fuse)
-    orc = oracle.OraclePack(d_in, d_out, task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
-                            seed=seed, bf16_storage=(prec == "bf16"))
+    orc = Oracles(prec, d_in, d_out, task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"], seed=seed)
     return pk, orc
 
 
@@ -93,85 +81,29 @@ def test_dropout_masks_bit_exact(tp, step):
             np.testing.assert_array_equal(pk.debug_masks(i, l, step, 200), orc.keep(i, l))
 
 
-# A ReLU decision whose pre-activation lies within rounding of zero may go
-# either way on the two sides; both results are valid subgradients.  In bf16
-# mode a one-ulp difference in a stored activation (the fp32 and fp64 values
-# straddling a bf16 rounding boundary) moves the next layer's pre-activations
-# by a fraction of an ulp of their rms; each layer turns more of them into
-# straddles, so the discrepancy grows with depth (in a 4-layer member of width
-# 1024 on 2048 rows it reaches ~1e-3 rms(Z) at the last layer).  One flip at
-# (row b, unit j) of layer l changes dW_l[j, :] by one of the B batch terms
-# and every upstream gradient by a fraction of a percent.  The test therefore
-# reads the GPU's stored activations, finds every flipped decision exactly
-# (GPU H > 0 versus oracle keep & Z > 0), and requires each flip to sit at an
-# oracle near-tie: |Z| below the larger of TIE * rms(Z) and twice the
-# layer's largest measured GPU-versus-oracle discrepancy of the
-# pre-activations near zero (units kept and positive on both sides with
-# |Z| < 0.05 rms(Z), where the GPU's pre-activation is its stored H times
-# 1 - p; the discrepancy comes from discrete one-ulp events, so its tail and
-# not its rms is what a flip has to be compared with).  Members without
-# flips are held to the strict elementwise bar everywhere, members with flips
-# to the strict bar on losses and logits and to the bar norm-wise on each
-# gradient tensor.
-TIE = {"fp32": 1e-5, "bf16": 5e-3}
+def _kat():
+    import json
+    import os
+    with open(os.path.join(os.path.dirname(__file__), "golden", "philox4x32_10_kat.json")) as f:
+        g = json.load(f)
+    return [([int(x, 16) for x in v["ctr"]], [int(x, 16) for x in v["key"]], [int(x, 16) for x in v["out"]])
+            for v in g["vectors"]]
 
 
-def _flips(pk, orc, i, L, prec, oi=None, p_drop=0.0):
-    """Flipped ReLU / dropout decisions of GPU member i (oracle member oi)."""
-    oi = i if oi is None else oi
-    n = 0
-    for l in range(L):
-        Hg = pk.debug_activations(i, l).astype(np.float64)
-        Zo = orc.preact(oi, l)
-        keep = orc.keep(oi, l) > 0
-        mo = (Zo > 0) & keep
-        diff = (Hg > 0) != mo
-        if diff.any():
-            zr = np.sqrt(np.mean(Zo ** 2))
-            near = keep & (Hg > 0) & (Zo > 0) & (Zo < 0.05 * zr)
-            noise = 0.0
-            if near.sum() >= 100:
-                zg = Hg[near] * (1.0 - float(np.float32(p_drop)))
-                noise = float(np.max(np.abs(zg - Zo[near])) / zr)
-            worst = float(np.max(np.abs(Zo[diff])) / zr)
-            assert worst < max(TIE[prec], 2.0 * noise), ("flip away from a near-tie", i, l, worst, noise)
-            n += int(diff.sum())
-    return n
-
-
-def _compare_step(pk, orc, hp, prec, loss_gpu, loss_orc, members=None, max_flip_members=None):
-    """GPU members `members` (default: all) against oracle members 0, 1, ...
-    (the oracle may hold only the sampled members; they are independent)."""
-    tol = TOL[prec]
-    members = list(range(len(hp["depth"]))) if members is None else list(members)
-    problems = {}
-    n_flip_members = 0
-    for oi, i in enumerate(members):
-        L = int(hp["depth"][i])
-        flips = _flips(pk, orc, i, L, prec, oi, float(hp["dropout"][i]))
-        n_flip_members += flips > 0
-        p = []
-        le = abs(loss_gpu[i] - loss_orc[oi]) / max(1.0, abs(loss_orc[oi]))
-        ge = rel_err(pk.logits(i), orc.logits(oi))
-        if le > tol or ge > tol:
-            p.append(("loss/logits", le, ge))
-        for l in range(L + 1):
-            gW, gb = pk.get_grads(i, l)
-            oW, ob = orc.get_grads(oi, l)
-            if flips == 0:
-                e = max(rel_err(gW, oW), rel_err(gb, ob))
-            else:
-                g = np.concatenate([gW.ravel(), gb]).astype(np.float64)
-                o = np.concatenate([oW.ravel(), ob])
-                e = float(np.linalg.norm(g - o) / max(np.linalg.norm(o), 1e-30))
-            if e > tol:
-                p.append(("grad", l, flips, e))
-        if p:
-            problems[i] = p
-    if max_flip_members is None:
-        max_flip_members = max(1, len(members) // 3)
-    assert n_flip_members <= max_flip_members, ("too many members with flips", n_flip_members)
-    return problems
+def test_device_philox_known_answers(tp):
+    """The device's Philox4x32-10 (the function behind every dropout mask
+    and initial value) reproduces Random123's published known-answer
+    vectors word for word, and the oracle's words on random counters."""
+    kat = _kat()
+    got = tp.debug_philox([c for c, _, _ in kat], [k for _, k, _ in kat])
+    for (_, _, out), g in zip(kat, got):
+        assert [int(w) for w in g] == out
+    rng = np.random.default_rng(17)
+    ctr = rng.integers(0, 2 ** 32, (500, 4), dtype=np.uint64).astype(np.uint32)
+    key = rng.integers(0, 2 ** 32, (500, 2), dtype=np.uint64).astype(np.uint32)
+    got = tp.debug_philox(ctr, key)
+    want = np.stack([oracle.philox4x32_10(c, k) for c, k in zip(ctr, key)])
+    np.testing.assert_array_equal(got, want)
 
 
 @pytest.mark.parametrize("prec", ["fp32", "bf16"])
@@ -188,7 +120,7 @@ def test_one_step_logits_losses_grads(tp, prec, task, d_out, B):
     loss = torch.zeros(len(hp["depth"]), dtype=torch.float32, device=DEV)
     pk.forward_backward(Xd, idxd, yd, 5, loss)
     lo = orc.train_step(X, idx, y, 5, update=False)
-    problems = _compare_step(pk, orc, hp, prec, loss.cpu().numpy(), lo)
+    problems = compare_step(pk, orc, hp, prec, loss.cpu().numpy())
     assert not problems, problems
 
 
@@ -209,7 +141,7 @@ def test_stacked_batches_one_step(tp, prec, task, d_out, B):
     loss = torch.zeros(m, dtype=torch.float32, device=DEV)
     pk.forward_backward(Xd, idxd, yd, 5, loss)
     lo = orc.train_step(X, idx, y, 5, update=False)
-    problems = _compare_step(pk, orc, hp, prec, loss.cpu().numpy(), lo)
+    problems = compare_step(pk, orc, hp, prec, loss.cpu().numpy())
     assert not problems, problems
     # the shared-batch step on row 3 gives member 3 the same result
     pk2, _ = pair(tp, task, d_in, d_out, hp, prec, 256)
@@ -243,23 +175,19 @@ def test_stacked_batches_ten_steps(tp, prec):
         pk.train_step(Xd, idxd, yd, step, loss)
         lo = orc.train_step(X, idx, y, step)
         margin = np.minimum(margin, [orc.margin(i) for i in range(m)])
-        lg = loss.cpu().numpy()
-        for i in range(m):
-            assert abs(lg[i] - lo[i]) <= TOL["bf16"] * max(1.0, abs(lo[i])), (step, i, lg[i], lo[i])
-    errs = {}
-    for i in range(m):
-        e = 0.0
-        for l in range(int(hp["depth"][i]) + 1):
-            W, b = pk.get_params(i, l)
-            Wo, bo = orc.get_params(i, l)
-            e = max(e, rel_err(W, Wo), rel_err(b, bo))
-        errs[i] = e
-    bad = {i: e for i, e in errs.items() if e > TOL[prec]}
-    if prec == "fp32":
-        ties = {i for i in bad if margin[i] < 1e-5}
-        assert all(errs[i] <= TOL["bf16"] for i in ties), (errs, margin)
-        bad = {i: e for i, e in bad.items() if i not in ties}
-    assert not bad, (errs, margin)
+        _check_losses(loss.cpu().numpy(), lo, prec, margin, step)
+    errs, problems, relaxed = compare_params(pk, orc, hp, prec, margin=margin)
+    assert not problems, (problems, errs, margin)
+    assert len(relaxed) <= m // 4, (relaxed, errs, margin)
+
+
+def _check_losses(lg, lo, prec, margin, step):
+    """Per-step member losses against the exact oracle at the mode's bar (in
+    fp32 mode a member whose oracle pre-activations came within 1e-5 rms of
+    a ReLU tie in some step is held at the bf16 bar)."""
+    for i in range(len(lo)):
+        bar = TOL[prec] if (prec == "bf16" or margin[i] >= 1e-5) else TOL["bf16"]
+        assert abs(lg[i] - lo[i]) <= bar * max(1.0, abs(lo[i])), (step, i, lg[i], lo[i], bar)
 
 
 @pytest.mark.parametrize("prec,fuse", [("fp32", False), ("bf16", False), ("bf16", True)])
@@ -281,25 +209,10 @@ def test_ten_steps_params(tp, prec, fuse, task, d_out):
         pk.train_step(Xd, idxd, yd, step, loss)
         lo = orc.train_step(X, idx, y, step)
         margin = np.minimum(margin, [orc.margin(i) for i in range(m)])
-        lg = loss.cpu().numpy()
-        for i in range(m):
-            assert abs(lg[i] - lo[i]) <= TOL["bf16"] * max(1.0, abs(lo[i])), (step, i, lg[i], lo[i])
-    errs = {}
-    for i in range(m):
-        e = 0.0
-        for l in range(int(hp["depth"][i]) + 1):
-            W, b = pk.get_params(i, l)
-            Wo, bo = orc.get_params(i, l)
-            e = max(e, rel_err(W, Wo), rel_err(b, bo))
-        errs[i] = e
-    tol = TOL[prec]
-    bad = {i: e for i, e in errs.items() if e > tol}
-    if prec == "fp32":
-        ties = {i for i in bad if margin[i] < 1e-5}
-        assert all(errs[i] <= TOL["bf16"] for i in ties), (errs, margin)
-        bad = {i: e for i, e in bad.items() if i not in ties}
-        assert len(ties) <= m // 4, (errs, margin)
-    assert not bad, (errs, margin)
+        _check_losses(loss.cpu().numpy(), lo, prec, margin, step)
+    errs, problems, relaxed = compare_params(pk, orc, hp, prec, margin=margin)
+    assert not problems, (problems, errs, margin)
+    assert len(relaxed) <= m // 4, (relaxed, errs, margin)
 
 
 def _adamw_of_own_grads(pk_step, pk_grads, hp, members, step_fn, t=1, tol=1e-5):
@@ -328,10 +241,11 @@ def test_split_column_tiles(tp, prec):
     gradients against the oracle, then the AdamW step of the separate pass
     and of the fused epilogue (bf16) against the oracle's AdamW of the GPU's
     own gradients, and three steps' parameters against the oracle (fp32, at
-    the bf16 bar: AdamW's first steps divide each gradient by its own
-    magnitude, so an entry whose gradient is near zero carries the gradient's
-    absolute error into a full-size update; the exact check of the update is
-    the one on the GPU's own gradients)."""
+    1e-4, a member that came within 1e-5 rms of a ReLU tie at the bf16 bar:
+    AdamW's first steps divide each gradient by its own magnitude, so an
+    entry whose gradient is near zero carries the gradient's absolute error
+    into a full-size update; the exact check of the update is the one on the
+    GPU's own gradients)."""
     d_in, d_out, B = 270, 3, 256
     hp = random_pack(4, d_in, d_out, seed=41, depth=(2, 3), dropout=(0.0, 0.3))
     hp["width"] = np.array([272, 336, 704, 528], dtype=np.int32)
@@ -344,23 +258,22 @@ def test_split_column_tiles(tp, prec):
     loss = torch.zeros(4, dtype=torch.float32, device=DEV)
     pk.forward_backward(Xd, idxd, yd, 3, loss)
     lo = orc.train_step(X, idx, y, 3, update=False)
-    problems = _compare_step(pk, orc, hp, prec, loss.cpu().numpy(), lo)
+    problems = compare_step(pk, orc, hp, prec, loss.cpu().numpy())
     assert not problems, problems
     for fuse in ((False, True) if prec == "bf16" else (False,)):
         pk_s, _ = pair(tp, "multiclass", d_in, d_out, hp, prec, 256, fuse=fuse)
         _adamw_of_own_grads(pk_s, pk, hp, range(4), lambda: pk_s.train_step(Xd, idxd, yd, 3, loss))
     if prec == "bf16":
         return
+    margin = np.full(4, np.inf)
     for step in range(3):
         idx = rng.choice(600, B, replace=False).astype(np.int32)
         (idxd,) = to_dev(idx)
         pk.train_step(Xd, idxd, yd, step, loss)
         orc.train_step(X, idx, y, step)
-    for i in range(4):
-        for l in range(int(hp["depth"][i]) + 1):
-            W, b = pk.get_params(i, l)
-            Wo, bo = orc.get_params(i, l)
-            assert max(rel_err(W, Wo), rel_err(b, bo)) <= TOL["bf16"], (i, l)
+        margin = np.minimum(margin, [orc.margin(i) for i in range(4)])
+    errs, problems, relaxed = compare_params(pk, orc, hp, prec, margin=margin)
+    assert not problems and len(relaxed) <= 1, (problems, errs, relaxed, margin)
 
 
 def _sample_members(wl, hp):
@@ -399,14 +312,13 @@ def test_full_size_sampled_members(tp, name):
     pk = gpu_pack(False)
     loss = torch.zeros(wl.m, dtype=torch.float32, device=DEV)
     pk.forward_backward(Xd, idxd, yd, 0, loss)
-    orc = oracle.OraclePack(wl.d_in, wl.d_out, wl.task, sub["depth"], sub["width"], sub["dropout"], sub["lr"],
-                            sub["wd"], seed=SEED_INIT, bf16_storage=True, member_id=sample)
-    lo = orc.train_step(X, idx, y, 0, update=False)
+    orc = Oracles("bf16", wl.d_in, wl.d_out, wl.task, sub["depth"], sub["width"], sub["dropout"], sub["lr"],
+                  sub["wd"], seed=SEED_INIT, member_id=sample)
+    orc.train_step(X, idx, y, 0, update=False)
     for oi, i in enumerate(sample):
         for l in range(int(hp["depth"][i])):
             np.testing.assert_array_equal(pk.debug_masks(i, l, 0, B), orc.keep(oi, l))
-    problems = _compare_step(pk, orc, hp, "bf16", loss.cpu().numpy(), lo, members=sample,
-                             max_flip_members=len(sample))
+    problems = compare_step(pk, orc, hp, "bf16", loss.cpu().numpy(), members=sample)
     assert not problems, problems
     for fuse in (False, True):
         pk_s = gpu_pack(fuse)
@@ -435,15 +347,123 @@ def test_full_size_stacked_sampled_members(tp):
                  max_batch=B, seed=SEED_INIT, precision="bf16")
     loss = torch.zeros(wl.m, dtype=torch.float32, device=DEV)
     pk.forward_backward(Xd, idxd, yd, 0, loss)
-    orc = oracle.OraclePack(wl.d_in, wl.d_out, wl.task, sub["depth"], sub["width"], sub["dropout"], sub["lr"],
-                            sub["wd"], seed=SEED_INIT, bf16_storage=True, member_id=sample)
-    lo = orc.train_step(X, idx[sample], y, 0, update=False)
+    orc = Oracles("bf16", wl.d_in, wl.d_out, wl.task, sub["depth"], sub["width"], sub["dropout"], sub["lr"],
+                  sub["wd"], seed=SEED_INIT, member_id=sample)
+    orc.train_step(X, idx[sample], y, 0, update=False)
     for oi, i in enumerate(sample):
         for l in range(int(hp["depth"][i])):
             np.testing.assert_array_equal(pk.debug_masks(i, l, 0, B), orc.keep(oi, l))
-    problems = _compare_step(pk, orc, hp, "bf16", loss.cpu().numpy(), lo, members=sample,
-                             max_flip_members=len(sample))
+    problems = compare_step(pk, orc, hp, "bf16", loss.cpu().numpy(), members=sample)
     assert not problems, problems
+
+
+def test_applied_masks_full_width_replayed(tp):
+    """The dropout masks the forward actually applies (Sec. 3.3: a mask per
+    member at its own rate), on the medium workload at full width and batch
+    (32 members, widths to 1024, B = 512, bf16, graph-replayed steps).
+    Before each step t the mask arena -- the words the forward epilogue
+    reads -- must hold exactly step t's keep bits of every active member and
+    layer (filled by the previous step's optimizer pass, or by the mask
+    kernel on a jump of the step counter or after an active-set change), and
+    after the step every unit that mask drops must read exactly 0 in the
+    stored activations while every stored non-zero unit is kept."""
+    from workloads import SEED_HP, SEED_INIT, WORKLOADS, make_data as wl_data, sample_hparams
+    wl = WORKLOADS["medium"]
+    hp = sample_hparams(wl, seed=SEED_HP)
+    B, m = wl.batch, wl.m
+    d = wl_data(wl, device="cpu", n_train=4 * B, n_val=0)
+    X, y = d["X_train"].numpy(), d["y_train"].numpy()
+    Xd, yd = to_dev(X, y)
+    pk = tp.Pack(wl.d_in, wl.d_out, wl.task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
+                 max_batch=B, seed=SEED_INIT, precision="bf16")
+    loss = torch.zeros(m, dtype=torch.float32, device=DEV)
+    rng = np.random.default_rng(12)
+    cache = {}
+
+    def want(i, l, step):
+        k = (i, l, step)
+        if k not in cache:
+            cache[k] = oracle.dropout_mask(SEED_INIT, i, l, step, B, int(hp["width"][i]), float(hp["dropout"][i]))
+        return cache[k]
+
+    def check_arena(step, active):
+        for i in np.flatnonzero(active):
+            for l in range(int(hp["depth"][i])):
+                keep, held = pk.debug_mask_arena(int(i), l, B)
+                assert held == step, (i, l, held, step)
+                np.testing.assert_array_equal(keep, want(int(i), l, step), err_msg=f"arena {i} {l} {step}")
+
+    def check_applied(step, active):
+        for i in np.flatnonzero(active):
+            for l in range(int(hp["depth"][i])):
+                H = pk.debug_activations(int(i), l)
+                kp = want(int(i), l, step).astype(bool)
+                assert not np.any(H[~kp]), ("a dropped unit is non-zero", i, l, step)
+                assert np.all(kp[H != 0]), (i, l, step)
+
+    def run(step, active, fb=False):
+        idx = rng.permutation(4 * B)[:B].astype(np.int32)
+        (idxd,) = to_dev(idx)
+        if fb:
+            pk.forward_backward(Xd, idxd, yd, step, loss)
+        else:
+            pk.train_step(Xd, idxd, yd, step, loss)
+        check_applied(step, active)
+
+    active = np.ones(m, dtype=np.uint8)
+    run(0, active)                       # first step: the mask kernel fills step 0
+    for t in range(1, 5):                # steady state: the optimizer pass filled step t
+        check_arena(t, active)
+        run(t, active)
+    run(100, active, fb=True)            # a jump: forward-backward leaves step 100's masks
+    check_arena(100, active)
+    run(100, active)
+    check_arena(101, active)
+    active[[3, 17]] = 0                  # an active-set change
+    pk.set_active(active)
+    run(101, active)
+    check_arena(102, active)
+    run(102, active)
+    active[:] = 1
+    pk.set_active(active)
+    run(103, active)
+    check_arena(104, active)
+    run(104, active)
+    check_arena(105, active)
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_full_width_ten_steps(tp, prec):
+    """Ten graph-replayed AdamW steps of the whole medium pack at full batch
+    (B = 512), and the parameters of one member of width 512 or more and
+    depth 3 or more against the oracle trained on that member alone
+    (members are independent, Sec. 3.6)."""
+    from workloads import SEED_HP, SEED_INIT, WORKLOADS, make_data as wl_data, sample_hparams
+    wl = WORKLOADS["medium"]
+    hp = sample_hparams(wl, seed=SEED_HP)
+    B, m = wl.batch, wl.m
+    cand = [i for i in range(m) if hp["depth"][i] >= 3 and hp["width"][i] >= 512]
+    i0 = min(cand, key=lambda i: int(hp["depth"][i]) * int(hp["width"][i]) ** 2)
+    d = wl_data(wl, device="cpu", n_train=6 * B, n_val=0)
+    X, y = d["X_train"].numpy(), d["y_train"].numpy()
+    Xd, yd = to_dev(X, y)
+    pk = tp.Pack(wl.d_in, wl.d_out, wl.task, hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
+                 max_batch=B, seed=SEED_INIT, precision=prec)
+    sub = {k: v[[i0]] for k, v in hp.items()}
+    orc = Oracles(prec, wl.d_in, wl.d_out, wl.task, sub["depth"], sub["width"], sub["dropout"], sub["lr"],
+                  sub["wd"], seed=SEED_INIT, member_id=[i0])
+    loss = torch.zeros(m, dtype=torch.float32, device=DEV)
+    rng = np.random.default_rng(21)
+    margin = np.full(1, np.inf)
+    for step in range(10):
+        idx = rng.permutation(6 * B)[:B].astype(np.int32)
+        (idxd,) = to_dev(idx)
+        pk.train_step(Xd, idxd, yd, step, loss)
+        lo = orc.train_step(X, idx, y, step)
+        margin = np.minimum(margin, [orc.margin(0)])
+        _check_losses(loss.cpu().numpy()[[i0]], lo, prec, margin, step)
+    errs, problems, relaxed = compare_params(pk, orc, hp, prec, members=[i0], margin=margin)
+    assert not problems, (problems, errs, margin)
 
 
 @pytest.mark.parametrize("prec", ["fp32", "bf16"])
@@ -455,9 +475,22 @@ def test_predict(tp, prec, task, d_out):
     X, y = make_data(task, 333, d_in, d_out, 4)   # fp32: 3 row chunks of 128, ragged tail; bf16: one of 384
     (Xd,) = to_dev(X)
     out = pk.predict(Xd).cpu().numpy()
-    ref = orc.predict(X)
-    for i in range(5):
-        assert rel_err(out[i], ref[i]) <= TOL[prec], i
+    _check_predictions(out, orc, X, prec)
+
+
+def _check_predictions(out, orc, X, prec):
+    """Predictions of every member against the exact oracle (bf16 mode: by
+    check_bf16_vs_exact, and against the bf16-storage oracle at 2e-2)."""
+    ref = orc.ex.predict(X)
+    if prec == "fp32":
+        for i in range(len(ref)):
+            assert rel_err(out[i], ref[i]) <= TOL[prec], i
+        return
+    ref_b = orc.bst.predict(X)
+    for i in range(len(ref)):
+        p = []
+        check_bf16_vs_exact("predictions", out[i], ref_b[i], ref[i], p, ("predict", i))
+        assert not p and rel_err(out[i], ref_b[i]) <= TOL[prec], (i, p, rel_err(out[i], ref_b[i]))
 
 
 @pytest.mark.parametrize("prec", ["fp32", "bf16"])
@@ -472,9 +505,7 @@ def test_predict_chunks(tp, prec):
     X, _ = make_data("multiclass", 8525, d_in, d_out, 8)
     (Xd,) = to_dev(X)
     full = pk.predict(Xd).cpu().numpy()
-    ref = orc.predict(X)
-    for i in range(5):
-        assert rel_err(full[i], ref[i]) <= TOL[prec], i
+    _check_predictions(full, orc, X, prec)
     np.testing.assert_array_equal(pk.predict(Xd[8192:].contiguous()).cpu().numpy(), full[:, 8192:])
     np.testing.assert_array_equal(pk.predict(Xd[:100].contiguous()).cpu().numpy(), full[:, :100])
     pk.set_active([1, 0, 1, 1, 1])
@@ -502,19 +533,19 @@ def test_inactive_members(tp, prec, fuse):
     lg = loss.cpu().numpy()
     assert np.isnan(lg[2]) and np.isnan(lo[2])
     np.testing.assert_array_equal(pk.get_params(2, 0)[0], frozen[0])
-    tol = TOL["fp32"] * 10 if prec == "fp32" else TOL["bf16"]
-    for i in (0, 1, 3):
-        for l in range(int(hp["depth"][i]) + 1):
-            assert rel_err(pk.get_params(i, l)[0], orc.get_params(i, l)[0]) <= tol
+    margin = np.array([orc.margin(i) for i in range(4)])
+    errs, problems, relaxed = compare_params(pk, orc, hp, prec, members=[0, 1, 3], margin=margin,
+                                             oracle_index=[0, 1, 3])
+    assert not problems and len(relaxed) <= 1, (problems, errs, relaxed)
     pk.set_active([1, 1, 1, 1])
     orc.set_active([1, 1, 1, 1])
     for step in (2, 3, 4):   # the re-activated member must train from its own latest weights
         pk.train_step(Xd, idxd, yd, step, loss)
         orc.train_step(X, idx, y, step)
+        margin = np.minimum(margin, [orc.margin(i) for i in range(4)])
     assert orc.member_steps(2) == 4
-    for i in range(4):
-        for l in range(int(hp["depth"][i]) + 1):
-            assert rel_err(pk.get_params(i, l)[0], orc.get_params(i, l)[0]) <= tol, (i, l)
+    errs, problems, relaxed = compare_params(pk, orc, hp, prec, margin=margin)
+    assert not problems and len(relaxed) <= 1, (problems, errs, relaxed)
 
 
 @pytest.mark.parametrize("task,score,d_out", [("multiclass", "loss", 10), ("multiclass", "accuracy", 10),

@@ -80,6 +80,9 @@ def test_reference_arm_fits_its_time_budget():
     d = json.loads(r.stdout.strip().splitlines()[-1])
     assert d["impl"] == "reference" and d["steps"] == 400 and d["value"] > 0
     sample = d["cpu_baseline"]["sample"]
-    assert "400 timed steps of" in sample and ("cut to fit" in sample or "the full batch" in sample)
+    assert "400 timed steps of" in sample and ("to fit the time budget" in sample or "the full batch" in sample)
+    # the same config keys as the GPU arm's line
+    assert set(d["config"]) == {"workload", "params", "gemm_flop_per_step", "l2", "parallelism", "batches",
+                                "optimizer", "embeddings"}
     assert d["e2e"]["h2d_bytes_per_step"] == 0
     assert wall < 120, wall

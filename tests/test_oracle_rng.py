@@ -145,3 +145,14 @@ def test_init_values(orc):
     # U(-b, b): mean 0, variance b^2 / 3
     assert abs(vals.mean()) < 5 * bound / np.sqrt(3 * len(vals))
     assert abs(vals.var() / (bound ** 2 / 3) - 1) < 0.1
+
+
+def test_dropout_mask_equals_elementwise_decisions(orc):
+    """The whole-layer mask (one counter per four columns) equals the
+    element-by-element decision, including a ragged last column group."""
+    seed, member, layer, step, p = 0xDEADBEEF12345678, 9, 3, 41, 0.37
+    B, w = 7, 30
+    m = orc.dropout_mask(seed, member, layer, step, B, w, p)
+    want = np.array([[orc.dropout_keep(seed, member, layer, step, r, c, p) for c in range(w)] for r in range(B)])
+    np.testing.assert_array_equal(m, want)
+    assert np.all(orc.dropout_mask(seed, member, layer, step, B, w, 0.0) == 1)
