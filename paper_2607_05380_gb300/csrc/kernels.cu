@@ -598,6 +598,258 @@ __global__ void __launch_bounds__(256, 2) k_head(HeadArgs<T> g) {
   }
 }
 
+constexpr int kStageWarps = 8;
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+// ----------------------------------------------- head + loss, staged (bf16)
+// The same work as k_head for one member on one 64-row block in bf16 mode,
+// with the block's H_L rows staged in shared memory by bulk copies (one per
+// row) so that H is read from HBM once and both passes run from shared
+// memory:
+//   1. logits: warp v takes the 8-column groups v, v + 8, ... and lane l rows
+//      l and l + 32 (16-byte loads; the row pitch is 16 bytes past a
+//      multiple of 128, so the eight rows of a quarter-warp fall in distinct
+//      banks), with the head weights read warp-uniformly (broadcast); the
+//      eight warps' partial logits are added in warp order through shared
+//      memory, and one thread per row takes its loss and dlogits;
+//   2. gradients: a thread owns 4 consecutive columns of a row set and walks
+//      its rows: dZ = (dlogits W_h) [H > 0] / (1 - p) stored in bf16, dW_h
+//      partials in registers; row sets (narrow members) are added in order
+//      through shared memory.
+// Shared memory: H [64][pitch] | partial logits [8][64][DO] | dlogits
+// [64][DOP] | row losses [64] | mbarrier.
+template <int DO>
+__global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
+  constexpr int DOP = DO == 1 ? 1 : (DO + 3) & ~3;
+  pdl_trigger();
+  pdl_wait();
+  const HeadJob jb = g.jobs[blockIdx.x];
+  const int r0 = jb.blk * kHeadRows;
+  if (r0 >= g.B_pad) return;
+  const MemberDev md = g.mem[jb.member];
+  const int w = md.w, d_out = g.d_out, ldh = jb.h_ld;
+  const int pitch = head_stage_pitch(w);
+  extern __shared__ __align__(128) unsigned char smem[];
+  unsigned char* Hs = smem;
+  float* zpart = reinterpret_cast<float*>(smem + (int64_t)kHeadRows * pitch);   // [8][64][DO]
+  float* dlog = zpart + kStageWarps * kHeadRows * DO;                          // [64][DOP]
+  float* lrow = dlog + kHeadRows * DOP;                                         // [64]
+  uint64_t* bar = reinterpret_cast<uint64_t*>(lrow + kHeadRows + 2);            // 8-byte aligned
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const __nv_bfloat16* __restrict__ H = g.act + jb.h_off + (int64_t)r0 * ldh;
+  const float* __restrict__ Wh = g.params + jb.w_off;
+  const float* __restrict__ bh = g.params + jb.b_off;
+  const uint32_t row_bytes = (uint32_t)w * 2u;
+
+  // stage the 64 rows (warp 0 issues one bulk copy per row)
+  if (threadIdx.x == 0) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_addr(bar)) : "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  __syncthreads();
+  if (warp == 0) {
+    if (lane == 0) {
+      asm volatile("fence.proxy.async.global;" ::: "memory");
+      asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
+                   "r"(row_bytes * (uint32_t)kHeadRows)
+                   : "memory");
+    }
+    __syncwarp();
+    for (int r = lane; r < kHeadRows; r += 32)
+      asm volatile(
+          "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+              smem_addr(Hs + (int64_t)r * pitch)),
+          "l"(H + (int64_t)r * ldh), "r"(row_bytes), "r"(smem_addr(bar))
+          : "memory");
+  }
+  {  // bounded wait for the copies (2 s); on expiry record site 20 and leave
+    uint32_t ok = 0;
+    uint64_t t0 = 0;
+    for (int it = 0;; ++it) {
+      asm volatile(
+          "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0;\n selp.u32 %0, 1, 0, p;\n}\n"
+          : "=r"(ok)
+          : "r"(smem_addr(bar))
+          : "memory");
+      if (ok) break;
+      uint64_t t;
+      asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+      if (it == 0) {
+        t0 = t;
+      } else if (t - t0 > 2000000000ull) {
+        if (g.err) atomicCAS(g.err, 0, 20);
+        return;
+      }
+    }
+  }
+
+  // 1. logits
+  {
+    float acc[2][DO];
+#pragma unroll
+    for (int q = 0; q < 2; ++q)
+#pragma unroll
+      for (int c = 0; c < DO; ++c) acc[q][c] = 0.f;
+    const int ng = w >> 3;
+    for (int gi = warp; gi < ng; gi += kStageWarps) {
+      float h[2][8];
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        const uint4 v = *reinterpret_cast<const uint4*>(Hs + (int64_t)(lane + 32 * q) * pitch + 16 * gi);
+        const __nv_bfloat16* b = reinterpret_cast<const __nv_bfloat16*>(&v);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) h[q][k] = __bfloat162float(b[k]);
+      }
+#pragma unroll
+      for (int c = 0; c < DO; ++c) {
+        if (c < d_out) {
+          const float4 wa = __ldg(reinterpret_cast<const float4*>(Wh + (int64_t)c * w + 8 * gi));
+          const float4 wb = __ldg(reinterpret_cast<const float4*>(Wh + (int64_t)c * w + 8 * gi + 4));
+          const float w8[8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
+#pragma unroll
+          for (int q = 0; q < 2; ++q)
+#pragma unroll
+            for (int k = 0; k < 8; ++k) acc[q][c] = fmaf(h[q][k], w8[k], acc[q][c]);
+        }
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < 2; ++q)
+#pragma unroll
+      for (int c = 0; c < DO; ++c) zpart[(warp * kHeadRows + lane + 32 * q) * DO + c] = acc[q][c];
+  }
+  __syncthreads();
+  if (threadIdx.x < kHeadRows) {
+    const int rl = threadIdx.x, r = r0 + rl;
+    float z[DO];
+#pragma unroll
+    for (int c = 0; c < DO; ++c) {
+      float v = 0.f;
+      for (int v8 = 0; v8 < kStageWarps; ++v8) v += zpart[(v8 * kHeadRows + rl) * DO + c];
+      z[c] = c < d_out ? v + bh[c] : 0.f;
+    }
+    float dl[DO];
+    float loss = 0.f;
+#pragma unroll
+    for (int c = 0; c < DO; ++c) dl[c] = 0.f;
+    if (r < g.B) {
+      const int32_t* idx = g.dyn ? g.dyn->idx : g.idx;
+      const void* yv = g.dyn ? g.dyn->y : g.y;
+      const int64_t row = idx ? (int64_t)idx[(int64_t)jb.member * g.idx_stride + r] : (int64_t)r;
+      loss = row_loss<DO>(g.task, d_out, z, yv, row, 1.f / (float)g.B, dl);
+      float* lg = g.logits + ((int64_t)jb.member * g.B_cap + r) * d_out;
+#pragma unroll
+      for (int c = 0; c < DO; ++c)
+        if (c < d_out) lg[c] = z[c];
+    }
+#pragma unroll
+    for (int c = 0; c < DOP; ++c) dlog[rl * DOP + c] = c < DO ? dl[c < DO ? c : 0] : 0.f;
+    lrow[rl] = loss;
+  }
+  __syncthreads();
+
+  // 2. dZ of the last hidden layer and the head-weight gradient partial
+  const int n_cg = w >> 2;
+  const int S = head_stage_split(w, DO);
+  const int rows_per_set = kHeadRows / S;
+  __nv_bfloat16* __restrict__ dZ = g.dz + jb.dz_off + (int64_t)r0 * w;
+  float* part = g.head_part + jb.part_off;
+  float a[DO][4];
+  int cg = 0, set = 0;
+  for (int u = threadIdx.x; u < n_cg * S; u += blockDim.x) {
+    cg = u % n_cg;
+    set = u / n_cg;
+    const int col = 4 * cg;
+    float Wr[DO][4];
+#pragma unroll
+    for (int c = 0; c < DO; ++c) {
+      if (c < d_out) {
+        const float4 v = __ldg(reinterpret_cast<const float4*>(Wh + (int64_t)c * w + col));
+        Wr[c][0] = v.x;
+        Wr[c][1] = v.y;
+        Wr[c][2] = v.z;
+        Wr[c][3] = v.w;
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) Wr[c][k] = 0.f;
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) a[c][k] = 0.f;
+    }
+    const int rb = set * rows_per_set;
+#pragma unroll 4
+    for (int rr = rb; rr < rb + rows_per_set; ++rr) {
+      const uint2 hv = *reinterpret_cast<const uint2*>(Hs + (int64_t)rr * pitch + 2 * col);
+      const __nv_bfloat16* hb = reinterpret_cast<const __nv_bfloat16*>(&hv);
+      float h[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) h[k] = __bfloat162float(hb[k]);
+      float dl[DOP];
+      if constexpr (DOP % 4 == 0) {
+#pragma unroll
+        for (int c = 0; c < DOP; c += 4) {
+          const float4 v = *reinterpret_cast<const float4*>(&dlog[rr * DOP + c]);
+          dl[c] = v.x;
+          dl[c + 1] = v.y;
+          dl[c + 2] = v.z;
+          dl[c + 3] = v.w;
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < DOP; ++c) dl[c] = dlog[rr * DOP + c];
+      }
+      float sacc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int c = 0; c < DO; ++c)
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          sacc[k] = fmaf(dl[c], Wr[c][k], sacc[k]);
+          a[c][k] = fmaf(dl[c], h[k], a[c][k]);
+        }
+      __align__(8) __nv_bfloat16 o[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) o[k] = __float2bfloat16_rn(h[k] > 0.f ? sacc[k] * md.scale : 0.f);
+      *reinterpret_cast<uint2*>(dZ + (int64_t)rr * w + col) = *reinterpret_cast<const uint2*>(o);
+    }
+    if (S == 1) {
+#pragma unroll
+      for (int c = 0; c < DO; ++c)
+        if (c < d_out)
+          *reinterpret_cast<float4*>(part + (int64_t)c * w + col) = make_float4(a[c][0], a[c][1], a[c][2], a[c][3]);
+    }
+  }
+  if (S > 1) {  // one (column group, row set) per thread; sets added in order (the H area is free now)
+    __syncthreads();
+    float* red = reinterpret_cast<float*>(Hs);   // [S][DO][w]
+    if (threadIdx.x < n_cg * S) {
+#pragma unroll
+      for (int c = 0; c < DO; ++c)
+        if (c < d_out)
+          *reinterpret_cast<float4*>(red + ((int64_t)set * DO + c) * w + 4 * cg) =
+              make_float4(a[c][0], a[c][1], a[c][2], a[c][3]);
+    }
+    __syncthreads();
+    for (int e = threadIdx.x; e < d_out * w; e += blockDim.x) {
+      const int c = e / w, k = e - c * w;
+      float v = 0.f;
+      for (int st = 0; st < S; ++st) v += red[((int64_t)st * DO + c) * w + k];
+      part[e] = v;
+    }
+  }
+  // bias partial and loss partial of the block (rows in order)
+  if (threadIdx.x < d_out) {
+    float v = 0.f;
+    for (int rr = 0; rr < kHeadRows; ++rr) v += dlog[rr * DOP + threadIdx.x];
+    part[(int64_t)d_out * w + threadIdx.x] = v;
+  }
+  if (threadIdx.x == 0) {
+    float sl = 0.f;
+    for (int rr = 0; rr < kHeadRows; ++rr) sl += lrow[rr];
+    g.loss_part[(int64_t)jb.member * g.n_blk_cap + jb.blk] = sl;
+  }
+}
+
 // Sum the per-block head partials (fixed order) into the head gradients and
 // the per-member mean loss; in update mode apply the member's AdamW to the
 // head parameters directly (the gradients are not stored).  Grid: member x
@@ -857,9 +1109,41 @@ void launch_gemm_simt(cudaStream_t st, const GemmArgs<T>& g, int tile_base, int 
   if (n_tiles > 0) launch_pdl(k_gemm_simt<T>, dim3(n_tiles), dim3(256), 0, st, g, tile_base);
 }
 
+template <int DO>
+static bool launch_head_stage(cudaStream_t st, const HeadArgs<__nv_bfloat16>& g, int n_jobs) {
+  const int64_t bytes = head_stage_smem(g.w_max, DO);
+  if (bytes > kHeadStageSmemMax) return false;
+  launch_pdl(k_head_stage<DO>, dim3(n_jobs), dim3(256), (size_t)bytes, st, g);
+  return true;
+}
+
+void head_stage_prepare() {
+  cudaFuncSetAttribute(k_head_stage<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kHeadStageSmemMax);
+  cudaFuncSetAttribute(k_head_stage<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, kHeadStageSmemMax);
+  cudaFuncSetAttribute(k_head_stage<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, kHeadStageSmemMax);
+  cudaFuncSetAttribute(k_head_stage<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, kHeadStageSmemMax);
+  cudaFuncSetAttribute(k_head_stage<10>, cudaFuncAttributeMaxDynamicSharedMemorySize, kHeadStageSmemMax);
+  cudaFuncSetAttribute(k_head_stage<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, kHeadStageSmemMax);
+}
+
 template <typename T>
 void launch_head(cudaStream_t st, const HeadArgs<T>& g, int n_jobs) {
   if (n_jobs <= 0) return;
+  if constexpr (std::is_same_v<T, __nv_bfloat16>) {
+    if (g.stage) {
+      bool done = false;
+      switch (head_bucket(g.d_out)) {
+        case 1: done = launch_head_stage<1>(st, g, n_jobs); break;
+        case 2: done = launch_head_stage<2>(st, g, n_jobs); break;
+        case 4: done = launch_head_stage<4>(st, g, n_jobs); break;
+        case 8: done = launch_head_stage<8>(st, g, n_jobs); break;
+        case 10: done = launch_head_stage<10>(st, g, n_jobs); break;
+        case 16: done = launch_head_stage<16>(st, g, n_jobs); break;
+        default: break;
+      }
+      if (done) return;
+    }
+  }
   switch (head_bucket(g.d_out)) {
     case 1: launch_pdl(k_head<T, 1>, dim3(n_jobs), dim3(256), 0, st, g); break;
     case 2: launch_pdl(k_head<T, 2>, dim3(n_jobs), dim3(256), 0, st, g); break;

@@ -59,7 +59,25 @@ struct HeadArgs {
   int32_t B, B_pad, B_cap, d_out, task, n_blk_cap;
   const StepDyn* dyn;     // non-NULL: take idx and y from here
   int32_t idx_stride;     // member i's rows are idx[i * idx_stride ..] (0: one shared batch)
+  int32_t w_max;          // widest member (bf16: shared-memory size of the staged head kernel)
+  int32_t stage;          // bf16: 1 = the staged head kernel where it fits in shared memory
+  int* err;               // device error word for a bounded wait that runs out (NULL: none)
 };
+
+// Staged head kernel (bf16): shared memory per block for members up to w_max
+// wide and DO classes, and the most a block may take.
+constexpr int kHeadStageSmemMax = 232448;
+__host__ __device__ constexpr int head_stage_pitch(int w) { return (int)round_up((int64_t)w * 2, 128) + 16; }
+__host__ __device__ constexpr int head_stage_split(int w, int DO) {
+  int S = 1;
+  while (S < 8 && (w / 4) * S * 2 <= 256 && S * 2 * DO <= 32) S *= 2;
+  return S;
+}
+__host__ __device__ constexpr int64_t head_stage_smem(int w_max, int DO) {
+  return (int64_t)kHeadRows * head_stage_pitch(w_max) +
+         4 * ((int64_t)8 * kHeadRows * DO + (int64_t)kHeadRows * (DO == 1 ? 1 : (DO + 3) & ~3) + kHeadRows) + 16;
+}
+void head_stage_prepare();
 
 struct HeadReduceArgs {
   const HeadReduceJob* jobs;

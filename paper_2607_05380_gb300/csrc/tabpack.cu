@@ -3,6 +3,7 @@
 // launch), the step orchestration on the pack's stream, and error handling.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <array>
 #include <cmath>
 #include <cstdarg>
@@ -882,6 +883,9 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
   hg.n_blk_cap = h->n_blk_cap;
   hg.dyn = dyn;
   hg.idx_stride = stacked ? B : 0;
+  hg.w_max = *std::max_element(h->width.begin(), h->width.end());
+  hg.stage = h->bf16 ? 1 : 0;
+  hg.err = h->bf16 && h->tc.enabled ? h->tc.err_dev : nullptr;
   launch_head<T>(h->st, hg, h->n_head_jobs);
   TP_LAUNCHED(h);
   h->launches++;
@@ -1413,6 +1417,7 @@ static tp_status create_impl(const tp_config* cfg, const int32_t* depth, const i
     h->d_emb.assign(d_emb, d_emb + cfg->m);
     h->fuse_adamw = false;   // the embedding parameters take the stand-alone AdamW pass
   }
+  if (h->bf16) head_stage_prepare();   // the staged head kernel's shared-memory limit (outside any capture)
   tp_status s = build_layout(h);
   if (s == TP_OK) s = alloc_all(h);
   if (s == TP_OK) s = build_schedule(h);

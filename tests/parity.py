@@ -214,11 +214,16 @@ def compare_step(pk, orc: Oracles, hp, prec, loss_gpu, members=None, emb_grads=N
                 p.append(("loss", "vs exact", lg, lxv, lb))
             check_bf16_vs_exact("logits", logit_g, orc.bst.logits(oi), orc.ex.logits(oi), p, "logits")
             grads_b = [orc.bst.get_grads(oi, l) for l in range(L + 1)]
+            flip_any = [f.any() for f in flips_b]
             for l in range(L + 1):
                 kind = "grad hidden" if l < L else "grad head"
                 # diagnostic: rows of layer l whose unit flipped against the
-                # bf16 model are held to the bar norm-wise
+                # bf16 model are held to the bar norm-wise, and so is the
+                # whole tensor when a layer above it flipped (the flip
+                # changes one row of the back-propagated gradient below it)
                 flip_rows = flips_b[l].any(axis=0) if l < L else np.zeros(grads_g[l][1].shape[0], dtype=bool)
+                if any(flip_any[l + 1:]):
+                    flip_rows = np.ones_like(flip_rows)
                 for t, name in ((0, "W"), (1, "b")):
                     g, ox, ob = grads_g[l][t], grads_x[l][t], grads_b[l][t]
                     check_bf16_vs_exact(kind, g, ob, ox, p, ("grad", l, name))
@@ -229,9 +234,9 @@ def compare_step(pk, orc: Oracles, hp, prec, loss_gpu, members=None, emb_grads=N
             if e > tol:
                 p.append(("logits vs bf16 model", e))
             if emb_grads is not None:
-                # a flipped first-layer decision changes one of B rows of dE,
-                # which every embedding gradient sums: norm-wise then
-                flip_b = any(f.any() for f in flips_b)
+                # a flipped decision changes one of B rows of dE, which every
+                # embedding gradient sums: norm-wise then
+                flip_b = any(flip_any)
                 for k, (g, ox, ob) in enumerate(emb_grads(i, oi)):
                     check_bf16_vs_exact("emb grad", g, ob, ox, p, ("emb grad", k))
                     e = nrm_err(g, ob) if flip_b else rel_err(g, ob)
