@@ -240,12 +240,15 @@ tp_status pack_select_greedy(const float* preds, int32_t P, int64_t N, int32_t d
  * embedding runtimes that forbid allocation calls after start-up.  It calls
  * no allocating routine.
  *   Limit: the problem must fit, N*d_out*8 + P*ceil(N/1024)*8 +
- *   (4 + m_ens + P)*4 + 768 <= 16 MiB (e.g. N = 100000 rows of 10 classes
- *   with P = 96 candidates); larger problems return TP_EINVAL with a message
- *   in pack_last_error(NULL) and do nothing.
- *   The first call on each device looks up the array's device address
- *   (cudaGetSymbolAddress, with that device current); make that first call
- *   before any stream capture.
+ *   (4 + m_ens + P)*4 + 1024 <= 16 MiB, with P*N*10 + 512 more bytes for
+ *   TP_SCORE_AUC (its sort keys and labels); e.g. N = 100000 rows of 10
+ *   classes with P = 96 candidates, or ROC-AUC on N = 20000 rows with P = 80.
+ *   Larger problems return TP_EINVAL with the exact need in the message of
+ *   pack_last_error(NULL) and do nothing.
+ *   The first call on each device (and the first after a device reset)
+ *   looks up the array's device address (cudaGetSymbolAddress, with that
+ *   device current); make that first call before any stream capture.
+ *   selected receives the *n_selected selected slots only.
  *   All calls share the one array and each call starts by clearing what it
  *   needs, so calls that overlap on the GPU (concurrent streams) race and
  *   must be serialised by the caller.                                        */
@@ -322,6 +325,20 @@ tp_status pack_debug_activations(tabpack_t* pack, int32_t member, int32_t layer,
  * whose epilogue evaluates the keep bits itself.  Synchronises.            */
 tp_status pack_debug_mask_arena(tabpack_t* pack, int32_t member, int32_t layer, int32_t B, uint8_t* keep,
                                 int64_t* step_held);
+
+/* Failure detection of the tensor-core products, for tests (the paper has
+ * no counterpart).  Every wait of the persistent GEMM launches that can give
+ * up (copy stages, accumulators, row-block dependencies) gives up after
+ * wait_s seconds (default 2): the CTA raises its abort flag, records the
+ * wait's site code in the pack's device error word, lets its own copies and
+ * MMAs finish, frees its tensor memory and exits, and the next
+ * synchronising call returns TP_ETIMEOUT naming the site (3: a row-block
+ * dependency).  poison != 0 also makes the first forward tile that waits
+ * on a dependency wait for a count the launch never reaches, so the next
+ * bf16 step's forward launch gives up there; the pack's results are then
+ * undefined and it should be destroyed.  bf16 mode; synchronises; captured
+ * step graphs are dropped.                                                 */
+tp_status pack_debug_gemm_timeout(tabpack_t* pack, double wait_s, int32_t poison);
 
 /* Philox4x32-10 (Salmon et al., SC'11) as the device evaluates it for the
  * dropout masks and the initial values: out[i] = the four words of counter

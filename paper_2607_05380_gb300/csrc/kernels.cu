@@ -622,7 +622,8 @@ __device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)
 template <int DO>
 __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
   constexpr int DOP = DO == 1 ? 1 : (DO + 3) & ~3;
-  pdl_trigger();
+  // no early trigger: the next kernels' CTAs (the backward GEMM's hold most
+  // of an SM's shared memory) must not park beside these blocks
   pdl_wait();
   const HeadJob jb = g.jobs[blockIdx.x];
   const int r0 = jb.blk * kHeadRows;
@@ -837,6 +838,7 @@ __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
       part[e] = v;
     }
   }
+  pdl_trigger();
   // bias partial and loss partial of the block (rows in order)
   if (threadIdx.x < d_out) {
     float v = 0.f;

@@ -27,9 +27,34 @@ static __device__ __align__(256) unsigned char g_select_scratch[kStaticScratchBy
 
 // Device address of g_select_scratch per device.  In host code the symbol
 // names a host-side stand-in, never the device array, so the address is
-// looked up once per device (with that device current) and cached.
-static void* g_scratch_addr[kMaxDevices] = {nullptr};
+// looked up with the device current and cached.  The cache entry remembers
+// the context it was taken in: after a device reset (or the primary context
+// being released and created again) the module is loaded anew, the context
+// handle changes and the address is looked up again.
+typedef int (*PFN_ctxGetCurrent)(void**);   // CUresult cuCtxGetCurrent(CUcontext*)
+
+struct ScratchAddr {
+  void* ctx = nullptr;
+  void* addr = nullptr;
+};
+static ScratchAddr g_scratch_addr[kMaxDevices];
 static std::mutex g_scratch_mu;
+
+static void* current_context() {
+  static PFN_ctxGetCurrent fn = nullptr;
+  static bool looked = false;
+  if (!looked) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = (PFN_ctxGetCurrent)p;
+    looked = true;
+  }
+  void* ctx = nullptr;
+  if (fn == nullptr || fn(&ctx) != 0) return nullptr;
+  return ctx;
+}
 
 static cudaError_t scratch_address(void** out) {
   int dev = 0;
@@ -37,13 +62,16 @@ static cudaError_t scratch_address(void** out) {
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
   std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (g_scratch_addr[dev] == nullptr) {
+  void* ctx = current_context();
+  ScratchAddr& c = g_scratch_addr[dev];
+  if (c.addr == nullptr || ctx == nullptr || c.ctx != ctx) {
     void* p = nullptr;
     e = cudaGetSymbolAddress(&p, g_select_scratch);
     if (e != cudaSuccess) return e;
-    g_scratch_addr[dev] = p;
+    c.addr = p;
+    c.ctx = ctx;
   }
-  *out = g_scratch_addr[dev];
+  *out = c.addr;
   return cudaSuccess;
 }
 
@@ -79,10 +107,10 @@ tp_status pack_select_greedy_static(const float* preds, int32_t P, int64_t N, in
   if (P > 65535) return static_fail(TP_EINVAL, "P > 65535");
   const int64_t need = select_scratch_bytes(P, N, d_out, m_ens, score);
   if (need > kStaticScratchBytes) {
-    char buf[256];
+    char buf[320];
     snprintf(buf, sizeof buf,
              "problem needs %lld bytes of scratch, the static array holds %lld (N * d_out * 8 + P * ceil(N/1024) * 8 "
-             "+ (4 + m_ens + P) * 4 + 768 must fit)",
+             "+ (4 + m_ens + P) * 4 + 1024, plus P * N * 10 + 512 for the ROC-AUC score, must fit)",
              (long long)need, (long long)kStaticScratchBytes);
     return static_fail(TP_EINVAL, buf);
   }
@@ -98,11 +126,15 @@ tp_status pack_select_greedy_static(const float* preds, int32_t P, int64_t N, in
   double cur = 0.0;
   e = cudaGetLastError();
   if (e == cudaSuccess) e = cudaMemcpyAsync(hdr, s.state, sizeof hdr, cudaMemcpyDeviceToHost, st);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(selected, s.state + 4, sizeof(int32_t) * m_ens, cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess) e = cudaMemcpyAsync(&cur, s.cur, sizeof(double), cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  // only the n selected slots reach the caller, as with pack_select_greedy
+  const int32_t n = hdr[0] < 0 ? 0 : (hdr[0] > m_ens ? m_ens : hdr[0]);
+  if (e == cudaSuccess && n > 0)
+    e = cudaMemcpyAsync(selected, s.state + 4, sizeof(int32_t) * n, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess && n > 0) e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return static_fail(TP_ECUDA, "select (static scratch)", e);
-  *n_selected = hdr[0];
+  *n_selected = n;
   if (final_score) *final_score = cur;
   return TP_OK;
 }

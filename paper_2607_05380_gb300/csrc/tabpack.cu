@@ -1783,6 +1783,22 @@ tp_status pack_debug_mask_arena(tabpack_t* h, int32_t member, int32_t layer, int
   return TP_OK;
 }
 
+tp_status pack_debug_gemm_timeout(tabpack_t* h, double wait_s, int32_t poison) {
+  if (!h) return fail(nullptr, TP_EINVAL, "null pack");
+  if (!h->bf16 || !h->tc.enabled) return fail(h, TP_ESTATE, "the tensor-core plan runs in bf16 mode only");
+  if (!(wait_s > 0.0) || wait_s > 60.0) return fail(h, TP_EINVAL, "wait budget must be in (0, 60] s");
+  TP_CUDA(h, cudaStreamSynchronize(h->st));
+  const uint64_t ns = (uint64_t)(wait_s * 1e9);
+  h->tc.wait_ns = ns;
+  h->tcs.wait_ns = ns;
+  h->tcp.wait_ns = ns;
+  // captured graphs hold the old launch arguments
+  for (auto& e : h->graphs) cudaGraphExecDestroy(e.exec);
+  h->graphs.clear();
+  if (poison) TP_TRY(tc_debug_poison(h->tc, h->st, h->err));
+  return TP_OK;
+}
+
 tp_status pack_debug_philox(const uint32_t* ctr, const uint32_t* key, int32_t n, uint32_t* out) {
   if (n < 1 || !ctr || !key || !out) return fail(nullptr, TP_EINVAL, "bad n or null pointer");
   std::vector<uint32_t> in((size_t)n * 6);

@@ -119,6 +119,7 @@ struct TcArgs {
   int* cnt;            // row-block completion counters
   int32_t kmaj_off;    // index distance to the same matrix's map with 128-row boxes (K-major loads)
   __nv_bfloat16* ns;   // Newton-Schulz arena (kNs launches)
+  uint64_t wait_ns;    // budget of every wait that can give up (TcPlan::wait_ns)
 };
 
 // ------------------------------------------------------------ PTX helpers
@@ -189,13 +190,14 @@ __device__ __forceinline__ void fence_proxy_async_global() {
 }
 
 // Bounded wait until counters p[0 .. n-1] each reach `need`.
-__device__ __noinline__ bool dep_wait(const int* p, int n, int need, volatile int* abort_flag, int* err, int site) {
+__device__ __noinline__ bool dep_wait(const int* p, int n, int need, volatile int* abort_flag, int* err,
+                                      uint64_t budget_ns, int site) {
   for (int j = 0; j < n; ++j) {
     if (ld_acquire(p + j) >= need) continue;
     const uint64_t t0 = global_ns();
     while (ld_acquire(p + j) < need) {
       if (*abort_flag) return false;
-      if (global_ns() - t0 > kWaitNs) {
+      if (global_ns() - t0 > budget_ns) {
         *abort_flag = 1;
         atomicCAS(err, 0, site);
         return false;
@@ -469,7 +471,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       bool dep_ok = true;
       if (lane == 0 && u.rows_live && tile.dep >= 0)
         dep_ok = dep_wait(g.cnt + tile.dep + (tile.dep_n ? rank : 0), tile.dep_n ? tile.dep_n : g.B_pad / kRowTile,
-                          tile.dep_need, abort_flag, g.err, 3);
+                          tile.dep_need, abort_flag, g.err, g.wait_ns, 3);
       if (!__shfl_sync(0xffffffffu, dep_ok, 0)) {
         ok = false;
         break;
@@ -478,7 +480,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       for (int k0 = 0; k0 < K; k0 += 64) {
         bool got = true;
         if (lane == 0) {
-          got = mbar_wait(&tl->empty[stage], phase ^ 1u, abort_flag, g.err, kWaitNs, 1);
+          got = mbar_wait(&tl->empty[stage], phase ^ 1u, abort_flag, g.err, g.wait_ns, 1);
           if (got && leader) mbar_expect_tx(&tl->full[stage], bytes);
         }
         if (!__shfl_sync(0xffffffffu, got, 0)) {
@@ -526,7 +528,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         const TcTile tile = g.tiles[t];
         if (!tile_live(tile, g.B_pad)) continue;
         const int K = tile.k_len ? tile.k_len : g.B_pad;
-        if (!mbar_wait(&tl->tempty[acc], acc_phase ^ 1u, abort_flag, g.err, kWaitNs, 5)) break;
+        if (!mbar_wait(&tl->tempty[acc], acc_phase ^ 1u, abort_flag, g.err, g.wait_ns, 5)) break;
         tc_fence_after();
         const uint32_t d = tmem + acc * kAccCols;
         const int a_mn = tile.kind == kWgrad, b_mn = !b_kmajor(tile.kind);
@@ -535,7 +537,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         const uint32_t ka = a_mn ? 2048 >> 4 : 32 >> 4, kb = b_mn ? 2048 >> 4 : 32 >> 4;
         uint32_t accum = 0;
         for (int k0 = 0; k0 < K; k0 += 64) {
-          if (!mbar_wait(&tl->full[stage], phase, abort_flag, g.err, kWaitNs, 6)) {
+          if (!mbar_wait(&tl->full[stage], phase, abort_flag, g.err, g.wait_ns, 6)) {
             ok = false;
             break;
           }
@@ -628,7 +630,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           bits[ci] = mb;
         }
       }
-      if (!mbar_wait(&tl->tfull[acc], acc_phase, abort_flag, g.err, kWaitNs, 7)) break;
+      if (!mbar_wait(&tl->tfull[acc], acc_phase, abort_flag, g.err, g.wait_ns, 7)) break;
       tc_fence_after();
       const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + acc * kAccCols;
       float lr = 0.f, wd_w = 0.f, wd_b = 0.f, ib1 = 1.f, ib2 = 1.f;
@@ -1291,6 +1293,7 @@ static tp_status launch(TcPlan& plan, cudaStream_t st, const std::pair<int, int>
   a.err = plan.err_dev;
   a.cnt = plan.cnt_dev;
   a.kmaj_off = plan.kmaj_off;
+  a.wait_ns = plan.wait_ns;
   const int cta = plan.cta;
   // every CTA resident at once (the dataflow waits rely on it)
   const int n_clu = std::max(1, std::min(rng.second, plan.max_clusters));
@@ -1374,6 +1377,35 @@ tp_status tc_check(TcPlan& plan, cudaStream_t st, std::string& err) {
     return TP_ETIMEOUT;
   }
   return TP_OK;
+}
+
+tp_status tc_debug_poison(TcPlan& plan, cudaStream_t st, std::string& err) {
+  const int n = plan.fwd_rng.second;
+  if (!plan.tiles_dev || n <= 0) {
+    err = "no forward tiles to poison";
+    return TP_ESTATE;
+  }
+  std::vector<TcTile> t((size_t)n);
+  if (cudaStreamSynchronize(st) != cudaSuccess ||
+      cudaMemcpy(t.data(), plan.tiles_dev + plan.fwd_rng.first, sizeof(TcTile) * n, cudaMemcpyDeviceToHost) !=
+          cudaSuccess) {
+    err = "reading the tile list failed";
+    return TP_ECUDA;
+  }
+  for (int i = 0; i < n; ++i)
+    if (t[i].dep >= 0) {
+      // a count the launch never reaches: the producer of this tile waits
+      // before it issues any copy, gives up after wait_ns and aborts its CTA
+      t[i].dep_need = 1 << 30;
+      if (cudaMemcpy(plan.tiles_dev + plan.fwd_rng.first + i, &t[i], sizeof(TcTile), cudaMemcpyHostToDevice) !=
+          cudaSuccess) {
+        err = "writing the tile list failed";
+        return TP_ECUDA;
+      }
+      return TP_OK;
+    }
+  err = "no forward tile waits on a dependency (a pack of depth-1 members)";
+  return TP_ESTATE;
 }
 
 void tc_free_plan(TcPlan& plan) {

@@ -63,6 +63,7 @@ struct TcPlan {
   int cta = 1;             // CTAs per tile (2: CTA pairs with cta_group::2 MMAs)
   int max_clusters = 0;    // tiles in flight at once (resident CTAs / cta)
   int* err_dev = nullptr;  // device error word (bounded waits that gave up)
+  uint64_t wait_ns = 2000000000ull;  // budget of every wait that can give up
   std::vector<int> map_act, map_dz, map_w;  // per (member * kMaxDepth + layer)
   std::vector<int> map_ns;                  // per Muon matrix: X0, X1, A, Bm
 };
@@ -113,6 +114,9 @@ tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, 
 tp_status tc_run_ns(TcPlan& plan, cudaStream_t st, int which, void* ns, const MemberDev* mem, std::string& err);
 // Reads and clears the device error word (synchronises the stream).
 tp_status tc_check(TcPlan& plan, cudaStream_t st, std::string& err);
+// Tests: the first forward tile with a dependency waits for a count the
+// launch never reaches (then its CTA gives up after plan.wait_ns).
+tp_status tc_debug_poison(TcPlan& plan, cudaStream_t st, std::string& err);
 void tc_free_plan(TcPlan& plan);
 
 }  // namespace tp
