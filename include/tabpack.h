@@ -328,8 +328,9 @@ tp_status pack_debug_mask_arena(tabpack_t* pack, int32_t member, int32_t layer, 
 
 /* Failure detection of the tensor-core products, for tests (the paper has
  * no counterpart).  Every wait of the persistent GEMM launches that can give
- * up (copy stages, accumulators, row-block dependencies) gives up after
- * wait_s seconds (default 2): the CTA raises its abort flag, records the
+ * up gives up after wait_s seconds (default 2) -- the producer's waits for a
+ * free stage or a row-block dependency -- or 2 wait_s -- the MMA and
+ * epilogue waits, which wait on the producer: the CTA raises its abort flag, records the
  * wait's site code in the pack's device error word, lets its own copies and
  * MMAs finish, frees its tensor memory and exits, and the next
  * synchronising call returns TP_ETIMEOUT naming the site (3: a row-block

@@ -604,9 +604,9 @@ __device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)
 
 // ----------------------------------------------- head + loss, staged (bf16)
 // The same work as k_head for one member on one 64-row block in bf16 mode,
-// with the block's H_L rows staged in shared memory by bulk copies (one per
-// row) so that H is read from HBM once and both passes run from shared
-// memory:
+// with the block's H_L rows (one bulk copy per row) and the head weights (one
+// bulk copy) staged in shared memory, so that H is read from HBM once and
+// both passes run from shared memory:
 //   1. logits: warp v takes the 8-column groups v, v + 8, ... and lane l rows
 //      l and l + 32 (16-byte loads; the row pitch is 16 bytes past a
 //      multiple of 128, so the eight rows of a quarter-warp fall in distinct
@@ -617,8 +617,8 @@ __device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)
 //      its rows: dZ = (dlogits W_h) [H > 0] / (1 - p) stored in bf16, dW_h
 //      partials in registers; row sets (narrow members) are added in order
 //      through shared memory.
-// Shared memory: H [64][pitch] | partial logits [8][64][DO] | dlogits
-// [64][DOP] | row losses [64] | mbarrier.
+// Shared memory: H [64][pitch] | W_h [DO][w] | partial logits [8][DO][64] |
+// dlogits [64][DOP] | row losses [64] | mbarrier.
 template <int DO>
 __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
   constexpr int DOP = DO == 1 ? 1 : (DO + 3) & ~3;
@@ -633,17 +633,19 @@ __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
   const int pitch = head_stage_pitch(w);
   extern __shared__ __align__(128) unsigned char smem[];
   unsigned char* Hs = smem;
-  float* zpart = reinterpret_cast<float*>(smem + (int64_t)kHeadRows * pitch);   // [8][64][DO]
+  float* Ws = reinterpret_cast<float*>(smem + (int64_t)kHeadRows * pitch);      // [d_out][w]
+  float* zpart = Ws + (int64_t)DO * w;                                          // [8][DO][64]
   float* dlog = zpart + kStageWarps * kHeadRows * DO;                          // [64][DOP]
   float* lrow = dlog + kHeadRows * DOP;                                         // [64]
   uint64_t* bar = reinterpret_cast<uint64_t*>(lrow + kHeadRows + 2);            // 8-byte aligned
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const __nv_bfloat16* __restrict__ H = g.act + jb.h_off + (int64_t)r0 * ldh;
-  const float* __restrict__ Wh = g.params + jb.w_off;
+  const float* __restrict__ Wg = g.params + jb.w_off;
   const float* __restrict__ bh = g.params + jb.b_off;
   const uint32_t row_bytes = (uint32_t)w * 2u;
+  const uint32_t w_bytes = (uint32_t)(d_out * w) * 4u;
 
-  // stage the 64 rows (warp 0 issues one bulk copy per row)
+  // stage the 64 rows and the head weights (warp 0 issues the bulk copies)
   if (threadIdx.x == 0) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_addr(bar)) : "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -653,8 +655,13 @@ __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
     if (lane == 0) {
       asm volatile("fence.proxy.async.global;" ::: "memory");
       asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
-                   "r"(row_bytes * (uint32_t)kHeadRows)
+                   "r"(row_bytes * (uint32_t)kHeadRows + w_bytes)
                    : "memory");
+      asm volatile(
+          "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+              smem_addr(Ws)),
+          "l"(Wg), "r"(w_bytes), "r"(smem_addr(bar))
+          : "memory");
     }
     __syncwarp();
     for (int r = lane; r < kHeadRows; r += 32)
@@ -693,6 +700,7 @@ __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
 #pragma unroll
       for (int c = 0; c < DO; ++c) acc[q][c] = 0.f;
     const int ng = w >> 3;
+#pragma unroll 2
     for (int gi = warp; gi < ng; gi += kStageWarps) {
       float h[2][8];
 #pragma unroll
@@ -705,8 +713,8 @@ __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
 #pragma unroll
       for (int c = 0; c < DO; ++c) {
         if (c < d_out) {
-          const float4 wa = __ldg(reinterpret_cast<const float4*>(Wh + (int64_t)c * w + 8 * gi));
-          const float4 wb = __ldg(reinterpret_cast<const float4*>(Wh + (int64_t)c * w + 8 * gi + 4));
+          const float4 wa = *reinterpret_cast<const float4*>(Ws + c * w + 8 * gi);
+          const float4 wb = *reinterpret_cast<const float4*>(Ws + c * w + 8 * gi + 4);
           const float w8[8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
 #pragma unroll
           for (int q = 0; q < 2; ++q)
@@ -718,7 +726,7 @@ __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
 #pragma unroll
     for (int q = 0; q < 2; ++q)
 #pragma unroll
-      for (int c = 0; c < DO; ++c) zpart[(warp * kHeadRows + lane + 32 * q) * DO + c] = acc[q][c];
+      for (int c = 0; c < DO; ++c) zpart[(warp * DO + c) * kHeadRows + lane + 32 * q] = acc[q][c];
   }
   __syncthreads();
   if (threadIdx.x < kHeadRows) {
@@ -727,7 +735,7 @@ __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
 #pragma unroll
     for (int c = 0; c < DO; ++c) {
       float v = 0.f;
-      for (int v8 = 0; v8 < kStageWarps; ++v8) v += zpart[(v8 * kHeadRows + rl) * DO + c];
+      for (int v8 = 0; v8 < kStageWarps; ++v8) v += zpart[(v8 * DO + c) * kHeadRows + rl];
       z[c] = c < d_out ? v + bh[c] : 0.f;
     }
     float dl[DO];
@@ -766,7 +774,7 @@ __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
 #pragma unroll
     for (int c = 0; c < DO; ++c) {
       if (c < d_out) {
-        const float4 v = __ldg(reinterpret_cast<const float4*>(Wh + (int64_t)c * w + col));
+        const float4 v = *reinterpret_cast<const float4*>(Ws + c * w + col);
         Wr[c][0] = v.x;
         Wr[c][1] = v.y;
         Wr[c][2] = v.z;

@@ -75,7 +75,8 @@ __host__ __device__ constexpr int head_stage_split(int w, int DO) {
 }
 __host__ __device__ constexpr int64_t head_stage_smem(int w_max, int DO) {
   return (int64_t)kHeadRows * head_stage_pitch(w_max) +
-         4 * ((int64_t)8 * kHeadRows * DO + (int64_t)kHeadRows * (DO == 1 ? 1 : (DO + 3) & ~3) + kHeadRows) + 16;
+         4 * ((int64_t)DO * w_max + (int64_t)8 * kHeadRows * DO + (int64_t)kHeadRows * (DO == 1 ? 1 : (DO + 3) & ~3) +
+              kHeadRows) + 16;
 }
 void head_stage_prepare();
 

@@ -154,7 +154,9 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // A wait that gives up records its site code in the error word (the first
 // one wins): 1 producer stage empty, 3 producer dependency, 5 MMA
 // accumulator free, 6 MMA stage full, 7 epilogue accumulator full, 10 final
-// copy drain, 12 final MMA drain.
+// copy drain, 12 final MMA drain.  The MMA and epilogue waits (5, 6, 7)
+// wait on another role of the same CTA and take twice the budget of the
+// producer's, so a stalled dependency is reported as its own site.
 __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* err,
                                             uint64_t budget_ns, int site) {
   if (mbar_try_wait(bar, parity)) return true;
@@ -528,7 +530,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         const TcTile tile = g.tiles[t];
         if (!tile_live(tile, g.B_pad)) continue;
         const int K = tile.k_len ? tile.k_len : g.B_pad;
-        if (!mbar_wait(&tl->tempty[acc], acc_phase ^ 1u, abort_flag, g.err, g.wait_ns, 5)) break;
+        if (!mbar_wait(&tl->tempty[acc], acc_phase ^ 1u, abort_flag, g.err, 2 * g.wait_ns, 5)) break;
         tc_fence_after();
         const uint32_t d = tmem + acc * kAccCols;
         const int a_mn = tile.kind == kWgrad, b_mn = !b_kmajor(tile.kind);
@@ -537,7 +539,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         const uint32_t ka = a_mn ? 2048 >> 4 : 32 >> 4, kb = b_mn ? 2048 >> 4 : 32 >> 4;
         uint32_t accum = 0;
         for (int k0 = 0; k0 < K; k0 += 64) {
-          if (!mbar_wait(&tl->full[stage], phase, abort_flag, g.err, g.wait_ns, 6)) {
+          if (!mbar_wait(&tl->full[stage], phase, abort_flag, g.err, 2 * g.wait_ns, 6)) {
             ok = false;
             break;
           }
@@ -630,7 +632,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           bits[ci] = mb;
         }
       }
-      if (!mbar_wait(&tl->tfull[acc], acc_phase, abort_flag, g.err, g.wait_ns, 7)) break;
+      if (!mbar_wait(&tl->tfull[acc], acc_phase, abort_flag, g.err, 2 * g.wait_ns, 7)) break;
       tc_fence_after();
       const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + acc * kAccCols;
       float lr = 0.f, wd_w = 0.f, wd_b = 0.f, ib1 = 1.f, ib2 = 1.f;
