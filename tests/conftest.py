@@ -17,3 +17,16 @@ def orc():
     import oracle
     oracle.build()
     return oracle
+
+
+def pytest_terminal_summary(terminalreporter, exitstatus, config):
+    """The bf16-mode distances the parity tests measured: per tensor kind,
+    the largest entrywise error of the GPU against the exact oracle and of
+    the oracle's own bf16-storage model against its exact mode."""
+    mod = sys.modules.get("parity")
+    stats = getattr(mod, "STATS", None) if mod else None
+    if not stats:
+        return
+    terminalreporter.section("bf16 mode against the exact oracle (largest entrywise relative error)")
+    for kind, (e_gpu, e_model) in sorted(stats.items()):
+        terminalreporter.write_line(f"{kind:14s} GPU {e_gpu:.3g}   oracle bf16-storage model {e_model:.3g}")
