@@ -33,12 +33,12 @@ from workloads import SEED_HP, SEED_INIT, WORKLOADS, make_data, sample_emb, samp
 METRIC = "member-samples/sec (fwd+bwd+AdamW)"
 
 # DRAM bytes (read + write) per step of the dominant kernels, from ncu captures of
-# the current kernels (summaries in profiles/; the wide figure is scaled from its
-# first 8 members by GEMM flops).  A workload without a capture reports null.
+# the current kernels (summaries in profiles/; the wide GEMM figure is the capture
+# of its first 4 members scaled to 16 by GEMM flops).  A workload without a capture
+# of the current kernel reports null.
 DRAM_TRAFFIC = {
-    ("medium", "k_tc_gemm"): 252.0e6,
     ("medium", "k_adamw"): 607.7e6,
-    ("wide", "k_tc_gemm"): 3.589e9,
+    ("wide", "k_tc_gemm"): 3.101e9,
 }
 UNIT = "member-samples/s"
 
