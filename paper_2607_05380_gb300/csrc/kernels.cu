@@ -926,8 +926,6 @@ __global__ void k_head_reduce(HeadReduceArgs g) {
 __global__ void __launch_bounds__(256) k_adamw(AdamArgs g) {
   pdl_trigger();
   pdl_wait();
-  // the next step's dropout masks: ALU work beside this pass's HBM streaming
-  fill_masks(g.mg, (int64_t)blockIdx.x * blockDim.x + threadIdx.x, (int64_t)gridDim.x * blockDim.x);
   const Chunk ch = g.chunks[blockIdx.x];
   const Segment s = g.segs[ch.seg];
   const MemberDev md = g.mem[s.member];
@@ -968,6 +966,10 @@ __global__ void __launch_bounds__(256) k_adamw(AdamArgs g) {
     g.v[o] = v;
     if (g.wq) g.wq[o] = __float2bfloat16_rn(p);
   }
+  // the next step's dropout masks: ALU work that other blocks' HBM streaming
+  // overlaps (after this block's own stores have left, so that it does not
+  // delay them)
+  fill_masks(g.mg, (int64_t)blockIdx.x * blockDim.x + threadIdx.x, (int64_t)gridDim.x * blockDim.x);
 }
 
 // ------------------------------------------------------------------- init
@@ -1143,7 +1145,9 @@ template <typename T>
 void launch_head(cudaStream_t st, const HeadArgs<T>& g, int n_jobs) {
   if (n_jobs <= 0) return;
   if constexpr (std::is_same_v<T, __nv_bfloat16>) {
-    if (g.stage) {
+    // one output on members wider than 512: the row-per-lane-group kernel
+    // measured faster (the staged block then runs one per SM)
+    if (g.stage && !(g.d_out == 1 && g.w_max > 512)) {
       bool done = false;
       switch (head_bucket(g.d_out)) {
         case 1: done = launch_head_stage<1>(st, g, n_jobs); break;
