@@ -317,6 +317,32 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
   return *reinterpret_cast<uint32_t*>(&t);
 }
 
+// One chunk of an epilogue warp's bf16 output -- its 32 rows (lane = row)
+// by 32 columns -- written as row segments: each lane puts its row's four
+// 16-byte groups into the warp's transpose buffer (XOR-swizzled by row, so
+// that both the row-wise write and the segment-wise read are free of bank
+// conflicts; stage_group), and flush_chunk reads them back four lanes per row,
+// so that every store instruction writes eight whole 64-byte row segments
+// instead of 32 half sectors of 32 different rows.
+__device__ __forceinline__ void stage_group(uint8_t* buf, int lane, int s, uint32_t a, uint32_t b, uint32_t c,
+                                            uint32_t d) {
+  *reinterpret_cast<uint4*>(buf + lane * 64 + 16 * (s ^ ((lane >> 1) & 3))) = make_uint4(a, b, c, d);
+}
+// out: the warp's first row at the chunk's first column; rows from rbase on
+// are valid below m_lim, columns below ncols.
+__device__ __forceinline__ void flush_chunk(uint8_t* buf, int lane, __nv_bfloat16* out, int64_t ldc, int rbase,
+                                            int m_lim, int ncols) {
+  __syncwarp();
+  const int seg = lane & 3;
+#pragma unroll 1
+  for (int j = 0; j < 4; ++j) {
+    const int rl = 8 * j + (lane >> 2);
+    const uint4 val = *reinterpret_cast<const uint4*>(buf + rl * 64 + 16 * (seg ^ ((rl >> 1) & 3)));
+    if (rbase + rl < m_lim && 8 * seg < ncols) *reinterpret_cast<uint4*>(out + (int64_t)rl * ldc + 8 * seg) = val;
+  }
+  __syncwarp();  // the buffer is reused by the next chunk
+}
+
 // a[i] for a runtime i < N (N = 4 or 8) without indexing (keeps a[] in registers)
 template <typename V, int N>
 __device__ __forceinline__ V pick(const V (&a)[N], int i) {
@@ -768,50 +794,49 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           continue;
         }
         if (tile.kind == kFwd) {  // ncols: a multiple of 8 (widths are multiples of 16)
-          float bias[32];
           const float bl = pick(bias_l, ci);
-#pragma unroll
-          for (int j = 0; j < 32; ++j) bias[j] = __shfl_sync(0xffffffffu, bl, j);
-          if (!live) continue;
+          if (ncols <= 0) continue;   // warp-uniform: every lane takes part in the store below
           const uint32_t keep = pick(bits, ci);
           const float sc = g.train ? md.scale : 1.f;
-          __nv_bfloat16* out = g.act + tile.c_off + (int64_t)r * tile.ldc + col0;
+          uint8_t* buf = reinterpret_cast<uint8_t*>(tr_all + (warp - 2) * 32 * 32);
 #pragma unroll
-          for (int s = 0; s < 4; ++s) {
-            if (8 * s >= ncols) break;
+          for (int sg = 0; sg < 4; ++sg) {
             uint32_t pk[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
               float h2[2];
 #pragma unroll
-              for (int u = 0; u < 2; ++u) {
-                const int j = 8 * s + 2 * e + u;
-                const float z = __uint_as_float(v[j]) + bias[j];
+              for (int u2 = 0; u2 < 2; ++u2) {
+                const int j = 8 * sg + 2 * e + u2;
+                const float z = __uint_as_float(v[j]) + __shfl_sync(0xffffffffu, bl, j);
                 const float a = z > 0.f ? z : 0.f;
-                h2[u] = ((keep >> j) & 1u) ? a * sc : 0.f;
+                h2[u2] = ((keep >> j) & 1u) ? a * sc : 0.f;
               }
               pk[e] = pack_bf16x2(h2[0], h2[1]);
             }
-            *reinterpret_cast<uint4*>(out + 8 * s) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            stage_group(buf, lane, sg, pk[0], pk[1], pk[2], pk[3]);
           }
+          const int rbase = u.m0 + 32 * q;
+          flush_chunk(buf, lane, g.act + tile.c_off + (int64_t)rbase * tile.ldc + col0, tile.ldc, rbase, m_lim, ncols);
         } else if (tile.kind == kDgrad) {
-          if (!live) continue;
+          if (ncols <= 0) continue;
           const uint32_t mb = pick(bits, ci);
           const float dsc = tile.aux_off >= 0 ? md.scale : 1.f;   // the first layer's input gradient: 1
-          __nv_bfloat16* out = g.dz + tile.c_off + (int64_t)r * tile.ldc + col0;
+          uint8_t* buf = reinterpret_cast<uint8_t*>(tr_all + (warp - 2) * 32 * 32);
 #pragma unroll
-          for (int s = 0; s < 4; ++s) {
-            if (8 * s >= ncols) break;
+          for (int sg = 0; sg < 4; ++sg) {
             uint32_t pk[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
-              const int j = 8 * s + 2 * e;
+              const int j = 8 * sg + 2 * e;
               const float x0 = ((mb >> j) & 1u) ? __uint_as_float(v[j]) * dsc : 0.f;
               const float x1 = ((mb >> (j + 1)) & 1u) ? __uint_as_float(v[j + 1]) * dsc : 0.f;
               pk[e] = pack_bf16x2(x0, x1);
             }
-            *reinterpret_cast<uint4*>(out + 8 * s) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            stage_group(buf, lane, sg, pk[0], pk[1], pk[2], pk[3]);
           }
+          const int rbase = u.m0 + 32 * q;
+          flush_chunk(buf, lane, g.dz + tile.c_off + (int64_t)rbase * tile.ldc + col0, tile.ldc, rbase, m_lim, ncols);
         }
       }
       // this warp has read its part of the accumulator: release it to the
@@ -826,9 +851,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       if (acc == 0) acc_phase ^= 1u;
       if (tile.sig >= 0 && u.rows_live) {  // publish this warp's part of the tile
         __syncwarp();
+        // the release of lane 0 after the warp barrier orders every lane's
+        // stores before the count (release is cumulative); the proxy fence
+        // serves the readers' tensor-map loads
         if (lane == 0) {
           fence_proxy_async_global();
-          __threadfence();
           red_release_add(g.cnt + tile.sig + rank, 1);
         }
       }
