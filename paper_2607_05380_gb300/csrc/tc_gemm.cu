@@ -18,6 +18,9 @@
 //   warp 1     MMA issuer: one thread issues tcgen05.mma (M=128, K=16 per
 //              instruction) into one of two TMEM accumulators (2 x 256
 //              fp32 columns) and commits each stage back to the producer.
+//   warp 10    publisher: per stored tile, the release count that tiles in
+//              other CTAs wait on (so that the epilogue warps do not wait for
+//              their stores to drain before starting the next tile)
 //   warps 2-9  epilogue: tcgen05.ld of the accumulator (warp w reads TMEM
 //              lanes 32 (w % 4) .. +31, i.e. those output rows; the two
 //              warps of a lane quarter take alternate 32-column chunks) and
@@ -63,7 +66,9 @@ constexpr int kEpiWarps = TP_EPI_WARPS;
 static_assert(kEpiWarps == 4 || kEpiWarps == 8, "one or two epilogue warps per TMEM lane quarter");
 constexpr int kEpiPerQ = kEpiWarps / 4;         // epilogue warps per lane quarter
 constexpr int kChunks = 8 / kEpiPerQ;           // 32-column chunks per warp of a 256-column tile
-constexpr int kThreads = 64 + 32 * kEpiWarps;   // producer warp, MMA warp, epilogue warps
+constexpr int kThreads = 96 + 32 * kEpiWarps;   // producer warp, MMA warp, epilogue warps, publisher warp
+constexpr int kPubWarp = 2 + kEpiWarps;
+constexpr int kPubSlots = 4;                    // tiles in flight between the epilogue and the publisher
 constexpr uint32_t kTmemCols = 512;
 constexpr int kAccCols = 256;
 constexpr uint64_t kWaitNs = 2000000000ull;
@@ -88,6 +93,8 @@ struct SmemTail {
   uint64_t empty[kStages];
   uint64_t tfull[2];
   uint64_t tempty[2];
+  uint64_t stored[kPubSlots];    // the epilogue warps have stored a tile (one arrival each)
+  uint64_t pub_free[kPubSlots];  // the publisher has counted it
   uint64_t done;
   uint32_t tmem_base;
   int abort;
@@ -154,9 +161,10 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // A wait that gives up records its site code in the error word (the first
 // one wins): 1 producer stage empty, 3 producer dependency, 5 MMA
 // accumulator free, 6 MMA stage full, 7 epilogue accumulator full, 10 final
-// copy drain, 12 final MMA drain.  The MMA and epilogue waits (5, 6, 7)
-// wait on another role of the same CTA and take twice the budget of the
-// producer's, so a stalled dependency is reported as its own site.
+// copy drain, 12 final MMA drain, 8 epilogue publish slot, 9 publisher.
+// The MMA and epilogue waits (5, 6, 7, 8) wait on another role of the same
+// CTA and take twice the budget of the producer's, the publisher's (9) four
+// times, so a stalled dependency is reported as its own site.
 __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* err,
                                             uint64_t budget_ns, int site) {
   if (mbar_try_wait(bar, parity)) return true;
@@ -427,6 +435,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       mbar_init(&tl->tfull[b], 1);
       mbar_init(&tl->tempty[b], kEpiWarps * kCta);  // one arrival per epilogue warp of the pair
     }
+    for (int b = 0; b < kPubSlots; ++b) {
+      mbar_init(&tl->stored[b], kEpiWarps);
+      mbar_init(&tl->pub_free[b], 1);
+    }
     mbar_init(&tl->done, 1);
     tl->abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -596,12 +608,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       int dummy_abort = 0;
       mbar_wait(&tl->done, 0, &dummy_abort, g.err, kWaitNs, 12);
     }
-  } else {
+  } else if (warp < kPubWarp) {
     // ------------------------------------------------------------ epilogue
     const int q = warp & 3;             // TMEM lane quarter this warp may access
     const int half = (warp - 2) >> 2;   // 0 for warps 2-5, 1 for warps 6-9
     const int row = 32 * q + lane;
     uint32_t acc = 0, acc_phase = 0;
+    int n_pub = 0;   // tiles handed to the publisher
     // Fused AdamW: the parameter rows of the CTA's next weight-gradient tile
     // stream into L2 while this tile's products run and its epilogue works.
     if (g.update && clu < g.n_tiles && g.tiles[clu].kind == kWgrad)
@@ -849,15 +862,42 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       }
       acc ^= 1u;
       if (acc == 0) acc_phase ^= 1u;
-      if (tile.sig >= 0 && u.rows_live) {  // publish this warp's part of the tile
+      if (tile.sig >= 0 && u.rows_live) {
+        // hand this warp's part of the tile to the publisher: the arrival
+        // (a release at CTA scope after the warp barrier) orders every
+        // lane's stores before the publisher's count.  A slot is reused
+        // once the publisher has counted its previous tile.
+        const int slot = n_pub % kPubSlots;
+        bool got = true;
+        if (n_pub >= kPubSlots && lane == 0)
+          got = mbar_wait(&tl->pub_free[slot], (uint32_t)((n_pub / kPubSlots) - 1) & 1u, abort_flag, g.err,
+                          2 * g.wait_ns, 8);
+        if (!__shfl_sync(0xffffffffu, got, 0)) break;
         __syncwarp();
-        // the release of lane 0 after the warp barrier orders every lane's
-        // stores before the count (release is cumulative); the proxy fence
-        // serves the readers' tensor-map loads
-        if (lane == 0) {
-          fence_proxy_async_global();
-          red_release_add(g.cnt + tile.sig + rank, 1);
-        }
+        if (lane == 0) mbar_arrive(&tl->stored[slot]);
+        ++n_pub;
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ publisher
+    // Per stored tile (the epilogue's order), once every epilogue warp has
+    // arrived: the count that other CTAs' tiles wait on.  The release is
+    // cumulative over the stores the arrivals ordered before it; the proxy
+    // fence serves the readers' tensor-map loads.
+    if (lane == 0) {
+      int n_pub = 0;
+      for (int t = clu; t < g.n_tiles; t += n_clu) {
+        const TcTile tile = g.tiles[t];
+        if (!tile_live(tile, g.B_pad)) continue;
+        const SubTile u = sub_tile(tile, rank, g.B_pad);
+        if (tile.sig < 0 || !u.rows_live) continue;
+        const int slot = n_pub % kPubSlots;
+        if (!mbar_wait(&tl->stored[slot], (uint32_t)(n_pub / kPubSlots) & 1u, abort_flag, g.err, 4 * g.wait_ns, 9))
+          break;
+        fence_proxy_async_global();
+        red_release_add(g.cnt + tile.sig + rank, kEpiWarps);
+        mbar_arrive(&tl->pub_free[slot]);
+        ++n_pub;
       }
     }
   }
