@@ -33,12 +33,13 @@ from workloads import SEED_HP, SEED_INIT, WORKLOADS, make_data, sample_emb, samp
 METRIC = "member-samples/sec (fwd+bwd+AdamW)"
 
 # DRAM bytes (read + write) per step of the dominant kernels, from ncu captures of
-# the current kernels (summaries in profiles/; the wide GEMM figure is the capture
-# of its first 4 members scaled to 16 by GEMM flops).  A workload without a capture
-# of the current kernel reports null.
+# the current kernels (summaries in profiles/; the wide figures are captures of its
+# first 4 members scaled to 16, the GEMM's by GEMM flops, AdamW's by parameters).
+# A workload without a capture of the current kernel reports null.
 DRAM_TRAFFIC = {
     ("medium", "k_adamw"): 607.7e6,
-    ("wide", "k_tc_gemm"): 3.101e9,
+    ("wide", "k_tc_gemm"): 3.155e9,
+    ("wide", "k_adamw"): 4.020e9,
 }
 UNIT = "member-samples/s"
 
