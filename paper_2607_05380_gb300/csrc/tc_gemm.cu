@@ -1257,12 +1257,14 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
   // tile per resident CTA (pair), taken from the two lists in proportion to
   // their lengths, every CTA alternates between tiles whose epilogue streams
   // parameters (fused AdamW) and tiles whose time goes to the tensor cores.
-  // Each tile still only waits for tiles earlier in the list.
+  // A level starts with a block of wgrad tiles, which wait for nothing,
+  // while the previous level's last dgrad rows finish.  Each tile still only
+  // waits for tiles earlier in the list.
   auto interleave = [&](const std::vector<TcTile>& a, const std::vector<TcTile>& b) {
     const size_t blk = (size_t)std::max(1, plan.max_clusters);
     size_t ia = 0, ib = 0;
     while (ia < a.size() || ib < b.size()) {
-      const bool take_a = ib >= b.size() || (ia < a.size() && ia * b.size() <= ib * a.size());
+      const bool take_a = ib >= b.size() || (ia < a.size() && ia * b.size() < ib * a.size());
       if (take_a) {
         const size_t e = std::min(a.size(), ia + blk);
         all.insert(all.end(), a.begin() + ia, a.begin() + e);
