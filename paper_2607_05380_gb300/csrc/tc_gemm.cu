@@ -199,24 +199,34 @@ __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
-// Bounded wait until counters p[0 .. n-1] each reach `need`.
+// Bounded wait, by the whole warp, until counters p[0 .. n-1] each reach
+// `need`.  Lane j polls counters j, j + 32, ...: a weight-gradient tile waits
+// on every row block of its operand (16 counters for 2048 rows), and one
+// lane reading them in turn paid 16 acquire round trips to L2 per tile even
+// when all were long complete.  The warp barrier orders every lane after all
+// lanes' acquires; the caller's proxy fence follows it.
 __device__ __noinline__ bool dep_wait(const int* p, int n, int need, volatile int* abort_flag, int* err,
-                                      uint64_t budget_ns, int site) {
-  for (int j = 0; j < n; ++j) {
+                                      uint64_t budget_ns, int site, int lane) {
+  bool mine = true;
+  for (int j = lane; mine && j < n; j += 32) {
     if (ld_acquire(p + j) >= need) continue;
     const uint64_t t0 = global_ns();
     while (ld_acquire(p + j) < need) {
-      if (*abort_flag) return false;
+      if (*abort_flag) {
+        mine = false;
+        break;
+      }
       if (global_ns() - t0 > budget_ns) {
         *abort_flag = 1;
         atomicCAS(err, 0, site);
-        return false;
+        mine = false;
+        break;
       }
       __nanosleep(32);
     }
   }
-  fence_proxy_async_global();
-  return true;
+  __syncwarp();
+  return __all_sync(0xffffffffu, mine);
 }
 
 // Bulk prefetch of `bytes` (a multiple of 16; 16-byte aligned address) into L2.
@@ -509,14 +519,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       const int xy0 = is_a ? u.m0 + 64 * bl : bn0 + (b_k ? 128 : 64) * qb;
       const uint32_t off = is_a ? (uint32_t)bl * kBoxBytes : (uint32_t)kABytes + (uint32_t)qb * boxB;
       bool dep_ok = true;
-      if (lane == 0 && u.rows_live && tile.dep >= 0)
+      if (u.rows_live && tile.dep >= 0)
         dep_ok = dep_wait(g.cnt + tile.dep + (tile.dep_n ? rank : 0), tile.dep_n ? tile.dep_n : g.B_pad / kRowTile,
-                          tile.dep_need, abort_flag, g.err, g.wait_ns, 3);
-      if (!__shfl_sync(0xffffffffu, dep_ok, 0)) {
+                          tile.dep_need, abort_flag, g.err, g.wait_ns, 3, lane);
+      if (!dep_ok) {
         ok = false;
         break;
       }
-      if (tile.dep >= 0) fence_proxy_async_global();  // every issuing lane, after lane 0's acquire
+      if (tile.dep >= 0) fence_proxy_async_global();  // every issuing lane, after the warp's acquires
       for (int k0 = 0; k0 < K; k0 += 64) {
         bool got = true;
         if (lane == 0) {
