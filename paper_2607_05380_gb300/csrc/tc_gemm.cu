@@ -259,6 +259,16 @@ __device__ __forceinline__ uint32_t mapa(uint32_t addr, uint32_t rank) {
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar) : "memory");
 }
+// Arrivals that order no memory accesses of the arriving thread.  A release
+// arrival waits until the thread's earlier global stores are performed at its
+// scope; the epilogue's accumulator hand-back follows tcgen05.wait::ld, which
+// has already completed every TMEM read it covers, so it needs no release.
+__device__ __forceinline__ void mbar_arrive_relaxed(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.relaxed.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster_relaxed(uint32_t bar) {
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar) : "memory");
+}
 __device__ __forceinline__ uint32_t cluster_rank() {
   uint32_t r;
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
@@ -650,8 +660,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       const int n_hi = min(tile.n_real, tile.n0 + tile.n_len);
       // Inputs that do not depend on the accumulator are prepared while the
       // tile's MMAs run: forward, this lane's bias value of each chunk
-      // (column = lane; broadcast by shuffles) and the 32 dropout keep bits of
-      // its row; dgrad, the 32 ReLU-mask bits of its row.
+      // (column = lane; later broadcast through shared memory) and the 32
+      // dropout keep bits of its row; dgrad, the 32 ReLU-mask bits of its row.
       float bias_l[kChunks];
       uint32_t bits[kChunks];
 #pragma unroll
@@ -822,8 +832,17 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           const uint32_t keep = pick(bits, ci);
           const float sc = g.train ? md.scale : 1.f;
           uint8_t* buf = reinterpret_cast<uint8_t*>(tr_all + (warp - 2) * 32 * 32);
+          // the chunk's 32 bias values sit past the 2 KB of staged rows and
+          // reach every lane as broadcast reads (8 shared loads instead of 32
+          // shuffles); the flush's closing warp barrier orders their reuse
+          float* bsm = reinterpret_cast<float*>(buf + 2048);
+          bsm[lane] = bl;
+          __syncwarp();
 #pragma unroll
           for (int sg = 0; sg < 4; ++sg) {
+            const float4 b0 = *reinterpret_cast<const float4*>(bsm + 8 * sg);
+            const float4 b1 = *reinterpret_cast<const float4*>(bsm + 8 * sg + 4);
+            const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
             uint32_t pk[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
@@ -831,7 +850,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
 #pragma unroll
               for (int u2 = 0; u2 < 2; ++u2) {
                 const int j = 8 * sg + 2 * e + u2;
-                const float z = __uint_as_float(v[j]) + __shfl_sync(0xffffffffu, bl, j);
+                const float z = __uint_as_float(v[j]) + bv[2 * e + u2];
                 const float a = z > 0.f ? z : 0.f;
                 h2[u2] = ((keep >> j) & 1u) ? a * sc : 0.f;
               }
@@ -867,8 +886,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
-        if constexpr (kCta == 2) mbar_arrive_cluster(mapa(smem_u32(&tl->tempty[acc]), 0));
-        else mbar_arrive(&tl->tempty[acc]);
+        if constexpr (kCta == 2) mbar_arrive_cluster_relaxed(mapa(smem_u32(&tl->tempty[acc]), 0));
+        else mbar_arrive_relaxed(&tl->tempty[acc]);
       }
       acc ^= 1u;
       if (acc == 0) acc_phase ^= 1u;
