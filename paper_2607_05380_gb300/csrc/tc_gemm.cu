@@ -714,32 +714,86 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         tmem_ld32(taddr + c, v);
         if constexpr (kNs) {
           // Newton-Schulz: out = alpha acc + beta aux, bf16 (kNsGram: A;
-          // kNsPoly: Bm = c (A A) + b A; kNsApply: X' = (Bm X) + a X)
-          if (!live) continue;
+          // kNsPoly: Bm = c (A A) + b A; kNsApply: X' = (Bm X) + a X).
+          // A and Bm are symmetric: element (r, col) is written where
+          // col >= r, and its mirror (col, r) where col > r, so each element
+          // has one writer; elements below the diagonal are left to their
+          // mirrors.
+          if (ncols <= 0) continue;  // warp-uniform: every lane takes part in the mirror below
+          const bool sym = tile.kind != kNsApply;
           const float al = tile.kind == kNsPoly ? kNsC : 1.f;
           const float be = tile.kind == kNsPoly ? kNsB : (tile.kind == kNsApply ? kNsA : 0.f);
           __nv_bfloat16* out = g.ns + tile.c_off + (int64_t)r * tile.ldc + col0;
           const __nv_bfloat16* aux = g.ns + tile.aux_off + (int64_t)r * tile.ld_aux + col0;
+          uint32_t pk[16];
 #pragma unroll
           for (int s = 0; s < 4; ++s) {
-            if (8 * s >= ncols) break;
             float ax[8];
 #pragma unroll
             for (int e = 0; e < 8; ++e) ax[e] = 0.f;
-            if (tile.kind != kNsGram) {
+            if (tile.kind != kNsGram && live && 8 * s < ncols) {
               const uint4 av = *reinterpret_cast<const uint4*>(aux + 8 * s);
               const __nv_bfloat16* ab = reinterpret_cast<const __nv_bfloat16*>(&av);
 #pragma unroll
               for (int e = 0; e < 8; ++e) ax[e] = __bfloat162float(ab[e]);
             }
-            uint32_t pk[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
               const int j = 8 * s + 2 * e;
-              pk[e] = pack_bf16x2(al * __uint_as_float(v[j]) + be * ax[2 * e],
-                                  al * __uint_as_float(v[j + 1]) + be * ax[2 * e + 1]);
+              pk[4 * s + e] = pack_bf16x2(al * __uint_as_float(v[j]) + be * ax[2 * e],
+                                          al * __uint_as_float(v[j + 1]) + be * ax[2 * e + 1]);
             }
-            *reinterpret_cast<uint4*>(out + 8 * s) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          }
+          if (live) {
+#pragma unroll
+            for (int s = 0; s < 4; ++s) {
+              if (8 * s >= ncols) break;
+              const int c8 = col0 + 8 * s;
+              if (!sym || c8 >= r) {
+                *reinterpret_cast<uint4*>(out + 8 * s) =
+                    make_uint4(pk[4 * s], pk[4 * s + 1], pk[4 * s + 2], pk[4 * s + 3]);
+              } else if (c8 + 7 >= r) {  // the group holding the diagonal element
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                  if (c8 + e >= r) {
+                    const uint32_t wv = pk[4 * s + (e >> 1)];
+                    reinterpret_cast<uint16_t*>(out)[8 * s + e] = (uint16_t)((e & 1) ? (wv >> 16) : (wv & 0xFFFFu));
+                  }
+              }
+            }
+          }
+          if (sym) {
+            // the mirror: stage the warp's 32 x 32 chunk (row pitch 68 bytes),
+            // then lane j writes row col0 + j of the output at columns
+            // rbase .. rbase + 31 (the warp's rows)
+            uint8_t* buf = reinterpret_cast<uint8_t*>(tr_all + (warp - 2) * 32 * 32);
+#pragma unroll
+            for (int e = 0; e < 16; ++e) *reinterpret_cast<uint32_t*>(buf + lane * 68 + 4 * e) = pk[e];
+            __syncwarp();
+            const int rbase = u.m0 + 32 * q;
+            const int cm = col0 + lane;  // the mirrored row
+            if (lane < ncols) {
+              uint32_t t2[16];
+#pragma unroll
+              for (int e = 0; e < 16; ++e) {
+                const uint32_t lo = *reinterpret_cast<const uint16_t*>(buf + (2 * e) * 68 + 2 * lane);
+                const uint32_t hi = *reinterpret_cast<const uint16_t*>(buf + (2 * e + 1) * 68 + 2 * lane);
+                t2[e] = lo | (hi << 16);
+              }
+              __nv_bfloat16* mo = g.ns + tile.c_off + (int64_t)cm * tile.ldc + rbase;
+              if (rbase + 31 < cm && rbase + 31 < m_lim) {  // every element is above the diagonal
+#pragma unroll
+                for (int s = 0; s < 4; ++s)
+                  *reinterpret_cast<uint4*>(mo + 8 * s) =
+                      make_uint4(t2[4 * s], t2[4 * s + 1], t2[4 * s + 2], t2[4 * s + 3]);
+              } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                  if (rbase + i < cm && rbase + i < m_lim)
+                    reinterpret_cast<uint16_t*>(mo)[i] = (uint16_t)((i & 1) ? (t2[i >> 1] >> 16) : (t2[i >> 1] & 0xFFFFu));
+              }
+            }
+            __syncwarp();  // the buffer is reused by the next chunk
           }
         } else if (tile.kind == kWgrad) {
           // Transpose the warp's 32 rows x 32 columns through shared memory
@@ -1357,7 +1411,15 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
           t.ld_aux = mt.c;
         }
         split_n(t.n_real, ns, 32);
+        const size_t first = v.size();
         emit(v, t, (int)ceil_div(mt.r, kRowTile), ns);
+        // A and Bm are symmetric: a tile whose elements all lie below the
+        // diagonal (every column < every row) is left out; the epilogue of the
+        // tiles on and above it writes each upper element and its mirror
+        if (t.kind != kNsApply)
+          v.erase(std::remove_if(v.begin() + first, v.end(),
+                                 [](const TcTile& x) { return x.n0 + x.n_len <= x.m0; }),
+                  v.end());
       }
       std::stable_sort(v.begin(), v.end(), [](const TcTile& a, const TcTile& b) {
         return (int64_t)a.k_len * a.n_len > (int64_t)b.k_len * b.n_len;
