@@ -129,7 +129,9 @@ __global__ void k_sel_solo(const double* __restrict__ partial, int32_t P, int32_
 // equal scores by binary search: AUC = (sum of the positives' ranks -
 // n_pos (n_pos + 1) / 2) / (n_pos n_neg).  Rank sums are half-integers, exact
 // in fp64, so the result does not depend on the order of the sum.
-__global__ void __launch_bounds__(kAucThreads) k_sel_auc(const double* __restrict__ S,
+// two blocks per SM (32 registers a thread), so that a pool of up to two
+// candidates per SM sorts in one wave
+__global__ void __launch_bounds__(kAucThreads, 2) k_sel_auc(const double* __restrict__ S,
                                                          const float* __restrict__ preds,
                                                          const int32_t* __restrict__ y, int64_t N,
                                                          const int32_t* __restrict__ state,
