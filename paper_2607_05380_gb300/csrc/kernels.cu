@@ -451,8 +451,10 @@ struct HeadLogits {
 //      = (dlogits W_h) * [H > 0] / (1 - p), and dW_h += dlogits^T H.  Narrow
 //      heads split the rows into jb.split sets, added in order in shared
 //      memory, so that every block writes one partial.
+// One output: three blocks per SM (80 registers a thread, no spills; the
+// kernel waits on memory, 64 to 68 us per wide step for three against two).
 template <typename T, int DO>
-__global__ void __launch_bounds__(256, 2) k_head(HeadArgs<T> g) {
+__global__ void __launch_bounds__(256, DO == 1 ? 3 : 2) k_head(HeadArgs<T> g) {
   constexpr int R = DO <= 4 ? 4 : 2;
   constexpr int G = head_cols(DO);
   constexpr int DOP = DO == 1 ? 1 : (DO + 3) & ~3;  // padded row of dlogits in shared memory
