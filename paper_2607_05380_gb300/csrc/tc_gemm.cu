@@ -498,12 +498,17 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
     uint32_t stage = 0, phase = 0;
     uint32_t issued_mask = 0, last_parity = 0;  // per stage: ever issued, parity of the last issue
     bool ok = true;
-    if (lane < 2 && clu < g.n_tiles) prefetch_tile_map(g, g.tiles[clu], lane);
-    for (int t = clu; ok && t < g.n_tiles; t += n_clu) {
-      const TcTile tile = g.tiles[t];
-      // the descriptors of this CTA's next tile reach the descriptor cache
-      // while this tile's copies stream
-      if (lane < 2 && t + n_clu < g.n_tiles) prefetch_tile_map(g, g.tiles[t + n_clu], lane);
+    // A tile's descriptor is read while the previous tile's copies stream,
+    // and its tensor maps reach the descriptor cache from the middle of that
+    // tile: at a tile boundary the producer goes straight to the dependency
+    // check and the copies (a global read there cost a round trip in which
+    // the ring drained).
+    TcTile tile{}, nxt{};
+    if (clu < g.n_tiles) tile = g.tiles[clu];
+    if (lane < 2 && clu < g.n_tiles) prefetch_tile_map(g, tile, lane);
+    for (int t = clu; ok && t < g.n_tiles; t += n_clu, tile = nxt) {
+      const bool has_next = t + n_clu < g.n_tiles;
+      if (has_next) nxt = g.tiles[t + n_clu];
       if (!tile_live(tile, g.B_pad)) continue;
       const SubTile u = sub_tile(tile, rank, g.B_pad);
       const int K = tile.k_len ? tile.k_len : g.B_pad;
@@ -537,7 +542,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         break;
       }
       if (tile.dep >= 0) fence_proxy_async_global();  // every issuing lane, after the warp's acquires
+      const int k_mid = (((K + 63) >> 6) >> 1) << 6;
       for (int k0 = 0; k0 < K; k0 += 64) {
+        if (k0 == k_mid && lane < 2 && has_next) prefetch_tile_map(g, nxt, lane);
         bool got = true;
         if (lane == 0) {
           got = mbar_wait(&tl->empty[stage], phase ^ 1u, abort_flag, g.err, g.wait_ns, 1);
@@ -584,8 +591,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       constexpr uint32_t kStageStep = G::kStageBytes >> 4;
       uint32_t stage = 0, phase = 0, acc = 0, acc_phase = 0;
       bool ok = true;
-      for (int t = clu; ok && t < g.n_tiles; t += n_clu) {
-        const TcTile tile = g.tiles[t];
+      // the next tile's descriptor is read while this tile's MMAs issue
+      TcTile tile{}, nxt{};
+      if (clu < g.n_tiles) tile = g.tiles[clu];
+      for (int t = clu; ok && t < g.n_tiles; t += n_clu, tile = nxt) {
+        if (t + n_clu < g.n_tiles) nxt = g.tiles[t + n_clu];
         if (!tile_live(tile, g.B_pad)) continue;
         const int K = tile.k_len ? tile.k_len : g.B_pad;
         if (!mbar_wait(&tl->tempty[acc], acc_phase ^ 1u, abort_flag, g.err, 2 * g.wait_ns, 5)) break;
