@@ -524,9 +524,13 @@ def measure(args, tp, torch, dist, dev, name, steps, warmup, world, rank, headli
             "traffic": DRAM_TRAFFIC.get((name, "k_tc_gemm")) if plain else None,
             "ms_per_step": gemm_ms, "peak_source": peak_note}
     gemm["frac"] = gemm["achieved"] / gemm["peak"]
+    n_adam = n_params
+    if args.muon:     # AdamW keeps the biases and the head; Muon the hidden weight matrices
+        n_adam -= sum(in0_of(wl, emb, i_) * int(w_) + (int(L_) - 1) * int(w_) ** 2
+                      for i_, (L_, w_) in enumerate(zip(hp["depth"], hp["width"])))
     if adam_ms > 0:   # AdamW as a separate pass (the default): 30 B per parameter
-        mem = {"kernel": "k_adamw", "bound": "hbm", "achieved": 30.0 * n_params / (adam_ms / 1e3) / 1e9,
-               "ms_per_step": adam_ms, "bytes_per_step": 30.0 * n_params}
+        mem = {"kernel": "k_adamw", "bound": "hbm", "achieved": 30.0 * n_adam / (adam_ms / 1e3) / 1e9,
+               "ms_per_step": adam_ms, "bytes_per_step": 30.0 * n_adam}
     else:             # --fuse-optimizer: AdamW in the wgrad epilogue, 26 B per parameter
         mem = {"kernel": "k_tc_gemm backward launches (fused AdamW: read p, m, v; write p, m, v, bf16 p)",
                "bound": "hbm", "achieved": 26.0 * n_params / (bwd_ms / 1e3) / 1e9, "ms_per_step": bwd_ms,

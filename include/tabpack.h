@@ -188,7 +188,8 @@ tp_status pack_forward_backward_stacked(tabpack_t* pack, const float* X, int64_t
  * momentum buffers start at zero; AdamW in the weight-gradient epilogue
  * (fuse_optimizer) is turned off.  Allocates the Newton-Schulz buffers
  * (2 r c + 2 r^2 elements per matrix, r = min(out, in), c = max) on the
- * first call; synchronises.                                                  */
+ * first call; synchronises.  TP_EINVAL when a matrix has 2^31 elements or
+ * more (out times the input width rounded up to 8).                         */
 tp_status pack_set_muon(tabpack_t* pack, const float* lr_muon, float momentum, int32_t ns_steps);
 
 /* The direction X of the last Muon step of hidden layer `layer` of `member`

@@ -1330,70 +1330,141 @@ void launch_emb_bwd(cudaStream_t st, const EmbArgs<T>& a, int n_active, int cols
 }
 
 // ------------------------------------------------------------------ Muon
-// One block per chunk of kMuonChunk elements of a Muon matrix (row-major
-// [rows, cols] in the arena).
+// One block of 256 threads per chunk of kMuonChunk elements of a Muon matrix
+// (row-major [rows, cols] in the arena).  Widths are multiples of 16 and
+// padded input widths multiples of 8, and arena blocks start 32-element
+// aligned, so every chunk holds a multiple of 4 elements at a 16-byte
+// boundary and 4 consecutive elements share a row: the kernels move float4
+// and 4-element vectors, each thread kMuonV of them, all loads first.  The
+// per-element arithmetic is fp32; doubles appear only in the partial sums
+// (GB300's FP64 rate is a small fraction of its FP32 rate).
+constexpr int kMuonV = kMuonChunk / 4 / 256;
+static_assert(kMuonChunk % 1024 == 0, "a Muon chunk is a whole number of float4 per thread");
+
 template <typename T>
 struct MuonChunk {
   MuonMat mt;
-  int64_t e0, e1;  // element range of the chunk
-  __device__ __forceinline__ MuonChunk(const MuonArgs<T>& a) {
-    mt = a.mats[a.chunk_mat[blockIdx.x]];
-    e0 = (int64_t)(blockIdx.x - mt.chunk0) * kMuonChunk;
-    e1 = min(e0 + kMuonChunk, (int64_t)mt.rows * mt.cols);
+  int e0, n4;  // the chunk's first element within the matrix; its float4 count
+  __device__ __forceinline__ MuonChunk(const MuonArgs<T>& a, int blk) {
+    mt = a.mats[a.chunk_mat[blk]];
+    e0 = (blk - mt.chunk0) * kMuonChunk;
+    n4 = (min(e0 + kMuonChunk, mt.rows * mt.cols) - e0) >> 2;
   }
-  // index of element e of W in X (transposed when tr)
-  __device__ __forceinline__ int64_t xi(int64_t e) const {
-    const int64_t i = e / mt.cols, j = e - i * mt.cols;
-    return mt.tr ? j * mt.c + i : i * mt.c + j;
+  // index in X of element e of W (transposed when tr)
+  __device__ __forceinline__ int xi(int e) const {
+    if (!mt.tr) return e;
+    const int i = e / mt.cols;
+    return (e - i * mt.cols) * mt.c + i;
   }
 };
 
+__device__ __forceinline__ float4 load4f(const float* p) { return *reinterpret_cast<const float4*>(p); }
+__device__ __forceinline__ float4 load4f(const __nv_bfloat16* p) {
+  const uint2 u = *reinterpret_cast<const uint2*>(p);
+  const float2 lo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.x));
+  const float2 hi = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
+  return make_float4(lo.x, lo.y, hi.x, hi.y);
+}
+
+// the momentum update of one element; returns U's element
+__device__ __forceinline__ float muon_mom(float g, float& m, float mu) {
+  m = mu * m + (1.f - mu) * g;
+  return (1.f - mu) * g + mu * m;
+}
+
 // momentum M <- mu M + (1 - mu) G; U = (1 - mu) G + mu M; the chunk's sum of
-// squares of U (per-thread partials, then a fixed-order tree)
+// squares of U (fp32 per thread, then fp64 in a fixed-order tree)
 template <typename T>
 __global__ void __launch_bounds__(256) k_muon_momentum(MuonArgs<T> a) {
   pdl_trigger();
   pdl_wait();
-  const MuonChunk<T> ck(a);
+  const MuonChunk<T> ck(a, blockIdx.x);
   const float mu = a.mu;
-  double ss = 0.0;
-  for (int64_t e = ck.e0 + threadIdx.x; e < ck.e1; e += blockDim.x) {
-    const int64_t o = ck.mt.w_off + e;
-    const float g = a.grads[o];
-    const float m = mu * a.mom[o] + (1.f - mu) * g;
-    a.mom[o] = m;
-    const float u = (1.f - mu) * g + mu * m;
-    ss += (double)u * (double)u;
+  const float4* G4 = reinterpret_cast<const float4*>(a.grads + ck.mt.w_off + ck.e0);
+  float4* M4 = reinterpret_cast<float4*>(a.mom + ck.mt.w_off + ck.e0);
+  float4 g[kMuonV], m[kMuonV];
+#pragma unroll
+  for (int k = 0; k < kMuonV; ++k) {
+    const int v = threadIdx.x + 256 * k;
+    if (v < ck.n4) {
+      g[k] = G4[v];
+      m[k] = M4[v];
+    }
   }
-  __shared__ double red[256];
-  red[threadIdx.x] = ss;
+  float ss = 0.f;
+#pragma unroll
+  for (int k = 0; k < kMuonV; ++k) {
+    const int v = threadIdx.x + 256 * k;
+    if (v < ck.n4) {
+      const float u0 = muon_mom(g[k].x, m[k].x, mu), u1 = muon_mom(g[k].y, m[k].y, mu);
+      const float u2 = muon_mom(g[k].z, m[k].z, mu), u3 = muon_mom(g[k].w, m[k].w, mu);
+      M4[v] = m[k];
+      ss = fmaf(u0, u0, ss);
+      ss = fmaf(u1, u1, ss);
+      ss = fmaf(u2, u2, ss);
+      ss = fmaf(u3, u3, ss);
+    }
+  }
+  double s = (double)ss;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  __shared__ double red[8];
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
   __syncthreads();
-  for (int s = 128; s > 0; s >>= 1) {
-    if (threadIdx.x < s) red[threadIdx.x] += red[threadIdx.x + s];
-    __syncthreads();
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int w = 0; w < 8; ++w) t += red[w];
+    a.part[blockIdx.x] = t;
   }
-  if (threadIdx.x == 0) a.part[blockIdx.x] = red[0];
 }
 
-// X0 = U / max(||U||_F, 1e-7), transposed when rows > cols
+// X0 = U / max(||U||_F, 1e-7), transposed when rows > cols.  Chunks in
+// reverse order: the momentum pass's last chunks are still in L2.
 template <typename T>
 __global__ void __launch_bounds__(256) k_muon_x0(MuonArgs<T> a) {
   pdl_trigger();
   pdl_wait();
-  const MuonChunk<T> ck(a);
+  const MuonChunk<T> ck(a, gridDim.x - 1 - blockIdx.x);
   __shared__ float inv_s;
-  if (threadIdx.x == 0) {
+  if (threadIdx.x < 32) {  // the matrix's norm from its chunks' partials, one warp
     double ss = 0.0;
-    for (int k = 0; k < ck.mt.n_chunks; ++k) ss += a.part[ck.mt.chunk0 + k];
-    inv_s = (float)(1.0 / fmax(sqrt(ss), 1e-7));
+    for (int k = threadIdx.x; k < ck.mt.n_chunks; k += 32) ss += a.part[ck.mt.chunk0 + k];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    if (threadIdx.x == 0) inv_s = (float)(1.0 / fmax(sqrt(ss), 1e-7));
+  }
+  const float mu = a.mu;
+  const float4* G4 = reinterpret_cast<const float4*>(a.grads + ck.mt.w_off + ck.e0);
+  const float4* M4 = reinterpret_cast<const float4*>(a.mom + ck.mt.w_off + ck.e0);
+  float4 g[kMuonV], m[kMuonV];
+#pragma unroll
+  for (int k = 0; k < kMuonV; ++k) {
+    const int v = threadIdx.x + 256 * k;
+    if (v < ck.n4) {
+      g[k] = __ldcs(G4 + v);
+      m[k] = M4[v];
+    }
   }
   __syncthreads();
-  const float inv = inv_s, mu = a.mu;
+  const float inv = inv_s;
   T* X = a.ns + ck.mt.x_off[0];
-  for (int64_t e = ck.e0 + threadIdx.x; e < ck.e1; e += blockDim.x) {
-    const int64_t o = ck.mt.w_off + e;
-    const float u = (1.f - mu) * a.grads[o] + mu * a.mom[o];
-    X[ck.xi(e)] = Elem<T>::from_f(u * inv);
+#pragma unroll
+  for (int k = 0; k < kMuonV; ++k) {
+    const int v = threadIdx.x + 256 * k;
+    if (v < ck.n4) {
+      const float4 u = make_float4(((1.f - mu) * g[k].x + mu * m[k].x) * inv, ((1.f - mu) * g[k].y + mu * m[k].y) * inv,
+                                   ((1.f - mu) * g[k].z + mu * m[k].z) * inv, ((1.f - mu) * g[k].w + mu * m[k].w) * inv);
+      const int e = ck.e0 + 4 * v;
+      if (!ck.mt.tr) {
+        store4(X + e, u);
+      } else {  // the 4 elements share a row of W: 4 entries of a column of X
+        const int x0 = ck.xi(e);
+        X[x0] = Elem<T>::from_f(u.x);
+        X[x0 + ck.mt.c] = Elem<T>::from_f(u.y);
+        X[x0 + 2 * ck.mt.c] = Elem<T>::from_f(u.z);
+        X[x0 + 3 * ck.mt.c] = Elem<T>::from_f(u.w);
+      }
+    }
   }
 }
 
@@ -1402,16 +1473,42 @@ template <typename T>
 __global__ void __launch_bounds__(256) k_muon_apply(MuonArgs<T> a) {
   pdl_trigger();
   pdl_wait();
-  const MuonChunk<T> ck(a);
+  const MuonChunk<T> ck(a, blockIdx.x);
   const float lr = ck.mt.lr, wd = a.mem[ck.mt.member].wd, sc = ck.mt.scale;
   const T* X = a.ns + ck.mt.x_off[a.x_final];
-  for (int64_t e = ck.e0 + threadIdx.x; e < ck.e1; e += blockDim.x) {
-    const int64_t o = ck.mt.w_off + e;
-    float p = a.params[o];
-    p = p - lr * wd * p;
-    p = p - lr * sc * Elem<T>::to_f(X[ck.xi(e)]);
-    a.params[o] = p;
-    if (a.wq_out) a.wq_out[o] = __float2bfloat16_rn(p);
+  float4* P4 = reinterpret_cast<float4*>(a.params + ck.mt.w_off + ck.e0);
+  float4 p[kMuonV], x[kMuonV];
+#pragma unroll
+  for (int k = 0; k < kMuonV; ++k) {
+    const int v = threadIdx.x + 256 * k;
+    if (v < ck.n4) {
+      p[k] = P4[v];
+      const int e = ck.e0 + 4 * v;
+      if (!ck.mt.tr) {
+        x[k] = load4f(X + e);
+      } else {
+        const int x0 = ck.xi(e);
+        x[k] = make_float4(Elem<T>::to_f(X[x0]), Elem<T>::to_f(X[x0 + ck.mt.c]), Elem<T>::to_f(X[x0 + 2 * ck.mt.c]),
+                           Elem<T>::to_f(X[x0 + 3 * ck.mt.c]));
+      }
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < kMuonV; ++k) {
+    const int v = threadIdx.x + 256 * k;
+    if (v < ck.n4) {
+      float4 q = p[k];
+      q.x = q.x - lr * wd * q.x;
+      q.y = q.y - lr * wd * q.y;
+      q.z = q.z - lr * wd * q.z;
+      q.w = q.w - lr * wd * q.w;
+      q.x = q.x - lr * sc * x[k].x;
+      q.y = q.y - lr * sc * x[k].y;
+      q.z = q.z - lr * sc * x[k].z;
+      q.w = q.w - lr * sc * x[k].w;
+      P4[v] = q;
+      if (a.wq_out) store4(a.wq_out + ck.mt.w_off + ck.e0 + 4 * v, q);
+    }
   }
 }
 

@@ -1558,6 +1558,11 @@ tp_status pack_set_muon(tabpack_t* h, const float* lr_muon, float momentum, int3
     return fail(h, TP_EINVAL, "momentum must be in [0, 1) and ns_steps in 1..32");
   for (int i = 0; i < h->cfg.m; ++i)
     if (!(lr_muon[i] >= 0.f)) return fail(h, TP_EINVAL, "lr_muon[%d] must be >= 0", i);
+  for (int i = 0; i < h->cfg.m; ++i) {
+    const int64_t in_max = std::max<int64_t>(h->in0_pad[i], h->width[i]);
+    if ((int64_t)h->width[i] * in_max > (int64_t)INT32_MAX)
+      return fail(h, TP_EINVAL, "member %d: a Muon matrix would have 2^31 elements or more", i);
+  }
   TP_TRY(sync_check(h));
   const int m = h->cfg.m;
   if (!h->muon) {

@@ -371,6 +371,11 @@ __device__ __forceinline__ void flush_chunk(uint8_t* buf, int lane, __nv_bfloat1
   __syncwarp();  // the buffer is reused by the next chunk
 }
 
+// Element (row, col) of a chunk staged by stage_group (16-bit).
+__device__ __forceinline__ uint32_t staged_elem(const uint8_t* buf, int row, int col) {
+  return *reinterpret_cast<const uint16_t*>(buf + row * 64 + 16 * ((col >> 3) ^ ((row >> 1) & 3)) + 2 * (col & 7));
+}
+
 // a[i] for a runtime i < N (N = 4 or 8) without indexing (keeps a[] in registers)
 template <typename V, int N>
 __device__ __forceinline__ V pick(const V (&a)[N], int i) {
@@ -724,16 +729,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         tmem_ld32(taddr + c, v);
         if constexpr (kNs) {
           // Newton-Schulz: out = alpha acc + beta aux, bf16 (kNsGram: A;
-          // kNsPoly: Bm = c (A A) + b A; kNsApply: X' = (Bm X) + a X).
-          // A and Bm are symmetric: element (r, col) is written where
-          // col >= r, and its mirror (col, r) where col > r, so each element
-          // has one writer; elements below the diagonal are left to their
-          // mirrors.
-          if (ncols <= 0) continue;  // warp-uniform: every lane takes part in the mirror below
+          // kNsPoly: Bm = c (A A) + b A; kNsApply: X' = (Bm X) + a X).  The
+          // warp's 32 x 32 chunk is staged in its buffer and leaves as whole
+          // 64-byte row segments.  A and Bm are symmetric and only the tiles
+          // on or above the diagonal run; chunk origins are 32-aligned, so a
+          // chunk lies wholly above, on or below the diagonal.  Above: the
+          // chunk and its transpose at the mirror position.  On: the chunk
+          // with its upper triangle mirrored into the lower.  Below (on a
+          // diagonal tile): nothing, its mirror writes it.
+          if (ncols <= 0) continue;  // warp-uniform
           const bool sym = tile.kind != kNsApply;
+          const int rbase = u.m0 + 32 * q;
+          if (sym && col0 < rbase) continue;  // warp-uniform
           const float al = tile.kind == kNsPoly ? kNsC : 1.f;
           const float be = tile.kind == kNsPoly ? kNsB : (tile.kind == kNsApply ? kNsA : 0.f);
-          __nv_bfloat16* out = g.ns + tile.c_off + (int64_t)r * tile.ldc + col0;
           const __nv_bfloat16* aux = g.ns + tile.aux_off + (int64_t)r * tile.ld_aux + col0;
           uint32_t pk[16];
 #pragma unroll
@@ -754,56 +763,41 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
                                           al * __uint_as_float(v[j + 1]) + be * ax[2 * e + 1]);
             }
           }
-          if (live) {
+          uint8_t* buf = reinterpret_cast<uint8_t*>(tr_all + (warp - 2) * 32 * 32);
+          __nv_bfloat16* out = g.ns + tile.c_off + (int64_t)rbase * tile.ldc + col0;
 #pragma unroll
-            for (int s = 0; s < 4; ++s) {
-              if (8 * s >= ncols) break;
-              const int c8 = col0 + 8 * s;
-              if (!sym || c8 >= r) {
-                *reinterpret_cast<uint4*>(out + 8 * s) =
-                    make_uint4(pk[4 * s], pk[4 * s + 1], pk[4 * s + 2], pk[4 * s + 3]);
-              } else if (c8 + 7 >= r) {  // the group holding the diagonal element
-#pragma unroll
-                for (int e = 0; e < 8; ++e)
-                  if (c8 + e >= r) {
-                    const uint32_t wv = pk[4 * s + (e >> 1)];
-                    reinterpret_cast<uint16_t*>(out)[8 * s + e] = (uint16_t)((e & 1) ? (wv >> 16) : (wv & 0xFFFFu));
-                  }
-              }
-            }
-          }
-          if (sym) {
-            // the mirror: stage the warp's 32 x 32 chunk (row pitch 68 bytes),
-            // then lane j writes row col0 + j of the output at columns
-            // rbase .. rbase + 31 (the warp's rows)
-            uint8_t* buf = reinterpret_cast<uint8_t*>(tr_all + (warp - 2) * 32 * 32);
-#pragma unroll
-            for (int e = 0; e < 16; ++e) *reinterpret_cast<uint32_t*>(buf + lane * 68 + 4 * e) = pk[e];
-            __syncwarp();
-            const int rbase = u.m0 + 32 * q;
-            const int cm = col0 + lane;  // the mirrored row
-            if (lane < ncols) {
+          for (int s = 0; s < 4; ++s) stage_group(buf, lane, s, pk[4 * s], pk[4 * s + 1], pk[4 * s + 2], pk[4 * s + 3]);
+          if (!sym || col0 > rbase) {
+            flush_chunk(buf, lane, out, tile.ldc, rbase, m_lim, ncols);
+            if (sym) {
+              // lane j gathers column j of the chunk: row col0 + j of the
+              // output at columns rbase .. rbase + 31
               uint32_t t2[16];
 #pragma unroll
-              for (int e = 0; e < 16; ++e) {
-                const uint32_t lo = *reinterpret_cast<const uint16_t*>(buf + (2 * e) * 68 + 2 * lane);
-                const uint32_t hi = *reinterpret_cast<const uint16_t*>(buf + (2 * e + 1) * 68 + 2 * lane);
-                t2[e] = lo | (hi << 16);
-              }
-              __nv_bfloat16* mo = g.ns + tile.c_off + (int64_t)cm * tile.ldc + rbase;
-              if (rbase + 31 < cm && rbase + 31 < m_lim) {  // every element is above the diagonal
+              for (int e = 0; e < 16; ++e)
+                t2[e] = staged_elem(buf, 2 * e, lane) | (staged_elem(buf, 2 * e + 1, lane) << 16);
+              __syncwarp();
 #pragma unroll
-                for (int s = 0; s < 4; ++s)
-                  *reinterpret_cast<uint4*>(mo + 8 * s) =
-                      make_uint4(t2[4 * s], t2[4 * s + 1], t2[4 * s + 2], t2[4 * s + 3]);
-              } else {
-#pragma unroll
-                for (int i = 0; i < 32; ++i)
-                  if (rbase + i < cm && rbase + i < m_lim)
-                    reinterpret_cast<uint16_t*>(mo)[i] = (uint16_t)((i & 1) ? (t2[i >> 1] >> 16) : (t2[i >> 1] & 0xFFFFu));
-              }
+              for (int s = 0; s < 4; ++s) stage_group(buf, lane, s, t2[4 * s], t2[4 * s + 1], t2[4 * s + 2], t2[4 * s + 3]);
+              flush_chunk(buf, lane, g.ns + tile.c_off + (int64_t)col0 * tile.ldc + rbase, tile.ldc, col0, col0 + ncols,
+                          min(32, m_lim - rbase));
             }
-            __syncwarp();  // the buffer is reused by the next chunk
+          } else {
+            // on the diagonal: row i keeps its columns j >= i and takes
+            // element (j, i) of the chunk for j < i
+            __syncwarp();
+            uint32_t t2[16];
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+              const int j0 = 2 * e, j1 = 2 * e + 1;
+              const uint32_t lo = j0 >= lane ? (pk[e] & 0xFFFFu) : staged_elem(buf, j0, lane);
+              const uint32_t hi = j1 >= lane ? (pk[e] >> 16) : staged_elem(buf, j1, lane);
+              t2[e] = lo | (hi << 16);
+            }
+            __syncwarp();
+#pragma unroll
+            for (int s = 0; s < 4; ++s) stage_group(buf, lane, s, t2[4 * s], t2[4 * s + 1], t2[4 * s + 2], t2[4 * s + 3]);
+            flush_chunk(buf, lane, out, tile.ldc, rbase, m_lim, ncols);
           }
         } else if (tile.kind == kWgrad) {
           // Transpose the warp's 32 rows x 32 columns through shared memory
