@@ -1373,11 +1373,13 @@ __device__ __forceinline__ float muon_mom(float g, float& m, float mu) {
 }
 
 // momentum M <- mu M + (1 - mu) G; U = (1 - mu) G + mu M; the chunk's sum of
-// squares of U (fp32 per thread, then fp64 in a fixed-order tree)
+// squares of U (fp32 per thread, then fp64 in a fixed-order tree).  Also
+// clears the counters of the Newton-Schulz launch that follows.
 template <typename T>
 __global__ void __launch_bounds__(256) k_muon_momentum(MuonArgs<T> a) {
   pdl_trigger();
   pdl_wait();
+  for (int i = blockIdx.x * 256 + threadIdx.x; i < a.n_ns_cnt; i += gridDim.x * 256) a.ns_cnt[i] = 0;
   const MuonChunk<T> ck(a, blockIdx.x);
   const float mu = a.mu;
   const float4* G4 = reinterpret_cast<const float4*>(a.grads + ck.mt.w_off + ck.e0);

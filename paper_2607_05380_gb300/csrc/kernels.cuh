@@ -42,6 +42,8 @@ struct MuonArgs {
   const MemberDev* mem;
   float mu;
   int32_t x_final;           // the X buffer that holds the result
+  int* ns_cnt;               // the Newton-Schulz launch's counters, cleared by the momentum kernel
+  int32_t n_ns_cnt;
 };
 
 template <typename T>

@@ -598,6 +598,7 @@ tp_status build_schedule(tabpack* h) {
     lay.mask_off = h->mask_words > 0 ? &h->mask_off : nullptr;
     lay.muon = h->muon ? &h->mmats : nullptr;
     lay.ns = h->ns;
+    lay.ns_steps = h->ns_steps;
     lay.in0_pad = &h->in0_pad;
     if (h->emb) {
       lay.xb = h->ex;
@@ -955,24 +956,28 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
     ma.mem = h->mem_dev;
     ma.mu = h->muon_mu;
     ma.x_final = h->ns_steps & 1;
+    ma.ns_cnt = h->bf16 ? h->tc.ns_cnt_dev : nullptr;
+    ma.n_ns_cnt = h->bf16 ? h->tc.n_ns_cnt : 0;
     int nl = 0;
     for (int phase = 0; phase < 2; ++phase) {
       launch_muon<T>(h->st, ma, h->n_muon_chunks, phase);
       TP_LAUNCHED(h);
       ++nl;
     }
-    for (int it = 0; it < h->ns_steps; ++it) {
-      const int p = it & 1;
-      const int which[3] = {p, 2, 3 + p};
-      for (int q = 0; q < 3; ++q) {
-        if (h->bf16) {
-          TP_TRY(tc_run_ns(h->tc, h->st, which[q], h->ns, h->mem_dev, h->err));
-        } else {
+    if (h->bf16) {  // every iteration in one tensor-core launch
+      TP_TRY(tc_run_ns(h->tc, h->st, h->ns, h->mem_dev, h->err));
+      TP_LAUNCHED(h);
+      ++nl;
+    } else {
+      for (int it = 0; it < h->ns_steps; ++it) {
+        const int p = it & 1;
+        const int which[3] = {p, 2, 3 + p};
+        for (int q = 0; q < 3; ++q) {
           auto g = gemm_args<T>(h, B, B_pad, step, 0);
           launch_gemm_simt<T>(h->st, g, h->ns_simt_rng[which[q]].first, h->ns_simt_rng[which[q]].second);
+          TP_LAUNCHED(h);
+          ++nl;
         }
-        TP_LAUNCHED(h);
-        ++nl;
       }
     }
     launch_muon<T>(h->st, ma, h->n_muon_chunks, 2);

@@ -538,10 +538,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
       const bool mn = is_a ? !a_k : !b_k;  // MN-major box: x = row / column, y = k
       const int xy0 = is_a ? u.m0 + 64 * bl : bn0 + (b_k ? 128 : 64) * qb;
       const uint32_t off = is_a ? (uint32_t)bl * kBoxBytes : (uint32_t)kABytes + (uint32_t)qb * boxB;
+      // Newton-Schulz tiles count on one counter per matrix and product,
+      // shared by the CTAs of a pair, and both CTAs wait: each loads half of
+      // B, which earlier tiles of the launch wrote.
       bool dep_ok = true;
-      if (u.rows_live && tile.dep >= 0)
-        dep_ok = dep_wait(g.cnt + tile.dep + (tile.dep_n ? rank : 0), tile.dep_n ? tile.dep_n : g.B_pad / kRowTile,
-                          tile.dep_need, abort_flag, g.err, g.wait_ns, 3, lane);
+      if ((u.rows_live || kNs) && tile.dep >= 0)
+        dep_ok = dep_wait(g.cnt + tile.dep + (tile.dep_n && !kNs ? rank : 0),
+                          tile.dep_n ? tile.dep_n : g.B_pad / kRowTile, tile.dep_need, abort_flag, g.err, g.wait_ns, 3,
+                          lane);
       if (!dep_ok) {
         ok = false;
         break;
@@ -705,6 +709,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           }
           bits[ci] = mb;
         }
+      }
+      // Newton-Schulz: the epilogue reads `aux` (A or X), which earlier
+      // tiles of the launch wrote, with plain loads; its own acquire of the
+      // tile's dependency orders them (and, through this tile's count, the
+      // later tiles that overwrite a buffer after it).
+      if constexpr (kNs) {
+        if (tile.dep >= 0 &&
+            !dep_wait(g.cnt + tile.dep, 1, tile.dep_need, abort_flag, g.err, 2 * g.wait_ns, 13, lane))
+          break;
       }
       if (!mbar_wait(&tl->tfull[acc], acc_phase, abort_flag, g.err, 2 * g.wait_ns, 7)) break;
       tc_fence_after();
@@ -982,7 +995,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         if (!mbar_wait(&tl->stored[slot], (uint32_t)(n_pub / kPubSlots) & 1u, abort_flag, g.err, 4 * g.wait_ns, 9))
           break;
         fence_proxy_async_global();
-        red_release_add(g.cnt + tile.sig + rank, kEpiWarps);
+        red_release_add(g.cnt + tile.sig + (kNs ? 0 : rank), kEpiWarps);
         mbar_arrive(&tl->pub_free[slot]);
         ++n_pub;
       }
@@ -1369,16 +1382,38 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
     all.insert(all.end(), VW[Lmax - 1].begin(), VW[Lmax - 1].end());
   }
   plan.bwd_rng = {plan.fwd_rng.second, (int)all.size() - plan.fwd_rng.second};
-  // Muon: the Newton-Schulz products of the active members' matrices, one
-  // launch per product kind (and X buffer), costliest tiles first
-  for (auto& r : plan.ns_rng) r = {(int)all.size(), 0};
-  if (lay.muon && plan.ns_maps) {
-    for (int which = 0; which < 5; ++which) {
+  // Muon: every Newton-Schulz iteration's three products of the active
+  // members' matrices in one launch, product after product (costliest tiles
+  // first within each).  Counters, per matrix j: 3 j + 0 / 1 / 2 count the
+  // stored X X^T / polynomial / update tiles (kEpiWarps per CTA with live
+  // rows), cumulatively over the iterations.  Iteration it's X X^T tiles
+  // wait for every update tile of iteration it - 1, its polynomial tiles for
+  // every X X^T tile of it, its update tiles for every polynomial tile of it.
+  // Every dependency lies in an earlier product of the list, and the chain
+  // orders each buffer's rewrite after the last reads of its previous
+  // contents (A and Bm each iteration, X every other).
+  plan.ns_rng = {(int)all.size(), 0};
+  if (lay.muon && plan.ns_maps && lay.ns_steps > 0) {
+    const int n_mat = (int)lay.muon->size();
+    if (plan.n_ns_cnt != 3 * n_mat) {
+      if (plan.ns_cnt_dev) cudaFree(plan.ns_cnt_dev);
+      plan.ns_cnt_dev = nullptr;
+      plan.n_ns_cnt = 3 * n_mat;
+      if (cudaMalloc(&plan.ns_cnt_dev, sizeof(int) * plan.n_ns_cnt) != cudaSuccess ||
+          cudaMemset(plan.ns_cnt_dev, 0, sizeof(int) * plan.n_ns_cnt) != cudaSuccess) {
+        plan.n_ns_cnt = 0;
+        err = "cudaMalloc(Newton-Schulz counters) failed";
+        return TP_ENOMEM;
+      }
+    }
+    // the tiles of one product of every active matrix (X buffer p), with
+    // per matrix the number of CTAs with live rows
+    std::vector<int> live[3];
+    auto product = [&](int kind, int p) {
       std::vector<TcTile> v;
-      for (size_t j = 0; j < lay.muon->size(); ++j) {
+      for (int j = 0; j < n_mat; ++j) {
         const MuonMat& mt = (*lay.muon)[j];
         if (!active[mt.member]) continue;
-        const int p = which == 0 || which == 3 ? 0 : 1;  // the X buffer read
         TcTile t{};
         t.member = mt.member;
         t.layer = mt.layer;
@@ -1387,15 +1422,13 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
         t.dep = -1;
         t.sig = -1;
         t.mask_off = -1;
-        if (which < 2) {          // A = X X^T
-          t.kind = kNsGram;
+        if (kind == kNsGram) {        // A = X X^T
           t.n_real = mt.r;
           t.k_len = mt.c;
           t.map_a = t.map_b = plan.map_ns[j * 4 + p];
           t.c_off = mt.a_off;
           t.ldc = mt.r;
-        } else if (which == 2) {  // Bm = b A + c A A
-          t.kind = kNsPoly;
+        } else if (kind == kNsPoly) { // Bm = b A + c A A
           t.n_real = mt.r;
           t.k_len = mt.r;
           t.map_a = t.map_b = plan.map_ns[j * 4 + 2];
@@ -1403,8 +1436,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
           t.ldc = mt.r;
           t.aux_off = mt.a_off;
           t.ld_aux = mt.r;
-        } else {                  // X' = a X + Bm X
-          t.kind = kNsApply;
+        } else {                      // X' = a X + Bm X
           t.n_real = mt.c;
           t.k_len = mt.r;
           t.map_a = plan.map_ns[j * 4 + 3];
@@ -1414,23 +1446,48 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
           t.aux_off = mt.x_off[p];
           t.ld_aux = mt.c;
         }
+        t.kind = kind;
         split_n(t.n_real, ns, 32);
         const size_t first = v.size();
         emit(v, t, (int)ceil_div(mt.r, kRowTile), ns);
         // A and Bm are symmetric: a tile whose elements all lie below the
         // diagonal (every column < every row) is left out; the epilogue of the
         // tiles on and above it writes each upper element and its mirror
-        if (t.kind != kNsApply)
+        if (kind != kNsApply)
           v.erase(std::remove_if(v.begin() + first, v.end(),
                                  [](const TcTile& x) { return x.n0 + x.n_len <= x.m0; }),
                   v.end());
+        int n_live = 0;
+        for (size_t e = first; e < v.size(); ++e) {
+          v[e].dep_n = 1;
+          v[e].sig = 3 * j + (kind - kNsGram);
+          for (int q = 0; q < cta; ++q) n_live += v[e].m0 + kRowTile * q < mt.r;
+        }
+        live[kind - kNsGram].resize(n_mat);
+        live[kind - kNsGram][j] = kEpiWarps * n_live;
       }
       std::stable_sort(v.begin(), v.end(), [](const TcTile& a, const TcTile& b) {
         return (int64_t)a.k_len * a.n_len > (int64_t)b.k_len * b.n_len;
       });
-      plan.ns_rng[which] = {(int)all.size(), (int)v.size()};
-      all.insert(all.end(), v.begin(), v.end());
+      return v;
+    };
+    static_assert(kNsPoly == kNsGram + 1 && kNsApply == kNsGram + 2, "Newton-Schulz kinds are consecutive");
+    for (int it = 0; it < lay.ns_steps; ++it) {
+      const int p = it & 1;  // the X buffer read by this iteration
+      for (int kind = kNsGram; kind <= kNsApply; ++kind) {
+        std::vector<TcTile> v = product(kind, kind == kNsPoly ? 0 : p);
+        for (TcTile& t : v) {
+          const int j = t.sig / 3;
+          const int prev = kind == kNsGram ? 2 : kind - kNsGram - 1;  // the product waited for
+          const int done = kind == kNsGram ? it : it + 1;              // its iterations completed
+          t.dep = done > 0 ? 3 * j + prev : -1;
+          t.dep_need = done > 0 ? done * live[prev][j] : 0;
+          if (kind == kNsApply && it + 1 == lay.ns_steps) t.sig = -1;  // nothing waits for the last update
+        }
+        all.insert(all.end(), v.begin(), v.end());
+      }
     }
+    plan.ns_rng = {plan.ns_rng.first, (int)all.size() - plan.ns_rng.first};
   }
   if ((int)all.size() + 1 > plan.cap_tiles) {
     if (plan.tiles_dev) cudaFree(plan.tiles_dev);
@@ -1457,7 +1514,7 @@ static tp_status launch(TcPlan& plan, cudaStream_t st, const std::pair<int, int>
   a.n_tiles = rng.second;
   a.maps = plan.maps_dev;
   a.err = plan.err_dev;
-  a.cnt = plan.cnt_dev;
+  a.cnt = ns ? plan.ns_cnt_dev : plan.cnt_dev;
   a.kmaj_off = plan.kmaj_off;
   a.wait_ns = plan.wait_ns;
   const int cta = plan.cta;
@@ -1520,13 +1577,13 @@ tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, 
   return launch(plan, st, plan.bwd_rng, a, err);
 }
 
-tp_status tc_run_ns(TcPlan& plan, cudaStream_t st, int which, void* ns, const MemberDev* mem, std::string& err) {
+tp_status tc_run_ns(TcPlan& plan, cudaStream_t st, void* ns, const MemberDev* mem, std::string& err) {
   TcArgs a{};
   a.B = 0;
   a.B_pad = 0;
   a.mem = mem;  // the epilogue reads every tile's member record
   a.ns = (__nv_bfloat16*)ns;
-  return launch(plan, st, plan.ns_rng[which], a, err, true);
+  return launch(plan, st, plan.ns_rng, a, err, true);
 }
 
 tp_status tc_check(TcPlan& plan, cudaStream_t st, std::string& err) {
@@ -1581,6 +1638,9 @@ void tc_free_plan(TcPlan& plan) {
   if (plan.cnt_dev) cudaFree(plan.cnt_dev);
   plan.cnt_dev = nullptr;
   plan.n_cnt = 0;
+  if (plan.ns_cnt_dev) cudaFree(plan.ns_cnt_dev);
+  plan.ns_cnt_dev = nullptr;
+  plan.n_ns_cnt = 0;
   plan.maps_dev = nullptr;
   plan.tiles_dev = nullptr;
   plan.cap_tiles = 0;

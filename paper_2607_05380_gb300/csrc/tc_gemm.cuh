@@ -51,9 +51,13 @@ struct TcPlan {
   TcTile* tiles_dev = nullptr;
   int cap_tiles = 0;
   std::pair<int, int> fwd_rng, bwd_rng;  // tile ranges of the forward / backward launch
-  // Newton-Schulz launches: kNsGram reading X0 / X1, kNsPoly, kNsApply
-  // reading X0 / X1 (writing the other)
-  std::pair<int, int> ns_rng[5] = {};
+  // The Newton-Schulz launch: every iteration's kNsGram, kNsPoly and
+  // kNsApply tiles, with their own completion counters (3 per Muon matrix),
+  // which must be zero before the launch (the Muon momentum kernel that
+  // precedes it clears them)
+  std::pair<int, int> ns_rng = {};
+  int* ns_cnt_dev = nullptr;
+  int n_ns_cnt = 0;
   bool ns_maps = false;    // the map table holds the Muon matrices' maps
   // Row-block completion counters: act of (member, layer) then dz of
   // (member, layer), B_cap / 128 each.  They must be zero before a launch
@@ -86,6 +90,7 @@ struct TcLayout {          // what the plan needs to know about the pack's arena
   // and the bf16 arena holding their X, A and Bm buffers
   const std::vector<MuonMat>* muon = nullptr;
   const void* ns = nullptr;
+  int ns_steps = 0;        // Newton-Schulz iterations per Muon step
   int64_t xb_stride = 0;   // > 0: a batch matrix per member (stacked batches), this many elements apart
   // Periodic embeddings: member i's first layer reads the matrix at xb +
   // x0_off[i] ([B_cap, in0_pad[i] + 16]) and, with de_off, its input gradient
@@ -109,9 +114,9 @@ tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, 
 // weight copy).
 tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, const MemberDev* mem, void* act,
                      void* dz, float* grads, int update, const AdamDev& adam, std::string& err);
-// One Newton-Schulz product launch over every Muon matrix: which = 0 / 1
-// kNsGram of X0 / X1, 2 kNsPoly, 3 / 4 kNsApply of X0 / X1.
-tp_status tc_run_ns(TcPlan& plan, cudaStream_t st, int which, void* ns, const MemberDev* mem, std::string& err);
+// Every Newton-Schulz iteration of every Muon matrix in one launch (X0 in
+// buffer 0; the result in buffer ns_steps & 1).
+tp_status tc_run_ns(TcPlan& plan, cudaStream_t st, void* ns, const MemberDev* mem, std::string& err);
 // Reads and clears the device error word (synchronises the stream).
 tp_status tc_check(TcPlan& plan, cudaStream_t st, std::string& err);
 // Tests: the first forward tile with a dependency waits for a count the
