@@ -357,18 +357,60 @@ __device__ __forceinline__ void stage_group(uint8_t* buf, int lane, int s, uint3
   *reinterpret_cast<uint4*>(buf + lane * 64 + 16 * (s ^ ((lane >> 1) & 3))) = make_uint4(a, b, c, d);
 }
 // out: the warp's first row at the chunk's first column; rows from rbase on
-// are valid below m_lim, columns below ncols.
+// are valid below m_lim, columns below ncols.  kAhead: the four shared
+// loads first, then the four stores (16 more registers, no load-to-store
+// round trip per row group).
+template <bool kAhead = false>
 __device__ __forceinline__ void flush_chunk(uint8_t* buf, int lane, __nv_bfloat16* out, int64_t ldc, int rbase,
                                             int m_lim, int ncols) {
   __syncwarp();
   const int seg = lane & 3;
+  if constexpr (kAhead) {
+    uint4 val[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int rl = 8 * j + (lane >> 2);
+      val[j] = *reinterpret_cast<const uint4*>(buf + rl * 64 + 16 * (seg ^ ((rl >> 1) & 3)));
+    }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int rl = 8 * j + (lane >> 2);
+      if (rbase + rl < m_lim && 8 * seg < ncols) *reinterpret_cast<uint4*>(out + (int64_t)rl * ldc + 8 * seg) = val[j];
+    }
+  } else {
 #pragma unroll 1
-  for (int j = 0; j < 4; ++j) {
-    const int rl = 8 * j + (lane >> 2);
-    const uint4 val = *reinterpret_cast<const uint4*>(buf + rl * 64 + 16 * (seg ^ ((rl >> 1) & 3)));
-    if (rbase + rl < m_lim && 8 * seg < ncols) *reinterpret_cast<uint4*>(out + (int64_t)rl * ldc + 8 * seg) = val;
+    for (int j = 0; j < 4; ++j) {
+      const int rl = 8 * j + (lane >> 2);
+      const uint4 val = *reinterpret_cast<const uint4*>(buf + rl * 64 + 16 * (seg ^ ((rl >> 1) & 3)));
+      if (rbase + rl < m_lim && 8 * seg < ncols) *reinterpret_cast<uint4*>(out + (int64_t)rl * ldc + 8 * seg) = val;
+    }
   }
   __syncwarp();  // the buffer is reused by the next chunk
+}
+
+// The transpose of a chunk staged by stage_group in `src`, staged the same
+// way in `dst`: per group S of source columns, ldmatrix .trans reads the four
+// 8 x 8 blocks of rows 8 k .. 8 k + 7 (k = 0..3) transposed and stmatrix
+// writes them as rows 8 S .. 8 S + 7, group k, of dst.  Lane l addresses row
+// l % 8 of block l / 8; the XOR swizzle keeps both conflict-free.  The
+// caller orders the staging before (warp barrier) and the reads after.
+__device__ __forceinline__ void stage_transpose(const uint8_t* src, uint8_t* dst, int lane) {
+  const int rr = lane & 7, blk = lane >> 3;
+#pragma unroll
+  for (int S = 0; S < 4; ++S) {
+    const int ri = 8 * blk + rr;
+    const uint32_t a = smem_u32(src + ri * 64 + 16 * (S ^ ((ri >> 1) & 3)));
+    uint32_t r0, r1, r2, r3;
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(a)
+                 : "memory");
+    const int ro = 8 * S + rr;
+    const uint32_t d = smem_u32(dst + ro * 64 + 16 * (blk ^ ((ro >> 1) & 3)));
+    asm volatile("stmatrix.sync.aligned.m8n8.x4.shared.b16 [%0], {%1, %2, %3, %4};" ::"r"(d), "r"(r0), "r"(r1),
+                 "r"(r2), "r"(r3)
+                 : "memory");
+  }
 }
 
 // Element (row, col) of a chunk staged by stage_group (16-bit).
@@ -719,6 +761,22 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
             !dep_wait(g.cnt + tile.dep, 1, tile.dep_need, abort_flag, g.err, 2 * g.wait_ns, 13, lane))
           break;
       }
+      // Newton-Schulz: this lane's 32 values of the aux term in chunk ci of
+      // its warp (zeros where the chunk is not written), loaded one chunk
+      // ahead -- the first while the tile's products run.
+      auto ns_aux = [&](int ci, uint4(&a)[4]) {
+        const int c = 32 * half + 32 * kEpiPerQ * ci;
+        const int col0 = tile.n0 + c;
+        const int ncols = min(32, n_hi - col0);
+        const bool need = tile.kind != kNsGram && row_ok && c < n_end && ncols > 0 &&
+                          (tile.kind == kNsApply || col0 >= u.m0 + 32 * q);
+        const __nv_bfloat16* p = g.ns + tile.aux_off + (int64_t)r * tile.ld_aux + col0;
+#pragma unroll
+        for (int s = 0; s < 4; ++s)
+          a[s] = need && 8 * s < ncols ? *reinterpret_cast<const uint4*>(p + 8 * s) : make_uint4(0u, 0u, 0u, 0u);
+      };
+      uint4 axn[4];
+      if constexpr (kNs) ns_aux(0, axn);
       if (!mbar_wait(&tl->tfull[acc], acc_phase, abort_flag, g.err, 2 * g.wait_ns, 7)) break;
       tc_fence_after();
       const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + acc * kAccCols;
@@ -747,33 +805,29 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           // 64-byte row segments.  A and Bm are symmetric and only the tiles
           // on or above the diagonal run; chunk origins are 32-aligned, so a
           // chunk lies wholly above, on or below the diagonal.  Above: the
-          // chunk and its transpose at the mirror position.  On: the chunk
+          // chunk, and its transpose (staged by ldmatrix / stmatrix in the
+          // buffer's second half) at the mirror position.  On: the chunk
           // with its upper triangle mirrored into the lower.  Below (on a
           // diagonal tile): nothing, its mirror writes it.
+          uint4 axc[4];
+#pragma unroll
+          for (int s = 0; s < 4; ++s) axc[s] = axn[s];
+          if (ci + 1 < kChunks) ns_aux(ci + 1, axn);
           if (ncols <= 0) continue;  // warp-uniform
           const bool sym = tile.kind != kNsApply;
           const int rbase = u.m0 + 32 * q;
           if (sym && col0 < rbase) continue;  // warp-uniform
           const float al = tile.kind == kNsPoly ? kNsC : 1.f;
           const float be = tile.kind == kNsPoly ? kNsB : (tile.kind == kNsApply ? kNsA : 0.f);
-          const __nv_bfloat16* aux = g.ns + tile.aux_off + (int64_t)r * tile.ld_aux + col0;
           uint32_t pk[16];
 #pragma unroll
           for (int s = 0; s < 4; ++s) {
-            float ax[8];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) ax[e] = 0.f;
-            if (tile.kind != kNsGram && live && 8 * s < ncols) {
-              const uint4 av = *reinterpret_cast<const uint4*>(aux + 8 * s);
-              const __nv_bfloat16* ab = reinterpret_cast<const __nv_bfloat16*>(&av);
-#pragma unroll
-              for (int e = 0; e < 8; ++e) ax[e] = __bfloat162float(ab[e]);
-            }
+            const __nv_bfloat16* ab = reinterpret_cast<const __nv_bfloat16*>(&axc[s]);
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
               const int j = 8 * s + 2 * e;
-              pk[4 * s + e] = pack_bf16x2(al * __uint_as_float(v[j]) + be * ax[2 * e],
-                                          al * __uint_as_float(v[j + 1]) + be * ax[2 * e + 1]);
+              pk[4 * s + e] = pack_bf16x2(al * __uint_as_float(v[j]) + be * __bfloat162float(ab[2 * e]),
+                                          al * __uint_as_float(v[j + 1]) + be * __bfloat162float(ab[2 * e + 1]));
             }
           }
           uint8_t* buf = reinterpret_cast<uint8_t*>(tr_all + (warp - 2) * 32 * 32);
@@ -781,19 +835,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
 #pragma unroll
           for (int s = 0; s < 4; ++s) stage_group(buf, lane, s, pk[4 * s], pk[4 * s + 1], pk[4 * s + 2], pk[4 * s + 3]);
           if (!sym || col0 > rbase) {
-            flush_chunk(buf, lane, out, tile.ldc, rbase, m_lim, ncols);
-            if (sym) {
-              // lane j gathers column j of the chunk: row col0 + j of the
-              // output at columns rbase .. rbase + 31
-              uint32_t t2[16];
-#pragma unroll
-              for (int e = 0; e < 16; ++e)
-                t2[e] = staged_elem(buf, 2 * e, lane) | (staged_elem(buf, 2 * e + 1, lane) << 16);
-              __syncwarp();
-#pragma unroll
-              for (int s = 0; s < 4; ++s) stage_group(buf, lane, s, t2[4 * s], t2[4 * s + 1], t2[4 * s + 2], t2[4 * s + 3]);
-              flush_chunk(buf, lane, g.ns + tile.c_off + (int64_t)col0 * tile.ldc + rbase, tile.ldc, col0, col0 + ncols,
-                          min(32, m_lim - rbase));
+            flush_chunk<true>(buf, lane, out, tile.ldc, rbase, m_lim, ncols);
+            if (sym) {  // rows col0 .. col0 + 31 of the output at columns rbase .. rbase + 31
+              stage_transpose(buf, buf + 2048, lane);
+              flush_chunk<true>(buf + 2048, lane, g.ns + tile.c_off + (int64_t)col0 * tile.ldc + rbase, tile.ldc, col0,
+                                col0 + ncols, min(32, m_lim - rbase));
             }
           } else {
             // on the diagonal: row i keeps its columns j >= i and takes
@@ -810,7 +856,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
             __syncwarp();
 #pragma unroll
             for (int s = 0; s < 4; ++s) stage_group(buf, lane, s, t2[4 * s], t2[4 * s + 1], t2[4 * s + 2], t2[4 * s + 3]);
-            flush_chunk(buf, lane, out, tile.ldc, rbase, m_lim, ncols);
+            flush_chunk<true>(buf, lane, out, tile.ldc, rbase, m_lim, ncols);
           }
         } else if (tile.kind == kWgrad) {
           // Transpose the warp's 32 rows x 32 columns through shared memory
