@@ -233,3 +233,40 @@ def test_muon_full_size_sampled_members(tp):
                 errs[(i, l, len(g_.shape))] = max(errs.get((i, l, len(g_.shape)), 0.0), e)
     bad = {k: e for k, e in errs.items() if e > TOL["bf16"]}
     assert not bad, bad
+
+
+@pytest.mark.parametrize("ctas", ["1", "2"])
+@pytest.mark.parametrize("ns_steps", [1, 2, 3])
+def test_muon_ns_steps_and_cta_pairs(tp, monkeypatch, ns_steps, ctas):
+    """The single Newton-Schulz launch of bf16 mode (every iteration's three
+    products, chained by per-matrix counters) for 1, 2 and 3 iterations (the
+    result in either X buffer), with single CTAs and with CTA pairs. Widths
+    384 and 640 leave the second CTA of a pair's last row tile without rows, so
+    it waits and loads its half of B only for its partner. The tall first
+    layers (384 and 640 outputs over 200 inputs) run transposed, and the middle
+    member is inactive. Bar, per active member and layer: the direction from
+    the GPU's own gradient within twice the error that the oracle's bf16 model
+    of the same iteration makes against the exact one (norm-wise), or 5e-3."""
+    monkeypatch.setenv("TP_GEMM_CTAS", ctas)
+    d_in, d_out, B = 200, 4, 256
+    hp = {"depth": np.array([2, 1, 2], dtype=np.int32), "width": np.array([384, 256, 640], dtype=np.int32),
+          "dropout": np.array([0.0, 0.1, 0.2], dtype=np.float32), "lr": np.full(3, 1e-3, dtype=np.float32),
+          "wd": np.full(3, 1e-4, dtype=np.float32)}
+    pk = tp.Pack(d_in, d_out, "multiclass", hp["depth"], hp["width"], hp["dropout"], hp["lr"], hp["wd"],
+                 max_batch=B, seed=4, precision="bf16")
+    pk.set_muon(np.full(3, 0.02, dtype=np.float32), ns_steps=ns_steps)
+    pk.set_active(np.array([1, 0, 1], dtype=np.uint8))
+    X, y = data("multiclass", 2 * B, d_in, d_out, 11)
+    Xd, yd = (torch.from_numpy(a).to(DEV) for a in (X, y))
+    idx = np.random.default_rng(2).permutation(2 * B)[:B].astype(np.int32)
+    pk.train_step(Xd, torch.from_numpy(idx).to(DEV), yd, 0)
+    errs = {}
+    for i in (0, 2):
+        for l in range(int(hp["depth"][i])):
+            G = pk.get_grads(i, l)[0].astype(np.float64)
+            O_ref = oracle.newton_schulz(G, steps=ns_steps)
+            e_orc = np.linalg.norm(oracle.newton_schulz(G, steps=ns_steps, bf16=True) - O_ref) / np.linalg.norm(O_ref)
+            e_gpu = np.linalg.norm(pk.muon_dir(i, l) - O_ref) / np.linalg.norm(O_ref)
+            if e_gpu > max(2.0 * e_orc, 5e-3):
+                errs[(i, l)] = (e_gpu, e_orc)
+    assert not errs, errs
