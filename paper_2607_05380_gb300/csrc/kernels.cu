@@ -1344,9 +1344,11 @@ static_assert(kMuonChunk % 1024 == 0, "a Muon chunk is a whole number of float4 
 template <typename T>
 struct MuonChunk {
   MuonMat mt;
+  int mat;     // its index in the matrix list
   int e0, n4;  // the chunk's first element within the matrix; its float4 count
   __device__ __forceinline__ MuonChunk(const MuonArgs<T>& a, int blk) {
-    mt = a.mats[a.chunk_mat[blk]];
+    mat = a.chunk_mat[blk];
+    mt = a.mats[mat];
     e0 = (blk - mt.chunk0) * kMuonChunk;
     n4 = (min(e0 + kMuonChunk, mt.rows * mt.cols) - e0) >> 2;
   }
@@ -1372,9 +1374,22 @@ __device__ __forceinline__ float muon_mom(float g, float& m, float mu) {
   return (1.f - mu) * g + mu * m;
 }
 
+// 1 / max(|U|_F, 1e-7) of a matrix from its chunks' sums of squares, by one
+// warp in a fixed order (lane j sums chunks j, j + 32, ...; then a butterfly):
+// the same value wherever it is computed.
+__device__ __forceinline__ float muon_inv_norm(const double* part, int chunk0, int n_chunks, int lane) {
+  double ss = 0.0;
+  for (int k = lane; k < n_chunks; k += 32) ss += __ldcg(part + chunk0 + k);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  return (float)(1.0 / fmax(sqrt(ss), 1e-7));
+}
+
 // momentum M <- mu M + (1 - mu) G; U = (1 - mu) G + mu M; the chunk's sum of
 // squares of U (fp32 per thread, then fp64 in a fixed-order tree).  Also
-// clears the counters of the Newton-Schulz launch that follows.
+// clears the counters of the Newton-Schulz launch that follows.  x0_fused:
+// U is also written as X0 (transposed when rows > cols), and the last chunk
+// of a matrix to finish stores the matrix's scale.
 template <typename T>
 __global__ void __launch_bounds__(256) k_muon_momentum(MuonArgs<T> a) {
   pdl_trigger();
@@ -1405,6 +1420,19 @@ __global__ void __launch_bounds__(256) k_muon_momentum(MuonArgs<T> a) {
       ss = fmaf(u1, u1, ss);
       ss = fmaf(u2, u2, ss);
       ss = fmaf(u3, u3, ss);
+      if (a.x0_fused) {
+        T* X = a.ns + ck.mt.x_off[0];
+        const int e = ck.e0 + 4 * v;
+        if (!ck.mt.tr) {
+          store4(X + e, make_float4(u0, u1, u2, u3));
+        } else {  // the 4 elements share a row of W: 4 entries of a column of X
+          const int x0 = ck.xi(e);
+          X[x0] = Elem<T>::from_f(u0);
+          X[x0 + ck.mt.c] = Elem<T>::from_f(u1);
+          X[x0 + 2 * ck.mt.c] = Elem<T>::from_f(u2);
+          X[x0 + 3 * ck.mt.c] = Elem<T>::from_f(u3);
+        }
+      }
     }
   }
   double s = (double)ss;
@@ -1413,10 +1441,25 @@ __global__ void __launch_bounds__(256) k_muon_momentum(MuonArgs<T> a) {
   __shared__ double red[8];
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
   __syncthreads();
+  __shared__ int last;
   if (threadIdx.x == 0) {
     double t = 0.0;
     for (int w = 0; w < 8; ++w) t += red[w];
     a.part[blockIdx.x] = t;
+    if (a.x0_fused) {
+      __threadfence();  // the partial before the arrival
+      last = atomicAdd(a.mat_done + ck.mat, 1) == ck.mt.n_chunks - 1;
+    }
+  }
+  if (!a.x0_fused) return;
+  __syncthreads();
+  if (last && threadIdx.x < 32) {
+    __threadfence();  // every arrival before the partials' reads
+    const float inv = muon_inv_norm(a.part, ck.mt.chunk0, ck.mt.n_chunks, threadIdx.x);
+    if (threadIdx.x == 0) {
+      a.ns_scale[ck.mat] = inv;
+      a.mat_done[ck.mat] = 0;
+    }
   }
 }
 
@@ -1429,11 +1472,8 @@ __global__ void __launch_bounds__(256) k_muon_x0(MuonArgs<T> a) {
   const MuonChunk<T> ck(a, gridDim.x - 1 - blockIdx.x);
   __shared__ float inv_s;
   if (threadIdx.x < 32) {  // the matrix's norm from its chunks' partials, one warp
-    double ss = 0.0;
-    for (int k = threadIdx.x; k < ck.mt.n_chunks; k += 32) ss += a.part[ck.mt.chunk0 + k];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-    if (threadIdx.x == 0) inv_s = (float)(1.0 / fmax(sqrt(ss), 1e-7));
+    const float inv = muon_inv_norm(a.part, ck.mt.chunk0, ck.mt.n_chunks, threadIdx.x);
+    if (threadIdx.x == 0) inv_s = inv;
   }
   const float mu = a.mu;
   const float4* G4 = reinterpret_cast<const float4*>(a.grads + ck.mt.w_off + ck.e0);

@@ -44,6 +44,13 @@ struct MuonArgs {
   int32_t x_final;           // the X buffer that holds the result
   int* ns_cnt;               // the Newton-Schulz launch's counters, cleared by the momentum kernel
   int32_t n_ns_cnt;
+  // x0_fused = 1 (the tensor-core iteration): the momentum kernel also writes
+  // U, unnormalised, as X0 and, from the last chunk of each matrix to finish,
+  // ns_scale[matrix] = 1 / max(|U|_F, 1e-7); mat_done counts the chunks done
+  // (back to 0 after each step).  k_muon_x0 is then not launched.
+  int32_t x0_fused;
+  float* ns_scale;
+  int* mat_done;
 };
 
 template <typename T>

@@ -96,6 +96,8 @@ struct tabpack {
   MuonMat* mmats_dev = nullptr;
   int32_t* mchunk_mat_dev = nullptr;
   double* mpart_dev = nullptr;
+  float* mscale_dev = nullptr;   // per matrix: 1 / |U|_F (bf16 mode)
+  int* mdone_dev = nullptr;      // per matrix: momentum chunks done (bf16 mode)
   int n_muon_chunks = 0;
   std::pair<int, int> ns_simt_rng[5] = {};  // CUDA-core Newton-Schulz tiles (fp32 mode)
 
@@ -721,12 +723,15 @@ void free_all(tabpack* h) {
   h->ex = nullptr;
   if (h->embm_dev) cudaFree(h->embm_dev);
   h->embm_dev = nullptr;
-  for (void* p : {h->ns, (void*)h->mmats_dev, (void*)h->mchunk_mat_dev, (void*)h->mpart_dev})
+  for (void* p : {h->ns, (void*)h->mmats_dev, (void*)h->mchunk_mat_dev, (void*)h->mpart_dev, (void*)h->mscale_dev,
+                  (void*)h->mdone_dev})
     if (p) cudaFree(p);
   h->ns = nullptr;
   h->mmats_dev = nullptr;
   h->mchunk_mat_dev = nullptr;
   h->mpart_dev = nullptr;
+  h->mscale_dev = nullptr;
+  h->mdone_dev = nullptr;
   for (void* p : h->allocs) cudaFree(p);
   h->allocs.clear();
   for (auto e : h->prof.pool) cudaEventDestroy(e);
@@ -958,14 +963,19 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
     ma.x_final = h->ns_steps & 1;
     ma.ns_cnt = h->bf16 ? h->tc.ns_cnt_dev : nullptr;
     ma.n_ns_cnt = h->bf16 ? h->tc.n_ns_cnt : 0;
+    // bf16: the momentum kernel writes U as X0 and 1 / |U|_F, which the
+    // first iteration's products apply; fp32: k_muon_x0 normalises X0
+    ma.x0_fused = h->bf16 ? 1 : 0;
+    ma.ns_scale = h->mscale_dev;
+    ma.mat_done = h->mdone_dev;
     int nl = 0;
-    for (int phase = 0; phase < 2; ++phase) {
+    for (int phase = 0; phase < (h->bf16 ? 1 : 2); ++phase) {
       launch_muon<T>(h->st, ma, h->n_muon_chunks, phase);
       TP_LAUNCHED(h);
       ++nl;
     }
     if (h->bf16) {  // every iteration in one tensor-core launch
-      TP_TRY(tc_run_ns(h->tc, h->st, h->ns, h->mem_dev, h->err));
+      TP_TRY(tc_run_ns(h->tc, h->st, h->ns, h->mscale_dev, h->mem_dev, h->err));
       TP_LAUNCHED(h);
       ++nl;
     } else {
@@ -1599,6 +1609,10 @@ tp_status pack_set_muon(tabpack_t* h, const float* lr_muon, float momentum, int3
     TP_CUDA(h, cudaMalloc((void**)&h->mmats_dev, sizeof(MuonMat) * h->mmats.size()));
     TP_CUDA(h, cudaMalloc((void**)&h->mchunk_mat_dev, sizeof(int32_t) * std::max<int64_t>(n_chunks, 1)));
     TP_CUDA(h, cudaMalloc((void**)&h->mpart_dev, sizeof(double) * std::max<int64_t>(n_chunks, 1)));
+    const size_t n_mat = std::max<size_t>(h->mmats.size(), 1);
+    TP_CUDA(h, cudaMalloc((void**)&h->mscale_dev, sizeof(float) * n_mat));
+    TP_CUDA(h, cudaMalloc((void**)&h->mdone_dev, sizeof(int) * n_mat));
+    TP_CUDA(h, cudaMemset(h->mdone_dev, 0, sizeof(int) * n_mat));
     // Muon's momentum starts at zero in the first-moment arena
     for (const MuonMat& mt : h->mmats)
       TP_CUDA(h, cudaMemset(h->adam_m + mt.w_off, 0, sizeof(float) * (size_t)mt.rows * mt.cols));

@@ -126,6 +126,7 @@ struct TcArgs {
   int* cnt;            // row-block completion counters
   int32_t kmaj_off;    // index distance to the same matrix's map with 128-row boxes (K-major loads)
   __nv_bfloat16* ns;   // Newton-Schulz arena (kNs launches)
+  const float* ns_scale;  // per Muon matrix: 1 / |U|_F (kNs launches)
   uint64_t wait_ns;    // budget of every wait that can give up (TcPlan::wait_ns)
 };
 
@@ -817,8 +818,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           const bool sym = tile.kind != kNsApply;
           const int rbase = u.m0 + 32 * q;
           if (sym && col0 < rbase) continue;  // warp-uniform
-          const float al = tile.kind == kNsPoly ? kNsC : 1.f;
-          const float be = tile.kind == kNsPoly ? kNsB : (tile.kind == kNsApply ? kNsA : 0.f);
+          // the first iteration reads U = |U|_F X0: A = s^2 (U U^T), X' = s (Bm U + a U)
+          const float sc = tile.ns_scale ? g.ns_scale[tile.ns_scale - 1] : 1.f;
+          const float al = tile.kind == kNsPoly ? kNsC : (tile.kind == kNsGram ? sc * sc : sc);
+          const float be = tile.kind == kNsPoly ? kNsB : (tile.kind == kNsApply ? kNsA * sc : 0.f);
           uint32_t pk[16];
 #pragma unroll
           for (int s = 0; s < 4; ++s) {
@@ -1437,7 +1440,9 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
   // every X X^T tile of it, its update tiles for every polynomial tile of it.
   // Every dependency lies in an earlier product of the list, and the chain
   // orders each buffer's rewrite after the last reads of its previous
-  // contents (A and Bm each iteration, X every other).
+  // contents (A and Bm each iteration, X every other).  Buffer 0 holds U
+  // unnormalised: the first iteration's X X^T and update tiles carry the
+  // matrix's 1 / |U|_F (ns_scale).
   plan.ns_rng = {(int)all.size(), 0};
   if (lay.muon && plan.ns_maps && lay.ns_steps > 0) {
     const int n_mat = (int)lay.muon->size();
@@ -1528,6 +1533,7 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
           const int done = kind == kNsGram ? it : it + 1;              // its iterations completed
           t.dep = done > 0 ? 3 * j + prev : -1;
           t.dep_need = done > 0 ? done * live[prev][j] : 0;
+          if (it == 0 && kind != kNsPoly) t.ns_scale = j + 1;
           if (kind == kNsApply && it + 1 == lay.ns_steps) t.sig = -1;  // nothing waits for the last update
         }
         all.insert(all.end(), v.begin(), v.end());
@@ -1623,12 +1629,14 @@ tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, 
   return launch(plan, st, plan.bwd_rng, a, err);
 }
 
-tp_status tc_run_ns(TcPlan& plan, cudaStream_t st, void* ns, const MemberDev* mem, std::string& err) {
+tp_status tc_run_ns(TcPlan& plan, cudaStream_t st, void* ns, const float* ns_scale, const MemberDev* mem,
+                    std::string& err) {
   TcArgs a{};
   a.B = 0;
   a.B_pad = 0;
   a.mem = mem;  // the epilogue reads every tile's member record
   a.ns = (__nv_bfloat16*)ns;
+  a.ns_scale = ns_scale;
   return launch(plan, st, plan.ns_rng, a, err, true);
 }
 

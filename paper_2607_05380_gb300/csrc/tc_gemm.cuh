@@ -32,10 +32,13 @@ struct TcTile {
   // mi of the tile waits until counters d .. d + n - 1 each reach dep_need
   // (dep_n = 1: d = dep + mi, n = 1; dep_n = 0: d = dep, n = the step's
   // B_pad / 128); after storing its output every epilogue warp adds 1 to
-  // counter sig + mi.  -1: none.
+  // counter sig + mi.  -1: none.  Newton-Schulz tiles: counters dep and
+  // sig themselves, shared by the CTAs of a pair (one per matrix and product).
   int32_t dep, dep_n, dep_need, sig;
   int32_t mask_off;        // kFwd of a member with dropout: word offset of its keep words in the
                            // mask arena ([ceil(n_real / 32), mask rows]); -1: none
+  int32_t ns_scale;        // kNsGram / kNsApply of the first iteration: 1 + the Muon matrix whose
+                           // 1 / |U|_F scales the product (X0 holds U unnormalised); 0: none
   int64_t c_off;           // output: act (kFwd), dz (kDgrad), weight offset in the arena (kWgrad)
   int64_t aux_off;         // kFwd: bias offset in params; kDgrad: H_l offset in act (mask);
                            // kWgrad: bias offset in the arena
@@ -114,9 +117,11 @@ tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, 
 // weight copy).
 tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, const MemberDev* mem, void* act,
                      void* dz, float* grads, int update, const AdamDev& adam, std::string& err);
-// Every Newton-Schulz iteration of every Muon matrix in one launch (X0 in
-// buffer 0; the result in buffer ns_steps & 1).
-tp_status tc_run_ns(TcPlan& plan, cudaStream_t st, void* ns, const MemberDev* mem, std::string& err);
+// Every Newton-Schulz iteration of every Muon matrix in one launch (U in
+// buffer 0, scaled by ns_scale[matrix] = 1 / |U|_F inside the first
+// iteration's products; the result in buffer ns_steps & 1).
+tp_status tc_run_ns(TcPlan& plan, cudaStream_t st, void* ns, const float* ns_scale, const MemberDev* mem,
+                    std::string& err);
 // Reads and clears the device error word (synchronises the stream).
 tp_status tc_check(TcPlan& plan, cudaStream_t st, std::string& err);
 // Tests: the first forward tile with a dependency waits for a count the

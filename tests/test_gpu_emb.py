@@ -194,7 +194,12 @@ def test_emb_eight_steps(tp, prec):
 def test_emb_muon_one_step(tp, prec):
     """Muon on the first layer's [width, d_in d_emb] matrix (AdamW on the
     embeddings): parameters after one step (fp32 against the oracle; bf16
-    by the bf16 rule)."""
+    by the bf16 rule against the exact oracle).  The bf16 kernel stores U and
+    applies 1 / |U|_F in fp32 inside the first Newton-Schulz products, while
+    the oracle's bf16-storage model rounds U / |U|_F: two bf16 roundings of
+    the same iteration, each within d of the exact result, so the diagnostic
+    comparison with the model is norm-wise within 2 d (triangle inequality)
+    where it misses 2e-2 elementwise."""
     d_in, m, B, d_out = 7, 4, 160, 3
     hp = random_pack(m, d_in, d_out, seed=95, width=(16, 96, 16), depth=(1, 2), dropout=(0.0, 0.0))
     em = sample_emb(m, d_in, seed=9)
@@ -208,7 +213,7 @@ def test_emb_muon_one_step(tp, prec):
     Xd, yd, idxd = to_dev(X, y, idx)
     pk.train_step(Xd, idxd, yd, 0)
     orc.train_step(X, idx, y, 0)
-    errs, problems, relaxed = compare_params(pk, orc, hp, prec, extra=emb_params(pk, orc))
+    errs, problems, relaxed = compare_params(pk, orc, hp, prec, extra=emb_params(pk, orc), diag_ratio=2.0)
     assert not problems and not relaxed, (problems, errs)
 
 
