@@ -181,7 +181,9 @@ tp_status pack_forward_backward_stacked(tabpack_t* pack, const float* X, int64_t
  *   X = U / max(||U||_F, 1e-7), transposed when out > in;
  *   ns_steps times: A = X X^T; Bm = b A + c A A; X = a X + Bm X,
  *   (a, b, c) = (3.4445, -4.7750, 2.0315) (on the tensor cores in bf16 mode,
- *   X, A and Bm stored in bf16; on CUDA cores in fp32 mode);
+ *   X, A and Bm stored in bf16, and U stored as X with 1 / max(||U||_F,
+ *   1e-7) applied in fp32 inside the first iteration's products; on CUDA
+ *   cores in fp32 mode);
  *   W <- W - lr_muon wd W;  W <- W - lr_muon max(1, out / in)^(1/2) X
  * (in = the real input width).  lr_muon: host [m]; wd: the member's weight
  * decay; momentum in [0, 1); ns_steps in 1..32 (5 in the paper's Muon).  The
