@@ -1330,14 +1330,15 @@ void launch_emb_bwd(cudaStream_t st, const EmbArgs<T>& a, int n_active, int cols
 }
 
 // ------------------------------------------------------------------ Muon
-// One block of 256 threads per chunk of kMuonChunk elements of a Muon matrix
-// (row-major [rows, cols] in the arena).  Widths are multiples of 16 and
+// One block of 256 threads per chunk of a Muon matrix (row-major [rows,
+// cols] in the arena): kMuonChunk consecutive elements, or for a transposed
+// matrix a 32 x 128 tile of W (muon_chunks).  Widths are multiples of 16 and
 // padded input widths multiples of 8, and arena blocks start 32-element
-// aligned, so every chunk holds a multiple of 4 elements at a 16-byte
-// boundary and 4 consecutive elements share a row: the kernels move float4
-// and 4-element vectors, each thread kMuonV of them, all loads first.  The
-// per-element arithmetic is fp32; doubles appear only in the partial sums
-// (GB300's FP64 rate is a small fraction of its FP32 rate).
+// aligned, so 4 consecutive elements of a chunk share a row and start at a
+// 16-byte boundary: the kernels move float4 and 4-element vectors, each
+// thread kMuonV of them, all loads first.  The per-element arithmetic is
+// fp32; doubles appear only in the partial sums (GB300's FP64 rate is a
+// small fraction of its FP32 rate).
 constexpr int kMuonV = kMuonChunk / 4 / 256;
 static_assert(kMuonChunk % 1024 == 0, "a Muon chunk is a whole number of float4 per thread");
 
@@ -1345,18 +1346,37 @@ template <typename T>
 struct MuonChunk {
   MuonMat mt;
   int mat;     // its index in the matrix list
-  int e0, n4;  // the chunk's first element within the matrix; its float4 count
+  int e0, n4;  // flat chunk: its first element within the matrix and its float4 count
+  int i0, j0;  // tile of a transposed matrix: its first row and column of W
   __device__ __forceinline__ MuonChunk(const MuonArgs<T>& a, int blk) {
     mat = a.chunk_mat[blk];
     mt = a.mats[mat];
-    e0 = (blk - mt.chunk0) * kMuonChunk;
-    n4 = (min(e0 + kMuonChunk, mt.rows * mt.cols) - e0) >> 2;
+    const int k = blk - mt.chunk0;
+    if (!mt.tr) {
+      e0 = k * kMuonChunk;
+      n4 = (min(e0 + kMuonChunk, mt.rows * mt.cols) - e0) >> 2;
+      i0 = j0 = 0;
+    } else {
+      const int tpr = (mt.cols + kMuonTileC - 1) / kMuonTileC;
+      i0 = (k / tpr) * kMuonTileR;
+      j0 = (k % tpr) * kMuonTileC;
+      e0 = n4 = 0;
+    }
   }
-  // index in X of element e of W (transposed when tr)
-  __device__ __forceinline__ int xi(int e) const {
-    if (!mt.tr) return e;
-    const int i = e / mt.cols;
-    return (e - i * mt.cols) * mt.c + i;
+  // Element offset in W (from w_off) of this chunk's float4 q (0 <= q <
+  // kMuonChunk / 4), or -1 outside the matrix.  Tiles: row q / 32, columns
+  // 4 (q % 32) .. + 3 of the tile, so a warp reads 512 contiguous bytes.
+  __device__ __forceinline__ int w_elem(int q) const {
+    if (!mt.tr) return q < n4 ? e0 + 4 * q : -1;
+    const int row = i0 + (q >> 5), col = j0 + 4 * (q & 31);
+    return row < mt.rows && col < mt.cols ? row * mt.cols + col : -1;
+  }
+  // Tiles: piece p (0 <= p < kMuonChunk / 4) of X's rows -- row j0 + p / 8,
+  // columns i0 + 4 (p % 8) .. + 3, i.e. W's column j0 + p / 8 at its rows
+  // i0 + 4 (p % 8) .. + 3 -- as an element offset in X, or -1 outside.
+  __device__ __forceinline__ int x_piece(int p) const {
+    const int j = j0 + (p >> 3), i = i0 + 4 * (p & 7);
+    return j < mt.cols && i < mt.rows ? j * mt.c + i : -1;
   }
 };
 
@@ -1367,6 +1387,12 @@ __device__ __forceinline__ float4 load4f(const __nv_bfloat16* p) {
   const float2 hi = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&u.y));
   return make_float4(lo.x, lo.y, hi.x, hi.y);
 }
+
+// A tile's X values staged in shared memory as [tile row][tile column] of W
+// (pitch kMuonTileC + 2: the column reads of x_piece order touch distinct
+// banks).
+template <typename T>
+using MuonStage = T[kMuonTileR][kMuonTileC + 2];
 
 // the momentum update of one element; returns U's element
 __device__ __forceinline__ float muon_mom(float g, float& m, float mu) {
@@ -1388,8 +1414,9 @@ __device__ __forceinline__ float muon_inv_norm(const double* part, int chunk0, i
 // momentum M <- mu M + (1 - mu) G; U = (1 - mu) G + mu M; the chunk's sum of
 // squares of U (fp32 per thread, then fp64 in a fixed-order tree).  Also
 // clears the counters of the Newton-Schulz launch that follows.  x0_fused:
-// U is also written as X0 (transposed when rows > cols), and the last chunk
-// of a matrix to finish stores the matrix's scale.
+// U is also written as X0 (a transposed matrix's tile through shared memory,
+// as whole row segments of X), and the last chunk of a matrix to finish
+// stores the matrix's scale.
 template <typename T>
 __global__ void __launch_bounds__(256) k_muon_momentum(MuonArgs<T> a) {
   pdl_trigger();
@@ -1397,42 +1424,52 @@ __global__ void __launch_bounds__(256) k_muon_momentum(MuonArgs<T> a) {
   for (int i = blockIdx.x * 256 + threadIdx.x; i < a.n_ns_cnt; i += gridDim.x * 256) a.ns_cnt[i] = 0;
   const MuonChunk<T> ck(a, blockIdx.x);
   const float mu = a.mu;
-  const float4* G4 = reinterpret_cast<const float4*>(a.grads + ck.mt.w_off + ck.e0);
-  float4* M4 = reinterpret_cast<float4*>(a.mom + ck.mt.w_off + ck.e0);
+  const float* G = a.grads + ck.mt.w_off;
+  float* M = a.mom + ck.mt.w_off;
+  T* X = a.ns + ck.mt.x_off[0];
+  __shared__ MuonStage<T> st;
   float4 g[kMuonV], m[kMuonV];
+  int ev[kMuonV];
 #pragma unroll
   for (int k = 0; k < kMuonV; ++k) {
-    const int v = threadIdx.x + 256 * k;
-    if (v < ck.n4) {
-      g[k] = G4[v];
-      m[k] = M4[v];
+    ev[k] = ck.w_elem(threadIdx.x + 256 * k);
+    if (ev[k] >= 0) {
+      g[k] = *reinterpret_cast<const float4*>(G + ev[k]);
+      m[k] = *reinterpret_cast<const float4*>(M + ev[k]);
     }
   }
   float ss = 0.f;
 #pragma unroll
   for (int k = 0; k < kMuonV; ++k) {
-    const int v = threadIdx.x + 256 * k;
-    if (v < ck.n4) {
-      const float u0 = muon_mom(g[k].x, m[k].x, mu), u1 = muon_mom(g[k].y, m[k].y, mu);
-      const float u2 = muon_mom(g[k].z, m[k].z, mu), u3 = muon_mom(g[k].w, m[k].w, mu);
-      M4[v] = m[k];
-      ss = fmaf(u0, u0, ss);
-      ss = fmaf(u1, u1, ss);
-      ss = fmaf(u2, u2, ss);
-      ss = fmaf(u3, u3, ss);
-      if (a.x0_fused) {
-        T* X = a.ns + ck.mt.x_off[0];
-        const int e = ck.e0 + 4 * v;
-        if (!ck.mt.tr) {
-          store4(X + e, make_float4(u0, u1, u2, u3));
-        } else {  // the 4 elements share a row of W: 4 entries of a column of X
-          const int x0 = ck.xi(e);
-          X[x0] = Elem<T>::from_f(u0);
-          X[x0 + ck.mt.c] = Elem<T>::from_f(u1);
-          X[x0 + 2 * ck.mt.c] = Elem<T>::from_f(u2);
-          X[x0 + 3 * ck.mt.c] = Elem<T>::from_f(u3);
-        }
+    if (ev[k] < 0) continue;
+    const float u0 = muon_mom(g[k].x, m[k].x, mu), u1 = muon_mom(g[k].y, m[k].y, mu);
+    const float u2 = muon_mom(g[k].z, m[k].z, mu), u3 = muon_mom(g[k].w, m[k].w, mu);
+    *reinterpret_cast<float4*>(M + ev[k]) = m[k];
+    ss = fmaf(u0, u0, ss);
+    ss = fmaf(u1, u1, ss);
+    ss = fmaf(u2, u2, ss);
+    ss = fmaf(u3, u3, ss);
+    if (a.x0_fused) {
+      if (!ck.mt.tr) {
+        store4(X + ev[k], make_float4(u0, u1, u2, u3));
+      } else {
+        const int q = threadIdx.x + 256 * k, r = q >> 5, c = 4 * (q & 31);
+        st[r][c] = Elem<T>::from_f(u0);
+        st[r][c + 1] = Elem<T>::from_f(u1);
+        st[r][c + 2] = Elem<T>::from_f(u2);
+        st[r][c + 3] = Elem<T>::from_f(u3);
       }
+    }
+  }
+  if (a.x0_fused && ck.mt.tr) {  // block-uniform
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < kMuonV; ++k) {
+      const int p = threadIdx.x + 256 * k, xo = ck.x_piece(p);
+      if (xo < 0) continue;
+      const int jj = p >> 3, i4 = 4 * (p & 7);
+      store4(X + xo, make_float4(Elem<T>::to_f(st[i4][jj]), Elem<T>::to_f(st[i4 + 1][jj]),
+                                 Elem<T>::to_f(st[i4 + 2][jj]), Elem<T>::to_f(st[i4 + 3][jj])));
     }
   }
   double s = (double)ss;
@@ -1463,8 +1500,9 @@ __global__ void __launch_bounds__(256) k_muon_momentum(MuonArgs<T> a) {
   }
 }
 
-// X0 = U / max(||U||_F, 1e-7), transposed when rows > cols.  Chunks in
-// reverse order: the momentum pass's last chunks are still in L2.
+// X0 = U / max(||U||_F, 1e-7), transposed when rows > cols (element by
+// element: this pass serves the fp32 mode).  Chunks in reverse order: the
+// momentum pass's last chunks are still in L2.
 template <typename T>
 __global__ void __launch_bounds__(256) k_muon_x0(MuonArgs<T> a) {
   pdl_trigger();
@@ -1476,15 +1514,16 @@ __global__ void __launch_bounds__(256) k_muon_x0(MuonArgs<T> a) {
     if (threadIdx.x == 0) inv_s = inv;
   }
   const float mu = a.mu;
-  const float4* G4 = reinterpret_cast<const float4*>(a.grads + ck.mt.w_off + ck.e0);
-  const float4* M4 = reinterpret_cast<const float4*>(a.mom + ck.mt.w_off + ck.e0);
+  const float* G = a.grads + ck.mt.w_off;
+  const float* M = a.mom + ck.mt.w_off;
   float4 g[kMuonV], m[kMuonV];
+  int ev[kMuonV];
 #pragma unroll
   for (int k = 0; k < kMuonV; ++k) {
-    const int v = threadIdx.x + 256 * k;
-    if (v < ck.n4) {
-      g[k] = __ldcs(G4 + v);
-      m[k] = M4[v];
+    ev[k] = ck.w_elem(threadIdx.x + 256 * k);
+    if (ev[k] >= 0) {
+      g[k] = __ldcs(reinterpret_cast<const float4*>(G + ev[k]));
+      m[k] = *reinterpret_cast<const float4*>(M + ev[k]);
     }
   }
   __syncthreads();
@@ -1492,65 +1531,76 @@ __global__ void __launch_bounds__(256) k_muon_x0(MuonArgs<T> a) {
   T* X = a.ns + ck.mt.x_off[0];
 #pragma unroll
   for (int k = 0; k < kMuonV; ++k) {
-    const int v = threadIdx.x + 256 * k;
-    if (v < ck.n4) {
-      const float4 u = make_float4(((1.f - mu) * g[k].x + mu * m[k].x) * inv, ((1.f - mu) * g[k].y + mu * m[k].y) * inv,
-                                   ((1.f - mu) * g[k].z + mu * m[k].z) * inv, ((1.f - mu) * g[k].w + mu * m[k].w) * inv);
-      const int e = ck.e0 + 4 * v;
-      if (!ck.mt.tr) {
-        store4(X + e, u);
-      } else {  // the 4 elements share a row of W: 4 entries of a column of X
-        const int x0 = ck.xi(e);
-        X[x0] = Elem<T>::from_f(u.x);
-        X[x0 + ck.mt.c] = Elem<T>::from_f(u.y);
-        X[x0 + 2 * ck.mt.c] = Elem<T>::from_f(u.z);
-        X[x0 + 3 * ck.mt.c] = Elem<T>::from_f(u.w);
-      }
+    const int e = ev[k];
+    if (e < 0) continue;
+    const float4 u = make_float4(((1.f - mu) * g[k].x + mu * m[k].x) * inv, ((1.f - mu) * g[k].y + mu * m[k].y) * inv,
+                                 ((1.f - mu) * g[k].z + mu * m[k].z) * inv, ((1.f - mu) * g[k].w + mu * m[k].w) * inv);
+    if (!ck.mt.tr) {
+      store4(X + e, u);
+    } else {  // the 4 elements share a row i of W: entries (j .. j + 3, i) of X
+      const int i = e / ck.mt.cols, j = e - i * ck.mt.cols;
+      const int x0 = j * ck.mt.c + i;
+      X[x0] = Elem<T>::from_f(u.x);
+      X[x0 + ck.mt.c] = Elem<T>::from_f(u.y);
+      X[x0 + 2 * ck.mt.c] = Elem<T>::from_f(u.z);
+      X[x0 + 3 * ck.mt.c] = Elem<T>::from_f(u.w);
     }
   }
 }
 
-// W <- W - lr wd W; W <- W - lr scale O, O = the final X (transposed back)
+// W <- W - lr wd W; W <- W - lr scale O, O = the final X (transposed back: a
+// transposed matrix's tile reads whole row segments of X into shared memory)
 template <typename T>
 __global__ void __launch_bounds__(256) k_muon_apply(MuonArgs<T> a) {
   pdl_trigger();
   pdl_wait();
   const MuonChunk<T> ck(a, blockIdx.x);
   const float lr = ck.mt.lr, wd = a.mem[ck.mt.member].wd, sc = ck.mt.scale;
-  const T* X = a.ns + ck.mt.x_off[a.x_final];
-  float4* P4 = reinterpret_cast<float4*>(a.params + ck.mt.w_off + ck.e0);
+  const T* X = a.ns + (a.x_final ? ck.mt.x_off[1] : ck.mt.x_off[0]);  // no runtime index into the record
+  float* P = a.params + ck.mt.w_off;
+  __shared__ MuonStage<T> st;
+  if (ck.mt.tr) {  // block-uniform
+#pragma unroll
+    for (int k = 0; k < kMuonV; ++k) {
+      const int p = threadIdx.x + 256 * k, xo = ck.x_piece(p);
+      if (xo < 0) continue;
+      const float4 v = load4f(X + xo);
+      const int jj = p >> 3, i4 = 4 * (p & 7);
+      st[i4][jj] = Elem<T>::from_f(v.x);
+      st[i4 + 1][jj] = Elem<T>::from_f(v.y);
+      st[i4 + 2][jj] = Elem<T>::from_f(v.z);
+      st[i4 + 3][jj] = Elem<T>::from_f(v.w);
+    }
+    __syncthreads();
+  }
   float4 p[kMuonV], x[kMuonV];
+  int ev[kMuonV];
 #pragma unroll
   for (int k = 0; k < kMuonV; ++k) {
-    const int v = threadIdx.x + 256 * k;
-    if (v < ck.n4) {
-      p[k] = P4[v];
-      const int e = ck.e0 + 4 * v;
-      if (!ck.mt.tr) {
-        x[k] = load4f(X + e);
-      } else {
-        const int x0 = ck.xi(e);
-        x[k] = make_float4(Elem<T>::to_f(X[x0]), Elem<T>::to_f(X[x0 + ck.mt.c]), Elem<T>::to_f(X[x0 + 2 * ck.mt.c]),
-                           Elem<T>::to_f(X[x0 + 3 * ck.mt.c]));
-      }
+    const int q = threadIdx.x + 256 * k, r = q >> 5, c = 4 * (q & 31);
+    ev[k] = ck.w_elem(q);
+    p[k] = x[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (ev[k] >= 0) {
+      p[k] = *reinterpret_cast<const float4*>(P + ev[k]);
+      x[k] = ck.mt.tr ? make_float4(Elem<T>::to_f(st[r][c]), Elem<T>::to_f(st[r][c + 1]),
+                                    Elem<T>::to_f(st[r][c + 2]), Elem<T>::to_f(st[r][c + 3]))
+                      : load4f(X + ev[k]);
     }
   }
 #pragma unroll
   for (int k = 0; k < kMuonV; ++k) {
-    const int v = threadIdx.x + 256 * k;
-    if (v < ck.n4) {
-      float4 q = p[k];
-      q.x = q.x - lr * wd * q.x;
-      q.y = q.y - lr * wd * q.y;
-      q.z = q.z - lr * wd * q.z;
-      q.w = q.w - lr * wd * q.w;
-      q.x = q.x - lr * sc * x[k].x;
-      q.y = q.y - lr * sc * x[k].y;
-      q.z = q.z - lr * sc * x[k].z;
-      q.w = q.w - lr * sc * x[k].w;
-      P4[v] = q;
-      if (a.wq_out) store4(a.wq_out + ck.mt.w_off + ck.e0 + 4 * v, q);
-    }
+    if (ev[k] < 0) continue;
+    float4 q = p[k];
+    q.x = q.x - lr * wd * q.x;
+    q.y = q.y - lr * wd * q.y;
+    q.z = q.z - lr * wd * q.z;
+    q.w = q.w - lr * wd * q.w;
+    q.x = q.x - lr * sc * x[k].x;
+    q.y = q.y - lr * sc * x[k].y;
+    q.z = q.z - lr * sc * x[k].z;
+    q.w = q.w - lr * sc * x[k].w;
+    *reinterpret_cast<float4*>(P + ev[k]) = q;
+    if (a.wq_out) store4(a.wq_out + ck.mt.w_off + ev[k], q);
   }
 }
 

@@ -84,8 +84,8 @@ struct tabpack {
 
   // Muon for the hidden-layer weights (pack_set_muon): one MuonMat per (member,
   // hidden layer), its X0, X1, A, Bm in the Newton-Schulz arena `ns` (the
-  // product precision), the flat list of kMuonChunk-element chunks of the
-  // active members' matrices and a sum-of-squares partial per chunk.  The
+  // product precision), the flat list of the element chunks (muon_chunks) of
+  // the active members' matrices and a sum-of-squares partial per chunk.  The
   // momentum buffers are the AdamW first-moment arena (AdamW skips these
   // matrices).
   bool muon = false;
@@ -567,7 +567,7 @@ tp_status build_schedule(tabpack* h) {
     for (size_t j = 0; j < h->mmats.size(); ++j) {
       MuonMat& mt = h->mmats[j];
       mt.chunk0 = (int32_t)cm.size();
-      mt.n_chunks = h->active[mt.member] ? (int32_t)ceil_div((int64_t)mt.rows * mt.cols, kMuonChunk) : 0;
+      mt.n_chunks = h->active[mt.member] ? (int32_t)muon_chunks(mt) : 0;
       for (int k = 0; k < mt.n_chunks; ++k) cm.push_back((int32_t)j);
     }
     TP_CUDA(h, cudaMemcpy(h->mmats_dev, h->mmats.data(), sizeof(MuonMat) * h->mmats.size(), cudaMemcpyHostToDevice));
@@ -1601,7 +1601,7 @@ tp_status pack_set_muon(tabpack_t* h, const float* lr_muon, float momentum, int3
         mt.a_off = take((int64_t)mt.r * mt.r);
         mt.bm_off = take((int64_t)mt.r * mt.r);
         mt.scale = (float)std::sqrt(std::max(1.0, (double)mt.rows / (double)real_cols));
-        n_chunks += ceil_div((int64_t)mt.rows * mt.cols, kMuonChunk);
+        n_chunks += muon_chunks(mt);
         h->mmats.push_back(mt);
       }
     TP_CUDA(h, cudaMalloc(&h->ns, h->elem * (size_t)std::max<int64_t>(off, 128)));

@@ -307,4 +307,14 @@ __host__ __device__ constexpr int head_split(int w, int d_out) {
 }
 __host__ __device__ constexpr int64_t ceil_div(int64_t x, int64_t a) { return (x + a - 1) / a; }
 
+// The element chunks of a Muon matrix: kMuonChunk consecutive elements of W,
+// or for a transposed one (tr) a kMuonTileR x kMuonTileC tile of W, so that
+// the element kernels can move its X rows (W's columns) as whole segments.
+constexpr int kMuonTileR = 32, kMuonTileC = 128;
+static_assert(kMuonTileR * kMuonTileC == kMuonChunk, "a tile is one chunk");
+__host__ __device__ constexpr int64_t muon_chunks(const MuonMat& mt) {
+  return mt.tr ? ceil_div(mt.rows, kMuonTileR) * ceil_div(mt.cols, kMuonTileC)
+               : ceil_div((int64_t)mt.rows * mt.cols, kMuonChunk);
+}
+
 }  // namespace tp
