@@ -864,6 +864,143 @@ __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
   }
 }
 
+// ------------------------------------------ one-output head, one pass (bf16)
+// The head of a one-output task (binary or regression) for one member on one
+// 64-row block, with H_L read once.  The block's 256 threads form S = 256 / T
+// row sets of T threads (T = w / 8 rounded up to a power of two, at least
+// 32); thread t of a set owns the 8-column group t, keeps its head weights
+// and its partial weight gradient in registers, and walks the set's rows
+// kOneRows at a time with the next rows' 16-byte loads in flight:
+//   1. partial logits of the rows, summed over the warp by shuffles and over
+//      the set's warps in warp order through shared memory, bias added; one
+//      thread per row takes its loss and dlogit;
+//   2. dZ of the last hidden layer = dlogit W_h [H > 0] / (1 - p) stored in
+//      bf16, and dW_h += dlogit H.
+// The sets' partials are added in set order, so each block writes one
+// partial of dW_h, db_h and the loss (rows in order), the layout k_head
+// writes for k_head_reduce.  Widths up to 2048.
+constexpr int kOneRows = 8;
+
+__global__ void __launch_bounds__(256, 2) k_head_one(HeadArgs<__nv_bfloat16> g) {
+  pdl_trigger();
+  pdl_wait();
+  const HeadJob jb = g.jobs[blockIdx.x];
+  const int r0 = jb.blk * kHeadRows;
+  if (r0 >= g.B_pad) return;
+  const MemberDev md = g.mem[jb.member];
+  const int w = md.w, ldh = jb.h_ld, ng = w >> 3;
+  int T = 32;
+  while (T < ng) T <<= 1;
+  const int S = 256 / T, set = threadIdx.x / T, t = threadIdx.x % T;
+  const int rows_set = kHeadRows / S, n_steps = rows_set / kOneRows, wpset = T >> 5;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const bool has = t < ng;
+  const int col = 8 * t;
+  __shared__ float zp[8][kOneRows];
+  __shared__ float dls[8][kOneRows];
+  __shared__ float dlrow[kHeadRows], lrow[kHeadRows];
+  __shared__ __align__(16) float red[8 * 256];  // [S][w]: S * w <= 8 * T * S = 2048
+  const __nv_bfloat16* __restrict__ H = g.act + jb.h_off + (int64_t)(r0 + set * rows_set) * ldh + col;
+  __nv_bfloat16* __restrict__ dZ = g.dz + jb.dz_off + (int64_t)(r0 + set * rows_set) * w + col;
+  const float bias = g.params[jb.b_off];
+  const float invB = 1.f / (float)g.B;
+  const int32_t* idx = g.dyn ? g.dyn->idx : g.idx;
+  const void* yv = g.dyn ? g.dyn->y : g.y;
+  float Wr[8], a[8];
+  if (has) load8(g.params + jb.w_off + col, Wr);
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    if (!has) Wr[k] = 0.f;
+    a[k] = 0.f;
+  }
+  uint4 cur[kOneRows], nxt[kOneRows];
+#pragma unroll
+  for (int u = 0; u < kOneRows; ++u) {
+    cur[u] = has ? *reinterpret_cast<const uint4*>(H + (int64_t)u * ldh) : make_uint4(0u, 0u, 0u, 0u);
+    nxt[u] = make_uint4(0u, 0u, 0u, 0u);
+  }
+  for (int st = 0; st < n_steps; ++st) {
+    if (has && st + 1 < n_steps)
+#pragma unroll
+      for (int u = 0; u < kOneRows; ++u)
+        nxt[u] = *reinterpret_cast<const uint4*>(H + (int64_t)((st + 1) * kOneRows + u) * ldh);
+    // 1. logits of the set's kOneRows rows
+    float p[kOneRows];
+#pragma unroll
+    for (int u = 0; u < kOneRows; ++u) {
+      const __nv_bfloat16* b = reinterpret_cast<const __nv_bfloat16*>(&cur[u]);
+      float s = 0.f;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) s = fmaf(__bfloat162float(b[k]), Wr[k], s);
+      p[u] = s;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+      for (int u = 0; u < kOneRows; ++u) p[u] += __shfl_xor_sync(0xffffffffu, p[u], o);
+    if (lane == 0)
+#pragma unroll
+      for (int u = 0; u < kOneRows; ++u) zp[warp][u] = p[u];
+    __syncthreads();
+    if (threadIdx.x < S * kOneRows) {
+      const int s2 = threadIdx.x / kOneRows, u = threadIdx.x % kOneRows;
+      float zz[1] = {0.f};
+      for (int v = 0; v < wpset; ++v) zz[0] += zp[s2 * wpset + v][u];
+      zz[0] += bias;
+      const int rl = s2 * rows_set + st * kOneRows + u, r = r0 + rl;
+      float dl[1] = {0.f}, loss = 0.f;
+      if (r < g.B) {
+        const int64_t row = idx ? (int64_t)idx[(int64_t)jb.member * g.idx_stride + r] : (int64_t)r;
+        loss = row_loss<1>(g.task, 1, zz, yv, row, invB, dl);
+        g.logits[(int64_t)jb.member * g.B_cap + r] = zz[0];
+      }
+      dls[s2][u] = dl[0];
+      dlrow[rl] = dl[0];
+      lrow[rl] = loss;
+    }
+    __syncthreads();
+    // 2. dZ of the last hidden layer and the weight-gradient partial
+#pragma unroll
+    for (int u = 0; u < kOneRows; ++u) {
+      const float dl = dls[set][u];
+      const __nv_bfloat16* b = reinterpret_cast<const __nv_bfloat16*>(&cur[u]);
+      float o[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const float h = __bfloat162float(b[k]);
+        o[k] = h > 0.f ? (dl * Wr[k]) * md.scale : 0.f;
+        a[k] = fmaf(dl, h, a[k]);
+      }
+      if (has) store8(dZ + (int64_t)(st * kOneRows + u) * w, o);
+    }
+#pragma unroll
+    for (int u = 0; u < kOneRows; ++u) cur[u] = nxt[u];
+  }
+  float* part = g.head_part + jb.part_off;
+  if (S == 1) {
+    if (has) store8(part + col, a);
+  } else {  // the sets' partials added in set order
+    if (has) store8(red + set * w + col, a);
+    __syncthreads();
+    for (int e = threadIdx.x; e < w; e += blockDim.x) {
+      float v = 0.f;
+      for (int s2 = 0; s2 < S; ++s2) v += red[s2 * w + e];
+      part[e] = v;
+    }
+  }
+  // bias and loss partials of the block (rows in order)
+  if (threadIdx.x == 0) {
+    float v = 0.f;
+    for (int rr = 0; rr < kHeadRows; ++rr) v += dlrow[rr];
+    part[w] = v;
+  }
+  if (threadIdx.x == 32) {
+    float v = 0.f;
+    for (int rr = 0; rr < kHeadRows; ++rr) v += lrow[rr];
+    g.loss_part[(int64_t)jb.member * g.n_blk_cap + jb.blk] = v;
+  }
+}
+
 // Sum the per-block head partials (fixed order) into the head gradients and
 // the per-member mean loss; in update mode apply the member's AdamW to the
 // head parameters directly (the gradients are not stored).  Grid: member x
@@ -1147,8 +1284,12 @@ template <typename T>
 void launch_head(cudaStream_t st, const HeadArgs<T>& g, int n_jobs) {
   if (n_jobs <= 0) return;
   if constexpr (std::is_same_v<T, __nv_bfloat16>) {
-    // one output on members wider than 512: the row-per-lane-group kernel
-    // measured faster (the staged block then runs one per SM)
+    // one output on members wider than 512: the one-pass kernel (the staged
+    // block would run one per SM)
+    if (g.d_out == 1 && g.w_max > 512 && g.w_max <= 2048) {
+      launch_pdl(k_head_one, dim3(n_jobs), dim3(256), 0, st, g);
+      return;
+    }
     if (g.stage && !(g.d_out == 1 && g.w_max > 512)) {
       bool done = false;
       switch (head_bucket(g.d_out)) {

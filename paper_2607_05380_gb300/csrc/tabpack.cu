@@ -496,6 +496,10 @@ tp_status build_schedule(tabpack* h) {
       hj.push_back(j);
     }
   }
+  // widest members' blocks first (a block's cost grows with the width), so
+  // that the blocks left for the last wave are the cheapest
+  std::stable_sort(hj.begin(), hj.end(),
+                   [h](const HeadJob& x, const HeadJob& y) { return h->width[x.member] > h->width[y.member]; });
   // element-wise chunks of the active members (init, fp32-mode AdamW)
   std::vector<Chunk> ch;
   for (int s = 0; s < (int)h->segs.size(); ++s) {

@@ -124,6 +124,29 @@ def test_one_step_logits_losses_grads(tp, prec, task, d_out, B):
     assert not problems, problems
 
 
+@pytest.mark.parametrize("task", ["binary", "regression"])
+@pytest.mark.parametrize("B", [256, 200])
+def test_one_output_head_widths(tp, task, B):
+    """The one-pass one-output head (bf16, widest member above 512): members
+    whose 8-column groups fill 32, 64, 128 and 256 threads of a block (widths
+    128, 272, 528, 1040, 1536, 2048; 1 to 8 row sets), a ragged batch whose
+    padded rows share blocks with real ones: one step's logits, losses and
+    gradients against the oracle."""
+    d_in = 70
+    hp = random_pack(6, d_in, 1, seed=23, depth=(1, 2), dropout=(0.0, 0.4))
+    hp["width"] = np.array([2048, 128, 1040, 272, 1536, 528], dtype=np.int32)
+    hp["depth"] = np.array([1, 2, 2, 2, 1, 2], dtype=np.int32)
+    pk, orc = pair(tp, task, d_in, 1, hp, "bf16", 256)
+    X, y = make_data(task, 500, d_in, 1, 3)
+    idx = np.random.default_rng(4).choice(500, B, replace=False).astype(np.int32)
+    Xd, yd, idxd = to_dev(X, y, idx)
+    loss = torch.zeros(6, dtype=torch.float32, device=DEV)
+    pk.forward_backward(Xd, idxd, yd, 2, loss)
+    orc.train_step(X, idx, y, 2, update=False)
+    problems = compare_step(pk, orc, hp, "bf16", loss.cpu().numpy())
+    assert not problems, problems
+
+
 @pytest.mark.parametrize("prec", ["fp32", "bf16"])
 @pytest.mark.parametrize("task,d_out", [("binary", 1), ("multiclass", 7), ("regression", 1)])
 @pytest.mark.parametrize("B", [256, 200])
