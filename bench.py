@@ -38,7 +38,7 @@ METRIC = "member-samples/sec (fwd+bwd+AdamW)"
 # A workload without a capture of the current kernel reports null.
 DRAM_TRAFFIC = {
     ("medium", "k_adamw"): 607.7e6,
-    ("wide", "k_tc_gemm"): 3.186e9,
+    ("wide", "k_tc_gemm"): 2.848e9,
     ("wide", "k_adamw"): 4.020e9,
 }
 UNIT = "member-samples/s"
@@ -465,6 +465,8 @@ def measure(args, tp, torch, dist, dev, name, steps, warmup, world, rank, headli
                    max_batch=B, seed=SEED_INIT, precision=args.precision, stream=stream,
                    fuse_optimizer=args.fuse_optimizer, d_emb=None if emb is None else emb["d_emb"],
                    freq=None if emb is None else emb["freq"])
+    if args.bias_path != "auto" and args.precision == "bf16":
+        pack.debug_bias_path(1 if args.bias_path == "colsums" else 0)
     loss = torch.zeros(wl.m, dtype=torch.float32, device=dev)
     lr_muon = None
     if args.muon:
@@ -651,6 +653,9 @@ def main():
     ap.add_argument("--members", type=int, default=0,
                     help="train only the first N members of the workload (profiling small cases)")
     ap.add_argument("--fuse-optimizer", action="store_true", help="AdamW inside the weight-gradient epilogue")
+    ap.add_argument("--bias-path", default="auto", choices=["auto", "colsums", "column"],
+                    help="bf16: hidden-layer bias gradients from dZ column sums (where the input width is a "
+                         "multiple of 256) or from a bias column; auto = the pack's own choice")
     ap.add_argument("--no-online", action="store_true", help="skip timing the online-ensemble epoch end")
     ap.add_argument("--online-score", default="loss", choices=["loss", "accuracy", "rmse", "auc"],
                     help="ensemble score of the timed online epoch end (auc: binary workloads)")

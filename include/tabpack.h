@@ -344,6 +344,19 @@ tp_status pack_debug_mask_arena(tabpack_t* pack, int32_t member, int32_t layer, 
  * step graphs are dropped.                                                 */
 tp_status pack_debug_gemm_timeout(tabpack_t* pack, double wait_s, int32_t poison);
 
+/* Where the bf16 tensor-core weight-gradient products take each hidden
+ * layer's bias gradient db_j = sum_b dZ[b, j] (Sec. 3.3 backward; the paper
+ * has no counterpart for the choice).  mode 1: for every layer whose input
+ * width is a multiple of 256, from column sums of dZ that the head kernel
+ * and the dgrad epilogues store while they write dZ (this saves a column
+ * tile of the product); mode 0: from a column of ones appended to the
+ * product's input, for every layer; mode -1: the pack's own choice (column
+ * sums when its backward products are tensor-bound: ideal tensor time of
+ * 300 us or more per step).  Both sum dZ as stored in bf16, in fp32.  For
+ * tests and measurements; bf16 mode only (TP_ESTATE otherwise), TP_EINVAL
+ * for another mode.  Synchronises; captured step graphs are dropped.      */
+tp_status pack_debug_bias_path(tabpack_t* pack, int32_t mode);
+
 /* Philox4x32-10 (Salmon et al., SC'11) as the device evaluates it for the
  * dropout masks and the initial values: out[i] = the four words of counter
  * ctr[i] (host uint32 [n, 4]) under key key[i] (host uint32 [n, 2]).  Runs

@@ -36,7 +36,7 @@ SYMBOLS = ["pack_create", "pack_destroy", "pack_set_stream", "pack_train_step", 
            "pack_online_members", "pack_online_ensemble", "pack_online_snapshot", "pack_online_predict",
            "pack_online_last_error", "pack_train_step_stacked", "pack_forward_backward_stacked", "pack_set_muon",
            "pack_debug_muon_dir", "pack_create_emb", "pack_get_emb", "pack_set_emb", "pack_member_emb",
-           "pack_debug_mask_arena", "pack_debug_philox", "pack_debug_gemm_timeout"]
+           "pack_debug_mask_arena", "pack_debug_philox", "pack_debug_gemm_timeout", "pack_debug_bias_path"]
 
 
 class TabpackError(RuntimeError):
@@ -120,6 +120,7 @@ def load_library(path: str = LIB_PATH):
         "pack_debug_mask_arena": (st, [P, i32, i32, i32, P, P]),
         "pack_debug_philox": (st, [P, P, i32, P]),
         "pack_debug_gemm_timeout": (st, [P, ctypes.c_double, i32]),
+        "pack_debug_bias_path": (st, [P, i32]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -354,6 +355,13 @@ class Pack:
         """Wait budget of the tensor-core launches; poison: one forward
         dependency that is never met (tests of the bounded waits)."""
         _check(load_library().pack_debug_gemm_timeout(self._h, float(wait_s), int(bool(poison))), self._h)
+
+    def debug_bias_path(self, mode):
+        """bf16: where the tensor-core weight-gradient products take the
+        bias gradient from -- 1: column sums of dZ for every layer whose
+        input width is a multiple of 256, 0: the bias column everywhere,
+        -1: the pack's own choice."""
+        _check(load_library().pack_debug_bias_path(self._h, int(mode)), self._h)
 
     def debug_activations(self, member, layer):
         out = np.zeros((self._B, int(self.width[member])), dtype=np.float32)

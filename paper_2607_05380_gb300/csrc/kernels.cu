@@ -471,6 +471,8 @@ __global__ void __launch_bounds__(256, DO == 1 ? 3 : 2) k_head(HeadArgs<T> g) {
   __shared__ __align__(16) float dlog[kHeadRows][DOP];
   __shared__ float lrow[kHeadRows];
   __shared__ __align__(16) float red[256 * G * DO];  // row-set partials when the rows are split
+  constexpr bool kColSums = std::is_same_v<T, __nv_bfloat16>;  // dZ column sums (tensor-core mode only)
+  __shared__ __align__(16) float redz[kColSums ? 256 * G : 4];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float invB = 1.f / (float)g.B;
 
@@ -517,10 +519,13 @@ __global__ void __launch_bounds__(256, DO == 1 ? 3 : 2) k_head(HeadArgs<T> g) {
   const int rows_per_set = kHeadRows / S;
   T* __restrict__ dZ = g.dz + jb.dz_off + (int64_t)r0 * w;
   float* part = g.head_part + jb.part_off;
+  float* dbp = kColSums && g.dbp && jb.colsum ? g.dbp + jb.dz_off / 32 + (int64_t)jb.blk * w : nullptr;
   for (int u = threadIdx.x; u < n_cg * S; u += blockDim.x) {
     const int cg = u % n_cg, set = u / n_cg;
     const int col = G * cg;
-    float Wr[DO][G], a[DO][G];
+    float Wr[DO][G], a[DO][G], cz[G];
+#pragma unroll
+    for (int k = 0; k < G; ++k) cz[k] = 0.f;
 #pragma unroll
     for (int c = 0; c < DO; ++c) {
       if (c < d_out) loadG<G>(Wh + (int64_t)c * w + col, Wr[c]);
@@ -565,7 +570,11 @@ __global__ void __launch_bounds__(256, DO == 1 ? 3 : 2) k_head(HeadArgs<T> g) {
           a[c][k] = fmaf(dl[c], h[k], a[c][k]);
         }
 #pragma unroll
-      for (int k = 0; k < G; ++k) s[k] = h[k] > 0.f ? s[k] * md.scale : 0.f;
+      for (int k = 0; k < G; ++k) {
+        s[k] = h[k] > 0.f ? s[k] * md.scale : 0.f;
+        if constexpr (kColSums)
+          if (dbp) cz[k] += __bfloat162float(__float2bfloat16_rn(s[k]));  // dZ as stored
+      }
       storeG<G>(dZ + (int64_t)rr * w + col, s);
       }
     }
@@ -573,10 +582,12 @@ __global__ void __launch_bounds__(256, DO == 1 ? 3 : 2) k_head(HeadArgs<T> g) {
 #pragma unroll
       for (int c = 0; c < DO; ++c)
         if (c < d_out) storeG<G>(part + (int64_t)c * w + col, a[c]);
+      if (dbp) storeG<G>(dbp + col, cz);
     } else {  // n_cg * S <= 256: one (column group, row set) per thread
 #pragma unroll
       for (int c = 0; c < DO; ++c)
         if (c < d_out) storeG<G>(&red[((set * DO + c) * n_cg + cg) * G], a[c]);
+      if constexpr (kColSums) storeG<G>(&redz[(set * n_cg + cg) * G], cz);
     }
   }
   if (S > 1) {  // the block's partial: row sets added in order
@@ -588,6 +599,13 @@ __global__ void __launch_bounds__(256, DO == 1 ? 3 : 2) k_head(HeadArgs<T> g) {
       for (int set = 0; set < S; ++set) v += red[((set * DO + c) * n_cg + cg) * G + kk];
       part[e] = v;
     }
+    if (dbp)
+      for (int e = threadIdx.x; e < w; e += blockDim.x) {
+        const int cg = e / G, kk = e - cg * G;
+        float v = 0.f;
+        for (int set = 0; set < S; ++set) v += redz[(set * n_cg + cg) * G + kk];
+        dbp[e] = v;
+      }
   }
   // bias partial and loss partial of the block (rows in order)
   if (threadIdx.x < d_out) {
@@ -768,12 +786,15 @@ __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
   const int rows_per_set = kHeadRows / S;
   __nv_bfloat16* __restrict__ dZ = g.dz + jb.dz_off + (int64_t)r0 * w;
   float* part = g.head_part + jb.part_off;
-  float a[DO][4];
+  float* dbp = g.dbp && jb.colsum ? g.dbp + jb.dz_off / 32 + (int64_t)jb.blk * w : nullptr;
+  float a[DO][4], cz[4] = {0.f, 0.f, 0.f, 0.f};
   int cg = 0, set = 0;
   for (int u = threadIdx.x; u < n_cg * S; u += blockDim.x) {
     cg = u % n_cg;
     set = u / n_cg;
     const int col = 4 * cg;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) cz[k] = 0.f;
     float Wr[DO][4];
 #pragma unroll
     for (int c = 0; c < DO; ++c) {
@@ -822,7 +843,10 @@ __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
         }
       __align__(8) __nv_bfloat16 o[4];
 #pragma unroll
-      for (int k = 0; k < 4; ++k) o[k] = __float2bfloat16_rn(h[k] > 0.f ? sacc[k] * md.scale : 0.f);
+      for (int k = 0; k < 4; ++k) {
+        o[k] = __float2bfloat16_rn(h[k] > 0.f ? sacc[k] * md.scale : 0.f);
+        if (dbp) cz[k] += __bfloat162float(o[k]);  // dZ as stored
+      }
       *reinterpret_cast<uint2*>(dZ + (int64_t)rr * w + col) = *reinterpret_cast<const uint2*>(o);
     }
     if (S == 1) {
@@ -830,17 +854,20 @@ __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
       for (int c = 0; c < DO; ++c)
         if (c < d_out)
           *reinterpret_cast<float4*>(part + (int64_t)c * w + col) = make_float4(a[c][0], a[c][1], a[c][2], a[c][3]);
+      if (dbp) *reinterpret_cast<float4*>(dbp + col) = make_float4(cz[0], cz[1], cz[2], cz[3]);
     }
   }
   if (S > 1) {  // one (column group, row set) per thread; sets added in order (the H area is free now)
     __syncthreads();
-    float* red = reinterpret_cast<float*>(Hs);   // [S][DO][w]
+    float* red = reinterpret_cast<float*>(Hs);   // [S][DO][w], then [S][w] of dZ column sums
+    float* redz = red + (int64_t)S * DO * w;     // S (DO + 1) w <= 24 w floats fit in 64 rows of H
     if (threadIdx.x < n_cg * S) {
 #pragma unroll
       for (int c = 0; c < DO; ++c)
         if (c < d_out)
           *reinterpret_cast<float4*>(red + ((int64_t)set * DO + c) * w + 4 * cg) =
               make_float4(a[c][0], a[c][1], a[c][2], a[c][3]);
+      *reinterpret_cast<float4*>(redz + (int64_t)set * w + 4 * cg) = make_float4(cz[0], cz[1], cz[2], cz[3]);
     }
     __syncthreads();
     for (int e = threadIdx.x; e < d_out * w; e += blockDim.x) {
@@ -849,6 +876,12 @@ __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
       for (int st = 0; st < S; ++st) v += red[((int64_t)st * DO + c) * w + k];
       part[e] = v;
     }
+    if (dbp)
+      for (int e = threadIdx.x; e < w; e += blockDim.x) {
+        float v = 0.f;
+        for (int st = 0; st < S; ++st) v += redz[(int64_t)st * w + e];
+        dbp[e] = v;
+      }
   }
   pdl_trigger();
   // bias partial and loss partial of the block (rows in order)
@@ -878,7 +911,8 @@ __global__ void __launch_bounds__(256) k_head_stage(HeadArgs<__nv_bfloat16> g) {
 //      bf16, and dW_h += dlogit H.
 // The sets' partials are added in set order, so each block writes one
 // partial of dW_h, db_h and the loss (rows in order), the layout k_head
-// writes for k_head_reduce.  Widths up to 2048.
+// writes for k_head_reduce, and (dbp) the column sums of its dZ rows.
+// Widths up to 2048.
 constexpr int kOneRows = 8;
 
 __global__ void __launch_bounds__(256, 2) k_head_one(HeadArgs<__nv_bfloat16> g) {
@@ -900,18 +934,20 @@ __global__ void __launch_bounds__(256, 2) k_head_one(HeadArgs<__nv_bfloat16> g) 
   __shared__ float dls[8][kOneRows];
   __shared__ float dlrow[kHeadRows], lrow[kHeadRows];
   __shared__ __align__(16) float red[8 * 256];  // [S][w]: S * w <= 8 * T * S = 2048
+  __shared__ __align__(16) float redz[8 * 256]; // the same for the column sums of dZ
   const __nv_bfloat16* __restrict__ H = g.act + jb.h_off + (int64_t)(r0 + set * rows_set) * ldh + col;
   __nv_bfloat16* __restrict__ dZ = g.dz + jb.dz_off + (int64_t)(r0 + set * rows_set) * w + col;
   const float bias = g.params[jb.b_off];
   const float invB = 1.f / (float)g.B;
   const int32_t* idx = g.dyn ? g.dyn->idx : g.idx;
   const void* yv = g.dyn ? g.dyn->y : g.y;
-  float Wr[8], a[8];
+  float Wr[8], a[8], cz[8];
   if (has) load8(g.params + jb.w_off + col, Wr);
 #pragma unroll
   for (int k = 0; k < 8; ++k) {
     if (!has) Wr[k] = 0.f;
     a[k] = 0.f;
+    cz[k] = 0.f;
   }
   uint4 cur[kOneRows], nxt[kOneRows];
 #pragma unroll
@@ -971,21 +1007,44 @@ __global__ void __launch_bounds__(256, 2) k_head_one(HeadArgs<__nv_bfloat16> g) 
         o[k] = h > 0.f ? (dl * Wr[k]) * md.scale : 0.f;
         a[k] = fmaf(dl, h, a[k]);
       }
-      if (has) store8(dZ + (int64_t)(st * kOneRows + u) * w, o);
+      uint4 pz;
+      __nv_bfloat162* pb = reinterpret_cast<__nv_bfloat162*>(&pz);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) pb[k] = __floats2bfloat162_rn(o[2 * k], o[2 * k + 1]);
+      if (has) *reinterpret_cast<uint4*>(dZ + (int64_t)(st * kOneRows + u) * w) = pz;
+      if (jb.colsum) {  // column sums of dZ as stored
+        const uint32_t* pw = reinterpret_cast<const uint32_t*>(&pz);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          cz[2 * k] += __uint_as_float(pw[k] << 16);
+          cz[2 * k + 1] += __uint_as_float(pw[k] & 0xFFFF0000u);
+        }
+      }
     }
 #pragma unroll
     for (int u = 0; u < kOneRows; ++u) cur[u] = nxt[u];
   }
   float* part = g.head_part + jb.part_off;
+  float* dbp = g.dbp && jb.colsum ? g.dbp + jb.dz_off / 32 + (int64_t)jb.blk * w : nullptr;
   if (S == 1) {
-    if (has) store8(part + col, a);
+    if (has) {
+      store8(part + col, a);
+      if (dbp) store8(dbp + col, cz);
+    }
   } else {  // the sets' partials added in set order
-    if (has) store8(red + set * w + col, a);
+    if (has) {
+      store8(red + set * w + col, a);
+      store8(redz + set * w + col, cz);
+    }
     __syncthreads();
     for (int e = threadIdx.x; e < w; e += blockDim.x) {
-      float v = 0.f;
-      for (int s2 = 0; s2 < S; ++s2) v += red[s2 * w + e];
+      float v = 0.f, vz = 0.f;
+      for (int s2 = 0; s2 < S; ++s2) {
+        v += red[s2 * w + e];
+        vz += redz[s2 * w + e];
+      }
       part[e] = v;
+      if (dbp) dbp[e] = vz;
     }
   }
   // bias and loss partials of the block (rows in order)

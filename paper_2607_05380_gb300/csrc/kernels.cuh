@@ -71,6 +71,9 @@ struct HeadArgs {
   int32_t w_max;          // widest member (bf16: shared-memory size of the staged head kernel)
   int32_t stage;          // bf16: 1 = the staged head kernel where it fits in shared memory
   int* err;               // device error word for a bounded wait that runs out (NULL: none)
+  float* dbp;             // bf16 tensor-core mode: the column sums of dZ_L as stored (bf16) over
+                          // each 64-row block (element dz_off / 32 + blk * w + j) of the jobs
+                          // with colsum set, from which the weight-gradient tiles take db
 };
 
 // Staged head kernel (bf16): shared memory per block for members up to w_max

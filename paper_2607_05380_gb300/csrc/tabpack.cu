@@ -36,6 +36,7 @@ struct tabpack {
   int d_in_pad = 0, ldx = 0, B_cap = 0, n_blk_cap = 0, Lmax = 0;
   cudaStream_t st = nullptr;
   bool bf16 = true;
+  bool bias_colsums = false;  // bf16: bias gradients from dZ column sums where bias_from_colsums
   std::vector<int32_t> depth, width;
   std::vector<float> dropout, lr, wd;
   std::vector<std::array<int64_t, kMaxDepth + 1>> W_off, b_off;
@@ -54,6 +55,10 @@ struct tabpack {
   bool fuse_adamw = false;  // bf16: AdamW in the wgrad epilogue (else a stand-alone pass)
   void *xb = nullptr, *act = nullptr, *dz = nullptr;
   float *logits = nullptr, *head_part = nullptr, *loss_part = nullptr, *loss_last = nullptr;
+  // bf16: column sums of dZ over 32-row groups (64-row blocks for the last
+  // hidden layer's, written by the head), element dz_off / 32 + g * w + j,
+  // for the layers whose bias gradient comes from them (bias_from_colsums)
+  float* dbp = nullptr;
   int32_t* t_dev = nullptr;
   float2* bias_corr = nullptr;
   uint8_t* active_dev = nullptr;
@@ -261,6 +266,21 @@ void drop_graphs(tabpack* h);
 void free_predict(tabpack* h);
 
 // ------------------------------------------------------------------ layout
+// Column sums of dZ save a weight-gradient column tile of every layer whose
+// input width is a multiple of 256, but add work to the head and to the
+// dgrad epilogues, which lie on the backward launch's dependency chain.
+// They pay where the backward is bound by tensor throughput, taken as an
+// ideal backward tensor time (nominal 2 PFLOP/s) of 300 us or more.
+bool auto_bias_colsums(const tabpack* h) {
+  if (!h->bf16) return false;
+  double flops = 0.0;
+  for (int i = 0; i < h->cfg.m; ++i) {
+    const double w = h->width[i], L = h->depth[i];
+    flops += 2.0 * h->B_cap * (w * h->in0_pad[i] + 2.0 * (L - 1.0) * w * w);
+  }
+  return flops / 2.0e15 >= 300e-6;
+}
+
 tp_status build_layout(tabpack* h) {
   const auto& c = h->cfg;
   const int m = c.m;
@@ -281,6 +301,7 @@ tp_status build_layout(tabpack* h) {
     }
   h->B_cap = (int)round_up(c.max_batch, kRowTile);
   h->n_blk_cap = h->B_cap / kHeadRows;
+  h->bias_colsums = auto_bias_colsums(h);
   h->W_off.resize(m);
   h->b_off.resize(m);
   h->act_off.resize(m);
@@ -488,6 +509,7 @@ tp_status build_schedule(tabpack* h) {
       j.blk = b;
       j.h_ld = ldh_of(h, i);
       j.split = head_split(h->width[i], h->cfg.d_out);
+      j.colsum = h->bias_colsums && bias_from_colsums(L == 1 ? h->in0_pad[i] : h->width[i]) ? 1 : 0;
       j.h_off = h->act_off[i][L - 1];
       j.dz_off = h->dz_off[i][L - 1];
       j.w_off = h->W_off[i][L];
@@ -601,6 +623,7 @@ tp_status build_schedule(tabpack* h) {
     lay.xb = h->xb;
     lay.act = h->act;
     lay.dz = h->dz;
+    lay.bias_colsums = h->bias_colsums;
     lay.mask_off = h->mask_words > 0 ? &h->mask_off : nullptr;
     lay.muon = h->muon ? &h->mmats : nullptr;
     lay.ns = h->ns;
@@ -656,6 +679,7 @@ tp_status alloc_all(tabpack* h) {
   TP_TRY(dalloc(h, &h->dz, h->elem * h->dz_elems));
   TP_TRY(dalloc(h, &h->logits, sizeof(float) * (size_t)m * h->B_cap * h->cfg.d_out));
   TP_TRY(dalloc(h, &h->head_part, sizeof(float) * h->head_part_elems));
+  if (h->bf16) TP_TRY(dalloc(h, &h->dbp, sizeof(float) * (size_t)(h->dz_elems / 32 + 32)));
   TP_TRY(dalloc(h, &h->loss_part, sizeof(float) * (size_t)m * h->n_blk_cap));
   TP_TRY(dalloc(h, &h->loss_last, sizeof(float) * m));
   TP_TRY(dalloc(h, &h->t_dev, sizeof(int32_t) * m));
@@ -896,6 +920,7 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
   hg.w_max = *std::max_element(h->width.begin(), h->width.end());
   hg.stage = h->bf16 ? 1 : 0;
   hg.err = h->bf16 && h->tc.enabled ? h->tc.err_dev : nullptr;
+  hg.dbp = h->bf16 ? h->dbp : nullptr;   // the tensor-core backward sums them into the bias gradients
   launch_head<T>(h->st, hg, h->n_head_jobs);
   TP_LAUNCHED(h);
   h->launches++;
@@ -927,8 +952,8 @@ tp_status run_step(tabpack* h, const float* X, int64_t n_rows, const int32_t* id
   const AdamDev ad = adam_dev(h, wq_next);
   if (h->bf16) {
     prof_begin(h, TP_PH_BWD, &slot);
-    TP_TRY(tc_run_bwd(plan, h->st, B, B_pad, h->wcur, h->mem_dev, h->act, h->dz, h->grads, fused ? 1 : 0, ad,
-                      h->err));
+    TP_TRY(tc_run_bwd(plan, h->st, B, B_pad, h->wcur, h->mem_dev, h->act, h->dz, h->grads, h->dbp, fused ? 1 : 0,
+                      ad, h->err));
     TP_LAUNCHED(h);
     h->launches++;
     prof_end(h, slot, 1, TP_PH_BWD);
@@ -1130,6 +1155,7 @@ tp_status ensure_stacked(tabpack* h) {
     lay.xb = h->xbs;
     lay.act = h->act;
     lay.dz = h->dz;
+    lay.bias_colsums = h->bias_colsums;
     lay.mask_off = h->mask_words > 0 ? &h->mask_off : nullptr;
     lay.xb_stride = h->xb_elems;
     TP_CUDA(h, cudaStreamSynchronize(h->st));
@@ -1825,6 +1851,16 @@ tp_status pack_debug_gemm_timeout(tabpack_t* h, double wait_s, int32_t poison) {
   h->graphs.clear();
   if (poison) TP_TRY(tc_debug_poison(h->tc, h->st, h->err));
   return TP_OK;
+}
+
+tp_status pack_debug_bias_path(tabpack_t* h, int32_t mode) {
+  if (!h) return fail(nullptr, TP_EINVAL, "null pack");
+  if (mode < -1 || mode > 1) return fail(h, TP_EINVAL, "mode must be -1, 0 or 1");
+  if (!h->bf16) return fail(h, TP_ESTATE, "the bias path choice exists in bf16 mode only");
+  TP_TRY(sync_check(h));
+  h->bias_colsums = mode < 0 ? auto_bias_colsums(h) : mode == 1;
+  h->s_stale = true;
+  return build_schedule(h);
 }
 
 tp_status pack_debug_philox(const uint32_t* ctr, const uint32_t* key, int32_t n, uint32_t* out) {

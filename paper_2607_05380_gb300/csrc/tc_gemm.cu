@@ -27,7 +27,10 @@
 //              the fused epilogue of the product kind:
 //                kFwd   z = acc + b; h = dropout(relu(z)) / (1 - p)   -> bf16
 //                kDgrad dz_prev = acc * [H_prev > 0] / (1 - p)          -> bf16
-//                kWgrad dW, db = acc (store) or AdamW(p, m, v; dW, db) with
+//                       (and, where the layer's wgrad wants them, its column
+//                       sums over each warp's 32 rows)
+//                kWgrad dW, db = acc (the bias column) or the sum of dZ's
+//                       column sums (store), or AdamW(p, m, v; dW, db) with
 //                       the fp32 master, the moments and the bf16 copy
 // Ragged K (member widths that are multiples of 16 but not of 64) issues
 // only the K=16 steps that exist; out-of-range operand rows and columns are
@@ -128,6 +131,7 @@ struct TcArgs {
   __nv_bfloat16* ns;   // Newton-Schulz arena (kNs launches)
   const float* ns_scale;  // per Muon matrix: 1 / |U|_F (kNs launches)
   uint64_t wait_ns;    // budget of every wait that can give up (TcPlan::wait_ns)
+  float* dbp;          // column-sum partials of dZ (kDgrad writes them, kWgrad reads them)
 };
 
 // ------------------------------------------------------------ PTX helpers
@@ -162,7 +166,8 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // A wait that gives up records its site code in the error word (the first
 // one wins): 1 producer stage empty, 3 producer dependency, 5 MMA
 // accumulator free, 6 MMA stage full, 7 epilogue accumulator full, 10 final
-// copy drain, 12 final MMA drain, 8 epilogue publish slot, 9 publisher.
+// copy drain, 12 final MMA drain, 8 epilogue publish slot, 9 publisher,
+// 13 epilogue Newton-Schulz dependency, 14 epilogue bias-partial dependency.
 // The MMA and epilogue waits (5, 6, 7, 8) wait on another role of the same
 // CTA and take twice the budget of the producer's, the publisher's (9) four
 // times, so a stalled dependency is reported as its own site.
@@ -228,6 +233,37 @@ __device__ __noinline__ bool dep_wait(const int* p, int n, int need, volatile in
   }
   __syncwarp();
   return __all_sync(0xffffffffu, mine);
+}
+
+// Column sums of a warp's 32 x 32 chunk (lane = row, c[j] = column j):
+// halving exchanges (16 + 8 + 4 + 2 + 1 shuffles), after which lane l
+// holds column l's sum in c[0].  The order of the additions is fixed.
+template <int W>
+__device__ __forceinline__ void colsum_halve(float (&c)[32], int lane) {
+  const bool up = (lane & W) != 0;
+#pragma unroll
+  for (int k = 0; k < W; ++k) {
+    const float keep = up ? c[W + k] : c[k];
+    const float send = up ? c[k] : c[W + k];
+    c[k] = keep + __shfl_xor_sync(0xffffffffu, send, W);
+  }
+}
+__device__ __forceinline__ float colsum32(float (&c)[32], int lane) {
+  colsum_halve<16>(c, lane);
+  colsum_halve<8>(c, lane);
+  colsum_halve<4>(c, lane);
+  colsum_halve<2>(c, lane);
+  colsum_halve<1>(c, lane);
+  return c[0];
+}
+
+// p[0] + p[ld] + ... + p[(n - 1) ld], added in that order (kept out of line:
+// inlined, its loop state raised the epilogue's register spills).
+__device__ __noinline__ float sum_strided(const float* p, int n, int ld) {
+  float s = 0.f;
+#pragma unroll 8
+  for (int i = 0; i < n; ++i) s += p[(int64_t)i * ld];
+  return s;
 }
 
 // Bulk prefetch of `bytes` (a multiple of 16; 16-byte aligned address) into L2.
@@ -458,7 +494,7 @@ __device__ __forceinline__ SubTile sub_tile(const TcTile& t, int mi, int B_pad) 
 // the weight columns of a tile a multiple of 8 (n0 a multiple of 16, in_pad of 8).
 __device__ __forceinline__ void prefetch_adam_rows(const TcArgs& g, const TcTile& t, int rank, int e, int lane) {
   const SubTile u = sub_tile(t, rank, g.B_pad);
-  const int cols = min(t.n_len, t.n_real - 1 - t.n0);
+  const int cols = min(t.n_len, (t.db_off >= 0 ? t.n_real : t.n_real - 1) - t.n0);
   if (!u.rows_live || cols <= 0) return;
   constexpr int kR = 128 / kEpiWarps;
   for (int k = lane; k < 3 * kR; k += 32) {
@@ -776,6 +812,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
         for (int s = 0; s < 4; ++s)
           a[s] = need && 8 * s < ncols ? *reinterpret_cast<const uint4*>(p + 8 * s) : make_uint4(0u, 0u, 0u, 0u);
       };
+      // Weight-gradient tiles of column 0: the bias gradient sums dZ's
+      // column-sum partials with plain loads.  Row blocks of dZ written in
+      // this launch are acquired here (their counts were reached before the
+      // tile's operands were loaded, so this does not wait).
+      const bool bias_tile = !kNs && tile.kind == kWgrad && tile.n0 == 0 && half == 0 && g.dbp != nullptr &&
+                             tile.db_off >= 0 && u.rows_live;
+      if (bias_tile && tile.dep >= 0 &&
+          !dep_wait(g.cnt + tile.dep, g.B_pad / kRowTile, tile.dep_need, abort_flag, g.err, 2 * g.wait_ns, 14, lane))
+        break;
       uint4 axn[4];
       if constexpr (kNs) ns_aux(0, axn);
       if (!mbar_wait(&tl->tfull[acc], acc_phase, abort_flag, g.err, 2 * g.wait_ns, 7)) break;
@@ -875,10 +920,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
                 make_float4(__uint_as_float(v[4 * gi]), __uint_as_float(v[4 * gi + 1]),
                             __uint_as_float(v[4 * gi + 2]), __uint_as_float(v[4 * gi + 3]));
           __syncwarp();
-          const int in_pad = tile.n_real - 1;  // a multiple of 8: a group is all weights or starts at the bias
+          // in_pad: a multiple of 8, so a float4 group is all weights or
+          // starts at the bias column (when the bias comes from the ones column)
+          const int in_pad = tile.db_off >= 0 ? tile.n_real : tile.n_real - 1;
           const int gc = lane & 7, rsub = lane >> 3;
           const int col = col0 + 4 * gc;
-          const bool is_w = col < in_pad && col < n_hi, is_b = col == in_pad && col < n_hi;
+          const bool is_w = col < in_pad && col < n_hi;
           const int rbase = u.m0 + 32 * q;
           const int nrows = min(32, m_lim - rbase);
           if (g.update) {
@@ -916,31 +963,36 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
                       make_uint2(pack_bf16x2(P[i].x, P[i].y), pack_bf16x2(P[i].z, P[i].w));
                 }
               }
-            } else if (is_b) {
+            }
+          } else {
+            if (is_w) {
+#pragma unroll
               for (int i = 0; i < 8; ++i) {
                 const int rr = 4 * i + rsub;
                 if (rr >= nrows) break;
-                const float gb = tr[rr * 32 + 4 * (gc ^ (rr & 7))];
-                const int64_t o = tile.aux_off + rbase + rr;
-                float pb = ad.params[o], mb = ad.m[o], vb = ad.v[o];
-                adamw_elem(pb, mb, vb, gb, lr, wd_b, ad.beta1, ad.beta2, ad.eps, ib1, ib2);
-                ad.params[o] = pb;
-                ad.m[o] = mb;
-                ad.v[o] = vb;
-                ad.wq_out[o] = __float2bfloat16_rn(pb);
+                *reinterpret_cast<float4*>(g.grads + tile.c_off + (int64_t)(rbase + rr) * tile.ldc + col) =
+                    *reinterpret_cast<const float4*>(tr + rr * 32 + 4 * (gc ^ (rr & 7)));
               }
             }
-          } else if (is_w || is_b) {
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              const int rr = 4 * i + rsub;
-              if (rr >= nrows) break;
-              const float* src = tr + rr * 32 + 4 * (gc ^ (rr & 7));
-              if (is_w)
-                *reinterpret_cast<float4*>(g.grads + tile.c_off + (int64_t)(rbase + rr) * tile.ldc + col) =
-                    *reinterpret_cast<const float4*>(src);
-              else
-                g.grads[tile.aux_off + rbase + rr] = src[0];
+          }
+          // db_j, lane = row j: from the bias column when this chunk holds it,
+          // or from dZ's column sums (partials of column j in batch order)
+          const int cb = in_pad - col0;
+          const bool col_b = tile.db_off < 0 && cb >= 0 && cb < 32 && in_pad < n_hi;
+          if ((col_b || (bias_tile && ci == 0)) && lane < nrows) {
+            const float gb = col_b ? tr[lane * 32 + 4 * ((cb >> 2) ^ (lane & 7)) + (cb & 3)]
+                                   : sum_strided(g.dbp + tile.db_off + rbase + lane, g.B_pad / tile.db_rows, tile.m_real);
+            const int64_t o = tile.aux_off + rbase + lane;
+            if (g.update) {
+              const AdamDev& ad = g.adam;
+              float pb = ad.params[o], mb = ad.m[o], vb = ad.v[o];
+              adamw_elem(pb, mb, vb, gb, lr, wd_b, ad.beta1, ad.beta2, ad.eps, ib1, ib2);
+              ad.params[o] = pb;
+              ad.m[o] = mb;
+              ad.v[o] = vb;
+              ad.wq_out[o] = __float2bfloat16_rn(pb);
+            } else {
+              g.grads[o] = gb;
             }
           }
           __syncwarp();  // the buffer is reused by the next chunk
@@ -982,23 +1034,33 @@ __global__ void __launch_bounds__(kThreads, 1) k_tc_gemm(const TcArgs g) {
           flush_chunk(buf, lane, g.act + tile.c_off + (int64_t)rbase * tile.ldc + col0, tile.ldc, rbase, m_lim, ncols);
         } else if (tile.kind == kDgrad) {
           if (ncols <= 0) continue;
-          const uint32_t mb = pick(bits, ci);
+          const uint32_t mb = row_ok ? pick(bits, ci) : 0u;
           const float dsc = tile.aux_off >= 0 ? md.scale : 1.f;   // the first layer's input gradient: 1
           uint8_t* buf = reinterpret_cast<uint8_t*>(tr_all + (warp - 2) * 32 * 32);
+          uint32_t pk[16];
 #pragma unroll
-          for (int sg = 0; sg < 4; ++sg) {
-            uint32_t pk[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const int j = 8 * sg + 2 * e;
-              const float x0 = ((mb >> j) & 1u) ? __uint_as_float(v[j]) * dsc : 0.f;
-              const float x1 = ((mb >> (j + 1)) & 1u) ? __uint_as_float(v[j + 1]) * dsc : 0.f;
-              pk[e] = pack_bf16x2(x0, x1);
-            }
-            stage_group(buf, lane, sg, pk[0], pk[1], pk[2], pk[3]);
+          for (int e = 0; e < 16; ++e) {
+            const int j = 2 * e;
+            const float x0 = ((mb >> j) & 1u) ? __uint_as_float(v[j]) * dsc : 0.f;
+            const float x1 = ((mb >> (j + 1)) & 1u) ? __uint_as_float(v[j + 1]) * dsc : 0.f;
+            pk[e] = pack_bf16x2(x0, x1);
           }
+#pragma unroll
+          for (int sg = 0; sg < 4; ++sg) stage_group(buf, lane, sg, pk[4 * sg], pk[4 * sg + 1], pk[4 * sg + 2], pk[4 * sg + 3]);
           const int rbase = u.m0 + 32 * q;
           flush_chunk(buf, lane, g.dz + tile.c_off + (int64_t)rbase * tile.ldc + col0, tile.ldc, rbase, m_lim, ncols);
+          // the column sums of the stored values over this warp's 32 rows,
+          // where the layer's weight-gradient tiles take db from them
+          if (tile.db_rows > 0 && g.dbp != nullptr) {
+            float x[32];
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+              x[2 * e] = __uint_as_float(pk[e] << 16);
+              x[2 * e + 1] = __uint_as_float(pk[e] & 0xFFFF0000u);
+            }
+            const float cs = colsum32(x, lane);
+            if (lane < ncols) g.dbp[tile.c_off / 32 + (int64_t)(rbase >> 5) * tile.ldc + col0 + lane] = cs;
+          }
         }
       }
       // this warp has read its part of the accumulator: release it to the
@@ -1376,14 +1438,20 @@ tp_status tc_build_plan(TcPlan& plan, const TcLayout& lay, std::string& err) {
         t.sig = cnt_dz(i, l - 1);
         t.c_off = (*lay.dz_off)[i][l - 1];
         t.aux_off = (*lay.act_off)[i][l - 1];
+        t.db_rows = lay.bias_colsums && bias_from_colsums(l - 1 == 0 ? in0p(i) : w) ? 32 : 0;  // dz_{l-1}'s column sums
         emit(vd, t, lay.B_cap / kRowTile, ns);
       }
+      // the weight columns, and the bias column unless the bias gradient
+      // comes from dZ's column sums (bias_from_colsums)
+      const bool cs = lay.bias_colsums && bias_from_colsums(in_pad);
       std::vector<std::pair<int, int>> nw;
-      split_n(in_pad + 1, nw);  // weight columns plus the bias column
+      split_n(cs ? in_pad : in_pad + 1, nw);
       TcTile t{};
       t.kind = kWgrad; t.member = i; t.layer = l;
       t.mask_off = -1;
-      t.m_real = w; t.n_real = in_pad + 1;
+      t.m_real = w; t.n_real = cs ? in_pad : in_pad + 1;
+      t.db_rows = from_head ? kHeadRows : 32;
+      t.db_off = cs ? (*lay.dz_off)[i][l] / 32 : -1;
       t.k_len = 0;
       t.map_a = plan.map_dz[(size_t)i * kMaxDepth + l];
       t.map_b = l == 0 ? (lay.xb_stride || lay.x0_off ? i : 0) : plan.map_act[(size_t)i * kMaxDepth + l - 1];
@@ -1615,7 +1683,7 @@ tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, 
 }
 
 tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, const MemberDev* mem, void* act,
-                     void* dz, float* grads, int update, const AdamDev& adam, std::string& err) {
+                     void* dz, float* grads, float* dbp, int update, const AdamDev& adam, std::string& err) {
   TcArgs a{};
   a.B = B;
   a.B_pad = B_pad;
@@ -1625,6 +1693,7 @@ tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, 
   a.act = (__nv_bfloat16*)act;
   a.dz = (__nv_bfloat16*)dz;
   a.grads = grads;
+  a.dbp = dbp;
   a.adam = adam;
   return launch(plan, st, plan.bwd_rng, a, err);
 }

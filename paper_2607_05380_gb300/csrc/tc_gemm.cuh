@@ -19,7 +19,11 @@ namespace tp {
 //   kFwd   C[b, j]  = sum_k H[b, k] W[j, k]         A = H (K-major), B = W (K-major)
 //   kDgrad C[b, k]  = sum_j dZ[b, j] W[j, k]        A = dZ (K-major), B = W (MN-major)
 //   kWgrad C[j, k]  = sum_b dZ[b, j] [H | 1][b, k]  A = dZ (MN-major), B = [H | 1] (MN-major);
-//          columns k < in_pad are dW, column in_pad is db
+//          columns k < in_pad are dW, column in_pad is db -- or, where the
+//          input width is a multiple of 256 (bias_from_colsums), B = H and
+//          the tiles with n0 = 0 write db_j = sum_b dZ[b, j] from the column
+//          sums that the producer of dZ (head kernel or dgrad epilogue)
+//          stored beside it, added in batch order
 struct TcTile {
   int32_t kind, member, layer;
   int32_t m0, n0, n_len;   // tile origin; n_len = MMA N (multiple of 16, <= 256)
@@ -39,9 +43,15 @@ struct TcTile {
                            // mask arena ([ceil(n_real / 32), mask rows]); -1: none
   int32_t ns_scale;        // kNsGram / kNsApply of the first iteration: 1 + the Muon matrix whose
                            // 1 / |U|_F scales the product (X0 holds U unnormalised); 0: none
+  int32_t db_rows;         // kWgrad: batch rows per column-sum partial of dZ (64: written by the
+                           // head kernel, 32: by dgrad epilogues); kDgrad: 32 = store the column
+                           // sums of the output, 0 = do not
   int64_t c_off;           // output: act (kFwd), dz (kDgrad), weight offset in the arena (kWgrad)
   int64_t aux_off;         // kFwd: bias offset in params; kDgrad: H_l offset in act (mask);
                            // kWgrad: bias offset in the arena
+  int64_t db_off;          // kWgrad: the column-sum partials of its dZ in the partial arena
+                           // ([B_pad / db_rows][w], partial after partial); -1: db from the
+                           // bias column
 };
 
 struct TcPlan {
@@ -89,6 +99,8 @@ struct TcLayout {          // what the plan needs to know about the pack's arena
   const void* act;
   const void* dz;
   bool fwd_only = false;   // forward tiles only (prediction): no dz maps, counters or backward tiles
+  bool bias_colsums = false;  // bias gradients from dZ column sums where bias_from_colsums (else the
+                              // bias column everywhere)
   // Muon: the matrices whose Newton-Schulz products get tiles (NULL: none)
   // and the bf16 arena holding their X, A and Bm buffers
   const std::vector<MuonMat>* muon = nullptr;
@@ -114,9 +126,13 @@ tp_status tc_run_fwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, 
 // Backward products (dgrad + wgrad) of every hidden layer (one launch).
 // update = 0: the weight and bias gradients are stored in `grads`;
 // update = 1: AdamW is applied in the epilogue (adam.wq_out = the other
-// weight copy).
+// weight copy).  dbp: the column-sum partials of dZ (float, element
+// dz_off / 32 + g * w + j for partial g of a [B_cap, w] dZ at dz_off) of
+// the layers whose bias gradient comes from them; the head kernel has
+// written those of each member's last hidden layer, the dgrad epilogues
+// write the others.
 tp_status tc_run_bwd(TcPlan& plan, cudaStream_t st, int B, int B_pad, int wcur, const MemberDev* mem, void* act,
-                     void* dz, float* grads, int update, const AdamDev& adam, std::string& err);
+                     void* dz, float* grads, float* dbp, int update, const AdamDev& adam, std::string& err);
 // Every Newton-Schulz iteration of every Muon matrix in one launch (U in
 // buffer 0, scaled by ns_scale[matrix] = 1 / |U|_F inside the first
 // iteration's products; the result in buffer ns_steps & 1).

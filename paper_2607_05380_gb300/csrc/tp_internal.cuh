@@ -106,6 +106,7 @@ struct HeadJob {          // head forward / loss / backward of one member on one
   int32_t member, blk;
   int32_t h_ld;           // pitch of H_L
   int32_t split;          // row sets of the gradient pass (head_split)
+  int32_t colsum, _pad;   // 1: store the column sums of dZ (bf16 tensor-core mode, bias_from_colsums)
   int64_t h_off;          // H_L in act
   int64_t dz_off;         // dZ_{L-1} in dz (pitch w)
   int64_t w_off, b_off;   // head weight / bias offsets in params
@@ -306,6 +307,14 @@ __host__ __device__ constexpr int head_split(int w, int d_out) {
   return S;
 }
 __host__ __device__ constexpr int64_t ceil_div(int64_t x, int64_t a) { return (x + a - 1) / a; }
+
+// Tensor-core weight-gradient products of a layer whose input width is a
+// multiple of 256 (the widest column tile) take the bias gradient from
+// column sums of dZ that its producer (head kernel or dgrad epilogue)
+// stores beside it: a bias column of ones in the B operand would cost a
+// whole extra column tile there.  Other widths keep the ones column, which
+// fits in the last tile's spare columns.  Both sum dZ as stored (bf16).
+__host__ __device__ constexpr bool bias_from_colsums(int in_pad) { return in_pad % 256 == 0; }
 
 // The element chunks of a Muon matrix: kMuonChunk consecutive elements of W,
 // or for a transposed one (tr) a kMuonTileR x kMuonTileC tile of W, so that

@@ -147,6 +147,38 @@ def test_one_output_head_widths(tp, task, B):
     assert not problems, problems
 
 
+@pytest.mark.parametrize("task,d_out", [("regression", 1), ("multiclass", 3)])
+@pytest.mark.parametrize("B", [256, 200])
+def test_bias_from_column_sums(tp, task, d_out, B):
+    """Layers whose input width is a multiple of 256 take the bias gradient
+    from column sums of dZ instead of a bias column (bf16; forced on here,
+    the pack's own choice keeps it for tensor-bound backward products):
+    d_in = 256 and widths 256, 512, 768, so every layer does, with column
+    sums written by the head (depth 1, and the last layer of deeper members)
+    and by dgrad epilogues; a 272-wide member beside them keeps the bias
+    column.  One step's logits, losses and gradients against the oracle,
+    then the AdamW step of the separate pass and of the fused epilogue
+    against the oracle's AdamW of the GPU's own gradients."""
+    d_in = 256
+    hp = random_pack(5, d_in, d_out, seed=29, depth=(1, 3), dropout=(0.0, 0.3))
+    hp["width"] = np.array([256, 512, 768, 256, 272], dtype=np.int32)
+    hp["depth"] = np.array([1, 2, 3, 3, 2], dtype=np.int32)
+    pk, orc = pair(tp, task, d_in, d_out, hp, "bf16", 256)
+    pk.debug_bias_path(1)
+    X, y = make_data(task, 500, d_in, d_out, 5)
+    idx = np.random.default_rng(6).choice(500, B, replace=False).astype(np.int32)
+    Xd, yd, idxd = to_dev(X, y, idx)
+    loss = torch.zeros(5, dtype=torch.float32, device=DEV)
+    pk.forward_backward(Xd, idxd, yd, 4, loss)
+    orc.train_step(X, idx, y, 4, update=False)
+    problems = compare_step(pk, orc, hp, "bf16", loss.cpu().numpy())
+    assert not problems, problems
+    for fuse in (False, True):
+        pk_s, _ = pair(tp, task, d_in, d_out, hp, "bf16", 256, fuse=fuse)
+        pk_s.debug_bias_path(1)
+        _adamw_of_own_grads(pk_s, pk, hp, range(5), lambda: pk_s.train_step(Xd, idxd, yd, 4, loss))
+
+
 @pytest.mark.parametrize("prec", ["fp32", "bf16"])
 @pytest.mark.parametrize("task,d_out", [("binary", 1), ("multiclass", 7), ("regression", 1)])
 @pytest.mark.parametrize("B", [256, 200])
