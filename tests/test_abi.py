@@ -120,3 +120,13 @@ def test_embedding_entry_points_reject_bad_arguments_without_a_gpu(lib_path):
     assert L.pack_get_emb(None, 0, 0, tp._hptr(out)) == tp.TP_EINVAL
     assert L.pack_set_emb(None, 0, tp._hptr(out)) == tp.TP_EINVAL
     assert L.pack_member_emb(None, 0, ctypes.byref(n)) == tp.TP_EINVAL
+
+
+def test_debug_hooks_reject_a_null_pack_without_a_gpu(lib_path):
+    """The tensor-core debug hooks check their pack before any GPU call."""
+    import paper_2607_05380_gb300 as tp
+    L = tp.load_library()
+    assert L.pack_debug_bias_path(None, 1) == tp.TP_EINVAL
+    assert L.pack_debug_bias_path(None, -1) == tp.TP_EINVAL
+    assert L.pack_debug_gemm_timeout(None, 1.0, 0) == tp.TP_EINVAL
+    assert L.pack_last_error(None)
