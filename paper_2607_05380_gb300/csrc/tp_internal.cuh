@@ -15,7 +15,8 @@
 //   dz     : dL/dZ_l of hidden layer l of member i, [B_cap, w_i] (T).
 // Column in_pad of xb and column w of every act matrix hold 1 (the next 15
 // columns 0): the weight-gradient product dZ^T [H | 1] then yields the bias
-// gradient dZ^T 1 as its extra output column.
+// gradient dZ^T 1 as its extra output column (except where the tensor-core
+// products take it from column sums of dZ, bias_from_colsums below).
 // T = __nv_bfloat16 in bf16 mode, float in fp32 mode.  Batches are padded to
 // B_pad = round_up(B, 128) rows; padded rows carry zero loss gradient, so they
 // add nothing to weight or bias gradients.
